@@ -1,0 +1,260 @@
+"""ctypes loader for the CPU oracle (oracle/auv_oracle.cpp).
+
+TEST INFRASTRUCTURE: only tests/, __graft_entry__.smoke() and the CPU-baseline
+leg of bench.py may import this module.  It never touches the CUDA library.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(HERE, "auv_oracle.cpp")
+LIB = os.path.join(HERE, "liboracle.so")
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle: plain C++17, -O2, no FMA contraction."""
+    if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < os.path.getmtime(SRC):
+        cmd = ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fno-fast-math",
+               "-shared", "-fPIC", "-o", LIB + ".tmp", SRC]
+        subprocess.check_call(cmd)
+        os.replace(LIB + ".tmp", LIB)
+    return LIB
+
+
+class OracleModel(C.Structure):
+    _fields_ = [
+        ("n_substeps", C.c_int32), ("episode_len", C.c_int32), ("seed", C.c_uint32),
+        ("dr_enable", C.c_int32),
+        ("dt", C.c_double), ("mass", C.c_double), ("inertia", C.c_double * 3),
+        ("added_mass", C.c_double * 6), ("damp_lin", C.c_double * 6),
+        ("damp_quad", C.c_double * 6), ("gravity", C.c_double * 3),
+        ("thrust_max", C.c_double), ("alloc", C.c_double * 48),
+        ("w_pos", C.c_double), ("w_att", C.c_double), ("w_act", C.c_double),
+        ("w_vs", C.c_double),
+        ("init_pos_range", C.c_float), ("init_att_range", C.c_float),
+        ("goal_pos_range", C.c_float), ("goal_yaw_range", C.c_float),
+        ("current_range", C.c_float), ("dr_scale_lo", C.c_float), ("dr_scale_hi", C.c_float),
+        ("dr_buoy_range", C.c_float), ("dr_cob_range", C.c_float),
+        ("hidden", C.c_int32), ("policy_out", C.c_int32), ("mlp_bf16", C.c_int32),
+        ("has_value", C.c_int32), ("logstd_fixed", C.c_float * 8),
+        ("logstd_min", C.c_float), ("logstd_max", C.c_float),
+    ]
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = C.CDLL(build())
+        P = C.c_void_p
+        _lib.oracle_model_size.restype = C.c_int
+        _lib.oracle_philox.argtypes = [C.c_uint32, C.c_uint32, P, P]
+        _lib.oracle_word_to_uniform.argtypes = [C.c_uint32]
+        _lib.oracle_word_to_uniform.restype = C.c_float
+        _lib.oracle_taylor_sin.argtypes = [C.c_float]
+        _lib.oracle_taylor_sin.restype = C.c_float
+        _lib.oracle_taylor_cos.argtypes = [C.c_float]
+        _lib.oracle_taylor_cos.restype = C.c_float
+        _lib.oracle_to_bf16.argtypes = [C.c_double]
+        _lib.oracle_to_bf16.restype = C.c_float
+        _lib.oracle_normals.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, P]
+        _lib.oracle_reset.argtypes = [P, C.c_int, P, P, P, P, P]
+        _lib.oracle_replay.argtypes = [P, C.c_int, C.c_int, P, P, P, P, P, C.c_int, P, P, P, P]
+        _lib.oracle_rollout.argtypes = [P, C.c_int, P, P, C.c_int, P, P, P, P, P, C.c_uint64,
+                                        C.c_int, P, P, P, P, P, P]
+        _lib.oracle_mlp.argtypes = [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, P]
+        _lib.oracle_observe.argtypes = [P, P, P, P]
+        _lib.oracle_reward.argtypes = [P, P, P, P]
+        _lib.oracle_reward.restype = C.c_double
+        _lib.oracle_allocate.argtypes = [P, P, P]
+        _lib.oracle_nu_dot.argtypes = [P, P, P, P, P]
+        _lib.oracle_integrate.argtypes = [P, C.c_int, P, P, P, C.c_double, C.c_int]
+        assert _lib.oracle_model_size() == C.sizeof(OracleModel), "OracleModel layout mismatch"
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+def model(w: dict) -> OracleModel:
+    """OracleModel from a workload dict (paper_2512_13359_gb300.workloads)."""
+    m = OracleModel()
+    m.n_substeps = int(w["substeps"])
+    m.episode_len = int(w["episode_len"])
+    m.seed = int(w["seed"]) & 0xFFFFFFFF
+    m.dr_enable = int(w["dr_enable"])
+    m.dt = float(w["dt"])
+    m.mass = float(w["mass"])
+    m.inertia[:] = [float(x) for x in w["inertia"]]
+    m.added_mass[:] = [float(x) for x in w["added_mass"]]
+    m.damp_lin[:] = [float(x) for x in w["damp_lin"]]
+    m.damp_quad[:] = [float(x) for x in w["damp_quad"]]
+    m.gravity[:] = [float(x) for x in w["gravity"]]
+    m.thrust_max = float(w["thrust_max"])
+    m.alloc[:] = [float(x) for x in np.asarray(w["alloc"], dtype=np.float64).reshape(-1)]
+    m.w_pos, m.w_att, m.w_act, m.w_vs = (float(w[k]) for k in ("w_pos", "w_att", "w_act", "w_vs"))
+    for k in ("init_pos_range", "init_att_range", "goal_pos_range", "goal_yaw_range",
+              "current_range", "dr_scale_lo", "dr_scale_hi", "dr_buoy_range", "dr_cob_range"):
+        setattr(m, k, float(w[k]))
+    m.hidden = int(w["hidden"])
+    m.policy_out = int(w["policy_out"])
+    m.mlp_bf16 = 1 if w["mlp"] == "bf16" else 0
+    m.has_value = int(w["has_value"])
+    m.logstd_fixed[:] = [float(x) for x in w["logstd_fixed"]]
+    m.logstd_min = float(w["logstd_min"])
+    m.logstd_max = float(w["logstd_max"])
+    return m
+
+
+class Batch:
+    """SoA env batch held by the oracle: state[19][n], params[17][n] (float64),
+    t_ep[n] (int32), episode[n] (uint32) for the listed env ids."""
+
+    def __init__(self, env_ids):
+        self.env_ids = np.ascontiguousarray(env_ids, dtype=np.uint32)
+        n = len(self.env_ids)
+        self.n = n
+        self.state = np.zeros((19, n), dtype=np.float64)
+        self.params = np.zeros((17, n), dtype=np.float64)
+        self.t_ep = np.zeros(n, dtype=np.int32)
+        self.episode = np.zeros(n, dtype=np.uint32)
+
+    def copy(self):
+        b = Batch(self.env_ids)
+        b.state[:] = self.state
+        b.params[:] = self.params
+        b.t_ep[:] = self.t_ep
+        b.episode[:] = self.episode
+        return b
+
+
+def reset(m: OracleModel, batch: Batch) -> Batch:
+    lib().oracle_reset(C.byref(m), batch.n, _p(batch.env_ids), _p(batch.state),
+                       _p(batch.params), _p(batch.t_ep), _p(batch.episode))
+    return batch
+
+
+def replay(m: OracleModel, batch: Batch, actions: np.ndarray, precision: str = "f64",
+           trace: bool = False):
+    """Action replay over T steps; actions[T][8][n] float32.  Mutates batch.
+    Returns (rew[T][n], done[T][n], trace[T][19][n] or None)."""
+    T = actions.shape[0]
+    n = batch.n
+    assert actions.shape == (T, 8, n)
+    act = np.ascontiguousarray(actions, dtype=np.float32)
+    rew = np.zeros((T, n), dtype=np.float64)
+    done = np.zeros((T, n), dtype=np.uint8)
+    tr = np.zeros((T, 19, n), dtype=np.float64) if trace else None
+    lib().oracle_replay(C.byref(m), 1 if precision == "f32" else 0, n, _p(batch.env_ids),
+                        _p(batch.state), _p(batch.params), _p(batch.t_ep), _p(batch.episode),
+                        T, _p(act), _p(rew), _p(done), _p(tr))
+    return rew, done, tr
+
+
+def rollout(m: OracleModel, batch: Batch, pol_w: np.ndarray, val_w, t_g0: int, T: int,
+            precision: str = "f64", want=("obs", "act", "logp", "value", "rew", "done")):
+    """Closed-loop rollout over T steps.  Mutates batch.  Returns a dict of
+    SoA arrays obs[T][18][n], act[T][8][n], logp[T][n], value[T][n],
+    rew[T][n], done[T][n] (those listed in `want`)."""
+    n = batch.n
+    out = {}
+    shapes = dict(obs=(T, 18, n), act=(T, 8, n), logp=(T, n), value=(T, n), rew=(T, n))
+    for k, s in shapes.items():
+        out[k] = np.zeros(s, dtype=np.float64) if k in want else None
+    if "value" in want and not m.has_value:
+        out["value"] = None
+    out["done"] = np.zeros((T, n), dtype=np.uint8)
+    pw = np.ascontiguousarray(pol_w, dtype=np.float32)
+    vw = None if val_w is None else np.ascontiguousarray(val_w, dtype=np.float32)
+    lib().oracle_rollout(C.byref(m), 1 if precision == "f32" else 0, _p(pw), _p(vw), n,
+                         _p(batch.env_ids), _p(batch.state), _p(batch.params), _p(batch.t_ep),
+                         _p(batch.episode), int(t_g0), T, _p(out["obs"]), _p(out["act"]),
+                         _p(out["logp"]), _p(out["value"]), _p(out["rew"]), _p(out["done"]))
+    return {k: v for k, v in out.items() if v is not None}
+
+
+def mlp(weights: np.ndarray, in_dim: int, hidden: int, out_dim: int, bf16: bool,
+        x: np.ndarray) -> np.ndarray:
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    n = x.shape[0]
+    out = np.zeros((n, out_dim), dtype=np.float64)
+    w = np.ascontiguousarray(weights, dtype=np.float32)
+    lib().oracle_mlp(_p(w), in_dim, hidden, out_dim, 1 if bf16 else 0, n, _p(x), _p(out))
+    return out
+
+
+def philox(key0: int, key1: int, ctr) -> np.ndarray:
+    c = np.ascontiguousarray(ctr, dtype=np.uint32)
+    out = np.zeros(4, dtype=np.uint32)
+    lib().oracle_philox(key0 & 0xFFFFFFFF, key1 & 0xFFFFFFFF, _p(c), _p(out))
+    return out
+
+
+def normals(env_id: int, seed: int, t_g: int) -> np.ndarray:
+    out = np.zeros(8, dtype=np.float64)
+    lib().oracle_normals(env_id, seed, t_g, _p(out))
+    return out
+
+
+def single_env(state: dict, params: dict):
+    """19- and 17-row single-env SoA vectors from field dicts (missing = 0,
+    scales default 1, quaternions default identity)."""
+    st = np.zeros(19)
+    pr = np.zeros(17)
+    st[3] = 1.0
+    pr[3] = 1.0
+    pr[7] = pr[8] = pr[9] = 1.0
+    for k, v in state.items():
+        idx = dict(p=0, q=3, nu=7, nu_prev=13)[k]
+        st[idx:idx + len(v)] = v
+    for k, v in params.items():
+        idx = dict(p_d=0, q_d=3, s_m=7, s_a=8, s_d=9, dB=10, r_b=11, V_c=14)[k]
+        v = np.atleast_1d(v)
+        pr[idx:idx + len(v)] = v
+    return st, pr
+
+
+def observe(st, pr):
+    obs = np.zeros(18)
+    th = np.zeros(1)
+    lib().oracle_observe(_p(np.ascontiguousarray(st, dtype=np.float64)),
+                         _p(np.ascontiguousarray(pr, dtype=np.float64)), _p(obs), _p(th))
+    return obs, float(th[0])
+
+
+def reward(m, st, pr, a_c):
+    return lib().oracle_reward(C.byref(m), _p(np.ascontiguousarray(st, dtype=np.float64)),
+                               _p(np.ascontiguousarray(pr, dtype=np.float64)),
+                               _p(np.ascontiguousarray(a_c, dtype=np.float64)))
+
+
+def allocate(m, a):
+    tau = np.zeros(6)
+    lib().oracle_allocate(C.byref(m), _p(np.ascontiguousarray(a, dtype=np.float64)), _p(tau))
+    return tau
+
+
+def nu_dot(m, st, pr, tau):
+    out = np.zeros(6)
+    lib().oracle_nu_dot(C.byref(m), _p(np.ascontiguousarray(st, dtype=np.float64)),
+                        _p(np.ascontiguousarray(pr, dtype=np.float64)),
+                        _p(np.ascontiguousarray(tau, dtype=np.float64)), _p(out))
+    return out
+
+
+def integrate(m, st, pr, tau, h, n_steps, method="euler"):
+    """Integrate one env's physics; returns the new 19-row state vector."""
+    s = np.ascontiguousarray(st, dtype=np.float64).copy()
+    lib().oracle_integrate(C.byref(m), 0 if method == "euler" else 1, _p(s),
+                           _p(np.ascontiguousarray(pr, dtype=np.float64)),
+                           _p(np.ascontiguousarray(tau, dtype=np.float64)), float(h),
+                           int(n_steps))
+    return s
