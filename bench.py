@@ -1,0 +1,396 @@
+#!/usr/bin/env python
+"""Throughput of the batched AUV rollout step on GB300 (env-steps/s).
+
+One bench step = one PPO collection pass of the 65,536-env workload: a
+T = 128-step rollout (observation, policy network, Gaussian action,
+thruster allocation, 4 physics substeps, reward, done, auto-reset) writing
+the full SoA trajectory (obs, act, logp, rew, done), followed by the value
+network over the stored observations.  Prints one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) each rank steps its own shard of envs (env ids offset
+by rank, weak scaling, no data-path collective); rank 0 prints.
+`--impl reference` times the CPU oracle (test infrastructure) on a bounded
+sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2512_13359_gb300 import workloads as W  # noqa: E402
+
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="ppo_65536")
+    ap.add_argument("--n-envs", type=int, default=None)
+    ap.add_argument("--rollout-steps", type=int, default=None)
+    ap.add_argument("--mlp", default=None, choices=[None, "fp32", "bf16"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "sm_max_mhz": 2070.0}, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work per env-step
+# ---------------------------------------------------------------------------
+def mlp_flops(hidden, out):
+    return 2 * (W.OBS_DIM * hidden + hidden * hidden + hidden * out)
+
+
+def traj_bytes_per_env_step(keys):
+    b = dict(obs=4 * W.OBS_DIM, act=4 * W.ACT_DIM, logp=4, value=4, rew=4, done=1)
+    return sum(b[k] for k in keys)
+
+
+# ---------------------------------------------------------------------------
+# reference arm / CPU baseline: the oracle on a bounded sample
+# ---------------------------------------------------------------------------
+def oracle_sample_rate(w, T, target_s, max_envs=4096):
+    """Time the CPU oracle on a sample of envs over T steps; env-steps/s on
+    one host core.  The sample grows until it takes about target_s."""
+    from oracle import oracle as O
+    m = O.model(w)
+    pw = W.policy_weights(w)
+    vw = W.value_weights(w) if w["has_value"] else None
+    n = 2
+    while True:
+        b = O.Batch(np.arange(n))
+        O.reset(m, b)
+        t0 = time.perf_counter()
+        O.rollout(m, b, pw, vw, 0, T)
+        dt = time.perf_counter() - t0
+        if dt >= target_s or n >= max_envs:
+            return n * T / dt, n, dt
+        n = min(max_envs, max(n * 2, int(n * target_s / max(dt, 1e-3)) + 1))
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from oracle import oracle as O
+    O.build()
+    T = w["steps"]
+    m = O.model(w)
+    pw = W.policy_weights(w)
+    vw = W.value_weights(w) if w["has_value"] else None
+    # size one bench step so that K + W steps take about a minute in total
+    rate, _, _ = oracle_sample_rate(w, T, 2.0)
+    per_step_s = max(1.0, 60.0 / max(1, args.steps + args.warmup))
+    n = max(1, int(rate * per_step_s / T))
+    times = []
+    for s in range(args.warmup + args.steps):
+        b = O.Batch(np.arange(n))
+        O.reset(m, b)
+        t0 = time.perf_counter()
+        O.rollout(m, b, pw, vw, 0, T)
+        if s >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    value = n * T / sec
+    sample = f"{n} envs x {T} steps of {w['name']} per step (env ids 0..{n - 1})"
+    line = {
+        "impl": "reference", "metric": "env-steps/s (physics+policy+reward)", "value": value,
+        "unit": "env-steps/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w["name"], "n_envs": w["n_envs"], "rollout_steps": T,
+                   "substeps": w["substeps"], "mlp": w["mlp"], "sample_envs": n},
+        "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "env-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def main():
+    args = parse()
+    over = {}
+    if args.n_envs:
+        over["n_envs"] = args.n_envs
+    if args.rollout_steps:
+        over["steps"] = args.rollout_steps
+    if args.mlp:
+        over["mlp"] = args.mlp
+    w = W.workload(args.workload, **over)
+    if args.impl == "reference":
+        run_reference(args, w)
+        return
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2512_13359_gb300 import auvenv, build
+    if rank == 0 or world == 1:
+        build.build()
+    if dist:
+        dist.barrier()
+
+    n = int(w["n_envs"])
+    T = int(w["steps"])
+    w["env_id_base"] = rank * n          # shard: rank r owns global env ids [r n, (r+1) n)
+    env = auvenv.Env(w)
+    pw = W.policy_weights(w)
+    vw = W.value_weights(w) if w["has_value"] else None
+    env.set_weights(pw, vw)
+    env.reset()
+    keys = ["obs", "act", "logp", "rew", "done"]
+    traj = env.alloc_traj(T, keys=keys)
+    value = torch.empty((T, n), dtype=torch.float32, device="cuda") if w["has_value"] else None
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+
+    def one_step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        env.rollout(T, traj)
+        if ev:
+            ev[1].record(stream)
+        if value is not None:
+            env.value(traj["obs"], value)
+        if ev:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+    st = env.status()
+    if st.code != 0:
+        raise RuntimeError(f"device status {st.code} after warm-up")
+
+    clocks = ClockSampler(local) if not args.no_clocks else None
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    events = []
+    for _ in range(args.steps):
+        flush.zero_()                       # evict L2 between timed steps
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        one_step(ev)
+        events.append(ev)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clock_info = clocks.stop() if clocks else None
+    roll_ms = [e[0].elapsed_time(e[1]) for e in events]
+    val_ms = [e[1].elapsed_time(e[2]) for e in events]
+    step_ms = sum(r + v for r, v in zip(roll_ms, val_ms)) / args.steps
+    if dist:
+        t = torch.tensor([step_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms = float(t.item())
+    env_steps = n * T * world
+    value_rate = env_steps / (step_ms * 1e-3)
+    st = env.status()
+    if st.code != 0:
+        raise RuntimeError(f"device status {st.code} after timed steps")
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        h_traj = env.alloc_traj(T, keys=keys, pinned_host=True)
+        h_val = torch.empty((T, n), dtype=torch.float32, pin_memory=True) if value is not None else None
+        h_pw = torch.from_numpy(pw).pin_memory()
+        h_vw = torch.from_numpy(vw).pin_memory() if vw is not None else None
+        h2d = h_pw.numel() * 4 + (h_vw.numel() * 4 if h_vw is not None else 0)
+        d2h = n * T * traj_bytes_per_env_step(keys + (["value"] if value is not None else []))
+        for _ in range(2):
+            env.set_weights(h_pw, h_vw)
+            env.rollout(T, h_traj)
+            if h_val is not None:
+                env.value(h_traj["obs"], h_val)
+            torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(max(1, min(args.steps, 5))):
+            env.set_weights(h_pw, h_vw)          # step inputs: policy + value weights, H2D
+            env.rollout(T, h_traj)               # trajectory written to pinned host memory
+            if h_val is not None:
+                env.value(h_traj["obs"], h_val)
+            torch.cuda.synchronize()
+        e2e_s = (time.perf_counter() - t0) / max(1, min(args.steps, 5))
+        if dist:
+            t = torch.tensor([e2e_s], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        e2e = {"value": env_steps / e2e_s, "unit": "env-steps/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+
+    # ---- roofline of the dominant kernel ----
+    peaks, peak_src = load_peaks()
+    roll_avg = sum(roll_ms) / len(roll_ms)
+    val_avg = sum(val_ms) / len(val_ms) if value is not None else 0.0
+    pol_fl = mlp_flops(w["hidden"], w["policy_out"])
+    val_fl = mlp_flops(w["hidden"], 1) if w["has_value"] else 0
+    sm_mhz = (clock_info or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+    n_sm = torch.cuda.get_device_properties(local).multi_processor_count
+    fp32_peak = 2 * 128 * n_sm * sm_mhz * 1e6 / 1e12   # TFLOP/s of the FP32 pipe
+    if w["mlp"] == "bf16":
+        if roll_avg >= val_avg:
+            kern, dur = "rollout_bf16", roll_avg
+            flops = n * T * (pol_fl + DYN_FLOPS_PER_ENV_STEP)
+        else:
+            kern, dur = "value_bf16", val_avg
+            flops = n * T * val_fl
+        achieved = flops / (dur * 1e-3) / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        roof = {"bound": "tensor", "kernel": kern, "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "peak_source": f"bf16 sustained, {peak_src}"}
+    else:
+        kern, dur = "rollout_fp32", roll_avg
+        flops = n * T * (pol_fl + val_fl + DYN_FLOPS_PER_ENV_STEP)
+        if value is not None and val_avg > roll_avg:
+            kern, dur, flops = "value_fp32", val_avg, n * T * val_fl
+        elif value is not None:
+            flops = n * T * (pol_fl + DYN_FLOPS_PER_ENV_STEP)
+        achieved = flops / (dur * 1e-3) / 1e12
+        roof = {"bound": "alu", "kernel": kern, "achieved": achieved, "peak": fp32_peak,
+                "unit": "TFLOP/s", "frac": achieved / fp32_peak, "traffic": None,
+                "peak_source": f"FP32 pipe 2*128*{n_sm} SMs*{sm_mhz:.0f} MHz"}
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        from oracle import oracle as O
+        O.build()
+        rate, n_s, dt = oracle_sample_rate(w, T, args.cpu_seconds)
+        cpu = {"value": rate, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n_s} envs x {T} steps of {w['name']} ({dt:.1f} s, one thread)"}
+
+    launches_per_step = 1 + (1 if value is not None else 0)
+    line = {
+        "metric": "env-steps/s (physics+policy+reward)", "value": value_rate,
+        "unit": "env-steps/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if w["mlp"] == "bf16" else "f32",
+        "data": "synthetic",
+        "config": {"workload": w["name"], "n_envs_per_gpu": n, "rollout_steps": T,
+                   "substeps": w["substeps"], "mlp": w["mlp"], "hidden": w["hidden"],
+                   "trajectory": keys + (["value"] if value is not None else []),
+                   "l2": "flushed between timed steps (2 x L2 buffer written)",
+                   "rollout_ms": roll_avg, "value_ms": val_avg},
+        "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+# Algorithmic FP32 flops of the physics part of one env-step (4 substeps,
+# allocation, observation, noise, reward), counted from the kernel source.
+DYN_FLOPS_PER_ENV_STEP = 2000
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,255 @@
+/*
+ * auvenv.h -- C ABI of the GB300 batched AUV rollout library (libauvenv.so).
+ *
+ * The library steps N independent underwater-vehicle environments of the
+ * 6-DOF position-control task of "Fast Policy Learning for 6-DOF Position
+ * Control of Underwater Vehicles" (arXiv 2512.13359): per control step it
+ * evaluates the policy network on each env's observation, samples a Gaussian
+ * action, maps it through the thruster allocation to a body wrench,
+ * integrates the rigid-body + hydrodynamic model, and computes the reward,
+ * the done flag and the automatic reset (paper §IV-A: batched simulation of
+ * independent environments sharing one model and integrator).
+ *
+ * Conventions shared by every entry point
+ *  - Return value: AUV_OK (0) or a negative AUV_ERR_* code; env_last_error()
+ *    gives a one-line reason.  No entry point aborts or traps.
+ *  - Asynchrony: every call that takes `stream` (a cudaStream_t; NULL = the
+ *    legacy default stream) only enqueues work on that stream and returns.
+ *    Device-side faults (non-finite state, a wait that timed out) are latched
+ *    in a device status block and reported by env_status().
+ *  - Layout: all per-env arrays are structure-of-arrays, env index fastest:
+ *    element (k, i) of a [K][N] array is at k*N + i; trajectory arrays are
+ *    [T][K][N] with element (t, k, i) at (t*K + k)*N + i.
+ *  - Ownership: the caller allocates and owns every state, parameter and
+ *    trajectory buffer (device memory, or host memory that is page-locked and
+ *    mapped, e.g. from cudaHostAlloc, for trajectory outputs).  The library
+ *    owns only its handle and a device workspace it allocates in env_create
+ *    and frees in env_destroy (packed network weights and the status block).
+ *  - The CUDA device is the one current on the calling thread at env_create;
+ *    later calls must be made with the same device current.
+ */
+#ifndef AUVENV_H
+#define AUVENV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AUV_ABI_VERSION 1
+
+/* status codes */
+#define AUV_OK 0
+#define AUV_ERR_INVALID (-1)      /* bad argument or configuration value     */
+#define AUV_ERR_SIZE (-2)         /* buffer missing, misaligned or wrong kind */
+#define AUV_ERR_CUDA (-3)         /* a CUDA runtime call failed              */
+#define AUV_ERR_TIMEOUT (-4)      /* a device-side bounded wait gave up      */
+#define AUV_ERR_NAN (-5)          /* non-finite state detected               */
+#define AUV_ERR_UNSUPPORTED (-6)  /* valid but not implemented combination   */
+
+/* network arithmetic */
+#define AUV_MLP_FP32 0   /* fp32 operands and accumulation on CUDA cores        */
+#define AUV_MLP_BF16 1   /* bf16 weights/activations, fp32 accumulation, tcgen05 */
+
+/* sizes fixed by the model */
+#define AUV_OBS_DIM 18      /* observation: dp_b(3), R_e column-major(9), v(3), w(3) */
+#define AUV_ACT_DIM 8       /* normalised thruster commands                        */
+#define AUV_STATE_FIELDS 19 /* p(3) q(4: w,x,y,z body->world) nu(6) nu_prev(6)     */
+#define AUV_PARAM_FIELDS 17 /* p_d(3) q_d(4) s_m s_a s_d dB r_b(3) V_c(3)          */
+
+/*
+ * Model and workload description.  Paper §IV-B (environment), §IV-C (domain
+ * randomisation), §IV-D (Fossen 6-DOF equations of motion), Eqs. (1)-(7)
+ * (action and reward), §V-A1 (episodes with a random reference).
+ * The equations of motion, in the body frame, with nu = [v; w]:
+ *   (M_RB + M_A) nu' = tau - C_RB(nu) nu - C_A(nu_r) nu_r - D(nu_r) nu_r
+ *                      - g(eta) + M_A nu_c'
+ * nu_r = nu - [R^T V_c; 0], M_RB = diag(m, m, m, I), M_A, D_L, D_Q diagonal,
+ * damping D(nu_r) nu_r = (D_L + D_Q |nu_r|) nu_r, weight at the origin,
+ * buoyancy B = m |g| + dB at r_b, tau = alloc * (thrust_max * clip(a, -1, 1)).
+ * Per episode the randomised scales multiply: s_m the mass and inertia, s_a
+ * the added mass, s_d both damping matrices.
+ */
+typedef struct auv_config {
+  uint32_t struct_size;   /* sizeof(auv_config): version guard               */
+  uint32_t n_envs;        /* N >= 1                                          */
+  uint32_t substeps;      /* physics substeps per control step, 1..64        */
+  uint32_t episode_len;   /* control steps per episode (time-limit done) >= 1 */
+  uint32_t seed;          /* Philox key word 1 (word 0 is the env id)        */
+  uint32_t env_id_base;   /* global id of local env 0: env i uses Philox key
+                             word 0 = env_id_base + i, so a shard of a larger
+                             batch reproduces that batch's envs exactly       */
+  uint32_t dr_enable;     /* 1: draw s_m, s_a, s_d, dB, r_b at every reset   */
+  float dt;               /* control period [s] > 0                          */
+  float mass;             /* m [kg]                                          */
+  float inertia[3];       /* principal moments about the CoG [kg m^2]        */
+  float added_mass[6];    /* diag(M_A)                                       */
+  float damp_lin[6];      /* diag(D_L)                                       */
+  float damp_quad[6];     /* diag(D_Q)                                       */
+  float gravity[3];       /* world gravity vector g_w [m/s^2]                */
+  float thrust_max;       /* newtons per thruster at |a| = 1                 */
+  float alloc[48];        /* allocation matrix, row-major [6][8]             */
+  float w_pos, w_att, w_act, w_vs;  /* reward weights (see env_rollout)      */
+  float init_pos_range;   /* initial position U[-r, r] per axis [m]          */
+  float init_att_range;   /* initial roll, pitch, yaw U[-r, r] [rad]         */
+  float goal_pos_range;   /* goal position U[-r, r] per axis [m]             */
+  float goal_yaw_range;   /* goal yaw U[-r, r] [rad], r <= pi                */
+  float current_range;    /* water current U[-r, r] per world axis [m/s]     */
+  float dr_scale_lo, dr_scale_hi;   /* s_m, s_a, s_d ~ U[lo, hi]             */
+  float dr_buoy_range;    /* dB ~ U[-r, r] [N]                               */
+  float dr_cob_range;     /* r_b ~ U[-r, r] per axis [m]                     */
+  uint32_t hidden;        /* hidden width H of both networks                 */
+  uint32_t policy_out;    /* 8: mean only (fixed log-std); 16: mean + log-std */
+  uint32_t mlp_mode;      /* AUV_MLP_FP32 or AUV_MLP_BF16                    */
+  uint32_t has_value;     /* 1: value network present                        */
+  float logstd_fixed[8];  /* log-std used when policy_out == 8               */
+  float logstd_min, logstd_max;     /* clamp of the log-std head             */
+} auv_config;
+
+/* Caller-owned device buffers holding the batch (SoA, see layout above). */
+typedef struct auv_buffers {
+  float* state;       /* [19][N] p, q, nu, nu_prev                       */
+  float* params;      /* [17][N] p_d, q_d, s_m, s_a, s_d, dB, r_b, V_c    */
+  int32_t* t_ep;      /* [N] control steps taken in the current episode  */
+  uint32_t* episode;  /* [N] index of the next episode's reset draw      */
+} auv_buffers;
+
+/* Trajectory outputs of env_rollout; any pointer may be NULL (not written).
+ * Device memory or mapped page-locked host memory, 4-byte aligned.        */
+typedef struct auv_traj {
+  float* obs;     /* [T][18][N] observation the action was taken from   */
+  float* act;     /* [T][8][N]  unclipped sampled action a_t            */
+  float* logp;    /* [T][N]     log pi(a_t | o_t)                       */
+  float* value;   /* [T][N]     V(o_t) (needs has_value)                */
+  float* rew;     /* [T][N]     reward r_t on the post-step state       */
+  uint8_t* done;  /* [T][N]     1 if the episode ended at this step     */
+} auv_traj;
+
+/* Device status block contents, read by env_status(). */
+typedef struct auv_status {
+  int32_t code;          /* AUV_OK, AUV_ERR_NAN or AUV_ERR_TIMEOUT (first latched) */
+  int32_t nan_flag;      /* 1 if any env produced a non-finite state               */
+  int32_t first_nan_env; /* smallest env id with a non-finite state, or -1         */
+  int32_t timeouts;      /* number of device waits that gave up                    */
+} auv_status;
+
+typedef struct auv_env auv_env;
+
+/* ABI version of the loaded library (AUV_ABI_VERSION it was built with). */
+int env_abi_version(void);
+
+/*
+ * env_create: validate `cfg`, bind the caller's buffers and allocate the
+ * library workspace on the current device.  Writes the handle to *out.
+ * Buffers must hold N elements per field and be 16-byte aligned.  Nothing is
+ * initialised: call env_set_weights and env_reset before stepping.  The
+ * global step counter (the action-noise stream index) starts at 0.
+ * Errors: AUV_ERR_INVALID (bad cfg value, NULL pointer, struct_size
+ * mismatch), AUV_ERR_UNSUPPORTED (hidden/policy_out/mode combination not
+ * built), AUV_ERR_CUDA.
+ */
+int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out);
+
+/* env_destroy: synchronise the device, free the workspace and the handle. */
+int env_destroy(auv_env* env);
+
+/* One-line description of the last error on this handle ("" if none). */
+const char* env_last_error(const auv_env* env);
+
+/*
+ * env_set_weights: load the policy (and value) network weights.  Layout per
+ * network, fp32, row-major [out][in]: W1[H][18] b1[H] W2[H][H] b2[H]
+ * W3[O][H] b3[O] with O = policy_out (policy) or 1 (value).  Pointers may be
+ * host or device memory; `value` must be non-NULL iff has_value.  The library
+ * converts them into its packed device layout (bf16 rounding to nearest even
+ * in AUV_MLP_BF16 mode) on `stream`; host memory is read before return.
+ */
+int env_set_weights(auv_env* env, const float* policy, const float* value, void* stream);
+
+/*
+ * env_reset: start a new episode for every env with mask[i] != 0 (all envs if
+ * mask is NULL; mask is device memory, [N] bytes).  Draws, from Philox4x32-10
+ * with key (env_id_base + i, seed) and counter (episode, 0, 1, 0..4), 20 uniforms:
+ * initial position, roll/pitch/yaw, goal position, goal yaw, current, s_m,
+ * s_a, s_d, dB, r_b (paper §IV-C, §V-A1); zero velocities; t_ep = 0;
+ * episode += 1.  Bit-exact across implementations of the same steps.
+ */
+int env_reset(auv_env* env, const uint8_t* mask, void* stream);
+
+/*
+ * env_rollout: T >= 1 control steps of the full hot path for all envs, state
+ * carried on chip.  Per step t and env: o_t = observation (paper §IV-B1,
+ * attitude as the rotation-matrix error of §V-A3); (mu, log sigma) = policy
+ * network; eps = 8 Box-Muller normals from Philox key (env id, seed), counter
+ * (t_g lo, t_g hi, 0, 0..1); a = mu + sigma eps; log pi = sum(-eps^2/2 -
+ * log sigma - log(2 pi)/2); tau = alloc (thrust_max clip(a, -1, 1)) (Eq. 1 and
+ * the thruster allocation of §V-B); nu_prev = nu; `substeps` semi-implicit
+ * Euler substeps of the equations of motion; r = -w_pos |p - p_d| - w_att
+ * theta_e - w_act |clip(a)|^2 - w_vs |nu - nu_prev|^2 (weighted norms of
+ * Eqs. 2-7); t_ep += 1; done = (t_ep == episode_len); on done the env resets
+ * as in env_reset.  The global step t_g advances by T.
+ */
+int env_rollout(auv_env* env, int T, const auv_traj* traj, void* stream);
+
+/* env_step: env_rollout with T = 1 writing only obs (the observation the
+ * step acted on), rew and done; each may be NULL. */
+int env_step(auv_env* env, float* obs_out, float* rew_out, uint8_t* done_out, void* stream);
+
+/*
+ * env_step_actions: action replay.  T control steps with the given
+ * normalised actions act[T][8][N] (device) instead of the policy: allocation,
+ * substeps, reward, done and auto-reset exactly as in env_rollout.  Writes
+ * rew[T][N], done[T][N] and, if non-NULL, state_trace[T][19][N] (state after
+ * each step, after any reset).  Does not advance t_g.
+ */
+int env_step_actions(auv_env* env, const float* act, int T, float* rew_out, uint8_t* done_out,
+                     float* state_trace, void* stream);
+
+/*
+ * env_value: the value network on stored observations, in the trajectory
+ * layout: obs[T][18][N] -> value[T][N] (device or mapped host memory),
+ * T >= 1, with the loaded value weights (needs has_value).  A PPO learner
+ * re-evaluates values this way; env_rollout calls it itself when given
+ * traj.value.
+ */
+int env_value(auv_env* env, const float* obs, int T, float* value, void* stream);
+
+/* env_observe: observation of the current state, obs[18][N] (device). */
+int env_observe(auv_env* env, float* obs_out, void* stream);
+
+/*
+ * env_policy_forward: evaluate the loaded networks on caller observations
+ * obs[n][18] (row-major, device) for n >= 1 rows: head[n][policy_out] (raw
+ * outputs: mean, then unclamped log-std) and, if value is non-NULL and
+ * has_value, value[n].  Same device arithmetic as env_rollout.
+ */
+int env_policy_forward(auv_env* env, const float* obs, int n, float* head, float* value,
+                       void* stream);
+
+/*
+ * env_draw_words: the raw Philox4x32-10 words of one stream for every env:
+ * out[4*n_blocks][N] (device, uint32) with block b of env i = Philox(key =
+ * (env_id_base + i, seed), counter = (index lo, index hi, stream_id, b)).  stream_id 0 =
+ * action noise (index = global step), 1 = reset (index = episode).
+ */
+int env_draw_words(auv_env* env, uint32_t stream_id, uint64_t index, int n_blocks,
+                   uint32_t* out, void* stream);
+
+/* Global step counter (action-noise stream index) get/set, for checkpoints. */
+int env_get_step(const auv_env* env, uint64_t* t_g);
+int env_set_step(auv_env* env, uint64_t t_g);
+
+/*
+ * env_status: synchronise `stream`, copy the device status block to *out and
+ * return out->code.  env_clear_status zeroes it (asynchronously on stream).
+ */
+int env_status(auv_env* env, auv_status* out, void* stream);
+int env_clear_status(auv_env* env, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AUVENV_H */

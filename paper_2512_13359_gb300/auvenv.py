@@ -1,0 +1,287 @@
+"""Python binding of libauvenv.so (include/auvenv.h): argument marshalling only.
+
+Every step of the rollout runs in the library's CUDA kernels; torch provides
+device memory and streams.  There is no CPU fallback: if the library is
+missing or cannot be loaded, LibraryMissing is raised.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+from . import workloads as W
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libauvenv.so")
+
+AUV_OK = 0
+AUV_ERR_INVALID = -1
+AUV_ERR_SIZE = -2
+AUV_ERR_CUDA = -3
+AUV_ERR_TIMEOUT = -4
+AUV_ERR_NAN = -5
+AUV_ERR_UNSUPPORTED = -6
+AUV_MLP_FP32 = 0
+AUV_MLP_BF16 = 1
+
+EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
+            "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
+            "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
+            "env_status", "env_clear_status")
+
+
+class LibraryMissing(RuntimeError):
+    pass
+
+
+class AuvError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"auvenv error {code}: {msg}")
+        self.code = code
+
+
+class AuvConfig(C.Structure):
+    _fields_ = [
+        ("struct_size", C.c_uint32), ("n_envs", C.c_uint32), ("substeps", C.c_uint32),
+        ("episode_len", C.c_uint32), ("seed", C.c_uint32), ("env_id_base", C.c_uint32),
+        ("dr_enable", C.c_uint32),
+        ("dt", C.c_float), ("mass", C.c_float), ("inertia", C.c_float * 3),
+        ("added_mass", C.c_float * 6), ("damp_lin", C.c_float * 6), ("damp_quad", C.c_float * 6),
+        ("gravity", C.c_float * 3), ("thrust_max", C.c_float), ("alloc", C.c_float * 48),
+        ("w_pos", C.c_float), ("w_att", C.c_float), ("w_act", C.c_float), ("w_vs", C.c_float),
+        ("init_pos_range", C.c_float), ("init_att_range", C.c_float),
+        ("goal_pos_range", C.c_float), ("goal_yaw_range", C.c_float),
+        ("current_range", C.c_float), ("dr_scale_lo", C.c_float), ("dr_scale_hi", C.c_float),
+        ("dr_buoy_range", C.c_float), ("dr_cob_range", C.c_float),
+        ("hidden", C.c_uint32), ("policy_out", C.c_uint32), ("mlp_mode", C.c_uint32),
+        ("has_value", C.c_uint32), ("logstd_fixed", C.c_float * 8),
+        ("logstd_min", C.c_float), ("logstd_max", C.c_float),
+    ]
+
+
+class AuvBuffers(C.Structure):
+    _fields_ = [("state", C.c_void_p), ("params", C.c_void_p), ("t_ep", C.c_void_p),
+                ("episode", C.c_void_p)]
+
+
+class AuvTraj(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("act", C.c_void_p), ("logp", C.c_void_p),
+                ("value", C.c_void_p), ("rew", C.c_void_p), ("done", C.c_void_p)]
+
+
+class AuvStatus(C.Structure):
+    _fields_ = [("code", C.c_int32), ("nan_flag", C.c_int32), ("first_nan_env", C.c_int32),
+                ("timeouts", C.c_int32)]
+
+
+_lib = None
+
+
+def lib(path: str | None = None):
+    """Load libauvenv.so (once).  Raises LibraryMissing if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise LibraryMissing(f"{p} not built; run paper_2512_13359_gb300.build.build()")
+    try:
+        L = C.CDLL(p)
+    except OSError as e:
+        raise LibraryMissing(f"cannot load {p}: {e}") from e
+    P, I = C.c_void_p, C.c_int
+    L.env_abi_version.restype = I
+    L.env_create.argtypes = [P, P, C.POINTER(P)]
+    L.env_destroy.argtypes = [P]
+    L.env_last_error.argtypes = [P]
+    L.env_last_error.restype = C.c_char_p
+    L.env_set_weights.argtypes = [P, P, P, P]
+    L.env_reset.argtypes = [P, P, P]
+    L.env_rollout.argtypes = [P, I, P, P]
+    L.env_value.argtypes = [P, P, I, P, P]
+    L.env_step.argtypes = [P, P, P, P, P]
+    L.env_step_actions.argtypes = [P, P, I, P, P, P, P]
+    L.env_observe.argtypes = [P, P, P]
+    L.env_policy_forward.argtypes = [P, P, I, P, P, P]
+    L.env_draw_words.argtypes = [P, C.c_uint32, C.c_uint64, I, P, P]
+    L.env_get_step.argtypes = [P, C.POINTER(C.c_uint64)]
+    L.env_set_step.argtypes = [P, C.c_uint64]
+    L.env_status.argtypes = [P, C.POINTER(AuvStatus), P]
+    L.env_clear_status.argtypes = [P, P]
+    for name in EXPORTED:
+        getattr(L, name).restype = getattr(L, name).restype or I
+    L.env_last_error.restype = C.c_char_p
+    _lib = L
+    return L
+
+
+def make_config(w: dict) -> AuvConfig:
+    c = AuvConfig()
+    c.struct_size = C.sizeof(AuvConfig)
+    c.n_envs = int(w["n_envs"])
+    c.substeps = int(w["substeps"])
+    c.episode_len = int(w["episode_len"])
+    c.seed = int(w["seed"]) & 0xFFFFFFFF
+    c.env_id_base = int(w.get("env_id_base", 0))
+    c.dr_enable = int(w["dr_enable"])
+    c.dt = float(w["dt"])
+    c.mass = float(w["mass"])
+    c.inertia[:] = [float(x) for x in w["inertia"]]
+    c.added_mass[:] = [float(x) for x in w["added_mass"]]
+    c.damp_lin[:] = [float(x) for x in w["damp_lin"]]
+    c.damp_quad[:] = [float(x) for x in w["damp_quad"]]
+    c.gravity[:] = [float(x) for x in w["gravity"]]
+    c.thrust_max = float(w["thrust_max"])
+    c.alloc[:] = [float(x) for x in np.asarray(w["alloc"], dtype=np.float64).reshape(-1)]
+    for k in ("w_pos", "w_att", "w_act", "w_vs", "init_pos_range", "init_att_range",
+              "goal_pos_range", "goal_yaw_range", "current_range", "dr_scale_lo", "dr_scale_hi",
+              "dr_buoy_range", "dr_cob_range", "logstd_min", "logstd_max"):
+        setattr(c, k, float(w[k]))
+    c.hidden = int(w["hidden"])
+    c.policy_out = int(w["policy_out"])
+    c.mlp_mode = AUV_MLP_BF16 if w["mlp"] == "bf16" else AUV_MLP_FP32
+    c.has_value = int(w["has_value"])
+    c.logstd_fixed[:] = [float(x) for x in w["logstd_fixed"]]
+    return c
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+class Env:
+    """A batch of N environments on the current CUDA device.
+
+    State lives in caller-owned torch tensors (SoA): state[19][N],
+    params[17][N], t_ep[N] (int32), episode[N] (int32 storage of uint32)."""
+
+    def __init__(self, workload: dict, device=None):
+        import torch
+        self.w = dict(workload)
+        self.n = int(workload["n_envs"])
+        self.device = torch.device(device or "cuda")
+        L = lib()
+        n = self.n
+        with torch.cuda.device(self.device):
+            self.state = torch.zeros((W.STATE_FIELDS, n), dtype=torch.float32, device=self.device)
+            self.params = torch.zeros((W.PARAM_FIELDS, n), dtype=torch.float32, device=self.device)
+            self.t_ep = torch.zeros(n, dtype=torch.int32, device=self.device)
+            self.episode = torch.zeros(n, dtype=torch.int32, device=self.device)
+            self.cfg = make_config(workload)
+            bufs = AuvBuffers(self.state.data_ptr(), self.params.data_ptr(),
+                              self.t_ep.data_ptr(), self.episode.data_ptr())
+            h = C.c_void_p()
+            rc = L.env_create(C.byref(self.cfg), C.byref(bufs), C.byref(h))
+            if rc != AUV_OK:
+                raise AuvError(rc, L.env_last_error(None).decode())
+        self.h = h
+
+    # -- helpers -------------------------------------------------------------
+    def _check(self, rc):
+        if rc != AUV_OK:
+            raise AuvError(rc, lib().env_last_error(self.h).decode())
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().env_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # -- entry points ----------------------------------------------------------
+    def set_weights(self, policy, value=None, stream=None):
+        """policy/value: torch tensors (host or device) or numpy float32 arrays."""
+        keep = []
+
+        def addr(x):
+            if x is None:
+                return None
+            if isinstance(x, np.ndarray):
+                a = np.ascontiguousarray(x, dtype=np.float32)
+                keep.append(a)
+                return a.ctypes.data_as(C.c_void_p)
+            x = x.contiguous()
+            keep.append(x)
+            return C.c_void_p(x.data_ptr())
+
+        self._check(lib().env_set_weights(self.h, addr(policy), addr(value), _stream(stream)))
+
+    def reset(self, mask=None, stream=None):
+        self._check(lib().env_reset(self.h, _ptr(mask), _stream(stream)))
+
+    def rollout(self, T: int, traj: dict, stream=None):
+        t = AuvTraj(*(traj.get(k).data_ptr() if traj.get(k) is not None else None
+                      for k in ("obs", "act", "logp", "value", "rew", "done")))
+        self._check(lib().env_rollout(self.h, int(T), C.byref(t), _stream(stream)))
+
+    def value(self, obs, value, stream=None):
+        """Value network on trajectory-layout observations obs[T][18][N] -> value[T][N]."""
+        self._check(lib().env_value(self.h, _ptr(obs), int(obs.shape[0]), _ptr(value),
+                                    _stream(stream)))
+
+    def step(self, obs=None, rew=None, done=None, stream=None):
+        self._check(lib().env_step(self.h, _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))
+
+    def step_actions(self, act, rew, done, trace=None, stream=None):
+        T = act.shape[0]
+        self._check(lib().env_step_actions(self.h, _ptr(act), int(T), _ptr(rew), _ptr(done),
+                                           _ptr(trace), _stream(stream)))
+
+    def observe(self, out, stream=None):
+        self._check(lib().env_observe(self.h, _ptr(out), _stream(stream)))
+
+    def policy_forward(self, obs, head, value=None, stream=None):
+        self._check(lib().env_policy_forward(self.h, _ptr(obs), int(obs.shape[0]), _ptr(head),
+                                             _ptr(value), _stream(stream)))
+
+    def draw_words(self, stream_id: int, index: int, n_blocks: int, out, stream=None):
+        self._check(lib().env_draw_words(self.h, int(stream_id), int(index), int(n_blocks),
+                                         _ptr(out), _stream(stream)))
+
+    @property
+    def t_g(self) -> int:
+        v = C.c_uint64()
+        self._check(lib().env_get_step(self.h, C.byref(v)))
+        return int(v.value)
+
+    @t_g.setter
+    def t_g(self, value: int):
+        self._check(lib().env_set_step(self.h, int(value)))
+
+    def status(self, stream=None) -> AuvStatus:
+        s = AuvStatus()
+        lib().env_status(self.h, C.byref(s), _stream(stream))
+        return s
+
+    def clear_status(self, stream=None):
+        self._check(lib().env_clear_status(self.h, _stream(stream)))
+
+    # -- allocation helpers ----------------------------------------------------
+    def alloc_traj(self, T: int, keys=("obs", "act", "logp", "value", "rew", "done"),
+                   pinned_host: bool = False) -> dict:
+        import torch
+        n = self.n
+        shapes = dict(obs=(T, W.OBS_DIM, n), act=(T, W.ACT_DIM, n), logp=(T, n), value=(T, n),
+                      rew=(T, n), done=(T, n))
+        out = {}
+        for k in keys:
+            if k == "value" and not self.w["has_value"]:
+                continue
+            dt = torch.uint8 if k == "done" else torch.float32
+            if pinned_host:
+                out[k] = torch.empty(shapes[k], dtype=dt, pin_memory=True)
+            else:
+                out[k] = torch.empty(shapes[k], dtype=dt, device=self.device)
+        return out

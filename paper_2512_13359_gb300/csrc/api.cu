@@ -1,0 +1,511 @@
+// api.cu -- the extern "C" entry points of libauvenv.so (include/auvenv.h):
+// argument and configuration validation, the library workspace, and the
+// dispatch of each call to its kernels on the caller's stream.
+#include <climits>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "auv_kernels.h"
+#include "auv_bf16.h"
+#include "auvenv.h"
+
+using auv::Buffers;
+using auv::Model;
+using auv::Status;
+using auv::Traj;
+
+struct auv_env {
+  auv_config cfg;
+  Model model;
+  Buffers buf;
+  int device;
+  uint64_t t_g;
+  char* workspace;          // device: [status | policy weights | value weights | staging]
+  Status* status;
+  float* w_policy_f32;      // fp32 mode: row-major weights as given
+  float* w_value_f32;
+  void* w_policy_packed;    // bf16 mode: packed operand images
+  void* w_value_packed;
+  float* staging;           // fp32 copy of the caller's weights (bf16 mode)
+  size_t policy_count, value_count;
+  bool weights_set;
+  char err[256];
+};
+
+namespace {
+
+thread_local char g_create_err[256] = "";
+
+int fail(auv_env* env, int code, const char* fmt, ...) {
+  char* dst = env ? env->err : g_create_err;
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(dst, 256, fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(auv_env* env, cudaError_t e, const char* what) {
+  return fail(env, AUV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+size_t mlp_count(size_t H, size_t out) { return H * 18 + H + H * H + H + out * H + out; }
+
+bool finite_pos(float x) { return std::isfinite(x) && x > 0.0f; }
+bool finite_nonneg(float x) { return std::isfinite(x) && x >= 0.0f; }
+
+enum PtrKind { kBad, kDevice, kHostMapped };
+
+// Classifies a pointer and returns the address a kernel must use.
+PtrKind classify(const void* p, void** dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return kBad;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+    *dev = const_cast<void*>(p);
+    return kDevice;
+  }
+  if (a.type == cudaMemoryTypeHost && a.devicePointer) {
+    *dev = a.devicePointer;
+    return kHostMapped;
+  }
+  return kBad;
+}
+
+int check_device_buffer(auv_env* env, const void* p, const char* name, size_t align) {
+  void* d = nullptr;
+  if (!p) return fail(env, AUV_ERR_INVALID, "%s is NULL", name);
+  if (reinterpret_cast<uintptr_t>(p) % align)
+    return fail(env, AUV_ERR_SIZE, "%s is not %zu-byte aligned", name, align);
+  if (classify(p, &d) != kDevice) return fail(env, AUV_ERR_SIZE, "%s is not device memory", name);
+  return AUV_OK;
+}
+
+// Output buffer: device memory or mapped page-locked host memory.
+int map_output(auv_env* env, void* p, const char* name, size_t align, void** dev) {
+  *dev = nullptr;
+  if (!p) return AUV_OK;
+  if (reinterpret_cast<uintptr_t>(p) % align)
+    return fail(env, AUV_ERR_SIZE, "%s is not %zu-byte aligned", name, align);
+  if (classify(p, dev) == kBad)
+    return fail(env, AUV_ERR_SIZE, "%s is neither device memory nor mapped page-locked host memory",
+                name);
+  return AUV_OK;
+}
+
+int validate_config(const auv_config* c) {
+  if (!c) return fail(nullptr, AUV_ERR_INVALID, "cfg is NULL");
+  if (c->struct_size != sizeof(auv_config))
+    return fail(nullptr, AUV_ERR_INVALID, "cfg->struct_size %u != sizeof(auv_config) %zu",
+                c->struct_size, sizeof(auv_config));
+  if (c->n_envs < 1 || c->n_envs > (1u << 30))
+    return fail(nullptr, AUV_ERR_INVALID, "n_envs %u outside [1, 2^30]", c->n_envs);
+  if ((uint64_t)c->env_id_base + c->n_envs > (1ull << 32))
+    return fail(nullptr, AUV_ERR_INVALID, "env_id_base + n_envs exceeds 2^32");
+  if (c->substeps < 1 || c->substeps > 64)
+    return fail(nullptr, AUV_ERR_INVALID, "substeps %u outside [1, 64]", c->substeps);
+  if (c->episode_len < 1 || c->episode_len > (uint32_t)INT_MAX)
+    return fail(nullptr, AUV_ERR_INVALID, "episode_len %u invalid", c->episode_len);
+  if (!finite_pos(c->dt)) return fail(nullptr, AUV_ERR_INVALID, "dt must be finite and > 0");
+  if (!finite_pos(c->mass)) return fail(nullptr, AUV_ERR_INVALID, "mass must be > 0");
+  for (int k = 0; k < 3; ++k)
+    if (!finite_pos(c->inertia[k])) return fail(nullptr, AUV_ERR_INVALID, "inertia must be > 0");
+  for (int k = 0; k < 6; ++k) {
+    if (!finite_nonneg(c->added_mass[k]) || !finite_nonneg(c->damp_lin[k]) ||
+        !finite_nonneg(c->damp_quad[k]))
+      return fail(nullptr, AUV_ERR_INVALID, "added mass and damping must be finite and >= 0");
+  }
+  for (int k = 0; k < 3; ++k)
+    if (!std::isfinite(c->gravity[k])) return fail(nullptr, AUV_ERR_INVALID, "gravity not finite");
+  if (!finite_nonneg(c->thrust_max)) return fail(nullptr, AUV_ERR_INVALID, "thrust_max invalid");
+  for (int k = 0; k < 48; ++k)
+    if (!std::isfinite(c->alloc[k])) return fail(nullptr, AUV_ERR_INVALID, "alloc not finite");
+  const float pi = 3.14159274f;
+  if (!finite_nonneg(c->init_pos_range) || !finite_nonneg(c->goal_pos_range) ||
+      !finite_nonneg(c->current_range) || !finite_nonneg(c->init_att_range) ||
+      !finite_nonneg(c->goal_yaw_range) || c->init_att_range > pi || c->goal_yaw_range > pi)
+    return fail(nullptr, AUV_ERR_INVALID,
+                "ranges must be finite and >= 0; attitude and goal-yaw ranges <= pi");
+  if (c->dr_enable > 1) return fail(nullptr, AUV_ERR_INVALID, "dr_enable must be 0 or 1");
+  if (c->dr_enable) {
+    if (!finite_pos(c->dr_scale_lo) || !(c->dr_scale_hi >= c->dr_scale_lo) ||
+        !std::isfinite(c->dr_scale_hi) || !finite_nonneg(c->dr_buoy_range) ||
+        !finite_nonneg(c->dr_cob_range))
+      return fail(nullptr, AUV_ERR_INVALID, "domain-randomisation ranges invalid");
+  }
+  if (!std::isfinite(c->w_pos) || !std::isfinite(c->w_att) || !std::isfinite(c->w_act) ||
+      !std::isfinite(c->w_vs))
+    return fail(nullptr, AUV_ERR_INVALID, "reward weights not finite");
+  if (c->policy_out != 8 && c->policy_out != 16)
+    return fail(nullptr, AUV_ERR_INVALID, "policy_out must be 8 or 16");
+  if (c->mlp_mode != AUV_MLP_FP32 && c->mlp_mode != AUV_MLP_BF16)
+    return fail(nullptr, AUV_ERR_INVALID, "unknown mlp_mode %u", c->mlp_mode);
+  if (c->has_value > 1) return fail(nullptr, AUV_ERR_INVALID, "has_value must be 0 or 1");
+  if (!(c->logstd_min <= c->logstd_max) || !std::isfinite(c->logstd_min) ||
+      !std::isfinite(c->logstd_max))
+    return fail(nullptr, AUV_ERR_INVALID, "logstd clamp invalid");
+  for (int k = 0; k < 8; ++k)
+    if (!std::isfinite(c->logstd_fixed[k]))
+      return fail(nullptr, AUV_ERR_INVALID, "logstd_fixed not finite");
+  if (c->mlp_mode == AUV_MLP_FP32 && c->hidden != 64 && c->hidden != 256)
+    return fail(nullptr, AUV_ERR_UNSUPPORTED, "fp32 networks are built for hidden 64 or 256");
+  if (c->mlp_mode == AUV_MLP_BF16 && (c->hidden != 256 || c->policy_out != 16))
+    return fail(nullptr, AUV_ERR_UNSUPPORTED,
+                "bf16 networks are built for hidden 256 with the 16-output policy head");
+  return AUV_OK;
+}
+
+Model build_model(const auv_config* c) {
+  Model M;
+  std::memset(&M, 0, sizeof(M));
+  M.n = (int)c->n_envs;
+  M.substeps = (int)c->substeps;
+  M.episode_len = (int)c->episode_len;
+  M.seed = c->seed;
+  M.id_base = c->env_id_base;
+  M.dr_enable = (int)c->dr_enable;
+  M.policy_out = (int)c->policy_out;
+  M.has_value = (int)c->has_value;
+  M.hidden = (int)c->hidden;
+  M.h = c->dt / (float)c->substeps;
+  M.mass = c->mass;
+  for (int k = 0; k < 3; ++k) M.inertia[k] = c->inertia[k];
+  for (int k = 0; k < 6; ++k) {
+    M.added[k] = c->added_mass[k];
+    M.dlin[k] = c->damp_lin[k];
+    M.dquad[k] = c->damp_quad[k];
+  }
+  const double g0 = c->gravity[0], g1 = c->gravity[1], g2 = c->gravity[2];
+  const double gn = std::sqrt(g0 * g0 + g1 * g1 + g2 * g2);
+  M.gnorm = (float)gn;
+  if (gn > 0) {
+    M.ghat[0] = (float)(g0 / gn);
+    M.ghat[1] = (float)(g1 / gn);
+    M.ghat[2] = (float)(g2 / gn);
+  }
+  for (int k = 0; k < 48; ++k) M.alloc_t[k] = c->alloc[k] * c->thrust_max;
+  M.w_pos = c->w_pos; M.w_att = c->w_att; M.w_act = c->w_act; M.w_vs = c->w_vs;
+  M.init_pos_range = c->init_pos_range;
+  M.init_att_range = c->init_att_range;
+  M.goal_pos_range = c->goal_pos_range;
+  M.goal_yaw_range = c->goal_yaw_range;
+  M.current_range = c->current_range;
+  M.dr_lo = c->dr_scale_lo; M.dr_hi = c->dr_scale_hi;
+  M.dr_buoy = c->dr_buoy_range; M.dr_cob = c->dr_cob_range;
+  for (int k = 0; k < 8; ++k) M.logstd_fixed[k] = c->logstd_fixed[k];
+  M.logstd_min = c->logstd_min; M.logstd_max = c->logstd_max;
+  return M;
+}
+
+int check_device(auv_env* env) {
+  int cur = -1;
+  cudaError_t e = cudaGetDevice(&cur);
+  if (e != cudaSuccess) return cuda_fail(env, e, "cudaGetDevice");
+  if (cur != env->device)
+    return fail(env, AUV_ERR_INVALID, "device %d is current but the env lives on device %d", cur,
+                env->device);
+  return AUV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int env_abi_version(void) { return AUV_ABI_VERSION; }
+
+const char* env_last_error(const auv_env* env) { return env ? env->err : g_create_err; }
+
+int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
+  g_create_err[0] = 0;
+  if (!out) return fail(nullptr, AUV_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  int rc = validate_config(cfg);
+  if (rc) return rc;
+  if (!buf) return fail(nullptr, AUV_ERR_INVALID, "buf is NULL");
+  if ((rc = check_device_buffer(nullptr, buf->state, "state", 16))) return rc;
+  if ((rc = check_device_buffer(nullptr, buf->params, "params", 16))) return rc;
+  if ((rc = check_device_buffer(nullptr, buf->t_ep, "t_ep", 16))) return rc;
+  if ((rc = check_device_buffer(nullptr, buf->episode, "episode", 16))) return rc;
+  auv_env* env = new (std::nothrow) auv_env;
+  if (!env) return fail(nullptr, AUV_ERR_INVALID, "out of host memory");
+  std::memset(env, 0, sizeof(*env));
+  env->cfg = *cfg;
+  env->model = build_model(cfg);
+  env->buf.state = buf->state;
+  env->buf.params = buf->params;
+  env->buf.t_ep = buf->t_ep;
+  env->buf.episode = buf->episode;
+  cudaGetDevice(&env->device);
+  env->policy_count = mlp_count(cfg->hidden, cfg->policy_out);
+  env->value_count = cfg->has_value ? mlp_count(cfg->hidden, 1) : 0;
+  // workspace: status (256 B) | fp32 policy | fp32 value | packed bf16 images
+  size_t off = 256;
+  const size_t pol_off = off;
+  off += ((env->policy_count * 4 + 255) / 256) * 256;
+  const size_t val_off = off;
+  off += ((env->value_count * 4 + 255) / 256) * 256;
+  size_t pol_pk_off = 0, val_pk_off = 0;
+  if (cfg->mlp_mode == AUV_MLP_BF16) {
+    pol_pk_off = off;
+    off += ((auv::bf16_policy_image_bytes() + 1023) / 1024) * 1024;
+    val_pk_off = off;
+    off += ((auv::bf16_value_image_bytes() + 1023) / 1024) * 1024;
+  }
+  cudaError_t e = cudaMalloc(&env->workspace, off);
+  if (e != cudaSuccess) {
+    delete env;
+    return cuda_fail(nullptr, e, "cudaMalloc(workspace)");
+  }
+  env->status = reinterpret_cast<Status*>(env->workspace);
+  env->w_policy_f32 = reinterpret_cast<float*>(env->workspace + pol_off);
+  env->w_value_f32 = cfg->has_value ? reinterpret_cast<float*>(env->workspace + val_off) : nullptr;
+  if (cfg->mlp_mode == AUV_MLP_BF16) {
+    env->w_policy_packed = env->workspace + pol_pk_off;
+    env->w_value_packed = env->workspace + val_pk_off;
+  }
+  Status s0 = {0, 0, INT_MAX, 0};
+  e = cudaMemcpy(env->status, &s0, sizeof(s0), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cudaFree(env->workspace);
+    delete env;
+    return cuda_fail(nullptr, e, "init status");
+  }
+  *out = env;
+  return AUV_OK;
+}
+
+int env_destroy(auv_env* env) {
+  if (!env) return AUV_ERR_INVALID;
+  cudaDeviceSynchronize();
+  cudaError_t e = cudaFree(env->workspace);
+  delete env;
+  return e == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
+}
+
+int env_set_weights(auv_env* env, const float* policy, const float* value, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!policy) return fail(env, AUV_ERR_INVALID, "policy weights are NULL");
+  if (env->cfg.has_value && !value) return fail(env, AUV_ERR_INVALID, "value weights are NULL");
+  if (!env->cfg.has_value && value)
+    return fail(env, AUV_ERR_INVALID, "value weights given but has_value = 0");
+  cudaError_t e = cudaMemcpyAsync(env->w_policy_f32, policy, env->policy_count * 4,
+                                  cudaMemcpyDefault, s);
+  if (e != cudaSuccess) return cuda_fail(env, e, "copy policy weights");
+  if (value) {
+    e = cudaMemcpyAsync(env->w_value_f32, value, env->value_count * 4, cudaMemcpyDefault, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "copy value weights");
+  }
+  if (env->cfg.mlp_mode == AUV_MLP_BF16) {
+    e = auv::launch_pack_bf16(env->model, env->w_policy_f32, env->w_value_f32,
+                              env->w_policy_packed, env->w_value_packed, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "pack bf16 weights");
+  }
+  // host sources are read before return
+  void* d = nullptr;
+  if (classify(policy, &d) != kDevice || (value && classify(value, &d) != kDevice)) {
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "synchronise weight upload");
+  }
+  env->weights_set = true;
+  return AUV_OK;
+}
+
+int env_reset(auv_env* env, const uint8_t* mask, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (mask && (rc = check_device_buffer(env, mask, "mask", 1))) return rc;
+  cudaError_t e = auv::launch_reset(env->model, env->buf, mask, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "reset kernel");
+}
+
+int env_rollout(auv_env* env, int T, const auv_traj* traj, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (T < 1) return fail(env, AUV_ERR_INVALID, "T must be >= 1");
+  if (!env->weights_set) return fail(env, AUV_ERR_INVALID, "weights not set");
+  Traj tr = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  if (traj) {
+    void* d;
+    if ((rc = map_output(env, traj->obs, "traj.obs", 4, &d))) return rc;
+    tr.obs = static_cast<float*>(d);
+    if ((rc = map_output(env, traj->act, "traj.act", 4, &d))) return rc;
+    tr.act = static_cast<float*>(d);
+    if ((rc = map_output(env, traj->logp, "traj.logp", 4, &d))) return rc;
+    tr.logp = static_cast<float*>(d);
+    if ((rc = map_output(env, traj->value, "traj.value", 4, &d))) return rc;
+    tr.value = static_cast<float*>(d);
+    if ((rc = map_output(env, traj->rew, "traj.rew", 4, &d))) return rc;
+    tr.rew = static_cast<float*>(d);
+    if ((rc = map_output(env, traj->done, "traj.done", 1, &d))) return rc;
+    tr.done = static_cast<uint8_t*>(d);
+  }
+  if (tr.value && !env->cfg.has_value)
+    return fail(env, AUV_ERR_INVALID, "traj.value requested but has_value = 0");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (env->cfg.mlp_mode == AUV_MLP_FP32) {
+    e = auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32, env->w_value_f32, tr, T,
+                                 env->t_g, env->status, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "fp32 rollout kernel");
+  } else {
+    if (tr.value && !tr.obs)
+      return fail(env, AUV_ERR_INVALID, "bf16 mode computes traj.value from traj.obs: give both");
+    e = auv::launch_rollout_bf16(env->model, env->buf, env->w_policy_packed, tr, T, env->t_g,
+                                 env->status, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "bf16 rollout kernel");
+    if (tr.value) {
+      e = auv::launch_value_bf16(env->model, env->w_value_packed, env->w_value_f32, tr.obs,
+                                 (size_t)T * env->model.n, env->model.n, tr.value, env->status, s);
+      if (e != cudaSuccess) return cuda_fail(env, e, "bf16 value kernel");
+    }
+  }
+  env->t_g += (uint64_t)T;
+  return AUV_OK;
+}
+
+int env_value(auv_env* env, const float* obs, int T, float* value, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (T < 1) return fail(env, AUV_ERR_INVALID, "T must be >= 1");
+  if (!env->cfg.has_value) return fail(env, AUV_ERR_INVALID, "has_value = 0");
+  if (!env->weights_set) return fail(env, AUV_ERR_INVALID, "weights not set");
+  void *o, *v;
+  if (!obs || !value) return fail(env, AUV_ERR_INVALID, "obs and value are required");
+  if ((rc = map_output(env, const_cast<float*>(obs), "obs", 4, &o))) return rc;
+  if ((rc = map_output(env, value, "value", 4, &v))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t rows = (size_t)T * env->model.n;
+  cudaError_t e;
+  if (env->cfg.mlp_mode == AUV_MLP_FP32)
+    e = auv::launch_value_fp32(env->model, env->w_value_f32, static_cast<const float*>(o), rows,
+                               env->model.n, static_cast<float*>(v), s);
+  else
+    e = auv::launch_value_bf16(env->model, env->w_value_packed, env->w_value_f32,
+                               static_cast<const float*>(o), rows, env->model.n,
+                               static_cast<float*>(v), env->status, s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "value kernel");
+}
+
+int env_step(auv_env* env, float* obs_out, float* rew_out, uint8_t* done_out, void* stream) {
+  auv_traj tr = {obs_out, nullptr, nullptr, nullptr, rew_out, done_out};
+  return env_rollout(env, 1, &tr, stream);
+}
+
+int env_step_actions(auv_env* env, const float* act, int T, float* rew_out, uint8_t* done_out,
+                     float* state_trace, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (T < 1) return fail(env, AUV_ERR_INVALID, "T must be >= 1");
+  if ((rc = check_device_buffer(env, act, "act", 4))) return rc;
+  void *rew, *done, *trace;
+  if (!rew_out || !done_out) return fail(env, AUV_ERR_INVALID, "rew_out and done_out are required");
+  if ((rc = map_output(env, rew_out, "rew_out", 4, &rew))) return rc;
+  if ((rc = map_output(env, done_out, "done_out", 1, &done))) return rc;
+  if ((rc = map_output(env, state_trace, "state_trace", 4, &trace))) return rc;
+  cudaError_t e = auv::launch_replay(env->model, env->buf, act, T, static_cast<float*>(rew),
+                                     static_cast<uint8_t*>(done), static_cast<float*>(trace),
+                                     env->status, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "replay kernel");
+}
+
+int env_observe(auv_env* env, float* obs_out, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  void* d;
+  if (!obs_out) return fail(env, AUV_ERR_INVALID, "obs_out is NULL");
+  if ((rc = map_output(env, obs_out, "obs_out", 4, &d))) return rc;
+  cudaError_t e = auv::launch_observe(env->model, env->buf, static_cast<float*>(d),
+                                      static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "observe kernel");
+}
+
+int env_policy_forward(auv_env* env, const float* obs, int n, float* head, float* value,
+                       void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (n < 1) return fail(env, AUV_ERR_INVALID, "n must be >= 1");
+  if (!env->weights_set) return fail(env, AUV_ERR_INVALID, "weights not set");
+  if ((rc = check_device_buffer(env, obs, "obs", 4))) return rc;
+  if ((rc = check_device_buffer(env, head, "head", 4))) return rc;
+  if (value && !env->cfg.has_value) return fail(env, AUV_ERR_INVALID, "value but has_value = 0");
+  if (value && (rc = check_device_buffer(env, value, "value", 4))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (env->cfg.mlp_mode == AUV_MLP_FP32)
+    e = auv::launch_forward_fp32(env->model, env->w_policy_f32, env->w_value_f32, obs, n, head,
+                                 value, s);
+  else
+    e = auv::launch_forward_bf16(env->model, env->w_policy_packed, env->w_value_packed,
+                                 env->w_value_f32, obs, n, head, value, env->status, s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "forward kernel");
+}
+
+int env_draw_words(auv_env* env, uint32_t stream_id, uint64_t index, int n_blocks, uint32_t* out,
+                   void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (n_blocks < 1 || n_blocks > 64) return fail(env, AUV_ERR_INVALID, "n_blocks outside [1, 64]");
+  if ((rc = check_device_buffer(env, out, "out", 4))) return rc;
+  cudaError_t e = auv::launch_draw_words(env->model, stream_id, index, n_blocks, out,
+                                         static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "draw-words kernel");
+}
+
+int env_get_step(const auv_env* env, uint64_t* t_g) {
+  if (!env || !t_g) return AUV_ERR_INVALID;
+  *t_g = env->t_g;
+  return AUV_OK;
+}
+
+int env_set_step(auv_env* env, uint64_t t_g) {
+  if (!env) return AUV_ERR_INVALID;
+  env->t_g = t_g;
+  return AUV_OK;
+}
+
+int env_status(auv_env* env, auv_status* out, void* stream) {
+  if (!env || !out) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(env, e, "synchronise");
+  Status st;
+  e = cudaMemcpy(&st, env->status, sizeof(st), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(env, e, "read status");
+  out->code = st.code;
+  out->nan_flag = st.nan_flag;
+  out->first_nan_env = st.first_nan_env == INT_MAX ? -1 : st.first_nan_env;
+  out->timeouts = st.timeouts;
+  if (st.code != 0)
+    fail(env, st.code, "device status %d (nan_flag %d, first env %d, timeouts %d)", st.code,
+         st.nan_flag, out->first_nan_env, st.timeouts);
+  return st.code;
+}
+
+int env_clear_status(auv_env* env, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  static const Status s0 = {0, 0, INT_MAX, 0};
+  cudaError_t e = cudaMemcpyAsync(env->status, &s0, sizeof(s0), cudaMemcpyHostToDevice,
+                                  static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "clear status");
+}
+
+}  // extern "C"

@@ -1,0 +1,32 @@
+// auv_bf16.h -- internal interface of the tensor-core (tcgen05, bf16 operands,
+// fp32 accumulation in tensor memory) network path.
+#pragma once
+
+#include "auv_kernels.h"
+
+namespace auv {
+
+// Bytes of the packed operand images the bf16 kernels stream into shared
+// memory (policy and value networks, hidden width 256).
+size_t bf16_policy_image_bytes();
+size_t bf16_value_image_bytes();
+
+// fp32 row-major weights -> packed bf16 images (round to nearest even).
+cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* wv_f32,
+                             void* wp_packed, void* wv_packed, cudaStream_t s);
+
+// Fused rollout with the policy network on tcgen05.
+cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp_packed,
+                                const Traj& tr, int T, uint64_t t_g0, Status* st, cudaStream_t s);
+
+// Value network over `rows` stored observations obs[t][18][n] (row r = t*n + i).
+cudaError_t launch_value_bf16(const Model& M, const void* wv_packed, const float* wv_f32,
+                              const float* obs, size_t rows, int n, float* value, Status* st,
+                              cudaStream_t s);
+
+// Networks on caller observations obs[n][18] (row-major).
+cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const void* wv_packed,
+                                const float* wv_f32, const float* obs, int n, float* head,
+                                float* value, Status* st, cudaStream_t s);
+
+}  // namespace auv

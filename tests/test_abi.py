@@ -1,0 +1,99 @@
+"""The C-ABI library builds, loads, exports every entry point that
+include/auvenv.h declares, and rejects bad configurations before touching
+the GPU (no compute calls here)."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "auvenv.h")
+
+
+@pytest.fixture(scope="module")
+def auvlib():
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    return auvenv.lib()
+
+
+def header_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\**\s*(env_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_entry_points():
+    names = header_functions()
+    for must in ("env_create", "env_reset", "env_step", "env_rollout", "env_step_actions"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(auvlib):
+    from paper_2512_13359_gb300 import auvenv
+    names = header_functions()
+    assert sorted(auvenv.EXPORTED) == names
+    out = subprocess.run(["nm", "-D", "--defined-only", auvenv.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT\s+(\w+)$", out, flags=re.M))
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        assert hasattr(auvlib, n)
+    assert auvlib.env_abi_version() == 1
+
+
+def test_config_struct_size_matches_header(auvlib):
+    """sizeof(auv_config) as compiled equals the binding's mirror: a create
+    with the binding's size passes the version guard, any other size fails."""
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    cfg = auvenv.make_config(W.workload("tiny_64"))
+    h = C.c_void_p()
+    cfg.struct_size = C.sizeof(auvenv.AuvConfig) + 4
+    rc = auvlib.env_create(C.byref(cfg), None, C.byref(h))
+    assert rc == auvenv.AUV_ERR_INVALID
+    assert b"struct_size" in auvlib.env_last_error(None)
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("n_envs", 0, -1), ("substeps", 0, -1), ("substeps", 65, -1), ("episode_len", 0, -1),
+    ("dt", 0.0, -1), ("dt", float("nan"), -1), ("mass", -1.0, -1), ("policy_out", 12, -1),
+    ("mlp_mode", 7, -1), ("goal_yaw_range", 4.0, -1), ("hidden", 128, -6),
+])
+def test_invalid_configs_are_rejected(auvlib, field, value, code):
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    cfg = auvenv.make_config(W.workload("tiny_64"))
+    setattr(cfg, field, value)
+    h = C.c_void_p()
+    rc = auvlib.env_create(C.byref(cfg), None, C.byref(h))
+    assert rc == code, auvlib.env_last_error(None)
+    assert not h.value
+
+
+def test_bf16_mode_requires_the_built_shape(auvlib):
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    cfg = auvenv.make_config(W.workload("ppo_65536", hidden=64))
+    h = C.c_void_p()
+    assert auvlib.env_create(C.byref(cfg), None, C.byref(h)) == auvenv.AUV_ERR_UNSUPPORTED
+
+
+def test_null_arguments(auvlib):
+    from paper_2512_13359_gb300 import auvenv
+    h = C.c_void_p()
+    assert auvlib.env_create(None, None, C.byref(h)) == auvenv.AUV_ERR_INVALID
+    assert auvlib.env_destroy(None) == auvenv.AUV_ERR_INVALID
+    assert auvlib.env_reset(None, None, None) == auvenv.AUV_ERR_INVALID
+    assert auvlib.env_rollout(None, 1, None, None) == auvenv.AUV_ERR_INVALID
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    from paper_2512_13359_gb300 import auvenv
+    saved = auvenv._lib
+    auvenv._lib = None
+    try:
+        with pytest.raises(auvenv.LibraryMissing):
+            auvenv.lib(str(tmp_path / "missing.so"))
+    finally:
+        auvenv._lib = saved
