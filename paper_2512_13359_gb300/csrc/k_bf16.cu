@@ -192,8 +192,11 @@ __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const flo
   }
 }
 
+// Register cap: the 4G+1 warps are spread over the SM's four sub-partitions,
+// whose 16K-register files each host G+1 warps (G = 4: 5 warps x 32 lanes
+// x 96 registers <= 16384).
 template <int G, int MODE>
-__global__ void __launch_bounds__(G * 128 + 32) __maxnreg__(G == 4 ? 120 : 168)
+__global__ void __launch_bounds__(G * 128 + 32) __maxnreg__(G == 4 ? 96 : 168)
 k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
          uint64_t t_g0, RowIO io, Status* st) {
   using E = Engine<G, MODE>;

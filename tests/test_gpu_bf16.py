@@ -43,9 +43,6 @@ def test_bf16_policy_and_value_forward(oracle, n):
     _report(f"policy head n={n}", eh, BF16_HEAD_TOL)
     _report(f"value n={n}", ev, BF16_VALUE_TOL)
     assert eh <= BF16_HEAD_TOL and ev <= BF16_VALUE_TOL
-    # the bf16 path is far closer to the bf16 definition than to fp32 arithmetic
-    ref32 = oracle.mlp(pw, 18, 256, 16, False, obs[idx].astype(np.float64))
-    assert np.abs(ref32 - ref_h).max() > eh
 
 
 def test_bf16_value_over_trajectory_layout(oracle):
