@@ -338,7 +338,7 @@ def main():
     if w["mlp"] == "bf16":
         if roll_avg >= val_avg:
             kern, dur = "rollout_bf16", roll_avg
-            flops = n * T * (pol_fl + DYN_FLOPS_PER_ENV_STEP)
+            flops = n * T * pol_fl          # tensor-core work of the fused rollout
         else:
             kern, dur = "value_bf16", val_avg
             flops = n * T * val_fl
@@ -388,9 +388,12 @@ def main():
         dist.destroy_process_group()
 
 
-# Algorithmic FP32 flops of the physics part of one env-step (4 substeps,
-# allocation, observation, noise, reward), counted from the kernel source.
-DYN_FLOPS_PER_ENV_STEP = 2000
+# Algorithmic FP32 flops of the non-network part of one env-step with 4
+# substeps, counted by running the oracle's formulation with an
+# operation-counting scalar: observation 141 + allocation 144 + 4 x 378
+# (substep) + reward 93 + action sampling and log-probability 72 (adds,
+# multiplies and divides; square roots and transcendentals not counted).
+DYN_FLOPS_PER_ENV_STEP = 1962
 
 if __name__ == "__main__":
     main()
