@@ -237,6 +237,33 @@ int env_policy_forward(auv_env* env, const float* obs, int n, float* head, float
 int env_draw_words(auv_env* env, uint32_t stream_id, uint64_t index, int n_blocks,
                    uint32_t* out, void* stream);
 
+/*
+ * env_policy_forward_noalloc: the same network evaluation as
+ * env_policy_forward in AUV_MLP_BF16 mode, for callers that must not allocate
+ * device memory, e.g. an on-vehicle control loop with a hard period (an
+ * allocation can synchronise the device) or a host application that owns a
+ * fixed device-memory budget.  The paper has no counterpart; this is a
+ * library convenience.
+ *  - No handle and no allocation: the packed weights and a status word live
+ *    in one static device array of 312.25 KiB that every GPU loading this
+ *    library holds until the process exits.  The first call on a device looks
+ *    up that array's address (once per device); make it before any stream
+ *    capture.
+ *  - hidden must be 256 and policy_out 16 (the built tensor-core shape);
+ *    larger values return AUV_ERR_SIZE (the packed weights would not fit
+ *    the array), other values AUV_ERR_UNSUPPORTED.
+ *  - policy[, value_w]: fp32 weights in the env_set_weights layout; obs[n][18]
+ *    (row-major); outputs head[n][policy_out] and, iff value_w is given,
+ *    value[n].  All device memory, 16-byte aligned; n >= 1.
+ *  - Every call on a device shares the array and leaves its contents there:
+ *    calls that overlap on the GPU (other streams, other host threads) race
+ *    on it and must be serialised by the caller.  Device-side wait timeouts
+ *    are not reported by this entry point.
+ */
+int env_policy_forward_noalloc(int hidden, int policy_out, const float* policy,
+                               const float* value_w, const float* obs, int n, float* head,
+                               float* value, void* stream);
+
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);

@@ -29,7 +29,7 @@ AUV_MLP_BF16 = 1
 EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
-            "env_status", "env_clear_status")
+            "env_status", "env_clear_status", "env_policy_forward_noalloc")
 
 
 class LibraryMissing(RuntimeError):
@@ -110,6 +110,7 @@ def lib(path: str | None = None):
     L.env_set_step.argtypes = [P, C.c_uint64]
     L.env_status.argtypes = [P, C.POINTER(AuvStatus), P]
     L.env_clear_status.argtypes = [P, P]
+    L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
