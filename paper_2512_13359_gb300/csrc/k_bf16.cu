@@ -7,8 +7,9 @@
 // One CTA per SM holds the network's weights in shared memory as pre-swizzled
 // bf16 images for the whole launch.  Its threads form G groups of 128 (one
 // row -- one environment -- per thread, which is also that row's tensor-memory
-// lane) plus one MMA-issuing warp.  The groups take turns on the tensor pipe:
-// while one group's network runs, the others integrate their environments.
+// lane) plus two MMA-issuing warps (layer 1; layers 2 and 3).  The groups take
+// turns on the tensor pipe: while one group's network runs, the others
+// integrate their environments.
 //
 // Per 128-row tile and control step:
 //   layer 1: A = observation tile (smem, K = 32 with 18 used), 4 N-chunks of 64
@@ -19,8 +20,9 @@
 //   layer 3 (policy): A = h2 chunk (smem), B = W3 K-slice, accumulated over
 //             the 4 chunks into a 16-column fp32 accumulator
 //
-// Tensor-memory columns: acc[0] 0..63, acc[1] 64..127, h1 128..255 (bf16
-// pairs), acc3 256..271.
+// Tensor-memory columns: h1 slots 0..127 and 128..255 (bf16 pairs), layer-1
+// accumulator X 256..319, layer-2 accumulators Y 320..383 and Z 384..447,
+// head accumulators 448..463 and 464..479.
 #include <climits>
 
 #include "auv_bf16.h"
@@ -60,7 +62,11 @@ constexpr uint32_t kObsTileBytes = kRows * 64;    // SW64, K = 32
 constexpr uint32_t kH2TileBytes = kRows * 128;    // SW128, K = 64
 
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColAcc0 = 0, kColAcc1 = 64, kColH1 = 128, kColAcc3 = 256;
+constexpr uint32_t kColH1 = 0;      // two h1 slots of 128 columns (bf16 pairs)
+constexpr uint32_t kColX = 256;     // layer-1 chunk accumulator (64 fp32 columns)
+constexpr uint32_t kColY = 320;     // layer-2 even-chunk accumulator
+constexpr uint32_t kColZ = 384;     // layer-2 odd-chunk accumulator
+constexpr uint32_t kColA3 = 448;    // two head accumulators of 16 columns
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per wait
 
@@ -132,14 +138,17 @@ __global__ void k_pack(const float* __restrict__ w, int out_dim, uint8_t* __rest
 // engine
 // -------------------------------------------------------------------------
 struct Barriers {
-  uint64_t obs_full[4];
-  uint64_t acc_full[4][2];
-  uint64_t acc3_full[4];
-  uint64_t acc_empty[2];
-  uint64_t h2_full[2];
-  uint64_t acc3_empty;
-  uint64_t h1_full;
-  uint64_t drain;
+  uint64_t obs_full[4];     // group g's observation tile written (128 arrivals)
+  uint64_t full_x[4];       // layer-1 chunk of group g in X (MMA commit)
+  uint64_t full_y[4];       // layer-2 even chunk of group g in Y
+  uint64_t full_z[4];       // layer-2 odd chunk of group g in Z
+  uint64_t acc3_full[4];    // head accumulator of group g complete
+  uint64_t empty_x, empty_y, empty_z;   // accumulator read back (128 arrivals)
+  uint64_t h1_full[2];      // h1 slot complete (128 arrivals)
+  uint64_t h2_full[2];      // h2 buffer written (128 arrivals)
+  uint64_t acc3_empty[2];   // head slot read back (128 arrivals)
+  uint64_t h1_free[2];      // layer-2 MMAs reading an h1 slot completed (commit)
+  uint64_t drain, drain1;
   uint32_t tmem_base;
   int abort;
 };
@@ -160,7 +169,7 @@ struct Engine {
   static constexpr uint32_t kOffH2 = kOffObs + G * kObsTileBytes;
   static constexpr uint32_t kOffBar = kOffH2 + (kPolicy ? 2 * kH2TileBytes : 0);
   static constexpr uint32_t kSmem = kOffBar + sizeof(Barriers) + 1024;   // + alignment slack
-  static constexpr int kThreads = G * kRows + 32;
+  static constexpr int kThreads = G * kRows + 64;
 };
 
 // Row r of the observation tile (bf16, K = 32, 64-byte swizzle): 4 pieces of
@@ -192,11 +201,32 @@ __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const flo
   }
 }
 
-// Register cap: the 4G+1 warps are spread over the SM's four sub-partitions,
-// whose 16K-register files each host G+1 warps (G = 4: 5 warps x 32 lanes
-// x 96 registers <= 16384).
+// Group-steps are numbered in the order the MMA warp serves them: iteration
+// it of every group that still has work, groups in ascending order (the
+// groups with work always form a prefix).  Index of (it, g):
+template <int G>
+__device__ __forceinline__ int step_index(int it, int g, const int (&iters)[G]) {
+  int k = g;
+#pragma unroll
+  for (int j = 0; j < G; ++j) k += min(it, iters[j]);
+  return k;
+}
+
+// Register cap: the 4G+2 warps are spread over the SM's four sub-partitions,
+// whose 16K-register files each host up to G+1 warps (G = 4: 5 warps x 32
+// lanes x 96 registers <= 16384).
+//
+// Schedule.  Two group-steps are in flight: while the tensor pipe runs layer 2
+// (and layer 3) of group-step k-1, it also runs layer 1 of group-step k, whose
+// epilogue fills the other h1 slot (the MMA thread's event loop is described
+// at its code).  Accumulator roles are fixed: X holds
+// layer-1 chunks, Y and Z the even and odd layer-2 chunks; h1 and the head
+// accumulator alternate between two slots by group-step parity.  Every reuse
+// of a buffer is ordered either by an "empty" barrier the MMA thread waits on
+// or by a commit: an epilogue only starts after a commit that covers every
+// MMA issued before it.
 template <int G, int MODE>
-__global__ void __launch_bounds__(G * 128 + 32) __maxnreg__(G == 4 ? 96 : 168)
+__global__ void __launch_bounds__(G * 128 + 64) __maxnreg__(G == 4 ? 96 : 168)
 k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
          uint64_t t_g0, RowIO io, Status* st) {
   using E = Engine<G, MODE>;
@@ -208,23 +238,28 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
   volatile int* abort = &bar->abort;
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
-  const bool is_mma_warp = warp == 4 * G;
+  const bool is_mma_warp = warp >= 4 * G;
 
   // ---- set-up: barriers, weights, tensor memory ----
   if (tid == 0) {
     for (int g = 0; g < G; ++g) {
       tc::mbar_init(&bar->obs_full[g], kRows);
-      tc::mbar_init(&bar->acc_full[g][0], 1);
-      tc::mbar_init(&bar->acc_full[g][1], 1);
+      tc::mbar_init(&bar->full_x[g], 1);
+      tc::mbar_init(&bar->full_y[g], 1);
+      tc::mbar_init(&bar->full_z[g], 1);
       tc::mbar_init(&bar->acc3_full[g], 1);
     }
-    tc::mbar_init(&bar->acc_empty[0], kRows);
-    tc::mbar_init(&bar->acc_empty[1], kRows);
-    tc::mbar_init(&bar->h2_full[0], kRows);
-    tc::mbar_init(&bar->h2_full[1], kRows);
-    tc::mbar_init(&bar->acc3_empty, kRows);
-    tc::mbar_init(&bar->h1_full, kRows);
+    tc::mbar_init(&bar->empty_x, kRows);
+    tc::mbar_init(&bar->empty_y, kRows);
+    tc::mbar_init(&bar->empty_z, kRows);
+    for (int s = 0; s < 2; ++s) {
+      tc::mbar_init(&bar->h1_full[s], kRows);
+      tc::mbar_init(&bar->h2_full[s], kRows);
+      tc::mbar_init(&bar->acc3_empty[s], kRows);
+      tc::mbar_init(&bar->h1_free[s], 1);
+    }
     tc::mbar_init(&bar->drain, 1);
+    tc::mbar_init(&bar->drain1, 1);
     bar->abort = 0;
     tc::mbar_fence_init();
   }
@@ -234,7 +269,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     for (uint32_t i = tid; i < E::kImage / 16; i += blockDim.x) dst[i] = __ldg(src + i);
   }
   tc::fence_async_smem();
-  if (is_mma_warp) {
+  if (warp == 4 * G) {
     tc::tmem_alloc(&bar->tmem_base, kTmemCols);
     tc::tmem_relinquish();
   }
@@ -249,99 +284,129 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
                                        : (int)((io.rows + kRows - 1) / kRows);
   const int slot0 = blockIdx.x * G;
   const int n_slots = gridDim.x * G;
-  auto group_iters = [&](int g) -> int {
+  int iters[G];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
     const int s = slot0 + g;
-    if (MODE == kRollout) return s < n_tiles ? T : 0;
-    return s < n_tiles ? (n_tiles - s - 1) / n_slots + 1 : 0;
-  };
+    iters[g] = MODE == kRollout ? (s < n_tiles ? T : 0)
+                                : (s < n_tiles ? (n_tiles - s - 1) / n_slots + 1 : 0);
+  }
 
   if (is_mma_warp) {
-    // =================== MMA issue (one elected lane) ===================
+    // =================== MMA issue: two streams, one elected lane each ===================
+    // Warp 4G issues layers 2 and 3 of each group-step once its h1 is
+    // complete, in the order L2 c0, L2 c1, L3 c0, L2 c2, L3 c1, L2 c3, L3 c2,
+    // L3 c3 (value mode: L2 c0..c3).  Warp 4G+1 issues layer 1 of each
+    // group-step into X chunk by chunk.  Each thread blocks (suspended by the
+    // hardware) only on the barrier of its own next operation, so neither
+    // stream waits behind the other's epilogue.  Before layer 1 of step k the
+    // layer-1 thread waits until the layer-2 MMAs of step k-2, which read the
+    // same h1 slot, have completed (h1_free).
     if ((tid & 31) == 0) {
       constexpr uint32_t kI64 = tc::idesc_bf16_f32(128, kChunk);
       constexpr uint32_t kI16 = tc::idesc_bf16_f32(128, kHeadOut);
-      const uint32_t tacc[2] = {tmem + kColAcc0, tmem + kColAcc1};
-      uint32_t use_acc[2] = {0, 0}, use_h1 = 0, use_h2[2] = {0, 0}, use_acc3 = 0;
-      uint32_t obs_phase[4] = {0, 0, 0, 0};
-      int max_iters = 0;
-      for (int g = 0; g < G; ++g) max_iters = max(max_iters, group_iters(g));
-      bool ok = true;
-      auto acquire_acc = [&](int b) -> bool {
-        const bool r = tc::mbar_wait(&bar->acc_empty[b], (use_acc[b] & 1u) ^ 1u, abort,
-                                     kWaitLimitNs);
-        ++use_acc[b];
-        tc::tc_fence_after();
-        return r;
-      };
-      auto issue_l2 = [&](int g, int c) -> bool {
-        const int b = c & 1;
-        if (!acquire_acc(b)) return false;
-#pragma unroll 1
-        for (int kk = 0; kk < 16; ++kk) {
-          const uint64_t bd = tc::smem_desc(
-              s_base + kOffW2 + (kk >> 2) * (kH * 128) + c * kChunk * 128 + (kk & 3) * 32, 1024, 2);
-          tc::mma_ts(tacc[b], tmem + kColH1 + kk * 8, bd, kI64, kk > 0 ? 1u : 0u);
+      int total = 0;
+#pragma unroll
+      for (int g = 0; g < G; ++g) total += iters[g];
+      auto advance = [&](int& it, int& g) {
+        ++g;
+        if (g >= G || iters[g] <= it) {
+          g = 0;
+          ++it;
         }
-        tc::mma_commit(&bar->acc_full[g][b]);
-        return true;
       };
-      for (int it = 0; it < max_iters && ok; ++it) {
-        for (int g = 0; g < G && ok; ++g) {
-          if (it >= group_iters(g)) continue;
-          // layer 1
-          ok = tc::mbar_wait(&bar->obs_full[g], obs_phase[g] & 1u, abort, kWaitLimitNs);
-          ++obs_phase[g];
+      bool ok = true;
+      int it = 0, g = 0;
+      if (warp == 4 * G) {
+        uint32_t u_y = 0, u_z = 0, u_h1[2] = {0, 0}, u_h2[2] = {0, 0}, u_a3[2] = {0, 0};
+        auto issue_l2 = [&](int k, int g2, int c) -> bool {
+          const int s2 = k & 1;
+          const bool odd = c & 1;
+          uint32_t& u = odd ? u_z : u_y;
+          const bool r = tc::mbar_wait(odd ? &bar->empty_z : &bar->empty_y, (u & 1u) ^ 1u, abort,
+                                       kWaitLimitNs);
+          ++u;
+          if (!r) return false;
+          tc::tc_fence_after();
+          const uint32_t d = tmem + (odd ? kColZ : kColY);
+#pragma unroll 1
+          for (int kk = 0; kk < 16; ++kk) {
+            const uint64_t bd = tc::smem_desc(
+                s_base + kOffW2 + (kk >> 2) * (kH * 128) + c * kChunk * 128 + (kk & 3) * 32, 1024, 2);
+            tc::mma_ts(d, tmem + kColH1 + s2 * 128 + kk * 8, bd, kI64, kk > 0 ? 1u : 0u);
+          }
+          tc::mma_commit(odd ? &bar->full_z[g2] : &bar->full_y[g2]);
+          if (c == kNChunks - 1) tc::mma_commit(&bar->h1_free[s2]);
+          return true;
+        };
+        auto issue_l3 = [&](int k, int g2, int c) -> bool {
+          const int s2 = k & 1;
+          if (c == 0) {
+            const bool r = tc::mbar_wait(&bar->acc3_empty[s2], (u_a3[s2] & 1u) ^ 1u, abort,
+                                         kWaitLimitNs);
+            ++u_a3[s2];
+            if (!r) return false;
+          }
+          const int hb = c & 1;
+          const bool r = tc::mbar_wait(&bar->h2_full[hb], u_h2[hb] & 1u, abort, kWaitLimitNs);
+          ++u_h2[hb];
+          if (!r) return false;
+          tc::tc_fence_after();
+          const uint32_t h2_s = s_base + E::kOffH2 + hb * kH2TileBytes;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = tc::smem_desc(h2_s + kk * 32, 1024, 2);
+            const uint64_t bd =
+                tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128) + kk * 32, 1024, 2);
+            tc::mma_ss(tmem + kColA3 + s2 * 16, ad, bd, kI16, (c > 0 || kk > 0) ? 1u : 0u);
+          }
+          if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g2]);
+          return true;
+        };
+        for (int k = 0; k < total && ok; ++k) {
+          const int s2 = k & 1;
+          ok = tc::mbar_wait(&bar->h1_full[s2], u_h1[s2] & 1u, abort, kWaitLimitNs);
+          ++u_h1[s2];
           if (!ok) break;
           tc::tc_fence_after();
+          if (kPolicy) {
+            ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l3(k, g, 0) && issue_l2(k, g, 2) &&
+                 issue_l3(k, g, 1) && issue_l2(k, g, 3) && issue_l3(k, g, 2) && issue_l3(k, g, 3);
+          } else {
+            ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          }
+          advance(it, g);
+        }
+      } else {
+        uint32_t u_x = 0, u_hf[2] = {0, 0}, u_obs[4] = {0, 0, 0, 0};
+        for (int k = 0; k < total && ok; ++k) {
+          const int s1 = k & 1;
+          ok = tc::mbar_wait(&bar->h1_free[s1], (u_hf[s1] & 1u) ^ 1u, abort, kWaitLimitNs);
+          ++u_hf[s1];
+          if (!ok) break;
+          ok = tc::mbar_wait(&bar->obs_full[g], u_obs[g] & 1u, abort, kWaitLimitNs);
+          ++u_obs[g];
           const uint32_t obs_s = s_base + E::kOffObs + g * kObsTileBytes;
           for (int c = 0; c < kNChunks && ok; ++c) {
-            const int b = c & 1;
-            if (!(ok = acquire_acc(b))) break;
+            ok = tc::mbar_wait(&bar->empty_x, (u_x & 1u) ^ 1u, abort, kWaitLimitNs);
+            ++u_x;
+            if (!ok) break;
+            tc::tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
               const uint64_t ad = tc::smem_desc(obs_s + kk * 32, 512, 4);
               const uint64_t bd = tc::smem_desc(s_base + kOffW1 + c * kChunk * 64 + kk * 32, 512, 4);
-              tc::mma_ss(tacc[b], ad, bd, kI64, kk);
+              tc::mma_ss(tmem + kColX, ad, bd, kI64, kk);
             }
-            tc::mma_commit(&bar->acc_full[g][b]);
+            tc::mma_commit(&bar->full_x[g]);
           }
-          if (!ok) break;
-          // layer 2 needs the whole of h1
-          ok = tc::mbar_wait(&bar->h1_full, use_h1 & 1u, abort, kWaitLimitNs);
-          ++use_h1;
-          if (!ok) break;
-          tc::tc_fence_after();
-          if (!kPolicy) {
-            for (int c = 0; c < kNChunks && ok; ++c) ok = issue_l2(g, c);
-            continue;
-          }
-          ok = issue_l2(g, 0) && issue_l2(g, 1);
-          if (!ok) break;
-          // layer 3 interleaved with the last two layer-2 chunks
-          ok = tc::mbar_wait(&bar->acc3_empty, (use_acc3 & 1u) ^ 1u, abort, kWaitLimitNs);
-          ++use_acc3;
-          for (int c = 0; c < kNChunks && ok; ++c) {
-            const int hb = c & 1;
-            ok = tc::mbar_wait(&bar->h2_full[hb], use_h2[hb] & 1u, abort, kWaitLimitNs);
-            ++use_h2[hb];
-            if (!ok) break;
-            tc::tc_fence_after();
-            const uint32_t h2_s = s_base + E::kOffH2 + hb * kH2TileBytes;
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t ad = tc::smem_desc(h2_s + kk * 32, 1024, 2);
-              const uint64_t bd = tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128) + kk * 32,
-                                                1024, 2);
-              tc::mma_ss(tmem + kColAcc3, ad, bd, kI16, (c > 0 || kk > 0) ? 1u : 0u);
-            }
-            if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g]);
-            if (c + 2 < kNChunks) ok = issue_l2(g, c + 2);
-          }
+          advance(it, g);
         }
       }
-      // drain: every issued MMA has completed before tensor memory is freed
-      tc::mma_commit(&bar->drain);
-      tc::mbar_wait(&bar->drain, 0, abort, kWaitLimitNs);
+      // drain: every MMA this thread issued has completed before tensor memory is freed
+      uint64_t* drain = warp == 4 * G ? &bar->drain : &bar->drain1;
+      tc::mma_commit(drain);
+      tc::mbar_wait(drain, 0, abort, kWaitLimitNs);
     }
     __syncwarp();
   } else {
@@ -353,45 +418,44 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     uint8_t* h2_tiles = smem + E::kOffH2;
     const float* b1 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB1P : kOffB1V));
     const float* b2 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB2P : kOffB2V));
-    uint32_t n_full[2] = {0, 0}, n_acc3 = 0;
+    uint32_t n_x = 0, n_y = 0, n_z = 0, n_acc3 = 0;
     bool ok = true;
 
-    auto wait_acc = [&](int b) -> bool {
-      const bool r = tc::mbar_wait(&bar->acc_full[g][b], n_full[b] & 1u, abort, kWaitLimitNs);
-      ++n_full[b];
-      tc::tc_fence_after();
-      return r;
-    };
-    // Layers 1 and 2 epilogues for this group's tile; value mode returns the
-    // head dot product, policy mode leaves the 16 head outputs in head[].
-    auto run_network = [&](float* head) -> bool {
-      for (int c = 0; c < kNChunks; ++c) {       // layer 1 -> h1 (tensor memory)
-        const int b = c & 1;
-        if (!wait_acc(b)) return false;
-        const uint32_t col = b ? kColAcc1 : kColAcc0;
+    // Layer 1-3 epilogues of this group's step k; value mode returns the
+    // head dot product in head[0], policy mode the 16 head outputs.
+    auto run_network = [&](int k, float* head) -> bool {
+      const int slot = k & 1;
+      for (int c = 0; c < kNChunks; ++c) {       // layer 1 (X) -> h1 slot
+        if (!tc::mbar_wait(&bar->full_x[g], n_x & 1u, abort, kWaitLimitNs)) return false;
+        ++n_x;
+        tc::tc_fence_after();
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           uint32_t acc[32], hv[16];
-          tc::tmem_ld32(lane_addr + col + 32 * half, acc);
+          tc::tmem_ld32(lane_addr + kColX + 32 * half, acc);
           tc::tmem_ld_wait(acc);
           if (half == 1) {
             tc::tc_fence_before();
-            tc::mbar_arrive(&bar->acc_empty[b]);
+            tc::mbar_arrive(&bar->empty_x);
           }
           bias_tanh32(acc, b1 + c * kChunk + 32 * half, hv);
-          tc::tmem_st16(lane_addr + kColH1 + c * 32 + half * 16, hv);
+          tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
         }
       }
       tc::tmem_st_wait();
       tc::tc_fence_before();
-      tc::mbar_arrive(&bar->h1_full);
+      tc::mbar_arrive(&bar->h1_full[slot]);
       float vsum = 0.0f;
       const float* w3v = reinterpret_cast<const float*>(smem + kOffW3V);
-      for (int c = 0; c < kNChunks; ++c) {       // layer 2
-        const int b = c & 1;
-        if (!wait_acc(b)) return false;
-        const uint32_t col = b ? kColAcc1 : kColAcc0;
-        uint8_t* h2 = h2_tiles + b * kH2TileBytes + row * 128;
+      for (int c = 0; c < kNChunks; ++c) {       // layer 2 (Y / Z)
+        const bool odd = c & 1;
+        uint32_t& n = odd ? n_z : n_y;
+        if (!tc::mbar_wait(odd ? &bar->full_z[g] : &bar->full_y[g], n & 1u, abort, kWaitLimitNs))
+          return false;
+        ++n;
+        tc::tc_fence_after();
+        const uint32_t col = odd ? kColZ : kColY;
+        uint8_t* h2 = h2_tiles + (c & 1) * kH2TileBytes + row * 128;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           uint32_t acc[32], hv[16];
@@ -399,7 +463,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           tc::tmem_ld_wait(acc);
           if (half == 1) {
             tc::tc_fence_before();
-            tc::mbar_arrive(&bar->acc_empty[b]);
+            tc::mbar_arrive(odd ? &bar->empty_z : &bar->empty_y);
           }
           bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
           if (kPolicy) {
@@ -418,7 +482,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         }
         if (kPolicy) {
           tc::fence_async_smem();
-          tc::mbar_arrive(&bar->h2_full[b]);
+          tc::mbar_arrive(&bar->h2_full[c & 1]);
         }
       }
       if (!kPolicy) {
@@ -429,26 +493,26 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       ++n_acc3;
       tc::tc_fence_after();
       uint32_t o3[16];
-      tc::tmem_ld16(lane_addr + kColAcc3, o3);
+      tc::tmem_ld16(lane_addr + kColA3 + slot * 16, o3);
       tc::tmem_ld_wait(o3);
       tc::tc_fence_before();
-      tc::mbar_arrive(&bar->acc3_empty);
+      tc::mbar_arrive(&bar->acc3_empty[slot]);
       const float* b3 = reinterpret_cast<const float*>(smem + kOffB3P);
 #pragma unroll
       for (int j = 0; j < kHeadOut; ++j) head[j] = __uint_as_float(o3[j]) + b3[j];
       return true;
     };
 
-    const int iters = group_iters(g);
+    const int my_iters = iters[g];
     if (MODE == kRollout) {
       const int tile = slot0 + g;
       const int i = tile * kRows + row;
-      const bool active = iters > 0 && i < M.n;
+      const bool active = my_iters > 0 && i < M.n;
       const size_t n = (size_t)M.n;
       Env e;
       if (active) load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
       bool bad = false;
-      for (int t = 0; t < iters && ok; ++t) {
+      for (int t = 0; t < my_iters && ok; ++t) {
         float o[kObs];
         if (active) {
           observe(e, o);
@@ -465,7 +529,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(head))) break;
+        if (!(ok = run_network(step_index<G>(t, g, iters), head))) break;
         __syncwarp();
         if (active) {
           const uint32_t id = M.id_base + (uint32_t)i;
@@ -497,7 +561,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
       }
     } else {
-      for (int it = 0; it < iters && ok; ++it) {
+      for (int it = 0; it < my_iters && ok; ++it) {
         const size_t r = (size_t)(slot0 + g + it * n_slots) * kRows + row;
         const bool active = r < io.rows;
         float o[kObs];
@@ -515,7 +579,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(head))) break;
+        if (!(ok = run_network(step_index<G>(it, g, iters), head))) break;
         __syncwarp();
         if (active) {
           if (MODE == kValueRows) {
@@ -535,7 +599,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     atomicAdd(&st->timeouts, 1);
     atomicCAS(&st->code, 0, -4);
   }
-  if (is_mma_warp) {
+  if (warp == 4 * G) {
     tc::tc_fence_after();
     tc::tmem_dealloc(tmem, kTmemCols);
   }
