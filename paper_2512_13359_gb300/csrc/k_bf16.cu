@@ -329,12 +329,13 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           if (!r) return false;
           tc::tc_fence_after();
           const uint32_t d = tmem + (odd ? kColZ : kColY);
-#pragma unroll 1
-          for (int kk = 0; kk < 16; ++kk) {
-            const uint64_t bd = tc::smem_desc(
-                s_base + kOffW2 + (kk >> 2) * (kH * 128) + c * kChunk * 128 + (kk & 3) * 32, 1024, 2);
-            tc::mma_ts(d, tmem + kColH1 + s2 * 128 + kk * 8, bd, kI64, kk > 0 ? 1u : 0u);
-          }
+          const uint32_t a0 = tmem + kColH1 + s2 * 128;
+          // descriptor start addresses are in 16-byte units: step K by adding offsets
+          const uint64_t b0 = tc::smem_desc(s_base + kOffW2 + c * kChunk * 128, 1024, 2);
+#pragma unroll
+          for (int kk = 0; kk < 16; ++kk)
+            tc::mma_ts(d, a0 + kk * 8, b0 + (uint64_t)(((kk >> 2) * (kH * 128) + (kk & 3) * 32) >> 4),
+                       kI64, kk > 0 ? 1u : 0u);
           tc::mma_commit(odd ? &bar->full_z[g2] : &bar->full_y[g2]);
           if (c == kNChunks - 1) tc::mma_commit(&bar->h1_free[s2]);
           return true;
@@ -352,14 +353,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           ++u_h2[hb];
           if (!r) return false;
           tc::tc_fence_after();
-          const uint32_t h2_s = s_base + E::kOffH2 + hb * kH2TileBytes;
+          const uint64_t a0 = tc::smem_desc(s_base + E::kOffH2 + hb * kH2TileBytes, 1024, 2);
+          const uint64_t b0 = tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128), 1024, 2);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            const uint64_t ad = tc::smem_desc(h2_s + kk * 32, 1024, 2);
-            const uint64_t bd =
-                tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128) + kk * 32, 1024, 2);
-            tc::mma_ss(tmem + kColA3 + s2 * 16, ad, bd, kI16, (c > 0 || kk > 0) ? 1u : 0u);
-          }
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_ss(tmem + kColA3 + s2 * 16, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), kI16,
+                       (c > 0 || kk > 0) ? 1u : 0u);
           if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g2]);
           return true;
         };
@@ -392,12 +391,10 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             ++u_x;
             if (!ok) break;
             tc::tc_fence_after();
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk) {
-              const uint64_t ad = tc::smem_desc(obs_s + kk * 32, 512, 4);
-              const uint64_t bd = tc::smem_desc(s_base + kOffW1 + c * kChunk * 64 + kk * 32, 512, 4);
-              tc::mma_ss(tmem + kColX, ad, bd, kI64, kk);
-            }
+            const uint64_t a0 = tc::smem_desc(obs_s, 512, 4);
+            const uint64_t b0 = tc::smem_desc(s_base + kOffW1 + c * kChunk * 64, 512, 4);
+            tc::mma_ss(tmem + kColX, a0, b0, kI64, 0u);
+            tc::mma_ss(tmem + kColX, a0 + 2, b0 + 2, kI64, 1u);
             tc::mma_commit(&bar->full_x[g]);
           }
           advance(it, g);
