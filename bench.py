@@ -213,9 +213,8 @@ def main():
         return
 
     import torch
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2512_13359_gb300 import shard
+    rank, world, local = shard.world()
     torch.cuda.set_device(local)
     dist = None
     if world > 1:
@@ -224,12 +223,10 @@ def main():
     from paper_2512_13359_gb300 import auvenv, build
     if rank == 0 or world == 1:
         build.build()
-    if dist:
-        dist.barrier()
+    shard.barrier(dist)
 
-    n = int(w["n_envs"])
     T = int(w["steps"])
-    w["env_id_base"] = rank * n          # shard: rank r owns global env ids [r n, (r+1) n)
+    w["env_id_base"], n = shard.env_range(rank, int(w["n_envs"]))
     env = auvenv.Env(w)
     pw = W.policy_weights(w)
     vw = W.value_weights(w) if w["has_value"] else None
@@ -260,8 +257,7 @@ def main():
         raise RuntimeError(f"device status {st.code} after warm-up")
 
     clocks = ClockSampler(local) if not args.no_clocks else None
-    if dist:
-        dist.barrier()
+    shard.barrier(dist)
     torch.cuda.synchronize()
     if clocks:
         clocks.start()
@@ -273,16 +269,12 @@ def main():
         one_step(ev)
         events.append(ev)
     torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
+    shard.barrier(dist)
     clock_info = clocks.stop() if clocks else None
     roll_ms = [e[0].elapsed_time(e[1]) for e in events]
     val_ms = [e[1].elapsed_time(e[2]) for e in events]
-    step_ms = sum(r + v for r, v in zip(roll_ms, val_ms)) / args.steps
-    if dist:
-        t = torch.tensor([step_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        step_ms = float(t.item())
+    step_ms = shard.max_over_ranks(sum(r + v for r, v in zip(roll_ms, val_ms)) / args.steps,
+                                   dist, "cuda")
     env_steps = n * T * world
     value_rate = env_steps / (step_ms * 1e-3)
     st = env.status()
@@ -304,8 +296,7 @@ def main():
             if h_val is not None:
                 env.value(h_traj["obs"], h_val)
             torch.cuda.synchronize()
-        if dist:
-            dist.barrier()
+        shard.barrier(dist)
         t0 = time.perf_counter()
         for _ in range(max(1, min(args.steps, 5))):
             env.set_weights(h_pw, h_vw)          # step inputs: policy + value weights, H2D
@@ -313,11 +304,8 @@ def main():
             if h_val is not None:
                 env.value(h_traj["obs"], h_val)
             torch.cuda.synchronize()
-        e2e_s = (time.perf_counter() - t0) / max(1, min(args.steps, 5))
-        if dist:
-            t = torch.tensor([e2e_s], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t.item())
+        e2e_s = shard.max_over_ranks((time.perf_counter() - t0) / max(1, min(args.steps, 5)),
+                                     dist, "cuda")
         e2e = {"value": env_steps / e2e_s, "unit": "env-steps/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 

@@ -275,6 +275,16 @@ int env_set_step(auv_env* env, uint64_t t_g);
 int env_status(auv_env* env, auv_status* out, void* stream);
 int env_clear_status(auv_env* env, void* stream);
 
+/*
+ * env_selftest_wait_timeout: failure-detection self-test.  Launches one
+ * thread that waits, with the same bounded wait the tensor-core kernels use
+ * on their mbarriers, on a barrier phase that nothing completes.  The wait
+ * gives up after limit_us microseconds (1 .. 5e6) and latches AUV_ERR_TIMEOUT
+ * and timeouts += 1 in the status block, read back by env_status; the CUDA
+ * context stays usable.  (A library check, not part of the paper's method.)
+ */
+int env_selftest_wait_timeout(auv_env* env, uint32_t limit_us, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

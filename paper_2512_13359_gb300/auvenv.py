@@ -29,7 +29,8 @@ AUV_MLP_BF16 = 1
 EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
-            "env_status", "env_clear_status", "env_policy_forward_noalloc")
+            "env_status", "env_clear_status", "env_selftest_wait_timeout",
+            "env_policy_forward_noalloc")
 
 
 class LibraryMissing(RuntimeError):
@@ -110,6 +111,7 @@ def lib(path: str | None = None):
     L.env_set_step.argtypes = [P, C.c_uint64]
     L.env_status.argtypes = [P, C.POINTER(AuvStatus), P]
     L.env_clear_status.argtypes = [P, P]
+    L.env_selftest_wait_timeout.argtypes = [P, C.c_uint32, P]
     L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
@@ -265,6 +267,9 @@ class Env:
         s = AuvStatus()
         lib().env_status(self.h, C.byref(s), _stream(stream))
         return s
+
+    def selftest_wait_timeout(self, limit_us: int, stream=None):
+        self._check(lib().env_selftest_wait_timeout(self.h, int(limit_us), _stream(stream)))
 
     def clear_status(self, stream=None):
         self._check(lib().env_clear_status(self.h, _stream(stream)))

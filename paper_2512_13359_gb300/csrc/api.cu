@@ -498,6 +498,17 @@ int env_status(auv_env* env, auv_status* out, void* stream) {
   return st.code;
 }
 
+int env_selftest_wait_timeout(auv_env* env, uint32_t limit_us, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (limit_us < 1 || limit_us > 5000000)
+    return fail(env, AUV_ERR_INVALID, "limit_us outside [1, 5e6]");
+  cudaError_t e = auv::launch_wait_selftest(env->status, (uint64_t)limit_us * 1000ull,
+                                            static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "wait self-test kernel");
+}
+
 int env_clear_status(auv_env* env, void* stream) {
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);

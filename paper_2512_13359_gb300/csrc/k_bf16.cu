@@ -643,7 +643,34 @@ int pick_groups(long tiles) {
   return best;
 }
 
+// Failure-detection self-test: one thread waits, with the engine's bounded
+// wait, on a barrier phase that nothing completes; the wait gives up after
+// `limit_ns` and the timeout is latched in the status block exactly as an
+// engine wait would latch it.
+__global__ void k_wait_selftest(Status* st, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile int* abort = &abort_flag;
+    if (!tc::mbar_wait(&bar, 0, abort, limit_ns)) {
+      atomicAdd(&st->timeouts, 1);
+      atomicCAS(&st->code, 0, -4);
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(Status* st, uint64_t limit_ns, cudaStream_t s) {
+  k_wait_selftest<<<1, 32, 0, s>>>(st, limit_ns);
+  return cudaGetLastError();
+}
 
 size_t bf16_policy_image_bytes() { return kPolicyImage; }
 size_t bf16_value_image_bytes() { return kValueImage; }

@@ -117,3 +117,25 @@ def test_bf16_rollout_is_deterministic(oracle):
     for k in t1:
         assert torch.equal(t1[k], t2[k]), k
     assert torch.equal(e1.state, e2.state)
+
+
+def test_sharded_batches_reproduce_the_full_batch(oracle):
+    """Two shards with env_id_base = 0 and n reproduce one batch of 2n envs
+    bit for bit (the multi-GPU partition, run here on one GPU)."""
+    torch = need_gpu()
+    n, T = 1000, 12
+    full_w = W.workload("ppo_65536", n_envs=2 * n, episode_len=7)
+    full = make_env(full_w)
+    full.reset()
+    tf = full.alloc_traj(T)
+    full.rollout(T, tf)
+    for r in range(2):
+        w = dict(full_w, n_envs=n, env_id_base=r * n)
+        e = make_env(w)
+        e.reset()
+        t = e.alloc_traj(T)
+        e.rollout(T, t)
+        sl = slice(r * n, (r + 1) * n)
+        for k in ("obs", "act", "logp", "rew", "done", "value"):
+            assert torch.equal(t[k], tf[k][..., sl]), k
+        assert torch.equal(e.state, full.state[:, sl])
