@@ -51,6 +51,8 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--sweep", action="store_true",
+                    help="batch-size sweep 1,024 .. 1,048,576 envs x 256 steps (one line per size)")
     return ap.parse_args()
 
 
@@ -200,6 +202,19 @@ def run_reference(args, w):
 # ---------------------------------------------------------------------------
 def main():
     args = parse()
+    if args.sweep:
+        base_steps = args.steps
+        for n in W.SWEEP_SIZES:
+            a = argparse.Namespace(**vars(args))
+            a.workload, a.n_envs, a.rollout_steps, a.sweep = "sweep", n, None, False
+            a.no_e2e, a.no_cpu_baseline = True, True
+            a.steps = max(3, min(base_steps, int(2e8 // (n * 256)) + 3))
+            run(a)
+        return
+    run(args)
+
+
+def run(args):
     over = {}
     if args.n_envs:
         over["n_envs"] = args.n_envs
