@@ -51,6 +51,8 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--replay", action="store_true",
+                    help="physics only: action replay (env_step_actions), FP32 roofline")
     ap.add_argument("--sweep", action="store_true",
                     help="batch-size sweep 1,024 .. 1,048,576 envs x 256 steps (one line per size)")
     return ap.parse_args()
@@ -200,8 +202,70 @@ def run_reference(args, w):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
+def run_replay(args):
+    """Dynamics step alone (allocation, substeps, reward, done, reset) over
+    given actions: the FP32-bound part of the rollout."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {}
+    if args.n_envs:
+        over["n_envs"] = args.n_envs
+    if args.rollout_steps:
+        over["steps"] = args.rollout_steps
+    w = W.workload(args.workload, **over)
+    n, T = int(w["n_envs"]), int(w["steps"])
+    env = auvenv.Env(w)
+    env.reset()
+    act = torch.from_numpy(W.replay_actions(1, T, n)).cuda()
+    rew = torch.empty((T, n), device="cuda")
+    done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        env.step_actions(act, rew, done)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0) if not args.no_clocks else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        env.step_actions(act, rew, done)
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    clock_info = clocks.stop() if clocks else None
+    step_ms = sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+    if env.status().code != 0:
+        raise RuntimeError("device status after replay")
+    peaks, _ = load_peaks()
+    sm_mhz = (clock_info or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    fp32_peak = 2 * 128 * n_sm * sm_mhz * 1e6 / 1e12
+    achieved = n * T * DYN_FLOPS_PER_ENV_STEP / (step_ms * 1e-3) / 1e12
+    line = {
+        "metric": "env-steps/s (physics only, action replay)", "value": n * T / (step_ms * 1e-3),
+        "unit": "env-steps/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w["name"], "n_envs_per_gpu": n, "rollout_steps": T,
+                   "substeps": w["substeps"], "l2": "flushed between timed steps"},
+        "roofline": {"bound": "alu", "kernel": "k_replay", "achieved": achieved, "peak": fp32_peak,
+                     "unit": "TFLOP/s", "frac": achieved / fp32_peak, "traffic": None,
+                     "peak_source": f"FP32 pipe 2*128*{n_sm} SMs*{sm_mhz:.0f} MHz"},
+        "gpu_launches": args.steps, "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.replay:
+        run_replay(args)
+        return
     if args.sweep:
         base_steps = args.steps
         for n in W.SWEEP_SIZES:
