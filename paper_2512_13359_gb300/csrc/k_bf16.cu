@@ -188,16 +188,20 @@ __device__ __forceinline__ void write_obs_row(uint8_t* tile, int r, const float 
   }
 }
 
-// 32 accumulator columns + bias -> tanh -> 16 bf16 pairs.
+// 32 accumulator columns + bias -> tanh -> 16 bf16 pairs.  The bias is added
+// two columns per instruction (packed fp32 add, round to nearest: the same
+// sums as scalar adds).
 __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const float* bias,
                                             uint32_t (&out)[16]) {
 #pragma unroll
   for (int j = 0; j < 16; j += 2) {
     const float4 b = *reinterpret_cast<const float4*>(bias + 2 * j);
-    out[j] = tc::tanh_bf16x2(tc::pack_bf16x2(__uint_as_float(acc[2 * j]) + b.x,
-                                             __uint_as_float(acc[2 * j + 1]) + b.y));
-    out[j + 1] = tc::tanh_bf16x2(tc::pack_bf16x2(__uint_as_float(acc[2 * j + 2]) + b.z,
-                                                 __uint_as_float(acc[2 * j + 3]) + b.w));
+    const float2 s0 = __fadd2_rn(make_float2(__uint_as_float(acc[2 * j]), __uint_as_float(acc[2 * j + 1])),
+                                 make_float2(b.x, b.y));
+    const float2 s1 = __fadd2_rn(make_float2(__uint_as_float(acc[2 * j + 2]), __uint_as_float(acc[2 * j + 3])),
+                                 make_float2(b.z, b.w));
+    out[j] = tc::tanh_bf16x2(tc::pack_bf16x2(s0.x, s0.y));
+    out[j + 1] = tc::tanh_bf16x2(tc::pack_bf16x2(s1.x, s1.y));
   }
 }
 
