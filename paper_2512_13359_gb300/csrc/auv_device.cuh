@@ -266,6 +266,38 @@ __device__ __forceinline__ void store_env(const Model& M, float* __restrict__ st
   ep[i] = e.ep;
 }
 
+// The per-episode parameters alone (goal, scales, buoyancy offset, centre
+// of buoyancy, current), for kernels that keep them in global memory while
+// the rest of the env state stays in registers.  The reload goes through L2
+// (ld.global.cg): it is coherent with this thread's own earlier stores of
+// the same kernel.  inv_m is not part of the arrays and is left as it is.
+__device__ __forceinline__ void store_params(const Model& M, float* pr, int i, const Env& e) {
+  const int n = M.n;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) pr[k * n + i] = e.pd[k];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) pr[(3 + k) * n + i] = e.qd[k];
+  pr[7 * n + i] = e.sm; pr[8 * n + i] = e.sa; pr[9 * n + i] = e.sd; pr[10 * n + i] = e.dB;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) pr[(11 + k) * n + i] = e.rb[k];
+#pragma unroll
+  for (int k = 0; k < 3; ++k) pr[(14 + k) * n + i] = e.Vc[k];
+}
+
+__device__ __forceinline__ void reload_params(const Model& M, const float* pr, int i, Env& e) {
+  const int n = M.n;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) e.pd[k] = __ldcg(pr + k * n + i);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) e.qd[k] = __ldcg(pr + (3 + k) * n + i);
+  e.sm = __ldcg(pr + 7 * n + i); e.sa = __ldcg(pr + 8 * n + i);
+  e.sd = __ldcg(pr + 9 * n + i); e.dB = __ldcg(pr + 10 * n + i);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) e.rb[k] = __ldcg(pr + (11 + k) * n + i);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) e.Vc[k] = __ldcg(pr + (14 + k) * n + i);
+}
+
 // ---------------------------------------------------------------------------
 // Dynamics
 // ---------------------------------------------------------------------------

@@ -312,9 +312,17 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       int total = 0;
 #pragma unroll
       for (int g = 0; g < G; ++g) total += iters[g];
+      // iters[] is read with a runtime index through selects, so that it stays
+      // in registers (likewise the per-slot barrier phases below are bits).
+      auto iters_at = [&](int gg) {
+        int v = 0;
+#pragma unroll
+        for (int j = 0; j < G; ++j) v = j == gg ? iters[j] : v;
+        return v;
+      };
       auto advance = [&](int& it, int& g) {
         ++g;
-        if (g >= G || iters[g] <= it) {
+        if (g >= G || iters_at(g) <= it) {
           g = 0;
           ++it;
         }
@@ -322,7 +330,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       bool ok = true;
       int it = 0, g = 0;
       if (warp == 4 * G) {
-        uint32_t u_y = 0, u_z = 0, u_h1[2] = {0, 0}, u_h2[2] = {0, 0}, u_a3[2] = {0, 0};
+        uint32_t u_y = 0, u_z = 0, u_h2[2] = {0, 0};
+        uint32_t p_h1 = 0, p_a3 = 0;   // phase bit of slot s at bit s
         auto issue_l2 = [&](int k, int g2, int c) -> bool {
           const int s2 = k & 1;
           const bool odd = c & 1;
@@ -347,9 +356,9 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         auto issue_l3 = [&](int k, int g2, int c) -> bool {
           const int s2 = k & 1;
           if (c == 0) {
-            const bool r = tc::mbar_wait(&bar->acc3_empty[s2], (u_a3[s2] & 1u) ^ 1u, abort,
+            const bool r = tc::mbar_wait(&bar->acc3_empty[s2], ((p_a3 >> s2) & 1u) ^ 1u, abort,
                                          kWaitLimitNs);
-            ++u_a3[s2];
+            p_a3 ^= 1u << s2;
             if (!r) return false;
           }
           const int hb = c & 1;
@@ -368,8 +377,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         };
         for (int k = 0; k < total && ok; ++k) {
           const int s2 = k & 1;
-          ok = tc::mbar_wait(&bar->h1_full[s2], u_h1[s2] & 1u, abort, kWaitLimitNs);
-          ++u_h1[s2];
+          ok = tc::mbar_wait(&bar->h1_full[s2], (p_h1 >> s2) & 1u, abort, kWaitLimitNs);
+          p_h1 ^= 1u << s2;
           if (!ok) break;
           tc::tc_fence_after();
           if (kPolicy) {
@@ -381,14 +390,14 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           advance(it, g);
         }
       } else {
-        uint32_t u_x = 0, u_hf[2] = {0, 0}, u_obs[4] = {0, 0, 0, 0};
+        uint32_t u_x = 0, p_hf = 0, p_obs = 0;   // phase bits per slot / group
         for (int k = 0; k < total && ok; ++k) {
           const int s1 = k & 1;
-          ok = tc::mbar_wait(&bar->h1_free[s1], (u_hf[s1] & 1u) ^ 1u, abort, kWaitLimitNs);
-          ++u_hf[s1];
+          ok = tc::mbar_wait(&bar->h1_free[s1], ((p_hf >> s1) & 1u) ^ 1u, abort, kWaitLimitNs);
+          p_hf ^= 1u << s1;
           if (!ok) break;
-          ok = tc::mbar_wait(&bar->obs_full[g], u_obs[g] & 1u, abort, kWaitLimitNs);
-          ++u_obs[g];
+          ok = tc::mbar_wait(&bar->obs_full[g], (p_obs >> g) & 1u, abort, kWaitLimitNs);
+          p_obs ^= 1u << g;
           const uint32_t obs_s = s_base + E::kOffObs + g * kObsTileBytes;
           for (int c = 0; c < kNChunks && ok; ++c) {
             ok = tc::mbar_wait(&bar->empty_x, (u_x & 1u) ^ 1u, abort, kWaitLimitNs);
@@ -419,16 +428,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     uint8_t* h2_tiles = smem + E::kOffH2;
     const float* b1 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB1P : kOffB1V));
     const float* b2 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB2P : kOffB2V));
-    uint32_t n_x = 0, n_y = 0, n_z = 0, n_acc3 = 0;
+    // Barrier phases need no counters: per group-step a group waits on its
+    // full_x barrier once per chunk (4 times), on full_y and full_z twice
+    // each and on acc3_full once, so the phase parities are c & 1,
+    // (c >> 1) & 1 and the parity of the group's own step count.
     bool ok = true;
 
     // Layer 1-3 epilogues of this group's step k; value mode returns the
     // head dot product in head[0], policy mode the 16 head outputs.
-    auto run_network = [&](int k, float* head) -> bool {
+    auto run_network = [&](int k, int it, float* head) -> bool {
       const int slot = k & 1;
       for (int c = 0; c < kNChunks; ++c) {       // layer 1 (X) -> h1 slot
-        if (!tc::mbar_wait(&bar->full_x[g], n_x & 1u, abort, kWaitLimitNs)) return false;
-        ++n_x;
+        if (!tc::mbar_wait(&bar->full_x[g], (uint32_t)c & 1u, abort, kWaitLimitNs)) return false;
         tc::tc_fence_after();
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -450,10 +461,9 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       const float* w3v = reinterpret_cast<const float*>(smem + kOffW3V);
       for (int c = 0; c < kNChunks; ++c) {       // layer 2 (Y / Z)
         const bool odd = c & 1;
-        uint32_t& n = odd ? n_z : n_y;
-        if (!tc::mbar_wait(odd ? &bar->full_z[g] : &bar->full_y[g], n & 1u, abort, kWaitLimitNs))
+        if (!tc::mbar_wait(odd ? &bar->full_z[g] : &bar->full_y[g], ((uint32_t)c >> 1) & 1u, abort,
+                           kWaitLimitNs))
           return false;
-        ++n;
         tc::tc_fence_after();
         const uint32_t col = odd ? kColZ : kColY;
         uint8_t* h2 = h2_tiles + (c & 1) * kH2TileBytes + row * 128;
@@ -490,8 +500,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         head[0] = vsum + *reinterpret_cast<const float*>(smem + kOffB3V);
         return true;
       }
-      if (!tc::mbar_wait(&bar->acc3_full[g], n_acc3 & 1u, abort, kWaitLimitNs)) return false;
-      ++n_acc3;
+      if (!tc::mbar_wait(&bar->acc3_full[g], (uint32_t)it & 1u, abort, kWaitLimitNs)) return false;
       tc::tc_fence_after();
       uint32_t o3[16];
       tc::tmem_ld16(lane_addr + kColA3 + slot * 16, o3);
@@ -504,8 +513,13 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       return true;
     };
 
-    const int my_iters = iters[g];
+    int my_iters = 0;
+#pragma unroll
+    for (int j = 0; j < G; ++j) my_iters = j == g ? iters[j] : my_iters;
     if (MODE == kRollout) {
+      int n_act = 0;
+#pragma unroll
+      for (int j = 0; j < G; ++j) n_act += iters[j] > 0 ? 1 : 0;
       const int tile = slot0 + g;
       const int i = tile * kRows + row;
       const bool active = my_iters > 0 && i < M.n;
@@ -530,9 +544,13 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(step_index<G>(t, g, iters), head))) break;
+        // every group with work runs T steps: the step index is t * n_act + g
+        if (!(ok = run_network(t * n_act + g, t, head))) break;
         __syncwarp();
         if (active) {
+          // The episode parameters are not held in registers across the
+          // network (they would not fit beside the accumulators).
+          reload_params(M, B.params, i, e);
           const uint32_t id = M.id_base + (uint32_t)i;
           float eps[kAct];
           action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
@@ -551,6 +569,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
           bool d;
           const float r = physics_step(M, id, e, a, &d);
+          if (d) store_params(M, B.params, i, e);
           if (tr.rew) tr.rew[(size_t)t * n + i] = r;
           if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
           bad |= !env_finite(e);
@@ -580,7 +599,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(step_index<G>(it, g, iters), head))) break;
+        if (!(ok = run_network(step_index<G>(it, g, iters), it, head))) break;
         __syncwarp();
         if (active) {
           if (MODE == kValueRows) {
