@@ -7,7 +7,7 @@
 // One CTA per SM holds the network's weights in shared memory as pre-swizzled
 // bf16 images for the whole launch.  Its threads form G groups of 128 (one
 // row -- one environment -- per thread, which is also that row's tensor-memory
-// lane) plus two MMA-issuing warps (layer 1; layers 2 and 3).  The groups take
+// lane) plus three MMA-issuing warps (layer 1, layer 2, layer 3).  The groups take
 // turns on the tensor pipe: while one group's network runs, the others
 // integrate their environments.
 //
@@ -148,7 +148,8 @@ struct Barriers {
   uint64_t h2_full[2];      // h2 buffer written (128 arrivals)
   uint64_t acc3_empty[2];   // head slot read back (128 arrivals)
   uint64_t h1_free[2];      // layer-2 MMAs reading an h1 slot completed (commit)
-  uint64_t drain, drain1;
+  uint64_t h2_empty[2];     // layer-3 MMAs reading an h2 buffer completed (commit)
+  uint64_t drain, drain1, drain2;
   uint32_t tmem_base;
   int abort;
 };
@@ -169,7 +170,7 @@ struct Engine {
   static constexpr uint32_t kOffH2 = kOffObs + G * kObsTileBytes;
   static constexpr uint32_t kOffBar = kOffH2 + (kPolicy ? 2 * kH2TileBytes : 0);
   static constexpr uint32_t kSmem = kOffBar + sizeof(Barriers) + 1024;   // + alignment slack
-  static constexpr int kThreads = G * kRows + 64;
+  static constexpr int kThreads = G * kRows + 96;
 };
 
 // Row r of the observation tile (bf16, K = 32, 64-byte swizzle): 4 pieces of
@@ -216,9 +217,9 @@ __device__ __forceinline__ int step_index(int it, int g, const int (&iters)[G]) 
   return k;
 }
 
-// Register cap: the 4G+2 warps are spread over the SM's four sub-partitions,
+// Register cap: the 4G+3 warps are spread over the SM's four sub-partitions,
 // whose 16K-register files each host up to G+1 warps (G = 4: 5 warps x 32
-// lanes x 96 registers <= 16384).
+// lanes x 96 registers <= 16384; G = 2: 3 x 32 x 168 <= 16384).
 //
 // Schedule.  Two group-steps are in flight: while the tensor pipe runs layer 2
 // (and layer 3) of group-step k-1, it also runs layer 1 of group-step k, whose
@@ -230,7 +231,7 @@ __device__ __forceinline__ int step_index(int it, int g, const int (&iters)[G]) 
 // or by a commit: an epilogue only starts after a commit that covers every
 // MMA issued before it.
 template <int G, int MODE>
-__global__ void __launch_bounds__(G * 128 + 64) __maxnreg__(G == 4 ? 96 : 168)
+__global__ void __launch_bounds__(G * 128 + 96) __maxnreg__(G == 4 ? 96 : 168)
 k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
          uint64_t t_g0, RowIO io, Status* st) {
   using E = Engine<G, MODE>;
@@ -261,9 +262,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       tc::mbar_init(&bar->h2_full[s], kRows);
       tc::mbar_init(&bar->acc3_empty[s], kRows);
       tc::mbar_init(&bar->h1_free[s], 1);
+      tc::mbar_init(&bar->h2_empty[s], 1);
     }
     tc::mbar_init(&bar->drain, 1);
     tc::mbar_init(&bar->drain1, 1);
+    tc::mbar_init(&bar->drain2, 1);
     bar->abort = 0;
     tc::mbar_fence_init();
   }
@@ -297,13 +300,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
   }
 
   if (is_mma_warp) {
-    // =================== MMA issue: two streams, one elected lane each ===================
-    // Warp 4G issues layers 2 and 3 of each group-step once its h1 is
-    // complete, in the order L2 c0, L2 c1, L3 c0, L2 c2, L3 c1, L2 c3, L3 c2,
-    // L3 c3 (value mode: L2 c0..c3).  Warp 4G+1 issues layer 1 of each
-    // group-step into X chunk by chunk.  Each thread blocks (suspended by the
-    // hardware) only on the barrier of its own next operation, so neither
-    // stream waits behind the other's epilogue.  Before layer 1 of step k the
+    // =================== MMA issue: three streams, one elected lane each ===================
+    // Warp 4G+1 issues layer 1 of each group-step into X chunk by chunk;
+    // warp 4G issues layer 2 (chunks c0..c3 into Y, Z, Y, Z) once the step's
+    // h1 is complete; warp 4G+2 issues layer 3 chunk by chunk as the h2
+    // buffers fill (policy modes).  Each thread blocks (suspended by the
+    // hardware) only on the barrier of its own next operation, so no stream
+    // waits behind another's epilogue: layer 2 of step k+1 starts as soon as
+    // its h1 and an accumulator are ready, while layer 3 of step k is still
+    // waiting for step k's last h2 chunk.  Before layer 1 of step k the
     // layer-1 thread waits until the layer-2 MMAs of step k-2, which read the
     // same h1 slot, have completed (h1_free).
     if ((tid & 31) == 0) {
@@ -330,8 +335,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       bool ok = true;
       int it = 0, g = 0;
       if (warp == 4 * G) {
-        uint32_t u_y = 0, u_z = 0, u_h2[2] = {0, 0};
-        uint32_t p_h1 = 0, p_a3 = 0;   // phase bit of slot s at bit s
+        uint32_t u_y = 0, u_z = 0;
+        uint32_t p_h1 = 0;   // phase bit of slot s at bit s
         auto issue_l2 = [&](int k, int g2, int c) -> bool {
           const int s2 = k & 1;
           const bool odd = c & 1;
@@ -353,39 +358,36 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           if (c == kNChunks - 1) tc::mma_commit(&bar->h1_free[s2]);
           return true;
         };
-        auto issue_l3 = [&](int k, int g2, int c) -> bool {
-          const int s2 = k & 1;
-          if (c == 0) {
-            const bool r = tc::mbar_wait(&bar->acc3_empty[s2], ((p_a3 >> s2) & 1u) ^ 1u, abort,
-                                         kWaitLimitNs);
-            p_a3 ^= 1u << s2;
-            if (!r) return false;
-          }
-          const int hb = c & 1;
-          const bool r = tc::mbar_wait(&bar->h2_full[hb], u_h2[hb] & 1u, abort, kWaitLimitNs);
-          ++u_h2[hb];
-          if (!r) return false;
-          tc::tc_fence_after();
-          const uint64_t a0 = tc::smem_desc(s_base + E::kOffH2 + hb * kH2TileBytes, 1024, 2);
-          const uint64_t b0 = tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128), 1024, 2);
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc::mma_ss(tmem + kColA3 + s2 * 16, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), kI16,
-                       (c > 0 || kk > 0) ? 1u : 0u);
-          if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g2]);
-          return true;
-        };
         for (int k = 0; k < total && ok; ++k) {
           const int s2 = k & 1;
           ok = tc::mbar_wait(&bar->h1_full[s2], (p_h1 >> s2) & 1u, abort, kWaitLimitNs);
           p_h1 ^= 1u << s2;
           if (!ok) break;
           tc::tc_fence_after();
-          if (kPolicy) {
-            ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l3(k, g, 0) && issue_l2(k, g, 2) &&
-                 issue_l3(k, g, 1) && issue_l2(k, g, 3) && issue_l3(k, g, 2) && issue_l3(k, g, 3);
-          } else {
-            ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          advance(it, g);
+        }
+      } else if (warp == 4 * G + 2) {
+        // layer 3: A = h2 buffer (c & 1), B = W3 K-slice c, into head slot k & 1
+        uint32_t p_h2 = 0, p_a3 = 0;   // phase bit of buffer / slot s at bit s
+        for (int k = 0; k < total && ok && kPolicy; ++k) {
+          const int s2 = k & 1;
+          ok = tc::mbar_wait(&bar->acc3_empty[s2], ((p_a3 >> s2) & 1u) ^ 1u, abort, kWaitLimitNs);
+          p_a3 ^= 1u << s2;
+          for (int c = 0; c < kNChunks && ok; ++c) {
+            const int hb = c & 1;
+            ok = tc::mbar_wait(&bar->h2_full[hb], (p_h2 >> hb) & 1u, abort, kWaitLimitNs);
+            p_h2 ^= 1u << hb;
+            if (!ok) break;
+            tc::tc_fence_after();
+            const uint64_t a0 = tc::smem_desc(s_base + E::kOffH2 + hb * kH2TileBytes, 1024, 2);
+            const uint64_t b0 = tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128), 1024, 2);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc::mma_ss(tmem + kColA3 + s2 * 16, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2),
+                         kI16, (c > 0 || kk > 0) ? 1u : 0u);
+            tc::mma_commit(&bar->h2_empty[hb]);
+            if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g]);
           }
           advance(it, g);
         }
@@ -414,7 +416,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         }
       }
       // drain: every MMA this thread issued has completed before tensor memory is freed
-      uint64_t* drain = warp == 4 * G ? &bar->drain : &bar->drain1;
+      uint64_t* drain = warp == 4 * G ? &bar->drain : (warp == 4 * G + 1 ? &bar->drain1 : &bar->drain2);
       tc::mma_commit(drain);
       tc::mbar_wait(drain, 0, abort, kWaitLimitNs);
     }
@@ -478,6 +480,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           }
           bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
           if (kPolicy) {
+            // Write j = 2k + (c >> 1) of h2 buffer c & 1 reuses it after
+            // layer 3 has consumed write j - 1 (completion j - 1 of h2_empty).
+            const int j = 2 * k + (c >> 1);
+            if (half == 0 && j > 0 &&
+                !tc::mbar_wait(&bar->h2_empty[c & 1], (uint32_t)(j - 1) & 1u, abort, kWaitLimitNs))
+              return false;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               const int pos = (4 * half + q) ^ (row & 7);
