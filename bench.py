@@ -363,25 +363,24 @@ def run(args):
     # ---- end to end through the C ABI with host buffers ----
     e2e = None
     if not args.no_e2e:
-        h_traj = env.alloc_traj(T, keys=keys, pinned_host=True)
-        h_val = torch.empty((T, n), dtype=torch.float32, pin_memory=True) if value is not None else None
+        # one env_rollout call per pass with page-locked host arrays (the
+        # library stages them through device buffers); traj.value makes the
+        # same call run the value pass
+        h_keys = keys + (["value"] if value is not None else [])
+        h_traj = env.alloc_traj(T, keys=h_keys, pinned_host=True)
         h_pw = torch.from_numpy(pw).pin_memory()
         h_vw = torch.from_numpy(vw).pin_memory() if vw is not None else None
         h2d = h_pw.numel() * 4 + (h_vw.numel() * 4 if h_vw is not None else 0)
-        d2h = n * T * traj_bytes_per_env_step(keys + (["value"] if value is not None else []))
+        d2h = n * T * traj_bytes_per_env_step(h_keys)
         for _ in range(2):
             env.set_weights(h_pw, h_vw)
             env.rollout(T, h_traj)
-            if h_val is not None:
-                env.value(h_traj["obs"], h_val)
             torch.cuda.synchronize()
         shard.barrier(dist)
         t0 = time.perf_counter()
         for _ in range(max(1, min(args.steps, 5))):
             env.set_weights(h_pw, h_vw)          # step inputs: policy + value weights, H2D
-            env.rollout(T, h_traj)               # trajectory written to pinned host memory
-            if h_val is not None:
-                env.value(h_traj["obs"], h_val)
+            env.rollout(T, h_traj)               # trajectory (and values) to host memory
             torch.cuda.synchronize()
         e2e_s = shard.max_over_ranks((time.perf_counter() - t0) / max(1, min(args.steps, 5)),
                                      dist, "cuda")

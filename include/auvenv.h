@@ -117,7 +117,9 @@ typedef struct auv_buffers {
 } auv_buffers;
 
 /* Trajectory outputs of env_rollout; any pointer may be NULL (not written).
- * Device memory or mapped page-locked host memory, 4-byte aligned.        */
+ * Device memory or mapped page-locked host memory, 4-byte aligned (done:
+ * any alignment).  Host arrays are filled through device staging buffers
+ * (see env_rollout).                                                      */
 typedef struct auv_traj {
   float* obs;     /* [T][18][N] observation the action was taken from   */
   float* act;     /* [T][8][N]  unclipped sampled action a_t            */
@@ -190,6 +192,15 @@ int env_reset(auv_env* env, const uint8_t* mask, void* stream);
  * theta_e - w_act |clip(a)|^2 - w_vs |nu - nu_prev|^2 (weighted norms of
  * Eqs. 2-7); t_ep += 1; done = (t_ep == episode_len); on done the env resets
  * as in env_reset.  The global step t_g advances by T.
+ * In AUV_MLP_BF16 mode traj.value (if given) comes from a value-network pass
+ * over traj.obs after the steps, so traj.obs is required with it.
+ * Host arrays (T >= 2): the steps run in segments into two device staging
+ * buffers (allocated on the first such call, about 2 x 128 MiB, kept until
+ * env_destroy); each finished segment is copied to the host arrays on a
+ * copy stream of the env while the next segment computes.  `stream` waits
+ * for the last copy, so its completion still means every array is written.
+ * With T = 1 host arrays are written in place through their device mapping.
+ * Results do not depend on where the arrays live.
  */
 int env_rollout(auv_env* env, int T, const auv_traj* traj, void* stream);
 

@@ -33,6 +33,14 @@ struct auv_env {
   size_t policy_count, value_count;
   bool weights_set;
   char err[256];
+  // Host trajectories (env_rollout): two device segment buffers, the copy
+  // stream that drains them, and the events ordering the two; made on first use.
+  char* stage = nullptr;
+  size_t stage_bytes = 0;
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t seg_done[2] = {nullptr, nullptr};
+  cudaEvent_t copy_done[2] = {nullptr, nullptr};
+  int last_copy = -1;       // buffer whose copy_done ends the last staged call
 };
 
 namespace {
@@ -283,6 +291,12 @@ int env_destroy(auv_env* env) {
   if (!env) return AUV_ERR_INVALID;
   cudaDeviceSynchronize();
   cudaError_t e = cudaFree(env->workspace);
+  if (env->stage) cudaFree(env->stage);
+  for (int b = 0; b < 2; ++b) {
+    if (env->seg_done[b]) cudaEventDestroy(env->seg_done[b]);
+    if (env->copy_done[b]) cudaEventDestroy(env->copy_done[b]);
+  }
+  if (env->copy_stream) cudaStreamDestroy(env->copy_stream);
   delete env;
   return e == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
 }
@@ -327,6 +341,115 @@ int env_reset(auv_env* env, const uint8_t* mask, void* stream) {
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "reset kernel");
 }
 
+namespace {
+
+// The kernels of T control steps from global step t_g0 (bf16 mode: the fused
+// rollout, then the value network over the observations just written).
+cudaError_t launch_rollout_any(auv_env* env, const Traj& tr, int T, uint64_t t_g0,
+                               cudaStream_t s) {
+  if (env->cfg.mlp_mode == AUV_MLP_FP32)
+    return auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32, env->w_value_f32, tr,
+                                    T, t_g0, env->status, s);
+  cudaError_t e = auv::launch_rollout_bf16(env->model, env->buf, env->w_policy_packed, tr, T,
+                                           t_g0, env->status, s);
+  if (e != cudaSuccess || !tr.value) return e;
+  return auv::launch_value_bf16(env->model, env->w_value_packed, env->w_value_f32, tr.obs,
+                                (size_t)T * env->model.n, env->model.n, tr.value, env->status, s);
+}
+
+constexpr int kTrajArrays = 6;   // obs, act, logp, value, rew, done (auv_traj order)
+
+void** traj_slot(Traj& t, int k) {
+  void** p[kTrajArrays] = {reinterpret_cast<void**>(&t.obs), reinterpret_cast<void**>(&t.act),
+                           reinterpret_cast<void**>(&t.logp), reinterpret_cast<void**>(&t.value),
+                           reinterpret_cast<void**>(&t.rew), reinterpret_cast<void**>(&t.done)};
+  return p[k];
+}
+
+// Host trajectory arrays are filled through device staging: the steps run in
+// segments of `seg` steps into one of two device segment buffers, and each
+// finished segment is copied to the caller's page-locked arrays on the env's
+// copy stream while the next segment computes.  The caller's stream waits
+// for the last copy, so its completion still means the arrays are written.
+int rollout_staged(auv_env* env, int T, const auv_traj* traj, Traj mapped,
+                   const bool host[kTrajArrays], cudaStream_t s) {
+  const size_t n = env->model.n;
+  const size_t row[kTrajArrays] = {18 * n * 4, 8 * n * 4, n * 4, n * 4, n * 4, n};
+  void* const dst[kTrajArrays] = {traj->obs, traj->act, traj->logp, traj->value, traj->rew,
+                                  traj->done};
+  size_t step_bytes = 0;
+  for (int k = 0; k < kTrajArrays; ++k)
+    if (host[k]) step_bytes += row[k];
+  // about 128 MiB per segment buffer: a power of two of steps in [4, T]
+  int seg = 4;
+  while (seg < T && (size_t)(2 * seg) * step_bytes <= ((size_t)1 << 27)) seg *= 2;
+  if (seg > T) seg = T;
+  size_t off[kTrajArrays], half = 0;
+  for (int k = 0; k < kTrajArrays; ++k) {
+    off[k] = half;
+    if (host[k]) half += ((size_t)seg * row[k] + 255) & ~(size_t)255;
+  }
+  cudaError_t e;
+  if (!env->copy_stream) {
+    if ((e = cudaStreamCreateWithFlags(&env->copy_stream, cudaStreamNonBlocking)) != cudaSuccess)
+      return cuda_fail(env, e, "create copy stream");
+    for (int b = 0; b < 2; ++b) {
+      if ((e = cudaEventCreateWithFlags(&env->seg_done[b], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&env->copy_done[b], cudaEventDisableTiming)) != cudaSuccess)
+        return cuda_fail(env, e, "create staging events");
+    }
+  }
+  if (2 * half > env->stage_bytes) {
+    if (env->stage) {   // the previous call's copies may still read the old buffers
+      if ((e = cudaStreamSynchronize(env->copy_stream)) != cudaSuccess)
+        return cuda_fail(env, e, "drain copy stream");
+      cudaFree(env->stage);
+      env->stage = nullptr;
+      env->stage_bytes = 0;
+      env->last_copy = -1;
+    }
+    if ((e = cudaMalloc(&env->stage, 2 * half)) != cudaSuccess)
+      return cuda_fail(env, e, "cudaMalloc(trajectory staging)");
+    env->stage_bytes = 2 * half;
+  }
+  // buffers are reused across calls: start after the previous call's copies
+  if (env->last_copy >= 0 && (e = cudaStreamWaitEvent(s, env->copy_done[env->last_copy], 0)) != cudaSuccess)
+    return cuda_fail(env, e, "order after previous copies");
+  int b = 0;
+  for (int t0 = 0, j = 0; t0 < T; t0 += seg, ++j) {
+    const int len = T - t0 < seg ? T - t0 : seg;
+    b = j & 1;
+    if (j >= 2 && (e = cudaStreamWaitEvent(s, env->copy_done[b], 0)) != cudaSuccess)
+      return cuda_fail(env, e, "wait for segment buffer");
+    Traj ts = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+    for (int k = 0; k < kTrajArrays; ++k) {
+      void* m = *traj_slot(mapped, k);
+      if (!m) continue;
+      *traj_slot(ts, k) = host[k] ? static_cast<void*>(env->stage + b * half + off[k])
+                                  : static_cast<void*>(static_cast<char*>(m) + (size_t)t0 * row[k]);
+    }
+    if ((e = launch_rollout_any(env, ts, len, env->t_g + (uint64_t)t0, s)) != cudaSuccess)
+      return cuda_fail(env, e, "rollout kernels");
+    if ((e = cudaEventRecord(env->seg_done[b], s)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(env->copy_stream, env->seg_done[b], 0)) != cudaSuccess)
+      return cuda_fail(env, e, "order segment copy");
+    for (int k = 0; k < kTrajArrays; ++k) {
+      if (!host[k]) continue;
+      e = cudaMemcpyAsync(static_cast<char*>(dst[k]) + (size_t)t0 * row[k], env->stage + b * half + off[k],
+                          (size_t)len * row[k], cudaMemcpyDeviceToHost, env->copy_stream);
+      if (e != cudaSuccess) return cuda_fail(env, e, "copy trajectory segment");
+    }
+    if ((e = cudaEventRecord(env->copy_done[b], env->copy_stream)) != cudaSuccess)
+      return cuda_fail(env, e, "record segment copy");
+  }
+  env->last_copy = b;
+  if ((e = cudaStreamWaitEvent(s, env->copy_done[b], 0)) != cudaSuccess)
+    return cuda_fail(env, e, "order after last copy");
+  return AUV_OK;
+}
+
+}  // namespace
+
 int env_rollout(auv_env* env, int T, const auv_traj* traj, void* stream) {
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);
@@ -334,40 +457,32 @@ int env_rollout(auv_env* env, int T, const auv_traj* traj, void* stream) {
   if (T < 1) return fail(env, AUV_ERR_INVALID, "T must be >= 1");
   if (!env->weights_set) return fail(env, AUV_ERR_INVALID, "weights not set");
   Traj tr = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  bool host[kTrajArrays] = {false, false, false, false, false, false};
+  bool any_host = false;
   if (traj) {
-    void* d;
-    if ((rc = map_output(env, traj->obs, "traj.obs", 4, &d))) return rc;
-    tr.obs = static_cast<float*>(d);
-    if ((rc = map_output(env, traj->act, "traj.act", 4, &d))) return rc;
-    tr.act = static_cast<float*>(d);
-    if ((rc = map_output(env, traj->logp, "traj.logp", 4, &d))) return rc;
-    tr.logp = static_cast<float*>(d);
-    if ((rc = map_output(env, traj->value, "traj.value", 4, &d))) return rc;
-    tr.value = static_cast<float*>(d);
-    if ((rc = map_output(env, traj->rew, "traj.rew", 4, &d))) return rc;
-    tr.rew = static_cast<float*>(d);
-    if ((rc = map_output(env, traj->done, "traj.done", 1, &d))) return rc;
-    tr.done = static_cast<uint8_t*>(d);
+    const char* names[kTrajArrays] = {"traj.obs", "traj.act", "traj.logp", "traj.value",
+                                      "traj.rew", "traj.done"};
+    void* const given[kTrajArrays] = {traj->obs, traj->act, traj->logp, traj->value, traj->rew,
+                                      traj->done};
+    for (int k = 0; k < kTrajArrays; ++k) {
+      void* d;
+      if ((rc = map_output(env, given[k], names[k], k == 5 ? 1 : 4, &d))) return rc;
+      *traj_slot(tr, k) = d;
+      host[k] = given[k] && classify(given[k], &d) == kHostMapped;
+      any_host |= host[k];
+    }
   }
   if (tr.value && !env->cfg.has_value)
     return fail(env, AUV_ERR_INVALID, "traj.value requested but has_value = 0");
+  if (env->cfg.mlp_mode != AUV_MLP_FP32 && tr.value && !tr.obs)
+    return fail(env, AUV_ERR_INVALID, "bf16 mode computes traj.value from traj.obs: give both");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e;
-  if (env->cfg.mlp_mode == AUV_MLP_FP32) {
-    e = auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32, env->w_value_f32, tr, T,
-                                 env->t_g, env->status, s);
-    if (e != cudaSuccess) return cuda_fail(env, e, "fp32 rollout kernel");
+  if (any_host && T >= 2) {
+    if ((rc = rollout_staged(env, T, traj, tr, host, s))) return rc;
   } else {
-    if (tr.value && !tr.obs)
-      return fail(env, AUV_ERR_INVALID, "bf16 mode computes traj.value from traj.obs: give both");
-    e = auv::launch_rollout_bf16(env->model, env->buf, env->w_policy_packed, tr, T, env->t_g,
-                                 env->status, s);
-    if (e != cudaSuccess) return cuda_fail(env, e, "bf16 rollout kernel");
-    if (tr.value) {
-      e = auv::launch_value_bf16(env->model, env->w_value_packed, env->w_value_f32, tr.obs,
-                                 (size_t)T * env->model.n, env->model.n, tr.value, env->status, s);
-      if (e != cudaSuccess) return cuda_fail(env, e, "bf16 value kernel");
-    }
+    // device arrays, or one step: host arrays are written in place (mapped)
+    cudaError_t e = launch_rollout_any(env, tr, T, env->t_g, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "rollout kernels");
   }
   env->t_g += (uint64_t)T;
   return AUV_OK;
