@@ -252,6 +252,32 @@ def test_split_rollout_is_deterministic(oracle):
     assert torch.equal(e1.state, e2.state)
 
 
+def test_checkpoint_resume_in_a_new_env(oracle):
+    """Checkpoint = the caller's state, params and counter buffers plus the
+    global step (env_get_step); restoring them into a fresh env (copy +
+    env_set_step) continues the rollout bit for bit, trajectory and state."""
+    torch = need_gpu()
+    w = W.workload("dr_16384", n_envs=1000, episode_len=17)
+    a = make_env(w)
+    a.reset()
+    a.rollout(25, a.alloc_traj(25))
+    snap = {k: getattr(a, k).clone() for k in ("state", "params", "t_ep", "episode")}
+    step = a.t_g
+    assert step == 25
+    b = make_env(w)
+    for k, v in snap.items():
+        getattr(b, k).copy_(v)
+    b.t_g = step
+    ta, tb = a.alloc_traj(30), b.alloc_traj(30)
+    a.rollout(30, ta)
+    b.rollout(30, tb)
+    for k in ta:
+        assert torch.equal(ta[k], tb[k]), k
+    for k in snap:
+        assert torch.equal(getattr(a, k), getattr(b, k)), k
+    assert b.t_g == a.t_g == 55
+
+
 def test_nan_state_is_reported(oracle):
     torch = need_gpu()
     w = W.workload("tiny_64", n_envs=300)
