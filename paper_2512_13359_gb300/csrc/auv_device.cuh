@@ -375,19 +375,35 @@ __device__ __forceinline__ void substep(const Model& M, Env& e, const float tau[
   float rbxk[3];
   cross3(e.rb, kb, rbxk);
   const float nur[6] = {vr[0], vr[1], vr[2], w[0], w[1], w[2]};
+  // Damping and the velocity update are the same for all six axes: two axes
+  // per packed fp32 instruction (each lane rounded as the scalar operation).
+  float damp[6];
+#pragma unroll
+  for (int j = 0; j < 3; ++j) {
+    const float2 an = make_float2(fabsf(nur[2 * j]), fabsf(nur[2 * j + 1]));
+    float2 t = __ffma2_rn(make_float2(M.dquad[2 * j], M.dquad[2 * j + 1]), an,
+                          make_float2(M.dlin[2 * j], M.dlin[2 * j + 1]));
+    t = __fmul2_rn(make_float2(e.sd, e.sd), t);
+    t = __fmul2_rn(t, make_float2(nur[2 * j], nur[2 * j + 1]));
+    damp[2 * j] = t.x;
+    damp[2 * j + 1] = t.y;
+  }
   float rhs[6];
 #pragma unroll
-  for (int k = 0; k < 3; ++k) {
-    const float damp = e.sd * (M.dlin[k] + M.dquad[k] * fabsf(nur[k])) * nur[k];
-    rhs[k] = tau[k] - m * wxv[k] - c0[k] - damp - e.dB * kb[k] - e.sa * M.added[k] * wxvc[k];
-  }
+  for (int k = 0; k < 3; ++k)
+    rhs[k] = tau[k] - m * wxv[k] - c0[k] - damp[k] - e.dB * kb[k] - e.sa * M.added[k] * wxvc[k];
 #pragma unroll
-  for (int k = 0; k < 3; ++k) {
-    const float damp = e.sd * (M.dlin[3 + k] + M.dquad[3 + k] * fabsf(nur[3 + k])) * nur[3 + k];
-    rhs[3 + k] = tau[3 + k] - wxIw[k] - c1[k] - c2[k] - damp - B * rbxk[k];
-  }
+  for (int k = 0; k < 3; ++k)
+    rhs[3 + k] = tau[3 + k] - wxIw[k] - c1[k] - c2[k] - damp[3 + k] - B * rbxk[k];
+  const float2 h2 = make_float2(M.h, M.h);
 #pragma unroll
-  for (int k = 0; k < 6; ++k) e.nu[k] = fmaf(M.h, rhs[k] * e.inv_m[k], e.nu[k]);
+  for (int j = 0; j < 3; ++j) {
+    const float2 nv = __ffma2_rn(h2, __fmul2_rn(make_float2(rhs[2 * j], rhs[2 * j + 1]),
+                                                make_float2(e.inv_m[2 * j], e.inv_m[2 * j + 1])),
+                                 make_float2(e.nu[2 * j], e.nu[2 * j + 1]));
+    e.nu[2 * j] = nv.x;
+    e.nu[2 * j + 1] = nv.y;
+  }
   // position with the new body velocity, attitude at the start of the substep
 #pragma unroll
   for (int i = 0; i < 3; ++i)
