@@ -27,6 +27,11 @@
 // a buoyancy offset, a centre-of-buoyancy offset and a water current.
 // Episodes: §V-A1 (fixed-length episodes with a fresh random reference).
 //
+// A second model, the paper's own environment (wrench action of Eq. 1,
+// inertia-box fluid model, effective gravity, 12-float axis-angle observation,
+// five-term reward of Eqs. 2-7), follows the Fossen model below under the
+// names paper_* / oracle_paper_*.
+//
 // Parity pins for every function here live in tests/test_oracle_*.py.
 
 #include <cmath>
@@ -686,6 +691,397 @@ void rk4_deriv(const OracleModel& m, const Env<R>& e, const R y[13], const R tau
   for (int k = 0; k < 6; ++k) dy[7 + k] = acc[k];
 }
 
+// ============================================================================
+// The paper's own environment (§IV-B "Environment Specifications", Eqs. (1)-(7),
+// §IV-C), next to the thruster-level Fossen model above:
+//  - action: a normalised body wrench a = [F; tau] in [-1, 1]^6, scaled by
+//    F_max and tau_max (Eq. 1);
+//  - dynamics: a free rigid body (no added mass) in still water under the
+//    "inertia" fluid model the paper names: the body is replaced by the
+//    uniform box that has its mass and principal moments, and that box feels
+//    quadratic pressure drag on its faces and viscous (Stokes) resistance;
+//    buoyancy is folded into an effective gravity acting at the centre of
+//    mass (centres of gravity and buoyancy coincide), randomised per episode;
+//  - observation (12): body-frame position error, axis-angle attitude error,
+//    body linear velocity, body angular velocity (§IV-B1);
+//  - reward: r_pos + r_att + r_act + r_vel + r_act-mavg (Eqs. 2-7).
+// Integration, noise streams and networks are those of the Fossen model.
+// ============================================================================
+struct PaperModel {
+  int32_t n_substeps;     // physics substeps per control step
+  int32_t episode_len;    // control steps per episode
+  uint32_t seed;          // second Philox key word
+  int32_t dr_enable;      // 1: draw the effective gravity offset
+  int32_t mavg_len;       // K: actions in the moving average, 1..8
+  int32_t pad0;
+  double dt;              // control period [s]
+  double mass;            // m [kg]
+  double inertia[3];      // principal moments about the centre of mass [kg m^2]
+  double f_max, tau_max;  // Eq. (1) scaling of the normalised wrench
+  double rho;             // fluid density [kg/m^3]
+  double visc;            // fluid dynamic viscosity [Pa s]
+  double g_eff;           // nominal effective gravity along world -z [m/s^2]
+  double w_pos, w_axes[3], w_att, w_act, w_vel, w_mavg;   // Eqs. (2)-(7)
+  float goal_pos_range;   // goal position U[-r, r] per axis [m]
+  float goal_att_range;   // goal roll, pitch, yaw U[-r, r] [rad]
+  float init_pos_range;   // initial position U[-r, r] per axis [m]
+  float init_att_range;   // initial roll, pitch, yaw U[-r, r] [rad]
+  float dr_gravity_range; // effective gravity offset U[-r, r] [m/s^2]
+  int32_t hidden;         // hidden width of both networks
+  int32_t policy_out;     // 6 (mean; fixed log-std) or 12 (mean and log-std head)
+  int32_t mlp_bf16;
+  int32_t has_value;
+  float logstd_fixed[6];
+  float logstd_min, logstd_max;
+};
+
+constexpr int kPObs = 12;
+constexpr int kPAct = 6;
+constexpr int kPHist = 8;                    // action-history slots kept (K <= 8)
+constexpr int kPStateF = 13 + 6 * kPHist;    // p(3) q(4) nu(6) history[8][6]
+constexpr int kPParamF = 8;                  // p_d(3) q_d(4) g_eff
+
+template <class R>
+struct PaperEnv {
+  R p[3], q[4], nu[6], hist[kPHist][6];
+  R p_d[3], q_d[4], g_eff;
+  int32_t t_ep;
+  uint32_t episode;
+};
+
+// Z-Y-X Euler angles -> unit quaternion q_z(yaw) (x) q_y(pitch) (x) q_x(roll),
+// float, fixed steps (bit-exact across implementations of the same steps).
+void euler_to_quat(float roll, float pitch, float yaw, float q[4]) {
+  float cr = taylor_cos(0.5f * roll), sr = taylor_sin(0.5f * roll);
+  float cp = taylor_cos(0.5f * pitch), sp = taylor_sin(0.5f * pitch);
+  float cy = taylor_cos(0.5f * yaw), sy = taylor_sin(0.5f * yaw);
+  float a = cy * cp, b = sy * sp, c = cy * sp, e = sy * cp;
+  q[0] = std::fmaf(a, cr, b * sr);
+  q[1] = std::fmaf(a, sr, -(b * cr));
+  q[2] = std::fmaf(c, cr, e * sr);
+  q[3] = std::fmaf(e, cr, -(c * sr));
+}
+
+// Episode start (§V-A1: a random 6-DOF reference per episode, §IV-C: the
+// effective gravity redrawn per environment).  Thirteen uniforms from the
+// reset stream, in this order: goal x, y, z; goal roll, pitch, yaw; gravity
+// offset; initial x, y, z; initial roll, pitch, yaw.  Velocities and the
+// action history start at zero.
+template <class R>
+void paper_apply_reset(const PaperModel& m, uint32_t env_id, PaperEnv<R>& e) {
+  uint32_t w[16];
+  draw_words(env_id, m.seed, e.episode, 1u, 4, w);
+  float u[13];
+  for (int j = 0; j < 13; ++j) u[j] = word_to_uniform(w[j]);
+  float qd[4], q0[4];
+  euler_to_quat(draw_sym(u[3], m.goal_att_range), draw_sym(u[4], m.goal_att_range),
+                draw_sym(u[5], m.goal_att_range), qd);
+  euler_to_quat(draw_sym(u[10], m.init_att_range), draw_sym(u[11], m.init_att_range),
+                draw_sym(u[12], m.init_att_range), q0);
+  for (int k = 0; k < 3; ++k) {
+    e.p_d[k] = draw_sym(u[k], m.goal_pos_range);
+    e.p[k] = draw_sym(u[7 + k], m.init_pos_range);
+  }
+  for (int k = 0; k < 4; ++k) { e.q_d[k] = qd[k]; e.q[k] = q0[k]; }
+  const float g0 = (float)m.g_eff;
+  e.g_eff = m.dr_enable ? g0 + draw_sym(u[6], m.dr_gravity_range) : g0;
+  for (int k = 0; k < 6; ++k) e.nu[k] = 0;
+  for (int j = 0; j < kPHist; ++j)
+    for (int k = 0; k < 6; ++k) e.hist[j][k] = 0;
+  e.t_ep = 0;
+  e.episode += 1u;
+}
+
+// Sides of the uniform box with the body's mass and principal moments:
+// I_x = m (b_y^2 + b_z^2) / 12 and so on, solved for the sides.
+template <class R>
+void paper_box(const PaperModel& m, R b[3]) {
+  const R I0 = (R)m.inertia[0], I1 = (R)m.inertia[1], I2 = (R)m.inertia[2], M = (R)m.mass;
+  b[0] = std::sqrt(6 * (I1 + I2 - I0) / M);
+  b[1] = std::sqrt(6 * (I0 + I2 - I1) / M);
+  b[2] = std::sqrt(6 * (I0 + I1 - I2) / M);
+}
+
+// Hydrodynamic wrench on the box moving with body velocity nu in still water,
+// every term kept separate: pressure drag -1/2 rho A_i |v_i| v_i on the face
+// areas A = (b_y b_z, b_x b_z, b_x b_y); its rotational counterpart
+// -rho/64 b_i (b_j^4 + b_k^4) |w_i| w_i (the pressure on the halves of the
+// faces moving into the fluid, integrated over the face); Stokes resistance
+// -3 pi mu d v and -pi mu d^3 w of the sphere of diameter d = (b_x+b_y+b_z)/3.
+template <class R>
+void paper_fluid(const PaperModel& m, const R nu[6], R f[6]) {
+  R b[3];
+  paper_box(m, b);
+  const R rho = (R)m.rho, mu = (R)m.visc, pi = (R)3.14159265358979323846;
+  const R d = (b[0] + b[1] + b[2]) / 3;
+  const R area[3] = {b[1] * b[2], b[0] * b[2], b[0] * b[1]};
+  for (int k = 0; k < 3; ++k) {
+    const int j = (k + 1) % 3, l = (k + 2) % 3;
+    const R v = nu[k], w = nu[3 + k];
+    const R drag_f = -(R)0.5 * rho * area[k] * std::fabs(v) * v;
+    const R visc_f = -3 * pi * mu * d * v;
+    const R b4 = b[j] * b[j] * b[j] * b[j] + b[l] * b[l] * b[l] * b[l];
+    const R drag_t = -rho / 64 * b[k] * b4 * std::fabs(w) * w;
+    const R visc_t = -pi * mu * d * d * d * w;
+    f[k] = drag_f + visc_f;
+    f[3 + k] = drag_t + visc_t;
+  }
+}
+
+// nu_dot = M_RB^{-1} (tau + fluid(nu) + R^T (0, 0, -m g_eff) - C_RB(nu) nu).
+template <class R>
+void paper_nu_dot(const PaperModel& m, const PaperEnv<R>& e, const R q[4], const R nu[6],
+                  const R tau[6], R out[6]) {
+  R Rm[3][3];
+  quat_to_rot(q, Rm);
+  const R v[3] = {nu[0], nu[1], nu[2]};
+  const R w[3] = {nu[3], nu[4], nu[5]};
+  const R M = (R)m.mass;
+  const R I[3] = {(R)m.inertia[0], (R)m.inertia[1], (R)m.inertia[2]};
+  R fl[6];
+  paper_fluid(m, nu, fl);
+  const R gw[3] = {0, 0, -M * e.g_eff};
+  R gb[3];
+  mat_t_vec(Rm, gw, gb);
+  R wxv[3], Iw[3] = {I[0] * w[0], I[1] * w[1], I[2] * w[2]}, wxIw[3];
+  cross(w, v, wxv);
+  cross(w, Iw, wxIw);
+  for (int k = 0; k < 3; ++k) {
+    out[k] = (tau[k] + fl[k] + gb[k] - M * wxv[k]) / M;
+    out[3 + k] = (tau[3 + k] + fl[3 + k] - wxIw[k]) / I[k];
+  }
+}
+
+// One semi-implicit Euler substep (the integrator of the Fossen model).
+template <class R>
+void paper_substep(const PaperModel& m, PaperEnv<R>& e, const R tau[6], R h) {
+  R acc[6];
+  paper_nu_dot(m, e, e.q, e.nu, tau, acc);
+  for (int k = 0; k < 6; ++k) e.nu[k] = e.nu[k] + h * acc[k];
+  R Rm[3][3];
+  quat_to_rot(e.q, Rm);
+  R pdot[3];
+  const R v[3] = {e.nu[0], e.nu[1], e.nu[2]};
+  mat_vec(Rm, v, pdot);
+  for (int k = 0; k < 3; ++k) e.p[k] = e.p[k] + h * pdot[k];
+  R phi[3] = {h * e.nu[3], h * e.nu[4], h * e.nu[5]};
+  R dq[4], qn[4];
+  quat_exp(phi, dq);
+  quat_mul(e.q, dq, qn);
+  R n = std::sqrt(qn[0] * qn[0] + qn[1] * qn[1] + qn[2] * qn[2] + qn[3] * qn[3]);
+  for (int k = 0; k < 4; ++k) e.q[k] = qn[k] / n;
+}
+
+// Axis-angle vector of q_e = conj(q_d) (x) q (the attitude of the body in the
+// goal frame), on the short way round: angle in [0, pi].
+template <class R>
+void paper_att_error(const PaperEnv<R>& e, R out[3]) {
+  const R qdc[4] = {e.q_d[0], -e.q_d[1], -e.q_d[2], -e.q_d[3]};
+  R qe[4];
+  quat_mul(qdc, e.q, qe);
+  if (qe[0] < 0)
+    for (int k = 0; k < 4; ++k) qe[k] = -qe[k];
+  const R vn = std::sqrt(qe[1] * qe[1] + qe[2] * qe[2] + qe[3] * qe[3]);
+  const R s = vn > 0 ? 2 * std::atan2(vn, qe[0]) / vn : 2 / qe[0];
+  for (int k = 0; k < 3; ++k) out[k] = s * qe[1 + k];
+}
+
+// Observation (§IV-B1): [R^T (p - p_d), axis-angle error, v, w].
+template <class R>
+void paper_observe(const PaperEnv<R>& e, R obs[kPObs]) {
+  R Rm[3][3];
+  quat_to_rot(e.q, Rm);
+  const R dp[3] = {e.p[0] - e.p_d[0], e.p[1] - e.p_d[1], e.p[2] - e.p_d[2]};
+  R dpb[3], th[3];
+  mat_t_vec(Rm, dp, dpb);
+  paper_att_error(e, th);
+  for (int k = 0; k < 3; ++k) { obs[k] = dpb[k]; obs[3 + k] = th[k]; }
+  for (int k = 0; k < 6; ++k) obs[6 + k] = e.nu[k];
+}
+
+// Reward (Eqs. 2-7) on the post-step state with the clipped action a_c and
+// the mean of the K previous clipped actions (zeros before the episode's
+// K-th step).
+template <class R>
+R paper_reward(const PaperModel& m, const PaperEnv<R>& e, const R a_c[kPAct]) {
+  R obs[kPObs];
+  paper_observe(e, obs);
+  R r_pos = 0, r_att = 0, r_act = 0, r_vel = 0, r_mavg = 0;
+  for (int k = 0; k < 3; ++k) {
+    const R dk = (R)m.w_axes[k] * obs[k];
+    r_pos += dk * dk;
+    r_att += obs[3 + k] * obs[3 + k];
+    r_act += a_c[3 + k] * a_c[3 + k];
+    r_vel += e.nu[3 + k] * e.nu[3 + k];
+  }
+  for (int k = 0; k < kPAct; ++k) {
+    R mean = 0;
+    for (int j = 0; j < m.mavg_len; ++j) mean += e.hist[j][k];
+    mean = mean / (R)m.mavg_len;
+    r_mavg += (a_c[k] - mean) * (a_c[k] - mean);
+  }
+  return -(R)m.w_pos * r_pos - (R)m.w_att * r_att - (R)m.w_act * r_act - (R)m.w_vel * r_vel -
+         (R)m.w_mavg * r_mavg;
+}
+
+// Eq. (1): clip to [-1, 1], scale forces by F_max and torques by tau_max.
+template <class R>
+void paper_wrench(const PaperModel& m, const R a[kPAct], R a_c[kPAct], R tau[6]) {
+  for (int k = 0; k < kPAct; ++k) a_c[k] = a[k] < -1 ? (R)-1 : (a[k] > 1 ? (R)1 : a[k]);
+  for (int k = 0; k < 3; ++k) {
+    tau[k] = (R)m.f_max * a_c[k];
+    tau[3 + k] = (R)m.tau_max * a_c[3 + k];
+  }
+}
+
+template <class R>
+R paper_control_step(const PaperModel& m, uint32_t env_id, PaperEnv<R>& e, const R a[kPAct],
+                     uint8_t* done) {
+  R a_c[kPAct], tau[6];
+  paper_wrench(m, a, a_c, tau);
+  const R h = (R)m.dt / (R)m.n_substeps;
+  for (int s = 0; s < m.n_substeps; ++s) paper_substep(m, e, tau, h);
+  R r = paper_reward(m, e, a_c);
+  for (int k = 0; k < kPAct; ++k) e.hist[e.t_ep % m.mavg_len][k] = a_c[k];
+  e.t_ep += 1;
+  *done = (e.t_ep == m.episode_len) ? 1 : 0;
+  if (*done) paper_apply_reset(m, env_id, e);
+  return r;
+}
+
+template <class R>
+void paper_load(const double* st, const double* pr, const int32_t* t_ep, const uint32_t* ep,
+                int n, int i, PaperEnv<R>& e) {
+  for (int k = 0; k < 3; ++k) e.p[k] = (R)st[k * n + i];
+  for (int k = 0; k < 4; ++k) e.q[k] = (R)st[(3 + k) * n + i];
+  for (int k = 0; k < 6; ++k) e.nu[k] = (R)st[(7 + k) * n + i];
+  for (int j = 0; j < kPHist; ++j)
+    for (int k = 0; k < 6; ++k) e.hist[j][k] = (R)st[(13 + 6 * j + k) * n + i];
+  for (int k = 0; k < 3; ++k) e.p_d[k] = (R)pr[k * n + i];
+  for (int k = 0; k < 4; ++k) e.q_d[k] = (R)pr[(3 + k) * n + i];
+  e.g_eff = (R)pr[7 * n + i];
+  e.t_ep = t_ep[i];
+  e.episode = ep[i];
+}
+
+template <class R>
+void paper_store_state(const PaperEnv<R>& e, int n, int i, double* st) {
+  for (int k = 0; k < 3; ++k) st[k * n + i] = (double)e.p[k];
+  for (int k = 0; k < 4; ++k) st[(3 + k) * n + i] = (double)e.q[k];
+  for (int k = 0; k < 6; ++k) st[(7 + k) * n + i] = (double)e.nu[k];
+  for (int j = 0; j < kPHist; ++j)
+    for (int k = 0; k < 6; ++k) st[(13 + 6 * j + k) * n + i] = (double)e.hist[j][k];
+}
+
+template <class R>
+void paper_store(const PaperEnv<R>& e, int n, int i, double* st, double* pr, int32_t* t_ep,
+                 uint32_t* ep) {
+  paper_store_state(e, n, i, st);
+  for (int k = 0; k < 3; ++k) pr[k * n + i] = (double)e.p_d[k];
+  for (int k = 0; k < 4; ++k) pr[(3 + k) * n + i] = (double)e.q_d[k];
+  pr[7 * n + i] = (double)e.g_eff;
+  t_ep[i] = e.t_ep;
+  ep[i] = e.episode;
+}
+
+template <class R>
+void paper_replay_impl(const PaperModel& m, int n, const uint32_t* env_ids, double* st,
+                       double* pr, int32_t* t_ep, uint32_t* ep, int T, const float* act,
+                       double* rew, uint8_t* done, double* trace) {
+  for (int i = 0; i < n; ++i) {
+    PaperEnv<R> e;
+    paper_load<R>(st, pr, t_ep, ep, n, i, e);
+    for (int t = 0; t < T; ++t) {
+      R a[kPAct];
+      for (int k = 0; k < kPAct; ++k) a[k] = (R)act[((size_t)t * kPAct + k) * n + i];
+      uint8_t d;
+      R r = paper_control_step(m, env_ids[i], e, a, &d);
+      rew[(size_t)t * n + i] = (double)r;
+      done[(size_t)t * n + i] = d;
+      if (trace) paper_store_state(e, n, i, trace + (size_t)t * kPStateF * n);
+    }
+    paper_store(e, n, i, st, pr, t_ep, ep);
+  }
+}
+
+template <class R>
+void paper_rollout_impl(const PaperModel& m, const float* pol_w, const float* val_w, int n,
+                        const uint32_t* env_ids, double* st, double* pr, int32_t* t_ep,
+                        uint32_t* ep, uint64_t t_g0, int T, double* obs_out, double* act_out,
+                        double* logp_out, double* value_out, double* rew_out,
+                        uint8_t* done_out) {
+  const double half_log_2pi = 0.91893853320467274178032973640562;
+  for (int i = 0; i < n; ++i) {
+    PaperEnv<R> e;
+    paper_load<R>(st, pr, t_ep, ep, n, i, e);
+    for (int t = 0; t < T; ++t) {
+      R obs[kPObs];
+      paper_observe(e, obs);
+      R out[12];
+      mlp_forward<R>(pol_w, kPObs, m.hidden, m.policy_out, m.mlp_bf16 != 0, obs, out);
+      R mu[kPAct], logstd[kPAct];
+      for (int k = 0; k < kPAct; ++k) {
+        mu[k] = out[k];
+        if (m.policy_out == 12) {
+          R ls = out[kPAct + k];
+          ls = ls < (R)m.logstd_min ? (R)m.logstd_min : ls;
+          logstd[k] = ls > (R)m.logstd_max ? (R)m.logstd_max : ls;
+        } else {
+          logstd[k] = (R)m.logstd_fixed[k];
+        }
+      }
+      // the first six of the eight normals of the action-noise stream
+      uint32_t w[8];
+      draw_words(env_ids[i], m.seed, t_g0 + (uint64_t)t, 0u, 2, w);
+      float u[8];
+      for (int k = 0; k < 8; ++k) u[k] = word_to_uniform(w[k]);
+      double eps[8];
+      box_muller8(u, eps);
+      R a[kPAct];
+      double logp = 0;
+      for (int k = 0; k < kPAct; ++k) {
+        a[k] = mu[k] + (R)std::exp((double)logstd[k]) * (R)eps[k];
+        logp += -0.5 * eps[k] * eps[k] - (double)logstd[k] - half_log_2pi;
+      }
+      if (value_out && m.has_value) {
+        R v;
+        mlp_forward<R>(val_w, kPObs, m.hidden, 1, m.mlp_bf16 != 0, obs, &v);
+        value_out[(size_t)t * n + i] = (double)v;
+      }
+      if (obs_out)
+        for (int k = 0; k < kPObs; ++k) obs_out[((size_t)t * kPObs + k) * n + i] = (double)obs[k];
+      if (act_out)
+        for (int k = 0; k < kPAct; ++k) act_out[((size_t)t * kPAct + k) * n + i] = (double)a[k];
+      if (logp_out) logp_out[(size_t)t * n + i] = logp;
+      uint8_t d;
+      R r = paper_control_step(m, env_ids[i], e, a, &d);
+      if (rew_out) rew_out[(size_t)t * n + i] = (double)r;
+      if (done_out) done_out[(size_t)t * n + i] = d;
+    }
+    paper_store(e, n, i, st, pr, t_ep, ep);
+  }
+}
+
+template <class R>
+void paper_rk4_deriv(const PaperModel& m, const PaperEnv<R>& e, const R y[13], const R tau[6],
+                     R dy[13]) {
+  const R q[4] = {y[3], y[4], y[5], y[6]};
+  const R nu[6] = {y[7], y[8], y[9], y[10], y[11], y[12]};
+  R Rm[3][3];
+  quat_to_rot(q, Rm);
+  const R v[3] = {nu[0], nu[1], nu[2]};
+  R pd[3];
+  mat_vec(Rm, v, pd);
+  const R wq[4] = {0, nu[3], nu[4], nu[5]};
+  R qd[4];
+  quat_mul(q, wq, qd);
+  R acc[6];
+  paper_nu_dot(m, e, q, nu, tau, acc);
+  for (int k = 0; k < 3; ++k) dy[k] = pd[k];
+  for (int k = 0; k < 4; ++k) dy[3 + k] = qd[k] / 2;
+  for (int k = 0; k < 6; ++k) dy[7 + k] = acc[k];
+}
+
 }  // namespace
 
 extern "C" {
@@ -820,6 +1216,108 @@ void oracle_integrate(const OracleModel* m, int method, double* st, const double
     }
   }
   store_state(e, 1, 0, st);
+}
+
+// ---- the paper's own environment ------------------------------------------
+int oracle_paper_model_size() { return (int)sizeof(PaperModel); }
+
+void oracle_paper_reset(const PaperModel* m, int n, const uint32_t* env_ids, double* st,
+                        double* pr, int32_t* t_ep, uint32_t* ep) {
+  for (int i = 0; i < n; ++i) {
+    PaperEnv<double> e;
+    std::memset(&e, 0, sizeof(e));
+    e.episode = ep[i];
+    paper_apply_reset(*m, env_ids[i], e);
+    paper_store(e, n, i, st, pr, t_ep, ep);
+  }
+}
+
+void oracle_paper_replay(const PaperModel* m, int precision, int n, const uint32_t* env_ids,
+                         double* st, double* pr, int32_t* t_ep, uint32_t* ep, int T,
+                         const float* act, double* rew, uint8_t* done, double* trace) {
+  if (precision == 1)
+    paper_replay_impl<float>(*m, n, env_ids, st, pr, t_ep, ep, T, act, rew, done, trace);
+  else
+    paper_replay_impl<double>(*m, n, env_ids, st, pr, t_ep, ep, T, act, rew, done, trace);
+}
+
+void oracle_paper_rollout(const PaperModel* m, int precision, const float* pol_w,
+                          const float* val_w, int n, const uint32_t* env_ids, double* st,
+                          double* pr, int32_t* t_ep, uint32_t* ep, uint64_t t_g0, int T,
+                          double* obs, double* act, double* logp, double* value, double* rew,
+                          uint8_t* done) {
+  if (precision == 1)
+    paper_rollout_impl<float>(*m, pol_w, val_w, n, env_ids, st, pr, t_ep, ep, t_g0, T, obs, act,
+                              logp, value, rew, done);
+  else
+    paper_rollout_impl<double>(*m, pol_w, val_w, n, env_ids, st, pr, t_ep, ep, t_g0, T, obs,
+                               act, logp, value, rew, done);
+}
+
+// Observation of one env (SoA with n = 1).
+void oracle_paper_observe(const double* st, const double* pr, double* obs) {
+  int32_t t = 0;
+  uint32_t e0 = 0;
+  PaperEnv<double> e;
+  paper_load<double>(st, pr, &t, &e0, 1, 0, e);
+  paper_observe(e, obs);
+}
+
+// Reward of one env's (post-step) state with clipped action a_c and its history.
+double oracle_paper_reward(const PaperModel* m, const double* st, const double* pr,
+                           const double* a_c) {
+  int32_t t = 0;
+  uint32_t e0 = 0;
+  PaperEnv<double> e;
+  paper_load<double>(st, pr, &t, &e0, 1, 0, e);
+  return paper_reward(*m, e, a_c);
+}
+
+void oracle_paper_wrench(const PaperModel* m, const double* a, double* a_c, double* tau) {
+  paper_wrench(*m, a, a_c, tau);
+}
+
+void oracle_paper_box(const PaperModel* m, double* b) { paper_box(*m, b); }
+
+void oracle_paper_nu_dot(const PaperModel* m, const double* st, const double* pr,
+                         const double* tau, double* out) {
+  int32_t t = 0;
+  uint32_t e0 = 0;
+  PaperEnv<double> e;
+  paper_load<double>(st, pr, &t, &e0, 1, 0, e);
+  paper_nu_dot(*m, e, e.q, e.nu, tau, out);
+}
+
+// Physics only, constant wrench: method 0 = the model's integrator, 1 = RK4.
+void oracle_paper_integrate(const PaperModel* m, int method, double* st, const double* pr,
+                            const double* tau, double h, int n_steps) {
+  int32_t t = 0;
+  uint32_t e0 = 0;
+  PaperEnv<double> e;
+  paper_load<double>(st, pr, &t, &e0, 1, 0, e);
+  for (int s = 0; s < n_steps; ++s) {
+    if (method == 0) {
+      paper_substep(*m, e, tau, h);
+    } else {
+      double y[13], k1[13], k2[13], k3[13], k4[13], yt[13];
+      for (int k = 0; k < 3; ++k) y[k] = e.p[k];
+      for (int k = 0; k < 4; ++k) y[3 + k] = e.q[k];
+      for (int k = 0; k < 6; ++k) y[7 + k] = e.nu[k];
+      paper_rk4_deriv(*m, e, y, tau, k1);
+      for (int k = 0; k < 13; ++k) yt[k] = y[k] + h / 2 * k1[k];
+      paper_rk4_deriv(*m, e, yt, tau, k2);
+      for (int k = 0; k < 13; ++k) yt[k] = y[k] + h / 2 * k2[k];
+      paper_rk4_deriv(*m, e, yt, tau, k3);
+      for (int k = 0; k < 13; ++k) yt[k] = y[k] + h * k3[k];
+      paper_rk4_deriv(*m, e, yt, tau, k4);
+      for (int k = 0; k < 13; ++k) y[k] = y[k] + h / 6 * (k1[k] + 2 * k2[k] + 2 * k3[k] + k4[k]);
+      double qn = std::sqrt(y[3] * y[3] + y[4] * y[4] + y[5] * y[5] + y[6] * y[6]);
+      for (int k = 0; k < 3; ++k) e.p[k] = y[k];
+      for (int k = 0; k < 4; ++k) e.q[k] = y[3 + k] / qn;
+      for (int k = 0; k < 6; ++k) e.nu[k] = y[7 + k];
+    }
+  }
+  paper_store_state(e, 1, 0, st);
 }
 
 }  // extern "C"

@@ -258,3 +258,208 @@ def integrate(m, st, pr, tau, h, n_steps, method="euler"):
                            _p(np.ascontiguousarray(tau, dtype=np.float64)), float(h),
                            int(n_steps))
     return s
+
+
+# ---------------------------------------------------------------------------
+# The paper's own environment (§IV-B; see PaperModel in auv_oracle.cpp)
+# ---------------------------------------------------------------------------
+PAPER_OBS, PAPER_ACT, PAPER_HIST = 12, 6, 8
+PAPER_STATE, PAPER_PARAM = 13 + 6 * PAPER_HIST, 8
+
+
+class PaperModel(C.Structure):
+    _fields_ = [
+        ("n_substeps", C.c_int32), ("episode_len", C.c_int32), ("seed", C.c_uint32),
+        ("dr_enable", C.c_int32), ("mavg_len", C.c_int32), ("pad0", C.c_int32),
+        ("dt", C.c_double), ("mass", C.c_double), ("inertia", C.c_double * 3),
+        ("f_max", C.c_double), ("tau_max", C.c_double), ("rho", C.c_double),
+        ("visc", C.c_double), ("g_eff", C.c_double),
+        ("w_pos", C.c_double), ("w_axes", C.c_double * 3), ("w_att", C.c_double),
+        ("w_act", C.c_double), ("w_vel", C.c_double), ("w_mavg", C.c_double),
+        ("goal_pos_range", C.c_float), ("goal_att_range", C.c_float),
+        ("init_pos_range", C.c_float), ("init_att_range", C.c_float),
+        ("dr_gravity_range", C.c_float),
+        ("hidden", C.c_int32), ("policy_out", C.c_int32), ("mlp_bf16", C.c_int32),
+        ("has_value", C.c_int32), ("logstd_fixed", C.c_float * 6),
+        ("logstd_min", C.c_float), ("logstd_max", C.c_float),
+    ]
+
+
+def _paper_lib():
+    L = lib()
+    if not getattr(L, "_paper_ready", False):
+        P = C.c_void_p
+        L.oracle_paper_model_size.restype = C.c_int
+        L.oracle_paper_reset.argtypes = [P, C.c_int, P, P, P, P, P]
+        L.oracle_paper_replay.argtypes = [P, C.c_int, C.c_int, P, P, P, P, P, C.c_int, P, P, P,
+                                          P]
+        L.oracle_paper_rollout.argtypes = [P, C.c_int, P, P, C.c_int, P, P, P, P, P,
+                                           C.c_uint64, C.c_int, P, P, P, P, P, P]
+        L.oracle_paper_observe.argtypes = [P, P, P]
+        L.oracle_paper_reward.argtypes = [P, P, P, P]
+        L.oracle_paper_reward.restype = C.c_double
+        L.oracle_paper_wrench.argtypes = [P, P, P, P]
+        L.oracle_paper_box.argtypes = [P, P]
+        L.oracle_paper_nu_dot.argtypes = [P, P, P, P, P]
+        L.oracle_paper_integrate.argtypes = [P, C.c_int, P, P, P, C.c_double, C.c_int]
+        assert L.oracle_paper_model_size() == C.sizeof(PaperModel), "PaperModel layout mismatch"
+        L._paper_ready = True
+    return L
+
+
+def paper_model(w: dict) -> PaperModel:
+    """PaperModel from a paper-model workload dict."""
+    m = PaperModel()
+    m.n_substeps = int(w["substeps"])
+    m.episode_len = int(w["episode_len"])
+    m.seed = int(w["seed"]) & 0xFFFFFFFF
+    m.dr_enable = int(w["dr_enable"])
+    m.mavg_len = int(w["mavg_len"])
+    m.dt = float(w["dt"])
+    m.mass = float(w["mass"])
+    m.inertia[:] = [float(x) for x in w["inertia"]]
+    m.f_max, m.tau_max = float(w["f_max"]), float(w["tau_max"])
+    m.rho, m.visc = float(w["fluid_density"]), float(w["fluid_viscosity"])
+    m.g_eff = float(w["g_eff"])
+    m.w_pos = float(w["w_pos"])
+    m.w_axes[:] = [float(x) for x in w["w_axes"]]
+    m.w_att, m.w_act, m.w_vel, m.w_mavg = (float(w[k]) for k in ("w_att", "w_act", "w_vel",
+                                                                   "w_mavg"))
+    for k in ("goal_pos_range", "goal_att_range", "init_pos_range", "init_att_range",
+              "dr_gravity_range"):
+        setattr(m, k, float(w[k]))
+    m.hidden = int(w["hidden"])
+    m.policy_out = int(w["policy_out"])
+    m.mlp_bf16 = 1 if w["mlp"] == "bf16" else 0
+    m.has_value = int(w["has_value"])
+    m.logstd_fixed[:] = [float(x) for x in w["logstd_fixed"][:6]]
+    m.logstd_min = float(w["logstd_min"])
+    m.logstd_max = float(w["logstd_max"])
+    return m
+
+
+class PaperBatch(Batch):
+    """SoA batch of the paper model: state[61][n] (p q nu, action history
+    [8][6]), params[8][n] (p_d q_d g_eff), t_ep, episode."""
+
+    def __init__(self, env_ids):
+        self.env_ids = np.ascontiguousarray(env_ids, dtype=np.uint32)
+        n = len(self.env_ids)
+        self.n = n
+        self.state = np.zeros((PAPER_STATE, n), dtype=np.float64)
+        self.params = np.zeros((PAPER_PARAM, n), dtype=np.float64)
+        self.t_ep = np.zeros(n, dtype=np.int32)
+        self.episode = np.zeros(n, dtype=np.uint32)
+
+    def copy(self):
+        b = PaperBatch(self.env_ids)
+        b.state[:] = self.state
+        b.params[:] = self.params
+        b.t_ep[:] = self.t_ep
+        b.episode[:] = self.episode
+        return b
+
+
+def paper_reset(m: PaperModel, batch: PaperBatch) -> PaperBatch:
+    _paper_lib().oracle_paper_reset(C.byref(m), batch.n, _p(batch.env_ids), _p(batch.state),
+                                    _p(batch.params), _p(batch.t_ep), _p(batch.episode))
+    return batch
+
+
+def paper_replay(m: PaperModel, batch: PaperBatch, actions: np.ndarray, precision="f64",
+                 trace=False):
+    """actions[T][6][n]; returns (rew[T][n], done[T][n], trace[T][61][n] or None)."""
+    T, n = actions.shape[0], batch.n
+    assert actions.shape == (T, PAPER_ACT, n)
+    act = np.ascontiguousarray(actions, dtype=np.float32)
+    rew = np.zeros((T, n))
+    done = np.zeros((T, n), dtype=np.uint8)
+    tr = np.zeros((T, PAPER_STATE, n)) if trace else None
+    _paper_lib().oracle_paper_replay(C.byref(m), 1 if precision == "f32" else 0, n,
+                                     _p(batch.env_ids), _p(batch.state), _p(batch.params),
+                                     _p(batch.t_ep), _p(batch.episode), T, _p(act), _p(rew),
+                                     _p(done), _p(tr))
+    return rew, done, tr
+
+
+def paper_rollout(m: PaperModel, batch: PaperBatch, pol_w, val_w, t_g0: int, T: int,
+                  precision="f64", want=("obs", "act", "logp", "value", "rew", "done")):
+    """obs[T][12][n], act[T][6][n], logp, value, rew, done (those in `want`)."""
+    n = batch.n
+    out = {}
+    shapes = dict(obs=(T, PAPER_OBS, n), act=(T, PAPER_ACT, n), logp=(T, n), value=(T, n),
+                  rew=(T, n))
+    for k, s in shapes.items():
+        out[k] = np.zeros(s) if k in want else None
+    if "value" in want and not m.has_value:
+        out["value"] = None
+    out["done"] = np.zeros((T, n), dtype=np.uint8)
+    pw = np.ascontiguousarray(pol_w, dtype=np.float32)
+    vw = None if val_w is None else np.ascontiguousarray(val_w, dtype=np.float32)
+    _paper_lib().oracle_paper_rollout(C.byref(m), 1 if precision == "f32" else 0, _p(pw),
+                                      _p(vw), n, _p(batch.env_ids), _p(batch.state),
+                                      _p(batch.params), _p(batch.t_ep), _p(batch.episode),
+                                      int(t_g0), T, _p(out["obs"]), _p(out["act"]),
+                                      _p(out["logp"]), _p(out["value"]), _p(out["rew"]),
+                                      _p(out["done"]))
+    return {k: v for k, v in out.items() if v is not None}
+
+
+def paper_single_env(state: dict, params: dict):
+    """61- and 8-row single-env vectors from field dicts (missing = 0,
+    quaternions default identity).  State keys p, q, nu, hist ([8][6]);
+    param keys p_d, q_d, g_eff."""
+    st = np.zeros(PAPER_STATE)
+    pr = np.zeros(PAPER_PARAM)
+    st[3] = 1.0
+    pr[3] = 1.0
+    for k, v in state.items():
+        if k == "hist":
+            st[13:13 + 6 * PAPER_HIST] = np.asarray(v, dtype=np.float64).reshape(-1)
+            continue
+        idx = dict(p=0, q=3, nu=7)[k]
+        st[idx:idx + len(v)] = v
+    for k, v in params.items():
+        idx = dict(p_d=0, q_d=3, g_eff=7)[k]
+        v = np.atleast_1d(v)
+        pr[idx:idx + len(v)] = v
+    return st, pr
+
+
+def _d(a):
+    return _p(np.ascontiguousarray(a, dtype=np.float64))
+
+
+def paper_observe(st, pr):
+    obs = np.zeros(PAPER_OBS)
+    _paper_lib().oracle_paper_observe(_d(st), _d(pr), _p(obs))
+    return obs
+
+
+def paper_reward(m, st, pr, a_c):
+    return _paper_lib().oracle_paper_reward(C.byref(m), _d(st), _d(pr), _d(a_c))
+
+
+def paper_wrench(m, a):
+    a_c, tau = np.zeros(PAPER_ACT), np.zeros(6)
+    _paper_lib().oracle_paper_wrench(C.byref(m), _d(a), _p(a_c), _p(tau))
+    return a_c, tau
+
+
+def paper_box(m):
+    b = np.zeros(3)
+    _paper_lib().oracle_paper_box(C.byref(m), _p(b))
+    return b
+
+
+def paper_nu_dot(m, st, pr, tau):
+    out = np.zeros(6)
+    _paper_lib().oracle_paper_nu_dot(C.byref(m), _d(st), _d(pr), _d(tau), _p(out))
+    return out
+
+
+def paper_integrate(m, st, pr, tau, h, n_steps, method="euler"):
+    s = np.ascontiguousarray(st, dtype=np.float64).copy()
+    _paper_lib().oracle_paper_integrate(C.byref(m), 0 if method == "euler" else 1, _p(s),
+                                        _d(pr), _d(tau), float(h), int(n_steps))
+    return s

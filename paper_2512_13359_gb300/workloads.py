@@ -13,6 +13,14 @@ references and initial states per episode (§V-A1) and per-env randomised
 parameters (§IV-C).  It publishes no vehicle constants; the presets below fix
 them (BlueROV2-Heavy-sized rigid body with diagonal added mass and linear plus
 quadratic damping, 8 thrusters) and the sizes of the five workloads.
+
+Two environment models exist (preset key "model"): "fossen", the
+thruster-level Fossen model with added mass, currents and domain-randomised
+parameters (18-float observation, 8 thruster commands), and "paper", the
+paper's own environment (§IV-B): a 6-D body-wrench action scaled by F_max and
+tau_max (Eq. 1), a free rigid body under the inertia-box fluid model with an
+effective gravity randomised per episode (§IV-C), a 12-float axis-angle
+observation and the five-term reward of Eqs. (2)-(7).
 """
 from __future__ import annotations
 
@@ -25,6 +33,14 @@ OBS_DIM = 18
 ACT_DIM = 8
 STATE_FIELDS = 19   # p(3) q(4) nu(6) nu_prev(6)
 PARAM_FIELDS = 17   # p_d(3) q_d(4) s_m s_a s_d dB r_b(3) V_c(3)
+
+# The paper model: 12-float observation, 6-D wrench action; state p q nu and
+# an 8-slot history of clipped actions; parameters p_d q_d g_eff.
+PAPER_OBS_DIM = 12
+PAPER_ACT_DIM = 6
+PAPER_HIST = 8
+PAPER_STATE_FIELDS = 13 + 6 * PAPER_HIST
+PAPER_PARAM_FIELDS = 8
 
 # Names of the SoA rows, for readable tests and snapshots.
 STATE_NAMES = (["p_x", "p_y", "p_z", "q_w", "q_x", "q_y", "q_z"]
@@ -79,6 +95,18 @@ _BASE = dict(
     trajectory="reward_done",
 )
 
+# Paper-model constants (§IV-B names the quantities, not their values): the
+# same rigid body without added mass; water; a neutrally buoyant nominal
+# vehicle whose effective gravity is randomised by +-0.2 m/s^2; goals within
+# +-2 m and +-60 degrees as in §V-A1; 512-step episodes.
+PAPER_MODEL = dict(
+    model="paper", f_max=40.0, tau_max=10.0, fluid_density=1000.0, fluid_viscosity=0.001,
+    g_eff=0.0, dr_gravity_range=0.2, w_axes=(1.0, 1.0, 1.0), w_pos=1.0, w_att=0.5,
+    w_act=0.01, w_vel=0.05, w_mavg=0.1, mavg_len=4, goal_pos_range=2.0,
+    goal_att_range=math.pi / 3, init_pos_range=0.0, init_att_range=0.0, episode_len=512,
+    policy_out=6, logstd_fixed=(0.0,) * 6,
+)
+
 # The five workloads.  "tiny" is the case the oracle finishes in seconds.
 WORKLOADS = {
     "tiny_64": dict(_BASE),
@@ -90,17 +118,46 @@ WORKLOADS = {
                       has_value=1, trajectory="full"),
 }
 WORKLOADS["sweep"] = dict(WORKLOADS["ppo_65536"], steps=256)
+# The paper's own environment: a small oracle-sized case and the paper's
+# largest setting (4,096 envs, one 512-step episode), with the 65,536-env
+# workload's network shapes (mean and log-std head, value network, bf16).
+WORKLOADS["paper_tiny"] = dict(_BASE, **PAPER_MODEL)
+WORKLOADS["paper_4096"] = dict(_BASE, **PAPER_MODEL, n_envs=4096, steps=512, substeps=4,
+                               hidden=256, dr_enable=1, mlp="bf16", has_value=1,
+                               trajectory="full")
+WORKLOADS["paper_4096"]["policy_out"] = 12
 SWEEP_SIZES = (1024, 4096, 16384, 65536, 262144, 1048576)
 
 
 def workload(name: str, **overrides) -> dict:
     """A deep copy of a preset with overrides, vehicle constants merged in."""
-    w = copy.deepcopy(WORKLOADS[name])
+    w = dict(model="fossen")
+    w.update(copy.deepcopy(WORKLOADS[name]))
     w.update(copy.deepcopy(VEHICLE))
     w["alloc"] = allocation_matrix()
     w["name"] = name
     w.update(overrides)
     return w
+
+
+def is_paper(w: dict) -> bool:
+    return w.get("model", "fossen") == "paper"
+
+
+def obs_dim(w: dict) -> int:
+    return PAPER_OBS_DIM if is_paper(w) else OBS_DIM
+
+
+def act_dim(w: dict) -> int:
+    return PAPER_ACT_DIM if is_paper(w) else ACT_DIM
+
+
+def state_fields(w: dict) -> int:
+    return PAPER_STATE_FIELDS if is_paper(w) else STATE_FIELDS
+
+
+def param_fields(w: dict) -> int:
+    return PAPER_PARAM_FIELDS if is_paper(w) else PARAM_FIELDS
 
 
 def mlp_shapes(in_dim: int, hidden: int, out_dim: int):
@@ -130,26 +187,31 @@ def mlp_weights(seed: int, in_dim: int, hidden: int, out_dim: int, stream: int =
 
 
 def policy_weights(w: dict, bias_std: float = 0.0) -> np.ndarray:
-    return mlp_weights(w["weight_seed"], OBS_DIM, w["hidden"], w["policy_out"], 0, bias_std)
+    return mlp_weights(w["weight_seed"], obs_dim(w), w["hidden"], w["policy_out"], 0, bias_std)
 
 
 def value_weights(w: dict, bias_std: float = 0.0) -> np.ndarray:
-    return mlp_weights(w["weight_seed"], OBS_DIM, w["hidden"], 1, 1, bias_std)
+    return mlp_weights(w["weight_seed"], obs_dim(w), w["hidden"], 1, 1, bias_std)
 
 
-def replay_actions(seed: int, T: int, n: int, scale: float = 0.7) -> np.ndarray:
-    """Normalised thruster commands [T][8][n] (float32) for action-replay runs:
+def replay_actions(seed: int, T: int, n: int, scale: float = 0.7,
+                   act: int = ACT_DIM) -> np.ndarray:
+    """Normalised commands [T][act][n] (float32) for action-replay runs:
     N(0, scale^2), so a share of them saturate at the +-1 clip."""
     rng = np.random.Generator(np.random.Philox(key=[seed, 7]))
-    return (rng.standard_normal((T, ACT_DIM, n)) * scale).astype(np.float32)
+    return (rng.standard_normal((T, act, n)) * scale).astype(np.float32)
 
 
-def random_observations(seed: int, n: int) -> np.ndarray:
-    """Observation-shaped inputs [n][18] for network-only checks: position
-    errors ~ +-2 m, rotation-matrix entries in [-1, 1], velocities ~ +-1."""
+def random_observations(seed: int, n: int, dim: int = OBS_DIM) -> np.ndarray:
+    """Observation-shaped inputs [n][dim] for network-only checks: position
+    errors ~ +-2 m, then attitude entries in [-1, 1] (rotation matrix, 18
+    floats) or +-pi/2 (axis-angle, 12 floats), velocities ~ +-1."""
     rng = np.random.Generator(np.random.Philox(key=[seed, 11]))
-    x = np.empty((n, OBS_DIM), dtype=np.float64)
+    x = np.empty((n, dim), dtype=np.float64)
     x[:, 0:3] = rng.uniform(-2, 2, (n, 3))
-    x[:, 3:12] = rng.uniform(-1, 1, (n, 9))
-    x[:, 12:18] = rng.uniform(-1, 1, (n, 6))
+    if dim == OBS_DIM:
+        x[:, 3:12] = rng.uniform(-1, 1, (n, 9))
+    else:
+        x[:, 3:6] = rng.uniform(-1.5, 1.5, (n, 3))
+    x[:, dim - 6:dim] = rng.uniform(-1, 1, (n, 6))
     return x.astype(np.float32)
