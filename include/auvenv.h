@@ -10,6 +10,20 @@
  * the done flag and the automatic reset (paper §IV-A: batched simulation of
  * independent environments sharing one model and integrator).
  *
+ * Two environment models (auv_config.model):
+ *  - AUV_MODEL_FOSSEN: the thruster-level model -- Fossen's 6-DOF equations
+ *    with added mass, Coriolis, linear + quadratic damping, restoring forces,
+ *    a water current and per-env randomised parameters; 8 thruster commands
+ *    through an allocation matrix; 18-float observation.
+ *  - AUV_MODEL_PAPER: the paper's own environment (§IV-B): a normalised body
+ *    wrench scaled by F_max and tau_max (Eq. 1); a free rigid body under the
+ *    inertia-box fluid model (quadratic drag and viscous resistance of the
+ *    uniform box with the body's mass and inertia); buoyancy folded into an
+ *    effective gravity randomised per episode (§IV-C); a 12-float
+ *    observation with the axis-angle attitude error (§IV-B1); the five-term
+ *    reward of Eqs. (2)-(7).
+ * The sizes that differ between the models are given by env_layout().
+ *
  * Conventions shared by every entry point
  *  - Return value: AUV_OK (0) or a negative AUV_ERR_* code; env_last_error()
  *    gives a one-line reason.  No entry point aborts or traps.
@@ -38,7 +52,7 @@
 extern "C" {
 #endif
 
-#define AUV_ABI_VERSION 1
+#define AUV_ABI_VERSION 2
 
 /* status codes */
 #define AUV_OK 0
@@ -53,11 +67,22 @@ extern "C" {
 #define AUV_MLP_FP32 0   /* fp32 operands and accumulation on CUDA cores        */
 #define AUV_MLP_BF16 1   /* bf16 weights/activations, fp32 accumulation, tcgen05 */
 
-/* sizes fixed by the model */
+/* environment models */
+#define AUV_MODEL_FOSSEN 0
+#define AUV_MODEL_PAPER 1
+
+/* sizes fixed by the Fossen model */
 #define AUV_OBS_DIM 18      /* observation: dp_b(3), R_e column-major(9), v(3), w(3) */
 #define AUV_ACT_DIM 8       /* normalised thruster commands                        */
 #define AUV_STATE_FIELDS 19 /* p(3) q(4: w,x,y,z body->world) nu(6) nu_prev(6)     */
 #define AUV_PARAM_FIELDS 17 /* p_d(3) q_d(4) s_m s_a s_d dB r_b(3) V_c(3)          */
+
+/* sizes fixed by the paper model */
+#define AUV_PAPER_OBS_DIM 12      /* dp_b(3), axis-angle error(3), v(3), w(3)        */
+#define AUV_PAPER_ACT_DIM 6       /* normalised wrench F(3), tau(3)                  */
+#define AUV_PAPER_HIST 8          /* action-history slots kept (mavg_len <= 8)       */
+#define AUV_PAPER_STATE_FIELDS 61 /* p(3) q(4) nu(6) history[8][6] of clipped actions */
+#define AUV_PAPER_PARAM_FIELDS 8  /* p_d(3) q_d(4) g_eff                             */
 
 /*
  * Model and workload description.  Paper §IV-B (environment), §IV-C (domain
@@ -106,9 +131,34 @@ typedef struct auv_config {
   uint32_t has_value;     /* 1: value network present                        */
   float logstd_fixed[8];  /* log-std used when policy_out == 8               */
   float logstd_min, logstd_max;     /* clamp of the log-std head             */
+  /* ---- model selection and the paper model (AUV_MODEL_PAPER) ----------- *
+   * The paper model uses n_envs, substeps, episode_len, seed, env_id_base,  *
+   * dr_enable, dt, mass, inertia, w_pos, w_att, w_act, init_pos_range,      *
+   * init_att_range, goal_pos_range, the network fields (policy_out 6: mean  *
+   * with logstd_fixed[0..5], or 12: mean + log-std head) and the fields     *
+   * below; it ignores the Fossen-only fields.                               */
+  uint32_t model;         /* AUV_MODEL_FOSSEN or AUV_MODEL_PAPER             */
+  float f_max, tau_max;   /* Eq. (1): force [N] and torque [N m] at |a| = 1  */
+  float fluid_density;    /* rho [kg/m^3] of the inertia-box fluid model     */
+  float fluid_viscosity;  /* mu [Pa s]                                       */
+  float g_eff;            /* nominal effective gravity along world -z [m/s^2] */
+  float dr_gravity_range; /* g_eff + U[-r, r] at every reset if dr_enable    */
+  float goal_att_range;   /* goal roll, pitch, yaw U[-r, r] [rad], r <= pi   */
+  float w_axes[3];        /* D = diag(w_x, w_y, w_z) of Eq. (3)              */
+  float w_vel, w_mavg;    /* Eq. (6) and Eq. (7) weights                     */
+  uint32_t mavg_len;      /* K: previous actions averaged in Eq. (7), 1..8   */
 } auv_config;
 
-/* Caller-owned device buffers holding the batch (SoA, see layout above). */
+/* Sizes of one model's arrays (see env_layout). */
+typedef struct auv_layout {
+  uint32_t obs_dim;       /* rows of an observation                          */
+  uint32_t act_dim;       /* rows of an action                               */
+  uint32_t state_fields;  /* rows of auv_buffers.state                       */
+  uint32_t param_fields;  /* rows of auv_buffers.params                      */
+} auv_layout;
+
+/* Caller-owned device buffers holding the batch (SoA, see layout above);
+ * row counts for the paper model from env_layout. */
 typedef struct auv_buffers {
   float* state;       /* [19][N] p, q, nu, nu_prev                       */
   float* params;      /* [17][N] p_d, q_d, s_m, s_a, s_d, dB, r_b, V_c    */
@@ -117,6 +167,8 @@ typedef struct auv_buffers {
 } auv_buffers;
 
 /* Trajectory outputs of env_rollout; any pointer may be NULL (not written).
+ * The row counts 18 and 8 below are the Fossen model's obs_dim and act_dim;
+ * the paper model writes obs[T][12][N] and act[T][6][N].
  * Device memory or mapped page-locked host memory, 4-byte aligned (done:
  * any alignment).  Host arrays are filled through device staging buffers
  * (see env_rollout).                                                      */
@@ -141,6 +193,10 @@ typedef struct auv_env auv_env;
 
 /* ABI version of the loaded library (AUV_ABI_VERSION it was built with). */
 int env_abi_version(void);
+
+/* env_layout: array sizes of environment model `model` (AUV_MODEL_*);
+ * AUV_ERR_INVALID for an unknown model. */
+int env_layout(uint32_t model, auv_layout* out);
 
 /*
  * env_create: validate `cfg`, bind the caller's buffers and allocate the
@@ -177,6 +233,9 @@ int env_set_weights(auv_env* env, const float* policy, const float* value, void*
  * initial position, roll/pitch/yaw, goal position, goal yaw, current, s_m,
  * s_a, s_d, dB, r_b (paper §IV-C, §V-A1); zero velocities; t_ep = 0;
  * episode += 1.  Bit-exact across implementations of the same steps.
+ * Paper model: 13 uniforms (counter blocks 0..3): goal position, goal roll,
+ * pitch, yaw, effective-gravity offset, initial position, initial roll,
+ * pitch, yaw; velocities and the action history zero.
  */
 int env_reset(auv_env* env, const uint8_t* mask, void* stream);
 
@@ -192,6 +251,13 @@ int env_reset(auv_env* env, const uint8_t* mask, void* stream);
  * theta_e - w_act |clip(a)|^2 - w_vs |nu - nu_prev|^2 (weighted norms of
  * Eqs. 2-7); t_ep += 1; done = (t_ep == episode_len); on done the env resets
  * as in env_reset.  The global step t_g advances by T.
+ * Paper model: o_t is [dp_b, axis-angle error of conj(q_d) (x) q, v, w]; a
+ * takes the first 6 of the 8 normals; a_c = clip(a, -1, 1); tau = [F_max
+ * a_c(0:3); tau_max a_c(3:6)] (Eq. 1); the substeps integrate M_RB nu' = tau +
+ * fluid wrench - C_RB(nu) nu + R^T (0, 0, -m g_eff); r = -w_pos |D dp_b|^2 -
+ * w_att |theta_e|^2 - w_act |a_c(3:6)|^2 - w_vel |w|^2 - w_mavg |a_c - mean
+ * of the previous mavg_len a_c|^2 (Eqs. 2-7, history zero after a reset),
+ * then a_c enters history slot (t_ep mod mavg_len).
  * In AUV_MLP_BF16 mode traj.value (if given) comes from a value-network pass
  * over traj.obs after the steps, so traj.obs is required with it.
  * Host arrays (T >= 2): the steps run in segments into two device staging
@@ -210,29 +276,30 @@ int env_step(auv_env* env, float* obs_out, float* rew_out, uint8_t* done_out, vo
 
 /*
  * env_step_actions: action replay.  T control steps with the given
- * normalised actions act[T][8][N] (device) instead of the policy: allocation,
- * substeps, reward, done and auto-reset exactly as in env_rollout.  Writes
- * rew[T][N], done[T][N] and, if non-NULL, state_trace[T][19][N] (state after
- * each step, after any reset).  Does not advance t_g.
+ * normalised actions act[T][act_dim][N] (device) instead of the policy:
+ * allocation (paper model: the Eq. (1) wrench), substeps, reward, done and
+ * auto-reset exactly as in env_rollout.  Writes rew[T][N], done[T][N] and,
+ * if non-NULL, state_trace[T][state_fields][N] (state after each step, after
+ * any reset).  Does not advance t_g.
  */
 int env_step_actions(auv_env* env, const float* act, int T, float* rew_out, uint8_t* done_out,
                      float* state_trace, void* stream);
 
 /*
  * env_value: the value network on stored observations, in the trajectory
- * layout: obs[T][18][N] -> value[T][N] (device or mapped host memory),
+ * layout: obs[T][obs_dim][N] -> value[T][N] (device or mapped host memory),
  * T >= 1, with the loaded value weights (needs has_value).  A PPO learner
  * re-evaluates values this way; env_rollout calls it itself when given
  * traj.value.
  */
 int env_value(auv_env* env, const float* obs, int T, float* value, void* stream);
 
-/* env_observe: observation of the current state, obs[18][N] (device). */
+/* env_observe: observation of the current state, obs[obs_dim][N] (device). */
 int env_observe(auv_env* env, float* obs_out, void* stream);
 
 /*
  * env_policy_forward: evaluate the loaded networks on caller observations
- * obs[n][18] (row-major, device) for n >= 1 rows: head[n][policy_out] (raw
+ * obs[n][obs_dim] (row-major, device) for n >= 1 rows: head[n][policy_out] (raw
  * outputs: mean, then unclamped log-std) and, if value is non-NULL and
  * has_value, value[n].  Same device arithmetic as env_rollout.
  */

@@ -25,12 +25,14 @@ AUV_ERR_NAN = -5
 AUV_ERR_UNSUPPORTED = -6
 AUV_MLP_FP32 = 0
 AUV_MLP_BF16 = 1
+AUV_MODEL_FOSSEN = 0
+AUV_MODEL_PAPER = 1
 
 EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
-            "env_policy_forward_noalloc")
+            "env_policy_forward_noalloc", "env_layout")
 
 
 class LibraryMissing(RuntimeError):
@@ -59,7 +61,17 @@ class AuvConfig(C.Structure):
         ("hidden", C.c_uint32), ("policy_out", C.c_uint32), ("mlp_mode", C.c_uint32),
         ("has_value", C.c_uint32), ("logstd_fixed", C.c_float * 8),
         ("logstd_min", C.c_float), ("logstd_max", C.c_float),
+        ("model", C.c_uint32), ("f_max", C.c_float), ("tau_max", C.c_float),
+        ("fluid_density", C.c_float), ("fluid_viscosity", C.c_float), ("g_eff", C.c_float),
+        ("dr_gravity_range", C.c_float), ("goal_att_range", C.c_float),
+        ("w_axes", C.c_float * 3), ("w_vel", C.c_float), ("w_mavg", C.c_float),
+        ("mavg_len", C.c_uint32),
     ]
+
+
+class AuvLayout(C.Structure):
+    _fields_ = [("obs_dim", C.c_uint32), ("act_dim", C.c_uint32), ("state_fields", C.c_uint32),
+                ("param_fields", C.c_uint32)]
 
 
 class AuvBuffers(C.Structure):
@@ -113,6 +125,7 @@ def lib(path: str | None = None):
     L.env_clear_status.argtypes = [P, P]
     L.env_selftest_wait_timeout.argtypes = [P, C.c_uint32, P]
     L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
+    L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
@@ -146,8 +159,23 @@ def make_config(w: dict) -> AuvConfig:
     c.policy_out = int(w["policy_out"])
     c.mlp_mode = AUV_MLP_BF16 if w["mlp"] == "bf16" else AUV_MLP_FP32
     c.has_value = int(w["has_value"])
-    c.logstd_fixed[:] = [float(x) for x in w["logstd_fixed"]]
+    ls = [float(x) for x in w["logstd_fixed"]]
+    c.logstd_fixed[:] = ls + [0.0] * (8 - len(ls))
+    c.model = AUV_MODEL_PAPER if W.is_paper(w) else AUV_MODEL_FOSSEN
+    for k in ("f_max", "tau_max", "fluid_density", "fluid_viscosity", "g_eff",
+              "dr_gravity_range", "goal_att_range", "w_vel", "w_mavg"):
+        setattr(c, k, float(w.get(k, 0.0)))
+    c.w_axes[:] = [float(x) for x in w.get("w_axes", (1.0, 1.0, 1.0))]
+    c.mavg_len = int(w.get("mavg_len", 1))
     return c
+
+
+def layout(model: int) -> AuvLayout:
+    out = AuvLayout()
+    rc = lib().env_layout(int(model), C.byref(out))
+    if rc != AUV_OK:
+        raise AuvError(rc, lib().env_last_error(None).decode())
+    return out
 
 
 def _ptr(t):
@@ -163,8 +191,9 @@ def _stream(stream):
 class Env:
     """A batch of N environments on the current CUDA device.
 
-    State lives in caller-owned torch tensors (SoA): state[19][N],
-    params[17][N], t_ep[N] (int32), episode[N] (int32 storage of uint32)."""
+    State lives in caller-owned torch tensors (SoA): state[S][N], params[P][N]
+    (S, P = 19, 17 for the Fossen model, 61, 8 for the paper model), t_ep[N]
+    (int32), episode[N] (int32 storage of uint32)."""
 
     def __init__(self, workload: dict, device=None):
         import torch
@@ -174,8 +203,10 @@ class Env:
         L = lib()
         n = self.n
         with torch.cuda.device(self.device):
-            self.state = torch.zeros((W.STATE_FIELDS, n), dtype=torch.float32, device=self.device)
-            self.params = torch.zeros((W.PARAM_FIELDS, n), dtype=torch.float32, device=self.device)
+            self.state = torch.zeros((W.state_fields(workload), n), dtype=torch.float32,
+                                     device=self.device)
+            self.params = torch.zeros((W.param_fields(workload), n), dtype=torch.float32,
+                                      device=self.device)
             self.t_ep = torch.zeros(n, dtype=torch.int32, device=self.device)
             self.episode = torch.zeros(n, dtype=torch.int32, device=self.device)
             self.cfg = make_config(workload)
@@ -230,7 +261,7 @@ class Env:
         self._check(lib().env_rollout(self.h, int(T), C.byref(t), _stream(stream)))
 
     def value(self, obs, value, stream=None):
-        """Value network on trajectory-layout observations obs[T][18][N] -> value[T][N]."""
+        """Value network on trajectory-layout observations obs[T][obs_dim][N] -> value[T][N]."""
         self._check(lib().env_value(self.h, _ptr(obs), int(obs.shape[0]), _ptr(value),
                                     _stream(stream)))
 
@@ -279,8 +310,8 @@ class Env:
                    pinned_host: bool = False) -> dict:
         import torch
         n = self.n
-        shapes = dict(obs=(T, W.OBS_DIM, n), act=(T, W.ACT_DIM, n), logp=(T, n), value=(T, n),
-                      rew=(T, n), done=(T, n))
+        shapes = dict(obs=(T, W.obs_dim(self.w), n), act=(T, W.act_dim(self.w), n), logp=(T, n),
+                      value=(T, n), rew=(T, n), done=(T, n))
         out = {}
         for k in keys:
             if k == "value" and not self.w["has_value"]:

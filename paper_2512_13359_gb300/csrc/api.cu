@@ -60,7 +60,13 @@ int cuda_fail(auv_env* env, cudaError_t e, const char* what) {
   return fail(env, AUV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-size_t mlp_count(size_t H, size_t out) { return H * 18 + H + H * H + H + out * H + out; }
+size_t mlp_count(size_t in, size_t H, size_t out) {
+  return H * in + H + H * H + H + out * H + out;
+}
+
+bool is_paper(const auv_config* c) { return c->model == AUV_MODEL_PAPER; }
+size_t obs_dim(const auv_config* c) { return is_paper(c) ? AUV_PAPER_OBS_DIM : AUV_OBS_DIM; }
+size_t act_dim(const auv_config* c) { return is_paper(c) ? AUV_PAPER_ACT_DIM : AUV_ACT_DIM; }
 
 bool finite_pos(float x) { return std::isfinite(x) && x > 0.0f; }
 bool finite_nonneg(float x) { return std::isfinite(x) && x >= 0.0f; }
@@ -106,6 +112,58 @@ int map_output(auv_env* env, void* p, const char* name, size_t align, void** dev
   return AUV_OK;
 }
 
+// Shared network and episode checks (both models).
+int validate_networks(const auv_config* c, uint32_t out_mean) {
+  if (c->policy_out != out_mean && c->policy_out != 2 * out_mean)
+    return fail(nullptr, AUV_ERR_INVALID, "policy_out must be %u or %u", out_mean, 2 * out_mean);
+  if (c->mlp_mode != AUV_MLP_FP32 && c->mlp_mode != AUV_MLP_BF16)
+    return fail(nullptr, AUV_ERR_INVALID, "unknown mlp_mode %u", c->mlp_mode);
+  if (c->has_value > 1) return fail(nullptr, AUV_ERR_INVALID, "has_value must be 0 or 1");
+  if (!(c->logstd_min <= c->logstd_max) || !std::isfinite(c->logstd_min) ||
+      !std::isfinite(c->logstd_max))
+    return fail(nullptr, AUV_ERR_INVALID, "logstd clamp invalid");
+  for (int k = 0; k < 8; ++k)
+    if (!std::isfinite(c->logstd_fixed[k]))
+      return fail(nullptr, AUV_ERR_INVALID, "logstd_fixed not finite");
+  if (c->mlp_mode == AUV_MLP_FP32 && c->hidden != 64 && c->hidden != 256)
+    return fail(nullptr, AUV_ERR_UNSUPPORTED, "fp32 networks are built for hidden 64 or 256");
+  if (c->mlp_mode == AUV_MLP_BF16 && (c->hidden != 256 || c->policy_out != 2 * out_mean))
+    return fail(nullptr, AUV_ERR_UNSUPPORTED,
+                "bf16 networks are built for hidden 256 with the mean + log-std head");
+  return AUV_OK;
+}
+
+// The paper model's own fields (the Fossen-only fields are ignored).
+int validate_paper(const auv_config* c) {
+  const float pi = 3.14159274f;
+  if (!finite_nonneg(c->f_max) || !finite_nonneg(c->tau_max))
+    return fail(nullptr, AUV_ERR_INVALID, "f_max and tau_max must be finite and >= 0");
+  if (!finite_nonneg(c->fluid_density) || !finite_nonneg(c->fluid_viscosity))
+    return fail(nullptr, AUV_ERR_INVALID, "fluid density and viscosity must be finite and >= 0");
+  const double I0 = c->inertia[0], I1 = c->inertia[1], I2 = c->inertia[2];
+  if (!(I1 + I2 > I0 && I0 + I2 > I1 && I0 + I1 > I2))
+    return fail(nullptr, AUV_ERR_INVALID,
+                "inertia violates the triangle inequality (no equivalent inertia box)");
+  if (!std::isfinite(c->g_eff) || !finite_nonneg(c->dr_gravity_range))
+    return fail(nullptr, AUV_ERR_INVALID, "effective gravity and its range must be finite");
+  if (!finite_nonneg(c->init_pos_range) || !finite_nonneg(c->goal_pos_range) ||
+      !finite_nonneg(c->init_att_range) || !finite_nonneg(c->goal_att_range) ||
+      c->init_att_range > pi || c->goal_att_range > pi)
+    return fail(nullptr, AUV_ERR_INVALID,
+                "ranges must be finite and >= 0; attitude ranges <= pi");
+  if (c->dr_enable > 1) return fail(nullptr, AUV_ERR_INVALID, "dr_enable must be 0 or 1");
+  if (!std::isfinite(c->w_pos) || !std::isfinite(c->w_att) || !std::isfinite(c->w_act) ||
+      !std::isfinite(c->w_vel) || !std::isfinite(c->w_mavg) || !std::isfinite(c->w_axes[0]) ||
+      !std::isfinite(c->w_axes[1]) || !std::isfinite(c->w_axes[2]))
+    return fail(nullptr, AUV_ERR_INVALID, "reward weights not finite");
+  if (c->mavg_len < 1 || c->mavg_len > AUV_PAPER_HIST)
+    return fail(nullptr, AUV_ERR_INVALID, "mavg_len %u outside [1, %d]", c->mavg_len,
+                AUV_PAPER_HIST);
+  if (c->mlp_mode == AUV_MLP_BF16)
+    return fail(nullptr, AUV_ERR_UNSUPPORTED, "the paper model runs fp32 networks only");
+  return validate_networks(c, AUV_PAPER_ACT_DIM);
+}
+
 int validate_config(const auv_config* c) {
   if (!c) return fail(nullptr, AUV_ERR_INVALID, "cfg is NULL");
   if (c->struct_size != sizeof(auv_config))
@@ -123,6 +181,9 @@ int validate_config(const auv_config* c) {
   if (!finite_pos(c->mass)) return fail(nullptr, AUV_ERR_INVALID, "mass must be > 0");
   for (int k = 0; k < 3; ++k)
     if (!finite_pos(c->inertia[k])) return fail(nullptr, AUV_ERR_INVALID, "inertia must be > 0");
+  if (c->model != AUV_MODEL_FOSSEN && c->model != AUV_MODEL_PAPER)
+    return fail(nullptr, AUV_ERR_INVALID, "unknown model %u", c->model);
+  if (is_paper(c)) return validate_paper(c);
   for (int k = 0; k < 6; ++k) {
     if (!finite_nonneg(c->added_mass[k]) || !finite_nonneg(c->damp_lin[k]) ||
         !finite_nonneg(c->damp_quad[k]))
@@ -149,23 +210,7 @@ int validate_config(const auv_config* c) {
   if (!std::isfinite(c->w_pos) || !std::isfinite(c->w_att) || !std::isfinite(c->w_act) ||
       !std::isfinite(c->w_vs))
     return fail(nullptr, AUV_ERR_INVALID, "reward weights not finite");
-  if (c->policy_out != 8 && c->policy_out != 16)
-    return fail(nullptr, AUV_ERR_INVALID, "policy_out must be 8 or 16");
-  if (c->mlp_mode != AUV_MLP_FP32 && c->mlp_mode != AUV_MLP_BF16)
-    return fail(nullptr, AUV_ERR_INVALID, "unknown mlp_mode %u", c->mlp_mode);
-  if (c->has_value > 1) return fail(nullptr, AUV_ERR_INVALID, "has_value must be 0 or 1");
-  if (!(c->logstd_min <= c->logstd_max) || !std::isfinite(c->logstd_min) ||
-      !std::isfinite(c->logstd_max))
-    return fail(nullptr, AUV_ERR_INVALID, "logstd clamp invalid");
-  for (int k = 0; k < 8; ++k)
-    if (!std::isfinite(c->logstd_fixed[k]))
-      return fail(nullptr, AUV_ERR_INVALID, "logstd_fixed not finite");
-  if (c->mlp_mode == AUV_MLP_FP32 && c->hidden != 64 && c->hidden != 256)
-    return fail(nullptr, AUV_ERR_UNSUPPORTED, "fp32 networks are built for hidden 64 or 256");
-  if (c->mlp_mode == AUV_MLP_BF16 && (c->hidden != 256 || c->policy_out != 16))
-    return fail(nullptr, AUV_ERR_UNSUPPORTED,
-                "bf16 networks are built for hidden 256 with the 16-output policy head");
-  return AUV_OK;
+  return validate_networks(c, AUV_ACT_DIM);
 }
 
 Model build_model(const auv_config* c) {
@@ -207,6 +252,33 @@ Model build_model(const auv_config* c) {
   M.dr_buoy = c->dr_buoy_range; M.dr_cob = c->dr_cob_range;
   for (int k = 0; k < 8; ++k) M.logstd_fixed[k] = c->logstd_fixed[k];
   M.logstd_min = c->logstd_min; M.logstd_max = c->logstd_max;
+  M.model = (int)c->model;
+  if (is_paper(c)) {
+    // inertia box: the uniform box with the body's mass and principal moments
+    const double m = c->mass, I0 = c->inertia[0], I1 = c->inertia[1], I2 = c->inertia[2];
+    const double b[3] = {std::sqrt(6 * (I1 + I2 - I0) / m), std::sqrt(6 * (I0 + I2 - I1) / m),
+                         std::sqrt(6 * (I0 + I1 - I2) / m)};
+    const double rho = c->fluid_density, mu = c->fluid_viscosity, pi = 3.14159265358979323846;
+    const double d = (b[0] + b[1] + b[2]) / 3;
+    for (int k = 0; k < 3; ++k) {
+      const int j = (k + 1) % 3, l = (k + 2) % 3;
+      M.kf_drag[k] = (float)(0.5 * rho * b[j] * b[l]);
+      M.kt_drag[k] = (float)(rho / 64 * b[k] * (std::pow(b[j], 4) + std::pow(b[l], 4)));
+      M.inv_inertia[k] = (float)(1.0 / c->inertia[k]);
+      M.w_axes[k] = c->w_axes[k];
+    }
+    M.c_visc_f = (float)(3 * pi * mu * d);
+    M.c_visc_t = (float)(pi * mu * d * d * d);
+    M.inv_mass = (float)(1.0 / m);
+    M.f_max = c->f_max;
+    M.tau_max = c->tau_max;
+    M.g_eff0 = c->g_eff;
+    M.dr_grav = c->dr_gravity_range;
+    M.goal_att_range = c->goal_att_range;
+    M.w_vel = c->w_vel;
+    M.w_mavg = c->w_mavg;
+    M.mavg_len = (int)c->mavg_len;
+  }
   return M;
 }
 
@@ -226,6 +298,18 @@ extern "C" {
 
 int env_abi_version(void) { return AUV_ABI_VERSION; }
 
+int env_layout(uint32_t model, auv_layout* out) {
+  if (!out) return fail(nullptr, AUV_ERR_INVALID, "out is NULL");
+  if (model == AUV_MODEL_FOSSEN) {
+    *out = {AUV_OBS_DIM, AUV_ACT_DIM, AUV_STATE_FIELDS, AUV_PARAM_FIELDS};
+  } else if (model == AUV_MODEL_PAPER) {
+    *out = {AUV_PAPER_OBS_DIM, AUV_PAPER_ACT_DIM, AUV_PAPER_STATE_FIELDS, AUV_PAPER_PARAM_FIELDS};
+  } else {
+    return fail(nullptr, AUV_ERR_INVALID, "unknown model %u", model);
+  }
+  return AUV_OK;
+}
+
 const char* env_last_error(const auv_env* env) { return env ? env->err : g_create_err; }
 
 int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
@@ -242,6 +326,7 @@ int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
   auv_env* env = new (std::nothrow) auv_env;
   if (!env) return fail(nullptr, AUV_ERR_INVALID, "out of host memory");
   std::memset(env, 0, sizeof(*env));
+  env->last_copy = -1;
   env->cfg = *cfg;
   env->model = build_model(cfg);
   env->buf.state = buf->state;
@@ -249,8 +334,8 @@ int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
   env->buf.t_ep = buf->t_ep;
   env->buf.episode = buf->episode;
   cudaGetDevice(&env->device);
-  env->policy_count = mlp_count(cfg->hidden, cfg->policy_out);
-  env->value_count = cfg->has_value ? mlp_count(cfg->hidden, 1) : 0;
+  env->policy_count = mlp_count(obs_dim(cfg), cfg->hidden, cfg->policy_out);
+  env->value_count = cfg->has_value ? mlp_count(obs_dim(cfg), cfg->hidden, 1) : 0;
   // workspace: status (256 B) | fp32 policy | fp32 value | packed bf16 images
   size_t off = 256;
   const size_t pol_off = off;
@@ -337,7 +422,9 @@ int env_reset(auv_env* env, const uint8_t* mask, void* stream) {
   int rc = check_device(env);
   if (rc) return rc;
   if (mask && (rc = check_device_buffer(env, mask, "mask", 1))) return rc;
-  cudaError_t e = auv::launch_reset(env->model, env->buf, mask, static_cast<cudaStream_t>(stream));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = is_paper(&env->cfg) ? auv::launch_paper_reset(env->model, env->buf, mask, s)
+                                      : auv::launch_reset(env->model, env->buf, mask, s);
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "reset kernel");
 }
 
@@ -348,8 +435,11 @@ namespace {
 cudaError_t launch_rollout_any(auv_env* env, const Traj& tr, int T, uint64_t t_g0,
                                cudaStream_t s) {
   if (env->cfg.mlp_mode == AUV_MLP_FP32)
-    return auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32, env->w_value_f32, tr,
-                                    T, t_g0, env->status, s);
+    return is_paper(&env->cfg)
+               ? auv::launch_paper_rollout_fp32(env->model, env->buf, env->w_policy_f32,
+                                                env->w_value_f32, tr, T, t_g0, env->status, s)
+               : auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32,
+                                          env->w_value_f32, tr, T, t_g0, env->status, s);
   cudaError_t e = auv::launch_rollout_bf16(env->model, env->buf, env->w_policy_packed, tr, T,
                                            t_g0, env->status, s);
   if (e != cudaSuccess || !tr.value) return e;
@@ -374,7 +464,8 @@ void** traj_slot(Traj& t, int k) {
 int rollout_staged(auv_env* env, int T, const auv_traj* traj, Traj mapped,
                    const bool host[kTrajArrays], cudaStream_t s) {
   const size_t n = env->model.n;
-  const size_t row[kTrajArrays] = {18 * n * 4, 8 * n * 4, n * 4, n * 4, n * 4, n};
+  const size_t row[kTrajArrays] = {obs_dim(&env->cfg) * n * 4, act_dim(&env->cfg) * n * 4,
+                                   n * 4, n * 4, n * 4, n};
   void* const dst[kTrajArrays] = {traj->obs, traj->act, traj->logp, traj->value, traj->rew,
                                   traj->done};
   size_t step_bytes = 0;
@@ -529,7 +620,11 @@ int env_step_actions(auv_env* env, const float* act, int T, float* rew_out, uint
   if ((rc = map_output(env, rew_out, "rew_out", 4, &rew))) return rc;
   if ((rc = map_output(env, done_out, "done_out", 1, &done))) return rc;
   if ((rc = map_output(env, state_trace, "state_trace", 4, &trace))) return rc;
-  cudaError_t e = auv::launch_replay(env->model, env->buf, act, T, static_cast<float*>(rew),
+  cudaError_t e = is_paper(&env->cfg)
+      ? auv::launch_paper_replay(env->model, env->buf, act, T, static_cast<float*>(rew),
+                                 static_cast<uint8_t*>(done), static_cast<float*>(trace),
+                                 env->status, static_cast<cudaStream_t>(stream))
+      : auv::launch_replay(env->model, env->buf, act, T, static_cast<float*>(rew),
                                      static_cast<uint8_t*>(done), static_cast<float*>(trace),
                                      env->status, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "replay kernel");
@@ -542,7 +637,10 @@ int env_observe(auv_env* env, float* obs_out, void* stream) {
   void* d;
   if (!obs_out) return fail(env, AUV_ERR_INVALID, "obs_out is NULL");
   if ((rc = map_output(env, obs_out, "obs_out", 4, &d))) return rc;
-  cudaError_t e = auv::launch_observe(env->model, env->buf, static_cast<float*>(d),
+  cudaError_t e = is_paper(&env->cfg)
+      ? auv::launch_paper_observe(env->model, env->buf, static_cast<float*>(d),
+                                  static_cast<cudaStream_t>(stream))
+      : auv::launch_observe(env->model, env->buf, static_cast<float*>(d),
                                       static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "observe kernel");
 }

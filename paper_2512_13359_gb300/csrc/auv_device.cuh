@@ -41,6 +41,17 @@ struct Model {
   float dr_lo, dr_hi, dr_buoy, dr_cob;
   float logstd_fixed[8];
   float logstd_min, logstd_max;
+  // ---- the paper model (model == 1; paper_device.cuh) ----
+  int model;          // 0 = Fossen, 1 = paper
+  int mavg_len;       // K of Eq. (7)
+  float f_max, tau_max;
+  float inv_mass, inv_inertia[3];
+  float kf_drag[3];   // 1/2 rho A_i, A = (b_y b_z, b_x b_z, b_x b_y) of the inertia box
+  float kt_drag[3];   // rho / 64 b_i (b_j^4 + b_k^4)
+  float c_visc_f;     // 3 pi mu d, d = mean box side
+  float c_visc_t;     // pi mu d^3
+  float g_eff0, dr_grav, goal_att_range;
+  float w_axes[3], w_vel, w_mavg;
 };
 
 // Device status block (mirrors auv_status; first_nan_env holds INT32_MAX
@@ -149,6 +160,20 @@ __device__ __forceinline__ void refresh_mass(const Model& M, Env& e) {
   e.inv_m[5] = 1.0f / (e.sm * M.inertia[2] + e.sa * M.added[5]);
 }
 
+// Z-Y-X Euler composition q_z(yaw) q_y(pitch) q_x(roll) from half angles,
+// every operation explicitly rounded (bit-exact reset draws).
+__device__ __forceinline__ void euler_quat(float roll, float pitch, float yaw, float q[4]) {
+  const float cr = reset_cos(__fmul_rn(0.5f, roll)), sr = reset_sin(__fmul_rn(0.5f, roll));
+  const float cp = reset_cos(__fmul_rn(0.5f, pitch)), sp = reset_sin(__fmul_rn(0.5f, pitch));
+  const float cy = reset_cos(__fmul_rn(0.5f, yaw)), sy = reset_sin(__fmul_rn(0.5f, yaw));
+  const float a = __fmul_rn(cy, cp), b = __fmul_rn(sy, sp);
+  const float c = __fmul_rn(cy, sp), d = __fmul_rn(sy, cp);
+  q[0] = __fmaf_rn(a, cr, __fmul_rn(b, sr));
+  q[1] = __fmaf_rn(a, sr, -__fmul_rn(b, cr));
+  q[2] = __fmaf_rn(c, cr, __fmul_rn(d, sr));
+  q[3] = __fmaf_rn(d, cr, -__fmul_rn(c, sr));
+}
+
 // New episode for env `id` at its current episode index; then episode += 1.
 // Draw order: p0 xyz, roll, pitch, yaw, goal xyz, goal yaw, current xyz,
 // s_m, s_a, s_d, dB, r_b xyz.
@@ -184,16 +209,7 @@ __device__ __forceinline__ void reset_env(const Model& M, uint32_t id, Env& e) {
     e.sm = 1.0f; e.sa = 1.0f; e.sd = 1.0f; e.dB = 0.0f;
     e.rb[0] = 0.0f; e.rb[1] = 0.0f; e.rb[2] = 0.0f;
   }
-  // Z-Y-X Euler composition q_z(yaw) q_y(pitch) q_x(roll) from half angles.
-  const float cr = reset_cos(__fmul_rn(0.5f, roll)), sr = reset_sin(__fmul_rn(0.5f, roll));
-  const float cp = reset_cos(__fmul_rn(0.5f, pitch)), sp = reset_sin(__fmul_rn(0.5f, pitch));
-  const float cy = reset_cos(__fmul_rn(0.5f, yaw)), sy = reset_sin(__fmul_rn(0.5f, yaw));
-  const float a = __fmul_rn(cy, cp), b = __fmul_rn(sy, sp);
-  const float c = __fmul_rn(cy, sp), d = __fmul_rn(sy, cp);
-  e.q[0] = __fmaf_rn(a, cr, __fmul_rn(b, sr));
-  e.q[1] = __fmaf_rn(a, sr, -__fmul_rn(b, cr));
-  e.q[2] = __fmaf_rn(c, cr, __fmul_rn(d, sr));
-  e.q[3] = __fmaf_rn(d, cr, -__fmul_rn(c, sr));
+  euler_quat(roll, pitch, yaw, e.q);
   e.qd[0] = reset_cos(__fmul_rn(0.5f, gyaw));
   e.qd[1] = 0.0f;
   e.qd[2] = 0.0f;
@@ -332,6 +348,40 @@ __device__ __forceinline__ void allocate(const Model& M, const float a[kAct], fl
   }
 }
 
+// Pose part of a semi-implicit Euler substep, shared by both models:
+// p += h R v (R: attitude at the start of the substep, v: new velocity), then
+// q = normalize(q (x) (cos a, sin(a) w/|w|)), a = h |w| / 2.
+__device__ __forceinline__ void advance_pose(float h, const float R[3][3], const float nu[6],
+                                             float p[3], float q[4]) {
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+    p[i] = fmaf(h, R[i][0] * nu[0] + R[i][1] * nu[1] + R[i][2] * nu[2], p[i]);
+  const float hw0 = 0.5f * h * nu[3], hw1 = 0.5f * h * nu[4], hw2 = 0.5f * h * nu[5];
+  const float a2 = hw0 * hw0 + hw1 * hw1 + hw2 * hw2;
+  float ca, sa_over_a;
+  if (a2 < 0.0625f) {
+    // cos a = 1 - a^2/2 + a^4/24 - a^6/720 + a^8/40320;
+    // sin(a)/a = 1 - a^2/6 + a^4/120 - a^6/5040 + a^8/362880 (|a| < 1/4)
+    ca = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 40320.0f, -1.0f / 720.0f), a2, 1.0f / 24.0f), a2, -0.5f),
+              a2, 1.0f);
+    sa_over_a = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 362880.0f, -1.0f / 5040.0f), a2, 1.0f / 120.0f),
+                          a2, -1.0f / 6.0f), a2, 1.0f);
+  } else {
+    const float a = sqrtf(a2);
+    float s;
+    sincosf(a, &s, &ca);
+    sa_over_a = s / a;
+  }
+  const float d1 = sa_over_a * hw0, d2 = sa_over_a * hw1, d3 = sa_over_a * hw2;
+  const float qw = q[0], qx = q[1], qy = q[2], qz = q[3];
+  float nw = qw * ca - qx * d1 - qy * d2 - qz * d3;
+  float nx = qw * d1 + qx * ca + qy * d3 - qz * d2;
+  float ny = qw * d2 - qx * d3 + qy * ca + qz * d1;
+  float nz = qw * d3 + qx * d2 - qy * d1 + qz * ca;
+  const float inv = rsqrtf(nw * nw + nx * nx + ny * ny + nz * nz);
+  q[0] = nw * inv; q[1] = nx * inv; q[2] = ny * inv; q[3] = nz * inv;
+}
+
 // One semi-implicit Euler substep of
 //   (M_RB + M_A) nu' = tau - C_RB(nu) nu - C_A(nu_r) nu_r - D(nu_r) nu_r
 //                      + restoring + M_A nu_c'
@@ -404,35 +454,7 @@ __device__ __forceinline__ void substep(const Model& M, Env& e, const float tau[
     e.nu[2 * j] = nv.x;
     e.nu[2 * j + 1] = nv.y;
   }
-  // position with the new body velocity, attitude at the start of the substep
-#pragma unroll
-  for (int i = 0; i < 3; ++i)
-    e.p[i] = fmaf(M.h, R[i][0] * e.nu[0] + R[i][1] * e.nu[1] + R[i][2] * e.nu[2], e.p[i]);
-  // attitude: q (x) (cos(a), sin(a) w/|w|), a = h |w| / 2
-  const float hw0 = 0.5f * M.h * e.nu[3], hw1 = 0.5f * M.h * e.nu[4], hw2 = 0.5f * M.h * e.nu[5];
-  const float a2 = hw0 * hw0 + hw1 * hw1 + hw2 * hw2;
-  float ca, sa_over_a;
-  if (a2 < 0.0625f) {
-    // cos a = 1 - a^2/2 + a^4/24 - a^6/720 + a^8/40320;
-    // sin(a)/a = 1 - a^2/6 + a^4/120 - a^6/5040 + a^8/362880 (|a| < 1/4)
-    ca = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 40320.0f, -1.0f / 720.0f), a2, 1.0f / 24.0f), a2, -0.5f),
-              a2, 1.0f);
-    sa_over_a = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 362880.0f, -1.0f / 5040.0f), a2, 1.0f / 120.0f),
-                          a2, -1.0f / 6.0f), a2, 1.0f);
-  } else {
-    const float a = sqrtf(a2);
-    float s;
-    sincosf(a, &s, &ca);
-    sa_over_a = s / a;
-  }
-  const float d1 = sa_over_a * hw0, d2 = sa_over_a * hw1, d3 = sa_over_a * hw2;
-  const float qw = e.q[0], qx = e.q[1], qy = e.q[2], qz = e.q[3];
-  float nw = qw * ca - qx * d1 - qy * d2 - qz * d3;
-  float nx = qw * d1 + qx * ca + qy * d3 - qz * d2;
-  float ny = qw * d2 - qx * d3 + qy * ca + qz * d1;
-  float nz = qw * d3 + qx * d2 - qy * d1 + qz * ca;
-  const float inv = rsqrtf(nw * nw + nx * nx + ny * ny + nz * nz);
-  e.q[0] = nw * inv; e.q[1] = nx * inv; e.q[2] = ny * inv; e.q[3] = nz * inv;
+  advance_pose(M.h, R, e.nu, e.p, e.q);
 }
 
 // q_e = conj(q_d) (x) q: attitude of the body in the goal frame.

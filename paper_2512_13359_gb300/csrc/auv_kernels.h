@@ -37,11 +37,22 @@ cudaError_t launch_draw_words(const Model& M, uint32_t stream_id, uint64_t index
 cudaError_t launch_rollout_fp32(const Model& M, const Buffers& B, const float* wp,
                                 const float* wv, const Traj& tr, int T, uint64_t t_g0, Status* st,
                                 cudaStream_t s);
-// Value network over stored observations obs[t][18][n] (row r = t*n + i).
+// Value network over stored observations obs[t][obs_dim][n] (row r = t*n + i).
 cudaError_t launch_value_fp32(const Model& M, const float* wv, const float* obs, size_t rows,
                               int n, float* value, cudaStream_t s);
 cudaError_t launch_forward_fp32(const Model& M, const float* wp, const float* wv,
                                 const float* obs, int n, float* head, float* value,
                                 cudaStream_t s);
+
+// The paper model's CUDA-core kernels (k_paper.cu)
+cudaError_t launch_paper_reset(const Model& M, const Buffers& B, const uint8_t* mask,
+                               cudaStream_t s);
+cudaError_t launch_paper_replay(const Model& M, const Buffers& B, const float* act, int T,
+                                float* rew, uint8_t* done, float* trace, Status* st,
+                                cudaStream_t s);
+cudaError_t launch_paper_observe(const Model& M, const Buffers& B, float* obs, cudaStream_t s);
+cudaError_t launch_paper_rollout_fp32(const Model& M, const Buffers& B, const float* wp,
+                                      const float* wv, const Traj& tr, int T, uint64_t t_g0,
+                                      Status* st, cudaStream_t s);
 
 }  // namespace auv

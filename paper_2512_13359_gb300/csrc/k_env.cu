@@ -5,6 +5,7 @@
 // registers across all T control steps and touches HBM only at the start and
 // the end (plus the trajectory rows it writes).
 #include "auv_kernels.h"
+#include "mlp_fp32.cuh"
 
 namespace auv {
 
@@ -76,55 +77,6 @@ __global__ void __launch_bounds__(256) k_draw_words(const Model M, uint32_t stre
   }
 }
 
-// ---------------------------------------------------------------------------
-// fp32 networks on CUDA cores: tanh(W1 x + b1) -> tanh(W2 h + b2) -> W3 h + b3.
-// Weights row-major [out][in] in global memory, read as warp-uniform loads
-// (one L1 transaction per warp); the first hidden layer of this thread's env
-// lives in its own shared-memory column hs[k * kTile] (conflict-free).  The
-// second hidden layer is consumed unit by unit by the output layer, so it is
-// never stored.
-// ---------------------------------------------------------------------------
-constexpr int kTile = 128;
-
-template <int H, int OUT>
-__device__ __forceinline__ void mlp_fp32(const float* __restrict__ w, const float x[kObs],
-                                         float* hs, float out[OUT]) {
-  const float* W1 = w;
-  const float* b1 = W1 + H * kObs;
-  const float* W2 = b1 + H;
-  const float* b2 = W2 + H * H;
-  const float* W3 = b2 + H;
-  const float* b3 = W3 + OUT * H;
-  for (int j = 0; j < H; ++j) {
-    float s = __ldg(b1 + j);
-    const float2* row = reinterpret_cast<const float2*>(W1 + j * kObs);
-#pragma unroll
-    for (int i2 = 0; i2 < kObs / 2; ++i2) {
-      const float2 wv = __ldg(row + i2);
-      s = fmaf(wv.x, x[2 * i2], s);
-      s = fmaf(wv.y, x[2 * i2 + 1], s);
-    }
-    hs[j * kTile] = tanhf(s);
-  }
-#pragma unroll
-  for (int o = 0; o < OUT; ++o) out[o] = __ldg(b3 + o);
-  for (int j = 0; j < H; ++j) {
-    float s0 = __ldg(b2 + j), s1 = 0.0f;
-    const float4* row = reinterpret_cast<const float4*>(W2 + (size_t)j * H);
-#pragma unroll 8
-    for (int k4 = 0; k4 < H / 4; ++k4) {
-      const float4 wv = __ldg(row + k4);
-      s0 = fmaf(wv.x, hs[(4 * k4 + 0) * kTile], s0);
-      s1 = fmaf(wv.y, hs[(4 * k4 + 1) * kTile], s1);
-      s0 = fmaf(wv.z, hs[(4 * k4 + 2) * kTile], s0);
-      s1 = fmaf(wv.w, hs[(4 * k4 + 3) * kTile], s1);
-    }
-    const float h2 = tanhf(s0 + s1);
-#pragma unroll
-    for (int o = 0; o < OUT; ++o) out[o] = fmaf(__ldg(W3 + o * H + j), h2, out[o]);
-  }
-}
-
 // Gaussian head: mean, log-std (fixed or clamped head), sampled action and
 // its log-density from the env's action-noise normals.
 __device__ __forceinline__ void sample_action(const Model& M, uint32_t id, uint64_t t_g,
@@ -159,12 +111,12 @@ __global__ void __launch_bounds__(kTile) k_rollout_fp32(const Model M, Buffers B
     float o[kObs];
     observe(e, o);
     float head[OUT];
-    mlp_fp32<H, OUT>(wp, o, hs, head);
+    mlp_fp32<kObs, H, OUT>(wp, o, hs, head);
     float a[kAct], lp;
     sample_action(M, M.id_base + (uint32_t)i, t_g0 + (uint64_t)t, head, a, &lp);
     if (tr.value) {
       float v[1];
-      mlp_fp32<H, 1>(wv, o, hs, v);
+      mlp_fp32<kObs, H, 1>(wv, o, hs, v);
       tr.value[(size_t)t * n + i] = v[0];
     }
     if (tr.obs) {
@@ -186,7 +138,7 @@ __global__ void __launch_bounds__(kTile) k_rollout_fp32(const Model M, Buffers B
   store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
 }
 
-template <int H, int OUT>
+template <int IN, int H, int OUT>
 __global__ void __launch_bounds__(kTile) k_forward_fp32(const float* __restrict__ wp,
                                                         const float* __restrict__ wv,
                                                         const float* __restrict__ obs, int n,
@@ -196,23 +148,23 @@ __global__ void __launch_bounds__(kTile) k_forward_fp32(const float* __restrict_
   const int i = blockIdx.x * kTile + threadIdx.x;
   if (i >= n) return;
   float* hs = hs_all + threadIdx.x;
-  float o[kObs];
+  float o[IN];
 #pragma unroll
-  for (int k = 0; k < kObs; ++k) o[k] = obs[(size_t)i * kObs + k];
+  for (int k = 0; k < IN; ++k) o[k] = obs[(size_t)i * IN + k];
   float h[OUT];
-  mlp_fp32<H, OUT>(wp, o, hs, h);
+  mlp_fp32<IN, H, OUT>(wp, o, hs, h);
 #pragma unroll
   for (int k = 0; k < OUT; ++k) head[(size_t)i * OUT + k] = h[k];
   if (value) {
     float v[1];
-    mlp_fp32<H, 1>(wv, o, hs, v);
+    mlp_fp32<IN, H, 1>(wv, o, hs, v);
     value[i] = v[0];
   }
 }
 
 // Value network on trajectory-layout observations: row r = t*n + i reads
-// obs[(t*18 + k)*n + i].
-template <int H>
+// obs[(t*IN + k)*n + i].
+template <int IN, int H>
 __global__ void __launch_bounds__(kTile) k_value_fp32(const float* __restrict__ wv,
                                                       const float* __restrict__ obs, size_t rows,
                                                       int n, float* __restrict__ value) {
@@ -221,11 +173,11 @@ __global__ void __launch_bounds__(kTile) k_value_fp32(const float* __restrict__ 
   if (r >= rows) return;
   float* hs = hs_all + threadIdx.x;
   const size_t t = r / (size_t)n, i = r % (size_t)n;
-  float o[kObs];
+  float o[IN];
 #pragma unroll
-  for (int k = 0; k < kObs; ++k) o[k] = obs[(t * kObs + k) * n + i];
+  for (int k = 0; k < IN; ++k) o[k] = obs[(t * IN + k) * n + i];
   float v[1];
-  mlp_fp32<H, 1>(wv, o, hs, v);
+  mlp_fp32<IN, H, 1>(wv, o, hs, v);
   value[r] = v[0];
 }
 
@@ -278,43 +230,57 @@ cudaError_t launch_rollout_fp32(const Model& M, const Buffers& B, const float* w
   return cudaErrorInvalidValue;
 }
 
-template <int H>
+template <int IN, int H>
 static cudaError_t value_fp32_impl(const float* wv, const float* obs, size_t rows, int n,
                                    float* value, cudaStream_t s) {
   const size_t smem = (size_t)H * kTile * sizeof(float);
-  cudaError_t err = cudaFuncSetAttribute(k_value_fp32<H>,
+  cudaError_t err = cudaFuncSetAttribute(k_value_fp32<IN, H>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
   const size_t blocks = (rows + kTile - 1) / kTile;
-  k_value_fp32<H><<<(unsigned)blocks, kTile, smem, s>>>(wv, obs, rows, n, value);
+  k_value_fp32<IN, H><<<(unsigned)blocks, kTile, smem, s>>>(wv, obs, rows, n, value);
   return cudaGetLastError();
 }
 
 cudaError_t launch_value_fp32(const Model& M, const float* wv, const float* obs, size_t rows,
                               int n, float* value, cudaStream_t s) {
-  if (M.hidden == 64) return value_fp32_impl<64>(wv, obs, rows, n, value, s);
-  if (M.hidden == 256) return value_fp32_impl<256>(wv, obs, rows, n, value, s);
+  const bool paper = M.model == 1;
+  if (M.hidden == 64)
+    return paper ? value_fp32_impl<12, 64>(wv, obs, rows, n, value, s)
+                 : value_fp32_impl<kObs, 64>(wv, obs, rows, n, value, s);
+  if (M.hidden == 256)
+    return paper ? value_fp32_impl<12, 256>(wv, obs, rows, n, value, s)
+                 : value_fp32_impl<kObs, 256>(wv, obs, rows, n, value, s);
   return cudaErrorInvalidValue;
 }
 
-template <int H, int OUT>
+template <int IN, int H, int OUT>
 static cudaError_t forward_fp32_impl(const float* wp, const float* wv, const float* obs, int n,
                                      float* head, float* value, cudaStream_t s) {
   const size_t smem = (size_t)H * kTile * sizeof(float);
-  cudaError_t err = cudaFuncSetAttribute(k_forward_fp32<H, OUT>,
+  cudaError_t err = cudaFuncSetAttribute(k_forward_fp32<IN, H, OUT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
-  k_forward_fp32<H, OUT><<<blocks_for(n, kTile), kTile, smem, s>>>(wp, wv, obs, n, head, value);
+  k_forward_fp32<IN, H, OUT><<<blocks_for(n, kTile), kTile, smem, s>>>(wp, wv, obs, n, head,
+                                                                        value);
   return cudaGetLastError();
 }
 
 cudaError_t launch_forward_fp32(const Model& M, const float* wp, const float* wv,
                                 const float* obs, int n, float* head, float* value,
                                 cudaStream_t s) {
-  if (M.hidden == 64 && M.policy_out == 8) return forward_fp32_impl<64, 8>(wp, wv, obs, n, head, value, s);
-  if (M.hidden == 64 && M.policy_out == 16) return forward_fp32_impl<64, 16>(wp, wv, obs, n, head, value, s);
-  if (M.hidden == 256 && M.policy_out == 8) return forward_fp32_impl<256, 8>(wp, wv, obs, n, head, value, s);
-  if (M.hidden == 256 && M.policy_out == 16) return forward_fp32_impl<256, 16>(wp, wv, obs, n, head, value, s);
+  const int H = M.hidden, O = M.policy_out;
+  if (M.model == 1) {
+    if (H == 64 && O == 6) return forward_fp32_impl<12, 64, 6>(wp, wv, obs, n, head, value, s);
+    if (H == 64 && O == 12) return forward_fp32_impl<12, 64, 12>(wp, wv, obs, n, head, value, s);
+    if (H == 256 && O == 6) return forward_fp32_impl<12, 256, 6>(wp, wv, obs, n, head, value, s);
+    if (H == 256 && O == 12) return forward_fp32_impl<12, 256, 12>(wp, wv, obs, n, head, value, s);
+    return cudaErrorInvalidValue;
+  }
+  if (H == 64 && O == 8) return forward_fp32_impl<kObs, 64, 8>(wp, wv, obs, n, head, value, s);
+  if (H == 64 && O == 16) return forward_fp32_impl<kObs, 64, 16>(wp, wv, obs, n, head, value, s);
+  if (H == 256 && O == 8) return forward_fp32_impl<kObs, 256, 8>(wp, wv, obs, n, head, value, s);
+  if (H == 256 && O == 16) return forward_fp32_impl<kObs, 256, 16>(wp, wv, obs, n, head, value, s);
   return cudaErrorInvalidValue;
 }
 

@@ -42,7 +42,7 @@ def test_library_exports_every_declared_symbol(auvlib):
     assert not missing, missing
     for n in names:
         assert hasattr(auvlib, n)
-    assert auvlib.env_abi_version() == 1
+    assert auvlib.env_abi_version() == 2
 
 
 def test_config_struct_size_matches_header(auvlib):
@@ -70,6 +70,44 @@ def test_invalid_configs_are_rejected(auvlib, field, value, code):
     rc = auvlib.env_create(C.byref(cfg), None, C.byref(h))
     assert rc == code, auvlib.env_last_error(None)
     assert not h.value
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("model", 5, -1), ("mavg_len", 0, -1), ("mavg_len", 9, -1), ("policy_out", 8, -1),
+    ("goal_att_range", 4.0, -1), ("fluid_density", -1.0, -1), ("f_max", float("inf"), -1),
+    ("hidden", 128, -6),
+])
+def test_invalid_paper_model_configs_are_rejected(auvlib, field, value, code):
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    cfg = auvenv.make_config(W.workload("paper_tiny"))
+    setattr(cfg, field, value)
+    h = C.c_void_p()
+    rc = auvlib.env_create(C.byref(cfg), None, C.byref(h))
+    assert rc == code, auvlib.env_last_error(None)
+    assert not h.value
+
+
+def test_paper_model_needs_an_inertia_box(auvlib):
+    """The inertia fluid model needs a box with the body's moments: each
+    principal moment below the sum of the other two."""
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    cfg = auvenv.make_config(W.workload("paper_tiny", inertia=(0.5, 0.1, 0.1)))
+    h = C.c_void_p()
+    assert auvlib.env_create(C.byref(cfg), None, C.byref(h)) == auvenv.AUV_ERR_INVALID
+    assert b"inertia box" in auvlib.env_last_error(None)
+
+
+def test_layout_of_each_model(auvlib):
+    from paper_2512_13359_gb300 import auvenv, workloads as W
+    f = auvenv.layout(auvenv.AUV_MODEL_FOSSEN)
+    assert (f.obs_dim, f.act_dim, f.state_fields, f.param_fields) == (
+        W.OBS_DIM, W.ACT_DIM, W.STATE_FIELDS, W.PARAM_FIELDS)
+    p = auvenv.layout(auvenv.AUV_MODEL_PAPER)
+    assert (p.obs_dim, p.act_dim, p.state_fields, p.param_fields) == (
+        W.PAPER_OBS_DIM, W.PAPER_ACT_DIM, W.PAPER_STATE_FIELDS, W.PAPER_PARAM_FIELDS)
+    out = auvenv.AuvLayout()
+    assert auvlib.env_layout(7, C.byref(out)) == auvenv.AUV_ERR_INVALID
+    assert auvlib.env_layout(0, None) == auvenv.AUV_ERR_INVALID
 
 
 def test_bf16_mode_requires_the_built_shape(auvlib):
