@@ -128,31 +128,42 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # algorithmic work per env-step
 # ---------------------------------------------------------------------------
-def mlp_flops(hidden, out):
-    return 2 * (W.OBS_DIM * hidden + hidden * hidden + hidden * out)
+def mlp_flops(in_dim, hidden, out):
+    return 2 * (in_dim * hidden + hidden * hidden + hidden * out)
 
 
-def traj_bytes_per_env_step(keys):
-    b = dict(obs=4 * W.OBS_DIM, act=4 * W.ACT_DIM, logp=4, value=4, rew=4, done=1)
+def traj_bytes_per_env_step(w, keys):
+    b = dict(obs=4 * W.obs_dim(w), act=4 * W.act_dim(w), logp=4, value=4, rew=4, done=1)
     return sum(b[k] for k in keys)
+
+
+def dyn_flops_per_env_step(w):
+    return PAPER_DYN_FLOPS_PER_ENV_STEP if W.is_paper(w) else DYN_FLOPS_PER_ENV_STEP
 
 
 # ---------------------------------------------------------------------------
 # reference arm / CPU baseline: the oracle on a bounded sample
 # ---------------------------------------------------------------------------
+def oracle_api(w):
+    """(model, batch class, reset, rollout) of the oracle for w's model."""
+    from oracle import oracle as O
+    if W.is_paper(w):
+        return O.paper_model(w), O.PaperBatch, O.paper_reset, O.paper_rollout
+    return O.model(w), O.Batch, O.reset, O.rollout
+
+
 def oracle_sample_rate(w, T, target_s, max_envs=4096):
     """Time the CPU oracle on a sample of envs over T steps; env-steps/s on
     one host core.  The sample grows until it takes about target_s."""
-    from oracle import oracle as O
-    m = O.model(w)
+    m, Batch, reset, rollout = oracle_api(w)
     pw = W.policy_weights(w)
     vw = W.value_weights(w) if w["has_value"] else None
     n = 2
     while True:
-        b = O.Batch(np.arange(n))
-        O.reset(m, b)
+        b = Batch(np.arange(n))
+        reset(m, b)
         t0 = time.perf_counter()
-        O.rollout(m, b, pw, vw, 0, T)
+        rollout(m, b, pw, vw, 0, T)
         dt = time.perf_counter() - t0
         if dt >= target_s or n >= max_envs:
             return n * T / dt, n, dt
@@ -166,7 +177,7 @@ def run_reference(args, w):
     from oracle import oracle as O
     O.build()
     T = w["steps"]
-    m = O.model(w)
+    m, Batch, reset, rollout = oracle_api(w)
     pw = W.policy_weights(w)
     vw = W.value_weights(w) if w["has_value"] else None
     # size one bench step so that K + W steps take about a minute in total
@@ -175,10 +186,10 @@ def run_reference(args, w):
     n = max(1, int(rate * per_step_s / T))
     times = []
     for s in range(args.warmup + args.steps):
-        b = O.Batch(np.arange(n))
-        O.reset(m, b)
+        b = Batch(np.arange(n))
+        reset(m, b)
         t0 = time.perf_counter()
-        O.rollout(m, b, pw, vw, 0, T)
+        rollout(m, b, pw, vw, 0, T)
         if s >= args.warmup:
             times.append(time.perf_counter() - t0)
     sec = sum(times) / len(times)
@@ -217,7 +228,7 @@ def run_replay(args):
     n, T = int(w["n_envs"]), int(w["steps"])
     env = auvenv.Env(w)
     env.reset()
-    act = torch.from_numpy(W.replay_actions(1, T, n)).cuda()
+    act = torch.from_numpy(W.replay_actions(1, T, n, act=W.act_dim(w))).cuda()
     rew = torch.empty((T, n), device="cuda")
     done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
     flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
@@ -245,7 +256,7 @@ def run_replay(args):
     sm_mhz = (clock_info or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     fp32_peak = 2 * 128 * n_sm * sm_mhz * 1e6 / 1e12
-    achieved = n * T * DYN_FLOPS_PER_ENV_STEP / (step_ms * 1e-3) / 1e12
+    achieved = n * T * dyn_flops_per_env_step(w) / (step_ms * 1e-3) / 1e12
     line = {
         "metric": "env-steps/s (physics only, action replay)", "value": n * T / (step_ms * 1e-3),
         "unit": "env-steps/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
@@ -371,7 +382,7 @@ def run(args):
         h_pw = torch.from_numpy(pw).pin_memory()
         h_vw = torch.from_numpy(vw).pin_memory() if vw is not None else None
         h2d = h_pw.numel() * 4 + (h_vw.numel() * 4 if h_vw is not None else 0)
-        d2h = n * T * traj_bytes_per_env_step(h_keys)
+        d2h = n * T * traj_bytes_per_env_step(w, h_keys)
         for _ in range(2):
             env.set_weights(h_pw, h_vw)
             env.rollout(T, h_traj)
@@ -396,8 +407,8 @@ def run(args):
     peaks, peak_src = load_peaks()
     roll_avg = sum(roll_ms) / len(roll_ms)
     val_avg = sum(val_ms) / len(val_ms) if value is not None else 0.0
-    pol_fl = mlp_flops(w["hidden"], w["policy_out"])
-    val_fl = mlp_flops(w["hidden"], 1) if w["has_value"] else 0
+    pol_fl = mlp_flops(W.obs_dim(w), w["hidden"], w["policy_out"])
+    val_fl = mlp_flops(W.obs_dim(w), w["hidden"], 1) if w["has_value"] else 0
     sm_mhz = (clock_info or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
     n_sm = torch.cuda.get_device_properties(local).multi_processor_count
     fp32_peak = 2 * 128 * n_sm * sm_mhz * 1e6 / 1e12   # TFLOP/s of the FP32 pipe
@@ -415,11 +426,11 @@ def run(args):
                 "peak_source": f"bf16 sustained, {peak_src}"}
     else:
         kern, dur = "rollout_fp32", roll_avg
-        flops = n * T * (pol_fl + val_fl + DYN_FLOPS_PER_ENV_STEP)
+        flops = n * T * (pol_fl + val_fl + dyn_flops_per_env_step(w))
         if value is not None and val_avg > roll_avg:
             kern, dur, flops = "value_fp32", val_avg, n * T * val_fl
         elif value is not None:
-            flops = n * T * (pol_fl + DYN_FLOPS_PER_ENV_STEP)
+            flops = n * T * (pol_fl + dyn_flops_per_env_step(w))
         achieved = flops / (dur * 1e-3) / 1e12
         roof = {"bound": "alu", "kernel": kern, "achieved": achieved, "peak": fp32_peak,
                 "unit": "TFLOP/s", "frac": achieved / fp32_peak, "traffic": None,
@@ -460,6 +471,11 @@ def run(args):
 # (substep) + reward 93 + action sampling and log-probability 72 (adds,
 # multiplies and divides; square roots and transcendentals not counted).
 DYN_FLOPS_PER_ENV_STEP = 1962
+# The paper model, counted the same way: observation 95 + wrench 6 + 4 x 245
+# (substep; the inertia-box constants, 78 flops that the oracle recomputes
+# in every substep, are per model, not per step) + reward 185 (including its
+# own observation of the post-step state) + sampling six actions 54.
+PAPER_DYN_FLOPS_PER_ENV_STEP = 1320
 
 if __name__ == "__main__":
     main()

@@ -159,8 +159,6 @@ int validate_paper(const auv_config* c) {
   if (c->mavg_len < 1 || c->mavg_len > AUV_PAPER_HIST)
     return fail(nullptr, AUV_ERR_INVALID, "mavg_len %u outside [1, %d]", c->mavg_len,
                 AUV_PAPER_HIST);
-  if (c->mlp_mode == AUV_MLP_BF16)
-    return fail(nullptr, AUV_ERR_UNSUPPORTED, "the paper model runs fp32 networks only");
   return validate_networks(c, AUV_PAPER_ACT_DIM);
 }
 

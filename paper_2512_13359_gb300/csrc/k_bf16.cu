@@ -26,6 +26,7 @@
 #include <climits>
 
 #include "auv_bf16.h"
+#include "paper_device.cuh"
 #include "tc_ptx.cuh"
 
 namespace auv {
@@ -80,15 +81,17 @@ __device__ __forceinline__ uint16_t bf16_bits(float x) {
 }
 
 // One thread per 16-byte piece of the W1/W2/W3 regions, then the vectors.
-__global__ void k_pack(const float* __restrict__ w, int out_dim, uint8_t* __restrict__ img) {
-  const int kObsDim = 18;
+// in_dim: network input width (18 or 12, <= 32); out_dim: 1 (value) or the
+// policy head width (<= 16; head rows out_dim..15 are packed as zeros).
+__global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
+                       uint8_t* __restrict__ img) {
   const float* W1 = w;
-  const float* b1 = W1 + kH * kObsDim;
+  const float* b1 = W1 + kH * in_dim;
   const float* W2 = b1 + kH;
   const float* b2 = W2 + kH * kH;
   const float* W3 = b2 + kH;
   const float* b3 = W3 + out_dim * kH;
-  const bool policy = out_dim == kHeadOut;
+  const bool policy = out_dim > 1;
   const int n_w1 = kH * 4, n_w2 = 4 * kH * 8, n_w3 = policy ? 4 * kHeadOut * 8 : 0;
   const int piece = blockIdx.x * blockDim.x + threadIdx.x;
   uint16_t v[8];
@@ -97,7 +100,7 @@ __global__ void k_pack(const float* __restrict__ w, int out_dim, uint8_t* __rest
     const int n = piece >> 2, p = piece & 3, q = p ^ ((n >> 1) & 3);
     for (int e = 0; e < 8; ++e) {
       const int k = 8 * q + e;
-      v[e] = k < kObsDim ? bf16_bits(W1[n * kObsDim + k]) : (uint16_t)0;
+      v[e] = k < in_dim ? bf16_bits(W1[n * in_dim + k]) : (uint16_t)0;
     }
     off = kOffW1 + n * 64 + p * 16;
   } else if (piece < n_w1 + n_w2) {
@@ -108,7 +111,8 @@ __global__ void k_pack(const float* __restrict__ w, int out_dim, uint8_t* __rest
   } else if (piece < n_w1 + n_w2 + n_w3) {
     const int id = piece - n_w1 - n_w2;
     const int a = id / (kHeadOut * 8), n = (id / 8) % kHeadOut, p = id & 7, q = p ^ (n & 7);
-    for (int e = 0; e < 8; ++e) v[e] = bf16_bits(W3[n * kH + 64 * a + 8 * q + e]);
+    for (int e = 0; e < 8; ++e)
+      v[e] = n < out_dim ? bf16_bits(W3[n * kH + 64 * a + 8 * q + e]) : (uint16_t)0;
     off = kOffW3 + a * (kHeadOut * 128) + n * 128 + p * 16;
   } else {
     const int id = piece - n_w1 - n_w2 - n_w3;   // vector entries, one float each
@@ -116,7 +120,8 @@ __global__ void k_pack(const float* __restrict__ w, int out_dim, uint8_t* __rest
     if (policy) {
       if (id < kH) f[(kOffB1P >> 2) + id] = b1[id];
       else if (id < 2 * kH) f[(kOffB2P >> 2) + id - kH] = b2[id - kH];
-      else if (id < 2 * kH + kHeadOut) f[(kOffB3P >> 2) + id - 2 * kH] = b3[id - 2 * kH];
+      else if (id < 2 * kH + kHeadOut)
+        f[(kOffB3P >> 2) + id - 2 * kH] = id - 2 * kH < out_dim ? b3[id - 2 * kH] : 0.0f;
     } else {
       if (id < kH) f[(kOffB1V >> 2) + id] = b1[id];
       else if (id < 2 * kH) f[(kOffB2V >> 2) + id - kH] = b2[id - kH];
@@ -154,11 +159,13 @@ struct Barriers {
   int abort;
 };
 
-struct RowIO {            // row modes: obs element (r, k) at ((r / ns) * 18 + k) * ns + r % ns
+struct RowIO {            // row modes: obs element (r, k) at ((r / ns) * obs_dim + k) * ns + r % ns
   const float* obs;
   size_t rows;
   int ns;
-  float* out;             // head[r][16] (policy) or value[r] (value)
+  float* out;             // head[r][out_dim] (policy) or value[r] (value)
+  int obs_dim;            // 18 (Fossen model) or 12 (paper model)
+  int out_dim;            // policy head width written per row
 };
 
 template <int G, int MODE>
@@ -174,13 +181,15 @@ struct Engine {
 };
 
 // Row r of the observation tile (bf16, K = 32, 64-byte swizzle): 4 pieces of
-// 16 bytes, piece q at position q ^ ((r >> 1) & 3).  Features 18..31 are zero.
-__device__ __forceinline__ void write_obs_row(uint8_t* tile, int r, const float o[kObs]) {
+// 16 bytes, piece q at position q ^ ((r >> 1) & 3).  Features NOBS..31 are zero.
+template <int NOBS>
+__device__ __forceinline__ void write_obs_row(uint8_t* tile, int r, const float o[NOBS]) {
+  static_assert(NOBS % 2 == 0 && NOBS <= 32, "observation width");
   uint32_t w[16];
 #pragma unroll
-  for (int j = 0; j < 9; ++j) w[j] = tc::pack_bf16x2(o[2 * j], o[2 * j + 1]);
+  for (int j = 0; j < NOBS / 2; ++j) w[j] = tc::pack_bf16x2(o[2 * j], o[2 * j + 1]);
 #pragma unroll
-  for (int j = 9; j < 16; ++j) w[j] = 0u;
+  for (int j = NOBS / 2; j < 16; ++j) w[j] = 0u;
   const int sw = (r >> 1) & 3;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -230,7 +239,9 @@ __device__ __forceinline__ int step_index(int it, int g, const int (&iters)[G]) 
 // of a buffer is ordered either by an "empty" barrier the MMA thread waits on
 // or by a commit: an epilogue only starts after a commit that covers every
 // MMA issued before it.
-template <int G, int MODE>
+// SIM selects the environment model of the fused rollout (0: Fossen,
+// 1: the paper model); the row modes ignore it.
+template <int G, int MODE, int SIM>
 __global__ void __launch_bounds__(G * 128 + 96) __maxnreg__(G == 4 ? 96 : 168)
 k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
          uint64_t t_g0, RowIO io, Status* st) {
@@ -524,7 +535,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     int my_iters = 0;
 #pragma unroll
     for (int j = 0; j < G; ++j) my_iters = j == g ? iters[j] : my_iters;
-    if (MODE == kRollout) {
+    if constexpr (MODE == kRollout && SIM == 0) {
       int n_act = 0;
 #pragma unroll
       for (int j = 0; j < G; ++j) n_act += iters[j] > 0 ? 1 : 0;
@@ -547,7 +558,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
 #pragma unroll
           for (int k = 0; k < kObs; ++k) o[k] = 0.0f;
         }
-        write_obs_row(obs_tile, row, o);
+        write_obs_row<kObs>(obs_tile, row, o);
         tc::fence_async_smem();
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
@@ -588,6 +599,69 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         if (bad) flag_nan(st, i);
         store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
       }
+    } else if constexpr (MODE == kRollout && SIM == 1) {
+      // The paper's own environment: 12-float observation, 6-D wrench
+      // action (mean head[0..5], clamped log-std head[6..11]), history in
+      // the state rows.
+      constexpr int kPO = paper::kObs, kPA = paper::kAct;
+      int n_act = 0;
+#pragma unroll
+      for (int j = 0; j < G; ++j) n_act += iters[j] > 0 ? 1 : 0;
+      const int tile = slot0 + g;
+      const int i = tile * kRows + row;
+      const bool active = my_iters > 0 && i < M.n;
+      const size_t n = (size_t)M.n;
+      paper::Env e;
+      if (active) paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+      bool bad = false;
+      for (int t = 0; t < my_iters && ok; ++t) {
+        float o[kPO];
+        if (active) {
+          paper::observe(e, o);
+          if (tr.obs) {
+#pragma unroll
+            for (int k = 0; k < kPO; ++k) tr.obs[((size_t)t * kPO + k) * n + i] = o[k];
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < kPO; ++k) o[k] = 0.0f;
+        }
+        write_obs_row<kPO>(obs_tile, row, o);
+        tc::fence_async_smem();
+        tc::mbar_arrive(&bar->obs_full[g]);
+        float head[kHeadOut];
+        __syncwarp();
+        if (!(ok = run_network(t * n_act + g, t, head))) break;
+        __syncwarp();
+        if (active) {
+          const uint32_t id = M.id_base + (uint32_t)i;
+          float eps[8];
+          action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
+          float a[kPA], lp = 0.0f;
+#pragma unroll
+          for (int k = 0; k < kPA; ++k) {
+            const float ls = fminf(fmaxf(head[kPA + k], M.logstd_min), M.logstd_max);
+            a[k] = fmaf(expf(ls), eps[k], head[k]);
+            lp += -0.5f * eps[k] * eps[k] - ls;
+          }
+          lp -= (float)kPA * 0.91893853320467274f;
+          if (tr.act) {
+#pragma unroll
+            for (int k = 0; k < kPA; ++k) tr.act[((size_t)t * kPA + k) * n + i] = a[k];
+          }
+          if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
+          bool d;
+          const float r = paper::physics_step(M, id, e, a, B.state, i, &d);
+          if (tr.rew) tr.rew[(size_t)t * n + i] = r;
+          if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
+          bad |= !paper::env_finite(e);
+        }
+        __syncwarp();
+      }
+      if (active) {
+        if (bad) flag_nan(st, i);
+        paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+      }
     } else {
       for (int it = 0; it < my_iters && ok; ++it) {
         const size_t r = (size_t)(slot0 + g + it * n_slots) * kRows + row;
@@ -595,14 +669,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         float o[kObs];
         if (active) {
           const size_t ns = (size_t)io.ns;
-          const size_t base = (r / ns) * kObs * ns + r % ns;
+          const size_t base = (r / ns) * (size_t)io.obs_dim * ns + r % ns;
 #pragma unroll
-          for (int k = 0; k < kObs; ++k) o[k] = __ldg(io.obs + base + (size_t)k * ns);
+          for (int k = 0; k < kObs; ++k)
+            o[k] = k < io.obs_dim ? __ldg(io.obs + base + (size_t)k * ns) : 0.0f;
         } else {
 #pragma unroll
           for (int k = 0; k < kObs; ++k) o[k] = 0.0f;
         }
-        write_obs_row(obs_tile, row, o);
+        write_obs_row<kObs>(obs_tile, row, o);
         tc::fence_async_smem();
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
@@ -614,7 +689,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             io.out[r] = head[0];
           } else {
 #pragma unroll
-            for (int k = 0; k < kHeadOut; ++k) io.out[r * kHeadOut + k] = head[k];
+            for (int k = 0; k < kHeadOut; ++k)
+              if (k < io.out_dim) io.out[r * io.out_dim + k] = head[k];
           }
         }
       }
@@ -644,15 +720,15 @@ int sm_count() {
   return cached;
 }
 
-template <int G, int MODE>
+template <int G, int MODE, int SIM = 0>
 cudaError_t launch_engine(int grid, const Model& M, const Buffers& B, const uint8_t* image,
                           const Traj& tr, int T, uint64_t t_g0, const RowIO& io, Status* st,
                           cudaStream_t s) {
   using E = Engine<G, MODE>;
-  cudaError_t err = cudaFuncSetAttribute(k_engine<G, MODE>,
+  cudaError_t err = cudaFuncSetAttribute(k_engine<G, MODE, SIM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, E::kSmem);
   if (err != cudaSuccess) return err;
-  k_engine<G, MODE><<<grid, E::kThreads, E::kSmem, s>>>(M, B, image, tr, T, t_g0, io, st);
+  k_engine<G, MODE, SIM><<<grid, E::kThreads, E::kSmem, s>>>(M, B, image, tr, T, t_g0, io, st);
   return cudaGetLastError();
 }
 
@@ -708,14 +784,15 @@ size_t bf16_value_image_bytes() { return kValueImage; }
 
 cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* wv_f32,
                              void* wp_packed, void* wv_packed, cudaStream_t s) {
-  (void)M;
+  const int in_dim = M.model == 1 ? 12 : kObs;
   const int pol_pieces = kH * 4 + 4 * kH * 8 + 4 * kHeadOut * 8 + 2 * kH + kHeadOut;
-  k_pack<<<(pol_pieces + 255) / 256, 256, 0, s>>>(wp_f32, kHeadOut,
+  k_pack<<<(pol_pieces + 255) / 256, 256, 0, s>>>(wp_f32, in_dim, M.policy_out,
                                                   static_cast<uint8_t*>(wp_packed));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || !wv_f32) return e;
   const int val_pieces = kH * 4 + 4 * kH * 8 + 3 * kH + 1;
-  k_pack<<<(val_pieces + 255) / 256, 256, 0, s>>>(wv_f32, 1, static_cast<uint8_t*>(wv_packed));
+  k_pack<<<(val_pieces + 255) / 256, 256, 0, s>>>(wv_f32, in_dim, 1,
+                                                  static_cast<uint8_t*>(wv_packed));
   return cudaGetLastError();
 }
 
@@ -725,7 +802,14 @@ cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp
   const int G = pick_groups(tiles);
   const int grid = (int)((tiles + G - 1) / G);
   const uint8_t* img = static_cast<const uint8_t*>(wp_packed);
-  const RowIO io = {nullptr, 0, 1, nullptr};
+  const RowIO io = {nullptr, 0, 1, nullptr, 0, 0};
+  if (M.model == 1) {
+    switch (G) {
+      case 4: return launch_engine<4, kRollout, 1>(grid, M, B, img, tr, T, t_g0, io, st, s);
+      case 2: return launch_engine<2, kRollout, 1>(grid, M, B, img, tr, T, t_g0, io, st, s);
+      default: return launch_engine<1, kRollout, 1>(grid, M, B, img, tr, T, t_g0, io, st, s);
+    }
+  }
   switch (G) {
     case 4: return launch_engine<4, kRollout>(grid, M, B, img, tr, T, t_g0, io, st, s);
     case 2: return launch_engine<2, kRollout>(grid, M, B, img, tr, T, t_g0, io, st, s);
@@ -753,7 +837,7 @@ cudaError_t launch_value_bf16(const Model& M, const void* wv_packed, const float
                               const float* obs, size_t rows, int n, float* value, Status* st,
                               cudaStream_t s) {
   (void)wv_f32;
-  const RowIO io = {obs, rows, n, value};
+  const RowIO io = {obs, rows, n, value, M.model == 1 ? 12 : kObs, 1};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), io, st, s);
 }
 
@@ -761,10 +845,11 @@ cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const voi
                                 const float* wv_f32, const float* obs, int n, float* head,
                                 float* value, Status* st, cudaStream_t s) {
   (void)wv_f32;
-  const RowIO io = {obs, (size_t)n, 1, head};
+  const int od = M.model == 1 ? 12 : kObs;
+  const RowIO io = {obs, (size_t)n, 1, head, od, M.policy_out};
   cudaError_t e = launch_rows<kPolicyRows>(M, static_cast<const uint8_t*>(wp_packed), io, st, s);
   if (e != cudaSuccess || !value) return e;
-  const RowIO iov = {obs, (size_t)n, 1, value};
+  const RowIO iov = {obs, (size_t)n, 1, value, od, 1};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), iov, st, s);
 }
 

@@ -3,8 +3,9 @@ inertia-box fluid model, effective gravity, 12-float axis-angle observation,
 five-term reward of Eqs. 2-7) through the C ABI against the oracle's paper
 model: resets bit-exact (including the zeroed action history), observation,
 action replay and the fp32 closed-loop rollout within the fp32 tolerances of
-the Fossen model, auto-resets inside the horizon, and host trajectories
-equal to device ones."""
+the Fossen model, auto-resets inside the horizon, host trajectories equal to
+device ones, and the tensor-core (bf16) networks and rollout within the bf16
+tolerances of the Fossen model's tensor-core path."""
 import numpy as np
 import pytest
 
@@ -121,3 +122,75 @@ def test_paper_host_trajectory_matches_device():
         outs.append({k: to_np(v).copy() for k, v in traj.items()})
     for k in outs[0]:
         assert np.array_equal(outs[0][k], outs[1][k]), k
+
+
+BF16_TOL = 3e-2     # network outputs, as for the Fossen model's bf16 path
+
+
+@pytest.mark.parametrize("n", [1, 300, 40000])
+def test_paper_bf16_forward(oracle, n):
+    torch = need_gpu()
+    w = W.workload("paper_4096", n_envs=64)
+    env = make_env(w, bias_std=0.1)
+    obs = W.random_observations(5, n, dim=12)
+    head = torch.empty((n, 12), device="cuda")
+    val = torch.empty((n,), device="cuda")
+    env.policy_forward(torch.from_numpy(obs).cuda(), head, val)
+    assert env.status().code == 0
+    idx = np.unique(np.r_[0, n - 1, np.random.default_rng(0).integers(0, n, 200)])
+    ref_h = oracle.mlp(W.policy_weights(w, 0.1), 12, 256, 12, True, obs[idx].astype(np.float64))
+    ref_v = oracle.mlp(W.value_weights(w, 0.1), 12, 256, 1, True, obs[idx].astype(np.float64))
+    eh = np.abs(to_np(head)[idx] - ref_h).max()
+    ev = np.abs(to_np(val)[idx] - ref_v[:, 0]).max()
+    print(f"[paper bf16] n={n}: head {eh:.3e} value {ev:.3e} (tol {BF16_TOL})")
+    assert eh <= BF16_TOL and ev <= BF16_TOL
+
+
+def test_paper_bf16_rollout(oracle):
+    """The paper workload's tensor-core rollout over one whole episode
+    (T = episode_len): step-0 observations to 1e-5, actions and log-probs
+    within the bf16 head tolerance, dones exact, values against the oracle's
+    bf16 value network, and the final state equal bit for bit to the next
+    episode's reset draw (history cleared)."""
+    torch = need_gpu()
+    n, T = 4096, 48
+    w = W.workload("paper_4096", n_envs=n, episode_len=T)
+    env = make_env(w)
+    env.reset()
+    traj = env.alloc_traj(T)
+    env.rollout(T, traj)
+    assert env.status().code == 0
+    m = oracle.paper_model(w)
+    sample = np.r_[0, 1, 2, 1000, 2047, 4095]
+    b = oracle.PaperBatch(sample)
+    oracle.paper_reset(m, b)
+    ref = oracle.paper_rollout(m, b, W.policy_weights(w), W.value_weights(w), 0, 1)
+    assert_close(to_np(traj["obs"])[0][:, sample], ref["obs"][0], 1e-5, what="obs step 0")
+    assert np.abs(to_np(traj["act"])[0][:, sample] - ref["act"][0]).max() <= 0.24
+    assert np.abs(to_np(traj["logp"])[0][sample] - ref["logp"][0]).max() <= 0.24
+    assert np.abs(to_np(traj["value"])[0][sample] - ref["value"][0]).max() <= BF16_TOL
+    done = to_np(traj["done"])
+    assert np.all(done[:-1] == 0) and np.all(done[-1] == 1)
+    full = oracle.PaperBatch(np.arange(n))
+    oracle.paper_reset(m, full)
+    oracle.paper_reset(m, full)
+    assert np.array_equal(to_np(env.state).view(np.uint32),
+                          full.state.astype(np.float32).view(np.uint32))
+    assert np.array_equal(to_np(env.params).view(np.uint32),
+                          full.params.astype(np.float32).view(np.uint32))
+
+
+def test_paper_bf16_value_over_trajectory_layout(oracle):
+    torch = need_gpu()
+    n, T = 1000, 5
+    w = W.workload("paper_4096", n_envs=n)
+    env = make_env(w, bias_std=0.1)
+    obs = W.random_observations(6, T * n, dim=12).reshape(T, n, 12).transpose(0, 2, 1).copy()
+    val = torch.empty((T, n), device="cuda")
+    env.value(torch.from_numpy(obs).cuda(), val)
+    vw = W.value_weights(w, 0.1)
+    g = to_np(val)
+    for t in (0, 2, 4):
+        idx = np.r_[0, 1, 500, 999]
+        ref = oracle.mlp(vw, 12, 256, 1, True, obs[t][:, idx].T.astype(np.float64))[:, 0]
+        assert np.abs(g[t, idx] - ref).max() <= BF16_TOL
