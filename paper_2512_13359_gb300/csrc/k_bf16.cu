@@ -215,6 +215,26 @@ __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const flo
   }
 }
 
+// The step's 8 action normals in the tensor-core path's precision class: the
+// Philox words and Box-Muller steps of action_noise, with the hardware
+// approximations of log and sin/cos (absolute error about 1e-6 on a normal,
+// far below the bf16 network's own error on the action it perturbs).
+__device__ __forceinline__ void action_noise_approx(uint32_t env, uint32_t seed, uint64_t t_g,
+                                                    float eps[8]) {
+  const uint32_t lo = (uint32_t)t_g, hi = (uint32_t)(t_g >> 32);
+  const uint4 a = philox10(lo, hi, 0u, 0u, env, seed);
+  const uint4 b = philox10(lo, hi, 0u, 1u, env, seed);
+  const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float r = sqrtf(-2.0f * __logf(uniform01(w[2 * k])));
+    float sn, cs;
+    __sincosf(6.28318530717958648f * uniform01(w[2 * k + 1]), &sn, &cs);
+    eps[2 * k] = r * cs;
+    eps[2 * k + 1] = r * sn;
+  }
+}
+
 // Group-steps are numbered in the order the MMA warp serves them: iteration
 // it of every group that still has work, groups in ascending order (the
 // groups with work always form a prefix).  Index of (it, g):
@@ -572,12 +592,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           reload_params(M, B.params, i, e);
           const uint32_t id = M.id_base + (uint32_t)i;
           float eps[kAct];
-          action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
+          action_noise_approx(id, M.seed, t_g0 + (uint64_t)t, eps);
           float a[kAct], lp = 0.0f;
 #pragma unroll
           for (int k = 0; k < kAct; ++k) {
             const float ls = fminf(fmaxf(head[kAct + k], M.logstd_min), M.logstd_max);
-            a[k] = fmaf(expf(ls), eps[k], head[k]);
+            a[k] = fmaf(__expf(ls), eps[k], head[k]);
             lp += -0.5f * eps[k] * eps[k] - ls;
           }
           lp -= (float)kAct * 0.91893853320467274f;
@@ -636,12 +656,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         if (active) {
           const uint32_t id = M.id_base + (uint32_t)i;
           float eps[8];
-          action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
+          action_noise_approx(id, M.seed, t_g0 + (uint64_t)t, eps);
           float a[kPA], lp = 0.0f;
 #pragma unroll
           for (int k = 0; k < kPA; ++k) {
             const float ls = fminf(fmaxf(head[kPA + k], M.logstd_min), M.logstd_max);
-            a[k] = fmaf(expf(ls), eps[k], head[k]);
+            a[k] = fmaf(__expf(ls), eps[k], head[k]);
             lp += -0.5f * eps[k] * eps[k] - ls;
           }
           lp -= (float)kPA * 0.91893853320467274f;
