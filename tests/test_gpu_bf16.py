@@ -62,9 +62,11 @@ def test_bf16_value_over_trajectory_layout(oracle):
         assert np.abs(g[t, idx] - ref).max() <= BF16_VALUE_TOL
 
 
-@pytest.mark.parametrize("n,T", [(65536, 128), (1000, 20), (300, 9)])
+@pytest.mark.parametrize("n,T", [(65536, 128), (1048576, 4), (1000, 20), (300, 9)])
 def test_bf16_rollout(oracle, n, T):
-    """The rollout as the benchmark launches it.  Step 0 starts from the
+    """The rollout as the benchmark launches it (65,536 envs x 128 steps; the
+    sweep's largest batch, 1,048,576 envs, several waves of CTAs; ragged
+    small batches).  Step 0 starts from the
     bit-exact reset state: its observation is compared at the fp32 tolerance,
     its action, log-probability and value at the bf16 tolerance.  The episode
     length equals T, so every env ends its episode on the last step and the
