@@ -53,6 +53,8 @@ def parse():
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--replay", action="store_true",
                     help="physics only: action replay (env_step_actions), FP32 roofline")
+    ap.add_argument("--gae", action="store_true",
+                    help="advantage estimation (env_gae) over one rollout, HBM roofline")
     ap.add_argument("--sweep", action="store_true",
                     help="batch-size sweep 1,024 .. 1,048,576 envs x 256 steps (one line per size)")
     return ap.parse_args()
@@ -272,10 +274,72 @@ def run_replay(args):
     print(json.dumps(line), flush=True)
 
 
+def run_gae(args):
+    """Advantage estimation (env_gae) over the workload's trajectory shape,
+    fed by one real rollout: the HBM-bound learner input pass, HBM roofline
+    (17 B per env-step + the bootstrap values)."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {}
+    if args.n_envs:
+        over["n_envs"] = args.n_envs
+    if args.rollout_steps:
+        over["steps"] = args.rollout_steps
+    w = W.workload(args.workload, **over)
+    n, T = int(w["n_envs"]), int(w["steps"])
+    env = auvenv.Env(w)
+    env.set_weights(W.policy_weights(w), W.value_weights(w) if w["has_value"] else None)
+    env.reset()
+    traj = env.alloc_traj(T, keys=("obs", "rew", "done", "value"))
+    env.rollout(T, traj)
+    last = torch.randn(n, device="cuda")
+    adv = torch.empty((T, n), device="cuda")
+    ret = torch.empty((T, n), device="cuda")
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        env.gae(traj["rew"], traj["done"], traj["value"], last, 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0) if not args.no_clocks else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        env.gae(traj["rew"], traj["done"], traj["value"], last, 0.99, 0.95, adv, ret)
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    clock_info = clocks.stop() if clocks else None
+    step_ms = sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+    peaks, src = load_peaks()
+    bytes_ = n * T * 17 + n * 4
+    achieved = bytes_ / (step_ms * 1e-3) / 1e9
+    line = {
+        "metric": "env-steps/s (advantage estimation)", "value": n * T / (step_ms * 1e-3),
+        "unit": "env-steps/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic (one rollout's rewards, dones, values)",
+        "config": {"workload": w["name"], "n_envs_per_gpu": n, "rollout_steps": T,
+                   "gamma": 0.99, "lambda": 0.95, "l2": "flushed between timed steps"},
+        "roofline": {"bound": "hbm", "kernel": "k_gae", "achieved": achieved,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                     "traffic": None, "peak_source": f"HBM copy, {src}"},
+        "gpu_launches": args.steps, "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.replay:
         run_replay(args)
+        return
+    if args.gae:
+        run_gae(args)
         return
     if args.sweep:
         base_steps = args.steps

@@ -342,6 +342,23 @@ int env_policy_forward_noalloc(int hidden, int policy_out, const float* policy,
                                const float* value_w, const float* obs, int n, float* head,
                                float* value, void* stream);
 
+/*
+ * env_gae: generalised advantage estimation over a rollout's trajectory --
+ * the advantage estimator of the PPO learner (paper §III-A; Schulman et al.
+ * 2016).  For t = T-1 .. 0 and every env:
+ *   delta_t = rew_t + gamma (1 - done_t) V_{t+1} - V_t,   V_T = last_value
+ *   adv_t   = delta_t + gamma lambda (1 - done_t) adv_{t+1},  adv_T = 0
+ *   ret_t   = adv_t + V_t   (the value target)
+ * A done step ends its episode: nothing of the next episode flows back.
+ * rew, value, adv, ret: [T][N] fp32; done: [T][N] u8; last_value: [N] (the
+ * value of the observation after the last step, e.g. env_observe then
+ * env_value).  All device memory, 4-byte aligned; adv and ret must not
+ * overlap the inputs.  T >= 1, 0 <= gamma, lambda <= 1.
+ */
+int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const float* value,
+            const float* last_value, float gamma, float lambda, float* adv, float* ret,
+            void* stream);
+
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);

@@ -32,7 +32,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
-            "env_policy_forward_noalloc", "env_layout")
+            "env_policy_forward_noalloc", "env_layout", "env_gae")
 
 
 class LibraryMissing(RuntimeError):
@@ -126,6 +126,7 @@ def lib(path: str | None = None):
     L.env_selftest_wait_timeout.argtypes = [P, C.c_uint32, P]
     L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
     L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
+    L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
@@ -264,6 +265,12 @@ class Env:
         """Value network on trajectory-layout observations obs[T][obs_dim][N] -> value[T][N]."""
         self._check(lib().env_value(self.h, _ptr(obs), int(obs.shape[0]), _ptr(value),
                                     _stream(stream)))
+
+    def gae(self, rew, done, value, last_value, gamma, lam, adv, ret, stream=None):
+        """Generalised advantage estimation over [T][N] trajectory arrays."""
+        self._check(lib().env_gae(self.h, int(rew.shape[0]), _ptr(rew), _ptr(done), _ptr(value),
+                                  _ptr(last_value), float(gamma), float(lam), _ptr(adv),
+                                  _ptr(ret), _stream(stream)))
 
     def step(self, obs=None, rew=None, done=None, stream=None):
         self._check(lib().env_step(self.h, _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))

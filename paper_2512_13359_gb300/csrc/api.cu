@@ -601,6 +601,36 @@ int env_value(auv_env* env, const float* obs, int T, float* value, void* stream)
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "value kernel");
 }
 
+int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const float* value,
+            const float* last_value, float gamma, float lambda, float* adv, float* ret,
+            void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (T < 1) return fail(env, AUV_ERR_INVALID, "T must be >= 1");
+  if (!(gamma >= 0.0f && gamma <= 1.0f) || !(lambda >= 0.0f && lambda <= 1.0f))
+    return fail(env, AUV_ERR_INVALID, "gamma and lambda must lie in [0, 1]");
+  if ((rc = check_device_buffer(env, rew, "rew", 4)) || (rc = check_device_buffer(env, done, "done", 1)) ||
+      (rc = check_device_buffer(env, value, "value", 4)) ||
+      (rc = check_device_buffer(env, last_value, "last_value", 4)) ||
+      (rc = check_device_buffer(env, adv, "adv", 4)) || (rc = check_device_buffer(env, ret, "ret", 4)))
+    return rc;
+  const size_t bytes = (size_t)T * env->model.n * 4;
+  auto overlap = [](const void* a, size_t na, const void* b, size_t nb) {
+    const char *pa = static_cast<const char*>(a), *pb = static_cast<const char*>(b);
+    return pa < pb + nb && pb < pa + na;
+  };
+  const size_t nd = (size_t)T * env->model.n, nl = (size_t)env->model.n * 4;
+  for (const void* out : {static_cast<const void*>(adv), static_cast<const void*>(ret)})
+    if (overlap(out, bytes, rew, bytes) || overlap(out, bytes, value, bytes) ||
+        overlap(out, bytes, done, nd) || overlap(out, bytes, last_value, nl))
+      return fail(env, AUV_ERR_INVALID, "adv and ret must not overlap the inputs");
+  if (overlap(adv, bytes, ret, bytes)) return fail(env, AUV_ERR_INVALID, "adv overlaps ret");
+  cudaError_t e = auv::launch_gae(env->model.n, T, rew, done, value, last_value, gamma, lambda,
+                                  adv, ret, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "gae kernel");
+}
+
 int env_step(auv_env* env, float* obs_out, float* rew_out, uint8_t* done_out, void* stream) {
   auv_traj tr = {obs_out, nullptr, nullptr, nullptr, rew_out, done_out};
   return env_rollout(env, 1, &tr, stream);

@@ -55,4 +55,9 @@ cudaError_t launch_paper_rollout_fp32(const Model& M, const Buffers& B, const fl
                                       const float* wv, const Traj& tr, int T, uint64_t t_g0,
                                       Status* st, cudaStream_t s);
 
+// PPO learner pieces (k_ppo.cu)
+cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, const float* value,
+                       const float* last_value, float gamma, float lam, float* adv, float* ret,
+                       cudaStream_t s);
+
 }  // namespace auv
