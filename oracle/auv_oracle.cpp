@@ -1082,6 +1082,56 @@ void paper_rk4_deriv(const PaperModel& m, const PaperEnv<R>& e, const R y[13], c
   for (int k = 0; k < 6; ++k) dy[7 + k] = acc[k];
 }
 
+
+// ----------------------------------------------------------------------------
+// Minibatch permutation of the PPO learner: a bijection on [0, M) for each
+// epoch, by a balanced four-round Feistel network (Luby & Rackoff 1988) on a
+// domain of 2^b >= M codes (b even, b >= 2), walked until it lands in [0, M)
+// ("cycle walking", Black & Rogaway 2002).  The round function is Philox4x32-10
+// with counter (right half, round, epoch low, epoch high) and key (seed low,
+// seed high); its first word, masked to b/2 bits, is the round value.
+// ----------------------------------------------------------------------------
+int perm_half_bits(uint64_t m) {
+  int b = 2;
+  while ((1ull << b) < m) b += 2;
+  return b / 2;
+}
+
+uint32_t feistel_encode(uint32_t x, int h, uint64_t seed, uint64_t epoch) {
+  const uint32_t mask = (h >= 32) ? 0xFFFFFFFFu : ((1u << h) - 1u);
+  uint32_t left = x >> h, right = x & mask;
+  for (uint32_t r = 0; r < 4; ++r) {
+    const uint32_t ctr[4] = {right, r, (uint32_t)epoch, (uint32_t)(epoch >> 32)};
+    uint32_t out[4];
+    philox4x32_10(ctr, (uint32_t)seed, (uint32_t)(seed >> 32), out);
+    const uint32_t next_right = left ^ (out[0] & mask);
+    left = right;
+    right = next_right;
+  }
+  return (left << h) | right;
+}
+
+uint32_t feistel_decode(uint32_t y, int h, uint64_t seed, uint64_t epoch) {
+  const uint32_t mask = (h >= 32) ? 0xFFFFFFFFu : ((1u << h) - 1u);
+  uint32_t left = y >> h, right = y & mask;
+  for (int r = 3; r >= 0; --r) {
+    // undo (L, R) -> (R, L ^ F_r(R)): the old right half is the new left
+    const uint32_t ctr[4] = {left, (uint32_t)r, (uint32_t)epoch, (uint32_t)(epoch >> 32)};
+    uint32_t out[4];
+    philox4x32_10(ctr, (uint32_t)seed, (uint32_t)(seed >> 32), out);
+    const uint32_t old_left = right ^ (out[0] & mask);
+    right = left;
+    left = old_left;
+  }
+  return (left << h) | right;
+}
+
+uint32_t minibatch_index(uint32_t j, uint32_t m, uint64_t seed, uint64_t epoch) {
+  const int h = perm_half_bits(m);
+  uint32_t x = feistel_encode(j, h, seed, epoch);
+  while (x >= m) x = feistel_encode(x, h, seed, epoch);
+  return x;
+}
 }  // namespace
 
 extern "C" {
@@ -1091,6 +1141,18 @@ int oracle_model_size() { return (int)sizeof(OracleModel); }
 
 void oracle_philox(uint32_t key0, uint32_t key1, const uint32_t* ctr, uint32_t* out) {
   philox4x32_10(ctr, key0, key1, out);
+}
+
+// Positions start .. start+count-1 of epoch `epoch`'s permutation of [0, m).
+void oracle_minibatch_perm(uint64_t seed, uint64_t epoch, uint32_t m, uint32_t start,
+                           uint32_t count, uint32_t* out) {
+  for (uint32_t k = 0; k < count; ++k) out[k] = minibatch_index(start + k, m, seed, epoch);
+}
+
+// One Feistel pass (no cycle walking) forward or back, for the pins.
+uint32_t oracle_feistel(uint32_t x, uint32_t m, uint64_t seed, uint64_t epoch, int inverse) {
+  const int h = perm_half_bits(m);
+  return inverse ? feistel_decode(x, h, seed, epoch) : feistel_encode(x, h, seed, epoch);
 }
 
 float oracle_word_to_uniform(uint32_t x) { return word_to_uniform(x); }

@@ -56,6 +56,10 @@ def lib():
         P = C.c_void_p
         _lib.oracle_model_size.restype = C.c_int
         _lib.oracle_philox.argtypes = [C.c_uint32, C.c_uint32, P, P]
+        _lib.oracle_minibatch_perm.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32,
+                                               C.c_uint32, P]
+        _lib.oracle_feistel.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.c_uint64, C.c_int]
+        _lib.oracle_feistel.restype = C.c_uint32
         _lib.oracle_word_to_uniform.argtypes = [C.c_uint32]
         _lib.oracle_word_to_uniform.restype = C.c_float
         _lib.oracle_taylor_sin.argtypes = [C.c_float]
@@ -196,6 +200,17 @@ def philox(key0: int, key1: int, ctr) -> np.ndarray:
     out = np.zeros(4, dtype=np.uint32)
     lib().oracle_philox(key0 & 0xFFFFFFFF, key1 & 0xFFFFFFFF, _p(c), _p(out))
     return out
+
+
+def minibatch_perm(seed: int, epoch: int, m: int, start: int, count: int) -> np.ndarray:
+    """Positions start .. start+count-1 of the learner's epoch permutation of [0, m)."""
+    out = np.zeros(count, dtype=np.uint32)
+    lib().oracle_minibatch_perm(seed, epoch, m, start, count, _p(out))
+    return out
+
+
+def feistel(x: int, m: int, seed: int, epoch: int, inverse: bool = False) -> int:
+    return int(lib().oracle_feistel(x, m, seed, epoch, 1 if inverse else 0))
 
 
 def normals(env_id: int, seed: int, t_g: int) -> np.ndarray:
