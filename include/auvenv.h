@@ -359,6 +359,136 @@ int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const fl
             const float* last_value, float gamma, float lambda, float* adv, float* ret,
             void* stream);
 
+/* ---------------------------------------------------------------------------
+ * PPO learner (paper §III-A: PPO with its clipped surrogate objective,
+ * Schulman et al. 2017) -- the update that consumes the rollout's trajectory.
+ *
+ * The learner owns fp32 master weights of the two networks the rollout runs
+ * (policy obs -> H -> H -> 2A: mean and log-std; value obs -> H -> H -> 1;
+ * tanh hidden layers), their Adam moments and its counters.  One gradient
+ * step on a minibatch of B samples computes, in float arithmetic:
+ *   mu, ls = policy head (ls clamped to [logstd_min, logstd_max])
+ *   logp   = sum_k -((a_k - mu_k) / e^ls_k)^2 / 2 - ls_k - log(2 pi) / 2
+ *   r      = exp(logp - logp_old)
+ *   A_n    = (adv - mean adv) / (std adv + 1e-8) over the minibatch (std with
+ *            B - 1 in the denominator; norm_adv = 0 uses adv as is)
+ *   L      = mean max(-A_n r, -A_n clip(r, 1 - clip_eps, 1 + clip_eps))
+ *          + vf_coef mean (V - ret)^2 / 2
+ *          - ent_coef mean sum_k (ls_k + (1 + log 2 pi) / 2)
+ * then the gradient of L (no gradient through an active log-std clamp),
+ * scaled to 2-norm max_grad_norm when larger (max_grad_norm <= 0: never),
+ * and one Adam step with bias correction:
+ *   m = b1 m + (1 - b1) g;  v = b2 v + (1 - b2) g^2
+ *   w -= lr (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) + adam_eps).
+ * The two networks form one parameter vector for the norm and for Adam.
+ *
+ * Minibatches: epoch e permutes the M = T * N trajectory rows (row
+ * r = t * N + i) by a four-round Feistel network on 2^b >= M codes (b even)
+ * with cycle walking; round j maps (L, R) -> (R, L ^ F_j(R)) with F_j(R) the
+ * first word of Philox4x32-10 at counter (R, j, e low, e high) and key (seed
+ * low, seed high), masked to b/2 bits.  Minibatch j of epoch e takes the rows
+ * at permutation positions j*B .. j*B + B - 1.
+ *
+ * Weight, gradient and moment vectors crossing this interface use the
+ * env_set_weights layout of each network, [W1 | b1 | W2 | b2 | W3 | b3]
+ * with W row-major [out][in]; a "parameter vector" is the policy's followed
+ * by the value network's (ppo_param_counts gives the two lengths).
+ * --------------------------------------------------------------------------- */
+#define AUV_PPO_FP32 0u   /* GEMMs on the CUDA cores in fp32                     */
+#define AUV_PPO_TF32 1u   /* GEMMs on the tensor cores, tf32 operands, fp32 sums */
+#define AUV_PPO_BF16 2u   /* GEMMs on the tensor cores, bf16 operands, fp32 sums */
+#define AUV_PPO_STATS 8   /* floats in a statistics record:                       */
+/* [0] surrogate (policy) loss, [1] value loss (mean (V - ret)^2 / 2),
+ * [2] entropy, [3] approx. KL mean(logp_old - logp), [4] clip fraction
+ * mean(|r - 1| > clip_eps), [5] gradient norm before clipping, [6] total loss
+ * L, [7] gradient steps the record covers.  ppo_update averages [0..6] over
+ * its steps. */
+
+typedef struct auv_ppo_config {
+  uint32_t struct_size;   /* sizeof(auv_ppo_config)                          */
+  uint32_t obs_dim;       /* network input width, 1 .. 64 (18 Fossen, 12 paper) */
+  uint32_t act_dim;       /* A, 1 .. 8: the policy head is 2A wide            */
+  uint32_t hidden;        /* H, a multiple of 8 in [8, 1024]                   */
+  uint32_t minibatch;     /* B samples per gradient step, 2 .. 2^22            */
+  uint32_t precision;     /* AUV_PPO_FP32 | AUV_PPO_TF32 | AUV_PPO_BF16        */
+  uint32_t norm_adv;      /* 1: normalise advantages per minibatch, 0: not     */
+  uint32_t reserved;      /* 0                                                 */
+  uint64_t seed;          /* key of the minibatch permutations                 */
+  float clip_eps;         /* > 0                                               */
+  float vf_coef, ent_coef;            /* finite                                */
+  float max_grad_norm;                /* <= 0: no clipping                     */
+  float lr, adam_beta1, adam_beta2, adam_eps;   /* lr >= 0, betas in [0, 1), eps > 0 */
+  float logstd_min, logstd_max;       /* the rollout's log-std clamp           */
+} auv_ppo_config;
+
+/* The trajectory a PPO update reads: the rollout's arrays (env_rollout with
+ * obs, act and logp) and env_gae's advantages and returns.  Device memory,
+ * 4-byte aligned, fp32.  obs [T][obs_dim][N], act [T][act_dim][N], logp, adv,
+ * ret [T][N].  T, N >= 1 and T * N <= 2^31. */
+typedef struct auv_ppo_batch {
+  const float* obs;
+  const float* act;
+  const float* logp;
+  const float* adv;
+  const float* ret;
+  uint32_t T, N;
+} auv_ppo_batch;
+
+typedef struct auv_ppo auv_ppo;
+
+/* Create a learner on the current device: weights zero (call ppo_set_weights),
+ * Adam moments zero, t = 0, epoch = 0.  AUV_ERR_INVALID on a bad config. */
+int ppo_create(const auv_ppo_config* cfg, auv_ppo** out);
+int ppo_destroy(auv_ppo* p);
+const char* ppo_last_error(const auv_ppo* p);
+int ppo_param_counts(const auv_ppo* p, uint64_t* n_policy, uint64_t* n_value);
+
+/* Load both networks (device or host memory, env_set_weights layout) and
+ * reset the Adam moments, t and epoch to 0.  Synchronises `stream`. */
+int ppo_set_weights(auv_ppo* p, const float* policy, const float* value, void* stream);
+/* Copy both networks out (device or host memory); synchronises `stream`. */
+int ppo_get_weights(auv_ppo* p, float* policy, float* value, void* stream);
+
+/* Adam state for checkpoints: moments m, v as parameter vectors (device or
+ * host memory), the step count t and the next epoch number.  get
+ * synchronises `stream`; set does too. */
+int ppo_get_state(auv_ppo* p, float* m, float* v, uint64_t* t, uint64_t* epoch, void* stream);
+int ppo_set_state(auv_ppo* p, const float* m, const float* v, uint64_t t, uint64_t epoch,
+                  void* stream);
+
+/*
+ * ppo_grads: the gradient of L on minibatch `minibatch` of epoch `epoch`
+ * (needs (minibatch + 1) * B <= T * N).  The gradient stays in the learner for
+ * ppo_apply; if grad is not NULL it is also written there as a parameter
+ * vector (device memory, 4-byte aligned), e.g. to be averaged over ranks
+ * before ppo_apply.  If stats is not NULL (device memory, AUV_PPO_STATS
+ * floats) the minibatch's record is written there ([5] = 0, [7] = 1).
+ * Asynchronous on `stream`.
+ */
+int ppo_grads(auv_ppo* p, const auv_ppo_batch* batch, uint64_t epoch, uint32_t minibatch,
+              float* grad, float* stats, void* stream);
+
+/* ppo_apply: clip and take one Adam step (t += 1) with the learner's last
+ * gradient (grad NULL) or with the parameter vector grad (device memory).
+ * stats, if not NULL, receives the gradient norm in [5] (others untouched). */
+int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream);
+
+/*
+ * ppo_update: `epochs` passes over the batch, each of n_minibatches gradient
+ * steps (minibatch j of epoch p->epoch, then p->epoch += 1), i.e. the whole
+ * PPO update of one rollout; needs n_minibatches * B <= T * N.  stats, if not
+ * NULL, receives the record averaged over the steps.  Asynchronous on
+ * `stream`; the weights (ppo_get_weights, or the pointers of ppo_weights) are
+ * the updated ones once it completes.
+ */
+int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t n_minibatches,
+               float* stats, void* stream);
+
+/* ppo_export_weights: write both networks, in the env_set_weights layout,
+ * to device memory (asynchronous on `stream`) -- e.g. straight into the
+ * buffers an env_set_weights call then reads. */
+int ppo_export_weights(auv_ppo* p, float* policy, float* value, void* stream);
+
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);

@@ -27,12 +27,22 @@ AUV_MLP_FP32 = 0
 AUV_MLP_BF16 = 1
 AUV_MODEL_FOSSEN = 0
 AUV_MODEL_PAPER = 1
+AUV_PPO_FP32 = 0
+AUV_PPO_TF32 = 1
+AUV_PPO_BF16 = 2
+AUV_PPO_STATS = 8
+PPO_PRECISION = {"fp32": AUV_PPO_FP32, "tf32": AUV_PPO_TF32, "bf16": AUV_PPO_BF16}
+PPO_STAT_NAMES = ("pg_loss", "v_loss", "entropy", "approx_kl", "clip_frac", "grad_norm", "loss",
+                  "steps")
 
 EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
-            "env_policy_forward_noalloc", "env_layout", "env_gae")
+            "env_policy_forward_noalloc", "env_layout", "env_gae",
+            "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
+            "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
+            "ppo_update", "ppo_export_weights")
 
 
 class LibraryMissing(RuntimeError):
@@ -84,6 +94,22 @@ class AuvTraj(C.Structure):
                 ("value", C.c_void_p), ("rew", C.c_void_p), ("done", C.c_void_p)]
 
 
+class PpoConfig(C.Structure):
+    _fields_ = [
+        ("struct_size", C.c_uint32), ("obs_dim", C.c_uint32), ("act_dim", C.c_uint32),
+        ("hidden", C.c_uint32), ("minibatch", C.c_uint32), ("precision", C.c_uint32),
+        ("norm_adv", C.c_uint32), ("reserved", C.c_uint32), ("seed", C.c_uint64),
+        ("clip_eps", C.c_float), ("vf_coef", C.c_float), ("ent_coef", C.c_float),
+        ("max_grad_norm", C.c_float), ("lr", C.c_float), ("adam_beta1", C.c_float),
+        ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("logstd_min", C.c_float),
+        ("logstd_max", C.c_float)]
+
+
+class PpoBatch(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("act", C.c_void_p), ("logp", C.c_void_p),
+                ("adv", C.c_void_p), ("ret", C.c_void_p), ("T", C.c_uint32), ("N", C.c_uint32)]
+
+
 class AuvStatus(C.Structure):
     _fields_ = [("code", C.c_int32), ("nan_flag", C.c_int32), ("first_nan_env", C.c_int32),
                 ("timeouts", C.c_int32)]
@@ -127,9 +153,24 @@ def lib(path: str | None = None):
     L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
     L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
+    U64, U32 = C.c_uint64, C.c_uint32
+    L.ppo_create.argtypes = [C.POINTER(PpoConfig), C.POINTER(P)]
+    L.ppo_destroy.argtypes = [P]
+    L.ppo_last_error.argtypes = [P]
+    L.ppo_last_error.restype = C.c_char_p
+    L.ppo_param_counts.argtypes = [P, C.POINTER(U64), C.POINTER(U64)]
+    L.ppo_set_weights.argtypes = [P, P, P, P]
+    L.ppo_get_weights.argtypes = [P, P, P, P]
+    L.ppo_export_weights.argtypes = [P, P, P, P]
+    L.ppo_get_state.argtypes = [P, P, P, C.POINTER(U64), C.POINTER(U64), P]
+    L.ppo_set_state.argtypes = [P, P, P, U64, U64, P]
+    L.ppo_grads.argtypes = [P, C.POINTER(PpoBatch), U64, U32, P, P, P]
+    L.ppo_apply.argtypes = [P, P, P, P]
+    L.ppo_update.argtypes = [P, C.POINTER(PpoBatch), U32, U32, P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
+    L.ppo_last_error.restype = C.c_char_p
     _lib = L
     return L
 
@@ -329,3 +370,116 @@ class Env:
             else:
                 out[k] = torch.empty(shapes[k], dtype=dt, device=self.device)
         return out
+
+
+PPO_DEFAULTS = dict(clip_eps=0.2, vf_coef=0.5, ent_coef=0.0, max_grad_norm=0.5, lr=3e-4,
+                    adam_beta1=0.9, adam_beta2=0.999, adam_eps=1e-8, logstd_min=-5.0,
+                    logstd_max=2.0, norm_adv=True)
+
+
+def make_ppo_config(obs_dim: int, act_dim: int, hidden: int, minibatch: int,
+                    precision: str = "fp32", seed: int = 0, **hp) -> PpoConfig:
+    h = dict(PPO_DEFAULTS, **hp)
+    c = PpoConfig()
+    c.struct_size = C.sizeof(PpoConfig)
+    c.obs_dim, c.act_dim, c.hidden, c.minibatch = obs_dim, act_dim, hidden, minibatch
+    c.precision = PPO_PRECISION[precision] if isinstance(precision, str) else int(precision)
+    c.norm_adv = 1 if h.pop("norm_adv") else 0
+    c.seed = seed
+    for k, v in h.items():
+        setattr(c, k, float(v))
+    return c
+
+
+class Learner:
+    """PPO learner (include/auvenv.h, ppo_*) on the current CUDA device.
+
+    Trajectory arguments are dicts of CUDA tensors in the rollout's layout:
+    obs [T][obs_dim][N], act [T][act_dim][N], logp, adv, ret [T][N]."""
+
+    def __init__(self, obs_dim: int, act_dim: int, hidden: int, minibatch: int,
+                 precision: str = "fp32", seed: int = 0, **hp):
+        import torch
+        self.cfg = make_ppo_config(obs_dim, act_dim, hidden, minibatch, precision, seed, **hp)
+        self.device = torch.device("cuda", torch.cuda.current_device())
+        L = lib()
+        h = C.c_void_p()
+        rc = L.ppo_create(C.byref(self.cfg), C.byref(h))
+        if rc != AUV_OK:
+            raise AuvError(rc, L.ppo_last_error(None).decode())
+        self.h = h
+        a, b = C.c_uint64(), C.c_uint64()
+        self._check(L.ppo_param_counts(h, C.byref(a), C.byref(b)))
+        self.n_policy, self.n_value = a.value, b.value
+
+    def _check(self, rc):
+        if rc != AUV_OK:
+            raise AuvError(rc, lib().ppo_last_error(self.h).decode())
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().ppo_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @staticmethod
+    def _batch(traj):
+        T, N = traj["logp"].shape
+        for k in ("obs", "act", "logp", "adv", "ret"):
+            if not traj[k].is_contiguous():
+                raise ValueError(f"{k} must be contiguous")
+        return PpoBatch(traj["obs"].data_ptr(), traj["act"].data_ptr(), traj["logp"].data_ptr(),
+                        traj["adv"].data_ptr(), traj["ret"].data_ptr(), T, N)
+
+    def set_weights(self, policy, value, stream=None):
+        p = np.ascontiguousarray(policy, dtype=np.float32)
+        v = np.ascontiguousarray(value, dtype=np.float32)
+        if p.size != self.n_policy or v.size != self.n_value:
+            raise ValueError("weight vector lengths do not match the networks")
+        self._check(lib().ppo_set_weights(self.h, p.ctypes.data_as(C.c_void_p),
+                                          v.ctypes.data_as(C.c_void_p), _stream(stream)))
+
+    def get_weights(self, stream=None):
+        p = np.empty(self.n_policy, dtype=np.float32)
+        v = np.empty(self.n_value, dtype=np.float32)
+        self._check(lib().ppo_get_weights(self.h, p.ctypes.data_as(C.c_void_p),
+                                          v.ctypes.data_as(C.c_void_p), _stream(stream)))
+        return p, v
+
+    def export_weights(self, policy, value, stream=None):
+        self._check(lib().ppo_export_weights(self.h, _ptr(policy), _ptr(value), _stream(stream)))
+
+    def get_state(self, stream=None):
+        n = self.n_policy + self.n_value
+        m = np.empty(n, dtype=np.float32)
+        v = np.empty(n, dtype=np.float32)
+        t, e = C.c_uint64(), C.c_uint64()
+        self._check(lib().ppo_get_state(self.h, m.ctypes.data_as(C.c_void_p),
+                                        v.ctypes.data_as(C.c_void_p), C.byref(t), C.byref(e),
+                                        _stream(stream)))
+        return dict(m=m, v=v, t=t.value, epoch=e.value)
+
+    def set_state(self, state, stream=None):
+        m = np.ascontiguousarray(state["m"], dtype=np.float32)
+        v = np.ascontiguousarray(state["v"], dtype=np.float32)
+        self._check(lib().ppo_set_state(self.h, m.ctypes.data_as(C.c_void_p),
+                                        v.ctypes.data_as(C.c_void_p), int(state["t"]),
+                                        int(state["epoch"]), _stream(stream)))
+
+    def grads(self, traj, epoch: int, minibatch: int, grad=None, stats=None, stream=None):
+        b = self._batch(traj)
+        self._check(lib().ppo_grads(self.h, C.byref(b), epoch, minibatch, _ptr(grad), _ptr(stats),
+                                    _stream(stream)))
+
+    def apply(self, grad=None, stats=None, stream=None):
+        self._check(lib().ppo_apply(self.h, _ptr(grad), _ptr(stats), _stream(stream)))
+
+    def update(self, traj, epochs: int, n_minibatches: int, stats=None, stream=None):
+        b = self._batch(traj)
+        self._check(lib().ppo_update(self.h, C.byref(b), epochs, n_minibatches, _ptr(stats),
+                                     _stream(stream)))

@@ -60,4 +60,66 @@ cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, cons
                        const float* last_value, float gamma, float lam, float* adv, float* ret,
                        cudaStream_t s);
 
+namespace ppo {
+
+// Shapes of one learner.  Each network is held "augmented": every layer's
+// input row carries a constant 1 after its features (then zeros up to a
+// multiple of 4 floats), and the layer's bias is the weight column that
+// meets it, so that a GEMM adds the bias and the weight-gradient GEMM yields
+// its gradient.  W1a [H][Dp], W2a [H][Hp], W3a [out][Hp].
+struct Dims {
+  int D, Dp;     // observation width and its padded, augmented row (>= D + 1)
+  int A;         // action width; policy head 2A
+  int H, Hp;     // hidden width and its augmented row (>= H + 1)
+  int B;         // minibatch
+};
+
+struct PermKey {        // Feistel permutation of [0, m) for one epoch
+  uint32_t m, mask;
+  int h;                // half width in bits
+  uint32_t k0, k1, e0, e1;
+};
+
+struct LossHp {
+  float clip_eps, vf_coef, ent_coef, logstd_min, logstd_max;
+  int norm_adv;
+};
+
+struct AdamHp {
+  float lr, b1, b2, eps, c1, c2;   // c1 = 1 - b1^t, c2 = 1 - b2^t
+  float max_norm;
+};
+
+struct Sample {                    // gathered minibatch, sample-major
+  float* X;                        // [B][Dp] (1 at column D)
+  float* act;                      // [B][A]
+  float* logp;                     // [B]
+  float* adv;                      // [B]
+  float* ret;                      // [B]
+  double* adv_part;                // [ceil(B/256)][2]: sums of adv and adv^2
+};
+
+constexpr int kNormBlocks = 256;   // blocks of the gradient-norm reduction
+
+size_t aug_count(int in, int in_p, int H, int Hp, int out);
+cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
+                          const float* act, const float* logp, const float* adv,
+                          const float* ret, uint32_t N, const Sample& out, cudaStream_t s);
+cudaError_t launch_tanh_fwd(float* h, int ld, int B, int H, cudaStream_t s);
+cudaError_t launch_tanh_bwd(float* g, int ldg, const float* h, int ldh, int B, int H,
+                            cudaStream_t s);
+cudaError_t launch_head(const Dims& d, const LossHp& hp, const float* y, const float* v,
+                        const Sample& smp, float* g_y, float* g_v, float* part, cudaStream_t s);
+cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, float* mb,
+                         float* acc, cudaStream_t s);
+cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
+                        const AdamHp& hp, float* mb, float* acc, cudaStream_t s);
+cudaError_t launch_finish(const float* acc, float* out, cudaStream_t s);
+// flat [W1|b1|W2|b2|W3|b3] <-> augmented [W1a|W2a|W3a] of one network
+cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int Hp, int out,
+                           bool to_aug, cudaStream_t s);
+cudaError_t launch_fill_ones(float* buf, int ld, int col, int rows, cudaStream_t s);
+
+}  // namespace ppo
+
 }  // namespace auv

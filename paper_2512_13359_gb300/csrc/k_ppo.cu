@@ -67,3 +67,377 @@ cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, cons
 }
 
 }  // namespace auv
+
+// ---------------------------------------------------------------------------
+// PPO minibatch update (Schulman et al. 2017).  The GEMMs of the two MLPs run
+// in cuBLAS (the host side); these kernels do everything around them: the
+// epoch permutation and minibatch gather, tanh forward and backward, the
+// per-sample loss and its gradient at the heads, the minibatch statistics,
+// the global gradient norm and Adam, and the weight-layout conversion.
+// ---------------------------------------------------------------------------
+namespace auv {
+namespace ppo {
+
+namespace {
+
+constexpr int kT = 256;
+constexpr float kHalfLog2Pi = 0.91893853320467274f;
+
+// Balanced Feistel network, four rounds; round j: (L, R) -> (R, L ^ F_j(R)),
+// F_j(R) = first Philox4x32-10 word at counter (R, j, epoch) and key seed.
+__device__ __forceinline__ uint32_t feistel(uint32_t x, const PermKey& p) {
+  uint32_t left = x >> p.h, right = x & p.mask;
+#pragma unroll 1
+  for (uint32_t j = 0; j < 4; ++j) {
+    const uint4 o = philox10(right, j, p.e0, p.e1, p.k0, p.k1);
+    const uint32_t next = left ^ (o.x & p.mask);
+    left = right;
+    right = next;
+  }
+  return (left << p.h) | right;
+}
+
+// Position j of the epoch's permutation of [0, m): cycle-walk the network
+// until it lands inside (it returns to j at the latest, so this ends).
+__device__ __forceinline__ uint32_t perm_index(uint32_t j, const PermKey& p) {
+  uint32_t x = feistel(j, p);
+  while (x >= p.m) x = feistel(x, p);
+  return x;
+}
+
+// Sum NV values over the block (blockDim.x = kT); the result is in thread 0.
+template <int NV, typename V>
+__device__ __forceinline__ void block_sum(V (&v)[NV], V* sh /* [NV][kT/32] */) {
+#pragma unroll
+  for (int k = 0; k < NV; ++k)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_down_sync(0xFFFFFFFFu, v[k], o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0)
+#pragma unroll
+    for (int k = 0; k < NV; ++k) sh[k * (kT / 32) + w] = v[k];
+  __syncthreads();
+  if (w == 0) {
+#pragma unroll
+    for (int k = 0; k < NV; ++k) {
+      v[k] = l < kT / 32 ? sh[k * (kT / 32) + l] : V(0);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_down_sync(0xFFFFFFFFu, v[k], o);
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, uint32_t start,
+                                               const float* __restrict__ obs,
+                                               const float* __restrict__ act,
+                                               const float* __restrict__ logp,
+                                               const float* __restrict__ adv,
+                                               const float* __restrict__ ret, uint32_t N,
+                                               Sample out) {
+  __shared__ double sh[2 * (kT / 32)];
+  const int b = blockIdx.x * kT + threadIdx.x;
+  double s[2] = {0.0, 0.0};
+  if (b < d.B) {
+    const uint32_t r = perm_index(start + (uint32_t)b, key);
+    const size_t t = r / N, i = r - (uint32_t)t * N, n = N;
+    float* x = out.X + (size_t)b * d.Dp;
+    for (int k = 0; k < d.D; ++k) x[k] = __ldg(obs + (t * d.D + k) * n + i);
+    x[d.D] = 1.0f;
+    for (int k = d.D + 1; k < d.Dp; ++k) x[k] = 0.0f;
+    for (int k = 0; k < d.A; ++k) out.act[(size_t)b * d.A + k] = __ldg(act + (t * d.A + k) * n + i);
+    const size_t o = t * n + i;
+    const float a = __ldg(adv + o);
+    out.logp[b] = __ldg(logp + o);
+    out.adv[b] = a;
+    out.ret[b] = __ldg(ret + o);
+    s[0] = a;
+    s[1] = (double)a * a;
+  }
+  block_sum<2>(s, sh);
+  if (threadIdx.x == 0) {
+    out.adv_part[2 * blockIdx.x] = s[0];
+    out.adv_part[2 * blockIdx.x + 1] = s[1];
+  }
+}
+
+__global__ void __launch_bounds__(kT) k_tanh_fwd(float* __restrict__ h, int ld, int B, int H4) {
+  const size_t n = (size_t)B * H4;
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const size_t row = e / H4, c = e - row * H4;
+    float4* p = reinterpret_cast<float4*>(h + row * ld) + c;
+    float4 z = *p;
+    z.x = tanhf(z.x); z.y = tanhf(z.y); z.z = tanhf(z.z); z.w = tanhf(z.w);
+    *p = z;
+  }
+}
+
+__global__ void __launch_bounds__(kT) k_tanh_bwd(float* __restrict__ g, int ldg,
+                                                 const float* __restrict__ h, int ldh, int B,
+                                                 int H4) {
+  const size_t n = (size_t)B * H4;
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const size_t row = e / H4, c = e - row * H4;
+    float4* pg = reinterpret_cast<float4*>(g + row * ldg) + c;
+    const float4 y = __ldg(reinterpret_cast<const float4*>(h + row * ldh) + c);
+    float4 v = *pg;
+    v.x *= 1.0f - y.x * y.x; v.y *= 1.0f - y.y * y.y;
+    v.z *= 1.0f - y.z * y.z; v.w *= 1.0f - y.w * y.w;
+    *pg = v;
+  }
+}
+
+// One thread per sample: log-density, ratio, clipped surrogate, value and
+// entropy terms, and dL/d(head) for both networks (already divided by B).
+// Every block first reduces the gather's advantage partial sums, in the same
+// order, so that all blocks normalise with the same mean and deviation.
+__global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __restrict__ y,
+                                             const float* __restrict__ v, Sample smp,
+                                             int n_part, float* __restrict__ g_y,
+                                             float* __restrict__ g_v, float* __restrict__ part) {
+  __shared__ double shd[2 * (kT / 32)];
+  __shared__ float shf[5 * (kT / 32)];
+  __shared__ double norm[2];
+  double s[2] = {0.0, 0.0};
+  for (int k = threadIdx.x; k < n_part; k += kT) {
+    s[0] += smp.adv_part[2 * k];
+    s[1] += smp.adv_part[2 * k + 1];
+  }
+  block_sum<2>(s, shd);
+  if (threadIdx.x == 0) {
+    const double mean = s[0] / d.B;
+    const double var = fmax((s[1] - s[0] * mean) / (d.B - 1), 0.0);
+    norm[0] = mean;
+    norm[1] = 1.0 / (sqrt(var) + 1e-8);
+  }
+  __syncthreads();
+  const int b = blockIdx.x * kT + threadIdx.x;
+  float st[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+  if (b < d.B) {
+    const float inv_b = 1.0f / (float)d.B;
+    const int A = d.A;
+    const float* yb = y + (size_t)b * 2 * A;
+    const float* ab = smp.act + (size_t)b * A;
+    const float an = hp.norm_adv ? (float)(((double)smp.adv[b] - norm[0]) * norm[1]) : smp.adv[b];
+    float dm[8], iv[8], z2[8];
+    bool in[8];
+    float lp = -(float)A * kHalfLog2Pi, ent = (float)A * (0.5f + kHalfLog2Pi);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (k < A) {
+        const float raw = yb[A + k];
+        const float ls = fminf(fmaxf(raw, hp.logstd_min), hp.logstd_max);
+        in[k] = raw >= hp.logstd_min && raw <= hp.logstd_max;
+        iv[k] = expf(-2.0f * ls);
+        dm[k] = ab[k] - yb[k];
+        z2[k] = dm[k] * dm[k] * iv[k];
+        lp += -0.5f * z2[k] - ls;
+        ent += ls;
+      }
+    }
+    const float lp_old = smp.logp[b];
+    const float r = expf(lp - lp_old);
+    const float lo = 1.0f - hp.clip_eps, hi = 1.0f + hp.clip_eps;
+    const bool unclipped = an > 0.0f ? r <= hi : r >= lo;
+    const float g_lp = unclipped ? -an * r * inv_b : 0.0f;
+    float* gy = g_y + (size_t)b * 2 * A;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (k < A) {
+        gy[k] = g_lp * dm[k] * iv[k];
+        gy[A + k] = in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f;
+      }
+    }
+    const float dv = v[b] - smp.ret[b];
+    g_v[b] = hp.vf_coef * dv * inv_b;
+    st[0] = fmaxf(-an * r, -an * fminf(fmaxf(r, lo), hi));
+    st[1] = 0.5f * dv * dv;
+    st[2] = ent;
+    st[3] = lp_old - lp;
+    st[4] = fabsf(r - 1.0f) > hp.clip_eps ? 1.0f : 0.0f;
+  }
+  block_sum<5>(st, shf);
+  if (threadIdx.x == 0)
+    for (int k = 0; k < 5; ++k) part[5 * blockIdx.x + k] = st[k];
+}
+
+__global__ void __launch_bounds__(kT) k_stats(int B, int n_part, float vf_coef, float ent_coef,
+                                              const float* __restrict__ part, float* mb,
+                                              float* acc) {
+  __shared__ double sh[5 * (kT / 32)];
+  double s[5] = {0, 0, 0, 0, 0};
+  for (int k = threadIdx.x; k < n_part; k += kT)
+    for (int j = 0; j < 5; ++j) s[j] += part[5 * k + j];
+  block_sum<5>(s, sh);
+  if (threadIdx.x == 0) {
+    float r[8];
+    for (int j = 0; j < 5; ++j) r[j] = (float)(s[j] / B);
+    r[5] = 0.0f;
+    r[6] = r[0] + vf_coef * r[1] - ent_coef * r[2];
+    r[7] = 1.0f;
+    for (int j = 0; j < 8; ++j) mb[j] = r[j];
+    if (acc)
+      for (int j = 0; j < 8; ++j)
+        if (j != 5) acc[j] += r[j];
+  }
+}
+
+__global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_t n,
+                                              float* __restrict__ part) {
+  __shared__ double sh[kT / 32];
+  double s[1] = {0.0};
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const float x = g[e];
+    s[0] += (double)x * x;
+  }
+  block_sum<1>(s, sh);
+  if (threadIdx.x == 0) part[blockIdx.x] = (float)s[0];
+}
+
+// Clip by the global norm (every block reduces the same partials in the
+// same order) and take one Adam step.
+__global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float* __restrict__ g,
+                                             float* __restrict__ m, float* __restrict__ v,
+                                             size_t n, const float* __restrict__ part, AdamHp hp,
+                                             float* mb, float* acc) {
+  __shared__ double sh[kT / 32];
+  __shared__ float scale_sh;
+  double s[1] = {0.0};
+  for (int k = threadIdx.x; k < kNormBlocks; k += kT) s[0] += part[k];
+  block_sum<1>(s, sh);
+  if (threadIdx.x == 0) {
+    const double norm = sqrt(s[0]);
+    scale_sh = hp.max_norm > 0.0f ? (float)fmin(1.0, hp.max_norm / (norm + 1e-6)) : 1.0f;
+    if (blockIdx.x == 0) {
+      mb[5] = (float)norm;
+      if (acc) acc[5] += (float)norm;
+    }
+  }
+  __syncthreads();
+  const float scale = scale_sh;
+  const float ib1 = 1.0f - hp.b1, ib2 = 1.0f - hp.b2;
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const float gi = g[e] * scale;
+    const float mi = hp.b1 * m[e] + ib1 * gi;
+    const float vi = hp.b2 * v[e] + ib2 * gi * gi;
+    m[e] = mi;
+    v[e] = vi;
+    w[e] -= hp.lr * (mi / hp.c1) / (sqrtf(vi / hp.c2) + hp.eps);
+  }
+}
+
+__global__ void k_finish(const float* __restrict__ acc, float* __restrict__ out) {
+  const int j = threadIdx.x;
+  if (j < 8) {
+    const float steps = acc[7];
+    out[j] = j == 7 ? steps : acc[j] / steps;
+  }
+}
+
+// Flat index of augmented element e (-1 for a padding element).
+__device__ __forceinline__ long long flat_index(size_t e, int in, int in_p, int H, int Hp,
+                                                int out) {
+  const size_t n1 = (size_t)H * in_p, n2 = (size_t)H * Hp;
+  const long long b1 = (long long)H * in, w2 = b1 + H, b2 = w2 + (long long)H * H,
+                  w3 = b2 + H, b3 = w3 + (long long)out * H;
+  if (e < n1) {
+    const int row = (int)(e / in_p), col = (int)(e - (size_t)row * in_p);
+    return col < in ? (long long)row * in + col : col == in ? b1 + row : -1;
+  }
+  e -= n1;
+  if (e < n2) {
+    const int row = (int)(e / Hp), col = (int)(e - (size_t)row * Hp);
+    return col < H ? w2 + (long long)row * H + col : col == H ? b2 + row : -1;
+  }
+  e -= n2;
+  const int row = (int)(e / Hp), col = (int)(e - (size_t)row * Hp);
+  return col < H ? w3 + (long long)row * H + col : col == H ? b3 + row : -1;
+}
+
+__global__ void __launch_bounds__(kT) k_convert(float* flat, float* aug, size_t n_aug, int in,
+                                                int in_p, int H, int Hp, int out, int to_aug) {
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n_aug; e += (size_t)gridDim.x * kT) {
+    const long long f = flat_index(e, in, in_p, H, Hp, out);
+    if (to_aug)
+      aug[e] = f >= 0 ? flat[f] : 0.0f;
+    else if (f >= 0)
+      flat[f] = aug[e];
+  }
+}
+
+__global__ void __launch_bounds__(kT) k_fill_ones(float* buf, int ld, int col, int rows) {
+  for (int r = blockIdx.x * kT + threadIdx.x; r < rows; r += gridDim.x * kT) {
+    float* p = buf + (size_t)r * ld;
+    p[col] = 1.0f;
+    for (int c = col + 1; c < ld; ++c) p[c] = 0.0f;
+  }
+}
+
+unsigned grid_for(size_t n) {
+  const size_t g = (n + kT - 1) / kT;
+  return (unsigned)(g < 152 * 8 ? (g > 0 ? g : 1) : 152 * 8);
+}
+
+}  // namespace
+
+size_t aug_count(int in, int in_p, int H, int Hp, int out) {
+  return (size_t)H * in_p + (size_t)H * Hp + (size_t)out * Hp;
+}
+
+cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
+                          const float* act, const float* logp, const float* adv,
+                          const float* ret, uint32_t N, const Sample& out, cudaStream_t s) {
+  k_gather<<<(d.B + kT - 1) / kT, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tanh_fwd(float* h, int ld, int B, int H, cudaStream_t s) {
+  k_tanh_fwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(h, ld, B, H / 4);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tanh_bwd(float* g, int ldg, const float* h, int ldh, int B, int H,
+                            cudaStream_t s) {
+  k_tanh_bwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(g, ldg, h, ldh, B, H / 4);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_head(const Dims& d, const LossHp& hp, const float* y, const float* v,
+                        const Sample& smp, float* g_y, float* g_v, float* part, cudaStream_t s) {
+  const int nb = (d.B + kT - 1) / kT;
+  k_head<<<nb, kT, 0, s>>>(d, hp, y, v, smp, nb, g_y, g_v, part);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, float* mb,
+                         float* acc, cudaStream_t s) {
+  k_stats<<<1, kT, 0, s>>>(d.B, (d.B + kT - 1) / kT, hp.vf_coef, hp.ent_coef, part, mb, acc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
+                        const AdamHp& hp, float* mb, float* acc, cudaStream_t s) {
+  k_sumsq<<<kNormBlocks, kT, 0, s>>>(g, n, part);
+  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, mb, acc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_finish(const float* acc, float* out, cudaStream_t s) {
+  k_finish<<<1, 32, 0, s>>>(acc, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int Hp, int out,
+                           bool to_aug, cudaStream_t s) {
+  const size_t n = aug_count(in, in_p, H, Hp, out);
+  k_convert<<<grid_for(n), kT, 0, s>>>(flat, aug, n, in, in_p, H, Hp, out, to_aug ? 1 : 0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fill_ones(float* buf, int ld, int col, int rows, cudaStream_t s) {
+  k_fill_ones<<<grid_for((size_t)rows), kT, 0, s>>>(buf, ld, col, rows);
+  return cudaGetLastError();
+}
+
+}  // namespace ppo
+}  // namespace auv

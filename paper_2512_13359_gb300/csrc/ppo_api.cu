@@ -1,0 +1,547 @@
+// ppo_api.cu -- the PPO learner's extern "C" entry points (include/auvenv.h):
+// validation, the learner's device memory, and the sequence of one gradient
+// step: gather -> forward GEMMs + tanh -> loss head -> backward GEMMs + tanh'
+// -> (gradient norm, Adam).  The dense products are plain GEMMs and run in
+// cuBLAS (fp32, tf32 or bf16 tensor-core compute on fp32 data); every other
+// step runs in the kernels of k_ppo.cu.
+//
+// Memory layout (one cudaMalloc): master weights, gradient and Adam moments
+// as augmented vectors [policy | value] (auv_kernels.h, ppo::Dims), a flat
+// staging vector, the gathered minibatch, and per network the activations
+// H1, H2 [B][Hp] (constant 1 at column H), the backward buffer G [B][H] and
+// the head output Y [B][out].  Everything a step touches is resident; no call
+// after ppo_create allocates.
+#include <cublas_v2.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "auv_kernels.h"
+#include "auvenv.h"
+
+namespace ppo = auv::ppo;
+
+struct auv_ppo {
+  auv_ppo_config cfg;
+  int device;
+  cublasHandle_t blas;
+  cublasComputeType_t ctype;
+  ppo::Dims d;
+  int out[2];                 // head widths: 2A (policy), 1 (value)
+  size_t n_flat[2], n_aug[2], n_aug_all;
+  char* mem;
+  float *w, *g, *m, *v;       // augmented [policy | value]
+  float* flat;                // staging, flat [policy | value]
+  ppo::Sample smp;
+  float *h1[2], *h2[2], *gb[2], *y[2];
+  float *g_y, *g_v;           // dL/d(head) [B][2A], [B]
+  float *head_part, *norm_part;
+  float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
+  void* blas_ws;
+  uint64_t t, epoch;
+  char err[256];
+};
+
+namespace {
+
+constexpr size_t kBlasWorkspace = 32u << 20;
+thread_local char g_err[256] = "";
+
+int fail(auv_ppo* p, int code, const char* fmt, ...) {
+  char* dst = p ? p->err : g_err;
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(dst, 256, fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(auv_ppo* p, cudaError_t e, const char* what) {
+  return fail(p, AUV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int blas_fail(auv_ppo* p, cublasStatus_t e, const char* what) {
+  return fail(p, AUV_ERR_CUDA, "%s: cuBLAS status %d", what, (int)e);
+}
+
+int round4(int x) { return (x + 3) & ~3; }
+
+bool is_device(const void* q) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, q) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+int check_dev(auv_ppo* p, const void* q, const char* name) {
+  if (!q) return fail(p, AUV_ERR_INVALID, "%s is NULL", name);
+  if (reinterpret_cast<uintptr_t>(q) % 4) return fail(p, AUV_ERR_SIZE, "%s not 4-byte aligned", name);
+  if (!is_device(q)) return fail(p, AUV_ERR_SIZE, "%s is not device memory", name);
+  return AUV_OK;
+}
+
+int check_device(auv_ppo* p) {
+  int cur = -1;
+  cudaError_t e = cudaGetDevice(&cur);
+  if (e != cudaSuccess) return cuda_fail(p, e, "cudaGetDevice");
+  if (cur != p->device)
+    return fail(p, AUV_ERR_INVALID, "device %d is current but the learner lives on device %d",
+                cur, p->device);
+  return AUV_OK;
+}
+
+int validate(const auv_ppo_config* c) {
+  if (!c) return fail(nullptr, AUV_ERR_INVALID, "cfg is NULL");
+  if (c->struct_size != sizeof(auv_ppo_config))
+    return fail(nullptr, AUV_ERR_INVALID, "cfg->struct_size %u != sizeof(auv_ppo_config) %zu",
+                c->struct_size, sizeof(auv_ppo_config));
+  if (c->obs_dim < 1 || c->obs_dim > 64) return fail(nullptr, AUV_ERR_INVALID, "obs_dim outside [1, 64]");
+  if (c->act_dim < 1 || c->act_dim > 8) return fail(nullptr, AUV_ERR_INVALID, "act_dim outside [1, 8]");
+  if (c->hidden < 8 || c->hidden > 1024 || c->hidden % 8)
+    return fail(nullptr, AUV_ERR_INVALID, "hidden must be a multiple of 8 in [8, 1024]");
+  if (c->minibatch < 2 || c->minibatch > (1u << 22))
+    return fail(nullptr, AUV_ERR_INVALID, "minibatch outside [2, 2^22]");
+  if (c->precision > AUV_PPO_BF16) return fail(nullptr, AUV_ERR_INVALID, "unknown precision %u", c->precision);
+  if (c->norm_adv > 1) return fail(nullptr, AUV_ERR_INVALID, "norm_adv must be 0 or 1");
+  if (c->reserved) return fail(nullptr, AUV_ERR_INVALID, "reserved must be 0");
+  if (!(std::isfinite(c->clip_eps) && c->clip_eps > 0.0f))
+    return fail(nullptr, AUV_ERR_INVALID, "clip_eps must be finite and > 0");
+  if (!std::isfinite(c->vf_coef) || !std::isfinite(c->ent_coef) || std::isnan(c->max_grad_norm) ||
+      std::isinf(c->max_grad_norm))
+    return fail(nullptr, AUV_ERR_INVALID, "loss coefficients and max_grad_norm must be finite");
+  if (!(std::isfinite(c->lr) && c->lr >= 0.0f)) return fail(nullptr, AUV_ERR_INVALID, "lr must be finite and >= 0");
+  if (!(c->adam_beta1 >= 0.0f && c->adam_beta1 < 1.0f && c->adam_beta2 >= 0.0f && c->adam_beta2 < 1.0f))
+    return fail(nullptr, AUV_ERR_INVALID, "Adam betas must lie in [0, 1)");
+  if (!(std::isfinite(c->adam_eps) && c->adam_eps > 0.0f))
+    return fail(nullptr, AUV_ERR_INVALID, "adam_eps must be finite and > 0");
+  if (!(std::isfinite(c->logstd_min) && std::isfinite(c->logstd_max) && c->logstd_min <= c->logstd_max))
+    return fail(nullptr, AUV_ERR_INVALID, "logstd clamp invalid");
+  return AUV_OK;
+}
+
+int check_batch(auv_ppo* p, const auv_ppo_batch* b) {
+  if (!b) return fail(p, AUV_ERR_INVALID, "batch is NULL");
+  if (b->T < 1 || b->N < 1) return fail(p, AUV_ERR_INVALID, "batch T and N must be >= 1");
+  if ((uint64_t)b->T * b->N > (1ull << 31)) return fail(p, AUV_ERR_SIZE, "T * N exceeds 2^31");
+  int rc;
+  if ((rc = check_dev(p, b->obs, "batch.obs")) || (rc = check_dev(p, b->act, "batch.act")) ||
+      (rc = check_dev(p, b->logp, "batch.logp")) || (rc = check_dev(p, b->adv, "batch.adv")) ||
+      (rc = check_dev(p, b->ret, "batch.ret")))
+    return rc;
+  return AUV_OK;
+}
+
+ppo::PermKey perm_key(const auv_ppo* p, uint32_t m, uint64_t epoch) {
+  ppo::PermKey k;
+  int bits = 2;
+  while ((1ull << bits) < m) bits += 2;
+  k.m = m;
+  k.h = bits / 2;
+  k.mask = k.h >= 32 ? 0xFFFFFFFFu : ((1u << k.h) - 1u);
+  k.k0 = (uint32_t)p->cfg.seed;
+  k.k1 = (uint32_t)(p->cfg.seed >> 32);
+  k.e0 = (uint32_t)epoch;
+  k.e1 = (uint32_t)(epoch >> 32);
+  return k;
+}
+
+ppo::LossHp loss_hp(const auv_ppo* p) {
+  const auv_ppo_config& c = p->cfg;
+  return {c.clip_eps, c.vf_coef, c.ent_coef, c.logstd_min, c.logstd_max, (int)c.norm_adv};
+}
+
+cublasStatus_t gemm(auv_ppo* p, cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
+                    const float* A, int lda, const float* B, int ldb, float* C, int ldc) {
+  const float one = 1.0f, zero = 0.0f;
+  return cublasGemmEx(p->blas, ta, tb, m, n, k, &one, A, CUDA_R_32F, lda, B, CUDA_R_32F, ldb,
+                      &zero, C, CUDA_R_32F, ldc, p->ctype, CUBLAS_GEMM_DEFAULT);
+}
+
+size_t net_offset(const auv_ppo* p, int net) { return net ? p->n_aug[0] : 0; }
+
+// Column-major view (cuBLAS): a sample-major [B][ld] array is an ld x B
+// matrix; a row-major weight [out][in_p] is an in_p x out matrix.
+//   Z1 = W1a^T X,  Z2 = W2a^T H1,  Y = W3a^T H2           (forward)
+//   gW3a = H2 gY^T, gH2 = W3 gY, gW2a = H1 gZ2^T, gH1 = W2 gZ2, gW1a = X gZ1^T
+int forward(auv_ppo* p, int net, cudaStream_t s) {
+  const ppo::Dims& d = p->d;
+  const float* w = p->w + net_offset(p, net);
+  const float *w1 = w, *w2 = w + (size_t)d.H * d.Dp, *w3 = w2 + (size_t)d.H * d.Hp;
+  cublasStatus_t bs;
+  cudaError_t e;
+  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Dp, w1, d.Dp, p->smp.X, d.Dp, p->h1[net], d.Hp)))
+    return blas_fail(p, bs, "forward layer 1");
+  if ((e = ppo::launch_tanh_fwd(p->h1[net], d.Hp, d.B, d.H, s))) return cuda_fail(p, e, "tanh 1");
+  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp, p->h2[net], d.Hp)))
+    return blas_fail(p, bs, "forward layer 2");
+  if ((e = ppo::launch_tanh_fwd(p->h2[net], d.Hp, d.B, d.H, s))) return cuda_fail(p, e, "tanh 2");
+  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Hp,
+                 p->y[net], p->out[net])))
+    return blas_fail(p, bs, "forward layer 3");
+  return AUV_OK;
+}
+
+int backward(auv_ppo* p, int net, const float* gy, cudaStream_t s) {
+  const ppo::Dims& d = p->d;
+  const int out = p->out[net];
+  const float* w = p->w + net_offset(p, net);
+  const float *w2 = w + (size_t)d.H * d.Dp, *w3 = w2 + (size_t)d.H * d.Hp;
+  float* g = p->g + net_offset(p, net);
+  float *g1 = g, *g2 = g + (size_t)d.H * d.Dp, *g3 = g2 + (size_t)d.H * d.Hp;
+  float* gz2 = p->gb[net];
+  float* gz1 = p->h2[net];      // H2 is dead once gZ2 exists
+  cublasStatus_t bs;
+  cudaError_t e;
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, out, d.B, p->h2[net], d.Hp, gy, out, g3, d.Hp)))
+    return blas_fail(p, bs, "gradient W3");
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, out, w3, d.Hp, gy, out, gz2, d.H)))
+    return blas_fail(p, bs, "gradient H2");
+  if ((e = ppo::launch_tanh_bwd(gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
+    return cuda_fail(p, e, "tanh' 2");
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp)))
+    return blas_fail(p, bs, "gradient W2");
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp)))
+    return blas_fail(p, bs, "gradient H1");
+  if ((e = ppo::launch_tanh_bwd(gz1, d.Hp, p->h1[net], d.Hp, d.B, d.H, s)))
+    return cuda_fail(p, e, "tanh' 1");
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->smp.X, d.Dp, gz1, d.Hp, g1, d.Dp)))
+    return blas_fail(p, bs, "gradient W1");
+  return AUV_OK;
+}
+
+int grads_impl(auv_ppo* p, const auv_ppo_batch* b, uint64_t epoch, uint32_t j, float* acc,
+               cudaStream_t s) {
+  const ppo::Dims& d = p->d;
+  const uint32_t m = b->T * b->N;
+  cudaError_t e = ppo::launch_gather(d, perm_key(p, m, epoch), j * (uint32_t)d.B, b->obs, b->act,
+                                     b->logp, b->adv, b->ret, b->N, p->smp, s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "gather");
+  int rc;
+  if ((rc = forward(p, 0, s)) || (rc = forward(p, 1, s))) return rc;
+  const ppo::LossHp hp = loss_hp(p);
+  if ((e = ppo::launch_head(d, hp, p->y[0], p->y[1], p->smp, p->g_y, p->g_v, p->head_part, s)))
+    return cuda_fail(p, e, "loss head");
+  if ((e = ppo::launch_stats(d, hp, p->head_part, p->mb, acc, s))) return cuda_fail(p, e, "statistics");
+  if ((rc = backward(p, 0, p->g_y, s)) || (rc = backward(p, 1, p->g_v, s))) return rc;
+  return AUV_OK;
+}
+
+int apply_impl(auv_ppo* p, float* acc, cudaStream_t s) {
+  const auv_ppo_config& c = p->cfg;
+  const uint64_t t = p->t + 1;
+  ppo::AdamHp hp;
+  hp.lr = c.lr;
+  hp.b1 = c.adam_beta1;
+  hp.b2 = c.adam_beta2;
+  hp.eps = c.adam_eps;
+  hp.c1 = (float)(1.0 - std::pow((double)c.adam_beta1, (double)t));
+  hp.c2 = (float)(1.0 - std::pow((double)c.adam_beta2, (double)t));
+  hp.max_norm = c.max_grad_norm;
+  if (!(hp.c1 > 0.0f)) hp.c1 = 1.0f;   // beta1 = 0 keeps the plain moment
+  if (!(hp.c2 > 0.0f)) hp.c2 = 1.0f;
+  cudaError_t e = ppo::launch_adam(p->w, p->g, p->m, p->v, p->n_aug_all, p->norm_part, hp, p->mb,
+                                   acc, s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "Adam");
+  p->t = t;
+  return AUV_OK;
+}
+
+// Convert both networks between a caller's flat parameter vector (device
+// memory) and an augmented learner vector.
+int convert(auv_ppo* p, float* flat_pol, float* flat_val, float* aug, bool to_aug,
+            cudaStream_t s) {
+  const ppo::Dims& d = p->d;
+  cudaError_t e = ppo::launch_convert(flat_pol, aug, d.D, d.Dp, d.H, d.Hp, p->out[0], to_aug, s);
+  if (e == cudaSuccess)
+    e = ppo::launch_convert(flat_val, aug + p->n_aug[0], d.D, d.Dp, d.H, d.Hp, p->out[1], to_aug, s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "weight layout conversion");
+}
+
+// Copy a caller's policy/value pair (device or host) into the flat staging
+// vector, then into the augmented vector dst.
+int load_pair(auv_ppo* p, const float* pol, const float* val, float* dst, cudaStream_t s) {
+  cudaError_t e = cudaMemcpyAsync(p->flat, pol, p->n_flat[0] * 4, cudaMemcpyDefault, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(p->flat + p->n_flat[0], val, p->n_flat[1] * 4, cudaMemcpyDefault, s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "copy in");
+  int rc = convert(p, p->flat, p->flat + p->n_flat[0], dst, true, s);
+  if (rc) return rc;
+  e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "synchronise");
+}
+
+int store_pair(auv_ppo* p, float* src, float* pol, float* val, cudaStream_t s) {
+  int rc = convert(p, p->flat, p->flat + p->n_flat[0], src, false, s);
+  if (rc) return rc;
+  cudaError_t e = cudaMemcpyAsync(pol, p->flat, p->n_flat[0] * 4, cudaMemcpyDefault, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(val, p->flat + p->n_flat[0], p->n_flat[1] * 4, cudaMemcpyDefault, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "copy out");
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ppo_last_error(const auv_ppo* p) { return p ? p->err : g_err; }
+
+int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
+  if (!out) return fail(nullptr, AUV_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  int rc = validate(cfg);
+  if (rc) return rc;
+  auv_ppo* p = new (std::nothrow) auv_ppo();
+  if (!p) return fail(nullptr, AUV_ERR_INVALID, "out of host memory");
+  p->cfg = *cfg;
+  cudaGetDevice(&p->device);
+  ppo::Dims& d = p->d;
+  d.D = (int)cfg->obs_dim;
+  d.Dp = round4(d.D + 1);
+  d.A = (int)cfg->act_dim;
+  d.H = (int)cfg->hidden;
+  d.Hp = round4(d.H + 1);
+  d.B = (int)cfg->minibatch;
+  p->out[0] = 2 * d.A;
+  p->out[1] = 1;
+  for (int k = 0; k < 2; ++k) {
+    const size_t o = (size_t)p->out[k];
+    p->n_flat[k] = (size_t)d.H * d.D + d.H + (size_t)d.H * d.H + d.H + o * d.H + o;
+    p->n_aug[k] = ppo::aug_count(d.D, d.Dp, d.H, d.Hp, p->out[k]);
+  }
+  p->n_aug_all = p->n_aug[0] + p->n_aug[1];
+  p->ctype = cfg->precision == AUV_PPO_FP32   ? CUBLAS_COMPUTE_32F
+             : cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32
+                                              : CUBLAS_COMPUTE_32F_FAST_16BF;
+  // one allocation, 256-byte aligned pieces
+  const size_t B = (size_t)d.B, nb = (B + 255) / 256;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) & ~(size_t)255;
+    return o;
+  };
+  const size_t o_w = take(p->n_aug_all * 4), o_g = take(p->n_aug_all * 4),
+               o_m = take(p->n_aug_all * 4), o_v = take(p->n_aug_all * 4),
+               o_flat = take((p->n_flat[0] + p->n_flat[1]) * 4), o_x = take(B * d.Dp * 4),
+               o_act = take(B * d.A * 4), o_lp = take(B * 4), o_adv = take(B * 4),
+               o_ret = take(B * 4), o_ap = take(nb * 2 * 8), o_gy = take(B * 2 * d.A * 4),
+               o_gv = take(B * 4), o_hp = take(nb * 5 * 4), o_np = take(ppo::kNormBlocks * 4),
+               o_mb = take(AUV_PPO_STATS * 4), o_acc = take(AUV_PPO_STATS * 4),
+               o_ws = take(kBlasWorkspace);
+  size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
+  for (int k = 0; k < 2; ++k) {
+    o_h1[k] = take(B * d.Hp * 4);
+    o_h2[k] = take(B * d.Hp * 4);
+    o_gb[k] = take(B * d.H * 4);
+    o_y[k] = take(B * p->out[k] * 4);
+  }
+  cudaError_t e = cudaMalloc(&p->mem, off);
+  if (e != cudaSuccess) {
+    delete p;
+    return cuda_fail(nullptr, e, "cudaMalloc(learner)");
+  }
+  char* base = p->mem;
+  p->w = reinterpret_cast<float*>(base + o_w);
+  p->g = reinterpret_cast<float*>(base + o_g);
+  p->m = reinterpret_cast<float*>(base + o_m);
+  p->v = reinterpret_cast<float*>(base + o_v);
+  p->flat = reinterpret_cast<float*>(base + o_flat);
+  p->smp.X = reinterpret_cast<float*>(base + o_x);
+  p->smp.act = reinterpret_cast<float*>(base + o_act);
+  p->smp.logp = reinterpret_cast<float*>(base + o_lp);
+  p->smp.adv = reinterpret_cast<float*>(base + o_adv);
+  p->smp.ret = reinterpret_cast<float*>(base + o_ret);
+  p->smp.adv_part = reinterpret_cast<double*>(base + o_ap);
+  p->g_y = reinterpret_cast<float*>(base + o_gy);
+  p->g_v = reinterpret_cast<float*>(base + o_gv);
+  p->head_part = reinterpret_cast<float*>(base + o_hp);
+  p->norm_part = reinterpret_cast<float*>(base + o_np);
+  p->mb = reinterpret_cast<float*>(base + o_mb);
+  p->acc = reinterpret_cast<float*>(base + o_acc);
+  p->blas_ws = base + o_ws;
+  for (int k = 0; k < 2; ++k) {
+    p->h1[k] = reinterpret_cast<float*>(base + o_h1[k]);
+    p->h2[k] = reinterpret_cast<float*>(base + o_h2[k]);
+    p->gb[k] = reinterpret_cast<float*>(base + o_gb[k]);
+    p->y[k] = reinterpret_cast<float*>(base + o_y[k]);
+  }
+  e = cudaMemset(p->mem, 0, off);
+  for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+    e = ppo::launch_fill_ones(p->h1[k], d.Hp, d.H, d.B, 0);
+    if (e == cudaSuccess) e = ppo::launch_fill_ones(p->h2[k], d.Hp, d.H, d.B, 0);
+  }
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cudaFree(p->mem);
+    delete p;
+    return cuda_fail(nullptr, e, "initialise learner memory");
+  }
+  cublasStatus_t bs = cublasCreate(&p->blas);
+  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetWorkspace(p->blas, p->blas_ws, kBlasWorkspace);
+  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetMathMode(p->blas, CUBLAS_DEFAULT_MATH);
+  if (bs != CUBLAS_STATUS_SUCCESS) {
+    if (p->blas) cublasDestroy(p->blas);
+    cudaFree(p->mem);
+    delete p;
+    return blas_fail(nullptr, bs, "cuBLAS handle");
+  }
+  *out = p;
+  return AUV_OK;
+}
+
+int ppo_destroy(auv_ppo* p) {
+  if (!p) return AUV_ERR_INVALID;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  cudaSetDevice(p->device);
+  cudaDeviceSynchronize();
+  cublasDestroy(p->blas);
+  cudaFree(p->mem);
+  if (prev >= 0) cudaSetDevice(prev);
+  delete p;
+  return AUV_OK;
+}
+
+int ppo_param_counts(const auv_ppo* p, uint64_t* n_policy, uint64_t* n_value) {
+  if (!p || !n_policy || !n_value) return AUV_ERR_INVALID;
+  *n_policy = p->n_flat[0];
+  *n_value = p->n_flat[1];
+  return AUV_OK;
+}
+
+int ppo_set_weights(auv_ppo* p, const float* policy, const float* value, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  if (!policy || !value) return fail(p, AUV_ERR_INVALID, "weights are NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t bytes = p->n_aug_all * 4;
+  cudaError_t e = cudaMemsetAsync(p->m, 0, bytes, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(p->v, 0, bytes, s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "clear Adam moments");
+  if ((rc = load_pair(p, policy, value, p->w, s))) return rc;
+  p->t = 0;
+  p->epoch = 0;
+  return AUV_OK;
+}
+
+int ppo_get_weights(auv_ppo* p, float* policy, float* value, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  if (!policy || !value) return fail(p, AUV_ERR_INVALID, "outputs are NULL");
+  return store_pair(p, p->w, policy, value, static_cast<cudaStream_t>(stream));
+}
+
+int ppo_export_weights(auv_ppo* p, float* policy, float* value, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc || (rc = check_dev(p, policy, "policy")) || (rc = check_dev(p, value, "value"))) return rc;
+  return convert(p, policy, value, p->w, false, static_cast<cudaStream_t>(stream));
+}
+
+int ppo_get_state(auv_ppo* p, float* m, float* v, uint64_t* t, uint64_t* epoch, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  if (!m || !v || !t || !epoch) return fail(p, AUV_ERR_INVALID, "outputs are NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = store_pair(p, p->m, m, m + p->n_flat[0], s))) return rc;
+  if ((rc = store_pair(p, p->v, v, v + p->n_flat[0], s))) return rc;
+  *t = p->t;
+  *epoch = p->epoch;
+  return AUV_OK;
+}
+
+int ppo_set_state(auv_ppo* p, const float* m, const float* v, uint64_t t, uint64_t epoch,
+                  void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  if (!m || !v) return fail(p, AUV_ERR_INVALID, "moments are NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = load_pair(p, m, m + p->n_flat[0], p->m, s))) return rc;
+  if ((rc = load_pair(p, v, v + p->n_flat[0], p->v, s))) return rc;
+  p->t = t;
+  p->epoch = epoch;
+  return AUV_OK;
+}
+
+int ppo_grads(auv_ppo* p, const auv_ppo_batch* batch, uint64_t epoch, uint32_t minibatch,
+              float* grad, float* stats, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc || (rc = check_batch(p, batch))) return rc;
+  if (((uint64_t)minibatch + 1) * p->d.B > (uint64_t)batch->T * batch->N)
+    return fail(p, AUV_ERR_SIZE, "minibatch %u needs %llu rows, the batch has %llu", minibatch,
+                (unsigned long long)(((uint64_t)minibatch + 1) * p->d.B),
+                (unsigned long long)batch->T * batch->N);
+  if (grad && (rc = check_dev(p, grad, "grad"))) return rc;
+  if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cublasStatus_t bs = cublasSetStream(p->blas, s);
+  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
+  if ((rc = grads_impl(p, batch, epoch, minibatch, nullptr, s))) return rc;
+  if (grad && (rc = convert(p, grad, grad + p->n_flat[0], p->g, false, s))) return rc;
+  if (stats) {
+    cudaError_t e = cudaMemcpyAsync(stats, p->mb, AUV_PPO_STATS * 4, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(p, e, "copy statistics");
+  }
+  return AUV_OK;
+}
+
+int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  if (grad && (rc = check_dev(p, grad, "grad"))) return rc;
+  if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (grad) {
+    cudaError_t e = cudaMemcpyAsync(p->flat, grad, (p->n_flat[0] + p->n_flat[1]) * 4,
+                                    cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(p, e, "copy gradient");
+    if ((rc = convert(p, p->flat, p->flat + p->n_flat[0], p->g, true, s))) return rc;
+  }
+  if ((rc = apply_impl(p, nullptr, s))) return rc;
+  if (stats) {
+    cudaError_t e = cudaMemcpyAsync(stats + 5, p->mb + 5, 4, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(p, e, "copy gradient norm");
+  }
+  return AUV_OK;
+}
+
+int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t n_minibatches,
+               float* stats, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc || (rc = check_batch(p, batch))) return rc;
+  if (epochs < 1 || n_minibatches < 1) return fail(p, AUV_ERR_INVALID, "epochs and n_minibatches must be >= 1");
+  if ((uint64_t)n_minibatches * p->d.B > (uint64_t)batch->T * batch->N)
+    return fail(p, AUV_ERR_SIZE, "%u minibatches of %d exceed the batch's %llu rows", n_minibatches,
+                p->d.B, (unsigned long long)batch->T * batch->N);
+  if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cublasStatus_t bs = cublasSetStream(p->blas, s);
+  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
+  cudaError_t e = cudaMemsetAsync(p->acc, 0, AUV_PPO_STATS * 4, s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "clear statistics");
+  for (uint32_t ep = 0; ep < epochs; ++ep) {
+    for (uint32_t j = 0; j < n_minibatches; ++j) {
+      if ((rc = grads_impl(p, batch, p->epoch, j, p->acc, s))) return rc;
+      if ((rc = apply_impl(p, p->acc, s))) return rc;
+    }
+    ++p->epoch;
+  }
+  if (stats && (e = ppo::launch_finish(p->acc, stats, s)) != cudaSuccess)
+    return cuda_fail(p, e, "statistics");
+  return AUV_OK;
+}
+
+}  // extern "C"

@@ -22,12 +22,14 @@ def auvlib():
 def header_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\**\s*(env_\w+)\s*\(", text, flags=re.M)))
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\**\s*((?:env|ppo)_\w+)\s*\(", text,
+                                 flags=re.M)))
 
 
 def test_header_declares_the_entry_points():
     names = header_functions()
-    for must in ("env_create", "env_reset", "env_step", "env_rollout", "env_step_actions"):
+    for must in ("env_create", "env_reset", "env_step", "env_rollout", "env_step_actions",
+                 "env_gae", "ppo_create", "ppo_grads", "ppo_apply", "ppo_update"):
         assert must in names
 
 
@@ -124,6 +126,45 @@ def test_null_arguments(auvlib):
     assert auvlib.env_destroy(None) == auvenv.AUV_ERR_INVALID
     assert auvlib.env_reset(None, None, None) == auvenv.AUV_ERR_INVALID
     assert auvlib.env_rollout(None, 1, None, None) == auvenv.AUV_ERR_INVALID
+
+
+def test_ppo_config_struct_size_matches_header(auvlib):
+    from paper_2512_13359_gb300 import auvenv
+    cfg = auvenv.make_ppo_config(18, 8, 256, 4096)
+    h = C.c_void_p()
+    cfg.struct_size = C.sizeof(auvenv.PpoConfig) - 4
+    assert auvlib.ppo_create(C.byref(cfg), C.byref(h)) == auvenv.AUV_ERR_INVALID
+    assert b"struct_size" in auvlib.ppo_last_error(None)
+
+
+@pytest.mark.parametrize("field,value,msg", [
+    ("obs_dim", 0, b"obs_dim"), ("obs_dim", 65, b"obs_dim"), ("act_dim", 9, b"act_dim"),
+    ("hidden", 100, b"hidden"), ("hidden", 2048, b"hidden"), ("minibatch", 1, b"minibatch"),
+    ("precision", 3, b"precision"), ("norm_adv", 2, b"norm_adv"), ("reserved", 1, b"reserved"),
+    ("clip_eps", 0.0, b"clip_eps"), ("clip_eps", float("nan"), b"clip_eps"),
+    ("vf_coef", float("inf"), b"finite"), ("max_grad_norm", float("nan"), b"finite"),
+    ("lr", -1e-3, b"lr"), ("adam_beta1", 1.0, b"betas"), ("adam_beta2", -0.1, b"betas"),
+    ("adam_eps", 0.0, b"adam_eps"), ("logstd_min", 3.0, b"logstd")])
+def test_invalid_ppo_configs_are_rejected(auvlib, field, value, msg):
+    from paper_2512_13359_gb300 import auvenv
+    cfg = auvenv.make_ppo_config(18, 8, 256, 4096)
+    setattr(cfg, field, value)
+    h = C.c_void_p()
+    assert auvlib.ppo_create(C.byref(cfg), C.byref(h)) == auvenv.AUV_ERR_INVALID
+    assert msg in auvlib.ppo_last_error(None)
+    assert not h.value
+
+
+def test_ppo_null_arguments(auvlib):
+    from paper_2512_13359_gb300 import auvenv
+    h = C.c_void_p()
+    E = auvenv.AUV_ERR_INVALID
+    assert auvlib.ppo_create(None, C.byref(h)) == E
+    assert auvlib.ppo_destroy(None) == E
+    assert auvlib.ppo_grads(None, None, 0, 0, None, None, None) == E
+    assert auvlib.ppo_apply(None, None, None, None) == E
+    assert auvlib.ppo_update(None, None, 1, 1, None, None) == E
+    assert auvlib.ppo_set_weights(None, None, None, None) == E
 
 
 def test_binding_fails_loudly_without_the_library(tmp_path):

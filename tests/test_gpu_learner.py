@@ -1,0 +1,282 @@
+"""GPU parity of the PPO learner (ppo_* entry points) against the oracle's
+float64 Learner: one minibatch's gradient and loss record in each GEMM
+precision (several minibatches of a ragged size, a trajectory whose row count
+is not a power of 4, both the Fossen and the paper network shapes), whole
+updates of several epochs (weights after every Adam step), the learner fed
+by a real rollout and env_gae, weight export into an env, checkpoint/resume,
+and argument rejection."""
+import numpy as np
+import pytest
+
+from paper_2512_13359_gb300 import workloads as W
+from parity_util import make_env, need_gpu, to_np
+
+pytestmark = pytest.mark.gpu
+
+# Gradient tolerance, relative to the largest gradient component of each
+# network: fp32 GEMMs sum in fp32 (1e-4); tf32 operands carry 10 mantissa
+# bits (2e-3); bf16 operands 7 (2e-2).
+GRAD_TOL = {"fp32": 1e-4, "tf32": 4e-3, "bf16": 3e-2}
+STAT_TOL = {"fp32": 1e-4, "tf32": 5e-3, "bf16": 3e-2}
+HP = dict(clip_eps=0.2, vf_coef=0.5, ent_coef=0.01, max_grad_norm=0.5, lr=3e-4,
+          adam_beta1=0.9, adam_beta2=0.999, adam_eps=1e-8, logstd_min=-5.0, logstd_max=2.0,
+          norm_adv=True)
+
+
+def _traj(seed, T, N, D, A, policy=None, dims=None):
+    """Random trajectory arrays in the rollout layout; the old log-probs are
+    the networks' own plus noise, so ratios straddle the clip range."""
+    rng = np.random.default_rng(seed)
+    obs = rng.normal(size=(T, D, N)).astype(np.float32)
+    act = rng.normal(size=(T, A, N)).astype(np.float32)
+    logp = (rng.normal(size=(T, N)) * 0.3 - 1.5 * A).astype(np.float32)
+    adv = (rng.normal(size=(T, N)) * 2.0 + 0.3).astype(np.float32)
+    ret = (rng.normal(size=(T, N)) * 3.0 - 5.0).astype(np.float32)
+    return dict(obs=obs, act=act, logp=logp, adv=adv, ret=ret)
+
+
+def _weights(D, H, A, seed=0, bias_std=0.1):
+    pw = W.mlp_weights(seed, D, H, 2 * A, 0, bias_std)
+    vw = W.mlp_weights(seed, D, H, 1, 1, bias_std)
+    return pw, vw
+
+
+def _on_rollout_policy(traj, pw, D, H, A, spread=0.3, seed=1):
+    """Replace logp by the policy's own log-density of act (plus noise)."""
+    from oracle import ppo_oracle as P
+    T, _, N = traj["obs"].shape
+    x = traj["obs"].transpose(0, 2, 1).reshape(-1, D).astype(np.float64)
+    a = traj["act"].transpose(0, 2, 1).reshape(-1, A).astype(np.float64)
+    _, _, y = P.mlp_forward(pw, D, H, 2 * A, x)
+    _, _, _, lp = P.gaussian_policy(y, a, HP)
+    noise = np.random.default_rng(seed).normal(size=lp.shape) * spread
+    traj["logp"] = (lp + noise).reshape(T, N).astype(np.float32)
+    return traj
+
+
+def _dev(torch, traj):
+    return {k: torch.from_numpy(np.ascontiguousarray(v)).cuda() for k, v in traj.items()}
+
+
+def _learner(D, A, H, B, precision, seed=7, **hp):
+    from paper_2512_13359_gb300 import auvenv
+    return auvenv.Learner(D, A, H, B, precision=precision, seed=seed, **dict(HP, **hp))
+
+
+def _check_grad(gpu, ref, n_pol, tol, what):
+    for name, sl in (("policy", slice(0, n_pol)), ("value", slice(n_pol, None))):
+        g, r = gpu[sl], ref[sl]
+        scale = np.abs(r).max()
+        err = np.abs(g - r).max() / scale
+        print(f"[{what}] {name}: max |g| {scale:.3e}, max err / max |g| {err:.3e} (tol {tol})")
+        assert err <= tol, (what, name, err)
+
+
+def _check_stats(stats, parts, tol, B):
+    names = ("pg_loss", "v_loss", "entropy", "approx_kl")
+    for k, name in enumerate(names):
+        ref = parts[name]
+        assert abs(stats[k] - ref) <= tol * max(1.0, abs(ref)), (name, stats[k], ref)
+    assert abs(stats[4] - parts["clip_frac"]) <= 2.0 / B + tol
+
+
+@pytest.mark.parametrize("D,A,H,T,N,B,epoch,mb", [
+    (18, 8, 64, 7, 333, 1000, 3, 1),       # ragged B, M = 2331 (cycle walking)
+    (12, 6, 256, 5, 1000, 777, 0, 4),      # the paper's shapes, last full minibatch
+    (18, 8, 256, 3, 4096, 4096, 11, 2)])   # the rollout's shapes
+def test_fp32_gradient_matches_oracle(D, A, H, T, N, B, epoch, mb):
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    pw, vw = _weights(D, H, A)
+    traj = _on_rollout_policy(_traj(D * 100 + H, T, N, D, A), pw, D, H, A)
+    L = _learner(D, A, H, B, "fp32")
+    L.set_weights(pw, vw)
+    grad = torch.empty(L.n_policy + L.n_value, device="cuda")
+    stats = torch.empty(8, device="cuda")
+    L.grads(_dev(torch, traj), epoch, mb, grad=grad, stats=stats)
+    ref = P.Learner(pw, vw, (D, H, A), HP, seed=7)
+    parts, g_ref = ref.grads(traj, epoch, mb, B)
+    _check_grad(to_np(grad), g_ref, L.n_policy, GRAD_TOL["fp32"], f"fp32 D{D} H{H} B{B}")
+    st = to_np(stats)
+    _check_stats(st, parts, STAT_TOL["fp32"], B)
+    assert st[5] == 0.0 and st[7] == 1.0
+    loss = parts["pg_loss"] + HP["vf_coef"] * parts["v_loss"] - HP["ent_coef"] * parts["entropy"]
+    assert abs(st[6] - loss) <= 1e-4 * max(1.0, abs(loss))
+
+
+@pytest.mark.parametrize("precision", ["tf32", "bf16"])
+def test_tensor_core_gradient_within_tolerance(precision):
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    D, A, H, T, N, B = 18, 8, 256, 4, 8192, 16384
+    pw, vw = _weights(D, H, A, seed=3)
+    traj = _on_rollout_policy(_traj(5, T, N, D, A), pw, D, H, A)
+    L = _learner(D, A, H, B, precision)
+    L.set_weights(pw, vw)
+    grad = torch.empty(L.n_policy + L.n_value, device="cuda")
+    stats = torch.empty(8, device="cuda")
+    L.grads(_dev(torch, traj), 2, 1, grad=grad, stats=stats)
+    parts, g_ref = P.Learner(pw, vw, (D, H, A), HP, seed=7).grads(traj, 2, 1, B)
+    _check_grad(to_np(grad), g_ref, L.n_policy, GRAD_TOL[precision], precision)
+    _check_stats(to_np(stats), parts, STAT_TOL[precision], B)
+
+
+def test_update_matches_oracle_step_by_step():
+    """Two epochs of three minibatches: after each ppo_update the weights
+    agree with the oracle's within a small fraction of the Adam step; the
+    averaged record agrees too.  adam_eps = 1e-5 keeps Adam from dividing
+    fp32 rounding noise of near-zero gradient components by itself."""
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    D, A, H, T, N, B = 18, 8, 64, 6, 500, 900
+    hp = dict(HP, adam_eps=1e-5, lr=1e-3)
+    pw, vw = _weights(D, H, A, seed=4)
+    traj = _on_rollout_policy(_traj(9, T, N, D, A), pw, D, H, A)
+    L = _learner(D, A, H, B, "fp32", **hp)
+    L.set_weights(pw, vw)
+    ref = P.Learner(pw, vw, (D, H, A), hp, seed=7)
+    dtraj = _dev(torch, traj)
+    stats = torch.empty(8, device="cuda")
+    for call in range(2):
+        L.update(dtraj, 2, 3, stats=stats)
+        r = ref.update(traj, 2, 3, B)
+        gp, gv = L.get_weights()
+        steps = 6 * (call + 1)
+        for got, want in ((gp, ref.policy), (gv, ref.value)):
+            err = np.abs(got - want).max()
+            print(f"[update] after {steps} steps: max |w - w_oracle| = {err:.3e} (lr {hp['lr']})")
+            assert err <= 2e-3 * hp["lr"] * steps + 1e-6
+        st = to_np(stats)
+        assert st[7] == 6.0
+        for k, name in enumerate(("pg_loss", "v_loss", "entropy", "approx_kl")):
+            assert abs(st[k] - r[name]) <= 1e-3 * max(1.0, abs(r[name])), name
+        assert abs(st[5] - r["grad_norm"]) <= 1e-3 * r["grad_norm"]
+    s = L.get_state()
+    assert s["t"] == 12 and s["epoch"] == 4
+
+
+def test_learner_on_a_rollout_and_gae():
+    """The learner's real input at the rollout's shapes: a bf16 rollout of
+    65,536 envs x 16 steps (episode ends inside), bootstrap value, env_gae,
+    then one tf32 minibatch of 65,536 samples against the oracle on the same
+    arrays."""
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    n, T, B = 65536, 16, 65536
+    w = W.workload("ppo_65536", n_envs=n, episode_len=10)
+    env = make_env(w)
+    env.reset()
+    traj = env.alloc_traj(T)
+    env.rollout(T, traj)
+    obs = torch.empty((1, 18, n), device="cuda")
+    env.observe(obs[0])
+    last = torch.empty((1, n), device="cuda")
+    env.value(obs, last)
+    adv = torch.empty((T, n), device="cuda")
+    ret = torch.empty((T, n), device="cuda")
+    env.gae(traj["rew"], traj["done"], traj["value"], last[0], 0.99, 0.95, adv, ret)
+    dtraj = dict(obs=traj["obs"], act=traj["act"], logp=traj["logp"], adv=adv, ret=ret)
+    pw, vw = W.policy_weights(w), W.value_weights(w)
+    hp = dict(HP, logstd_min=w["logstd_min"], logstd_max=w["logstd_max"])
+    L = _learner(18, 8, 256, B, "tf32", **hp)
+    L.set_weights(pw, vw)
+    grad = torch.empty(L.n_policy + L.n_value, device="cuda")
+    stats = torch.empty(8, device="cuda")
+    L.grads(dtraj, 0, 0, grad=grad, stats=stats)
+    host = {k: to_np(v) for k, v in dtraj.items()}
+    parts, g_ref = P.Learner(pw, vw, (18, 256, 8), hp, seed=7).grads(host, 0, 0, B)
+    _check_grad(to_np(grad), g_ref, L.n_policy, GRAD_TOL["tf32"], "rollout tf32")
+    st = to_np(stats)
+    _check_stats(st, parts, STAT_TOL["tf32"], B)
+    # the rollout's own log-probs came from bf16 networks: ratios near 1
+    assert abs(st[3]) < 0.05
+
+
+def test_weights_export_set_get_and_env_roundtrip():
+    torch = need_gpu()
+    D, A, H = 18, 8, 256
+    pw, vw = _weights(D, H, A, seed=6, bias_std=0.3)
+    L = _learner(D, A, H, 512, "fp32")
+    L.set_weights(pw, vw)
+    gp, gv = L.get_weights()
+    assert np.array_equal(gp, pw) and np.array_equal(gv, vw)
+    tp = torch.empty(L.n_policy, device="cuda")
+    tv = torch.empty(L.n_value, device="cuda")
+    L.export_weights(tp, tv)
+    assert np.array_equal(to_np(tp), pw) and np.array_equal(to_np(tv), vw)
+    w = W.workload("ppo_65536", n_envs=256)
+    env = make_env(w, policy=False)
+    env.set_weights(tp, tv)          # device pointers straight from the learner
+    obs = torch.from_numpy(W.random_observations(3, 256)).cuda()
+    head = torch.empty((256, 16), device="cuda")
+    env.policy_forward(obs, head)
+    env2 = make_env(w, policy=False)
+    env2.set_weights(pw, vw)
+    head2 = torch.empty((256, 16), device="cuda")
+    env2.policy_forward(obs, head2)
+    assert torch.equal(head, head2)
+
+
+def test_checkpoint_resume_is_bit_exact():
+    torch = need_gpu()
+    D, A, H, T, N, B = 12, 6, 64, 4, 700, 600
+    pw, vw = _weights(D, H, A, seed=8)
+    traj = _dev(torch, _on_rollout_policy(_traj(10, T, N, D, A), pw, D, H, A))
+    a = _learner(D, A, H, B, "fp32")
+    a.set_weights(pw, vw)
+    a.update(traj, 1, 4)
+    saved_w, saved_s = a.get_weights(), a.get_state()
+    a.update(traj, 2, 4)
+    b = _learner(D, A, H, B, "fp32")
+    b.set_weights(*saved_w)
+    b.set_state(saved_s)
+    b.update(traj, 2, 4)
+    for x, y in zip(a.get_weights(), b.get_weights()):
+        assert np.array_equal(x, y)
+    sa, sb = a.get_state(), b.get_state()
+    assert np.array_equal(sa["m"], sb["m"]) and np.array_equal(sa["v"], sb["v"])
+    assert (sa["t"], sa["epoch"]) == (sb["t"], sb["epoch"]) == (12, 3)
+
+
+def test_external_gradient_apply_equals_internal():
+    """ppo_grads -> (caller's vector, e.g. averaged over ranks) -> ppo_apply
+    gives the same weights as applying the learner's own gradient."""
+    torch = need_gpu()
+    D, A, H, T, N, B = 18, 8, 64, 3, 800, 1024
+    pw, vw = _weights(D, H, A, seed=12)
+    traj = _dev(torch, _on_rollout_policy(_traj(11, T, N, D, A), pw, D, H, A))
+    a, b = _learner(D, A, H, B, "fp32"), _learner(D, A, H, B, "fp32")
+    a.set_weights(pw, vw)
+    b.set_weights(pw, vw)
+    g = torch.empty(a.n_policy + a.n_value, device="cuda")
+    stats = torch.zeros(8, device="cuda")
+    a.grads(traj, 0, 1)
+    a.apply()
+    b.grads(traj, 0, 1, grad=g)
+    b.apply(grad=g, stats=stats)
+    for x, y in zip(a.get_weights(), b.get_weights()):
+        assert np.array_equal(x, y)
+    assert float(stats[5]) > 0.0
+
+
+def test_learner_rejects_bad_arguments():
+    torch = need_gpu()
+    from paper_2512_13359_gb300 import auvenv
+    D, A, H, T, N, B = 18, 8, 64, 2, 100, 128
+    L = _learner(D, A, H, B, "fp32")
+    L.set_weights(*_weights(D, H, A))
+    traj = _dev(torch, _traj(1, T, N, D, A))
+    with pytest.raises(auvenv.AuvError) as ei:
+        L.grads(traj, 0, 2)                           # rows 256..383 of 200
+    assert ei.value.code == auvenv.AUV_ERR_SIZE
+    with pytest.raises(auvenv.AuvError):
+        L.update(traj, 1, 2)                          # 2 x 128 > 200
+    with pytest.raises(auvenv.AuvError) as ei:
+        L.update(traj, 0, 1)
+    assert ei.value.code == auvenv.AUV_ERR_INVALID
+    host = {k: v.cpu() for k, v in traj.items()}
+    with pytest.raises(auvenv.AuvError) as ei:
+        L.grads(host, 0, 0)                           # host arrays
+    assert ei.value.code == auvenv.AUV_ERR_SIZE
+    with pytest.raises(ValueError):
+        L.set_weights(np.zeros(3), np.zeros(3))
