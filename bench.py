@@ -53,6 +53,13 @@ def parse():
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--replay", action="store_true",
                     help="physics only: action replay (env_step_actions), FP32 roofline")
+    ap.add_argument("--ppo", action="store_true",
+                    help="time the PPO update (ppo_update) on one rollout's trajectory")
+    ap.add_argument("--ppo-precision", default="bf16", choices=["fp32", "tf32", "bf16"])
+    ap.add_argument("--minibatch", type=int, default=65536)
+    ap.add_argument("--epochs", type=int, default=4)
+    ap.add_argument("--n-minibatches", type=int, default=None,
+                    help="minibatches per epoch (default: all rows / minibatch)")
     ap.add_argument("--gae", action="store_true",
                     help="advantage estimation (env_gae) over one rollout, HBM roofline")
     ap.add_argument("--sweep", action="store_true",
@@ -333,8 +340,106 @@ def run_gae(args):
     print(json.dumps(line), flush=True)
 
 
+def ppo_flops_per_sample(d, h, a):
+    """Algorithmic flops of one PPO sample: forward of both MLPs
+    (2 x multiply-adds), their weight gradients (same count) and the input
+    gradients of layers 2 and 3 (layer 1's input gradient is not needed)."""
+    fwd = mlp_flops(d, h, 2 * a) + mlp_flops(d, h, 1)
+    return 3 * fwd - 2 * (2 * d * h)
+
+
+def run_ppo(args):
+    """The PPO update (ppo_update: epochs x minibatches of gather, forward,
+    loss head, backward, Adam) over the trajectory of one rollout of the
+    workload plus env_gae.  Tensor roofline: algorithmic flops of the two
+    MLPs' forward and backward per sample."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {}
+    if args.n_envs:
+        over["n_envs"] = args.n_envs
+    if args.rollout_steps:
+        over["steps"] = args.rollout_steps
+    w = W.workload(args.workload, **over)
+    n, T = int(w["n_envs"]), int(w["steps"])
+    D, A, H = W.obs_dim(w), W.act_dim(w), int(w["hidden"])
+    env = auvenv.Env(w)
+    env.set_weights(W.policy_weights(w), W.value_weights(w))
+    env.reset()
+    traj = env.alloc_traj(T)
+    env.rollout(T, traj)
+    obs = torch.empty((1, D, n), device="cuda")
+    env.observe(obs[0])
+    last = torch.empty((1, n), device="cuda")
+    env.value(obs, last)
+    adv = torch.empty((T, n), device="cuda")
+    ret = torch.empty((T, n), device="cuda")
+    env.gae(traj["rew"], traj["done"], traj["value"], last[0], 0.99, 0.95, adv, ret)
+    batch = dict(obs=traj["obs"], act=traj["act"], logp=traj["logp"], adv=adv, ret=ret)
+    B = args.minibatch
+    n_mb = args.n_minibatches or (n * T) // B
+    L = auvenv.Learner(D, A, H, B, precision=args.ppo_precision, seed=1,
+                       logstd_min=w["logstd_min"], logstd_max=w["logstd_max"])
+    L.set_weights(W.policy_weights(w), W.value_weights(w))
+    stats = torch.empty(8, device="cuda")
+    for _ in range(args.warmup):
+        L.update(batch, args.epochs, n_mb, stats=stats)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0) if not args.no_clocks else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ms = []
+    for _ in range(args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        L.update(batch, args.epochs, n_mb, stats=stats)
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    clock_info = clocks.stop() if clocks else None
+    step_ms = sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+    samples = args.epochs * n_mb * B
+    fps = ppo_flops_per_sample(D, H, A)
+    achieved = samples * fps / (step_ms * 1e-3) / 1e12
+    peaks, src = load_peaks()
+    if args.ppo_precision == "fp32":
+        mhz = peaks.get("sm_max_mhz", 2070.0)
+        peak, bound, psrc = 152 * 128 * 2 * mhz * 1e6 / 1e12, "alu", f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz"
+    else:
+        ratio = 1.0 if args.ppo_precision == "bf16" else 1.1 / 2.25
+        peak = peaks["bf16_tflops_sustained"] * ratio
+        bound, psrc = "tensor", (f"bf16 sustained, {src}" + ("" if ratio == 1.0 else
+                                 " x tf32/bf16 nominal 1.1/2.25"))
+    st = stats.cpu().numpy().tolist()
+    launches_per_step = 1 + 10 + 1 + 1 + 14 + 2     # gather, fwd, head, stats, bwd, norm+Adam
+    line = {
+        "metric": "PPO update samples/s", "value": samples / (step_ms * 1e-3),
+        "unit": "samples/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if args.ppo_precision == "fp32" else args.ppo_precision,
+        "data": "synthetic (one rollout of the workload, env_gae advantages)",
+        "config": {"workload": w["name"], "n_envs": n, "rollout_steps": T, "rows": n * T,
+                   "minibatch": B, "minibatches_per_epoch": n_mb, "epochs": args.epochs,
+                   "precision": args.ppo_precision,
+                   "l2": "working set per step larger than L2 when B >= 32768"},
+        "roofline": {"bound": bound, "kernel": "whole update (cuBLAS GEMMs + own kernels)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "peak_source": psrc,
+                     "flops_per_sample": fps},
+        "update_stats": dict(zip(auvenv.PPO_STAT_NAMES, st)),
+        "gpu_launches": args.steps * args.epochs * n_mb * launches_per_step,
+        "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.ppo:
+        run_ppo(args)
+        return
     if args.replay:
         run_replay(args)
         return

@@ -72,6 +72,9 @@ struct Dims {
   int A;         // action width; policy head 2A
   int H, Hp;     // hidden width and its augmented row (>= H + 1)
   int B;         // minibatch
+  int ld_pol;    // row length of the policy head arrays Y, dL/dY (>= 2A)
+  int ld_val;    // row length of the value head arrays (>= 1)
+  int bf16;      // activations and head gradients stored as bf16
 };
 
 struct PermKey {        // Feistel permutation of [0, m) for one epoch
@@ -91,7 +94,6 @@ struct AdamHp {
 };
 
 struct Sample {                    // gathered minibatch, sample-major
-  float* X;                        // [B][Dp] (1 at column D)
   float* act;                      // [B][A]
   float* logp;                     // [B]
   float* adv;                      // [B]
@@ -102,23 +104,29 @@ struct Sample {                    // gathered minibatch, sample-major
 constexpr int kNormBlocks = 256;   // blocks of the gradient-norm reduction
 
 size_t aug_count(int in, int in_p, int H, int Hp, int out);
+// X [B][Dp]: the gathered observations with the constant 1 at column D,
+// fp32 or bf16 (Dims::bf16), as are the activation arguments below.
 cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
                           const float* act, const float* logp, const float* adv,
-                          const float* ret, uint32_t N, const Sample& out, cudaStream_t s);
-cudaError_t launch_tanh_fwd(float* h, int ld, int B, int H, cudaStream_t s);
-cudaError_t launch_tanh_bwd(float* g, int ldg, const float* h, int ldh, int B, int H,
+                          const float* ret, uint32_t N, const Sample& out, void* X,
+                          cudaStream_t s);
+cudaError_t launch_tanh_fwd(bool bf16, void* h, int ld, int B, int H, cudaStream_t s);
+cudaError_t launch_tanh_bwd(bool bf16, void* g, int ldg, const void* h, int ldh, int B, int H,
                             cudaStream_t s);
+// y [B][ld_pol], v [B][ld_val] fp32 head outputs; g_y, g_v the same shapes.
 cudaError_t launch_head(const Dims& d, const LossHp& hp, const float* y, const float* v,
-                        const Sample& smp, float* g_y, float* g_v, float* part, cudaStream_t s);
+                        const Sample& smp, void* g_y, void* g_v, float* part, cudaStream_t s);
 cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, float* mb,
                          float* acc, cudaStream_t s);
+// wb (bf16 copy of w, may be NULL) is rewritten with the new weights.
 cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
-                        const AdamHp& hp, float* mb, float* acc, cudaStream_t s);
+                        const AdamHp& hp, float* mb, float* acc, void* wb, cudaStream_t s);
+cudaError_t launch_to_bf16(const float* w, void* wb, size_t n, cudaStream_t s);
 cudaError_t launch_finish(const float* acc, float* out, cudaStream_t s);
 // flat [W1|b1|W2|b2|W3|b3] <-> augmented [W1a|W2a|W3a] of one network
 cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int Hp, int out,
                            bool to_aug, cudaStream_t s);
-cudaError_t launch_fill_ones(float* buf, int ld, int col, int rows, cudaStream_t s);
+cudaError_t launch_fill_ones(bool bf16, void* buf, int ld, int col, int rows, cudaStream_t s);
 
 }  // namespace ppo
 

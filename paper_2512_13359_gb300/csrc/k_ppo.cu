@@ -10,6 +10,8 @@
 // runs their recursion, so that every warp keeps 3 kU coalesced loads in
 // flight (16-step blocks: 3.1 TB/s at 65,536 envs x 128 steps, 4.3 TB/s at
 // 262,144; 8- and 32-step blocks measured slower).
+#include <cuda_bf16.h>
+
 #include "auv_kernels.h"
 
 namespace auv {
@@ -83,6 +85,12 @@ namespace {
 constexpr int kT = 256;
 constexpr float kHalfLog2Pi = 0.91893853320467274f;
 
+// Activation storage: fp32, or bf16 (round to nearest even) in bf16 mode.
+__device__ __forceinline__ float ld_act(const float* p) { return *p; }
+__device__ __forceinline__ float ld_act(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void st_act(float* p, float x) { *p = x; }
+__device__ __forceinline__ void st_act(__nv_bfloat16* p, float x) { *p = __float2bfloat16_rn(x); }
+
 // Balanced Feistel network, four rounds; round j: (L, R) -> (R, L ^ F_j(R)),
 // F_j(R) = first Philox4x32-10 word at counter (R, j, epoch) and key seed.
 __device__ __forceinline__ uint32_t feistel(uint32_t x, const PermKey& p) {
@@ -128,23 +136,24 @@ __device__ __forceinline__ void block_sum(V (&v)[NV], V* sh /* [NV][kT/32] */) {
   __syncthreads();
 }
 
+template <typename TX>
 __global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, uint32_t start,
                                                const float* __restrict__ obs,
                                                const float* __restrict__ act,
                                                const float* __restrict__ logp,
                                                const float* __restrict__ adv,
                                                const float* __restrict__ ret, uint32_t N,
-                                               Sample out) {
+                                               Sample out, TX* __restrict__ X) {
   __shared__ double sh[2 * (kT / 32)];
   const int b = blockIdx.x * kT + threadIdx.x;
   double s[2] = {0.0, 0.0};
   if (b < d.B) {
     const uint32_t r = perm_index(start + (uint32_t)b, key);
     const size_t t = r / N, i = r - (uint32_t)t * N, n = N;
-    float* x = out.X + (size_t)b * d.Dp;
-    for (int k = 0; k < d.D; ++k) x[k] = __ldg(obs + (t * d.D + k) * n + i);
-    x[d.D] = 1.0f;
-    for (int k = d.D + 1; k < d.Dp; ++k) x[k] = 0.0f;
+    TX* x = X + (size_t)b * d.Dp;
+    for (int k = 0; k < d.D; ++k) st_act(x + k, __ldg(obs + (t * d.D + k) * n + i));
+    st_act(x + d.D, 1.0f);
+    for (int k = d.D + 1; k < d.Dp; ++k) st_act(x + k, 0.0f);
     for (int k = 0; k < d.A; ++k) out.act[(size_t)b * d.A + k] = __ldg(act + (t * d.A + k) * n + i);
     const size_t o = t * n + i;
     const float a = __ldg(adv + o);
@@ -172,6 +181,44 @@ __global__ void __launch_bounds__(kT) k_tanh_fwd(float* __restrict__ h, int ld, 
   }
 }
 
+__global__ void __launch_bounds__(kT) k_tanh_fwd_bf16(__nv_bfloat16* __restrict__ h, int ld,
+                                                      int B, int H8) {
+  const size_t n = (size_t)B * H8;
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const size_t row = e / H8, c = e - row * H8;
+    uint4* p = reinterpret_cast<uint4*>(h + row * ld) + c;
+    uint4 u = *p;
+    __nv_bfloat162* v = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 z = __bfloat1622float2(v[k]);
+      v[k] = __floats2bfloat162_rn(tanhf(z.x), tanhf(z.y));
+    }
+    *p = u;
+  }
+}
+
+__global__ void __launch_bounds__(kT) k_tanh_bwd_bf16(__nv_bfloat16* __restrict__ g, int ldg,
+                                                      const __nv_bfloat16* __restrict__ h,
+                                                      int ldh, int B, int H8) {
+  const size_t n = (size_t)B * H8;
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
+    const size_t row = e / H8, c = e - row * H8;
+    uint4* pg = reinterpret_cast<uint4*>(g + row * ldg) + c;
+    uint4 hv = __ldg(reinterpret_cast<const uint4*>(h + row * ldh) + c);
+    uint4 gv = *pg;
+    __nv_bfloat162* gg = reinterpret_cast<__nv_bfloat162*>(&gv);
+    const __nv_bfloat162* hh = reinterpret_cast<const __nv_bfloat162*>(&hv);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 y = __bfloat1622float2(hh[k]);
+      const float2 x = __bfloat1622float2(gg[k]);
+      gg[k] = __floats2bfloat162_rn(x.x * (1.0f - y.x * y.x), x.y * (1.0f - y.y * y.y));
+    }
+    *pg = gv;
+  }
+}
+
 __global__ void __launch_bounds__(kT) k_tanh_bwd(float* __restrict__ g, int ldg,
                                                  const float* __restrict__ h, int ldh, int B,
                                                  int H4) {
@@ -191,10 +238,11 @@ __global__ void __launch_bounds__(kT) k_tanh_bwd(float* __restrict__ g, int ldg,
 // entropy terms, and dL/d(head) for both networks (already divided by B).
 // Every block first reduces the gather's advantage partial sums, in the same
 // order, so that all blocks normalise with the same mean and deviation.
+template <typename TG>
 __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __restrict__ y,
                                              const float* __restrict__ v, Sample smp,
-                                             int n_part, float* __restrict__ g_y,
-                                             float* __restrict__ g_v, float* __restrict__ part) {
+                                             int n_part, TG* __restrict__ g_y,
+                                             TG* __restrict__ g_v, float* __restrict__ part) {
   __shared__ double shd[2 * (kT / 32)];
   __shared__ float shf[5 * (kT / 32)];
   __shared__ double norm[2];
@@ -216,7 +264,7 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
   if (b < d.B) {
     const float inv_b = 1.0f / (float)d.B;
     const int A = d.A;
-    const float* yb = y + (size_t)b * 2 * A;
+    const float* yb = y + (size_t)b * d.ld_pol;
     const float* ab = smp.act + (size_t)b * A;
     const float an = hp.norm_adv ? (float)(((double)smp.adv[b] - norm[0]) * norm[1]) : smp.adv[b];
     float dm[8], iv[8], z2[8];
@@ -240,16 +288,16 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
     const float lo = 1.0f - hp.clip_eps, hi = 1.0f + hp.clip_eps;
     const bool unclipped = an > 0.0f ? r <= hi : r >= lo;
     const float g_lp = unclipped ? -an * r * inv_b : 0.0f;
-    float* gy = g_y + (size_t)b * 2 * A;
+    TG* gy = g_y + (size_t)b * d.ld_pol;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       if (k < A) {
-        gy[k] = g_lp * dm[k] * iv[k];
-        gy[A + k] = in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f;
+        st_act(gy + k, g_lp * dm[k] * iv[k]);
+        st_act(gy + A + k, in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f);
       }
     }
-    const float dv = v[b] - smp.ret[b];
-    g_v[b] = hp.vf_coef * dv * inv_b;
+    const float dv = v[(size_t)b * d.ld_val] - smp.ret[b];
+    st_act(g_v + (size_t)b * d.ld_val, hp.vf_coef * dv * inv_b);
     st[0] = fmaxf(-an * r, -an * fminf(fmaxf(r, lo), hi));
     st[1] = 0.5f * dv * dv;
     st[2] = ent;
@@ -299,7 +347,8 @@ __global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_
 __global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float* __restrict__ g,
                                              float* __restrict__ m, float* __restrict__ v,
                                              size_t n, const float* __restrict__ part, AdamHp hp,
-                                             float* mb, float* acc) {
+                                             float* mb, float* acc,
+                                             __nv_bfloat16* __restrict__ wb) {
   __shared__ double sh[kT / 32];
   __shared__ float scale_sh;
   double s[1] = {0.0};
@@ -322,8 +371,16 @@ __global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float*
     const float vi = hp.b2 * v[e] + ib2 * gi * gi;
     m[e] = mi;
     v[e] = vi;
-    w[e] -= hp.lr * (mi / hp.c1) / (sqrtf(vi / hp.c2) + hp.eps);
+    const float wi = w[e] - hp.lr * (mi / hp.c1) / (sqrtf(vi / hp.c2) + hp.eps);
+    w[e] = wi;
+    if (wb) wb[e] = __float2bfloat16_rn(wi);
   }
+}
+
+__global__ void __launch_bounds__(kT) k_to_bf16(const float* __restrict__ w,
+                                                __nv_bfloat16* __restrict__ wb, size_t n) {
+  for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT)
+    wb[e] = __float2bfloat16_rn(w[e]);
 }
 
 __global__ void k_finish(const float* __restrict__ acc, float* __restrict__ out) {
@@ -365,11 +422,12 @@ __global__ void __launch_bounds__(kT) k_convert(float* flat, float* aug, size_t 
   }
 }
 
-__global__ void __launch_bounds__(kT) k_fill_ones(float* buf, int ld, int col, int rows) {
+template <typename TX>
+__global__ void __launch_bounds__(kT) k_fill_ones(TX* buf, int ld, int col, int rows) {
   for (int r = blockIdx.x * kT + threadIdx.x; r < rows; r += gridDim.x * kT) {
-    float* p = buf + (size_t)r * ld;
-    p[col] = 1.0f;
-    for (int c = col + 1; c < ld; ++c) p[c] = 0.0f;
+    TX* p = buf + (size_t)r * ld;
+    st_act(p + col, 1.0f);
+    for (int c = col + 1; c < ld; ++c) st_act(p + c, 0.0f);
   }
 }
 
@@ -386,26 +444,48 @@ size_t aug_count(int in, int in_p, int H, int Hp, int out) {
 
 cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
                           const float* act, const float* logp, const float* adv,
-                          const float* ret, uint32_t N, const Sample& out, cudaStream_t s) {
-  k_gather<<<(d.B + kT - 1) / kT, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out);
+                          const float* ret, uint32_t N, const Sample& out, void* X,
+                          cudaStream_t s) {
+  const unsigned nb = (d.B + kT - 1) / kT;
+  if (d.bf16)
+    k_gather<<<nb, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out,
+                               static_cast<__nv_bfloat16*>(X));
+  else
+    k_gather<<<nb, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out,
+                               static_cast<float*>(X));
   return cudaGetLastError();
 }
 
-cudaError_t launch_tanh_fwd(float* h, int ld, int B, int H, cudaStream_t s) {
-  k_tanh_fwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(h, ld, B, H / 4);
+cudaError_t launch_tanh_fwd(bool bf16, void* h, int ld, int B, int H, cudaStream_t s) {
+  if (bf16)
+    k_tanh_fwd_bf16<<<grid_for((size_t)B * H / 8), kT, 0, s>>>(static_cast<__nv_bfloat16*>(h), ld,
+                                                               B, H / 8);
+  else
+    k_tanh_fwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(static_cast<float*>(h), ld, B, H / 4);
   return cudaGetLastError();
 }
 
-cudaError_t launch_tanh_bwd(float* g, int ldg, const float* h, int ldh, int B, int H,
+cudaError_t launch_tanh_bwd(bool bf16, void* g, int ldg, const void* h, int ldh, int B, int H,
                             cudaStream_t s) {
-  k_tanh_bwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(g, ldg, h, ldh, B, H / 4);
+  if (bf16)
+    k_tanh_bwd_bf16<<<grid_for((size_t)B * H / 8), kT, 0, s>>>(
+        static_cast<__nv_bfloat16*>(g), ldg, static_cast<const __nv_bfloat16*>(h), ldh, B, H / 8);
+  else
+    k_tanh_bwd<<<grid_for((size_t)B * H / 4), kT, 0, s>>>(static_cast<float*>(g), ldg,
+                                                          static_cast<const float*>(h), ldh, B,
+                                                          H / 4);
   return cudaGetLastError();
 }
 
 cudaError_t launch_head(const Dims& d, const LossHp& hp, const float* y, const float* v,
-                        const Sample& smp, float* g_y, float* g_v, float* part, cudaStream_t s) {
+                        const Sample& smp, void* g_y, void* g_v, float* part, cudaStream_t s) {
   const int nb = (d.B + kT - 1) / kT;
-  k_head<<<nb, kT, 0, s>>>(d, hp, y, v, smp, nb, g_y, g_v, part);
+  if (d.bf16)
+    k_head<<<nb, kT, 0, s>>>(d, hp, y, v, smp, nb, static_cast<__nv_bfloat16*>(g_y),
+                             static_cast<__nv_bfloat16*>(g_v), part);
+  else
+    k_head<<<nb, kT, 0, s>>>(d, hp, y, v, smp, nb, static_cast<float*>(g_y),
+                             static_cast<float*>(g_v), part);
   return cudaGetLastError();
 }
 
@@ -416,9 +496,15 @@ cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, flo
 }
 
 cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
-                        const AdamHp& hp, float* mb, float* acc, cudaStream_t s) {
+                        const AdamHp& hp, float* mb, float* acc, void* wb, cudaStream_t s) {
   k_sumsq<<<kNormBlocks, kT, 0, s>>>(g, n, part);
-  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, mb, acc);
+  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, mb, acc,
+                                    static_cast<__nv_bfloat16*>(wb));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_to_bf16(const float* w, void* wb, size_t n, cudaStream_t s) {
+  k_to_bf16<<<grid_for(n), kT, 0, s>>>(w, static_cast<__nv_bfloat16*>(wb), n);
   return cudaGetLastError();
 }
 
@@ -434,8 +520,12 @@ cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_fill_ones(float* buf, int ld, int col, int rows, cudaStream_t s) {
-  k_fill_ones<<<grid_for((size_t)rows), kT, 0, s>>>(buf, ld, col, rows);
+cudaError_t launch_fill_ones(bool bf16, void* buf, int ld, int col, int rows, cudaStream_t s) {
+  if (bf16)
+    k_fill_ones<<<grid_for((size_t)rows), kT, 0, s>>>(static_cast<__nv_bfloat16*>(buf), ld, col,
+                                                      rows);
+  else
+    k_fill_ones<<<grid_for((size_t)rows), kT, 0, s>>>(static_cast<float*>(buf), ld, col, rows);
   return cudaGetLastError();
 }
 

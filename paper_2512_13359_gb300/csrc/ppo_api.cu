@@ -2,15 +2,19 @@
 // validation, the learner's device memory, and the sequence of one gradient
 // step: gather -> forward GEMMs + tanh -> loss head -> backward GEMMs + tanh'
 // -> (gradient norm, Adam).  The dense products are plain GEMMs and run in
-// cuBLAS (fp32, tf32 or bf16 tensor-core compute on fp32 data); every other
-// step runs in the kernels of k_ppo.cu.
+// cuBLAS; every other step runs in the kernels of k_ppo.cu.  Precision modes:
+//   fp32  fp32 activations, fp32 GEMMs on the CUDA cores;
+//   tf32  fp32 activations, tensor-core GEMMs with tf32 operands;
+//   bf16  bf16 activations, backward signals and weight copy (the GEMM
+//         operands), tensor-core GEMMs with fp32 sums; the heads' outputs
+//         and the weight gradients stay fp32, as do the master weights.
 //
 // Memory layout (one cudaMalloc): master weights, gradient and Adam moments
-// as augmented vectors [policy | value] (auv_kernels.h, ppo::Dims), a flat
-// staging vector, the gathered minibatch, and per network the activations
-// H1, H2 [B][Hp] (constant 1 at column H), the backward buffer G [B][H] and
-// the head output Y [B][out].  Everything a step touches is resident; no call
-// after ppo_create allocates.
+// as augmented vectors [policy | value] (auv_kernels.h, ppo::Dims), the bf16
+// weight copy, a flat staging vector, the gathered minibatch, and per
+// network the activations H1, H2 [B][Hp] (constant 1 at column H), the
+// backward buffer G [B][H] and the head output Y [B][ld].  Everything a step
+// touches is resident; no call after ppo_create allocates.
 #include <cublas_v2.h>
 
 #include <cmath>
@@ -33,11 +37,17 @@ struct auv_ppo {
   int out[2];                 // head widths: 2A (policy), 1 (value)
   size_t n_flat[2], n_aug[2], n_aug_all;
   char* mem;
+  bool bf16;
+  cudaDataType_t act_t;       // storage type of X, H1, H2, G, dL/d(head)
+  size_t esz;                 // its size in bytes
   float *w, *g, *m, *v;       // augmented [policy | value]
+  void* wb;                   // bf16 copy of w (bf16 mode)
   float* flat;                // staging, flat [policy | value]
   ppo::Sample smp;
-  float *h1[2], *h2[2], *gb[2], *y[2];
-  float *g_y, *g_v;           // dL/d(head) [B][2A], [B]
+  void* X;                    // [B][Dp]
+  void *h1[2], *h2[2], *gb[2];
+  float* y[2];                // head outputs [B][ld_pol], [B][ld_val]
+  void *g_y, *g_v;            // dL/d(head), same shapes
   float *head_part, *norm_part;
   float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
   void* blas_ws;
@@ -67,7 +77,7 @@ int blas_fail(auv_ppo* p, cublasStatus_t e, const char* what) {
   return fail(p, AUV_ERR_CUDA, "%s: cuBLAS status %d", what, (int)e);
 }
 
-int round4(int x) { return (x + 3) & ~3; }
+int round8(int x) { return (x + 7) & ~7; }
 
 bool is_device(const void* q) {
   cudaPointerAttributes a;
@@ -155,14 +165,25 @@ ppo::LossHp loss_hp(const auv_ppo* p) {
   return {c.clip_eps, c.vf_coef, c.ent_coef, c.logstd_min, c.logstd_max, (int)c.norm_adv};
 }
 
+// C = op(A) op(B) with A, B in the activation type; C in that type too
+// (c32 = false) or fp32 (c32 = true).
 cublasStatus_t gemm(auv_ppo* p, cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
-                    const float* A, int lda, const float* B, int ldb, float* C, int ldc) {
+                    const void* A, int lda, const void* B, int ldb, void* C, int ldc, bool c32) {
   const float one = 1.0f, zero = 0.0f;
-  return cublasGemmEx(p->blas, ta, tb, m, n, k, &one, A, CUDA_R_32F, lda, B, CUDA_R_32F, ldb,
-                      &zero, C, CUDA_R_32F, ldc, p->ctype, CUBLAS_GEMM_DEFAULT);
+  return cublasGemmEx(p->blas, ta, tb, m, n, k, &one, A, p->act_t, lda, B, p->act_t, ldb, &zero, C,
+                      c32 ? CUDA_R_32F : p->act_t, ldc, p->ctype, CUBLAS_GEMM_DEFAULT);
 }
 
 size_t net_offset(const auv_ppo* p, int net) { return net ? p->n_aug[0] : 0; }
+
+// The GEMM operand copy of network `net`'s augmented weights.
+const char* weights_for_gemm(const auv_ppo* p, int net) {
+  const size_t o = net_offset(p, net);
+  return p->bf16 ? static_cast<const char*>(p->wb) + o * 2
+                 : reinterpret_cast<const char*>(p->w + o);
+}
+
+int ld_head(const auv_ppo* p, int net) { return net ? p->d.ld_val : p->d.ld_pol; }
 
 // Column-major view (cuBLAS): a sample-major [B][ld] array is an ld x B
 // matrix; a row-major weight [out][in_p] is an in_p x out matrix.
@@ -170,46 +191,55 @@ size_t net_offset(const auv_ppo* p, int net) { return net ? p->n_aug[0] : 0; }
 //   gW3a = H2 gY^T, gH2 = W3 gY, gW2a = H1 gZ2^T, gH1 = W2 gZ2, gW1a = X gZ1^T
 int forward(auv_ppo* p, int net, cudaStream_t s) {
   const ppo::Dims& d = p->d;
-  const float* w = p->w + net_offset(p, net);
-  const float *w1 = w, *w2 = w + (size_t)d.H * d.Dp, *w3 = w2 + (size_t)d.H * d.Hp;
+  const size_t es = p->esz;
+  const char* w = weights_for_gemm(p, net);
+  const char *w1 = w, *w2 = w + (size_t)d.H * d.Dp * es, *w3 = w2 + (size_t)d.H * d.Hp * es;
   cublasStatus_t bs;
   cudaError_t e;
-  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Dp, w1, d.Dp, p->smp.X, d.Dp, p->h1[net], d.Hp)))
+  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Dp, w1, d.Dp, p->X, d.Dp, p->h1[net],
+                 d.Hp, false)))
     return blas_fail(p, bs, "forward layer 1");
-  if ((e = ppo::launch_tanh_fwd(p->h1[net], d.Hp, d.B, d.H, s))) return cuda_fail(p, e, "tanh 1");
-  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp, p->h2[net], d.Hp)))
+  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h1[net], d.Hp, d.B, d.H, s)))
+    return cuda_fail(p, e, "tanh 1");
+  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp,
+                 p->h2[net], d.Hp, false)))
     return blas_fail(p, bs, "forward layer 2");
-  if ((e = ppo::launch_tanh_fwd(p->h2[net], d.Hp, d.B, d.H, s))) return cuda_fail(p, e, "tanh 2");
+  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h2[net], d.Hp, d.B, d.H, s)))
+    return cuda_fail(p, e, "tanh 2");
   if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Hp,
-                 p->y[net], p->out[net])))
+                 p->y[net], ld_head(p, net), true)))
     return blas_fail(p, bs, "forward layer 3");
   return AUV_OK;
 }
 
-int backward(auv_ppo* p, int net, const float* gy, cudaStream_t s) {
+int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
   const ppo::Dims& d = p->d;
-  const int out = p->out[net];
-  const float* w = p->w + net_offset(p, net);
-  const float *w2 = w + (size_t)d.H * d.Dp, *w3 = w2 + (size_t)d.H * d.Hp;
+  const size_t es = p->esz;
+  const int out = p->out[net], ldy = ld_head(p, net);
+  const char* w = weights_for_gemm(p, net);
+  const char *w2 = w + (size_t)d.H * d.Dp * es, *w3 = w2 + (size_t)d.H * d.Hp * es;
   float* g = p->g + net_offset(p, net);
   float *g1 = g, *g2 = g + (size_t)d.H * d.Dp, *g3 = g2 + (size_t)d.H * d.Hp;
-  float* gz2 = p->gb[net];
-  float* gz1 = p->h2[net];      // H2 is dead once gZ2 exists
+  void* gz2 = p->gb[net];
+  void* gz1 = p->h2[net];       // H2 is dead once gZ2 exists
   cublasStatus_t bs;
   cudaError_t e;
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, out, d.B, p->h2[net], d.Hp, gy, out, g3, d.Hp)))
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, out, d.B, p->h2[net], d.Hp, gy, ldy, g3, d.Hp,
+                 true)))
     return blas_fail(p, bs, "gradient W3");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, out, w3, d.Hp, gy, out, gz2, d.H)))
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, out, w3, d.Hp, gy, ldy, gz2, d.H, false)))
     return blas_fail(p, bs, "gradient H2");
-  if ((e = ppo::launch_tanh_bwd(gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_bwd(p->bf16, gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 2");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp)))
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+                 true)))
     return blas_fail(p, bs, "gradient W2");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp)))
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp, false)))
     return blas_fail(p, bs, "gradient H1");
-  if ((e = ppo::launch_tanh_bwd(gz1, d.Hp, p->h1[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_bwd(p->bf16, gz1, d.Hp, p->h1[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 1");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->smp.X, d.Dp, gz1, d.Hp, g1, d.Dp)))
+  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+                 true)))
     return blas_fail(p, bs, "gradient W1");
   return AUV_OK;
 }
@@ -219,7 +249,7 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, uint64_t epoch, uint32_t j, f
   const ppo::Dims& d = p->d;
   const uint32_t m = b->T * b->N;
   cudaError_t e = ppo::launch_gather(d, perm_key(p, m, epoch), j * (uint32_t)d.B, b->obs, b->act,
-                                     b->logp, b->adv, b->ret, b->N, p->smp, s);
+                                     b->logp, b->adv, b->ret, b->N, p->smp, p->X, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "gather");
   int rc;
   if ((rc = forward(p, 0, s)) || (rc = forward(p, 1, s))) return rc;
@@ -245,7 +275,7 @@ int apply_impl(auv_ppo* p, float* acc, cudaStream_t s) {
   if (!(hp.c1 > 0.0f)) hp.c1 = 1.0f;   // beta1 = 0 keeps the plain moment
   if (!(hp.c2 > 0.0f)) hp.c2 = 1.0f;
   cudaError_t e = ppo::launch_adam(p->w, p->g, p->m, p->v, p->n_aug_all, p->norm_part, hp, p->mb,
-                                   acc, s);
+                                   acc, p->wb, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "Adam");
   p->t = t;
   return AUV_OK;
@@ -271,6 +301,8 @@ int load_pair(auv_ppo* p, const float* pol, const float* val, float* dst, cudaSt
   if (e != cudaSuccess) return cuda_fail(p, e, "copy in");
   int rc = convert(p, p->flat, p->flat + p->n_flat[0], dst, true, s);
   if (rc) return rc;
+  if (dst == p->w && p->bf16 && (e = ppo::launch_to_bf16(p->w, p->wb, p->n_aug_all, s)))
+    return cuda_fail(p, e, "bf16 weight copy");
   e = cudaStreamSynchronize(s);
   return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "synchronise");
 }
@@ -302,11 +334,17 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   cudaGetDevice(&p->device);
   ppo::Dims& d = p->d;
   d.D = (int)cfg->obs_dim;
-  d.Dp = round4(d.D + 1);
+  d.Dp = round8(d.D + 1);     // rows of 16-byte multiples in fp32 and bf16
   d.A = (int)cfg->act_dim;
   d.H = (int)cfg->hidden;
-  d.Hp = round4(d.H + 1);
+  d.Hp = round8(d.H + 1);
   d.B = (int)cfg->minibatch;
+  d.ld_pol = round8(2 * d.A);
+  d.ld_val = 8;
+  d.bf16 = cfg->precision == AUV_PPO_BF16;
+  p->bf16 = d.bf16 != 0;
+  p->act_t = p->bf16 ? CUDA_R_16BF : CUDA_R_32F;
+  p->esz = p->bf16 ? 2 : 4;
   p->out[0] = 2 * d.A;
   p->out[1] = 1;
   for (int k = 0; k < 2; ++k) {
@@ -315,9 +353,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     p->n_aug[k] = ppo::aug_count(d.D, d.Dp, d.H, d.Hp, p->out[k]);
   }
   p->n_aug_all = p->n_aug[0] + p->n_aug[1];
-  p->ctype = cfg->precision == AUV_PPO_FP32   ? CUBLAS_COMPUTE_32F
-             : cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32
-                                              : CUBLAS_COMPUTE_32F_FAST_16BF;
+  p->ctype = cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
   // one allocation, 256-byte aligned pieces
   const size_t B = (size_t)d.B, nb = (B + 255) / 256;
   size_t off = 0;
@@ -326,20 +362,22 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     off += (bytes + 255) & ~(size_t)255;
     return o;
   };
+  const size_t es = p->esz;
   const size_t o_w = take(p->n_aug_all * 4), o_g = take(p->n_aug_all * 4),
                o_m = take(p->n_aug_all * 4), o_v = take(p->n_aug_all * 4),
-               o_flat = take((p->n_flat[0] + p->n_flat[1]) * 4), o_x = take(B * d.Dp * 4),
+               o_wb = take(p->bf16 ? p->n_aug_all * 2 : 0),
+               o_flat = take((p->n_flat[0] + p->n_flat[1]) * 4), o_x = take(B * d.Dp * es),
                o_act = take(B * d.A * 4), o_lp = take(B * 4), o_adv = take(B * 4),
-               o_ret = take(B * 4), o_ap = take(nb * 2 * 8), o_gy = take(B * 2 * d.A * 4),
-               o_gv = take(B * 4), o_hp = take(nb * 5 * 4), o_np = take(ppo::kNormBlocks * 4),
-               o_mb = take(AUV_PPO_STATS * 4), o_acc = take(AUV_PPO_STATS * 4),
-               o_ws = take(kBlasWorkspace);
+               o_ret = take(B * 4), o_ap = take(nb * 2 * 8), o_gy = take(B * d.ld_pol * es),
+               o_gv = take(B * d.ld_val * es), o_hp = take(nb * 5 * 4),
+               o_np = take(ppo::kNormBlocks * 4), o_mb = take(AUV_PPO_STATS * 4),
+               o_acc = take(AUV_PPO_STATS * 4), o_ws = take(kBlasWorkspace);
   size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
   for (int k = 0; k < 2; ++k) {
-    o_h1[k] = take(B * d.Hp * 4);
-    o_h2[k] = take(B * d.Hp * 4);
-    o_gb[k] = take(B * d.H * 4);
-    o_y[k] = take(B * p->out[k] * 4);
+    o_h1[k] = take(B * d.Hp * es);
+    o_h2[k] = take(B * d.Hp * es);
+    o_gb[k] = take(B * d.H * es);
+    o_y[k] = take(B * (k ? d.ld_val : d.ld_pol) * 4);
   }
   cudaError_t e = cudaMalloc(&p->mem, off);
   if (e != cudaSuccess) {
@@ -351,30 +389,31 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   p->g = reinterpret_cast<float*>(base + o_g);
   p->m = reinterpret_cast<float*>(base + o_m);
   p->v = reinterpret_cast<float*>(base + o_v);
+  p->wb = p->bf16 ? base + o_wb : nullptr;
   p->flat = reinterpret_cast<float*>(base + o_flat);
-  p->smp.X = reinterpret_cast<float*>(base + o_x);
+  p->X = base + o_x;
   p->smp.act = reinterpret_cast<float*>(base + o_act);
   p->smp.logp = reinterpret_cast<float*>(base + o_lp);
   p->smp.adv = reinterpret_cast<float*>(base + o_adv);
   p->smp.ret = reinterpret_cast<float*>(base + o_ret);
   p->smp.adv_part = reinterpret_cast<double*>(base + o_ap);
-  p->g_y = reinterpret_cast<float*>(base + o_gy);
-  p->g_v = reinterpret_cast<float*>(base + o_gv);
+  p->g_y = base + o_gy;
+  p->g_v = base + o_gv;
   p->head_part = reinterpret_cast<float*>(base + o_hp);
   p->norm_part = reinterpret_cast<float*>(base + o_np);
   p->mb = reinterpret_cast<float*>(base + o_mb);
   p->acc = reinterpret_cast<float*>(base + o_acc);
   p->blas_ws = base + o_ws;
   for (int k = 0; k < 2; ++k) {
-    p->h1[k] = reinterpret_cast<float*>(base + o_h1[k]);
-    p->h2[k] = reinterpret_cast<float*>(base + o_h2[k]);
-    p->gb[k] = reinterpret_cast<float*>(base + o_gb[k]);
+    p->h1[k] = base + o_h1[k];
+    p->h2[k] = base + o_h2[k];
+    p->gb[k] = base + o_gb[k];
     p->y[k] = reinterpret_cast<float*>(base + o_y[k]);
   }
   e = cudaMemset(p->mem, 0, off);
   for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
-    e = ppo::launch_fill_ones(p->h1[k], d.Hp, d.H, d.B, 0);
-    if (e == cudaSuccess) e = ppo::launch_fill_ones(p->h2[k], d.Hp, d.H, d.B, 0);
+    e = ppo::launch_fill_ones(p->bf16, p->h1[k], d.Hp, d.H, d.B, 0);
+    if (e == cudaSuccess) e = ppo::launch_fill_ones(p->bf16, p->h2[k], d.Hp, d.H, d.B, 0);
   }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
