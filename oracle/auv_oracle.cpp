@@ -233,6 +233,56 @@ ResetDraw reset_draw(const OracleModel& m, uint32_t env_id, uint32_t episode) {
 // ----------------------------------------------------------------------------
 // Rigid-body kinematics helpers (Hamilton quaternion, body -> world).
 // ----------------------------------------------------------------------------
+// ----------------------------------------------------------------------------
+// Forward-mode automatic differentiation: a dual number v + d e (e^2 = 0)
+// carries a value and its derivative along one direction through every
+// operation of the templated model code below, so that running the model in
+// Dual yields the exact directional derivative of any output (the oracle of
+// the adjoint kernels).  Comparisons look at the value only.  The model's
+// math calls are unqualified so that double and float keep std:: and Dual
+// finds the rules here.
+// ----------------------------------------------------------------------------
+using std::atan2;
+using std::cos;
+using std::fabs;
+using std::sin;
+using std::sqrt;
+
+struct Dual {
+  double v, d;
+  Dual(double x = 0.0) : v(x), d(0.0) {}
+  Dual(double x, double dx) : v(x), d(dx) {}
+  explicit operator double() const { return v; }
+  explicit operator float() const { return (float)v; }
+};
+inline Dual operator+(Dual a, Dual b) { return Dual(a.v + b.v, a.d + b.d); }
+inline Dual operator-(Dual a, Dual b) { return Dual(a.v - b.v, a.d - b.d); }
+inline Dual operator-(Dual a) { return Dual(-a.v, -a.d); }
+inline Dual operator*(Dual a, Dual b) { return Dual(a.v * b.v, a.d * b.v + a.v * b.d); }
+inline Dual operator/(Dual a, Dual b) {
+  return Dual(a.v / b.v, (a.d * b.v - a.v * b.d) / (b.v * b.v));
+}
+inline Dual& operator+=(Dual& a, Dual b) { return a = a + b; }
+inline Dual& operator-=(Dual& a, Dual b) { return a = a - b; }
+inline Dual& operator*=(Dual& a, Dual b) { return a = a * b; }
+inline Dual& operator/=(Dual& a, Dual b) { return a = a / b; }
+inline bool operator<(Dual a, Dual b) { return a.v < b.v; }
+inline bool operator>(Dual a, Dual b) { return a.v > b.v; }
+inline bool operator<=(Dual a, Dual b) { return a.v <= b.v; }
+inline bool operator>=(Dual a, Dual b) { return a.v >= b.v; }
+inline bool operator==(Dual a, Dual b) { return a.v == b.v; }
+inline bool operator!=(Dual a, Dual b) { return a.v != b.v; }
+inline Dual sqrt(Dual a) {
+  const double s = std::sqrt(a.v);
+  return Dual(s, a.d == 0.0 ? 0.0 : a.d / (2.0 * s));
+}
+inline Dual fabs(Dual a) { return a.v < 0.0 ? -a : a; }
+inline Dual sin(Dual a) { return Dual(std::sin(a.v), std::cos(a.v) * a.d); }
+inline Dual cos(Dual a) { return Dual(std::cos(a.v), -std::sin(a.v) * a.d); }
+inline Dual atan2(Dual y, Dual x) {
+  return Dual(std::atan2(y.v, x.v), (x.v * y.d - y.v * x.d) / (x.v * x.v + y.v * y.v));
+}
+
 template <class R>
 void quat_to_rot(const R q[4], R Rm[3][3]) {
   R w = q[0], x = q[1], y = q[2], z = q[3];
@@ -342,14 +392,14 @@ void nu_dot(const OracleModel& m, const Env<R>& e, const R q[4], const R nu[6],
   }
   // Linear plus quadratic damping on the relative velocity.
   R damp[6];
-  for (int k = 0; k < 6; ++k) damp[k] = (dl[k] + dq[k] * std::fabs(nur[k])) * nur[k];
+  for (int k = 0; k < 6; ++k) damp[k] = (dl[k] + dq[k] * fabs(nur[k])) * nur[k];
   // Restoring forces: weight W at the CoG (origin), buoyancy B = W + dB at r_b.
   // With k = R^T g_hat the body-frame gravity direction, the net force is
   // W k - B k = -dB k and the buoyancy moment is r_b x (-B k).
   R rest[6];
   {
     const R g[3] = {(R)m.gravity[0], (R)m.gravity[1], (R)m.gravity[2]};
-    const R gnorm = std::sqrt(g[0] * g[0] + g[1] * g[1] + g[2] * g[2]);
+    const R gnorm = sqrt(g[0] * g[0] + g[1] * g[1] + g[2] * g[2]);
     R kb[3] = {0, 0, 0};
     if (gnorm > 0) {
       const R ghat[3] = {g[0] / gnorm, g[1] / gnorm, g[2] / gnorm};
@@ -381,14 +431,14 @@ void nu_dot(const OracleModel& m, const Env<R>& e, const R q[4], const R nu[6],
 // Exponential map of a rotation vector phi = h w as a unit quaternion.
 template <class R>
 void quat_exp(const R phi[3], R dq[4]) {
-  R ang = std::sqrt(phi[0] * phi[0] + phi[1] * phi[1] + phi[2] * phi[2]);
+  R ang = sqrt(phi[0] * phi[0] + phi[1] * phi[1] + phi[2] * phi[2]);
   if (ang == 0) {
     dq[0] = 1; dq[1] = dq[2] = dq[3] = 0;
     return;
   }
   R half = ang / 2;
-  R s = std::sin(half) / ang;
-  dq[0] = std::cos(half);
+  R s = sin(half) / ang;
+  dq[0] = cos(half);
   dq[1] = s * phi[0]; dq[2] = s * phi[1]; dq[3] = s * phi[2];
 }
 
@@ -410,7 +460,7 @@ void substep(const OracleModel& m, Env<R>& e, const R tau[6], R h) {
   R dq[4], qn[4];
   quat_exp(phi, dq);
   quat_mul(e.q, dq, qn);
-  R n = std::sqrt(qn[0] * qn[0] + qn[1] * qn[1] + qn[2] * qn[2] + qn[3] * qn[3]);
+  R n = sqrt(qn[0] * qn[0] + qn[1] * qn[1] + qn[2] * qn[2] + qn[3] * qn[3]);
   for (int k = 0; k < 4; ++k) e.q[k] = qn[k] / n;
 }
 
@@ -443,8 +493,8 @@ R attitude_angle(const Env<R>& e) {
   const R qdc[4] = {e.q_d[0], -e.q_d[1], -e.q_d[2], -e.q_d[3]};
   R qe[4];
   quat_mul(qdc, e.q, qe);
-  R vn = std::sqrt(qe[1] * qe[1] + qe[2] * qe[2] + qe[3] * qe[3]);
-  return 2 * std::atan2(vn, std::fabs(qe[0]));
+  R vn = sqrt(qe[1] * qe[1] + qe[2] * qe[2] + qe[3] * qe[3]);
+  return 2 * atan2(vn, fabs(qe[0]));
 }
 
 // Reward: -w_pos ||dp|| - w_att theta_e - w_act ||a_c||^2 - w_vs ||nu - nu_prev||^2,
@@ -457,7 +507,7 @@ R reward(const OracleModel& m, const Env<R>& e, const R a_c[kAct]) {
   for (int k = 0; k < kAct; ++k) a2 += a_c[k] * a_c[k];
   R v2 = 0;
   for (int k = 0; k < 6; ++k) v2 += (e.nu[k] - e.nu_prev[k]) * (e.nu[k] - e.nu_prev[k]);
-  return -(R)m.w_pos * std::sqrt(d2) - (R)m.w_att * attitude_angle(e) -
+  return -(R)m.w_pos * sqrt(d2) - (R)m.w_att * attitude_angle(e) -
          (R)m.w_act * a2 - (R)m.w_vs * v2;
 }
 
@@ -797,9 +847,9 @@ void paper_apply_reset(const PaperModel& m, uint32_t env_id, PaperEnv<R>& e) {
 template <class R>
 void paper_box(const PaperModel& m, R b[3]) {
   const R I0 = (R)m.inertia[0], I1 = (R)m.inertia[1], I2 = (R)m.inertia[2], M = (R)m.mass;
-  b[0] = std::sqrt(6 * (I1 + I2 - I0) / M);
-  b[1] = std::sqrt(6 * (I0 + I2 - I1) / M);
-  b[2] = std::sqrt(6 * (I0 + I1 - I2) / M);
+  b[0] = sqrt(6 * (I1 + I2 - I0) / M);
+  b[1] = sqrt(6 * (I0 + I2 - I1) / M);
+  b[2] = sqrt(6 * (I0 + I1 - I2) / M);
 }
 
 // Hydrodynamic wrench on the box moving with body velocity nu in still water,
@@ -818,10 +868,10 @@ void paper_fluid(const PaperModel& m, const R nu[6], R f[6]) {
   for (int k = 0; k < 3; ++k) {
     const int j = (k + 1) % 3, l = (k + 2) % 3;
     const R v = nu[k], w = nu[3 + k];
-    const R drag_f = -(R)0.5 * rho * area[k] * std::fabs(v) * v;
+    const R drag_f = -(R)0.5 * rho * area[k] * fabs(v) * v;
     const R visc_f = -3 * pi * mu * d * v;
     const R b4 = b[j] * b[j] * b[j] * b[j] + b[l] * b[l] * b[l] * b[l];
-    const R drag_t = -rho / 64 * b[k] * b4 * std::fabs(w) * w;
+    const R drag_t = -rho / 64 * b[k] * b4 * fabs(w) * w;
     const R visc_t = -pi * mu * d * d * d * w;
     f[k] = drag_f + visc_f;
     f[3 + k] = drag_t + visc_t;
@@ -868,7 +918,7 @@ void paper_substep(const PaperModel& m, PaperEnv<R>& e, const R tau[6], R h) {
   R dq[4], qn[4];
   quat_exp(phi, dq);
   quat_mul(e.q, dq, qn);
-  R n = std::sqrt(qn[0] * qn[0] + qn[1] * qn[1] + qn[2] * qn[2] + qn[3] * qn[3]);
+  R n = sqrt(qn[0] * qn[0] + qn[1] * qn[1] + qn[2] * qn[2] + qn[3] * qn[3]);
   for (int k = 0; k < 4; ++k) e.q[k] = qn[k] / n;
 }
 
@@ -881,8 +931,8 @@ void paper_att_error(const PaperEnv<R>& e, R out[3]) {
   quat_mul(qdc, e.q, qe);
   if (qe[0] < 0)
     for (int k = 0; k < 4; ++k) qe[k] = -qe[k];
-  const R vn = std::sqrt(qe[1] * qe[1] + qe[2] * qe[2] + qe[3] * qe[3]);
-  const R s = vn > 0 ? 2 * std::atan2(vn, qe[0]) / vn : 2 / qe[0];
+  const R vn = sqrt(qe[1] * qe[1] + qe[2] * qe[2] + qe[3] * qe[3]);
+  const R s = vn > 0 ? 2 * atan2(vn, qe[0]) / vn : 2 / qe[0];
   for (int k = 0; k < 3; ++k) out[k] = s * qe[1 + k];
 }
 
@@ -1191,6 +1241,41 @@ void oracle_replay(const OracleModel* m, int precision, int n, const uint32_t* e
     replay_impl<double>(*m, n, env_ids, st, pr, t_ep, ep, T, act, rew, done, trace);
 }
 
+// Action-replay window objective J = sum_t coef[t] r_t + sum_k lam_T[k] x_T[k]
+// (x = p, q, nu after the last step; lam_T may be NULL) from the batch's
+// state, and its directional derivative along (dir_s0 on x_0 = p, q, nu;
+// dir_act on the actions), computed in Dual.  The batch is not modified.
+void oracle_adjoint_window(const OracleModel* m, int n, const uint32_t* env_ids,
+                           const double* st, const double* pr, const int32_t* t_ep,
+                           const uint32_t* ep, int T, const double* act, const double* coef,
+                           const double* lam_T, const double* dir_s0, const double* dir_act,
+                           double* J, double* dJ) {
+  for (int i = 0; i < n; ++i) {
+    Env<Dual> e;
+    load_env<Dual>(st, pr, t_ep, ep, n, i, e);
+    for (int k = 0; k < 3; ++k) e.p[k].d = dir_s0[(0 + k) * n + i];
+    for (int k = 0; k < 4; ++k) e.q[k].d = dir_s0[(3 + k) * n + i];
+    for (int k = 0; k < 6; ++k) e.nu[k].d = dir_s0[(7 + k) * n + i];
+    Dual obj = 0.0;
+    for (int t = 0; t < T; ++t) {
+      Dual a[kAct];
+      for (int k = 0; k < kAct; ++k) {
+        const size_t o = ((size_t)t * kAct + k) * n + i;
+        a[k] = Dual(act[o], dir_act[o]);
+      }
+      uint8_t d;
+      obj += Dual(coef[t]) * control_step(*m, env_ids[i], e, a, &d);
+    }
+    if (lam_T) {
+      for (int k = 0; k < 3; ++k) obj += Dual(lam_T[(0 + k) * n + i]) * e.p[k];
+      for (int k = 0; k < 4; ++k) obj += Dual(lam_T[(3 + k) * n + i]) * e.q[k];
+      for (int k = 0; k < 6; ++k) obj += Dual(lam_T[(7 + k) * n + i]) * e.nu[k];
+    }
+    J[i] = obj.v;
+    dJ[i] = obj.d;
+  }
+}
+
 void oracle_rollout(const OracleModel* m, int precision, const float* pol_w,
                     const float* val_w, int n, const uint32_t* env_ids, double* st,
                     double* pr, int32_t* t_ep, uint32_t* ep, uint64_t t_g0, int T,
@@ -1271,7 +1356,7 @@ void oracle_integrate(const OracleModel* m, int method, double* st, const double
       for (int k = 0; k < 13; ++k) yt[k] = y[k] + h * k3[k];
       rk4_deriv(*m, e, yt, tau, k4);
       for (int k = 0; k < 13; ++k) y[k] = y[k] + h / 6 * (k1[k] + 2 * k2[k] + 2 * k3[k] + k4[k]);
-      double qn = std::sqrt(y[3] * y[3] + y[4] * y[4] + y[5] * y[5] + y[6] * y[6]);
+      double qn = sqrt(y[3] * y[3] + y[4] * y[4] + y[5] * y[5] + y[6] * y[6]);
       for (int k = 0; k < 3; ++k) e.p[k] = y[k];
       for (int k = 0; k < 4; ++k) e.q[k] = y[3 + k] / qn;
       for (int k = 0; k < 6; ++k) e.nu[k] = y[7 + k];
@@ -1373,7 +1458,7 @@ void oracle_paper_integrate(const PaperModel* m, int method, double* st, const d
       for (int k = 0; k < 13; ++k) yt[k] = y[k] + h * k3[k];
       paper_rk4_deriv(*m, e, yt, tau, k4);
       for (int k = 0; k < 13; ++k) y[k] = y[k] + h / 6 * (k1[k] + 2 * k2[k] + 2 * k3[k] + k4[k]);
-      double qn = std::sqrt(y[3] * y[3] + y[4] * y[4] + y[5] * y[5] + y[6] * y[6]);
+      double qn = sqrt(y[3] * y[3] + y[4] * y[4] + y[5] * y[5] + y[6] * y[6]);
       for (int k = 0; k < 3; ++k) e.p[k] = y[k];
       for (int k = 0; k < 4; ++k) e.q[k] = y[3 + k] / qn;
       for (int k = 0; k < 6; ++k) e.nu[k] = y[7 + k];

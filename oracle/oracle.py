@@ -56,6 +56,8 @@ def lib():
         P = C.c_void_p
         _lib.oracle_model_size.restype = C.c_int
         _lib.oracle_philox.argtypes = [C.c_uint32, C.c_uint32, P, P]
+        _lib.oracle_adjoint_window.argtypes = [C.POINTER(OracleModel), C.c_int, P, P, P, P, P,
+                                               C.c_int, P, P, P, P, P, P, P]
         _lib.oracle_minibatch_perm.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32,
                                                C.c_uint32, P]
         _lib.oracle_feistel.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.c_uint64, C.c_int]
@@ -144,6 +146,29 @@ def reset(m: OracleModel, batch: Batch) -> Batch:
     lib().oracle_reset(C.byref(m), batch.n, _p(batch.env_ids), _p(batch.state),
                        _p(batch.params), _p(batch.t_ep), _p(batch.episode))
     return batch
+
+
+def adjoint_window(m: OracleModel, batch: Batch, actions, coef, lam_T, dir_s0, dir_act):
+    """J = sum_t coef[t] r_t + <lam_T, x_T> of an action-replay window from the
+    batch's state (x = p, q, nu: 13 rows) and its directional derivative
+    along (dir_s0 [13][n], dir_act [T][8][n]), by forward-mode dual numbers.
+    The batch is not modified.  Returns (J[n], dJ[n])."""
+    act = np.ascontiguousarray(actions, dtype=np.float64)
+    T = act.shape[0]
+    n = batch.n
+    assert act.shape == (T, 8, n)
+    coef = np.ascontiguousarray(coef, dtype=np.float64)
+    assert coef.shape == (T,)
+    lam = None if lam_T is None else np.ascontiguousarray(lam_T, dtype=np.float64)
+    ds0 = np.ascontiguousarray(dir_s0, dtype=np.float64)
+    da = np.ascontiguousarray(dir_act, dtype=np.float64)
+    assert ds0.shape == (13, n) and da.shape == act.shape
+    J = np.zeros(n)
+    dJ = np.zeros(n)
+    lib().oracle_adjoint_window(C.byref(m), n, _p(batch.env_ids), _p(batch.state),
+                                _p(batch.params), _p(batch.t_ep), _p(batch.episode), T, _p(act),
+                                _p(coef), _p(lam), _p(ds0), _p(da), _p(J), _p(dJ))
+    return J, dJ
 
 
 def replay(m: OracleModel, batch: Batch, actions: np.ndarray, precision: str = "f64",

@@ -1,0 +1,131 @@
+"""Pins for the oracle of the adjoint kernels: the directional derivative of
+an action-replay window objective J = sum_t coef_t r_t + <lam_T, x_T>
+computed by forward-mode dual numbers over the model code (oracle
+adjoint_window) against central differences of the same J in double, a
+one-substep closed form, linearity in the direction, the gradient cut at an
+episode end, and zero derivative through clipped thruster commands."""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2512_13359_gb300 import workloads as W
+
+
+def _setup(n=6, T=5, seed=0, warm=7, **over):
+    """A batch moved off its reset state by `warm` replay steps (so that
+    velocities, angular rates and the current are all non-zero), and
+    actions for the window away from the clip edges."""
+    w = W.workload("ppo_65536", n_envs=n, w_vs=0.05, **over)
+    m = O.model(w)
+    b = O.Batch(np.arange(n) + 11)
+    O.reset(m, b)
+    rng = np.random.default_rng(seed)
+    if warm:
+        O.replay(m, b, W.replay_actions(seed + 1, warm, n, scale=0.8))
+    act = rng.uniform(-0.95, 0.95, (T, 8, n))
+    return w, m, b, act, rng
+
+
+def _dirs(rng, T, n):
+    return rng.normal(size=(13, n)), rng.normal(size=(T, 8, n))
+
+
+def _shifted(b, act, ds0, da, h):
+    b2 = b.copy()
+    b2.state[0:13] = b.state[0:13] + h * ds0
+    return b2, act + h * da
+
+
+def test_dual_derivative_matches_central_differences():
+    T, n = 6, 5
+    w, m, b, act, rng = _setup(n=n, T=T)
+    coef = rng.normal(size=T)
+    lam = rng.normal(size=(13, n))
+    ds0, da = _dirs(rng, T, n)
+    zero0, zeroa = np.zeros((13, n)), np.zeros((T, 8, n))
+    J, dJ = O.adjoint_window(m, b, act, coef, lam, ds0, da)
+    h = 1e-6
+    bp, ap = _shifted(b, act, ds0, da, h)
+    bm, am = _shifted(b, act, ds0, da, -h)
+    Jp, _ = O.adjoint_window(m, bp, ap, coef, lam, zero0, zeroa)
+    Jm, _ = O.adjoint_window(m, bm, am, coef, lam, zero0, zeroa)
+    fd = (Jp - Jm) / (2 * h)
+    assert np.all(np.abs(dJ) > 1e-3)
+    assert np.allclose(dJ, fd, rtol=1e-6, atol=1e-9), (dJ, fd)
+    # the window leaves the batch untouched
+    J2, _ = O.adjoint_window(m, b, act, coef, lam, zero0, zeroa)
+    assert np.array_equal(J, J2)
+
+
+def test_one_substep_from_rest_closed_form():
+    """From rest, with no current, no buoyancy offset and the centre of
+    buoyancy at the origin, one substep gives nu' = h M^-1 tau and
+    p' = p + h R(q) v', so that for lam_T on (p, nu) and coef = 0
+    dJ/da_j = sum_k lam_nu,k h B_kj / M_k + lam_p . h R(q) (h B_vj / M_v)
+    with B = alloc * thrust_max."""
+    n, T = 4, 1
+    w, m, b, act, rng = _setup(n=n, T=T, warm=0, substeps=1, dr_enable=0, current_range=0.0)
+    assert np.all(b.state[7:13] == 0) and np.all(b.params[10:17] == 0)
+    lam = np.zeros((13, n))
+    lam[0:3] = rng.normal(size=(3, n))
+    lam[7:13] = rng.normal(size=(6, n))
+    h = float(w["dt"])
+    Minv = 1.0 / (np.r_[[w["mass"]] * 3, w["inertia"]] + np.asarray(w["added_mass"]))
+    Bm = np.asarray(w["alloc"], dtype=np.float64).reshape(6, 8) * w["thrust_max"]
+    for j in range(8):
+        da = np.zeros((T, 8, n))
+        da[0, j] = 1.0
+        _, dJ = O.adjoint_window(m, b, act, np.zeros(T), lam, np.zeros((13, n)), da)
+        for i in range(n):
+            q = b.state[3:7, i]
+            wq, x, y, z = q
+            R = np.array([[1 - 2 * (y * y + z * z), 2 * (x * y - wq * z), 2 * (x * z + wq * y)],
+                          [2 * (x * y + wq * z), 1 - 2 * (x * x + z * z), 2 * (y * z - wq * x)],
+                          [2 * (x * z - wq * y), 2 * (y * z + wq * x), 1 - 2 * (x * x + y * y)]])
+            dnu = h * Minv * Bm[:, j]
+            want = lam[7:13, i] @ dnu + lam[0:3, i] @ (h * R @ dnu[0:3])
+            assert dJ[i] == pytest.approx(want, rel=1e-12, abs=1e-15)
+
+
+def test_derivative_is_linear_in_the_direction():
+    T, n = 4, 3
+    w, m, b, act, rng = _setup(n=n, T=T, seed=3)
+    coef, lam = rng.normal(size=T), rng.normal(size=(13, n))
+    s1, a1 = _dirs(rng, T, n)
+    s2, a2 = _dirs(rng, T, n)
+    _, d1 = O.adjoint_window(m, b, act, coef, lam, s1, a1)
+    _, d2 = O.adjoint_window(m, b, act, coef, lam, s2, a2)
+    _, d12 = O.adjoint_window(m, b, act, coef, lam, s1 + 2 * s2, a1 + 2 * a2)
+    assert np.allclose(d12, d1 + 2 * d2, rtol=1e-12, atol=1e-14)
+
+
+def test_episode_end_cuts_the_gradient():
+    """With the episode ending at window step 2, nothing before or at that
+    step (actions 0..2, the initial state) reaches rewards of steps 3.. or
+    the terminal state; actions after it do."""
+    T, n = 6, 4
+    w, m, b, act, rng = _setup(n=n, T=T, warm=0, episode_len=3)
+    coef = np.r_[0.0, 0.0, 0.0, rng.normal(size=3)]
+    lam = rng.normal(size=(13, n))
+    ds0, da = _dirs(rng, T, n)
+    da_before = da.copy()
+    da_before[3:] = 0
+    _, dJ = O.adjoint_window(m, b, act, coef, lam, ds0, da_before)
+    assert np.all(dJ == 0.0)
+    da_after = da.copy()
+    da_after[:3] = 0
+    _, dJ = O.adjoint_window(m, b, act, coef, lam, np.zeros((13, n)), da_after)
+    assert np.all(np.abs(dJ) > 0)
+
+
+def test_clipped_commands_have_zero_derivative():
+    T, n = 3, 4
+    w, m, b, act, rng = _setup(n=n, T=T, seed=5)
+    act[:, 2] = 1.4          # thruster 2 saturated high at every step
+    act[:, 5] = -1.7         # thruster 5 saturated low
+    coef, lam = rng.normal(size=T), rng.normal(size=(13, n))
+    da = np.zeros((T, 8, n))
+    da[:, 2] = rng.normal(size=(T, n))
+    da[:, 5] = rng.normal(size=(T, n))
+    _, dJ = O.adjoint_window(m, b, act, coef, lam, np.zeros((13, n)), da)
+    assert np.all(dJ == 0.0)
