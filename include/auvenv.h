@@ -489,6 +489,35 @@ int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t
  * buffers an env_set_weights call then reads. */
 int ppo_export_weights(auv_ppo* p, float* policy, float* value, void* stream);
 
+/*
+ * env_adjoint: reverse-mode adjoint of the control step over a window of
+ * actions -- the back-propagation through the dynamics of SHAC (paper
+ * §III-A, short-horizon actor-critic; Xu et al. 2022).  From each env's
+ * current state x_0 = (p, q, nu) the window takes T control steps with the
+ * given actions (the rollout's own step: allocation with clip, substeps,
+ * reward, auto-reset) and forms
+ *   J = sum_t coef[t] r_t + <lam_T, x_T>
+ * with x_T the state after the last step.  Outputs dJ/da_t (grad_act) and
+ * dJ/dx_0 (lam_0).  An episode end inside the window replaces the state by
+ * its reset draw: nothing before it reaches later rewards or x_T.  The
+ * clip's derivative is taken as 1 on [-1, 1] and 0 outside.
+ *   act [T][8][N], grad_act [T][8][N]: device memory.
+ *   coef [T]: device memory.
+ *   lam_T [13][N] (rows p, q, nu): device memory, or NULL for 0.
+ *   lam_0 [13][N], rew_out [T][N] (fp32), done_out [T][N] (u8): optional
+ *   outputs, device or mapped page-locked host memory.
+ * The env's state, episode counters and step counter are not changed (step
+ * with env_step_actions to advance).  Fossen model only
+ * (AUV_ERR_UNSUPPORTED for the paper model); 1 <= T <= AUV_ADJOINT_MAX_T;
+ * at most AUV_ADJOINT_MAX_SUBSTEPS substeps (AUV_ERR_UNSUPPORTED).  The first
+ * call at a given N * T allocates the window's scratch (30 floats per
+ * env-step) on the device.
+ */
+#define AUV_ADJOINT_MAX_T 64
+#define AUV_ADJOINT_MAX_SUBSTEPS 8
+int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const float* lam_T,
+                float* grad_act, float* lam_0, float* rew_out, uint8_t* done_out, void* stream);
+
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);

@@ -39,7 +39,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
-            "env_policy_forward_noalloc", "env_layout", "env_gae",
+            "env_policy_forward_noalloc", "env_layout", "env_gae", "env_adjoint",
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
             "ppo_update", "ppo_export_weights")
@@ -153,6 +153,7 @@ def lib(path: str | None = None):
     L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
     L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
+    L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
     U64, U32 = C.c_uint64, C.c_uint32
     L.ppo_create.argtypes = [C.POINTER(PpoConfig), C.POINTER(P)]
     L.ppo_destroy.argtypes = [P]
@@ -312,6 +313,16 @@ class Env:
         self._check(lib().env_gae(self.h, int(rew.shape[0]), _ptr(rew), _ptr(done), _ptr(value),
                                   _ptr(last_value), float(gamma), float(lam), _ptr(adv),
                                   _ptr(ret), _stream(stream)))
+
+    def adjoint(self, act, coef, grad_act, lam_T=None, lam_0=None, rew=None, done=None,
+                stream=None):
+        """Reverse-mode adjoint of an action window from the current state
+        (env_adjoint): fills grad_act [T][8][N] and, if given, lam_0 [13][N],
+        rew and done [T][N]."""
+        T = act.shape[0]
+        self._check(lib().env_adjoint(self.h, T, _ptr(act), _ptr(coef), _ptr(lam_T),
+                                      _ptr(grad_act), _ptr(lam_0), _ptr(rew), _ptr(done),
+                                      _stream(stream)))
 
     def step(self, obs=None, rew=None, done=None, stream=None):
         self._check(lib().env_step(self.h, _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))

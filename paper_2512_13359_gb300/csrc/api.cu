@@ -41,6 +41,9 @@ struct auv_env {
   cudaEvent_t seg_done[2] = {nullptr, nullptr};
   cudaEvent_t copy_done[2] = {nullptr, nullptr};
   int last_copy = -1;       // buffer whose copy_done ends the last staged call
+  // Adjoint windows (env_adjoint): per-step inputs of the forward pass.
+  float* adj_scratch = nullptr;
+  size_t adj_scratch_floats = 0;
 };
 
 namespace {
@@ -375,6 +378,7 @@ int env_destroy(auv_env* env) {
   cudaDeviceSynchronize();
   cudaError_t e = cudaFree(env->workspace);
   if (env->stage) cudaFree(env->stage);
+  if (env->adj_scratch) cudaFree(env->adj_scratch);
   for (int b = 0; b < 2; ++b) {
     if (env->seg_done[b]) cudaEventDestroy(env->seg_done[b]);
     if (env->copy_done[b]) cudaEventDestroy(env->copy_done[b]);
@@ -656,6 +660,48 @@ int env_step_actions(auv_env* env, const float* act, int T, float* rew_out, uint
                                      static_cast<uint8_t*>(done), static_cast<float*>(trace),
                                      env->status, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "replay kernel");
+}
+
+int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const float* lam_T,
+                float* grad_act, float* lam_0, float* rew_out, uint8_t* done_out, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (is_paper(&env->cfg))
+    return fail(env, AUV_ERR_UNSUPPORTED, "the adjoint is built for the Fossen model");
+  if (T < 1 || T > AUV_ADJOINT_MAX_T)
+    return fail(env, AUV_ERR_INVALID, "T outside [1, %d]", AUV_ADJOINT_MAX_T);
+  if (env->model.substeps > AUV_ADJOINT_MAX_SUBSTEPS)
+    return fail(env, AUV_ERR_UNSUPPORTED, "the adjoint supports at most %d substeps",
+                AUV_ADJOINT_MAX_SUBSTEPS);
+  if ((rc = check_device_buffer(env, act, "act", 4)) || (rc = check_device_buffer(env, coef, "coef", 4)) ||
+      (rc = check_device_buffer(env, grad_act, "grad_act", 4)))
+    return rc;
+  if (lam_T && (rc = check_device_buffer(env, lam_T, "lam_T", 4))) return rc;
+  void *l0 = nullptr, *rew = nullptr, *done = nullptr;
+  if ((rc = map_output(env, lam_0, "lam_0", 4, &l0)) || (rc = map_output(env, rew_out, "rew_out", 4, &rew)) ||
+      (rc = map_output(env, done_out, "done_out", 1, &done)))
+    return rc;
+  const size_t need = auv::adjoint_scratch_floats(env->model.n, T);
+  if (need > env->adj_scratch_floats) {
+    if (env->adj_scratch) {
+      cudaError_t e = cudaFree(env->adj_scratch);
+      env->adj_scratch = nullptr;
+      env->adj_scratch_floats = 0;
+      if (e != cudaSuccess) return cuda_fail(env, e, "free adjoint scratch");
+    }
+    cudaError_t e = cudaMalloc(&env->adj_scratch, need * sizeof(float));
+    if (e != cudaSuccess) {
+      env->adj_scratch = nullptr;
+      return cuda_fail(env, e, "cudaMalloc(adjoint scratch)");
+    }
+    env->adj_scratch_floats = need;
+  }
+  cudaError_t e = auv::launch_adjoint(env->model, env->buf, act, T, coef, lam_T, grad_act,
+                                      static_cast<float*>(l0), static_cast<float*>(rew),
+                                      static_cast<uint8_t*>(done), env->adj_scratch, env->status,
+                                      static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "adjoint kernel");
 }
 
 int env_observe(auv_env* env, float* obs_out, void* stream) {

@@ -55,6 +55,15 @@ cudaError_t launch_paper_rollout_fp32(const Model& M, const Buffers& B, const fl
                                       const float* wv, const Traj& tr, int T, uint64_t t_g0,
                                       Status* st, cudaStream_t s);
 
+// Reverse-mode adjoint of the Fossen control step over an action window
+// (k_adjoint.cu).  scratch: adjoint_scratch_floats(n, T) floats.  T <= 64,
+// M.substeps <= 8.
+size_t adjoint_scratch_floats(int n, int T);
+cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, int T,
+                           const float* coef, const float* lam_T, float* g_act, float* lam_0,
+                           float* rew, uint8_t* done, float* scratch, Status* st,
+                           cudaStream_t s);
+
 // PPO learner pieces (k_ppo.cu)
 cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, const float* value,
                        const float* last_value, float gamma, float lam, float* adv, float* ret,
