@@ -60,6 +60,9 @@ def parse():
     ap.add_argument("--epochs", type=int, default=4)
     ap.add_argument("--n-minibatches", type=int, default=None,
                     help="minibatches per epoch (default: all rows / minibatch)")
+    ap.add_argument("--adjoint", action="store_true",
+                    help="time the control-step adjoint (env_adjoint) over an action window")
+    ap.add_argument("--window", type=int, default=32, help="adjoint window length")
     ap.add_argument("--gae", action="store_true",
                     help="advantage estimation (env_gae) over one rollout, HBM roofline")
     ap.add_argument("--sweep", action="store_true",
@@ -435,8 +438,86 @@ def run_ppo(args):
     print(json.dumps(line), flush=True)
 
 
+# FP32 operations one env-step of env_adjoint executes (forward pass, the
+# backward pass's recompute of the step, and the VJPs), by substep count,
+# FFMA counted twice: smsp__sass_thread_inst_executed_op_{fadd,fmul,ffma}_pred_on
+# of k_adjoint from one ncu capture of `bench.py --adjoint --n-envs 8192`,
+# divided by its 262,144 env-steps (674 FADD + 1273 FMUL + 2021 FFMA).
+ADJOINT_FLOPS_PER_ENV_STEP = {4: 5988.2}
+
+
+def run_adjoint(args):
+    """The reverse-mode adjoint of the Fossen control step over an action
+    window (env_adjoint) from the workload's state: forward re-simulation,
+    then the backward sweep.  One step = one window over all envs."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {}
+    if args.n_envs:
+        over["n_envs"] = args.n_envs
+    w = W.workload(args.workload, **over)
+    n, T = int(w["n_envs"]), int(args.window)
+    env = auvenv.Env(w)
+    env.reset()
+    warm = torch.from_numpy(W.replay_actions(1, 8, n, scale=0.8)).cuda()
+    rew0 = torch.empty((8, n), device="cuda")
+    done0 = torch.empty((8, n), dtype=torch.uint8, device="cuda")
+    env.step_actions(warm, rew0, done0)
+    act = torch.from_numpy(W.replay_actions(2, T, n, scale=0.9)).cuda()
+    coef = torch.tensor([0.99 ** t / (n * T) for t in range(T)], dtype=torch.float32,
+                        device="cuda")
+    lam_T = torch.randn((13, n), device="cuda") / (n * T)
+    g = torch.empty((T, 8, n), device="cuda")
+    lam_0 = torch.empty((13, n), device="cuda")
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        env.adjoint(act, coef, g, lam_T=lam_T, lam_0=lam_0)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0) if not args.no_clocks else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        env.adjoint(act, coef, g, lam_T=lam_T, lam_0=lam_0)
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    clock_info = clocks.stop() if clocks else None
+    assert env.status().code == 0
+    step_ms = sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+    rate = n * T / (step_ms * 1e-3)
+    peaks, src = load_peaks()
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+    fps = ADJOINT_FLOPS_PER_ENV_STEP.get(int(w["substeps"]))
+    achieved = None if fps is None else rate * fps / 1e12
+    line = {
+        "metric": "adjoint env-steps/s", "value": rate, "unit": "env-steps/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (workload state after 8 replayed steps, random actions)",
+        "config": {"workload": w["name"], "n_envs": n, "window": T,
+                   "substeps": int(w["substeps"]), "l2": "flushed between timed steps"},
+        "roofline": {"bound": "alu", "kernel": "k_adjoint", "achieved": achieved, "peak": peak,
+                     "unit": "TFLOP/s", "frac": None if achieved is None else achieved / peak,
+                     "traffic": None,
+                     "peak_source": f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz",
+                     "flops_per_env_step": fps},
+        "gpu_launches": args.steps, "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.adjoint:
+        run_adjoint(args)
+        return
     if args.ppo:
         run_ppo(args)
         return
