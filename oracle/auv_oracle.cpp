@@ -1199,6 +1199,20 @@ void oracle_minibatch_perm(uint64_t seed, uint64_t epoch, uint32_t m, uint32_t s
   for (uint32_t k = 0; k < count; ++k) out[k] = minibatch_index(start + k, m, seed, epoch);
 }
 
+// Replay-buffer sample indices: draw `draw`, sample b takes the first word
+// of Philox4x32-10 at counter (b, 0x52420000, draw low, draw high) and key
+// (seed low, seed high) and maps it to [0, size) by the multiply-high
+// floor(word * size / 2^32).
+void oracle_rbuf_indices(uint64_t seed, uint64_t draw, uint32_t size, uint32_t count,
+                         uint32_t* out) {
+  for (uint32_t b = 0; b < count; ++b) {
+    const uint32_t ctr[4] = {b, 0x52420000u, (uint32_t)draw, (uint32_t)(draw >> 32)};
+    uint32_t w[4];
+    philox4x32_10(ctr, (uint32_t)seed, (uint32_t)(seed >> 32), w);
+    out[b] = (uint32_t)(((uint64_t)w[0] * (uint64_t)size) >> 32);
+  }
+}
+
 // One Feistel pass (no cycle walking) forward or back, for the pins.
 uint32_t oracle_feistel(uint32_t x, uint32_t m, uint64_t seed, uint64_t epoch, int inverse) {
   const int h = perm_half_bits(m);

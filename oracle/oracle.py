@@ -56,6 +56,7 @@ def lib():
         P = C.c_void_p
         _lib.oracle_model_size.restype = C.c_int
         _lib.oracle_philox.argtypes = [C.c_uint32, C.c_uint32, P, P]
+        _lib.oracle_rbuf_indices.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32, P]
         _lib.oracle_adjoint_window.argtypes = [C.POINTER(OracleModel), C.c_int, P, P, P, P, P,
                                                C.c_int, P, P, P, P, P, P, P]
         _lib.oracle_minibatch_perm.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32,
@@ -231,6 +232,13 @@ def minibatch_perm(seed: int, epoch: int, m: int, start: int, count: int) -> np.
     """Positions start .. start+count-1 of the learner's epoch permutation of [0, m)."""
     out = np.zeros(count, dtype=np.uint32)
     lib().oracle_minibatch_perm(seed, epoch, m, start, count, _p(out))
+    return out
+
+
+def rbuf_indices(seed: int, draw: int, size: int, count: int) -> np.ndarray:
+    """Replay-buffer sample indices of draw `draw` (see oracle_rbuf_indices)."""
+    out = np.zeros(count, dtype=np.uint32)
+    lib().oracle_rbuf_indices(seed, draw, size, count, _p(out))
     return out
 
 
