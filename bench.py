@@ -63,6 +63,10 @@ def parse():
     ap.add_argument("--adjoint", action="store_true",
                     help="time the control-step adjoint (env_adjoint) over an action window")
     ap.add_argument("--window", type=int, default=32, help="adjoint window length")
+    ap.add_argument("--rbuf", action="store_true",
+                    help="time replay-buffer insert (a rollout's trajectory) and sampling")
+    ap.add_argument("--invalloc", action="store_true",
+                    help="time the inverse thruster allocation over the envs")
     ap.add_argument("--gae", action="store_true",
                     help="advantage estimation (env_gae) over one rollout, HBM roofline")
     ap.add_argument("--sweep", action="store_true",
@@ -513,8 +517,110 @@ def run_adjoint(args):
     print(json.dumps(line), flush=True)
 
 
+def _timed(args, fn, flush=None):
+    import torch
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(args.steps):
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+
+
+def run_rbuf(args):
+    """Replay buffer (rbuf_insert of one 65,536 x 128 rollout trajectory,
+    then rbuf_sample of 65,536-transition minibatches).  HBM roofline:
+    (2 D + A + 1) * 4 + 1 bytes read and written per transition."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {"n_envs": args.n_envs} if args.n_envs else {}
+    w = W.workload(args.workload, **over)
+    n, T = int(w["n_envs"]), int(w["steps"])
+    D, A = W.obs_dim(w), W.act_dim(w)
+    env = auvenv.Env(w)
+    env.set_weights(W.policy_weights(w), W.value_weights(w) if w["has_value"] else None)
+    env.reset()
+    traj = env.alloc_traj(T, keys=("obs", "act", "rew", "done"))
+    env.rollout(T, traj)
+    last = torch.empty((D, n), device="cuda")
+    env.observe(last)
+    rb = auvenv.ReplayBuffer(D, A, 1 << 24)
+    rec = (2 * D + A + 1) * 4 + 1
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    ins_ms = _timed(args, lambda: rb.insert(traj["obs"], traj["act"], traj["rew"], traj["done"],
+                                            last), flush)
+    B = 65536
+    out = rb.sample(B, 1, 0)
+    draws = iter(range(1, 10 ** 9))
+    smp_ms = _timed(args, lambda: rb.sample(B, 1, next(draws), out=out), flush)
+    peaks, src = load_peaks()
+    ins_gbs = 2 * rec * n * T / (ins_ms * 1e-3) / 1e9
+    smp_gbs = 2 * rec * B / (smp_ms * 1e-3) / 1e9
+    line = {
+        "metric": "replay-buffer sampled transitions/s", "value": B / (smp_ms * 1e-3),
+        "unit": "transitions/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": smp_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic (one rollout of the workload)",
+        "config": {"workload": w["name"], "capacity": 1 << 24, "minibatch": B,
+                   "inserted_per_call": n * T, "l2": "flushed between timed steps"},
+        "insert": {"transitions_per_s": n * T / (ins_ms * 1e-3), "ms": ins_ms,
+                   "achieved_gbs": ins_gbs, "frac": ins_gbs / peaks["hbm_gbs"]},
+        "roofline": {"bound": "hbm", "kernel": "k_rb_sample", "achieved": smp_gbs,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": smp_gbs / peaks["hbm_gbs"],
+                     "traffic": None, "peak_source": f"HBM copy, {src}",
+                     "bytes_per_transition": 2 * rec},
+        "gpu_launches": args.steps, "clocks": None,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_invalloc(args):
+    """Inverse thruster allocation (env_inverse_allocate) of one wrench per
+    env; HBM roofline 56 B per row (6 floats in, 8 out)."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    n = args.n_envs or (1 << 24)
+    w = W.workload("ppo_65536", n_envs=1024)
+    env = auvenv.Env(w)
+    wrench = torch.randn((6, n), device="cuda") * 30.0
+    cmd = torch.empty((8, n), device="cuda")
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    ms = _timed(args, lambda: env.inverse_allocate(wrench, cmd), flush)
+    peaks, src = load_peaks()
+    gbs = 56 * n / (ms * 1e-3) / 1e9
+    line = {
+        "metric": "inverse allocations/s", "value": n / (ms * 1e-3), "unit": "rows/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (N(0, 30^2) wrenches)",
+        "config": {"workload": "inverse allocation of the ppo_65536 vehicle", "rows": n,
+                   "l2": "flushed between timed steps"},
+        "roofline": {"bound": "hbm", "kernel": "k_inverse_alloc", "achieved": gbs,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": gbs / peaks["hbm_gbs"],
+                     "traffic": None, "peak_source": f"HBM copy, {src}"},
+        "gpu_launches": args.steps, "clocks": None,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.rbuf:
+        run_rbuf(args)
+        return
+    if args.invalloc:
+        run_invalloc(args)
+        return
     if args.adjoint:
         run_adjoint(args)
         return

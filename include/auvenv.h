@@ -518,6 +518,53 @@ int ppo_export_weights(auv_ppo* p, float* policy, float* value, void* stream);
 int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const float* lam_T,
                 float* grad_act, float* lam_0, float* rew_out, uint8_t* done_out, void* stream);
 
+/*
+ * env_inverse_allocate: thruster commands for body-frame wrenches, the map
+ * the paper's controllers go through at deployment (§V-B: the policy's
+ * forces and torques -> individual thrusters through the allocation matrix).
+ * With Bm = alloc * thrust_max (the env's 6 x 8 matrix), the commands are
+ * the minimum-norm solution of Bm u = tau clipped to the thrusters' range:
+ *   cmd = clip(pinv(Bm) tau, -1, 1)
+ * (pinv = Bm^T (Bm Bm^T)^-1, formed once in double on the host).
+ * wrench [6][n]: device memory; cmd [8][n]: device or mapped page-locked
+ * host memory.  AUV_ERR_UNSUPPORTED if the allocation has rank < 6.
+ * (The PWM interpolation after it is vehicle-specific and not built.)
+ */
+int env_inverse_allocate(auv_env* env, int n, const float* wrench, float* cmd, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Replay buffer for off-policy learning (DroQ, paper §III-A; Hiraoka et al.
+ * 2022): a device ring of `capacity` transitions (obs, act, rew, next_obs,
+ * done), stored sample-major.
+ *
+ * rbuf_insert adds a rollout's T x N transitions: transition (t, i) goes to
+ * slot (head + t*N + i) mod capacity with obs = obs[t][.][i], act =
+ * act[t][.][i], rew / done = [t][i], next_obs = obs[t+1][.][i] (last_obs for
+ * t = T-1: the observation after the last step).  After an auto-reset the
+ * next observation is the new episode's first: a time-limit end is stored
+ * as a terminal transition (done = 1).  Inputs are the rollout's arrays in
+ * device memory: obs [T][D][N], act [T][A][N], rew [T][N] fp32, done [T][N]
+ * u8, last_obs [D][N].  head and size advance on the host at the call.
+ *
+ * rbuf_sample draws B transitions uniformly from the filled slots: sample b
+ * of draw `draw` takes the first word w of Philox4x32-10 at counter
+ * (b, 0x52420000, draw low, draw high) with key (seed low, seed high) and
+ * reads slot floor(w * size / 2^32).  Outputs (device memory): obs and
+ * next_obs [B][D], act [B][A], rew [B] fp32, done [B] u8, and optionally
+ * the slots idx [B] (u32).  AUV_ERR_INVALID when the buffer is empty.
+ * Both calls are asynchronous on `stream`; a sample sees every insert
+ * issued before it on the same stream.
+ * --------------------------------------------------------------------------- */
+typedef struct auv_rbuf auv_rbuf;
+int rbuf_create(uint32_t obs_dim, uint32_t act_dim, uint64_t capacity, auv_rbuf** out);
+int rbuf_destroy(auv_rbuf* r);
+const char* rbuf_last_error(const auv_rbuf* r);
+int rbuf_size(const auv_rbuf* r, uint64_t* size, uint64_t* head);
+int rbuf_insert(auv_rbuf* r, int T, int N, const float* obs, const float* act, const float* rew,
+                const uint8_t* done, const float* last_obs, void* stream);
+int rbuf_sample(auv_rbuf* r, uint32_t B, uint64_t seed, uint64_t draw, float* obs, float* act,
+                float* rew, float* next_obs, uint8_t* done, uint32_t* idx, void* stream);
+
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);

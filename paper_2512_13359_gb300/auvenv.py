@@ -40,6 +40,8 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
             "env_policy_forward_noalloc", "env_layout", "env_gae", "env_adjoint",
+            "env_inverse_allocate", "rbuf_create", "rbuf_destroy", "rbuf_last_error",
+            "rbuf_size", "rbuf_insert", "rbuf_sample",
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
             "ppo_update", "ppo_export_weights")
@@ -154,6 +156,14 @@ def lib(path: str | None = None):
     L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
+    L.env_inverse_allocate.argtypes = [P, I, P, P, P]
+    L.rbuf_create.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(P)]
+    L.rbuf_destroy.argtypes = [P]
+    L.rbuf_last_error.argtypes = [P]
+    L.rbuf_last_error.restype = C.c_char_p
+    L.rbuf_size.argtypes = [P, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]
+    L.rbuf_insert.argtypes = [P, I, I, P, P, P, P, P, P]
+    L.rbuf_sample.argtypes = [P, C.c_uint32, C.c_uint64, C.c_uint64, P, P, P, P, P, P, P]
     U64, U32 = C.c_uint64, C.c_uint32
     L.ppo_create.argtypes = [C.POINTER(PpoConfig), C.POINTER(P)]
     L.ppo_destroy.argtypes = [P]
@@ -172,6 +182,7 @@ def lib(path: str | None = None):
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
     L.ppo_last_error.restype = C.c_char_p
+    L.rbuf_last_error.restype = C.c_char_p
     _lib = L
     return L
 
@@ -323,6 +334,11 @@ class Env:
         self._check(lib().env_adjoint(self.h, T, _ptr(act), _ptr(coef), _ptr(lam_T),
                                       _ptr(grad_act), _ptr(lam_0), _ptr(rew), _ptr(done),
                                       _stream(stream)))
+
+    def inverse_allocate(self, wrench, cmd, stream=None):
+        """Thruster commands cmd [8][n] for wrenches [6][n] (env_inverse_allocate)."""
+        self._check(lib().env_inverse_allocate(self.h, wrench.shape[1], _ptr(wrench), _ptr(cmd),
+                                               _stream(stream)))
 
     def step(self, obs=None, rew=None, done=None, stream=None):
         self._check(lib().env_step(self.h, _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))
@@ -494,3 +510,57 @@ class Learner:
         b = self._batch(traj)
         self._check(lib().ppo_update(self.h, C.byref(b), epochs, n_minibatches, _ptr(stats),
                                      _stream(stream)))
+
+
+class ReplayBuffer:
+    """Device replay buffer (include/auvenv.h, rbuf_*) on the current device."""
+
+    def __init__(self, obs_dim: int, act_dim: int, capacity: int):
+        L = lib()
+        h = C.c_void_p()
+        rc = L.rbuf_create(obs_dim, act_dim, capacity, C.byref(h))
+        if rc != AUV_OK:
+            raise AuvError(rc, L.rbuf_last_error(None).decode())
+        self.h = h
+        self.obs_dim, self.act_dim, self.capacity = obs_dim, act_dim, capacity
+
+    def _check(self, rc):
+        if rc != AUV_OK:
+            raise AuvError(rc, lib().rbuf_last_error(self.h).decode())
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().rbuf_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def size(self):
+        a, b = C.c_uint64(), C.c_uint64()
+        self._check(lib().rbuf_size(self.h, C.byref(a), C.byref(b)))
+        return a.value, b.value
+
+    def insert(self, obs, act, rew, done, last_obs, stream=None):
+        T, _, N = obs.shape
+        self._check(lib().rbuf_insert(self.h, T, N, _ptr(obs), _ptr(act), _ptr(rew), _ptr(done),
+                                      _ptr(last_obs), _stream(stream)))
+
+    def sample(self, B: int, seed: int, draw: int, out=None, with_idx=False, stream=None):
+        import torch
+        if out is None:
+            out = dict(obs=torch.empty((B, self.obs_dim), device="cuda"),
+                       act=torch.empty((B, self.act_dim), device="cuda"),
+                       rew=torch.empty(B, device="cuda"),
+                       next_obs=torch.empty((B, self.obs_dim), device="cuda"),
+                       done=torch.empty(B, dtype=torch.uint8, device="cuda"))
+            if with_idx:
+                out["idx"] = torch.empty(B, dtype=torch.int32, device="cuda")
+        self._check(lib().rbuf_sample(self.h, B, seed, draw, _ptr(out["obs"]), _ptr(out["act"]),
+                                      _ptr(out["rew"]), _ptr(out["next_obs"]), _ptr(out["done"]),
+                                      _ptr(out.get("idx")), _stream(stream)))
+        return out

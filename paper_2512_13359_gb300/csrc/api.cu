@@ -44,6 +44,9 @@ struct auv_env {
   // Adjoint windows (env_adjoint): per-step inputs of the forward pass.
   float* adj_scratch = nullptr;
   size_t adj_scratch_floats = 0;
+  // Inverse allocation (env_inverse_allocate): made on first use.
+  bool inv_ready = false;
+  auv::InvAlloc inv;
 };
 
 namespace {
@@ -702,6 +705,25 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
                                       static_cast<uint8_t*>(done), env->adj_scratch, env->status,
                                       static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "adjoint kernel");
+}
+
+int env_inverse_allocate(auv_env* env, int n, const float* wrench, float* cmd, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (n < 1) return fail(env, AUV_ERR_INVALID, "n must be >= 1");
+  if ((rc = check_device_buffer(env, wrench, "wrench", 4))) return rc;
+  void* out = nullptr;
+  if (!cmd) return fail(env, AUV_ERR_INVALID, "cmd is NULL");
+  if ((rc = map_output(env, cmd, "cmd", 4, &out))) return rc;
+  if (!env->inv_ready) {
+    if (!auv::pinv_6x8(env->model.alloc_t, env->inv.pinv))
+      return fail(env, AUV_ERR_UNSUPPORTED, "the allocation matrix has rank < 6");
+    env->inv_ready = true;
+  }
+  cudaError_t e = auv::launch_inverse_alloc(n, env->inv, wrench, static_cast<float*>(out),
+                                            static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "inverse allocation kernel");
 }
 
 int env_observe(auv_env* env, float* obs_out, void* stream) {

@@ -64,6 +64,14 @@ cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, i
                            float* rew, uint8_t* done, float* scratch, Status* st,
                            cudaStream_t s);
 
+// Inverse thruster allocation (rbuf.cu): commands = clip(pinv u-map, -1, 1).
+struct InvAlloc {
+  float pinv[48];   // [8][6]: pseudo-inverse of alloc * thrust_max
+};
+bool pinv_6x8(const float* alloc_t, float* out);
+cudaError_t launch_inverse_alloc(int n, const InvAlloc& ia, const float* wrench, float* cmd,
+                                 cudaStream_t s);
+
 // PPO learner pieces (k_ppo.cu)
 cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, const float* value,
                        const float* last_value, float gamma, float lam, float* adv, float* ret,
