@@ -282,6 +282,14 @@ inline Dual cos(Dual a) { return Dual(std::cos(a.v), -std::sin(a.v) * a.d); }
 inline Dual atan2(Dual y, Dual x) {
   return Dual(std::atan2(y.v, x.v), (x.v * y.d - y.v * x.d) / (x.v * x.v + y.v * y.v));
 }
+inline Dual tanh(Dual a) {
+  const double t = std::tanh(a.v);
+  return Dual(t, (1.0 - t * t) * a.d);
+}
+inline Dual exp(Dual a) {
+  const double e = std::exp(a.v);
+  return Dual(e, e * a.d);
+}
 
 template <class R>
 void quat_to_rot(const R q[4], R Rm[3][3]) {
@@ -1284,6 +1292,82 @@ void oracle_adjoint_window(const OracleModel* m, int n, const uint32_t* env_ids,
       for (int k = 0; k < 3; ++k) obj += Dual(lam_T[(0 + k) * n + i]) * e.p[k];
       for (int k = 0; k < 4; ++k) obj += Dual(lam_T[(3 + k) * n + i]) * e.q[k];
       for (int k = 0; k < 6; ++k) obj += Dual(lam_T[(7 + k) * n + i]) * e.nu[k];
+    }
+    J[i] = obj.v;
+    dJ[i] = obj.d;
+  }
+}
+
+// The MLP of the rollout with its weights as dual numbers: values w (float,
+// the flat [W1 | b1 | W2 | b2 | W3 | b3] layout) and tangents dw (NULL for 0).
+void mlp_dual(const float* w, const double* dw, int in_dim, int hidden, int out_dim,
+              const Dual* x, Dual* out) {
+  auto W = [&](size_t k) { return Dual((double)w[k], dw ? dw[k] : 0.0); };
+  const size_t oW1 = 0, ob1 = oW1 + (size_t)hidden * in_dim, oW2 = ob1 + hidden,
+               ob2 = oW2 + (size_t)hidden * hidden, oW3 = ob2 + hidden,
+               ob3 = oW3 + (size_t)out_dim * hidden;
+  Dual* h1 = new Dual[hidden];
+  Dual* h2 = new Dual[hidden];
+  for (int j = 0; j < hidden; ++j) {
+    Dual s = 0.0;
+    for (int i = 0; i < in_dim; ++i) s += W(oW1 + (size_t)j * in_dim + i) * x[i];
+    h1[j] = tanh(s + W(ob1 + j));
+  }
+  for (int j = 0; j < hidden; ++j) {
+    Dual s = 0.0;
+    for (int i = 0; i < hidden; ++i) s += W(oW2 + (size_t)j * hidden + i) * h1[i];
+    h2[j] = tanh(s + W(ob2 + j));
+  }
+  for (int j = 0; j < out_dim; ++j) {
+    Dual s = 0.0;
+    for (int i = 0; i < hidden; ++i) s += W(oW3 + (size_t)j * hidden + i) * h2[i];
+    out[j] = s + W(ob3 + j);
+  }
+  delete[] h1;
+  delete[] h2;
+}
+
+// SHAC's window objective of each env in closed loop (paper §III-A; Xu et al.
+// 2022): from the batch's state, T control steps with the reparameterised
+// Gaussian policy a = mu(o) + exp(clamp(ls(o))) eps (eps: the rollout's
+// action noise at global step t_g0 + t; policy head 2 x 8), then
+//   J = sum_t coef[t] r_t + coef_V V(o_T)
+// (value network at the observation after the last step; none if val_w is
+// NULL).  Returns J and its directional derivative along the policy-weight
+// direction dpol, in forward-mode dual numbers.  The batch is not modified.
+void oracle_shac_window(const OracleModel* m, const float* pol_w, const double* dpol,
+                        const float* val_w, int n, const uint32_t* env_ids, const double* st,
+                        const double* pr, const int32_t* t_ep, const uint32_t* ep,
+                        uint64_t t_g0, int T, const double* coef, double coef_V, double* J,
+                        double* dJ) {
+  for (int i = 0; i < n; ++i) {
+    Env<Dual> e;
+    load_env<Dual>(st, pr, t_ep, ep, n, i, e);
+    Dual obj = 0.0;
+    for (int t = 0; t < T; ++t) {
+      Dual o[kObs], y[2 * kAct], a[kAct];
+      observe(e, o);
+      mlp_dual(pol_w, dpol, kObs, m->hidden, 2 * kAct, o, y);
+      double eps[8];
+      uint32_t w[8];
+      draw_words(env_ids[i], m->seed, t_g0 + (uint64_t)t, 0u, 2, w);
+      float u[8];
+      for (int k = 0; k < 8; ++k) u[k] = word_to_uniform(w[k]);
+      box_muller8(u, eps);
+      for (int k = 0; k < kAct; ++k) {
+        Dual ls = y[kAct + k];
+        if (ls < Dual(m->logstd_min)) ls = Dual(m->logstd_min);
+        if (ls > Dual(m->logstd_max)) ls = Dual(m->logstd_max);
+        a[k] = y[k] + exp(ls) * Dual(eps[k]);
+      }
+      uint8_t d;
+      obj += Dual(coef[t]) * control_step(*m, env_ids[i], e, a, &d);
+    }
+    if (val_w) {
+      Dual o[kObs], v[1];
+      observe(e, o);
+      mlp_dual(val_w, nullptr, kObs, m->hidden, 1, o, v);
+      obj += Dual(coef_V) * v[0];
     }
     J[i] = obj.v;
     dJ[i] = obj.d;

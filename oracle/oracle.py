@@ -56,6 +56,8 @@ def lib():
         P = C.c_void_p
         _lib.oracle_model_size.restype = C.c_int
         _lib.oracle_philox.argtypes = [C.c_uint32, C.c_uint32, P, P]
+        _lib.oracle_shac_window.argtypes = [C.POINTER(OracleModel), P, P, P, C.c_int, P, P, P, P,
+                                            P, C.c_uint64, C.c_int, P, C.c_double, P, P]
         _lib.oracle_rbuf_indices.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32, P]
         _lib.oracle_adjoint_window.argtypes = [C.POINTER(OracleModel), C.c_int, P, P, P, P, P,
                                                C.c_int, P, P, P, P, P, P, P]
@@ -169,6 +171,26 @@ def adjoint_window(m: OracleModel, batch: Batch, actions, coef, lam_T, dir_s0, d
     lib().oracle_adjoint_window(C.byref(m), n, _p(batch.env_ids), _p(batch.state),
                                 _p(batch.params), _p(batch.t_ep), _p(batch.episode), T, _p(act),
                                 _p(coef), _p(lam), _p(ds0), _p(da), _p(J), _p(dJ))
+    return J, dJ
+
+
+def shac_window(m: OracleModel, batch: Batch, pol_w, dpol, val_w, t_g0: int, T: int, coef,
+                coef_V: float):
+    """SHAC window objective per env in closed loop (policy head 16, noise
+    of global steps t_g0 ..) and its directional derivative along the
+    policy-weight direction dpol (or None).  The batch is not modified.
+    Returns (J[n], dJ[n])."""
+    pw = np.ascontiguousarray(pol_w, dtype=np.float32)
+    dp = None if dpol is None else np.ascontiguousarray(dpol, dtype=np.float64)
+    vw = None if val_w is None else np.ascontiguousarray(val_w, dtype=np.float32)
+    coef = np.ascontiguousarray(coef, dtype=np.float64)
+    assert coef.shape == (T,) and m.policy_out == 16
+    n = batch.n
+    J = np.zeros(n)
+    dJ = np.zeros(n)
+    lib().oracle_shac_window(C.byref(m), _p(pw), _p(dp), _p(vw), n, _p(batch.env_ids),
+                             _p(batch.state), _p(batch.params), _p(batch.t_ep), _p(batch.episode),
+                             t_g0, T, _p(coef), float(coef_V), _p(J), _p(dJ))
     return J, dJ
 
 

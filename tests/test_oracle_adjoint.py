@@ -3,7 +3,10 @@ an action-replay window objective J = sum_t coef_t r_t + <lam_T, x_T>
 computed by forward-mode dual numbers over the model code (oracle
 adjoint_window) against central differences of the same J in double, a
 one-substep closed form, linearity in the direction, the gradient cut at an
-episode end, and zero derivative through clipped thruster commands."""
+episode end, and zero derivative through clipped thruster commands.  The
+closed-loop window of SHAC (policy network inside, terminal critic): its
+value equals the oracle's own rollout, its weight derivative matches central
+differences, and the critic term alone is linear in the direction."""
 import numpy as np
 import pytest
 
@@ -129,3 +132,75 @@ def test_clipped_commands_have_zero_derivative():
     da[:, 5] = rng.normal(size=(T, n))
     _, dJ = O.adjoint_window(m, b, act, coef, lam, np.zeros((13, n)), da)
     assert np.all(dJ == 0.0)
+
+
+# ---------------------------------------------------------------------------
+# Closed loop (SHAC's window with the policy network and a terminal critic)
+# ---------------------------------------------------------------------------
+def _smooth_policy(w, scale_mu=0.15, ls_bias=-3.0):
+    """Policy weights whose actions stay inside the thrusters' range (small
+    mean, sigma = e^-3), so the window objective is smooth in the weights."""
+    pw = W.policy_weights(w).astype(np.float64)
+    H = w["hidden"]
+    o3 = H * 18 + H + H * H + H
+    W3 = pw[o3:o3 + 16 * H].reshape(16, H)
+    W3[:8] *= scale_mu
+    W3[8:] *= 0.1
+    pw[o3 + 16 * H + 8:o3 + 16 * H + 16] = ls_bias
+    return pw.astype(np.float32)
+
+
+def _closed_loop_setup(n=4, T=5, seed=0, **over):
+    w = W.workload("ppo_65536", n_envs=n, hidden=16, w_vs=0.05, mlp="fp32", **over)
+    m = O.model(w)
+    b = O.Batch(np.arange(n) + 3)
+    O.reset(m, b)
+    O.replay(m, b, W.replay_actions(seed + 1, 4, n, scale=0.8))
+    return w, m, b
+
+
+def test_shac_window_value_equals_the_rollout():
+    T, n = 6, 4
+    w, m, b = _closed_loop_setup(n, T)
+    pw = W.policy_weights(w)
+    coef = np.random.default_rng(1).uniform(0.5, 1.5, T)
+    J, _ = O.shac_window(m, b, pw, None, None, 100, T, coef, 0.0)
+    ref = O.rollout(m, b.copy(), pw, None, 100, T, want=("rew",))
+    assert np.allclose(J, coef @ ref["rew"], rtol=1e-12, atol=1e-12)
+
+
+def test_shac_window_derivative_matches_central_differences():
+    T, n = 5, 3
+    w, m, b = _closed_loop_setup(n, T, seed=2)
+    pw = _smooth_policy(w)
+    vw = W.value_weights(w, 0.1)
+    rng = np.random.default_rng(3)
+    coef = rng.uniform(0.5, 1.5, T)
+    d = rng.normal(size=pw.size) * np.abs(pw).mean()
+    J, dJ = O.shac_window(m, b, pw, d, vw, 7, T, coef, 0.7)
+    h = 2e-3
+    Jp, _ = O.shac_window(m, b, (pw + h * d).astype(np.float32), None, vw, 7, T, coef, 0.7)
+    Jm, _ = O.shac_window(m, b, (pw - h * d).astype(np.float32), None, vw, 7, T, coef, 0.7)
+    fd = (Jp - Jm) / (2 * h)
+    assert np.all(np.abs(dJ) > 1e-4)
+    # the perturbed weights are rounded to float32 (the oracle's weight type):
+    # that noise, ~1e-5 of the largest derivative here, bounds the agreement
+    assert np.all(np.abs(dJ - fd) <= 3e-4 * np.abs(fd) + 3e-5 * np.abs(fd).max()), (dJ, fd)
+
+
+def test_shac_terminal_critic_alone():
+    """With coef = 0 only the critic term reaches the weights (through the
+    final state); its derivative is linear in the direction."""
+    T, n = 4, 3
+    w, m, b = _closed_loop_setup(n, T, seed=4)
+    pw = _smooth_policy(w)
+    vw = W.value_weights(w, 0.1)
+    rng = np.random.default_rng(5)
+    d1, d2 = rng.normal(size=pw.size), rng.normal(size=pw.size)
+    _, a = O.shac_window(m, b, pw, d1, vw, 0, T, np.zeros(T), 1.0)
+    _, c = O.shac_window(m, b, pw, d2, vw, 0, T, np.zeros(T), 1.0)
+    _, ac = O.shac_window(m, b, pw, d1 - 3 * d2, vw, 0, T, np.zeros(T), 1.0)
+    assert np.all(np.abs(a) > 0)
+    assert np.allclose(ac, a - 3 * c, rtol=1e-10, atol=1e-14)
+    _, z = O.shac_window(m, b, pw, d1, None, 0, T, np.zeros(T), 1.0)
+    assert np.all(z == 0.0)
