@@ -519,6 +519,32 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
                 float* grad_act, float* lam_0, float* rew_out, uint8_t* done_out, void* stream);
 
 /*
+ * env_shac_window: SHAC's actor gradient over one window in closed loop
+ * (paper §III-A: short-horizon actor-critic; Xu et al. 2022).  From each
+ * env's current state the policy `policy` (env_set_weights layout,
+ * 18 -> hidden -> hidden -> 16: mean and log-std of the 8 commands) acts for
+ * T steps with the reparameterised action a = mu + exp(clamp(ls)) eps (eps:
+ * the rollout's action noise at the env's global steps), and the env
+ * advances (state, counters, global step += T).  With the critic `value`
+ * (same layout, head 1; NULL for none) at the observation after the last
+ * step,
+ *   J = sum over envs [ sum_t coef[t] r_t + coef_V V(o_T) ],
+ * and grad (device memory, the policy's length) receives dJ/d(policy) by
+ * back-propagation through the dynamics, the policy network and the
+ * observation.  Gradients stop at the window's start and at episode ends
+ * inside it (the state after an end is a reset draw).  Optional outputs:
+ * J_out [N] each env's J; rew_out, done_out [T][N]; device or mapped
+ * page-locked host memory.  policy, value, coef [T], grad: device memory.
+ * Fossen model, 1 <= T <= AUV_ADJOINT_MAX_T, at most
+ * AUV_ADJOINT_MAX_SUBSTEPS substeps, hidden a multiple of 8 up to 1024.
+ * The first call at a given (N, T) allocates the window's workspace
+ * (activations of every step: about T N (2 hidden + 80) floats).
+ */
+int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
+                    const float* coef, float coef_V, float* grad, float* J_out, float* rew_out,
+                    uint8_t* done_out, void* stream);
+
+/*
  * env_inverse_allocate: thruster commands for body-frame wrenches, the map
  * the paper's controllers go through at deployment (§V-B: the policy's
  * forces and torques -> individual thrusters through the allocation matrix).

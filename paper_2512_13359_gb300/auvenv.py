@@ -40,7 +40,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
             "env_policy_forward_noalloc", "env_layout", "env_gae", "env_adjoint",
-            "env_inverse_allocate", "rbuf_create", "rbuf_destroy", "rbuf_last_error",
+            "env_inverse_allocate", "env_shac_window", "rbuf_create", "rbuf_destroy", "rbuf_last_error",
             "rbuf_size", "rbuf_insert", "rbuf_sample",
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
@@ -157,6 +157,7 @@ def lib(path: str | None = None):
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
     L.env_inverse_allocate.argtypes = [P, I, P, P, P]
+    L.env_shac_window.argtypes = [P, P, P, I, P, C.c_float, P, P, P, P, P]
     L.rbuf_create.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(P)]
     L.rbuf_destroy.argtypes = [P]
     L.rbuf_last_error.argtypes = [P]
@@ -334,6 +335,14 @@ class Env:
         self._check(lib().env_adjoint(self.h, T, _ptr(act), _ptr(coef), _ptr(lam_T),
                                       _ptr(grad_act), _ptr(lam_0), _ptr(rew), _ptr(done),
                                       _stream(stream)))
+
+    def shac_window(self, policy, value, coef, coef_V, grad, J=None, rew=None, done=None,
+                    stream=None):
+        """SHAC actor gradient over a window of len(coef) steps in closed loop
+        (env_shac_window); the env advances."""
+        self._check(lib().env_shac_window(self.h, _ptr(policy), _ptr(value), coef.shape[0],
+                                          _ptr(coef), float(coef_V), _ptr(grad), _ptr(J),
+                                          _ptr(rew), _ptr(done), _stream(stream)))
 
     def inverse_allocate(self, wrench, cmd, stream=None):
         """Thruster commands cmd [8][n] for wrenches [6][n] (env_inverse_allocate)."""

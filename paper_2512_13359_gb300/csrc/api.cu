@@ -8,6 +8,8 @@
 #include <cstring>
 #include <new>
 
+#include <cublas_v2.h>
+
 #include "auv_kernels.h"
 #include "auv_bf16.h"
 #include "auvenv.h"
@@ -47,6 +49,12 @@ struct auv_env {
   // Inverse allocation (env_inverse_allocate): made on first use.
   bool inv_ready = false;
   auv::InvAlloc inv;
+  // SHAC windows (env_shac_window): workspace for the last (N, T, H) and a
+  // cuBLAS handle, made on first use.
+  char* shac_ws = nullptr;
+  size_t shac_ws_bytes = 0;
+  int shac_T = 0;
+  cublasHandle_t blas = nullptr;
 };
 
 namespace {
@@ -382,6 +390,8 @@ int env_destroy(auv_env* env) {
   cudaError_t e = cudaFree(env->workspace);
   if (env->stage) cudaFree(env->stage);
   if (env->adj_scratch) cudaFree(env->adj_scratch);
+  if (env->shac_ws) cudaFree(env->shac_ws);
+  if (env->blas) cublasDestroy(env->blas);
   for (int b = 0; b < 2; ++b) {
     if (env->seg_done[b]) cudaEventDestroy(env->seg_done[b]);
     if (env->copy_done[b]) cudaEventDestroy(env->copy_done[b]);
@@ -705,6 +715,69 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
                                       static_cast<uint8_t*>(done), env->adj_scratch, env->status,
                                       static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? AUV_OK : cuda_fail(env, e, "adjoint kernel");
+}
+
+int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
+                    const float* coef, float coef_V, float* grad, float* J_out, float* rew_out,
+                    uint8_t* done_out, void* stream) {
+  if (!env) return AUV_ERR_INVALID;
+  int rc = check_device(env);
+  if (rc) return rc;
+  if (is_paper(&env->cfg))
+    return fail(env, AUV_ERR_UNSUPPORTED, "the SHAC window is built for the Fossen model");
+  if (T < 1 || T > AUV_ADJOINT_MAX_T)
+    return fail(env, AUV_ERR_INVALID, "T outside [1, %d]", AUV_ADJOINT_MAX_T);
+  if (env->model.substeps > AUV_ADJOINT_MAX_SUBSTEPS)
+    return fail(env, AUV_ERR_UNSUPPORTED, "the SHAC window supports at most %d substeps",
+                AUV_ADJOINT_MAX_SUBSTEPS);
+  const int H = (int)env->cfg.hidden;
+  if (H < 8 || H > 1024 || H % 8)
+    return fail(env, AUV_ERR_UNSUPPORTED, "the SHAC window needs hidden a multiple of 8 in [8, 1024]");
+  if (!std::isfinite(coef_V)) return fail(env, AUV_ERR_INVALID, "coef_V not finite");
+  if ((rc = check_device_buffer(env, policy, "policy", 4)) ||
+      (rc = check_device_buffer(env, coef, "coef", 4)) ||
+      (rc = check_device_buffer(env, grad, "grad", 4)))
+    return rc;
+  if (value && (rc = check_device_buffer(env, value, "value", 4))) return rc;
+  void *J = nullptr, *rew = nullptr, *done = nullptr;
+  if ((rc = map_output(env, J_out, "J_out", 4, &J)) ||
+      (rc = map_output(env, rew_out, "rew_out", 4, &rew)) ||
+      (rc = map_output(env, done_out, "done_out", 1, &done)))
+    return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const auv::shac::Layout L = auv::shac::layout(env->model.n, T, H);
+  if (!env->blas) {
+    cublasStatus_t bs = cublasCreate(&env->blas);
+    if (bs != CUBLAS_STATUS_SUCCESS) {
+      env->blas = nullptr;
+      return fail(env, AUV_ERR_CUDA, "cuBLAS handle: status %d", (int)bs);
+    }
+  }
+  if (L.bytes > env->shac_ws_bytes || T != env->shac_T) {
+    if (L.bytes > env->shac_ws_bytes) {
+      if (env->shac_ws) {
+        cudaError_t e = cudaFree(env->shac_ws);
+        env->shac_ws = nullptr;
+        env->shac_ws_bytes = 0;
+        if (e != cudaSuccess) return cuda_fail(env, e, "free SHAC workspace");
+      }
+      cudaError_t e = cudaMalloc(&env->shac_ws, L.bytes);
+      if (e != cudaSuccess) {
+        env->shac_ws = nullptr;
+        return cuda_fail(env, e, "cudaMalloc(SHAC workspace)");
+      }
+      env->shac_ws_bytes = L.bytes;
+    }
+    cudaError_t e = auv::shac::init(L, env->shac_ws, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "initialise SHAC workspace");
+    env->shac_T = T;
+  }
+  rc = auv::shac::run_window(env->blas, env->model, env->buf, env->status, L, env->shac_ws,
+                             env->t_g, policy, value, coef, coef_V, grad, static_cast<float*>(J),
+                             static_cast<float*>(rew), static_cast<uint8_t*>(done), s, env->err);
+  if (rc != AUV_OK) return rc;
+  env->t_g += (uint64_t)T;
+  return AUV_OK;
 }
 
 int env_inverse_allocate(auv_env* env, int n, const float* wrench, float* cmd, void* stream) {

@@ -64,6 +64,35 @@ cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, i
                            float* rew, uint8_t* done, float* scratch, Status* st,
                            cudaStream_t s);
 
+// SHAC in closed loop (k_adjoint.cu kernels, shac.cu orchestration).
+namespace shac {
+struct Layout {
+  int n, T, H, Dp, Hp;
+  size_t n_aug_p, n_aug_v;
+  size_t o_X, o_H1, o_H2, o_Y, o_G, o_GX, o_gY, o_lam, o_done, o_rew, o_VH1, o_VH2, o_V, o_gYv,
+      o_wp, o_wv, o_gp, o_sc, bytes;
+};
+Layout layout(int n, int T, int H);
+cudaError_t init(const Layout& L, char* base, cudaStream_t s);
+// blas: a cublasHandle_t.  Returns AUV_OK or an AUV_ERR_* code with err set.
+int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
+               char* base, uint64_t t_g0, const float* policy, const float* value,
+               const float* coef, float coef_V, float* grad, float* J, float* rew_out,
+               uint8_t* done_out, cudaStream_t s, char* err);
+cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
+                       cudaStream_t s);
+cudaError_t launch_step(const Model& M, const Buffers& B, const float* Y, int ldy, uint64_t t_g,
+                        float* rew, uint8_t* done, Status* st, cudaStream_t s);
+cudaError_t launch_bwd(const Model& M, const float* sc, const float* Y, int ldy,
+                       const uint8_t* done, uint64_t t_g, const float* coef, float* lam,
+                       float* gY, cudaStream_t s);
+cudaError_t launch_obs_vjp(const Model& M, const Buffers& B, const float* sc, const float* gX,
+                           int ldx, float* lam, cudaStream_t s);
+cudaError_t launch_objective(int n, int T, const float* rew, const float* coef, const float* V,
+                             int ldv, float coef_V, float* J, cudaStream_t s);
+cudaError_t launch_fill_col(int n, float* buf, int ld, float v, cudaStream_t s);
+}  // namespace shac
+
 // Inverse thruster allocation (rbuf.cu): commands = clip(pinv u-map, -1, 1).
 struct InvAlloc {
   float pinv[48];   // [8][6]: pseudo-inverse of alloc * thrust_max

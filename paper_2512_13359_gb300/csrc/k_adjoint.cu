@@ -424,9 +424,266 @@ __global__ void __launch_bounds__(kAdjThreads) k_adjoint(
   }
 }
 
+// ---------------------------------------------------------------------------
+// SHAC in closed loop: the window's steps one at a time, with the policy
+// network's products done outside (cuBLAS) between these kernels.
+// ---------------------------------------------------------------------------
+
+// dJ/d(state) += (d obs / d state)^T lo for the observation of auv_device.cuh.
+__device__ void obs_vjp(const Env& e, const float lo[kObs], X& lx) {
+  float R[3][3];
+  quat_rot(e.q, R);
+  const float dp[3] = {e.p[0] - e.pd[0], e.p[1] - e.pd[1], e.p[2] - e.pd[2]};
+  float LR[3][3];
+#pragma unroll
+  for (int j = 0; j < 3; ++j) {
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      LR[j][i] = lo[i] * dp[j];                  // o_i = sum_j R[j][i] dp_j
+      lx.p[j] += R[j][i] * lo[i];
+    }
+  }
+  rot_vjp(e.q, LR, lx.q);
+  float qe[4], LRe[3][3];
+  attitude_error(e, qe);
+#pragma unroll
+  for (int j = 0; j < 3; ++j) {
+#pragma unroll
+    for (int i = 0; i < 3; ++i) LRe[i][j] = lo[3 + 3 * j + i];   // o_{3+3j+i} = R(qe)[i][j]
+  }
+  float lqe[4] = {0.f, 0.f, 0.f, 0.f};
+  rot_vjp(qe, LRe, lqe);
+  const float aw = e.qd[0], ax = -e.qd[1], ay = -e.qd[2], az = -e.qd[3];
+  lx.q[0] += aw * lqe[0] + ax * lqe[1] + ay * lqe[2] + az * lqe[3];
+  lx.q[1] += -ax * lqe[0] + aw * lqe[1] + az * lqe[2] - ay * lqe[3];
+  lx.q[2] += -ay * lqe[0] - az * lqe[1] + aw * lqe[2] + ax * lqe[3];
+  lx.q[3] += -az * lqe[0] + ay * lqe[1] - ax * lqe[2] + aw * lqe[3];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lx.nu[k] += lo[12 + k];
+}
+
+__device__ __forceinline__ void load_lam(const float* __restrict__ lam, size_t n, int i, X& lx) {
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lx.p[k] = lam[k * n + i];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lx.q[k] = lam[(3 + k) * n + i];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lx.nu[k] = lam[(7 + k) * n + i];
+}
+
+__device__ __forceinline__ void store_lam(float* __restrict__ lam, size_t n, int i, const X& lx) {
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lam[k * n + i] = lx.p[k];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lam[(3 + k) * n + i] = lx.q[k];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lam[(7 + k) * n + i] = lx.nu[k];
+}
+
+// Reparameterised action a = mu + exp(clamp(ls)) eps from a policy head row.
+__device__ __forceinline__ void shac_action(const Model& M, const float* __restrict__ y,
+                                            const float eps[kAct], float a[kAct],
+                                            float sig[kAct], bool in[kAct]) {
+#pragma unroll
+  for (int k = 0; k < kAct; ++k) {
+    const float raw = y[kAct + k];
+    in[k] = raw >= M.logstd_min && raw <= M.logstd_max;
+    sig[k] = expf(fminf(fmaxf(raw, M.logstd_min), M.logstd_max));
+    a[k] = fmaf(sig[k], eps[k], y[k]);
+  }
+}
+
+// Observation row of the network input (augmented: 1 at column kObs, zeros
+// up to ldx) of each env's current state; with sc, also the step's scratch.
+__global__ void __launch_bounds__(kAdjThreads) k_shac_obs(const Model M, Buffers B,
+                                                          float* __restrict__ sc,
+                                                          float* __restrict__ X, int ldx) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  Env e;
+  load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  if (sc) save_step(sc, (size_t)M.n, i, e);
+  float o[kObs];
+  observe(e, o);
+  float* x = X + (size_t)i * ldx;
+#pragma unroll
+  for (int k = 0; k < kObs; ++k) x[k] = o[k];
+  x[kObs] = 1.0f;
+  for (int k = kObs + 1; k < ldx; ++k) x[k] = 0.0f;
+}
+
+// One closed-loop step from the policy head Y [N][ldy]: action, physics,
+// episode bookkeeping; the env's buffers are advanced.
+__global__ void __launch_bounds__(kAdjThreads) k_shac_step(const Model M, Buffers B,
+                                                           const float* __restrict__ Y, int ldy,
+                                                           uint64_t t_g, float* __restrict__ rew,
+                                                           uint8_t* __restrict__ done,
+                                                           Status* st) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  Env e;
+  load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  const uint32_t id = M.id_base + (uint32_t)i;
+  float eps[kAct], a[kAct], sig[kAct];
+  bool in[kAct];
+  action_noise(id, M.seed, t_g, eps);
+  shac_action(M, Y + (size_t)i * ldy, eps, a, sig, in);
+  bool d;
+  const float r = physics_step(M, id, e, a, &d);
+  if (!env_finite(e)) flag_nan(st, i);
+  store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  rew[i] = r;
+  done[i] = d ? 1 : 0;
+}
+
+// Backward of one closed-loop step: lam (dJ/d post-step state, [13][N]) is
+// replaced by dJ/d pre-step state through the physics, and the policy head's
+// gradient is written to gY [N][ldy] (mean, then the log-std head through
+// a = mu + sigma eps; zero where the clamp is active).
+__global__ void __launch_bounds__(kAdjThreads) k_shac_bwd(const Model M,
+                                                          const float* __restrict__ sc,
+                                                          const float* __restrict__ Y, int ldy,
+                                                          const uint8_t* __restrict__ done,
+                                                          uint64_t t_g, const float* __restrict__ coef,
+                                                          float* __restrict__ lam,
+                                                          float* __restrict__ gY) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  const size_t n = (size_t)M.n;
+  const uint32_t id = M.id_base + (uint32_t)i;
+  X lx;
+  if (done[i]) {
+#pragma unroll
+    for (int k = 0; k < 3; ++k) lx.p[k] = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) lx.q[k] = 0.f;
+#pragma unroll
+    for (int k = 0; k < 6; ++k) lx.nu[k] = 0.f;
+  } else {
+    load_lam(lam, n, i, lx);
+  }
+  Env es;
+  load_step(M, sc, n, i, es);
+  float eps[kAct], a[kAct], sig[kAct], a_c[kAct], tau[6], nup[6];
+  bool in[kAct];
+  action_noise(id, M.seed, t_g, eps);
+  shac_action(M, Y + (size_t)i * ldy, eps, a, sig, in);
+  allocate(M, a, a_c, tau);
+#pragma unroll
+  for (int k = 0; k < 6; ++k) nup[k] = es.nu[k];
+  X xs[8];
+  for (int s = 0; s < M.substeps; ++s) {
+    get_x(es, xs[s]);
+    substep(M, es, tau);
+  }
+  float la[kAct], lnup[6], ltau[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  reward_vjp(M, es, a_c, nup, __ldg(coef), lx, lnup, la);
+  for (int s = M.substeps - 1; s >= 0; --s) substep_vjp(M, es, xs[s], tau, lx, ltau);
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lx.nu[k] += lnup[k];
+  float* g = gY + (size_t)i * ldy;
+#pragma unroll
+  for (int k = 0; k < kAct; ++k) {
+    float ga = la[k];
+#pragma unroll
+    for (int r = 0; r < 6; ++r) ga = fmaf(M.alloc_t[r * kAct + k], ltau[r], ga);
+    if (!(a[k] >= -1.0f && a[k] <= 1.0f)) ga = 0.0f;
+    g[k] = ga;
+    g[kAct + k] = in[k] ? ga * sig[k] * eps[k] : 0.0f;
+  }
+  store_lam(lam, n, i, lx);
+}
+
+// lam += (d obs / d state)^T gX at the state of scratch sc (or of the env's
+// buffers when sc is NULL); gX [N][ldx], first kObs columns.
+__global__ void __launch_bounds__(kAdjThreads) k_shac_obs_vjp(const Model M, Buffers B,
+                                                              const float* __restrict__ sc,
+                                                              const float* __restrict__ gX,
+                                                              int ldx, float* __restrict__ lam) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  const size_t n = (size_t)M.n;
+  Env e;
+  if (sc) {
+    load_step(M, sc, n, i, e);
+  } else {
+    load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  }
+  float lo[kObs];
+#pragma unroll
+  for (int k = 0; k < kObs; ++k) lo[k] = gX[(size_t)i * ldx + k];
+  X lx;
+  load_lam(lam, n, i, lx);
+  obs_vjp(e, lo, lx);
+  store_lam(lam, n, i, lx);
+}
+
+// J_i = sum_t coef_t r_t + coef_V V_i (V [N][ldv], column 0; NULL for none).
+__global__ void __launch_bounds__(kAdjThreads) k_shac_objective(int n, int T,
+                                                                const float* __restrict__ rew,
+                                                                const float* __restrict__ coef,
+                                                                const float* __restrict__ V,
+                                                                int ldv, float coef_V,
+                                                                float* __restrict__ J) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= n) return;
+  float s = 0.0f;
+  for (int t = 0; t < T; ++t) s = fmaf(__ldg(coef + t), rew[(size_t)t * n + i], s);
+  if (V) s = fmaf(coef_V, V[(size_t)i * ldv], s);
+  J[i] = s;
+}
+
+__global__ void __launch_bounds__(kAdjThreads) k_fill_col(int n, float* __restrict__ buf, int ld,
+                                                          float v) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i < n) buf[(size_t)i * ld] = v;
+}
+
 }  // namespace
 
 size_t adjoint_scratch_floats(int n, int T) { return (size_t)T * kScratchF * (size_t)n; }
+
+namespace shac {
+
+static unsigned blocks(int n) { return (n + kAdjThreads - 1) / kAdjThreads; }
+
+cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
+                       cudaStream_t s) {
+  k_shac_obs<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_step(const Model& M, const Buffers& B, const float* Y, int ldy, uint64_t t_g,
+                        float* rew, uint8_t* done, Status* st, cudaStream_t s) {
+  k_shac_step<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, Y, ldy, t_g, rew, done, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bwd(const Model& M, const float* sc, const float* Y, int ldy,
+                       const uint8_t* done, uint64_t t_g, const float* coef, float* lam,
+                       float* gY, cudaStream_t s) {
+  k_shac_bwd<<<blocks(M.n), kAdjThreads, 0, s>>>(M, sc, Y, ldy, done, t_g, coef, lam, gY);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_obs_vjp(const Model& M, const Buffers& B, const float* sc, const float* gX,
+                           int ldx, float* lam, cudaStream_t s) {
+  k_shac_obs_vjp<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, gX, ldx, lam);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_objective(int n, int T, const float* rew, const float* coef, const float* V,
+                             int ldv, float coef_V, float* J, cudaStream_t s) {
+  k_shac_objective<<<blocks(n), kAdjThreads, 0, s>>>(n, T, rew, coef, V, ldv, coef_V, J);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fill_col(int n, float* buf, int ld, float v, cudaStream_t s) {
+  k_fill_col<<<blocks(n), kAdjThreads, 0, s>>>(n, buf, ld, v);
+  return cudaGetLastError();
+}
+
+}  // namespace shac
 
 cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, int T,
                            const float* coef, const float* lam_T, float* g_act, float* lam_0,

@@ -1,0 +1,204 @@
+// shac.cu -- SHAC's actor gradient over a window in closed loop (paper §III-A:
+// short-horizon actor-critic; Xu et al. 2022): the policy acts through the
+// differentiable step for T steps, and back-propagation through the
+// dynamics, the policy network and the observation gives dJ/dtheta of
+//   J = sum_i [ sum_t coef_t r_t,i + coef_V V(o_T,i) ]
+// (theta: the policy weights; V: the terminal critic; actions reparameterised
+// as a = mu(o) + exp(clamp(ls(o))) eps with the rollout's action noise eps).
+//
+// Per step the per-env work (observation, action, physics and their VJPs)
+// runs in the k_shac_* kernels of k_adjoint.cu; the policy network's dense
+// products run in cuBLAS (fp32 compute) on the augmented layout of the PPO
+// learner (a constant-1 input column carries each bias).  Forward: for each
+// step, observation -> policy GEMMs (activations kept for every step) ->
+// action and physics (the env advances).  Backward, t = T-1 .. 0: physics
+// VJP of step t (the state adjoint lam and the head gradient), the policy's
+// backward (weight gradients accumulated over steps, input gradient), then
+// the observation VJP into lam.  The terminal critic seeds lam with
+// coef_V dV(o(x_T))/dx_T through the value network's input gradient.
+#include <cublas_v2.h>
+
+#include <cstdio>
+
+#include "auv_kernels.h"
+#include "auvenv.h"
+
+namespace auv {
+namespace shac {
+
+namespace {
+
+int round8(int x) { return (x + 7) & ~7; }
+
+struct Gemm {
+  cublasHandle_t h;
+  cublasStatus_t operator()(cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
+                            const float* A, int lda, const float* B, int ldb, float* C, int ldc,
+                            float beta = 0.0f) const {
+    const float one = 1.0f;
+    return cublasGemmEx(h, ta, tb, m, n, k, &one, A, CUDA_R_32F, lda, B, CUDA_R_32F, ldb, &beta,
+                        C, CUDA_R_32F, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+  }
+};
+
+constexpr int kLdy = 16;   // policy head row (2 x 8)
+constexpr int kLdv = 8;    // value head row
+
+}  // namespace
+
+Layout layout(int n, int T, int H) {
+  Layout L;
+  L.n = n;
+  L.T = T;
+  L.H = H;
+  L.Dp = round8(kObs + 1);
+  L.Hp = round8(H + 1);
+  L.n_aug_p = ppo::aug_count(kObs, L.Dp, H, L.Hp, 2 * kAct);
+  L.n_aug_v = ppo::aug_count(kObs, L.Dp, H, L.Hp, 1);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) & ~(size_t)255;
+    return o;
+  };
+  const size_t N = (size_t)n;
+  L.o_X = take((T + 1) * N * L.Dp * 4);
+  L.o_H1 = take(T * N * L.Hp * 4);
+  L.o_H2 = take(T * N * L.Hp * 4);
+  L.o_Y = take(T * N * kLdy * 4);
+  L.o_G = take(N * H * 4);
+  L.o_GX = take(N * L.Dp * 4);
+  L.o_gY = take(N * kLdy * 4);
+  L.o_lam = take(13 * N * 4);
+  L.o_done = take(T * N);
+  L.o_rew = take(T * N * 4);
+  L.o_VH1 = take(N * L.Hp * 4);
+  L.o_VH2 = take(N * L.Hp * 4);
+  L.o_V = take(N * kLdv * 4);
+  L.o_gYv = take(N * kLdv * 4);
+  L.o_wp = take(L.n_aug_p * 4);
+  L.o_wv = take(L.n_aug_v * 4);
+  L.o_gp = take(L.n_aug_p * 4);
+  L.o_sc = take(adjoint_scratch_floats(n, T) * 4);
+  L.bytes = off;
+  return L;
+}
+
+cudaError_t init(const Layout& L, char* base, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(base, 0, L.bytes, s);
+  float* h1 = reinterpret_cast<float*>(base + L.o_H1);
+  float* h2 = reinterpret_cast<float*>(base + L.o_H2);
+  const int rows = L.T * L.n;
+  if (e == cudaSuccess) e = ppo::launch_fill_ones(false, h1, L.Hp, L.H, rows, s);
+  if (e == cudaSuccess) e = ppo::launch_fill_ones(false, h2, L.Hp, L.H, rows, s);
+  if (e == cudaSuccess)
+    e = ppo::launch_fill_ones(false, base + L.o_VH1, L.Hp, L.H, L.n, s);
+  if (e == cudaSuccess)
+    e = ppo::launch_fill_ones(false, base + L.o_VH2, L.Hp, L.H, L.n, s);
+  return e;
+}
+
+int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
+               char* base, uint64_t t_g0, const float* policy, const float* value,
+               const float* coef, float coef_V, float* grad, float* J, float* rew_out,
+               uint8_t* done_out, cudaStream_t s, char* err) {
+  const int n = L.n, T = L.T, H = L.H, Dp = L.Dp, Hp = L.Hp;
+  const size_t N = (size_t)n;
+  auto F = [&](size_t o) { return reinterpret_cast<float*>(base + o); };
+  float *X = F(L.o_X), *H1 = F(L.o_H1), *H2 = F(L.o_H2), *Y = F(L.o_Y), *G = F(L.o_G),
+        *GX = F(L.o_GX), *gY = F(L.o_gY), *lam = F(L.o_lam), *rew = F(L.o_rew),
+        *VH1 = F(L.o_VH1), *VH2 = F(L.o_VH2), *V = F(L.o_V), *gYv = F(L.o_gYv),
+        *wp = F(L.o_wp), *wv = F(L.o_wv), *gp = F(L.o_gp), *sc = F(L.o_sc);
+  uint8_t* done = reinterpret_cast<uint8_t*>(base + L.o_done);
+  auto Xs = [&](int t) { return X + (size_t)t * N * Dp; };
+  auto H1s = [&](int t) { return H1 + (size_t)t * N * Hp; };
+  auto H2s = [&](int t) { return H2 + (size_t)t * N * Hp; };
+  auto Ys = [&](int t) { return Y + (size_t)t * N * kLdy; };
+  auto SCs = [&](int t) { return sc + (size_t)t * adjoint_scratch_floats(n, 1); };
+  const float *w1 = wp, *w2 = wp + (size_t)H * Dp, *w3 = w2 + (size_t)H * Hp;
+  float *g1 = gp, *g2 = gp + (size_t)H * Dp, *g3 = g2 + (size_t)H * Hp;
+  const float *v1 = wv, *v2 = wv + (size_t)H * Dp, *v3 = v2 + (size_t)H * Hp;
+
+  cublasHandle_t h = static_cast<cublasHandle_t>(blas);
+  Gemm gemm{h};
+  cublasStatus_t bs = cublasSetStream(h, s);
+  cudaError_t e = cudaSuccess;
+  auto cfail = [&](cudaError_t x, const char* what) {
+    snprintf(err, 256, "%s: %s", what, cudaGetErrorString(x));
+    return AUV_ERR_CUDA;
+  };
+  auto bfail = [&](cublasStatus_t x, const char* what) {
+    snprintf(err, 256, "%s: cuBLAS status %d", what, (int)x);
+    return AUV_ERR_CUDA;
+  };
+  if (bs) return bfail(bs, "cublasSetStream");
+  const auto T_ = CUBLAS_OP_T, N_ = CUBLAS_OP_N;
+
+  // weights into the augmented layout; gradient accumulator to zero
+  if ((e = ppo::launch_convert(const_cast<float*>(policy), wp, kObs, Dp, H, Hp, 2 * kAct, true, s)))
+    return cfail(e, "policy weights");
+  if (value &&
+      (e = ppo::launch_convert(const_cast<float*>(value), wv, kObs, Dp, H, Hp, 1, true, s)))
+    return cfail(e, "value weights");
+  if ((e = cudaMemsetAsync(gp, 0, L.n_aug_p * 4, s))) return cfail(e, "clear gradient");
+
+  // ---- forward ----
+  for (int t = 0; t < T; ++t) {
+    if ((e = launch_obs(M, B, SCs(t), Xs(t), Dp, s))) return cfail(e, "observation");
+    if ((bs = gemm(T_, N_, H, n, Dp, w1, Dp, Xs(t), Dp, H1s(t), Hp))) return bfail(bs, "policy 1");
+    if ((e = ppo::launch_tanh_fwd(false, H1s(t), Hp, n, H, s))) return cfail(e, "tanh");
+    if ((bs = gemm(T_, N_, H, n, Hp, w2, Hp, H1s(t), Hp, H2s(t), Hp))) return bfail(bs, "policy 2");
+    if ((e = ppo::launch_tanh_fwd(false, H2s(t), Hp, n, H, s))) return cfail(e, "tanh");
+    if ((bs = gemm(T_, N_, 2 * kAct, n, Hp, w3, Hp, H2s(t), Hp, Ys(t), kLdy)))
+      return bfail(bs, "policy 3");
+    if ((e = launch_step(M, B, Ys(t), kLdy, t_g0 + (uint64_t)t, rew + (size_t)t * N,
+                         done + (size_t)t * N, st, s)))
+      return cfail(e, "step");
+  }
+  if ((e = cudaMemsetAsync(lam, 0, 13 * N * 4, s))) return cfail(e, "clear adjoint");
+  // ---- terminal critic: lam = coef_V dV(o(x_T))/dx_T ----
+  if (value) {
+    if ((e = launch_obs(M, B, nullptr, Xs(T), Dp, s))) return cfail(e, "observation");
+    if ((bs = gemm(T_, N_, H, n, Dp, v1, Dp, Xs(T), Dp, VH1, Hp))) return bfail(bs, "value 1");
+    if ((e = ppo::launch_tanh_fwd(false, VH1, Hp, n, H, s))) return cfail(e, "tanh");
+    if ((bs = gemm(T_, N_, H, n, Hp, v2, Hp, VH1, Hp, VH2, Hp))) return bfail(bs, "value 2");
+    if ((e = ppo::launch_tanh_fwd(false, VH2, Hp, n, H, s))) return cfail(e, "tanh");
+    if ((bs = gemm(T_, N_, 1, n, Hp, v3, Hp, VH2, Hp, V, kLdv))) return bfail(bs, "value 3");
+    if ((e = launch_fill_col(n, gYv, kLdv, coef_V, s))) return cfail(e, "critic seed");
+    if ((bs = gemm(N_, N_, H, n, 1, v3, Hp, gYv, kLdv, G, H))) return bfail(bs, "value dH2");
+    if ((e = ppo::launch_tanh_bwd(false, G, H, VH2, Hp, n, H, s))) return cfail(e, "tanh'");
+    if ((bs = gemm(N_, N_, H, n, H, v2, Hp, G, H, VH2, Hp))) return bfail(bs, "value dH1");
+    if ((e = ppo::launch_tanh_bwd(false, VH2, Hp, VH1, Hp, n, H, s))) return cfail(e, "tanh'");
+    if ((bs = gemm(N_, N_, Dp, n, H, v1, Dp, VH2, Hp, GX, Dp))) return bfail(bs, "value dX");
+    if ((e = launch_obs_vjp(M, B, nullptr, GX, Dp, lam, s))) return cfail(e, "observation VJP");
+  }
+  if (J && (e = launch_objective(n, T, rew, coef, value ? V : nullptr, kLdv, coef_V, J, s)))
+    return cfail(e, "objective");
+  // ---- backward through the window ----
+  for (int t = T - 1; t >= 0; --t) {
+    if ((e = launch_bwd(M, SCs(t), Ys(t), kLdy, done + (size_t)t * N, t_g0 + (uint64_t)t,
+                        coef + t, lam, gY, s)))
+      return cfail(e, "step VJP");
+    if ((bs = gemm(N_, T_, Hp, 2 * kAct, n, H2s(t), Hp, gY, kLdy, g3, Hp, 1.0f)))
+      return bfail(bs, "dW3");
+    if ((bs = gemm(N_, N_, H, n, 2 * kAct, w3, Hp, gY, kLdy, G, H))) return bfail(bs, "dH2");
+    if ((e = ppo::launch_tanh_bwd(false, G, H, H2s(t), Hp, n, H, s))) return cfail(e, "tanh'");
+    if ((bs = gemm(N_, T_, Hp, H, n, H1s(t), Hp, G, H, g2, Hp, 1.0f))) return bfail(bs, "dW2");
+    if ((bs = gemm(N_, N_, H, n, H, w2, Hp, G, H, H2s(t), Hp))) return bfail(bs, "dH1");
+    if ((e = ppo::launch_tanh_bwd(false, H2s(t), Hp, H1s(t), Hp, n, H, s)))
+      return cfail(e, "tanh'");
+    if ((bs = gemm(N_, T_, Dp, H, n, Xs(t), Dp, H2s(t), Hp, g1, Dp, 1.0f))) return bfail(bs, "dW1");
+    if ((bs = gemm(N_, N_, Dp, n, H, w1, Dp, H2s(t), Hp, GX, Dp))) return bfail(bs, "dX");
+    if ((e = launch_obs_vjp(M, B, SCs(t), GX, Dp, lam, s))) return cfail(e, "observation VJP");
+  }
+  if ((e = ppo::launch_convert(grad, gp, kObs, Dp, H, Hp, 2 * kAct, false, s)))
+    return cfail(e, "gradient layout");
+  if (rew_out && (e = cudaMemcpyAsync(rew_out, rew, T * N * 4, cudaMemcpyDefault, s)))
+    return cfail(e, "copy rewards");
+  if (done_out && (e = cudaMemcpyAsync(done_out, done, T * N, cudaMemcpyDefault, s)))
+    return cfail(e, "copy dones");
+  return AUV_OK;
+}
+
+}  // namespace shac
+}  // namespace auv
