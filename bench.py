@@ -62,7 +62,9 @@ def parse():
                     help="minibatches per epoch (default: all rows / minibatch)")
     ap.add_argument("--adjoint", action="store_true",
                     help="time the control-step adjoint (env_adjoint) over an action window")
-    ap.add_argument("--window", type=int, default=32, help="adjoint window length")
+    ap.add_argument("--window", type=int, default=32, help="adjoint / SHAC window length")
+    ap.add_argument("--shac", action="store_true",
+                    help="time SHAC's closed-loop window (env_shac_window)")
     ap.add_argument("--rbuf", action="store_true",
                     help="time replay-buffer insert (a rollout's trajectory) and sampling")
     ap.add_argument("--invalloc", action="store_true",
@@ -613,8 +615,56 @@ def run_invalloc(args):
     print(json.dumps(line), flush=True)
 
 
+def run_shac(args):
+    """SHAC's actor gradient over one window in closed loop (env_shac_window):
+    forward with the policy network, then back-propagation through the
+    dynamics, the network and the observation, with the terminal critic.
+    FP32 roofline: the policy network's forward, weight gradients and input
+    gradients (3 x 148,480 flop per env-step) plus the physics forward and
+    adjoint (5,988 flop per env-step, k_adjoint's count)."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    over = {"n_envs": args.n_envs} if args.n_envs else {}
+    w = W.workload(args.workload, mlp="fp32", **over)
+    n, T, H = int(w["n_envs"]), int(args.window), int(w["hidden"])
+    env = auvenv.Env(w)
+    env.reset()
+    pw = torch.from_numpy(W.policy_weights(w, 0.05)).cuda()
+    vw = torch.from_numpy(W.value_weights(w, 0.1)).cuda()
+    coef = torch.tensor([0.99 ** t / (n * T) for t in range(T)], dtype=torch.float32,
+                        device="cuda")
+    grad = torch.empty_like(pw)
+    ms = _timed(args, lambda: env.shac_window(pw, vw, coef, 0.99 ** T / n, grad))
+    assert env.status().code == 0
+    rate = n * T / (ms * 1e-3)
+    fps = 3 * mlp_flops(W.obs_dim(w), H, 16) + ADJOINT_FLOPS_PER_ENV_STEP.get(int(w["substeps"]), 0)
+    peaks, src = load_peaks()
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+    achieved = rate * fps / 1e12
+    line = {
+        "metric": "SHAC window env-steps/s", "value": rate, "unit": "env-steps/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (workload resets, seeded random policy and critic)",
+        "config": {"workload": w["name"], "n_envs": n, "window": T, "hidden": H,
+                   "l2": "working set per window (activations of every step) larger than L2"},
+        "roofline": {"bound": "alu", "kernel": "whole window (cuBLAS fp32 GEMMs + own kernels)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "peak_source": f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz",
+                     "flops_per_env_step": fps},
+        "gpu_launches": args.steps * (17 * T + 16), "clocks": None,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.shac:
+        run_shac(args)
+        return
     if args.rbuf:
         run_rbuf(args)
         return
