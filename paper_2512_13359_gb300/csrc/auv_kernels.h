@@ -135,8 +135,20 @@ struct LossHp {
 };
 
 struct AdamHp {
-  float lr, b1, b2, eps, c1, c2;   // c1 = 1 - b1^t, c2 = 1 - b2^t
+  float lr, b1, b2, eps;
   float max_norm;
+};
+
+// Per-step variables of an update, in device memory so that one captured
+// step (a CUDA graph) can be replayed: step s of the update gathers
+// minibatch s mod n_mb of epoch epoch0 + s / n_mb, and Adam takes its step
+// t + 1 (bias corrections 1 - b^(t+1)); launch_step_advance then moves to
+// the next step.
+struct StepCtl {
+  unsigned long long epoch0;
+  unsigned long long t;
+  unsigned int n_mb;
+  unsigned int step;
 };
 
 struct Sample {                    // gathered minibatch, sample-major
@@ -152,10 +164,12 @@ constexpr int kNormBlocks = 256;   // blocks of the gradient-norm reduction
 size_t aug_count(int in, int in_p, int H, int Hp, int out);
 // X [B][Dp]: the gathered observations with the constant 1 at column D,
 // fp32 or bf16 (Dims::bf16), as are the activation arguments below.
-cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
+// k: the permutation of the batch's rows (its epoch words are taken from ctl).
+cudaError_t launch_gather(const Dims& d, const PermKey& k, const StepCtl* ctl, const float* obs,
                           const float* act, const float* logp, const float* adv,
                           const float* ret, uint32_t N, const Sample& out, void* X,
                           cudaStream_t s);
+cudaError_t launch_step_advance(StepCtl* ctl, cudaStream_t s);
 cudaError_t launch_tanh_fwd(bool bf16, void* h, int ld, int B, int H, cudaStream_t s);
 cudaError_t launch_tanh_bwd(bool bf16, void* g, int ldg, const void* h, int ldh, int B, int H,
                             cudaStream_t s);
@@ -166,7 +180,8 @@ cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, flo
                          float* acc, cudaStream_t s);
 // wb (bf16 copy of w, may be NULL) is rewritten with the new weights.
 cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
-                        const AdamHp& hp, float* mb, float* acc, void* wb, cudaStream_t s);
+                        const AdamHp& hp, const StepCtl* ctl, float* mb, float* acc, void* wb,
+                        cudaStream_t s);
 cudaError_t launch_to_bf16(const float* w, void* wb, size_t n, cudaStream_t s);
 cudaError_t launch_finish(const float* acc, float* out, cudaStream_t s);
 // flat [W1|b1|W2|b2|W3|b3] <-> augmented [W1a|W2a|W3a] of one network

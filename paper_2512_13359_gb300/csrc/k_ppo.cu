@@ -137,7 +137,7 @@ __device__ __forceinline__ void block_sum(V (&v)[NV], V* sh /* [NV][kT/32] */) {
 }
 
 template <typename TX>
-__global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, uint32_t start,
+__global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, const StepCtl* ctl,
                                                const float* __restrict__ obs,
                                                const float* __restrict__ act,
                                                const float* __restrict__ logp,
@@ -146,15 +146,34 @@ __global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, uint32_t sta
                                                Sample out, TX* __restrict__ X) {
   __shared__ double sh[2 * (kT / 32)];
   const int b = blockIdx.x * kT + threadIdx.x;
+  const unsigned long long epoch = ctl->epoch0 + ctl->step / ctl->n_mb;
+  const uint32_t start = (ctl->step % ctl->n_mb) * (uint32_t)d.B;
+  key.e0 = (uint32_t)epoch;
+  key.e1 = (uint32_t)(epoch >> 32);
   double s[2] = {0.0, 0.0};
   if (b < d.B) {
     const uint32_t r = perm_index(start + (uint32_t)b, key);
     const size_t t = r / N, i = r - (uint32_t)t * N, n = N;
     TX* x = X + (size_t)b * d.Dp;
-    for (int k = 0; k < d.D; ++k) st_act(x + k, __ldg(obs + (t * d.D + k) * n + i));
+    // loads in chunks of 8 so that several are in flight per thread
+    for (int k0 = 0; k0 < d.D; k0 += 8) {
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (k0 + j < d.D) v[j] = __ldg(obs + (t * d.D + k0 + j) * n + i);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (k0 + j < d.D) st_act(x + k0 + j, v[j]);
+    }
     st_act(x + d.D, 1.0f);
     for (int k = d.D + 1; k < d.Dp; ++k) st_act(x + k, 0.0f);
-    for (int k = 0; k < d.A; ++k) out.act[(size_t)b * d.A + k] = __ldg(act + (t * d.A + k) * n + i);
+    float av[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k < d.A) av[k] = __ldg(act + (t * d.A + k) * n + i);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k < d.A) out.act[(size_t)b * d.A + k] = av[k];
     const size_t o = t * n + i;
     const float a = __ldg(adv + o);
     out.logp[b] = __ldg(logp + o);
@@ -347,16 +366,21 @@ __global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_
 __global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float* __restrict__ g,
                                              float* __restrict__ m, float* __restrict__ v,
                                              size_t n, const float* __restrict__ part, AdamHp hp,
-                                             float* mb, float* acc,
+                                             const StepCtl* ctl, float* mb, float* acc,
                                              __nv_bfloat16* __restrict__ wb) {
   __shared__ double sh[kT / 32];
-  __shared__ float scale_sh;
+  __shared__ float scale_sh, c1_sh, c2_sh;
   double s[1] = {0.0};
   for (int k = threadIdx.x; k < kNormBlocks; k += kT) s[0] += part[k];
   block_sum<1>(s, sh);
   if (threadIdx.x == 0) {
     const double norm = sqrt(s[0]);
     scale_sh = hp.max_norm > 0.0f ? (float)fmin(1.0, hp.max_norm / (norm + 1e-6)) : 1.0f;
+    // bias corrections of step t + 1; beta = 0 keeps the plain moment
+    const double t1 = (double)(ctl->t + 1ull);
+    const double c1 = 1.0 - pow((double)hp.b1, t1), c2 = 1.0 - pow((double)hp.b2, t1);
+    c1_sh = c1 > 0.0 ? (float)c1 : 1.0f;
+    c2_sh = c2 > 0.0 ? (float)c2 : 1.0f;
     if (blockIdx.x == 0) {
       mb[5] = (float)norm;
       if (acc) acc[5] += (float)norm;
@@ -364,6 +388,7 @@ __global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float*
   }
   __syncthreads();
   const float scale = scale_sh;
+  const float c1 = c1_sh, c2 = c2_sh;
   const float ib1 = 1.0f - hp.b1, ib2 = 1.0f - hp.b2;
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
     const float gi = g[e] * scale;
@@ -371,7 +396,7 @@ __global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float*
     const float vi = hp.b2 * v[e] + ib2 * gi * gi;
     m[e] = mi;
     v[e] = vi;
-    const float wi = w[e] - hp.lr * (mi / hp.c1) / (sqrtf(vi / hp.c2) + hp.eps);
+    const float wi = w[e] - hp.lr * (mi / c1) / (sqrtf(vi / c2) + hp.eps);
     w[e] = wi;
     if (wb) wb[e] = __float2bfloat16_rn(wi);
   }
@@ -381,6 +406,11 @@ __global__ void __launch_bounds__(kT) k_to_bf16(const float* __restrict__ w,
                                                 __nv_bfloat16* __restrict__ wb, size_t n) {
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT)
     wb[e] = __float2bfloat16_rn(w[e]);
+}
+
+__global__ void k_step_advance(StepCtl* ctl) {
+  ctl->step += 1u;
+  ctl->t += 1ull;
 }
 
 __global__ void k_finish(const float* __restrict__ acc, float* __restrict__ out) {
@@ -442,17 +472,22 @@ size_t aug_count(int in, int in_p, int H, int Hp, int out) {
   return (size_t)H * in_p + (size_t)H * Hp + (size_t)out * Hp;
 }
 
-cudaError_t launch_gather(const Dims& d, const PermKey& k, uint32_t start, const float* obs,
+cudaError_t launch_gather(const Dims& d, const PermKey& k, const StepCtl* ctl, const float* obs,
                           const float* act, const float* logp, const float* adv,
                           const float* ret, uint32_t N, const Sample& out, void* X,
                           cudaStream_t s) {
   const unsigned nb = (d.B + kT - 1) / kT;
   if (d.bf16)
-    k_gather<<<nb, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out,
+    k_gather<<<nb, kT, 0, s>>>(d, k, ctl, obs, act, logp, adv, ret, N, out,
                                static_cast<__nv_bfloat16*>(X));
   else
-    k_gather<<<nb, kT, 0, s>>>(d, k, start, obs, act, logp, adv, ret, N, out,
+    k_gather<<<nb, kT, 0, s>>>(d, k, ctl, obs, act, logp, adv, ret, N, out,
                                static_cast<float*>(X));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_step_advance(StepCtl* ctl, cudaStream_t s) {
+  k_step_advance<<<1, 1, 0, s>>>(ctl);
   return cudaGetLastError();
 }
 
@@ -496,9 +531,10 @@ cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, flo
 }
 
 cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
-                        const AdamHp& hp, float* mb, float* acc, void* wb, cudaStream_t s) {
+                        const AdamHp& hp, const StepCtl* ctl, float* mb, float* acc, void* wb,
+                        cudaStream_t s) {
   k_sumsq<<<kNormBlocks, kT, 0, s>>>(g, n, part);
-  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, mb, acc,
+  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, ctl, mb, acc,
                                     static_cast<__nv_bfloat16*>(wb));
   return cudaGetLastError();
 }

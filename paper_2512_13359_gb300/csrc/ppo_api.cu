@@ -50,8 +50,16 @@ struct auv_ppo {
   void *g_y, *g_v;            // dL/d(head), same shapes
   float *head_part, *norm_part;
   float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
+  ppo::StepCtl* ctl;          // device: per-step variables
   void* blas_ws;
   uint64_t t, epoch;
+  // One gradient step captured as a CUDA graph for ppo_update, replayed on a
+  // private stream; valid for the batch it was captured with.
+  cudaStream_t gstream = nullptr;
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  cudaGraphExec_t step_graph = nullptr;
+  auv_ppo_batch graph_batch;
+  bool graph_failed = false;
   char err[256];
 };
 
@@ -244,12 +252,20 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
   return AUV_OK;
 }
 
-int grads_impl(auv_ppo* p, const auv_ppo_batch* b, uint64_t epoch, uint32_t j, float* acc,
-               cudaStream_t s) {
+// The step variables for the next launches on s (copied from pageable host
+// memory: the call returns once the source has been staged).
+int set_ctl(auv_ppo* p, uint64_t epoch0, uint32_t n_mb, uint32_t step, uint64_t t,
+            cudaStream_t s) {
+  const ppo::StepCtl c = {epoch0, t, n_mb, step};
+  cudaError_t e = cudaMemcpyAsync(p->ctl, &c, sizeof(c), cudaMemcpyHostToDevice, s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "step control");
+}
+
+int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
   const ppo::Dims& d = p->d;
   const uint32_t m = b->T * b->N;
-  cudaError_t e = ppo::launch_gather(d, perm_key(p, m, epoch), j * (uint32_t)d.B, b->obs, b->act,
-                                     b->logp, b->adv, b->ret, b->N, p->smp, p->X, s);
+  cudaError_t e = ppo::launch_gather(d, perm_key(p, m, 0), p->ctl, b->obs, b->act, b->logp,
+                                     b->adv, b->ret, b->N, p->smp, p->X, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "gather");
   int rc;
   if ((rc = forward(p, 0, s)) || (rc = forward(p, 1, s))) return rc;
@@ -261,24 +277,58 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, uint64_t epoch, uint32_t j, f
   return AUV_OK;
 }
 
+// Adam step t + 1 with t from the step control (the caller advances p->t).
 int apply_impl(auv_ppo* p, float* acc, cudaStream_t s) {
   const auv_ppo_config& c = p->cfg;
-  const uint64_t t = p->t + 1;
   ppo::AdamHp hp;
   hp.lr = c.lr;
   hp.b1 = c.adam_beta1;
   hp.b2 = c.adam_beta2;
   hp.eps = c.adam_eps;
-  hp.c1 = (float)(1.0 - std::pow((double)c.adam_beta1, (double)t));
-  hp.c2 = (float)(1.0 - std::pow((double)c.adam_beta2, (double)t));
   hp.max_norm = c.max_grad_norm;
-  if (!(hp.c1 > 0.0f)) hp.c1 = 1.0f;   // beta1 = 0 keeps the plain moment
-  if (!(hp.c2 > 0.0f)) hp.c2 = 1.0f;
-  cudaError_t e = ppo::launch_adam(p->w, p->g, p->m, p->v, p->n_aug_all, p->norm_part, hp, p->mb,
-                                   acc, p->wb, s);
-  if (e != cudaSuccess) return cuda_fail(p, e, "Adam");
-  p->t = t;
-  return AUV_OK;
+  cudaError_t e = ppo::launch_adam(p->w, p->g, p->m, p->v, p->n_aug_all, p->norm_part, hp, p->ctl,
+                                   p->mb, acc, p->wb, s);
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "Adam");
+}
+
+// One whole gradient step of an update (gather .. Adam, then the step
+// control advances), captured once per batch into p->step_graph on the
+// private stream.  On any capture failure the update launches directly.
+bool same_batch(const auv_ppo_batch& a, const auv_ppo_batch& b) {
+  return a.obs == b.obs && a.act == b.act && a.logp == b.logp && a.adv == b.adv &&
+         a.ret == b.ret && a.T == b.T && a.N == b.N;
+}
+
+void drop_graph(auv_ppo* p) {
+  if (p->step_graph) cudaGraphExecDestroy(p->step_graph);
+  p->step_graph = nullptr;
+}
+
+bool capture_step(auv_ppo* p, const auv_ppo_batch* b) {
+  drop_graph(p);
+  if (!p->gstream &&
+      (cudaStreamCreateWithFlags(&p->gstream, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaEventCreateWithFlags(&p->ev_in, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&p->ev_out, cudaEventDisableTiming) != cudaSuccess))
+    return false;
+  if (cublasSetStream(p->blas, p->gstream) != CUBLAS_STATUS_SUCCESS) return false;
+  if (cudaStreamBeginCapture(p->gstream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+    return false;
+  const bool ok = grads_impl(p, b, p->acc, p->gstream) == AUV_OK &&
+                  apply_impl(p, p->acc, p->gstream) == AUV_OK &&
+                  ppo::launch_step_advance(p->ctl, p->gstream) == cudaSuccess;
+  cudaGraph_t g = nullptr;
+  const cudaError_t e = cudaStreamEndCapture(p->gstream, &g);
+  bool done = ok && e == cudaSuccess && g &&
+              cudaGraphInstantiate(&p->step_graph, g, 0) == cudaSuccess;
+  if (g) cudaGraphDestroy(g);
+  if (!done) {
+    p->step_graph = nullptr;
+    cudaGetLastError();
+    return false;
+  }
+  p->graph_batch = *b;
+  return true;
 }
 
 // Convert both networks between a caller's flat parameter vector (device
@@ -371,7 +421,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_ret = take(B * 4), o_ap = take(nb * 2 * 8), o_gy = take(B * d.ld_pol * es),
                o_gv = take(B * d.ld_val * es), o_hp = take(nb * 5 * 4),
                o_np = take(ppo::kNormBlocks * 4), o_mb = take(AUV_PPO_STATS * 4),
-               o_acc = take(AUV_PPO_STATS * 4), o_ws = take(kBlasWorkspace);
+               o_acc = take(AUV_PPO_STATS * 4), o_ctl = take(sizeof(ppo::StepCtl)),
+               o_ws = take(kBlasWorkspace);
   size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
   for (int k = 0; k < 2; ++k) {
     o_h1[k] = take(B * d.Hp * es);
@@ -403,6 +454,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   p->norm_part = reinterpret_cast<float*>(base + o_np);
   p->mb = reinterpret_cast<float*>(base + o_mb);
   p->acc = reinterpret_cast<float*>(base + o_acc);
+  p->ctl = reinterpret_cast<ppo::StepCtl*>(base + o_ctl);
   p->blas_ws = base + o_ws;
   for (int k = 0; k < 2; ++k) {
     p->h1[k] = base + o_h1[k];
@@ -440,6 +492,10 @@ int ppo_destroy(auv_ppo* p) {
   cudaGetDevice(&prev);
   cudaSetDevice(p->device);
   cudaDeviceSynchronize();
+  drop_graph(p);
+  if (p->ev_in) cudaEventDestroy(p->ev_in);
+  if (p->ev_out) cudaEventDestroy(p->ev_out);
+  if (p->gstream) cudaStreamDestroy(p->gstream);
   cublasDestroy(p->blas);
   cudaFree(p->mem);
   if (prev >= 0) cudaSetDevice(prev);
@@ -526,7 +582,8 @@ int ppo_grads(auv_ppo* p, const auv_ppo_batch* batch, uint64_t epoch, uint32_t m
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cublasStatus_t bs = cublasSetStream(p->blas, s);
   if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
-  if ((rc = grads_impl(p, batch, epoch, minibatch, nullptr, s))) return rc;
+  if ((rc = set_ctl(p, epoch, 1u << 31, minibatch, p->t, s))) return rc;
+  if ((rc = grads_impl(p, batch, nullptr, s))) return rc;
   if (grad && (rc = convert(p, grad, grad + p->n_flat[0], p->g, false, s))) return rc;
   if (stats) {
     cudaError_t e = cudaMemcpyAsync(stats, p->mb, AUV_PPO_STATS * 4, cudaMemcpyDeviceToDevice, s);
@@ -548,7 +605,9 @@ int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream) {
     if (e != cudaSuccess) return cuda_fail(p, e, "copy gradient");
     if ((rc = convert(p, p->flat, p->flat + p->n_flat[0], p->g, true, s))) return rc;
   }
+  if ((rc = set_ctl(p, p->epoch, 1u << 31, 0, p->t, s))) return rc;
   if ((rc = apply_impl(p, nullptr, s))) return rc;
+  p->t += 1;
   if (stats) {
     cudaError_t e = cudaMemcpyAsync(stats + 5, p->mb + 5, 4, cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) return cuda_fail(p, e, "copy gradient norm");
@@ -567,19 +626,39 @@ int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t
                 p->d.B, (unsigned long long)batch->T * batch->N);
   if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cublasStatus_t bs = cublasSetStream(p->blas, s);
-  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
-  cudaError_t e = cudaMemsetAsync(p->acc, 0, AUV_PPO_STATS * 4, s);
-  if (e != cudaSuccess) return cuda_fail(p, e, "clear statistics");
-  for (uint32_t ep = 0; ep < epochs; ++ep) {
-    for (uint32_t j = 0; j < n_minibatches; ++j) {
-      if ((rc = grads_impl(p, batch, p->epoch, j, p->acc, s))) return rc;
-      if ((rc = apply_impl(p, p->acc, s))) return rc;
-    }
-    ++p->epoch;
+  const uint64_t steps = (uint64_t)epochs * n_minibatches;
+  // replay the captured step on the private stream when it can be had
+  if (!p->graph_failed && (!p->step_graph || !same_batch(p->graph_batch, *batch)) &&
+      !capture_step(p, batch))
+    p->graph_failed = true;
+  const bool graph = p->step_graph != nullptr && !p->graph_failed;
+  cudaStream_t r = s;
+  cudaError_t e;
+  if (graph) {
+    if ((e = cudaEventRecord(p->ev_in, s)) || (e = cudaStreamWaitEvent(p->gstream, p->ev_in, 0)))
+      return cuda_fail(p, e, "order update after caller");
+    r = p->gstream;
+  } else {
+    cublasStatus_t bs = cublasSetStream(p->blas, s);
+    if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
   }
-  if (stats && (e = ppo::launch_finish(p->acc, stats, s)) != cudaSuccess)
+  if ((rc = set_ctl(p, p->epoch, n_minibatches, 0, p->t, r))) return rc;
+  if ((e = cudaMemsetAsync(p->acc, 0, AUV_PPO_STATS * 4, r)))
+    return cuda_fail(p, e, "clear statistics");
+  for (uint64_t k = 0; k < steps; ++k) {
+    if (graph) {
+      if ((e = cudaGraphLaunch(p->step_graph, r))) return cuda_fail(p, e, "launch step graph");
+    } else {
+      if ((rc = grads_impl(p, batch, p->acc, r)) || (rc = apply_impl(p, p->acc, r))) return rc;
+      if ((e = ppo::launch_step_advance(p->ctl, r))) return cuda_fail(p, e, "advance step");
+    }
+  }
+  if (stats && (e = ppo::launch_finish(p->acc, stats, r)) != cudaSuccess)
     return cuda_fail(p, e, "statistics");
+  if (graph && ((e = cudaEventRecord(p->ev_out, r)) || (e = cudaStreamWaitEvent(s, p->ev_out, 0))))
+    return cuda_fail(p, e, "order caller after update");
+  p->t += steps;
+  p->epoch += epochs;
   return AUV_OK;
 }
 

@@ -304,3 +304,32 @@ def test_learner_rejects_bad_arguments():
     assert ei.value.code == auvenv.AUV_ERR_SIZE
     with pytest.raises(ValueError):
         L.set_weights(np.zeros(3), np.zeros(3))
+
+
+def test_update_graph_equals_step_by_step_calls():
+    """ppo_update replays one captured step per minibatch; the same steps
+    through ppo_grads + ppo_apply (direct launches) give the same weights
+    and moments, and a second batch (new arrays) is captured afresh."""
+    torch = need_gpu()
+    D, A, H, T, N, B = 18, 8, 64, 4, 600, 700
+    pw, vw = _weights(D, H, A, seed=21)
+    traj = _dev(torch, _on_rollout_policy(_traj(22, T, N, D, A), pw, D, H, A))
+    a, b = _learner(D, A, H, B, "fp32"), _learner(D, A, H, B, "fp32")
+    a.set_weights(pw, vw)
+    b.set_weights(pw, vw)
+    a.update(traj, 2, 3)
+    for e in range(2):
+        for j in range(3):
+            b.grads(traj, e, j)
+            b.apply()
+    for x, y in zip(a.get_weights(), b.get_weights()):
+        assert np.abs(x - y).max() <= 1e-6 * max(1.0, np.abs(y).max())
+    sa, sb = a.get_state(), b.get_state()
+    assert (sa["t"], sa["epoch"]) == (6, 2) and sb["t"] == 6
+    traj2 = {k: v.clone() for k, v in traj.items()}
+    a.update(traj2, 1, 3)
+    for j in range(3):
+        b.grads(traj2, 2, j)
+        b.apply()
+    for x, y in zip(a.get_weights(), b.get_weights()):
+        assert np.abs(x - y).max() <= 1e-6 * max(1.0, np.abs(y).max())
