@@ -397,6 +397,10 @@ int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const fl
 #define AUV_PPO_FP32 0u   /* GEMMs on the CUDA cores in fp32                     */
 #define AUV_PPO_TF32 1u   /* GEMMs on the tensor cores, tf32 operands, fp32 sums */
 #define AUV_PPO_BF16 2u   /* GEMMs on the tensor cores, bf16 operands, fp32 sums */
+#define AUV_PPO_VALUE_ONLY 1u /* flags: train the value network alone on
+ * L = vf_coef mean (V - ret)^2 / 2 (the critic regression of SHAC, whose
+ * TD(lambda) targets are env_gae's returns); the policy is neither run nor
+ * changed, and batch.act, .logp, .adv may be NULL. */
 #define AUV_PPO_STATS 8   /* floats in a statistics record:                       */
 /* [0] surrogate (policy) loss, [1] value loss (mean (V - ret)^2 / 2),
  * [2] entropy, [3] approx. KL mean(logp_old - logp), [4] clip fraction
@@ -412,7 +416,7 @@ typedef struct auv_ppo_config {
   uint32_t minibatch;     /* B samples per gradient step, 2 .. 2^22            */
   uint32_t precision;     /* AUV_PPO_FP32 | AUV_PPO_TF32 | AUV_PPO_BF16        */
   uint32_t norm_adv;      /* 1: normalise advantages per minibatch, 0: not     */
-  uint32_t reserved;      /* 0                                                 */
+  uint32_t flags;         /* AUV_PPO_VALUE_ONLY or 0                           */
   uint64_t seed;          /* key of the minibatch permutations                 */
   float clip_eps;         /* > 0                                               */
   float vf_coef, ent_coef;            /* finite                                */
@@ -533,16 +537,19 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
  * back-propagation through the dynamics, the policy network and the
  * observation.  Gradients stop at the window's start and at episode ends
  * inside it (the state after an end is a reset draw).  Optional outputs:
- * J_out [N] each env's J; rew_out, done_out [T][N]; device or mapped
- * page-locked host memory.  policy, value, coef [T], grad: device memory.
+ * J_out [N] each env's J; obs_out [T][18][N] the observation of each step
+ * (the rollout's layout: with rew_out, done_out [T][N], env_value and
+ * env_gae it gives the critic's TD(lambda) targets); device or mapped
+ * page-locked host memory for J_out, rew_out, done_out, device memory for
+ * obs_out.  policy, value, coef [T], grad: device memory.
  * Fossen model, 1 <= T <= AUV_ADJOINT_MAX_T, at most
  * AUV_ADJOINT_MAX_SUBSTEPS substeps, hidden a multiple of 8 up to 1024.
  * The first call at a given (N, T) allocates the window's workspace
  * (activations of every step: about T N (2 hidden + 80) floats).
  */
 int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
-                    const float* coef, float coef_V, float* grad, float* J_out, float* rew_out,
-                    uint8_t* done_out, void* stream);
+                    const float* coef, float coef_V, float* grad, float* J_out, float* obs_out,
+                    float* rew_out, uint8_t* done_out, void* stream);
 
 /*
  * env_inverse_allocate: thruster commands for body-frame wrenches, the map

@@ -19,7 +19,9 @@ reset state's value, its rewards) flows back across it.
 The minibatch update of PPO (clipped surrogate, value and entropy terms,
 chain-rule gradients of the two tanh MLPs, global-norm clipping, Adam) and
 the learner that runs epochs of minibatches drawn by the Feistel permutation
-of the C++ oracle (oracle_minibatch_perm).  The paper names PPO but prints
+of the C++ oracle (oracle_minibatch_perm).  With hp["value_only"] the loss is
+the value term alone (the critic regression of SHAC, whose targets are the
+TD(lambda) returns = the GAE returns above) and the policy is not trained.  The paper names PPO but prints
 none of its constants or loss weights: every hyperparameter is an input.
 """
 from __future__ import annotations
@@ -120,10 +122,15 @@ def ppo_loss(pw, vw, dims, x, a, logp_old, adv, ret, hp):
     pg = np.mean(np.maximum(-an * r, -an * np.clip(r, 1 - eps, 1 + eps)))
     vl = 0.5 * np.mean((v[:, 0] - ret) ** 2)
     ent = np.mean(np.sum(ls + 0.5 * (1.0 + LOG_2PI), axis=1))
+    kl = float(np.mean(logp_old - logp))
+    cf = float(np.mean(np.abs(r - 1.0) > eps))
+    if hp.get("value_only"):
+        # critic regression (SHAC's value step): only the value term
+        pg, ent, kl, cf = 0.0, 0.0, 0.0, 0.0
+        return hp["vf_coef"] * vl, dict(pg_loss=pg, v_loss=vl, entropy=ent, approx_kl=kl,
+                                        clip_frac=cf)
     loss = pg + hp["vf_coef"] * vl - hp["ent_coef"] * ent
-    return loss, dict(pg_loss=pg, v_loss=vl, entropy=ent,
-                      approx_kl=float(np.mean(logp_old - logp)),
-                      clip_frac=float(np.mean(np.abs(r - 1.0) > eps)))
+    return loss, dict(pg_loss=pg, v_loss=vl, entropy=ent, approx_kl=kl, clip_frac=cf)
 
 
 def ppo_grads(pw, vw, dims, x, a, logp_old, adv, ret, hp):
@@ -144,6 +151,8 @@ def ppo_grads(pw, vw, dims, x, a, logp_old, adv, ret, hp):
     g_y[:, :A] = g_logp[:, None] * d / sig2
     g_y[:, A:] = (g_logp[:, None] * (d * d / sig2 - 1.0) - hp["ent_coef"] / B) * inside
     g_v = hp["vf_coef"] * (v - ret[:, None]) / B
+    if hp.get("value_only"):
+        g_y = np.zeros_like(g_y)
     gp = mlp_backward(pw, in_dim, H, 2 * A, x, h1, h2, g_y)
     gv = mlp_backward(vw, in_dim, H, 1, x, vh1, vh2, g_v)
     _, parts = ppo_loss(pw, vw, dims, x, a, logp_old, adv, ret, hp)

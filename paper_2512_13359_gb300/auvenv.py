@@ -31,6 +31,7 @@ AUV_PPO_FP32 = 0
 AUV_PPO_TF32 = 1
 AUV_PPO_BF16 = 2
 AUV_PPO_STATS = 8
+AUV_PPO_VALUE_ONLY = 1
 PPO_PRECISION = {"fp32": AUV_PPO_FP32, "tf32": AUV_PPO_TF32, "bf16": AUV_PPO_BF16}
 PPO_STAT_NAMES = ("pg_loss", "v_loss", "entropy", "approx_kl", "clip_frac", "grad_norm", "loss",
                   "steps")
@@ -100,7 +101,7 @@ class PpoConfig(C.Structure):
     _fields_ = [
         ("struct_size", C.c_uint32), ("obs_dim", C.c_uint32), ("act_dim", C.c_uint32),
         ("hidden", C.c_uint32), ("minibatch", C.c_uint32), ("precision", C.c_uint32),
-        ("norm_adv", C.c_uint32), ("reserved", C.c_uint32), ("seed", C.c_uint64),
+        ("norm_adv", C.c_uint32), ("flags", C.c_uint32), ("seed", C.c_uint64),
         ("clip_eps", C.c_float), ("vf_coef", C.c_float), ("ent_coef", C.c_float),
         ("max_grad_norm", C.c_float), ("lr", C.c_float), ("adam_beta1", C.c_float),
         ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("logstd_min", C.c_float),
@@ -157,7 +158,7 @@ def lib(path: str | None = None):
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
     L.env_inverse_allocate.argtypes = [P, I, P, P, P]
-    L.env_shac_window.argtypes = [P, P, P, I, P, C.c_float, P, P, P, P, P]
+    L.env_shac_window.argtypes = [P, P, P, I, P, C.c_float, P, P, P, P, P, P]
     L.rbuf_create.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(P)]
     L.rbuf_destroy.argtypes = [P]
     L.rbuf_last_error.argtypes = [P]
@@ -337,12 +338,12 @@ class Env:
                                       _stream(stream)))
 
     def shac_window(self, policy, value, coef, coef_V, grad, J=None, rew=None, done=None,
-                    stream=None):
+                    obs=None, stream=None):
         """SHAC actor gradient over a window of len(coef) steps in closed loop
         (env_shac_window); the env advances."""
         self._check(lib().env_shac_window(self.h, _ptr(policy), _ptr(value), coef.shape[0],
                                           _ptr(coef), float(coef_V), _ptr(grad), _ptr(J),
-                                          _ptr(rew), _ptr(done), _stream(stream)))
+                                          _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))
 
     def inverse_allocate(self, wrench, cmd, stream=None):
         """Thruster commands cmd [8][n] for wrenches [6][n] (env_inverse_allocate)."""
@@ -421,6 +422,7 @@ def make_ppo_config(obs_dim: int, act_dim: int, hidden: int, minibatch: int,
     c.obs_dim, c.act_dim, c.hidden, c.minibatch = obs_dim, act_dim, hidden, minibatch
     c.precision = PPO_PRECISION[precision] if isinstance(precision, str) else int(precision)
     c.norm_adv = 1 if h.pop("norm_adv") else 0
+    c.flags = AUV_PPO_VALUE_ONLY if h.pop("value_only", False) else 0
     c.seed = seed
     for k, v in h.items():
         setattr(c, k, float(v))
@@ -465,12 +467,13 @@ class Learner:
 
     @staticmethod
     def _batch(traj):
-        T, N = traj["logp"].shape
+        """obs, ret required; act, logp, adv may be absent (value-only learner)."""
+        T, N = traj["ret"].shape
         for k in ("obs", "act", "logp", "adv", "ret"):
-            if not traj[k].is_contiguous():
+            if traj.get(k) is not None and not traj[k].is_contiguous():
                 raise ValueError(f"{k} must be contiguous")
-        return PpoBatch(traj["obs"].data_ptr(), traj["act"].data_ptr(), traj["logp"].data_ptr(),
-                        traj["adv"].data_ptr(), traj["ret"].data_ptr(), T, N)
+        ptr = lambda k: traj[k].data_ptr() if traj.get(k) is not None else None
+        return PpoBatch(ptr("obs"), ptr("act"), ptr("logp"), ptr("adv"), ptr("ret"), T, N)
 
     def set_weights(self, policy, value, stream=None):
         p = np.ascontiguousarray(policy, dtype=np.float32)

@@ -718,8 +718,8 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
 }
 
 int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
-                    const float* coef, float coef_V, float* grad, float* J_out, float* rew_out,
-                    uint8_t* done_out, void* stream) {
+                    const float* coef, float coef_V, float* grad, float* J_out, float* obs_out,
+                    float* rew_out, uint8_t* done_out, void* stream) {
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);
   if (rc) return rc;
@@ -739,6 +739,7 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
       (rc = check_device_buffer(env, grad, "grad", 4)))
     return rc;
   if (value && (rc = check_device_buffer(env, value, "value", 4))) return rc;
+  if (obs_out && (rc = check_device_buffer(env, obs_out, "obs_out", 4))) return rc;
   void *J = nullptr, *rew = nullptr, *done = nullptr;
   if ((rc = map_output(env, J_out, "J_out", 4, &J)) ||
       (rc = map_output(env, rew_out, "rew_out", 4, &rew)) ||
@@ -774,7 +775,8 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
   }
   rc = auv::shac::run_window(env->blas, env->model, env->buf, env->status, L, env->shac_ws,
                              env->t_g, policy, value, coef, coef_V, grad, static_cast<float*>(J),
-                             static_cast<float*>(rew), static_cast<uint8_t*>(done), s, env->err);
+                             obs_out, static_cast<float*>(rew), static_cast<uint8_t*>(done), s,
+                             env->err);
   if (rc != AUV_OK) return rc;
   env->t_g += (uint64_t)T;
   return AUV_OK;

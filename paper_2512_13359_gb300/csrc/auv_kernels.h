@@ -77,10 +77,11 @@ cudaError_t init(const Layout& L, char* base, cudaStream_t s);
 // blas: a cublasHandle_t.  Returns AUV_OK or an AUV_ERR_* code with err set.
 int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
-               const float* coef, float coef_V, float* grad, float* J, float* rew_out,
-               uint8_t* done_out, cudaStream_t s, char* err);
+               const float* coef, float coef_V, float* grad, float* J, float* obs_out,
+               float* rew_out, uint8_t* done_out, cudaStream_t s, char* err);
+// obs_fm: optional [T][18][N] output of step t's observation.
 cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
-                       cudaStream_t s);
+                       float* obs_fm, int t, cudaStream_t s);
 cudaError_t launch_step(const Model& M, const Buffers& B, const float* Y, int ldy, uint64_t t_g,
                         float* rew, uint8_t* done, Status* st, cudaStream_t s);
 cudaError_t launch_bwd(const Model& M, const float* sc, const float* Y, int ldy,
@@ -121,6 +122,7 @@ struct Dims {
   int ld_pol;    // row length of the policy head arrays Y, dL/dY (>= 2A)
   int ld_val;    // row length of the value head arrays (>= 1)
   int bf16;      // activations and head gradients stored as bf16
+  int value_only;  // critic regression: the policy is not run
 };
 
 struct PermKey {        // Feistel permutation of [0, m) for one epoch

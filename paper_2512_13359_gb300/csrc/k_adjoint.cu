@@ -497,7 +497,8 @@ __device__ __forceinline__ void shac_action(const Model& M, const float* __restr
 // up to ldx) of each env's current state; with sc, also the step's scratch.
 __global__ void __launch_bounds__(kAdjThreads) k_shac_obs(const Model M, Buffers B,
                                                           float* __restrict__ sc,
-                                                          float* __restrict__ X, int ldx) {
+                                                          float* __restrict__ X, int ldx,
+                                                          float* __restrict__ obs_fm, int t) {
   const int i = blockIdx.x * kAdjThreads + threadIdx.x;
   if (i >= M.n) return;
   Env e;
@@ -510,6 +511,10 @@ __global__ void __launch_bounds__(kAdjThreads) k_shac_obs(const Model M, Buffers
   for (int k = 0; k < kObs; ++k) x[k] = o[k];
   x[kObs] = 1.0f;
   for (int k = kObs + 1; k < ldx; ++k) x[k] = 0.0f;
+  if (obs_fm) {
+#pragma unroll
+    for (int k = 0; k < kObs; ++k) obs_fm[((size_t)t * kObs + k) * M.n + i] = o[k];
+  }
 }
 
 // One closed-loop step from the policy head Y [N][ldy]: action, physics,
@@ -648,8 +653,8 @@ namespace shac {
 static unsigned blocks(int n) { return (n + kAdjThreads - 1) / kAdjThreads; }
 
 cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
-                       cudaStream_t s) {
-  k_shac_obs<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx);
+                       float* obs_fm, int t, cudaStream_t s) {
+  k_shac_obs<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx, obs_fm, t);
   return cudaGetLastError();
 }
 

@@ -167,20 +167,22 @@ __global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, const StepCt
     }
     st_act(x + d.D, 1.0f);
     for (int k = d.D + 1; k < d.Dp; ++k) st_act(x + k, 0.0f);
-    float av[8];
-#pragma unroll
-    for (int k = 0; k < 8; ++k)
-      if (k < d.A) av[k] = __ldg(act + (t * d.A + k) * n + i);
-#pragma unroll
-    for (int k = 0; k < 8; ++k)
-      if (k < d.A) out.act[(size_t)b * d.A + k] = av[k];
     const size_t o = t * n + i;
-    const float a = __ldg(adv + o);
-    out.logp[b] = __ldg(logp + o);
-    out.adv[b] = a;
     out.ret[b] = __ldg(ret + o);
-    s[0] = a;
-    s[1] = (double)a * a;
+    if (!d.value_only) {
+      float av[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (k < d.A) av[k] = __ldg(act + (t * d.A + k) * n + i);
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (k < d.A) out.act[(size_t)b * d.A + k] = av[k];
+      const float a = __ldg(adv + o);
+      out.logp[b] = __ldg(logp + o);
+      out.adv[b] = a;
+      s[0] = a;
+      s[1] = (double)a * a;
+    }
   }
   block_sum<2>(s, sh);
   if (threadIdx.x == 0) {
@@ -280,7 +282,11 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
   __syncthreads();
   const int b = blockIdx.x * kT + threadIdx.x;
   float st[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
-  if (b < d.B) {
+  if (b < d.B && d.value_only) {
+    const float dv = v[(size_t)b * d.ld_val] - smp.ret[b];
+    st_act(g_v + (size_t)b * d.ld_val, hp.vf_coef * dv * (1.0f / (float)d.B));
+    st[1] = 0.5f * dv * dv;
+  } else if (b < d.B) {
     const float inv_b = 1.0f / (float)d.B;
     const int A = d.A;
     const float* yb = y + (size_t)b * d.ld_pol;
@@ -331,6 +337,7 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
 __global__ void __launch_bounds__(kT) k_stats(int B, int n_part, float vf_coef, float ent_coef,
                                               const float* __restrict__ part, float* mb,
                                               float* acc) {
+  // (value-only steps leave the policy terms of part at 0)
   __shared__ double sh[5 * (kT / 32)];
   double s[5] = {0, 0, 0, 0, 0};
   for (int k = threadIdx.x; k < n_part; k += kT)

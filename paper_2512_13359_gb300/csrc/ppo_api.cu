@@ -126,7 +126,7 @@ int validate(const auv_ppo_config* c) {
     return fail(nullptr, AUV_ERR_INVALID, "minibatch outside [2, 2^22]");
   if (c->precision > AUV_PPO_BF16) return fail(nullptr, AUV_ERR_INVALID, "unknown precision %u", c->precision);
   if (c->norm_adv > 1) return fail(nullptr, AUV_ERR_INVALID, "norm_adv must be 0 or 1");
-  if (c->reserved) return fail(nullptr, AUV_ERR_INVALID, "reserved must be 0");
+  if (c->flags & ~AUV_PPO_VALUE_ONLY) return fail(nullptr, AUV_ERR_INVALID, "unknown flags %#x", c->flags);
   if (!(std::isfinite(c->clip_eps) && c->clip_eps > 0.0f))
     return fail(nullptr, AUV_ERR_INVALID, "clip_eps must be finite and > 0");
   if (!std::isfinite(c->vf_coef) || !std::isfinite(c->ent_coef) || std::isnan(c->max_grad_norm) ||
@@ -147,9 +147,11 @@ int check_batch(auv_ppo* p, const auv_ppo_batch* b) {
   if (b->T < 1 || b->N < 1) return fail(p, AUV_ERR_INVALID, "batch T and N must be >= 1");
   if ((uint64_t)b->T * b->N > (1ull << 31)) return fail(p, AUV_ERR_SIZE, "T * N exceeds 2^31");
   int rc;
-  if ((rc = check_dev(p, b->obs, "batch.obs")) || (rc = check_dev(p, b->act, "batch.act")) ||
-      (rc = check_dev(p, b->logp, "batch.logp")) || (rc = check_dev(p, b->adv, "batch.adv")) ||
-      (rc = check_dev(p, b->ret, "batch.ret")))
+  if ((rc = check_dev(p, b->obs, "batch.obs")) || (rc = check_dev(p, b->ret, "batch.ret")))
+    return rc;
+  if (p->d.value_only) return AUV_OK;     // act, logp, adv are not read
+  if ((rc = check_dev(p, b->act, "batch.act")) || (rc = check_dev(p, b->logp, "batch.logp")) ||
+      (rc = check_dev(p, b->adv, "batch.adv")))
     return rc;
   return AUV_OK;
 }
@@ -268,12 +270,13 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
                                      b->adv, b->ret, b->N, p->smp, p->X, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "gather");
   int rc;
-  if ((rc = forward(p, 0, s)) || (rc = forward(p, 1, s))) return rc;
+  if ((!d.value_only && (rc = forward(p, 0, s))) || (rc = forward(p, 1, s))) return rc;
   const ppo::LossHp hp = loss_hp(p);
   if ((e = ppo::launch_head(d, hp, p->y[0], p->y[1], p->smp, p->g_y, p->g_v, p->head_part, s)))
     return cuda_fail(p, e, "loss head");
   if ((e = ppo::launch_stats(d, hp, p->head_part, p->mb, acc, s))) return cuda_fail(p, e, "statistics");
-  if ((rc = backward(p, 0, p->g_y, s)) || (rc = backward(p, 1, p->g_v, s))) return rc;
+  if ((!d.value_only && (rc = backward(p, 0, p->g_y, s))) || (rc = backward(p, 1, p->g_v, s)))
+    return rc;
   return AUV_OK;
 }
 
@@ -392,6 +395,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   d.ld_pol = round8(2 * d.A);
   d.ld_val = 8;
   d.bf16 = cfg->precision == AUV_PPO_BF16;
+  d.value_only = (cfg->flags & AUV_PPO_VALUE_ONLY) ? 1 : 0;
   p->bf16 = d.bf16 != 0;
   p->act_t = p->bf16 ? CUDA_R_16BF : CUDA_R_32F;
   p->esz = p->bf16 ? 2 : 4;

@@ -100,8 +100,8 @@ cudaError_t init(const Layout& L, char* base, cudaStream_t s) {
 
 int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
-               const float* coef, float coef_V, float* grad, float* J, float* rew_out,
-               uint8_t* done_out, cudaStream_t s, char* err) {
+               const float* coef, float coef_V, float* grad, float* J, float* obs_out,
+               float* rew_out, uint8_t* done_out, cudaStream_t s, char* err) {
   const int n = L.n, T = L.T, H = L.H, Dp = L.Dp, Hp = L.Hp;
   const size_t N = (size_t)n;
   auto F = [&](size_t o) { return reinterpret_cast<float*>(base + o); };
@@ -144,7 +144,7 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
 
   // ---- forward ----
   for (int t = 0; t < T; ++t) {
-    if ((e = launch_obs(M, B, SCs(t), Xs(t), Dp, s))) return cfail(e, "observation");
+    if ((e = launch_obs(M, B, SCs(t), Xs(t), Dp, obs_out, t, s))) return cfail(e, "observation");
     if ((bs = gemm(T_, N_, H, n, Dp, w1, Dp, Xs(t), Dp, H1s(t), Hp))) return bfail(bs, "policy 1");
     if ((e = ppo::launch_tanh_fwd(false, H1s(t), Hp, n, H, s))) return cfail(e, "tanh");
     if ((bs = gemm(T_, N_, H, n, Hp, w2, Hp, H1s(t), Hp, H2s(t), Hp))) return bfail(bs, "policy 2");
@@ -158,7 +158,7 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   if ((e = cudaMemsetAsync(lam, 0, 13 * N * 4, s))) return cfail(e, "clear adjoint");
   // ---- terminal critic: lam = coef_V dV(o(x_T))/dx_T ----
   if (value) {
-    if ((e = launch_obs(M, B, nullptr, Xs(T), Dp, s))) return cfail(e, "observation");
+    if ((e = launch_obs(M, B, nullptr, Xs(T), Dp, nullptr, 0, s))) return cfail(e, "observation");
     if ((bs = gemm(T_, N_, H, n, Dp, v1, Dp, Xs(T), Dp, VH1, Hp))) return bfail(bs, "value 1");
     if ((e = ppo::launch_tanh_fwd(false, VH1, Hp, n, H, s))) return cfail(e, "tanh");
     if ((bs = gemm(T_, N_, H, n, Hp, v2, Hp, VH1, Hp, VH2, Hp))) return bfail(bs, "value 2");

@@ -333,3 +333,32 @@ def test_update_graph_equals_step_by_step_calls():
         b.apply()
     for x, y in zip(a.get_weights(), b.get_weights()):
         assert np.abs(x - y).max() <= 1e-6 * max(1.0, np.abs(y).max())
+
+
+def test_value_only_learner_matches_oracle():
+    """AUV_PPO_VALUE_ONLY: the critic regression (value term alone) with
+    act, logp and adv absent; the policy gradient is zero and an update
+    leaves the policy bit for bit."""
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    D, A, H, T, N, B = 18, 8, 64, 5, 400, 900
+    pw, vw = _weights(D, H, A, seed=31)
+    traj = _traj(32, T, N, D, A)
+    L = _learner(D, A, H, B, "fp32", value_only=True)
+    L.set_weights(pw, vw)
+    dev = {k: torch.from_numpy(traj[k]).cuda() for k in ("obs", "ret")}
+    grad = torch.empty(L.n_policy + L.n_value, device="cuda")
+    stats = torch.empty(8, device="cuda")
+    L.grads(dev, 1, 1, grad=grad, stats=stats)
+    hp = dict(HP, value_only=True)
+    parts, g_ref = P.Learner(pw, vw, (D, H, A), hp, seed=7).grads(traj, 1, 1, B)
+    g = to_np(grad)
+    assert np.all(g[:L.n_policy] == 0.0) and np.all(g_ref[:L.n_policy] == 0.0)
+    scale = np.abs(g_ref[L.n_policy:]).max()
+    assert np.abs(g[L.n_policy:] - g_ref[L.n_policy:]).max() <= 1e-4 * scale
+    st = to_np(stats)
+    assert st[0] == 0.0 and st[2] == 0.0
+    assert abs(st[1] - parts["v_loss"]) <= 1e-4 * parts["v_loss"]
+    L.update(dev, 2, 2)
+    gp, gv = L.get_weights()
+    assert np.array_equal(gp, pw) and not np.array_equal(gv, vw)

@@ -152,3 +152,63 @@ def test_shac_window_rejects_bad_arguments():
     with pytest.raises(auvenv.AuvError) as ei:
         pe.shac_window(pw, None, coef[:4], 0.0, g)
     assert ei.value.code == auvenv.AUV_ERR_UNSUPPORTED
+
+
+def test_shac_critic_targets_and_regression(oracle):
+    """SHAC's critic step from the window's outputs: the observations the
+    window returns (the rollout's layout) equal the oracle's closed-loop
+    rollout's, the TD(lambda) targets are env_gae's returns over the
+    window's rewards, dones and critic values (bootstrap at the final
+    observation), and the value-only learner's gradient on (obs, targets)
+    matches the oracle's critic regression."""
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    from paper_2512_13359_gb300 import auvenv
+    n, T, H = 256, 8, 64
+    w = W.workload("ppo_65536", n_envs=n, hidden=H, mlp="fp32", has_value=1, episode_len=6)
+    env = make_env(w)                       # the env's own value network is the critic
+    env.reset()
+    b = oracle.Batch(np.arange(n))
+    b.state[:] = to_np(env.state)
+    b.params[:] = to_np(env.params)
+    b.t_ep[:] = to_np(env.t_ep)
+    b.episode[:] = to_np(env.episode).view(np.uint32)
+    t_g0 = env.t_g
+    pw = W.policy_weights(w, 0.05)
+    vw = W.value_weights(w)
+    obs = torch.empty((T, 18, n), device="cuda")
+    rew = torch.empty((T, n), device="cuda")
+    done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
+    grad = torch.empty(pw.size, device="cuda")
+    coef = torch.full((T,), 1.0 / (n * T), device="cuda")
+    env.shac_window(torch.from_numpy(pw).cuda(), torch.from_numpy(vw).cuda(), coef, 0.5 / n, grad,
+                    obs=obs, rew=rew, done=done)
+    m = oracle.model(w)
+    ref = oracle.rollout(m, b, pw, None, t_g0, T, want=("obs", "rew"))
+    assert np.abs(to_np(obs) - ref["obs"]).max() <= 1e-4
+    assert np.array_equal(to_np(done), ref["done"])
+    # critic values of every step and of the final observation, TD(lambda) targets
+    val = torch.empty((T, n), device="cuda")
+    env.value(obs, val)
+    last_obs = torch.empty((1, 18, n), device="cuda")
+    env.observe(last_obs[0])
+    last = torch.empty((1, n), device="cuda")
+    env.value(last_obs, last)
+    adv = torch.empty((T, n), device="cuda")
+    ret = torch.empty((T, n), device="cuda")
+    env.gae(rew, done, val, last[0], 0.99, 0.95, adv, ret)
+    r_adv, r_ret = P.gae(to_np(rew), to_np(done), to_np(val), to_np(last[0]), 0.99, 0.95)
+    assert np.abs(to_np(ret) - r_ret).max() <= 2e-5 * max(1.0, np.abs(r_ret).max())
+    # critic regression on (obs, targets)
+    L = auvenv.Learner(18, 8, H, 512, precision="fp32", seed=4, value_only=True, vf_coef=1.0)
+    L.set_weights(pw, vw)
+    g = torch.empty(L.n_policy + L.n_value, device="cuda")
+    L.grads(dict(obs=obs, ret=ret), 0, 1, grad=g)
+    host = dict(obs=to_np(obs), ret=to_np(ret), act=np.zeros((T, 8, n), np.float32),
+                logp=np.zeros((T, n), np.float32), adv=np.zeros((T, n), np.float32))
+    hp = dict(clip_eps=0.2, vf_coef=1.0, ent_coef=0.0, max_grad_norm=0.5, lr=3e-4,
+              adam_beta1=0.9, adam_beta2=0.999, adam_eps=1e-8, logstd_min=-5.0,
+              logstd_max=2.0, norm_adv=True, value_only=True)
+    _, g_ref = P.Learner(pw, vw, (18, H, 8), hp, seed=4).grads(host, 0, 1, 512)
+    gv, rv = to_np(g)[L.n_policy:], g_ref[L.n_policy:]
+    assert np.abs(gv - rv).max() <= 1e-4 * np.abs(rv).max()

@@ -307,3 +307,17 @@ def test_learner_update_counts_and_moves():
     L0 = P.Learner(pw, vw, (in_dim, H, A), dict(HP, lr=0.0), seed=3)
     L0.update(traj, 1, 2, 64)
     assert np.array_equal(L0.policy, pw) and np.array_equal(L0.value, vw)
+
+
+def test_value_only_is_the_critic_regression():
+    """value_only: the loss is c_v mean((V - R)^2) / 2, the policy gradient
+    is zero, and the value gradient equals the full loss's (whose value part
+    does not depend on the policy)."""
+    pw, vw, dims, x, a, lp_old, adv, ret = _problem(17)
+    hp = dict(HP, value_only=True)
+    loss, parts = P.ppo_loss(pw, vw, dims, x, a, lp_old, adv, ret, hp)
+    assert loss == pytest.approx(HP["vf_coef"] * parts["v_loss"], rel=1e-15)
+    assert parts["pg_loss"] == 0.0 and parts["entropy"] == 0.0
+    _, gp, gv = P.ppo_grads(pw, vw, dims, x, a, lp_old, adv, ret, hp)
+    _, _, gv_full = P.ppo_grads(pw, vw, dims, x, a, lp_old, adv, ret, HP)
+    assert np.all(gp == 0.0) and np.array_equal(gv, gv_full)
