@@ -635,25 +635,30 @@ def run_shac(args):
     coef = torch.tensor([0.99 ** t / (n * T) for t in range(T)], dtype=torch.float32,
                         device="cuda")
     grad = torch.empty_like(pw)
-    ms = _timed(args, lambda: env.shac_window(pw, vw, coef, 0.99 ** T / n, grad))
+    prec = "tf32" if args.ppo_precision in ("tf32", "bf16") else "fp32"
+    ms = _timed(args, lambda: env.shac_window(pw, vw, coef, 0.99 ** T / n, grad, precision=prec))
     assert env.status().code == 0
     rate = n * T / (ms * 1e-3)
     fps = 3 * mlp_flops(W.obs_dim(w), H, 16) + ADJOINT_FLOPS_PER_ENV_STEP.get(int(w["substeps"]), 0)
     peaks, src = load_peaks()
     mhz = peaks.get("sm_max_mhz", 2070.0)
-    peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+    if prec == "tf32":
+        peak = peaks["bf16_tflops_sustained"] * 1.1 / 2.25
+        bound, psrc = "tensor", f"bf16 sustained, {src}, x tf32/bf16 nominal 1.1/2.25"
+    else:
+        peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+        bound, psrc = "alu", f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz"
     achieved = rate * fps / 1e12
     line = {
         "metric": "SHAC window env-steps/s", "value": rate, "unit": "env-steps/s", "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "scaling": "weak", "vs_baseline": None, "dtype": "tf32" if prec == "tf32" else "f32",
         "data": "synthetic (workload resets, seeded random policy and critic)",
-        "config": {"workload": w["name"], "n_envs": n, "window": T, "hidden": H,
+        "config": {"workload": w["name"], "n_envs": n, "window": T, "hidden": H, "precision": prec,
                    "l2": "working set per window (activations of every step) larger than L2"},
-        "roofline": {"bound": "alu", "kernel": "whole window (cuBLAS fp32 GEMMs + own kernels)",
+        "roofline": {"bound": bound, "kernel": "whole window (cuBLAS GEMMs + own kernels)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "traffic": None,
-                     "peak_source": f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz",
+                     "frac": achieved / peak, "traffic": None, "peak_source": psrc,
                      "flops_per_env_step": fps},
         "gpu_launches": args.steps * (17 * T + 16), "clocks": None,
     }

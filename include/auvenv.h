@@ -542,14 +542,18 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
  * env_gae it gives the critic's TD(lambda) targets); device or mapped
  * page-locked host memory for J_out, rew_out, done_out, device memory for
  * obs_out.  policy, value, coef [T], grad: device memory.
+ * precision: AUV_PPO_FP32 (network products on the CUDA cores in fp32) or
+ * AUV_PPO_TF32 (on the tensor cores, tf32 operands, fp32 sums); the physics
+ * and its adjoint are fp32 either way.
  * Fossen model, 1 <= T <= AUV_ADJOINT_MAX_T, at most
  * AUV_ADJOINT_MAX_SUBSTEPS substeps, hidden a multiple of 8 up to 1024.
  * The first call at a given (N, T) allocates the window's workspace
  * (activations of every step: about T N (2 hidden + 80) floats).
  */
 int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
-                    const float* coef, float coef_V, float* grad, float* J_out, float* obs_out,
-                    float* rew_out, uint8_t* done_out, void* stream);
+                    const float* coef, float coef_V, uint32_t precision, float* grad,
+                    float* J_out, float* obs_out, float* rew_out, uint8_t* done_out,
+                    void* stream);
 
 /*
  * env_inverse_allocate: thruster commands for body-frame wrenches, the map

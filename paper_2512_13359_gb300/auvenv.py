@@ -158,7 +158,7 @@ def lib(path: str | None = None):
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
     L.env_inverse_allocate.argtypes = [P, I, P, P, P]
-    L.env_shac_window.argtypes = [P, P, P, I, P, C.c_float, P, P, P, P, P, P]
+    L.env_shac_window.argtypes = [P, P, P, I, P, C.c_float, C.c_uint32, P, P, P, P, P, P]
     L.rbuf_create.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(P)]
     L.rbuf_destroy.argtypes = [P]
     L.rbuf_last_error.argtypes = [P]
@@ -338,12 +338,13 @@ class Env:
                                       _stream(stream)))
 
     def shac_window(self, policy, value, coef, coef_V, grad, J=None, rew=None, done=None,
-                    obs=None, stream=None):
+                    obs=None, precision="fp32", stream=None):
         """SHAC actor gradient over a window of len(coef) steps in closed loop
         (env_shac_window); the env advances."""
         self._check(lib().env_shac_window(self.h, _ptr(policy), _ptr(value), coef.shape[0],
-                                          _ptr(coef), float(coef_V), _ptr(grad), _ptr(J),
-                                          _ptr(obs), _ptr(rew), _ptr(done), _stream(stream)))
+                                          _ptr(coef), float(coef_V), PPO_PRECISION[precision],
+                                          _ptr(grad), _ptr(J), _ptr(obs), _ptr(rew), _ptr(done),
+                                          _stream(stream)))
 
     def inverse_allocate(self, wrench, cmd, stream=None):
         """Thruster commands cmd [8][n] for wrenches [6][n] (env_inverse_allocate)."""

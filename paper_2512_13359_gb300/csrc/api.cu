@@ -718,8 +718,9 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
 }
 
 int env_shac_window(auv_env* env, const float* policy, const float* value, int T,
-                    const float* coef, float coef_V, float* grad, float* J_out, float* obs_out,
-                    float* rew_out, uint8_t* done_out, void* stream) {
+                    const float* coef, float coef_V, uint32_t precision, float* grad,
+                    float* J_out, float* obs_out, float* rew_out, uint8_t* done_out,
+                    void* stream) {
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);
   if (rc) return rc;
@@ -734,6 +735,8 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
   if (H < 8 || H > 1024 || H % 8)
     return fail(env, AUV_ERR_UNSUPPORTED, "the SHAC window needs hidden a multiple of 8 in [8, 1024]");
   if (!std::isfinite(coef_V)) return fail(env, AUV_ERR_INVALID, "coef_V not finite");
+  if (precision != AUV_PPO_FP32 && precision != AUV_PPO_TF32)
+    return fail(env, AUV_ERR_INVALID, "precision must be AUV_PPO_FP32 or AUV_PPO_TF32");
   if ((rc = check_device_buffer(env, policy, "policy", 4)) ||
       (rc = check_device_buffer(env, coef, "coef", 4)) ||
       (rc = check_device_buffer(env, grad, "grad", 4)))
@@ -774,7 +777,8 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
     env->shac_T = T;
   }
   rc = auv::shac::run_window(env->blas, env->model, env->buf, env->status, L, env->shac_ws,
-                             env->t_g, policy, value, coef, coef_V, grad, static_cast<float*>(J),
+                             env->t_g, policy, value, coef, coef_V, precision == AUV_PPO_TF32,
+                             grad, static_cast<float*>(J),
                              obs_out, static_cast<float*>(rew), static_cast<uint8_t*>(done), s,
                              env->err);
   if (rc != AUV_OK) return rc;

@@ -77,8 +77,8 @@ cudaError_t init(const Layout& L, char* base, cudaStream_t s);
 // blas: a cublasHandle_t.  Returns AUV_OK or an AUV_ERR_* code with err set.
 int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
-               const float* coef, float coef_V, float* grad, float* J, float* obs_out,
-               float* rew_out, uint8_t* done_out, cudaStream_t s, char* err);
+               const float* coef, float coef_V, bool tf32, float* grad, float* J,
+               float* obs_out, float* rew_out, uint8_t* done_out, cudaStream_t s, char* err);
 // obs_fm: optional [T][18][N] output of step t's observation.
 cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
                        float* obs_fm, int t, cudaStream_t s);

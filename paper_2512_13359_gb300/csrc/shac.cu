@@ -32,12 +32,13 @@ int round8(int x) { return (x + 7) & ~7; }
 
 struct Gemm {
   cublasHandle_t h;
+  cublasComputeType_t ct;
   cublasStatus_t operator()(cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
                             const float* A, int lda, const float* B, int ldb, float* C, int ldc,
                             float beta = 0.0f) const {
     const float one = 1.0f;
     return cublasGemmEx(h, ta, tb, m, n, k, &one, A, CUDA_R_32F, lda, B, CUDA_R_32F, ldb, &beta,
-                        C, CUDA_R_32F, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+                        C, CUDA_R_32F, ldc, ct, CUBLAS_GEMM_DEFAULT);
   }
 };
 
@@ -100,8 +101,8 @@ cudaError_t init(const Layout& L, char* base, cudaStream_t s) {
 
 int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
-               const float* coef, float coef_V, float* grad, float* J, float* obs_out,
-               float* rew_out, uint8_t* done_out, cudaStream_t s, char* err) {
+               const float* coef, float coef_V, bool tf32, float* grad, float* J,
+               float* obs_out, float* rew_out, uint8_t* done_out, cudaStream_t s, char* err) {
   const int n = L.n, T = L.T, H = L.H, Dp = L.Dp, Hp = L.Hp;
   const size_t N = (size_t)n;
   auto F = [&](size_t o) { return reinterpret_cast<float*>(base + o); };
@@ -120,7 +121,7 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   const float *v1 = wv, *v2 = wv + (size_t)H * Dp, *v3 = v2 + (size_t)H * Hp;
 
   cublasHandle_t h = static_cast<cublasHandle_t>(blas);
-  Gemm gemm{h};
+  Gemm gemm{h, tf32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F};
   cublasStatus_t bs = cublasSetStream(h, s);
   cudaError_t e = cudaSuccess;
   auto cfail = [&](cudaError_t x, const char* what) {

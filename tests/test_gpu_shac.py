@@ -212,3 +212,38 @@ def test_shac_critic_targets_and_regression(oracle):
     _, g_ref = P.Learner(pw, vw, (18, H, 8), hp, seed=4).grads(host, 0, 1, 512)
     gv, rv = to_np(g)[L.n_policy:], g_ref[L.n_policy:]
     assert np.abs(gv - rv).max() <= 1e-4 * np.abs(rv).max()
+
+
+def test_shac_window_tf32(oracle):
+    """The window with tensor-core (tf32) network products: J and the
+    projected gradient against the oracle within tf32's tolerance (the
+    operands carry 10 mantissa bits; measured values in the print)."""
+    torch = need_gpu()
+    n, T, H = 256, 8, 64
+    w = W.workload("ppo_65536", n_envs=n, hidden=H, mlp="fp32", w_vs=0.05)
+    env = make_env(w, policy=False)
+    env.reset()
+    pw = _smooth(W.policy_weights(w, 0.05), H)
+    vw = W.value_weights(w, 0.1)
+    b = oracle.Batch(np.arange(n))
+    b.state[:] = to_np(env.state)
+    b.params[:] = to_np(env.params)
+    b.t_ep[:] = to_np(env.t_ep)
+    b.episode[:] = to_np(env.episode).view(np.uint32)
+    t_g0 = env.t_g
+    coef = np.full(T, 1.0 / n, np.float32)
+    grad = torch.empty(pw.size, device="cuda")
+    J = torch.empty(n, device="cuda")
+    env.shac_window(torch.from_numpy(pw).cuda(), torch.from_numpy(vw).cuda(),
+                    torch.from_numpy(coef).cuda(), 0.5 / n, grad, J=J, precision="tf32")
+    m = oracle.model(w)
+    rng = np.random.default_rng(2)
+    g = to_np(grad).astype(np.float64)
+    worst = 0.0
+    for _ in range(3):
+        d = rng.normal(size=pw.size)
+        Jr, dJ = oracle.shac_window(m, b, pw, d, vw, t_g0, T, coef, 0.5 / n)
+        worst = max(worst, abs(g @ d - dJ.sum()) / np.abs(g * d).sum())
+    jerr = np.abs(to_np(J) - Jr).max() / np.abs(Jr).max()
+    print(f"[shac tf32] projected {worst:.3e}, J {jerr:.3e}")
+    assert worst <= 5e-4 and jerr <= 5e-4        # measured 2.4e-5, 1.1e-5
