@@ -7,6 +7,12 @@ data path.  Local env i of rank r is global env r * n + i; its Philox streams
 are keyed by the global id (auv_config.env_id_base), so any sharding of a
 batch reproduces the unsharded batch exactly.  torch.distributed is used only
 to align ranks and to take the slowest rank's time.
+
+The learner is the one place with an exchange: a data-parallel PPO update
+computes each rank's minibatch gradient (ppo_grads, a flat parameter
+vector), averages the vectors over ranks (mean_over_ranks, one all-reduce
+per gradient step) and takes the same Adam step everywhere (ppo_apply with
+the averaged vector), so every rank's weights stay identical.
 """
 from __future__ import annotations
 
@@ -43,3 +49,13 @@ def max_over_ranks(value: float, dist=None, device=None) -> float:
 def barrier(dist=None):
     if dist is not None and dist.is_initialized() and dist.get_world_size() > 1:
         dist.barrier()
+
+
+def mean_over_ranks(vec, dist=None):
+    """Average a tensor over all ranks in place (sum all-reduce, then divide):
+    the gradient exchange of a data-parallel update.  Returns vec."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return vec
+    dist.all_reduce(vec, op=dist.ReduceOp.SUM)
+    vec.div_(dist.get_world_size())
+    return vec
