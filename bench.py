@@ -349,6 +349,27 @@ def run_gae(args):
     print(json.dumps(line), flush=True)
 
 
+# DRAM bytes (read + write) of one rollout launch of the 65,536-env x
+# 128-step workload, from one ncu capture (dram__bytes_read.sum +
+# dram__bytes_write.sum, 1 pass, `bench.py --steps 1 --warmup 1 --no-e2e
+# --no-cpu-baseline --no-clocks`; profiles/k_engine_ppo_65536_T128_dram.md),
+# valid while the engine's sources hash to ENGINE_SRC_HASH.
+ROLLOUT_TRAFFIC_65536x128 = 10_797_056 + 903_473_664
+ENGINE_SRC_HASH = "03ff566322b868e8"
+ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
+
+
+def rollout_traffic(w, n, T):
+    import hashlib
+    if w["name"] != "ppo_65536" or n != 65536 or T != 128:
+        return None
+    h = hashlib.sha256()
+    for f in ENGINE_SRCS:
+        with open(os.path.join(ROOT, "paper_2512_13359_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return ROLLOUT_TRAFFIC_65536x128 if h.hexdigest()[:16] == ENGINE_SRC_HASH else None
+
+
 def ppo_flops_per_sample(d, h, a):
     """Algorithmic flops of one PPO sample: forward of both MLPs
     (2 x multiply-adds), their weight gradients (same count) and the input
@@ -833,7 +854,8 @@ def run(args):
         achieved = flops / (dur * 1e-3) / 1e12
         peak = peaks["bf16_tflops_sustained"]
         roof = {"bound": "tensor", "kernel": kern, "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": rollout_traffic(w, n, T) if kern == "rollout_bf16" else None,
                 "peak_source": f"bf16 sustained, {peak_src}"}
     else:
         kern, dur = "rollout_fp32", roll_avg
