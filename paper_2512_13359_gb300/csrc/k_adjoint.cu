@@ -342,7 +342,7 @@ __device__ void reward_vjp(const Model& M, const Env& e, const float a_c[kAct],
   }
 }
 
-__global__ void __launch_bounds__(kAdjThreads) k_adjoint(
+__global__ void __launch_bounds__(kAdjThreads, 4) k_adjoint(
     const Model M, Buffers B, const float* __restrict__ act, int T,
     const float* __restrict__ coef, const float* __restrict__ lam_T, float* __restrict__ g_act,
     float* __restrict__ lam_0, float* __restrict__ rew, uint8_t* __restrict__ done,
@@ -545,7 +545,7 @@ __global__ void __launch_bounds__(kAdjThreads) k_shac_step(const Model M, Buffer
 // replaced by dJ/d pre-step state through the physics, and the policy head's
 // gradient is written to gY [N][ldy] (mean, then the log-std head through
 // a = mu + sigma eps; zero where the clamp is active).
-__global__ void __launch_bounds__(kAdjThreads) k_shac_bwd(const Model M,
+__global__ void __launch_bounds__(kAdjThreads, 4) k_shac_bwd(const Model M,
                                                           const float* __restrict__ sc,
                                                           const float* __restrict__ Y, int ldy,
                                                           const uint8_t* __restrict__ done,
