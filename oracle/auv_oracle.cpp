@@ -1477,6 +1477,45 @@ void oracle_paper_reset(const PaperModel* m, int n, const uint32_t* env_ids, dou
   }
 }
 
+// The paper model's action-replay window objective
+// J = sum_t coef[t] r_t + <lam_T, x_T> over its whole state x = (p, q, nu,
+// action history: rows 0..60), and the directional derivative along
+// (dir_s0 [61][n], dir_act [T][6][n]) in Dual.  The batch is not modified.
+void oracle_paper_adjoint_window(const PaperModel* m, int n, const uint32_t* env_ids,
+                                 const double* st, const double* pr, const int32_t* t_ep,
+                                 const uint32_t* ep, int T, const double* act,
+                                 const double* coef, const double* lam_T, const double* dir_s0,
+                                 const double* dir_act, double* J, double* dJ) {
+  for (int i = 0; i < n; ++i) {
+    PaperEnv<Dual> e;
+    paper_load<Dual>(st, pr, t_ep, ep, n, i, e);
+    for (int k = 0; k < 3; ++k) e.p[k].d = dir_s0[k * n + i];
+    for (int k = 0; k < 4; ++k) e.q[k].d = dir_s0[(3 + k) * n + i];
+    for (int k = 0; k < 6; ++k) e.nu[k].d = dir_s0[(7 + k) * n + i];
+    for (int j = 0; j < kPHist; ++j)
+      for (int k = 0; k < 6; ++k) e.hist[j][k].d = dir_s0[(13 + 6 * j + k) * n + i];
+    Dual obj = 0.0;
+    for (int t = 0; t < T; ++t) {
+      Dual a[kPAct];
+      for (int k = 0; k < kPAct; ++k) {
+        const size_t o = ((size_t)t * kPAct + k) * n + i;
+        a[k] = Dual(act[o], dir_act[o]);
+      }
+      uint8_t d;
+      obj += Dual(coef[t]) * paper_control_step(*m, env_ids[i], e, a, &d);
+    }
+    if (lam_T) {
+      for (int k = 0; k < 3; ++k) obj += Dual(lam_T[k * n + i]) * e.p[k];
+      for (int k = 0; k < 4; ++k) obj += Dual(lam_T[(3 + k) * n + i]) * e.q[k];
+      for (int k = 0; k < 6; ++k) obj += Dual(lam_T[(7 + k) * n + i]) * e.nu[k];
+      for (int j = 0; j < kPHist; ++j)
+        for (int k = 0; k < 6; ++k) obj += Dual(lam_T[(13 + 6 * j + k) * n + i]) * e.hist[j][k];
+    }
+    J[i] = obj.v;
+    dJ[i] = obj.d;
+  }
+}
+
 void oracle_paper_replay(const PaperModel* m, int precision, int n, const uint32_t* env_ids,
                          double* st, double* pr, int32_t* t_ep, uint32_t* ep, int T,
                          const float* act, double* rew, uint8_t* done, double* trace) {

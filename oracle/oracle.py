@@ -372,6 +372,8 @@ def _paper_lib():
         L.oracle_paper_box.argtypes = [P, P]
         L.oracle_paper_nu_dot.argtypes = [P, P, P, P, P]
         L.oracle_paper_integrate.argtypes = [P, C.c_int, P, P, P, C.c_double, C.c_int]
+        L.oracle_paper_adjoint_window.argtypes = [P, C.c_int, P, P, P, P, P, C.c_int, P, P, P,
+                                                  P, P, P, P]
         assert L.oracle_paper_model_size() == C.sizeof(PaperModel), "PaperModel layout mismatch"
         L._paper_ready = True
     return L
@@ -450,6 +452,28 @@ def paper_replay(m: PaperModel, batch: PaperBatch, actions: np.ndarray, precisio
                                      _p(batch.t_ep), _p(batch.episode), T, _p(act), _p(rew),
                                      _p(done), _p(tr))
     return rew, done, tr
+
+
+def paper_adjoint_window(m: PaperModel, batch: PaperBatch, actions, coef, lam_T, dir_s0,
+                         dir_act):
+    """The paper model's window objective (state rows 0..60: p, q, nu and
+    the action history) and its directional derivative, in dual numbers.
+    Returns (J[n], dJ[n]); the batch is not modified."""
+    act = np.ascontiguousarray(actions, dtype=np.float64)
+    T, n = act.shape[0], batch.n
+    assert act.shape == (T, PAPER_ACT, n)
+    coef = np.ascontiguousarray(coef, dtype=np.float64)
+    lam = None if lam_T is None else np.ascontiguousarray(lam_T, dtype=np.float64)
+    ds0 = np.ascontiguousarray(dir_s0, dtype=np.float64)
+    da = np.ascontiguousarray(dir_act, dtype=np.float64)
+    assert ds0.shape == (PAPER_STATE, n) and da.shape == act.shape
+    J = np.zeros(n)
+    dJ = np.zeros(n)
+    _paper_lib().oracle_paper_adjoint_window(C.byref(m), n, _p(batch.env_ids), _p(batch.state),
+                                             _p(batch.params), _p(batch.t_ep),
+                                             _p(batch.episode), T, _p(act), _p(coef), _p(lam),
+                                             _p(ds0), _p(da), _p(J), _p(dJ))
+    return J, dJ
 
 
 def paper_rollout(m: PaperModel, batch: PaperBatch, pol_w, val_w, t_g0: int, T: int,
