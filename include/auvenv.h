@@ -505,17 +505,21 @@ int ppo_export_weights(auv_ppo* p, float* policy, float* value, void* stream);
  * dJ/dx_0 (lam_0).  An episode end inside the window replaces the state by
  * its reset draw: nothing before it reaches later rewards or x_T.  The
  * clip's derivative is taken as 1 on [-1, 1] and 0 outside.
- *   act [T][8][N], grad_act [T][8][N]: device memory.
+ * Shapes by model (A = env_layout's act_dim, S = the adjoint's state rows):
+ *   Fossen: A = 8, S = 13 (p, q, nu; nu_prev is overwritten by every step);
+ *   paper:  A = 6, S = 61 (p, q, nu and the 8 x 6 action-history rows of its
+ *           state layout: the moving-average reward term makes an action
+ *           reach later rewards through them).
+ *   act [T][A][N], grad_act [T][A][N]: device memory.
  *   coef [T]: device memory.
- *   lam_T [13][N] (rows p, q, nu): device memory, or NULL for 0.
- *   lam_0 [13][N], rew_out [T][N] (fp32), done_out [T][N] (u8): optional
+ *   lam_T [S][N]: device memory, or NULL for 0.
+ *   lam_0 [S][N], rew_out [T][N] (fp32), done_out [T][N] (u8): optional
  *   outputs, device or mapped page-locked host memory.
  * The env's state, episode counters and step counter are not changed (step
- * with env_step_actions to advance).  Fossen model only
- * (AUV_ERR_UNSUPPORTED for the paper model); 1 <= T <= AUV_ADJOINT_MAX_T;
- * at most AUV_ADJOINT_MAX_SUBSTEPS substeps (AUV_ERR_UNSUPPORTED).  The first
- * call at a given N * T allocates the window's scratch (30 floats per
- * env-step) on the device.
+ * with env_step_actions to advance).  1 <= T <= AUV_ADJOINT_MAX_T; at most
+ * AUV_ADJOINT_MAX_SUBSTEPS substeps (AUV_ERR_UNSUPPORTED).  The first call at
+ * a given N * T allocates the window's scratch (30 floats per env-step plus
+ * 61 per env) on the device.
  */
 #define AUV_ADJOINT_MAX_T 64
 #define AUV_ADJOINT_MAX_SUBSTEPS 8

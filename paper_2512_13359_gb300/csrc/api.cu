@@ -680,8 +680,6 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);
   if (rc) return rc;
-  if (is_paper(&env->cfg))
-    return fail(env, AUV_ERR_UNSUPPORTED, "the adjoint is built for the Fossen model");
   if (T < 1 || T > AUV_ADJOINT_MAX_T)
     return fail(env, AUV_ERR_INVALID, "T outside [1, %d]", AUV_ADJOINT_MAX_T);
   if (env->model.substeps > AUV_ADJOINT_MAX_SUBSTEPS)

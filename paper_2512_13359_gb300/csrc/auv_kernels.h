@@ -59,6 +59,7 @@ cudaError_t launch_paper_rollout_fp32(const Model& M, const Buffers& B, const fl
 // (k_adjoint.cu).  scratch: adjoint_scratch_floats(n, T) floats.  T <= 64,
 // M.substeps <= 8.
 size_t adjoint_scratch_floats(int n, int T);
+size_t adjoint_step_floats(int n);   // one Fossen step's slice of the scratch
 cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, int T,
                            const float* coef, const float* lam_T, float* g_act, float* lam_0,
                            float* rew, uint8_t* done, float* scratch, Status* st,

@@ -20,6 +20,7 @@
 // update, velocity update, the right-hand side of the equations of motion),
 // allocation and the command clip.  The env's buffers are read, not written.
 #include "auv_kernels.h"
+#include "paper_device.cuh"
 
 namespace auv {
 
@@ -107,6 +108,73 @@ __device__ __forceinline__ void rot_vjp(const float q[4], const float L[3][3], f
                    2.0f * z * L[1][1] + y * L[1][2] + x * L[2][0] + y * L[2][1]);
 }
 
+// Vector-Jacobian product of the pose part of a substep (auv_device.cuh:
+// advance_pose, shared by both models): p1 = p + h R(q) v1 and
+// q1 = normalize(q (x) (cos a, sin(a)/a hw)), hw = h w1 / 2, a = |hw|.  On
+// entry lx holds dJ/d(p1, q1, nu1); on exit lnu1 = dJ/dnu1 (the direct part
+// plus the pose's), LR = dJ/dR from the position update, lq = dJ/dq from the
+// attitude product; lx.p is unchanged (p1 = p + ...).
+__device__ void pose_vjp(float h, const float q[4], const float R[3][3], const float nu1[6],
+                         const X& lx, float lnu1[6], float LR[3][3], float lq[4]) {
+  const float hw[3] = {0.5f * h * nu1[3], 0.5f * h * nu1[4], 0.5f * h * nu1[5]};
+  const float a2 = hw[0] * hw[0] + hw[1] * hw[1] + hw[2] * hw[2];
+  float ca, s, g;     // cos a, sin(a)/a, (a cos a - sin a)/a^3
+  if (a2 < 0.25f) {
+    ca = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 40320.0f, -1.0f / 720.0f), a2, 1.0f / 24.0f), a2, -0.5f),
+              a2, 1.0f);
+    s = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 362880.0f, -1.0f / 5040.0f), a2, 1.0f / 120.0f), a2,
+                  -1.0f / 6.0f),
+             a2, 1.0f);
+    g = fmaf(fmaf(fmaf(fmaf(a2, -1.0f / 3991680.0f, 1.0f / 45360.0f), a2, -1.0f / 840.0f), a2,
+                  1.0f / 30.0f),
+             a2, -1.0f / 3.0f);
+  } else {
+    const float a = sqrtf(a2);
+    float sn;
+    sincosf(a, &sn, &ca);
+    s = sn / a;
+    g = (a * ca - sn) / (a2 * a);
+  }
+  const float d[4] = {ca, s * hw[0], s * hw[1], s * hw[2]};
+  const float qw = q[0], qx = q[1], qy = q[2], qz = q[3];
+  const float u[4] = {qw * d[0] - qx * d[1] - qy * d[2] - qz * d[3],
+                      qw * d[1] + qx * d[0] + qy * d[3] - qz * d[2],
+                      qw * d[2] - qx * d[3] + qy * d[0] + qz * d[1],
+                      qw * d[3] + qx * d[2] - qy * d[1] + qz * d[0]};
+  const float inv_u = rsqrtf(u[0] * u[0] + u[1] * u[1] + u[2] * u[2] + u[3] * u[3]);
+  const float q1[4] = {u[0] * inv_u, u[1] * inv_u, u[2] * inv_u, u[3] * inv_u};
+  // q1 = u / |u|
+  const float dot = lx.q[0] * q1[0] + lx.q[1] * q1[1] + lx.q[2] * q1[2] + lx.q[3] * q1[3];
+  float lu[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lu[k] = (lx.q[k] - dot * q1[k]) * inv_u;
+  // u = q (x) d
+  lq[0] = d[0] * lu[0] + d[1] * lu[1] + d[2] * lu[2] + d[3] * lu[3];
+  lq[1] = -d[1] * lu[0] + d[0] * lu[1] - d[3] * lu[2] + d[2] * lu[3];
+  lq[2] = -d[2] * lu[0] + d[3] * lu[1] + d[0] * lu[2] - d[1] * lu[3];
+  lq[3] = -d[3] * lu[0] - d[2] * lu[1] + d[1] * lu[2] + d[0] * lu[3];
+  const float ld0 = qw * lu[0] + qx * lu[1] + qy * lu[2] + qz * lu[3];
+  const float ld[3] = {-qx * lu[0] + qw * lu[1] + qz * lu[2] - qy * lu[3],
+                       -qy * lu[0] - qz * lu[1] + qw * lu[2] + qx * lu[3],
+                       -qz * lu[0] + qy * lu[1] - qx * lu[2] + qw * lu[3]};
+  // d = (cos a, s(a) hw), a = |hw|
+  const float hl = hw[0] * ld[0] + hw[1] * ld[1] + hw[2] * ld[2];
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    const float lhw = -s * hw[k] * ld0 + s * ld[k] + g * hw[k] * hl;
+    lnu1[3 + k] = lx.nu[3 + k] + 0.5f * h * lhw;
+  }
+  // p1 = p + h R v1
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+#pragma unroll
+    for (int j = 0; j < 3; ++j) LR[i][j] = h * lx.p[i] * nu1[j];
+  }
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+    lnu1[j] = lx.nu[j] + h * (R[0][j] * lx.p[0] + R[1][j] * lx.p[1] + R[2][j] * lx.p[2]);
+}
+
 // Vector-Jacobian product of one substep (auv_device.cuh: substep) taken
 // from input x with wrench tau: on entry lx is dJ/d(output), on exit
 // dJ/d(input); ltau accumulates dJ/dtau.
@@ -154,68 +222,8 @@ __device__ void substep_vjp(const Model& M, const Env& e, const X& x, const floa
   }
 #pragma unroll
   for (int k = 0; k < 6; ++k) nu1[k] = x.nu[k] + M.h * (rhs[k] * e.inv_m[k]);
-  // attitude update: u = q (x) (ca, s hw), q1 = u / |u|, hw = h w1 / 2
-  const float hw[3] = {0.5f * M.h * nu1[3], 0.5f * M.h * nu1[4], 0.5f * M.h * nu1[5]};
-  const float a2 = hw[0] * hw[0] + hw[1] * hw[1] + hw[2] * hw[2];
-  float ca, s, g;     // cos a, sin(a)/a, (a cos a - sin a)/a^3
-  if (a2 < 0.25f) {
-    ca = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 40320.0f, -1.0f / 720.0f), a2, 1.0f / 24.0f), a2, -0.5f),
-              a2, 1.0f);
-    s = fmaf(fmaf(fmaf(fmaf(a2, 1.0f / 362880.0f, -1.0f / 5040.0f), a2, 1.0f / 120.0f), a2,
-                  -1.0f / 6.0f),
-             a2, 1.0f);
-    g = fmaf(fmaf(fmaf(fmaf(a2, -1.0f / 3991680.0f, 1.0f / 45360.0f), a2, -1.0f / 840.0f), a2,
-                  1.0f / 30.0f),
-             a2, -1.0f / 3.0f);
-  } else {
-    const float a = sqrtf(a2);
-    float sn;
-    sincosf(a, &sn, &ca);
-    s = sn / a;
-    g = (a * ca - sn) / (a2 * a);
-  }
-  const float d[4] = {ca, s * hw[0], s * hw[1], s * hw[2]};
-  const float qw = x.q[0], qx = x.q[1], qy = x.q[2], qz = x.q[3];
-  const float u[4] = {qw * d[0] - qx * d[1] - qy * d[2] - qz * d[3],
-                      qw * d[1] + qx * d[0] + qy * d[3] - qz * d[2],
-                      qw * d[2] - qx * d[3] + qy * d[0] + qz * d[1],
-                      qw * d[3] + qx * d[2] - qy * d[1] + qz * d[0]};
-  const float inv_u = rsqrtf(u[0] * u[0] + u[1] * u[1] + u[2] * u[2] + u[3] * u[3]);
-  const float q1[4] = {u[0] * inv_u, u[1] * inv_u, u[2] * inv_u, u[3] * inv_u};
-
-  // ---- reverse ----
-  // q1 = u / |u|
-  const float dot = lx.q[0] * q1[0] + lx.q[1] * q1[1] + lx.q[2] * q1[2] + lx.q[3] * q1[3];
-  float lu[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) lu[k] = (lx.q[k] - dot * q1[k]) * inv_u;
-  // u = q (x) d
-  float lq[4] = {d[0] * lu[0] + d[1] * lu[1] + d[2] * lu[2] + d[3] * lu[3],
-                 -d[1] * lu[0] + d[0] * lu[1] - d[3] * lu[2] + d[2] * lu[3],
-                 -d[2] * lu[0] + d[3] * lu[1] + d[0] * lu[2] - d[1] * lu[3],
-                 -d[3] * lu[0] - d[2] * lu[1] + d[1] * lu[2] + d[0] * lu[3]};
-  const float ld0 = qw * lu[0] + qx * lu[1] + qy * lu[2] + qz * lu[3];
-  const float ld[3] = {-qx * lu[0] + qw * lu[1] + qz * lu[2] - qy * lu[3],
-                       -qy * lu[0] - qz * lu[1] + qw * lu[2] + qx * lu[3],
-                       -qz * lu[0] + qy * lu[1] - qx * lu[2] + qw * lu[3]};
-  // d = (cos a, s(a) hw), a = |hw|
-  const float hl = hw[0] * ld[0] + hw[1] * ld[1] + hw[2] * ld[2];
-  float lnu1[6];
-#pragma unroll
-  for (int k = 0; k < 3; ++k) {
-    const float lhw = -s * hw[k] * ld0 + s * ld[k] + g * hw[k] * hl;
-    lnu1[3 + k] = lx.nu[3 + k] + 0.5f * M.h * lhw;
-  }
-  // p1 = p + h R v1
-  float LR[3][3];
-#pragma unroll
-  for (int i = 0; i < 3; ++i) {
-#pragma unroll
-    for (int j = 0; j < 3; ++j) LR[i][j] = M.h * lx.p[i] * nu1[j];
-  }
-#pragma unroll
-  for (int j = 0; j < 3; ++j)
-    lnu1[j] = lx.nu[j] + M.h * (R[0][j] * lx.p[0] + R[1][j] * lx.p[1] + R[2][j] * lx.p[2]);
+  float lnu1[6], LR[3][3], lq[4];
+  pose_vjp(M.h, x.q, R, nu1, lx, lnu1, LR, lq);
   // nu1 = nu + h M^-1 rhs
   float lr[6];
 #pragma unroll
@@ -644,9 +652,287 @@ __global__ void __launch_bounds__(kAdjThreads) k_fill_col(int n, float* __restri
   if (i < n) buf[(size_t)i * ld] = v;
 }
 
+// ---------------------------------------------------------------------------
+// The paper model (paper_device.cuh): its state adds the K-slot history of
+// clipped actions (rows 13 + 6 j + k), which the reward's moving-average
+// term reads, so the adjoint carries those rows too.
+// ---------------------------------------------------------------------------
+constexpr int kPScratchF = 28;   // x(13) pd(3) qd(4) g t_ep mean of the history(6)
+
+// lq += (d theta / dq)^T lth for the axis-angle error of paper_device.cuh:
+// qe = conj(q_d) (x) q, flipped to w >= 0; theta = s v, s = 2 atan2(|v|, w) / |v|.
+__device__ void att_error_vjp(const paper::Env& e, const float lth[3], float lq[4]) {
+  const float aw = e.qd[0], ax = -e.qd[1], ay = -e.qd[2], az = -e.qd[3];
+  const float bw = e.q[0], bx = e.q[1], by = e.q[2], bz = e.q[3];
+  float w = aw * bw - ax * bx - ay * by - az * bz;
+  float v[3] = {aw * bx + ax * bw + ay * bz - az * by, aw * by - ax * bz + ay * bw + az * bx,
+                aw * bz + ax * by - ay * bx + az * bw};
+  const float sg = w < 0.0f ? -1.0f : 1.0f;
+  w *= sg;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) v[k] *= sg;
+  const float vn2 = v[0] * v[0] + v[1] * v[1] + v[2] * v[2], vn = sqrtf(vn2);
+  const float den = vn2 + w * w;
+  float s, c;      // s, and (ds/d|v|) / |v|
+  if (vn > 1e-3f * w) {
+    s = 2.0f * atan2f(vn, w) / vn;
+    c = (2.0f * w / den - s) / vn2;
+  } else {         // series in r = |v| / w: s = (2/w)(1 - r^2/3 + r^4/5)
+    const float iw = 1.0f / w, r2 = vn2 * iw * iw;
+    s = 2.0f * iw * (1.0f - r2 / 3.0f + r2 * r2 / 5.0f);
+    c = 4.0f * iw * iw * iw * (-1.0f / 3.0f + 2.0f * r2 / 5.0f);
+  }
+  const float tv = lth[0] * v[0] + lth[1] * v[1] + lth[2] * v[2];
+  float lqe[4];
+  lqe[0] = sg * tv * (-2.0f / den);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lqe[1 + k] = sg * (s * lth[k] + tv * c * v[k]);
+  lq[0] += aw * lqe[0] + ax * lqe[1] + ay * lqe[2] + az * lqe[3];
+  lq[1] += -ax * lqe[0] + aw * lqe[1] + az * lqe[2] - ay * lqe[3];
+  lq[2] += -ay * lqe[0] - az * lqe[1] + aw * lqe[2] + ax * lqe[3];
+  lq[3] += -az * lqe[0] + ay * lqe[1] - ax * lqe[2] + aw * lqe[3];
+}
+
+// dJ/d(state) += (d obs / d state)^T lo for the paper model's observation
+// [R^T (p - p_d), theta, v, w].
+__device__ void paper_obs_vjp(const paper::Env& e, const float lo[paper::kObs], X& lx) {
+  float R[3][3];
+  quat_rot(e.q, R);
+  const float dp[3] = {e.p[0] - e.pd[0], e.p[1] - e.pd[1], e.p[2] - e.pd[2]};
+  float LR[3][3];
+#pragma unroll
+  for (int j = 0; j < 3; ++j) {
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      LR[j][i] = lo[i] * dp[j];
+      lx.p[j] += R[j][i] * lo[i];
+    }
+  }
+  rot_vjp(e.q, LR, lx.q);
+  att_error_vjp(e, lo + 3, lx.q);
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lx.nu[k] += lo[6 + k];
+}
+
+// VJP of one paper-model substep (paper_device.cuh: substep).
+__device__ void paper_substep_vjp(const Model& M, const paper::Env& e, const X& x,
+                                  const float tau[6], X& lx, float ltau[6]) {
+  float R[3][3];
+  quat_rot(x.q, R);
+  const float v[3] = {x.nu[0], x.nu[1], x.nu[2]};
+  const float w[3] = {x.nu[3], x.nu[4], x.nu[5]};
+  const float m = M.mass, mg = m * e.g;
+  float wxv[3], Iw[3], wxIw[3], nu1[6];
+  cross3(w, v, wxv);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) Iw[k] = M.inertia[k] * w[k];
+  cross3(w, Iw, wxIw);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    const float f = -M.kf_drag[k] * fabsf(v[k]) * v[k] - M.c_visc_f * v[k];
+    const float t = -M.kt_drag[k] * fabsf(w[k]) * w[k] - M.c_visc_t * w[k];
+    const float lin = tau[k] + f - mg * R[2][k] - m * wxv[k];
+    const float rot = tau[3 + k] + t - wxIw[k];
+    nu1[k] = fmaf(M.h, lin * M.inv_mass, x.nu[k]);
+    nu1[3 + k] = fmaf(M.h, rot * M.inv_inertia[k], x.nu[3 + k]);
+  }
+  float lnu1[6], LR[3][3], lq[4];
+  pose_vjp(M.h, x.q, R, nu1, lx, lnu1, LR, lq);
+  float llin[3], lrot[3], lv[3], lw[3], ly[3], lt[3] = {0.f, 0.f, 0.f};
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    llin[k] = M.h * M.inv_mass * lnu1[k];
+    lrot[k] = M.h * M.inv_inertia[k] * lnu1[3 + k];
+    ltau[k] += llin[k];
+    ltau[3 + k] += lrot[k];
+    lv[k] = llin[k] * (-2.0f * M.kf_drag[k] * fabsf(v[k]) - M.c_visc_f);
+    lw[k] = lrot[k] * (-2.0f * M.kt_drag[k] * fabsf(w[k]) - M.c_visc_t);
+    LR[2][k] -= mg * llin[k];
+    ly[k] = -m * llin[k];
+  }
+  cross_vjp(w, v, ly, lw, lv);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) ly[k] = -lrot[k];
+  cross_vjp(w, Iw, ly, lw, lt);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lw[k] += M.inertia[k] * lt[k];
+  rot_vjp(x.q, LR, lq);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lx.q[k] = lq[k];
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    lx.nu[k] = lnu1[k] + lv[k];
+    lx.nu[3 + k] = lnu1[3 + k] + lw[k];
+  }
+}
+
+__global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
+    const Model M, Buffers B, const float* __restrict__ act, int T,
+    const float* __restrict__ coef, const float* __restrict__ lam_T, float* __restrict__ g_act,
+    float* __restrict__ lam_0, float* __restrict__ rew, uint8_t* __restrict__ done,
+    float* __restrict__ scratch, Status* st) {
+  using namespace paper;
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  const size_t n = (size_t)M.n;
+  const uint32_t id = M.id_base + (uint32_t)i;
+  const int K = M.mavg_len;
+  const float inv_k = 1.0f / (float)K;
+  float* hsc = scratch + (size_t)T * kPScratchF * n;    // [61][n]: rows 13.. the history
+  paper::Env e;
+  paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  for (int r = 13; r < paper::kStateF; ++r) hsc[r * n + i] = B.state[r * n + i];
+  uint64_t ends = 0;
+  for (int t = 0; t < T; ++t) {
+    float mean[6];
+#pragma unroll
+    for (int k = 0; k < 6; ++k) {
+      float sum = 0.0f;
+      for (int j = 0; j < K; ++j) sum += hsc[(13 + 6 * j + k) * n + i];
+      mean[k] = sum * inv_k;
+    }
+    float* sc = scratch + (size_t)t * kPScratchF * n;
+    const float v[kPScratchF] = {e.p[0], e.p[1], e.p[2], e.q[0], e.q[1], e.q[2], e.q[3],
+                                 e.nu[0], e.nu[1], e.nu[2], e.nu[3], e.nu[4], e.nu[5],
+                                 e.pd[0], e.pd[1], e.pd[2], e.qd[0], e.qd[1], e.qd[2], e.qd[3],
+                                 e.g, __int_as_float(e.t_ep), mean[0], mean[1], mean[2], mean[3],
+                                 mean[4], mean[5]};
+#pragma unroll
+    for (int k = 0; k < kPScratchF; ++k) sc[k * n + i] = v[k];
+    float a[paper::kAct];
+#pragma unroll
+    for (int k = 0; k < paper::kAct; ++k) a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
+    bool d;
+    const float r = paper::physics_step(M, id, e, a, hsc, i, &d);
+    if (d) ends |= 1ull << t;
+    if (rew) rew[(size_t)t * n + i] = r;
+    if (done) done[(size_t)t * n + i] = d ? 1 : 0;
+  }
+  X lx;
+  float lh[paper::kHist][6];
+#pragma unroll
+  for (int k = 0; k < kX; ++k) {
+    const float v = lam_T ? __ldg(lam_T + k * n + i) : 0.0f;
+    if (k < 3) lx.p[k] = v;
+    else if (k < 7) lx.q[k - 3] = v;
+    else lx.nu[k - 7] = v;
+  }
+  for (int j = 0; j < paper::kHist; ++j)
+#pragma unroll
+    for (int k = 0; k < 6; ++k) lh[j][k] = lam_T ? __ldg(lam_T + (13 + 6 * j + k) * n + i) : 0.0f;
+  X xs[8];
+  for (int t = T - 1; t >= 0; --t) {
+    if ((ends >> t) & 1ull) {
+#pragma unroll
+      for (int k = 0; k < 3; ++k) lx.p[k] = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) lx.q[k] = 0.f;
+#pragma unroll
+      for (int k = 0; k < 6; ++k) lx.nu[k] = 0.f;
+      for (int j = 0; j < paper::kHist; ++j)
+#pragma unroll
+        for (int k = 0; k < 6; ++k) lh[j][k] = 0.f;
+    }
+    const float* sc = scratch + (size_t)t * kPScratchF * n;
+    float v[kPScratchF];
+#pragma unroll
+    for (int k = 0; k < kPScratchF; ++k) v[k] = sc[k * n + i];
+    paper::Env es;
+#pragma unroll
+    for (int k = 0; k < 3; ++k) { es.p[k] = v[k]; es.pd[k] = v[13 + k]; }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) { es.q[k] = v[3 + k]; es.qd[k] = v[16 + k]; }
+#pragma unroll
+    for (int k = 0; k < 6; ++k) es.nu[k] = v[7 + k];
+    es.g = v[20];
+    const int t_ep = __float_as_int(v[21]);
+    float a[paper::kAct], a_c[paper::kAct], tau[6], la[paper::kAct];
+#pragma unroll
+    for (int k = 0; k < paper::kAct; ++k) {
+      a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
+      a_c[k] = fminf(fmaxf(a[k], -1.0f), 1.0f);
+    }
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      tau[k] = M.f_max * a_c[k];
+      tau[3 + k] = M.tau_max * a_c[3 + k];
+    }
+    for (int s = 0; s < M.substeps; ++s) {
+#pragma unroll
+      for (int k = 0; k < 3; ++k) xs[s].p[k] = es.p[k];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) xs[s].q[k] = es.q[k];
+#pragma unroll
+      for (int k = 0; k < 6; ++k) xs[s].nu[k] = es.nu[k];
+      paper::substep(M, es, tau);
+    }
+    // the history slot written after this step's reward held a_c
+    const int slot = t_ep % K;
+#pragma unroll
+    for (int k = 0; k < 6; ++k) {
+      la[k] = lh[slot][k];
+      lh[slot][k] = 0.0f;
+    }
+    // reward on the post-step state
+    const float c = __ldg(coef + t);
+    float o[paper::kObs], lo[paper::kObs];
+    paper::observe(es, o);
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      lo[k] = -c * M.w_pos * 2.0f * M.w_axes[k] * M.w_axes[k] * o[k];
+      lo[3 + k] = -c * M.w_att * 2.0f * o[3 + k];
+      lo[6 + k] = 0.0f;
+      lo[9 + k] = -c * M.w_vel * 2.0f * o[9 + k];
+      la[3 + k] += -c * M.w_act * 2.0f * a_c[3 + k];
+    }
+    paper_obs_vjp(es, lo, lx);
+#pragma unroll
+    for (int k = 0; k < 6; ++k) {
+      const float dk = a_c[k] - v[22 + k];
+      la[k] += -c * M.w_mavg * 2.0f * dk;
+      const float lm = c * M.w_mavg * 2.0f * dk * inv_k;
+      for (int j = 0; j < K; ++j) lh[j][k] += lm;
+    }
+    float ltau[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int s = M.substeps - 1; s >= 0; --s) paper_substep_vjp(M, es, xs[s], tau, lx, ltau);
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      la[k] += M.f_max * ltau[k];
+      la[3 + k] += M.tau_max * ltau[3 + k];
+    }
+#pragma unroll
+    for (int k = 0; k < paper::kAct; ++k)
+      g_act[((size_t)t * paper::kAct + k) * n + i] = (a[k] >= -1.0f && a[k] <= 1.0f) ? la[k] : 0.0f;
+  }
+  float s = 0.0f;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) s += lx.p[k];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) s += lx.q[k];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) s += lx.nu[k];
+  if (!isfinite(s)) flag_nan(st, i);
+  if (lam_0) {
+#pragma unroll
+    for (int k = 0; k < 3; ++k) lam_0[k * n + i] = lx.p[k];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) lam_0[(3 + k) * n + i] = lx.q[k];
+#pragma unroll
+    for (int k = 0; k < 6; ++k) lam_0[(7 + k) * n + i] = lx.nu[k];
+    for (int j = 0; j < paper::kHist; ++j)
+#pragma unroll
+      for (int k = 0; k < 6; ++k) lam_0[(13 + 6 * j + k) * n + i] = lh[j][k];
+  }
+}
+
 }  // namespace
 
-size_t adjoint_scratch_floats(int n, int T) { return (size_t)T * kScratchF * (size_t)n; }
+size_t adjoint_step_floats(int n) { return (size_t)kScratchF * (size_t)n; }
+
+size_t adjoint_scratch_floats(int n, int T) {
+  // Fossen: T steps of 30 floats; paper: T steps of 28 plus a 61-row history copy
+  return ((size_t)T * kScratchF + paper::kStateF) * (size_t)n;
+}
 
 namespace shac {
 
@@ -694,6 +980,11 @@ cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, i
                            const float* coef, const float* lam_T, float* g_act, float* lam_0,
                            float* rew, uint8_t* done, float* scratch, Status* st,
                            cudaStream_t s) {
+  if (M.model == 1) {
+    k_paper_adjoint<<<(M.n + kAdjThreads - 1) / kAdjThreads, kAdjThreads, 0, s>>>(
+        M, B, act, T, coef, lam_T, g_act, lam_0, rew, done, scratch, st);
+    return cudaGetLastError();
+  }
   k_adjoint<<<(M.n + kAdjThreads - 1) / kAdjThreads, kAdjThreads, 0, s>>>(
       M, B, act, T, coef, lam_T, g_act, lam_0, rew, done, scratch, st);
   return cudaGetLastError();

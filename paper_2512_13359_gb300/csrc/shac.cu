@@ -115,7 +115,7 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   auto H1s = [&](int t) { return H1 + (size_t)t * N * Hp; };
   auto H2s = [&](int t) { return H2 + (size_t)t * N * Hp; };
   auto Ys = [&](int t) { return Y + (size_t)t * N * kLdy; };
-  auto SCs = [&](int t) { return sc + (size_t)t * adjoint_scratch_floats(n, 1); };
+  auto SCs = [&](int t) { return sc + (size_t)t * adjoint_step_floats(n); };
   const float *w1 = wp, *w2 = wp + (size_t)H * Dp, *w3 = w2 + (size_t)H * Hp;
   float *g1 = gp, *g2 = gp + (size_t)H * Dp, *g3 = g2 + (size_t)H * Hp;
   const float *v1 = wv, *v2 = wv + (size_t)H * Dp, *v3 = v2 + (size_t)H * Hp;

@@ -4,7 +4,8 @@ forward-mode dual numbers: for random directions (d_x0, d_a) the GPU's
 the same window objective J = sum_t coef_t r_t + <lam_T, x_T>, per env;
 unit directions check single components; windows with and without episode
 ends, ragged env counts, the full-size window sampled, saturated thrusters,
-and argument rejection."""
+the paper model (its adjoint state includes the action-history rows), and
+argument rejection."""
 import numpy as np
 import pytest
 
@@ -158,7 +159,51 @@ def test_adjoint_rejects_bad_arguments():
     with pytest.raises(auvenv.AuvError) as ei:
         env16.adjoint(act[:4], coef[:4], g[:4])
     assert ei.value.code == auvenv.AUV_ERR_UNSUPPORTED
-    pe = make_env(W.workload("paper_tiny", n_envs=n), policy=False)
-    with pytest.raises(auvenv.AuvError) as ei:
-        pe.adjoint(act[:4, :6].contiguous(), coef[:4], g[:4])
-    assert ei.value.code == auvenv.AUV_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("n,T,L,K", [(300, 10, 500, 4), (129, 12, 9, 3), (64, 6, 500, 8)])
+def test_paper_adjoint_matches_dual_numbers(oracle, n, T, L, K):
+    """The paper model: 61 adjoint rows (p, q, nu, the 8 x 6 history), the
+    moving-average term carrying gradient from later rewards to earlier
+    actions, episode ends inside the window."""
+    torch = need_gpu()
+    w = W.workload("paper_tiny", n_envs=n, substeps=4, dr_enable=1, mavg_len=K, g_eff=0.05,
+                   episode_len=L)
+    env = make_env(w, policy=False)
+    env.reset()
+    warm = torch.from_numpy(W.replay_actions(n + 1, 5, n, scale=0.8, act=6)).cuda()
+    env.step_actions(warm, torch.empty((5, n), device="cuda"),
+                     torch.empty((5, n), dtype=torch.uint8, device="cuda"))
+    rng = np.random.default_rng(n + T)
+    act = rng.uniform(-1.1, 1.1, (T, 6, n)).astype(np.float32)
+    coef = (0.99 ** np.arange(T)).astype(np.float32)
+    lam_T = rng.normal(size=(61, n)).astype(np.float32)
+    st0 = to_np(env.state).copy()
+    g = torch.empty((T, 6, n), device="cuda")
+    l0 = torch.empty((61, n), device="cuda")
+    done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
+    env.adjoint(torch.from_numpy(act).cuda(), torch.from_numpy(coef).cuda(), g,
+                lam_T=torch.from_numpy(lam_T).cuda(), lam_0=l0, done=done)
+    assert env.status().code == 0
+    assert np.array_equal(to_np(env.state), st0)
+    if L < 5 + T:
+        assert to_np(done).any()
+    m = oracle.paper_model(w)
+    b = oracle.PaperBatch(np.arange(n))
+    b.state[:] = st0
+    b.params[:] = to_np(env.params)
+    b.t_ep[:] = to_np(env.t_ep)
+    b.episode[:] = to_np(env.episode).view(np.uint32)
+    G, L0 = to_np(g), to_np(l0)
+    worst = 0.0
+    for _ in range(3):
+        ds0 = rng.normal(size=(61, n))
+        da = rng.normal(size=(T, 6, n))
+        _, dJ = oracle.paper_adjoint_window(m, b, act.astype(np.float64), coef, lam_T, ds0, da)
+        terms = G * da
+        got = terms.sum(axis=(0, 1)) + (L0 * ds0).sum(axis=0)
+        scale = np.abs(terms).sum(axis=(0, 1)) + np.abs(L0 * ds0).sum(axis=0)
+        worst = max(worst, float((np.abs(got - dJ) / np.maximum(scale, 1e-6)).max()))
+    print(f"[paper adjoint n{n} T{T} L{L} K{K}] {worst:.3e} (tol {ADJ_TOL})")
+    assert worst <= ADJ_TOL
+    assert np.all(G[np.abs(act) > 1.0] == 0.0)
