@@ -471,6 +471,9 @@ def run_ppo(args):
 # of k_adjoint from one ncu capture of `bench.py --adjoint --n-envs 8192`,
 # divided by its 262,144 env-steps (674 FADD + 1273 FMUL + 2021 FFMA).
 ADJOINT_FLOPS_PER_ENV_STEP = {4: 5988.2}
+# The paper model's k_paper_adjoint, counted the same way (4 substeps,
+# history of K = 4): `bench.py --adjoint --workload paper_4096 --n-envs 8192`.
+PAPER_ADJOINT_FLOPS_PER_ENV_STEP = {4: 4452.3}   # 409 FADD + 979 FMUL + 1532 FFMA
 
 
 def run_adjoint(args):
@@ -485,18 +488,20 @@ def run_adjoint(args):
         over["n_envs"] = args.n_envs
     w = W.workload(args.workload, **over)
     n, T = int(w["n_envs"]), int(args.window)
+    A = W.act_dim(w)
+    S = 61 if W.is_paper(w) else 13
     env = auvenv.Env(w)
     env.reset()
-    warm = torch.from_numpy(W.replay_actions(1, 8, n, scale=0.8)).cuda()
+    warm = torch.from_numpy(W.replay_actions(1, 8, n, scale=0.8, act=A)).cuda()
     rew0 = torch.empty((8, n), device="cuda")
     done0 = torch.empty((8, n), dtype=torch.uint8, device="cuda")
     env.step_actions(warm, rew0, done0)
-    act = torch.from_numpy(W.replay_actions(2, T, n, scale=0.9)).cuda()
+    act = torch.from_numpy(W.replay_actions(2, T, n, scale=0.9, act=A)).cuda()
     coef = torch.tensor([0.99 ** t / (n * T) for t in range(T)], dtype=torch.float32,
                         device="cuda")
-    lam_T = torch.randn((13, n), device="cuda") / (n * T)
-    g = torch.empty((T, 8, n), device="cuda")
-    lam_0 = torch.empty((13, n), device="cuda")
+    lam_T = torch.randn((S, n), device="cuda") / (n * T)
+    g = torch.empty((T, A, n), device="cuda")
+    lam_0 = torch.empty((S, n), device="cuda")
     flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
     for _ in range(args.warmup):
         env.adjoint(act, coef, g, lam_T=lam_T, lam_0=lam_0)
@@ -521,7 +526,8 @@ def run_adjoint(args):
     peaks, src = load_peaks()
     mhz = peaks.get("sm_max_mhz", 2070.0)
     peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
-    fps = ADJOINT_FLOPS_PER_ENV_STEP.get(int(w["substeps"]))
+    table = PAPER_ADJOINT_FLOPS_PER_ENV_STEP if W.is_paper(w) else ADJOINT_FLOPS_PER_ENV_STEP
+    fps = table.get(int(w["substeps"]))
     achieved = None if fps is None else rate * fps / 1e12
     line = {
         "metric": "adjoint env-steps/s", "value": rate, "unit": "env-steps/s", "n_gpus": 1,
@@ -530,7 +536,9 @@ def run_adjoint(args):
         "data": "synthetic (workload state after 8 replayed steps, random actions)",
         "config": {"workload": w["name"], "n_envs": n, "window": T,
                    "substeps": int(w["substeps"]), "l2": "flushed between timed steps"},
-        "roofline": {"bound": "alu", "kernel": "k_adjoint", "achieved": achieved, "peak": peak,
+        "roofline": {"bound": "alu",
+                     "kernel": "k_paper_adjoint" if W.is_paper(w) else "k_adjoint",
+                     "achieved": achieved, "peak": peak,
                      "unit": "TFLOP/s", "frac": None if achieved is None else achieved / peak,
                      "traffic": None,
                      "peak_source": f"FP32 FMA, 152 SMs x 128 lanes at {mhz:.0f} MHz",
