@@ -1516,6 +1516,49 @@ void oracle_paper_adjoint_window(const PaperModel* m, int n, const uint32_t* env
   }
 }
 
+// SHAC's closed-loop window on the paper model: policy 12 -> H -> H -> 12
+// (means and log-stds of the 6 wrench commands) acting with the first six
+// action normals, the value network at the final observation; J and its
+// derivative along the policy-weight direction dpol, in Dual.
+void oracle_paper_shac_window(const PaperModel* m, const float* pol_w, const double* dpol,
+                              const float* val_w, int n, const uint32_t* env_ids,
+                              const double* st, const double* pr, const int32_t* t_ep,
+                              const uint32_t* ep, uint64_t t_g0, int T, const double* coef,
+                              double coef_V, double* J, double* dJ) {
+  for (int i = 0; i < n; ++i) {
+    PaperEnv<Dual> e;
+    paper_load<Dual>(st, pr, t_ep, ep, n, i, e);
+    Dual obj = 0.0;
+    for (int t = 0; t < T; ++t) {
+      Dual o[kPObs], y[2 * kPAct], a[kPAct];
+      paper_observe(e, o);
+      mlp_dual(pol_w, dpol, kPObs, m->hidden, 2 * kPAct, o, y);
+      uint32_t w[8];
+      draw_words(env_ids[i], m->seed, t_g0 + (uint64_t)t, 0u, 2, w);
+      float u[8];
+      for (int k = 0; k < 8; ++k) u[k] = word_to_uniform(w[k]);
+      double eps[8];
+      box_muller8(u, eps);
+      for (int k = 0; k < kPAct; ++k) {
+        Dual ls = y[kPAct + k];
+        if (ls < Dual(m->logstd_min)) ls = Dual(m->logstd_min);
+        if (ls > Dual(m->logstd_max)) ls = Dual(m->logstd_max);
+        a[k] = y[k] + exp(ls) * Dual(eps[k]);
+      }
+      uint8_t d;
+      obj += Dual(coef[t]) * paper_control_step(*m, env_ids[i], e, a, &d);
+    }
+    if (val_w) {
+      Dual o[kPObs], v[1];
+      paper_observe(e, o);
+      mlp_dual(val_w, nullptr, kPObs, m->hidden, 1, o, v);
+      obj += Dual(coef_V) * v[0];
+    }
+    J[i] = obj.v;
+    dJ[i] = obj.d;
+  }
+}
+
 void oracle_paper_replay(const PaperModel* m, int precision, int n, const uint32_t* env_ids,
                          double* st, double* pr, int32_t* t_ep, uint32_t* ep, int T,
                          const float* act, double* rew, uint8_t* done, double* trace) {

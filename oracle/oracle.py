@@ -374,6 +374,8 @@ def _paper_lib():
         L.oracle_paper_integrate.argtypes = [P, C.c_int, P, P, P, C.c_double, C.c_int]
         L.oracle_paper_adjoint_window.argtypes = [P, C.c_int, P, P, P, P, P, C.c_int, P, P, P,
                                                   P, P, P, P]
+        L.oracle_paper_shac_window.argtypes = [P, P, P, P, C.c_int, P, P, P, P, P, C.c_uint64,
+                                               C.c_int, P, C.c_double, P, P]
         assert L.oracle_paper_model_size() == C.sizeof(PaperModel), "PaperModel layout mismatch"
         L._paper_ready = True
     return L
@@ -473,6 +475,25 @@ def paper_adjoint_window(m: PaperModel, batch: PaperBatch, actions, coef, lam_T,
                                              _p(batch.params), _p(batch.t_ep),
                                              _p(batch.episode), T, _p(act), _p(coef), _p(lam),
                                              _p(ds0), _p(da), _p(J), _p(dJ))
+    return J, dJ
+
+
+def paper_shac_window(m: PaperModel, batch: PaperBatch, pol_w, dpol, val_w, t_g0: int, T: int,
+                      coef, coef_V: float):
+    """SHAC's closed-loop window on the paper model (policy head 12) and its
+    derivative along the policy-weight direction dpol (or None)."""
+    pw = np.ascontiguousarray(pol_w, dtype=np.float32)
+    dp = None if dpol is None else np.ascontiguousarray(dpol, dtype=np.float64)
+    vw = None if val_w is None else np.ascontiguousarray(val_w, dtype=np.float32)
+    coef = np.ascontiguousarray(coef, dtype=np.float64)
+    assert coef.shape == (T,) and m.policy_out == 12
+    n = batch.n
+    J = np.zeros(n)
+    dJ = np.zeros(n)
+    _paper_lib().oracle_paper_shac_window(C.byref(m), _p(pw), _p(dp), _p(vw), n,
+                                          _p(batch.env_ids), _p(batch.state), _p(batch.params),
+                                          _p(batch.t_ep), _p(batch.episode), t_g0, T, _p(coef),
+                                          float(coef_V), _p(J), _p(dJ))
     return J, dJ
 
 

@@ -259,3 +259,36 @@ def test_paper_action_reaches_later_rewards_through_the_history():
     m0 = O.paper_model(dict(w, w_mavg=0.0))
     _, without = O.paper_adjoint_window(m0, b, act, coef, None, np.zeros((61, n)), da)
     assert np.all(np.abs(with_hist - without) > 1e-8)
+
+
+def test_paper_shac_window_value_and_derivative():
+    """The paper model's closed-loop window: its value equals the oracle's
+    own paper rollout, and its weight derivative matches central differences
+    (smooth policy: small means, sigma = e^-3)."""
+    T, n, H = 5, 3, 16
+    w = W.workload("paper_tiny", n_envs=n, hidden=H, policy_out=12, mlp="fp32", mavg_len=3,
+                   substeps=2)
+    m = O.paper_model(w)
+    b = O.PaperBatch(np.arange(n) + 5)
+    O.paper_reset(m, b)
+    O.paper_replay(m, b, W.replay_actions(3, 4, n, scale=0.8, act=6))
+    pw = W.policy_weights(w).astype(np.float64)
+    o3 = H * 12 + H + H * H + H
+    W3 = pw[o3:o3 + 12 * H].reshape(12, H)
+    W3[:6] *= 0.15
+    W3[6:] *= 0.1
+    pw[o3 + 12 * H + 6:o3 + 12 * H + 12] = -3.0
+    pw = pw.astype(np.float32)
+    coef = np.random.default_rng(4).uniform(0.5, 1.5, T)
+    J, _ = O.paper_shac_window(m, b, pw, None, None, 50, T, coef, 0.0)
+    ref = O.paper_rollout(m, b.copy(), pw, None, 50, T)
+    assert np.allclose(J, coef @ ref["rew"], rtol=1e-12, atol=1e-12)
+    vw = W.value_weights(w, 0.1)
+    d = np.random.default_rng(5).normal(size=pw.size) * np.abs(pw).mean()
+    _, dJ = O.paper_shac_window(m, b, pw, d, vw, 50, T, coef, 0.7)
+    h = 2e-3
+    Jp, _ = O.paper_shac_window(m, b, (pw + h * d).astype(np.float32), None, vw, 50, T, coef, 0.7)
+    Jm, _ = O.paper_shac_window(m, b, (pw - h * d).astype(np.float32), None, vw, 50, T, coef, 0.7)
+    fd = (Jp - Jm) / (2 * h)
+    assert np.all(np.abs(dJ) > 1e-5)
+    assert np.all(np.abs(dJ - fd) <= 3e-4 * np.abs(fd) + 3e-5 * np.abs(fd).max()), (dJ, fd)
