@@ -530,7 +530,8 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
  * env_shac_window: SHAC's actor gradient over one window in closed loop
  * (paper §III-A: short-horizon actor-critic; Xu et al. 2022).  From each
  * env's current state the policy `policy` (env_set_weights layout,
- * 18 -> hidden -> hidden -> 16: mean and log-std of the 8 commands) acts for
+ * obs -> hidden -> hidden -> 2A: means and log-stds of the A commands; the
+ * Fossen model 18 -> .. -> 16, the paper model 12 -> .. -> 12) acts for
  * T steps with the reparameterised action a = mu + exp(clamp(ls)) eps (eps:
  * the rollout's action noise at the env's global steps), and the env
  * advances (state, counters, global step += T).  With the critic `value`
@@ -541,7 +542,7 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
  * back-propagation through the dynamics, the policy network and the
  * observation.  Gradients stop at the window's start and at episode ends
  * inside it (the state after an end is a reset draw).  Optional outputs:
- * J_out [N] each env's J; obs_out [T][18][N] the observation of each step
+ * J_out [N] each env's J; obs_out [T][obs][N] the observation of each step
  * (the rollout's layout: with rew_out, done_out [T][N], env_value and
  * env_gae it gives the critic's TD(lambda) targets); device or mapped
  * page-locked host memory for J_out, rew_out, done_out, device memory for
@@ -549,7 +550,8 @@ int env_adjoint(auv_env* env, int T, const float* act, const float* coef, const 
  * precision: AUV_PPO_FP32 (network products on the CUDA cores in fp32) or
  * AUV_PPO_TF32 (on the tensor cores, tf32 operands, fp32 sums); the physics
  * and its adjoint are fp32 either way.
- * Fossen model, 1 <= T <= AUV_ADJOINT_MAX_T, at most
+ * Either model (the paper model's adjoint carries its action-history rows
+ * between steps, as env_adjoint's does); 1 <= T <= AUV_ADJOINT_MAX_T, at most
  * AUV_ADJOINT_MAX_SUBSTEPS substeps, hidden a multiple of 8 up to 1024.
  * The first call at a given (N, T) allocates the window's workspace
  * (activations of every step: about T N (2 hidden + 80) floats).

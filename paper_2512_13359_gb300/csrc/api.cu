@@ -722,8 +722,6 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
   if (!env) return AUV_ERR_INVALID;
   int rc = check_device(env);
   if (rc) return rc;
-  if (is_paper(&env->cfg))
-    return fail(env, AUV_ERR_UNSUPPORTED, "the SHAC window is built for the Fossen model");
   if (T < 1 || T > AUV_ADJOINT_MAX_T)
     return fail(env, AUV_ERR_INVALID, "T outside [1, %d]", AUV_ADJOINT_MAX_T);
   if (env->model.substeps > AUV_ADJOINT_MAX_SUBSTEPS)
@@ -747,7 +745,7 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
       (rc = map_output(env, done_out, "done_out", 1, &done)))
     return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const auv::shac::Layout L = auv::shac::layout(env->model.n, T, H);
+  const auv::shac::Layout L = auv::shac::layout(env->model.n, T, H, is_paper(&env->cfg));
   if (!env->blas) {
     cublasStatus_t bs = cublasCreate(&env->blas);
     if (bs != CUBLAS_STATUS_SUCCESS) {

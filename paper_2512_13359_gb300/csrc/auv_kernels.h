@@ -69,11 +69,14 @@ cudaError_t launch_adjoint(const Model& M, const Buffers& B, const float* act, i
 namespace shac {
 struct Layout {
   int n, T, H, Dp, Hp;
+  int D, out, S;     // network input, policy head width, adjoint rows (model)
   size_t n_aug_p, n_aug_v;
   size_t o_X, o_H1, o_H2, o_Y, o_G, o_GX, o_gY, o_lam, o_done, o_rew, o_VH1, o_VH2, o_V, o_gYv,
       o_wp, o_wv, o_gp, o_sc, bytes;
 };
-Layout layout(int n, int T, int H);
+// paper: the paper model (input 12, head 12, 61 adjoint rows), else Fossen
+// (18, 16, 13).
+Layout layout(int n, int T, int H, bool paper);
 cudaError_t init(const Layout& L, char* base, cudaStream_t s);
 // blas: a cublasHandle_t.  Returns AUV_OK or an AUV_ERR_* code with err set.
 int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,

@@ -766,6 +766,111 @@ __device__ void paper_substep_vjp(const Model& M, const paper::Env& e, const X& 
   }
 }
 
+// Save the step's input (x, goal, g, t_ep and the mean of the history rows of
+// st) to the step scratch sc [28][n].
+__device__ __forceinline__ void paper_save_step(const Model& M, const paper::Env& e,
+                                                const float* st, float* sc, size_t n, int i) {
+  float mean[6];
+  const float inv_k = 1.0f / (float)M.mavg_len;
+#pragma unroll
+  for (int k = 0; k < 6; ++k) {
+    float sum = 0.0f;
+    for (int j = 0; j < M.mavg_len; ++j) sum += st[(13 + 6 * j + k) * n + i];
+    mean[k] = sum * inv_k;
+  }
+  const float v[kPScratchF] = {e.p[0], e.p[1], e.p[2], e.q[0], e.q[1], e.q[2], e.q[3],
+                               e.nu[0], e.nu[1], e.nu[2], e.nu[3], e.nu[4], e.nu[5],
+                               e.pd[0], e.pd[1], e.pd[2], e.qd[0], e.qd[1], e.qd[2], e.qd[3],
+                               e.g, __int_as_float(e.t_ep), mean[0], mean[1], mean[2], mean[3],
+                               mean[4], mean[5]};
+#pragma unroll
+  for (int k = 0; k < kPScratchF; ++k) sc[k * n + i] = v[k];
+}
+
+__device__ __forceinline__ void paper_load_step(const float* sc, size_t n, int i, paper::Env& e,
+                                                int* t_ep, float mean[6]) {
+  float v[kPScratchF];
+#pragma unroll
+  for (int k = 0; k < kPScratchF; ++k) v[k] = sc[k * n + i];
+#pragma unroll
+  for (int k = 0; k < 3; ++k) { e.p[k] = v[k]; e.pd[k] = v[13 + k]; }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) { e.q[k] = v[3 + k]; e.qd[k] = v[16 + k]; }
+#pragma unroll
+  for (int k = 0; k < 6; ++k) { e.nu[k] = v[7 + k]; mean[k] = v[22 + k]; }
+  e.g = v[20];
+  *t_ep = __float_as_int(v[21]);
+}
+
+// Backward of one paper-model control step taken from the input saved in sc
+// with actions a: on entry (lx, lh) = dJ/d(post-step state) (the reset cut
+// already applied), on exit dJ/d(pre-step state); la = dJ/da (zero where the
+// command saturates).
+__device__ void paper_step_vjp(const Model& M, const float* sc, size_t n, int i,
+                               const float a[paper::kAct], float coef, X& lx,
+                               float (&lh)[paper::kHist][6], float la[paper::kAct]) {
+  const int K = M.mavg_len;
+  const float inv_k = 1.0f / (float)K;
+  paper::Env es;
+  int t_ep;
+  float mean[6];
+  paper_load_step(sc, n, i, es, &t_ep, mean);
+  float a_c[paper::kAct], tau[6];
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k) a_c[k] = fminf(fmaxf(a[k], -1.0f), 1.0f);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    tau[k] = M.f_max * a_c[k];
+    tau[3 + k] = M.tau_max * a_c[3 + k];
+  }
+  X xs[8];
+  for (int s = 0; s < M.substeps; ++s) {
+#pragma unroll
+    for (int k = 0; k < 3; ++k) xs[s].p[k] = es.p[k];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) xs[s].q[k] = es.q[k];
+#pragma unroll
+    for (int k = 0; k < 6; ++k) xs[s].nu[k] = es.nu[k];
+    paper::substep(M, es, tau);
+  }
+  // the history slot written after this step's reward held a_c
+  const int slot = t_ep % K;
+#pragma unroll
+  for (int k = 0; k < 6; ++k) {
+    la[k] = lh[slot][k];
+    lh[slot][k] = 0.0f;
+  }
+  // reward on the post-step state
+  float o[paper::kObs], lo[paper::kObs];
+  paper::observe(es, o);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    lo[k] = -coef * M.w_pos * 2.0f * M.w_axes[k] * M.w_axes[k] * o[k];
+    lo[3 + k] = -coef * M.w_att * 2.0f * o[3 + k];
+    lo[6 + k] = 0.0f;
+    lo[9 + k] = -coef * M.w_vel * 2.0f * o[9 + k];
+    la[3 + k] += -coef * M.w_act * 2.0f * a_c[3 + k];
+  }
+  paper_obs_vjp(es, lo, lx);
+#pragma unroll
+  for (int k = 0; k < 6; ++k) {
+    const float dk = a_c[k] - mean[k];
+    la[k] += -coef * M.w_mavg * 2.0f * dk;
+    const float lm = coef * M.w_mavg * 2.0f * dk * inv_k;
+    for (int j = 0; j < K; ++j) lh[j][k] += lm;
+  }
+  float ltau[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int s = M.substeps - 1; s >= 0; --s) paper_substep_vjp(M, es, xs[s], tau, lx, ltau);
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    la[k] += M.f_max * ltau[k];
+    la[3 + k] += M.tau_max * ltau[3 + k];
+  }
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k)
+    if (!(a[k] >= -1.0f && a[k] <= 1.0f)) la[k] = 0.0f;
+}
+
 __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
     const Model M, Buffers B, const float* __restrict__ act, int T,
     const float* __restrict__ coef, const float* __restrict__ lam_T, float* __restrict__ g_act,
@@ -776,29 +881,13 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
   if (i >= M.n) return;
   const size_t n = (size_t)M.n;
   const uint32_t id = M.id_base + (uint32_t)i;
-  const int K = M.mavg_len;
-  const float inv_k = 1.0f / (float)K;
   float* hsc = scratch + (size_t)T * kPScratchF * n;    // [61][n]: rows 13.. the history
   paper::Env e;
   paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   for (int r = 13; r < paper::kStateF; ++r) hsc[r * n + i] = B.state[r * n + i];
   uint64_t ends = 0;
   for (int t = 0; t < T; ++t) {
-    float mean[6];
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      float sum = 0.0f;
-      for (int j = 0; j < K; ++j) sum += hsc[(13 + 6 * j + k) * n + i];
-      mean[k] = sum * inv_k;
-    }
-    float* sc = scratch + (size_t)t * kPScratchF * n;
-    const float v[kPScratchF] = {e.p[0], e.p[1], e.p[2], e.q[0], e.q[1], e.q[2], e.q[3],
-                                 e.nu[0], e.nu[1], e.nu[2], e.nu[3], e.nu[4], e.nu[5],
-                                 e.pd[0], e.pd[1], e.pd[2], e.qd[0], e.qd[1], e.qd[2], e.qd[3],
-                                 e.g, __int_as_float(e.t_ep), mean[0], mean[1], mean[2], mean[3],
-                                 mean[4], mean[5]};
-#pragma unroll
-    for (int k = 0; k < kPScratchF; ++k) sc[k * n + i] = v[k];
+    paper_save_step(M, e, hsc, scratch + (size_t)t * kPScratchF * n, n, i);
     float a[paper::kAct];
 #pragma unroll
     for (int k = 0; k < paper::kAct; ++k) a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
@@ -820,7 +909,6 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
   for (int j = 0; j < paper::kHist; ++j)
 #pragma unroll
     for (int k = 0; k < 6; ++k) lh[j][k] = lam_T ? __ldg(lam_T + (13 + 6 * j + k) * n + i) : 0.0f;
-  X xs[8];
   for (int t = T - 1; t >= 0; --t) {
     if ((ends >> t) & 1ull) {
 #pragma unroll
@@ -833,76 +921,13 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
 #pragma unroll
         for (int k = 0; k < 6; ++k) lh[j][k] = 0.f;
     }
-    const float* sc = scratch + (size_t)t * kPScratchF * n;
-    float v[kPScratchF];
+    float a[paper::kAct], la[paper::kAct];
 #pragma unroll
-    for (int k = 0; k < kPScratchF; ++k) v[k] = sc[k * n + i];
-    paper::Env es;
-#pragma unroll
-    for (int k = 0; k < 3; ++k) { es.p[k] = v[k]; es.pd[k] = v[13 + k]; }
-#pragma unroll
-    for (int k = 0; k < 4; ++k) { es.q[k] = v[3 + k]; es.qd[k] = v[16 + k]; }
-#pragma unroll
-    for (int k = 0; k < 6; ++k) es.nu[k] = v[7 + k];
-    es.g = v[20];
-    const int t_ep = __float_as_int(v[21]);
-    float a[paper::kAct], a_c[paper::kAct], tau[6], la[paper::kAct];
-#pragma unroll
-    for (int k = 0; k < paper::kAct; ++k) {
-      a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
-      a_c[k] = fminf(fmaxf(a[k], -1.0f), 1.0f);
-    }
-#pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      tau[k] = M.f_max * a_c[k];
-      tau[3 + k] = M.tau_max * a_c[3 + k];
-    }
-    for (int s = 0; s < M.substeps; ++s) {
-#pragma unroll
-      for (int k = 0; k < 3; ++k) xs[s].p[k] = es.p[k];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) xs[s].q[k] = es.q[k];
-#pragma unroll
-      for (int k = 0; k < 6; ++k) xs[s].nu[k] = es.nu[k];
-      paper::substep(M, es, tau);
-    }
-    // the history slot written after this step's reward held a_c
-    const int slot = t_ep % K;
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      la[k] = lh[slot][k];
-      lh[slot][k] = 0.0f;
-    }
-    // reward on the post-step state
-    const float c = __ldg(coef + t);
-    float o[paper::kObs], lo[paper::kObs];
-    paper::observe(es, o);
-#pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      lo[k] = -c * M.w_pos * 2.0f * M.w_axes[k] * M.w_axes[k] * o[k];
-      lo[3 + k] = -c * M.w_att * 2.0f * o[3 + k];
-      lo[6 + k] = 0.0f;
-      lo[9 + k] = -c * M.w_vel * 2.0f * o[9 + k];
-      la[3 + k] += -c * M.w_act * 2.0f * a_c[3 + k];
-    }
-    paper_obs_vjp(es, lo, lx);
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      const float dk = a_c[k] - v[22 + k];
-      la[k] += -c * M.w_mavg * 2.0f * dk;
-      const float lm = c * M.w_mavg * 2.0f * dk * inv_k;
-      for (int j = 0; j < K; ++j) lh[j][k] += lm;
-    }
-    float ltau[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int s = M.substeps - 1; s >= 0; --s) paper_substep_vjp(M, es, xs[s], tau, lx, ltau);
-#pragma unroll
-    for (int k = 0; k < 3; ++k) {
-      la[k] += M.f_max * ltau[k];
-      la[3 + k] += M.tau_max * ltau[3 + k];
-    }
+    for (int k = 0; k < paper::kAct; ++k) a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
+    paper_step_vjp(M, scratch + (size_t)t * kPScratchF * n, n, i, a, __ldg(coef + t), lx, lh, la);
 #pragma unroll
     for (int k = 0; k < paper::kAct; ++k)
-      g_act[((size_t)t * paper::kAct + k) * n + i] = (a[k] >= -1.0f && a[k] <= 1.0f) ? la[k] : 0.0f;
+      g_act[((size_t)t * paper::kAct + k) * n + i] = la[k];
   }
   float s = 0.0f;
 #pragma unroll
@@ -925,6 +950,139 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
   }
 }
 
+// ---- SHAC in closed loop on the paper model ----
+
+// Observation row (12 + the constant 1, zeros up to ldx) of each env's state;
+// with sc, the step's scratch (its history mean from the env's state rows).
+__global__ void __launch_bounds__(kAdjThreads) k_shac_obs_paper(const Model M, Buffers B,
+                                                                float* __restrict__ sc,
+                                                                float* __restrict__ X, int ldx,
+                                                                float* __restrict__ obs_fm,
+                                                                int t) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  paper::Env e;
+  paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  if (sc) paper_save_step(M, e, B.state, sc, (size_t)M.n, i);
+  float o[paper::kObs];
+  paper::observe(e, o);
+  float* x = X + (size_t)i * ldx;
+#pragma unroll
+  for (int k = 0; k < paper::kObs; ++k) x[k] = o[k];
+  x[paper::kObs] = 1.0f;
+  for (int k = paper::kObs + 1; k < ldx; ++k) x[k] = 0.0f;
+  if (obs_fm) {
+#pragma unroll
+    for (int k = 0; k < paper::kObs; ++k) obs_fm[((size_t)t * paper::kObs + k) * M.n + i] = o[k];
+  }
+}
+
+// a = mu + exp(clamp(ls)) eps for the 6 wrench commands (eps: the first six
+// action normals).
+__device__ __forceinline__ void paper_shac_action(const Model& M, const float* __restrict__ y,
+                                                  const float eps[8], float a[paper::kAct],
+                                                  float sig[paper::kAct], bool in[paper::kAct]) {
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k) {
+    const float raw = y[paper::kAct + k];
+    in[k] = raw >= M.logstd_min && raw <= M.logstd_max;
+    sig[k] = expf(fminf(fmaxf(raw, M.logstd_min), M.logstd_max));
+    a[k] = fmaf(sig[k], eps[k], y[k]);
+  }
+}
+
+__global__ void __launch_bounds__(kAdjThreads) k_shac_step_paper(const Model M, Buffers B,
+                                                                 const float* __restrict__ Y,
+                                                                 int ldy, uint64_t t_g,
+                                                                 float* __restrict__ rew,
+                                                                 uint8_t* __restrict__ done,
+                                                                 Status* st) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  paper::Env e;
+  paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  const uint32_t id = M.id_base + (uint32_t)i;
+  float eps[8], a[paper::kAct], sig[paper::kAct];
+  bool in[paper::kAct];
+  action_noise(id, M.seed, t_g, eps);
+  paper_shac_action(M, Y + (size_t)i * ldy, eps, a, sig, in);
+  bool d;
+  const float r = paper::physics_step(M, id, e, a, B.state, i, &d);
+  if (!paper::env_finite(e)) flag_nan(st, i);
+  paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  rew[i] = r;
+  done[i] = d ? 1 : 0;
+}
+
+// Backward of one closed-loop paper step: lam [61][N] (rows 0..12 the pose
+// and velocity, 13.. the history) from post- to pre-step, head gradient gY.
+__global__ void __launch_bounds__(kAdjThreads) k_shac_bwd_paper(
+    const Model M, const float* __restrict__ sc, const float* __restrict__ Y, int ldy,
+    const uint8_t* __restrict__ done, uint64_t t_g, const float* __restrict__ coef,
+    float* __restrict__ lam, float* __restrict__ gY) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  const size_t n = (size_t)M.n;
+  const uint32_t id = M.id_base + (uint32_t)i;
+  X lx;
+  float lh[paper::kHist][6];
+  const bool cut = done[i] != 0;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lx.p[k] = cut ? 0.f : lam[k * n + i];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lx.q[k] = cut ? 0.f : lam[(3 + k) * n + i];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lx.nu[k] = cut ? 0.f : lam[(7 + k) * n + i];
+  for (int j = 0; j < paper::kHist; ++j)
+#pragma unroll
+    for (int k = 0; k < 6; ++k) lh[j][k] = cut ? 0.f : lam[(13 + 6 * j + k) * n + i];
+  float eps[8], a[paper::kAct], sig[paper::kAct], la[paper::kAct];
+  bool in[paper::kAct];
+  action_noise(id, M.seed, t_g, eps);
+  paper_shac_action(M, Y + (size_t)i * ldy, eps, a, sig, in);
+  paper_step_vjp(M, sc, n, i, a, __ldg(coef), lx, lh, la);
+  float* g = gY + (size_t)i * ldy;
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k) {
+    g[k] = la[k];
+    g[paper::kAct + k] = in[k] ? la[k] * sig[k] * eps[k] : 0.0f;
+  }
+#pragma unroll
+  for (int k = 0; k < 3; ++k) lam[k * n + i] = lx.p[k];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) lam[(3 + k) * n + i] = lx.q[k];
+#pragma unroll
+  for (int k = 0; k < 6; ++k) lam[(7 + k) * n + i] = lx.nu[k];
+  for (int j = 0; j < paper::kHist; ++j)
+#pragma unroll
+    for (int k = 0; k < 6; ++k) lam[(13 + 6 * j + k) * n + i] = lh[j][k];
+}
+
+// lam (rows 0..12) += (d obs / d state)^T gX at the step's input (sc) or at
+// the env's current state (sc NULL).
+__global__ void __launch_bounds__(kAdjThreads) k_shac_obs_vjp_paper(
+    const Model M, Buffers B, const float* __restrict__ sc, const float* __restrict__ gX,
+    int ldx, float* __restrict__ lam) {
+  const int i = blockIdx.x * kAdjThreads + threadIdx.x;
+  if (i >= M.n) return;
+  const size_t n = (size_t)M.n;
+  paper::Env e;
+  if (sc) {
+    int t_ep;
+    float mean[6];
+    paper_load_step(sc, n, i, e, &t_ep, mean);
+  } else {
+    paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  }
+  float lo[paper::kObs];
+#pragma unroll
+  for (int k = 0; k < paper::kObs; ++k) lo[k] = gX[(size_t)i * ldx + k];
+  X lx;
+  load_lam(lam, n, i, lx);
+  paper_obs_vjp(e, lo, lx);
+  store_lam(lam, n, i, lx);
+}
+
 }  // namespace
 
 size_t adjoint_step_floats(int n) { return (size_t)kScratchF * (size_t)n; }
@@ -940,26 +1098,38 @@ static unsigned blocks(int n) { return (n + kAdjThreads - 1) / kAdjThreads; }
 
 cudaError_t launch_obs(const Model& M, const Buffers& B, float* sc, float* X, int ldx,
                        float* obs_fm, int t, cudaStream_t s) {
-  k_shac_obs<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx, obs_fm, t);
+  if (M.model == 1)
+    k_shac_obs_paper<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx, obs_fm, t);
+  else
+    k_shac_obs<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, X, ldx, obs_fm, t);
   return cudaGetLastError();
 }
 
 cudaError_t launch_step(const Model& M, const Buffers& B, const float* Y, int ldy, uint64_t t_g,
                         float* rew, uint8_t* done, Status* st, cudaStream_t s) {
-  k_shac_step<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, Y, ldy, t_g, rew, done, st);
+  if (M.model == 1)
+    k_shac_step_paper<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, Y, ldy, t_g, rew, done, st);
+  else
+    k_shac_step<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, Y, ldy, t_g, rew, done, st);
   return cudaGetLastError();
 }
 
 cudaError_t launch_bwd(const Model& M, const float* sc, const float* Y, int ldy,
                        const uint8_t* done, uint64_t t_g, const float* coef, float* lam,
                        float* gY, cudaStream_t s) {
-  k_shac_bwd<<<blocks(M.n), kAdjThreads, 0, s>>>(M, sc, Y, ldy, done, t_g, coef, lam, gY);
+  if (M.model == 1)
+    k_shac_bwd_paper<<<blocks(M.n), kAdjThreads, 0, s>>>(M, sc, Y, ldy, done, t_g, coef, lam, gY);
+  else
+    k_shac_bwd<<<blocks(M.n), kAdjThreads, 0, s>>>(M, sc, Y, ldy, done, t_g, coef, lam, gY);
   return cudaGetLastError();
 }
 
 cudaError_t launch_obs_vjp(const Model& M, const Buffers& B, const float* sc, const float* gX,
                            int ldx, float* lam, cudaStream_t s) {
-  k_shac_obs_vjp<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, gX, ldx, lam);
+  if (M.model == 1)
+    k_shac_obs_vjp_paper<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, gX, ldx, lam);
+  else
+    k_shac_obs_vjp<<<blocks(M.n), kAdjThreads, 0, s>>>(M, B, sc, gX, ldx, lam);
   return cudaGetLastError();
 }
 

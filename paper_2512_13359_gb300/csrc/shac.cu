@@ -22,6 +22,7 @@
 
 #include "auv_kernels.h"
 #include "auvenv.h"
+#include "paper_device.cuh"
 
 namespace auv {
 namespace shac {
@@ -42,20 +43,23 @@ struct Gemm {
   }
 };
 
-constexpr int kLdy = 16;   // policy head row (2 x 8)
+constexpr int kLdy = 16;   // policy head row (2 x 8, or 2 x 6 padded)
 constexpr int kLdv = 8;    // value head row
 
 }  // namespace
 
-Layout layout(int n, int T, int H) {
+Layout layout(int n, int T, int H, bool paper) {
   Layout L;
   L.n = n;
   L.T = T;
   L.H = H;
-  L.Dp = round8(kObs + 1);
+  L.D = paper ? paper::kObs : kObs;
+  L.out = 2 * (paper ? paper::kAct : kAct);
+  L.S = paper ? paper::kStateF : 13;
+  L.Dp = round8(L.D + 1);
   L.Hp = round8(H + 1);
-  L.n_aug_p = ppo::aug_count(kObs, L.Dp, H, L.Hp, 2 * kAct);
-  L.n_aug_v = ppo::aug_count(kObs, L.Dp, H, L.Hp, 1);
+  L.n_aug_p = ppo::aug_count(L.D, L.Dp, H, L.Hp, L.out);
+  L.n_aug_v = ppo::aug_count(L.D, L.Dp, H, L.Hp, 1);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -70,7 +74,7 @@ Layout layout(int n, int T, int H) {
   L.o_G = take(N * H * 4);
   L.o_GX = take(N * L.Dp * 4);
   L.o_gY = take(N * kLdy * 4);
-  L.o_lam = take(13 * N * 4);
+  L.o_lam = take((size_t)L.S * N * 4);
   L.o_done = take(T * N);
   L.o_rew = take(T * N * 4);
   L.o_VH1 = take(N * L.Hp * 4);
@@ -136,10 +140,11 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   const auto T_ = CUBLAS_OP_T, N_ = CUBLAS_OP_N;
 
   // weights into the augmented layout; gradient accumulator to zero
-  if ((e = ppo::launch_convert(const_cast<float*>(policy), wp, kObs, Dp, H, Hp, 2 * kAct, true, s)))
+  const int D = L.D, out = L.out;
+  if ((e = ppo::launch_convert(const_cast<float*>(policy), wp, D, Dp, H, Hp, out, true, s)))
     return cfail(e, "policy weights");
   if (value &&
-      (e = ppo::launch_convert(const_cast<float*>(value), wv, kObs, Dp, H, Hp, 1, true, s)))
+      (e = ppo::launch_convert(const_cast<float*>(value), wv, D, Dp, H, Hp, 1, true, s)))
     return cfail(e, "value weights");
   if ((e = cudaMemsetAsync(gp, 0, L.n_aug_p * 4, s))) return cfail(e, "clear gradient");
 
@@ -150,13 +155,13 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
     if ((e = ppo::launch_tanh_fwd(false, H1s(t), Hp, n, H, s))) return cfail(e, "tanh");
     if ((bs = gemm(T_, N_, H, n, Hp, w2, Hp, H1s(t), Hp, H2s(t), Hp))) return bfail(bs, "policy 2");
     if ((e = ppo::launch_tanh_fwd(false, H2s(t), Hp, n, H, s))) return cfail(e, "tanh");
-    if ((bs = gemm(T_, N_, 2 * kAct, n, Hp, w3, Hp, H2s(t), Hp, Ys(t), kLdy)))
+    if ((bs = gemm(T_, N_, out, n, Hp, w3, Hp, H2s(t), Hp, Ys(t), kLdy)))
       return bfail(bs, "policy 3");
     if ((e = launch_step(M, B, Ys(t), kLdy, t_g0 + (uint64_t)t, rew + (size_t)t * N,
                          done + (size_t)t * N, st, s)))
       return cfail(e, "step");
   }
-  if ((e = cudaMemsetAsync(lam, 0, 13 * N * 4, s))) return cfail(e, "clear adjoint");
+  if ((e = cudaMemsetAsync(lam, 0, (size_t)L.S * N * 4, s))) return cfail(e, "clear adjoint");
   // ---- terminal critic: lam = coef_V dV(o(x_T))/dx_T ----
   if (value) {
     if ((e = launch_obs(M, B, nullptr, Xs(T), Dp, nullptr, 0, s))) return cfail(e, "observation");
@@ -180,9 +185,9 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
     if ((e = launch_bwd(M, SCs(t), Ys(t), kLdy, done + (size_t)t * N, t_g0 + (uint64_t)t,
                         coef + t, lam, gY, s)))
       return cfail(e, "step VJP");
-    if ((bs = gemm(N_, T_, Hp, 2 * kAct, n, H2s(t), Hp, gY, kLdy, g3, Hp, 1.0f)))
+    if ((bs = gemm(N_, T_, Hp, out, n, H2s(t), Hp, gY, kLdy, g3, Hp, 1.0f)))
       return bfail(bs, "dW3");
-    if ((bs = gemm(N_, N_, H, n, 2 * kAct, w3, Hp, gY, kLdy, G, H))) return bfail(bs, "dH2");
+    if ((bs = gemm(N_, N_, H, n, out, w3, Hp, gY, kLdy, G, H))) return bfail(bs, "dH2");
     if ((e = ppo::launch_tanh_bwd(false, G, H, H2s(t), Hp, n, H, s))) return cfail(e, "tanh'");
     if ((bs = gemm(N_, T_, Hp, H, n, H1s(t), Hp, G, H, g2, Hp, 1.0f))) return bfail(bs, "dW2");
     if ((bs = gemm(N_, N_, H, n, H, w2, Hp, G, H, H2s(t), Hp))) return bfail(bs, "dH1");
@@ -192,7 +197,7 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
     if ((bs = gemm(N_, N_, Dp, n, H, w1, Dp, H2s(t), Hp, GX, Dp))) return bfail(bs, "dX");
     if ((e = launch_obs_vjp(M, B, SCs(t), GX, Dp, lam, s))) return cfail(e, "observation VJP");
   }
-  if ((e = ppo::launch_convert(grad, gp, kObs, Dp, H, Hp, 2 * kAct, false, s)))
+  if ((e = ppo::launch_convert(grad, gp, D, Dp, H, Hp, out, false, s)))
     return cfail(e, "gradient layout");
   if (rew_out && (e = cudaMemcpyAsync(rew_out, rew, T * N * 4, cudaMemcpyDefault, s)))
     return cfail(e, "copy rewards");

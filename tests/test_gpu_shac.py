@@ -132,6 +132,61 @@ def test_shac_window_advances_like_a_replay(oracle):
     assert np.abs(st[:13] - b.state[:13]).max() <= 1e-4
 
 
+@pytest.mark.parametrize("n,T,L,smooth", [(100, 6, 500, True), (130, 10, 7, False)])
+def test_paper_shac_window_matches_dual_numbers(oracle, n, T, L, smooth):
+    """The paper model in closed loop: policy 12 -> 64 -> 64 -> 12, the
+    critic, the 61-row adjoint with the action history, episode ends."""
+    torch = need_gpu()
+    H = 64
+    w = W.workload("paper_tiny", n_envs=n, hidden=H, policy_out=12, mlp="fp32", mavg_len=3,
+                   substeps=4, dr_enable=1, g_eff=0.05, episode_len=L)
+    env = make_env(w, policy=False)
+    env.reset()
+    warm = torch.from_numpy(W.replay_actions(n, 3, n, scale=0.8, act=6)).cuda()
+    env.step_actions(warm, torch.empty((3, n), device="cuda"),
+                     torch.empty((3, n), dtype=torch.uint8, device="cuda"))
+    pw = W.policy_weights(w, 0.05).astype(np.float64)
+    if smooth:
+        o3 = H * 12 + H + H * H + H
+        W3 = pw[o3:o3 + 12 * H].reshape(12, H)
+        W3[:6] *= 0.15
+        W3[6:] *= 0.1
+        pw[o3 + 12 * H + 6:o3 + 12 * H + 12] = -3.0
+    pw = pw.astype(np.float32)
+    vw = W.value_weights(w, 0.1)
+    b = oracle.PaperBatch(np.arange(n))
+    b.state[:] = to_np(env.state)
+    b.params[:] = to_np(env.params)
+    b.t_ep[:] = to_np(env.t_ep)
+    b.episode[:] = to_np(env.episode).view(np.uint32)
+    t_g0 = env.t_g
+    coef = (0.99 ** np.arange(T) / n).astype(np.float32)
+    grad = torch.empty(pw.size, device="cuda")
+    J = torch.empty(n, device="cuda")
+    done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
+    env.shac_window(torch.from_numpy(pw).cuda(), torch.from_numpy(vw).cuda(),
+                    torch.from_numpy(coef).cuda(), 0.6 / n, grad, J=J, done=done)
+    assert env.status().code == 0
+    if L < 3 + T:
+        assert to_np(done).any()
+    m = oracle.paper_model(w)
+    g = to_np(grad).astype(np.float64)
+    rng = np.random.default_rng(n)
+    worst = 0.0
+    for k in range(3):
+        d = rng.normal(size=pw.size)
+        Jr, dJ = oracle.paper_shac_window(m, b, pw, d, vw, t_g0, T, coef, 0.6 / n)
+        if k == 0:
+            assert np.abs(to_np(J) - Jr).max() <= 1e-4 * max(np.abs(Jr).max(), 1e-6)
+        worst = max(worst, abs(g @ d - dJ.sum()) / np.abs(g * d).sum())
+    print(f"[paper shac n{n} T{T} L{L} smooth={smooth}] {worst:.3e} (tol {SHAC_TOL})")
+    assert worst <= SHAC_TOL
+    ref = oracle.paper_rollout(m, b, pw, None, t_g0, T, want=("rew",))
+    assert np.array_equal(to_np(done), ref["done"])
+    assert np.abs(to_np(env.state)[:13] - b.state[:13]).max() <= 1e-4
+    assert np.abs(to_np(env.state)[13:] - b.state[13:]).max() <= 1e-6
+
+
 def test_shac_window_rejects_bad_arguments():
     torch = need_gpu()
     from paper_2512_13359_gb300 import auvenv
@@ -148,10 +203,6 @@ def test_shac_window_rejects_bad_arguments():
     with pytest.raises(auvenv.AuvError) as ei:
         env.shac_window(pw.cpu(), None, coef[:4], 0.0, g)        # host weights
     assert ei.value.code == auvenv.AUV_ERR_SIZE
-    pe = make_env(W.workload("paper_tiny", n_envs=n), policy=False)
-    with pytest.raises(auvenv.AuvError) as ei:
-        pe.shac_window(pw, None, coef[:4], 0.0, g)
-    assert ei.value.code == auvenv.AUV_ERR_UNSUPPORTED
 
 
 def test_shac_critic_targets_and_regression(oracle):
