@@ -341,7 +341,8 @@ def run_gae(args):
         "dtype": "f32", "data": "synthetic (one rollout's rewards, dones, values)",
         "config": {"workload": w["name"], "n_envs_per_gpu": n, "rollout_steps": T,
                    "gamma": 0.99, "lambda": 0.95, "l2": "flushed between timed steps"},
-        "roofline": {"bound": "hbm", "kernel": "k_gae", "achieved": achieved,
+        "roofline": {"bound": "hbm", "kernel": "k_gae_chunked" if 8 < T <= 512 else "k_gae",
+                     "achieved": achieved,
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
                      "traffic": None, "peak_source": f"HBM copy, {src}"},
         "gpu_launches": args.steps, "clocks": clock_info,

@@ -58,13 +58,96 @@ __global__ void __launch_bounds__(256) k_gae(int n, int T, const float* __restri
   }
 }
 
+// The same recursion split over C time chunks of L <= LC steps: warp c
+// of a block runs chunk c for 32 envs (coalesced loads).  Pass one goes
+// backwards over the chunk from a zero carry and keeps only the chunk's
+// (A', P): its advantage at the chunk start given zero advantage after the
+// chunk, and the product of gamma lambda (1 - d_t) over it, so that the true
+// start value is A' + P A_next.  The block combines those in shared memory
+// to the true advantage just after each chunk, and pass two reruns the
+// chunk's recursion from it.  C times more threads than k_gae; 8-step chunks
+// keep 48 warps resident per SM, 16-step ones 32.
+template <int C, int LC>
+__global__ void __launch_bounds__(32 * C, (LC <= 8 ? 48 : 32) / C) k_gae_chunked(int n, int T, const float* __restrict__ rew,
+                                                        const uint8_t* __restrict__ done,
+                                                        const float* __restrict__ value,
+                                                        const float* __restrict__ last_value,
+                                                        float gamma, float gl,
+                                                        float* __restrict__ adv,
+                                                        float* __restrict__ ret) {
+  __shared__ float sA[C][32], sP[C][32];
+  const int lane = threadIdx.x & 31, c = threadIdx.x >> 5;
+  const int i = blockIdx.x * 32 + lane;
+  const int L = (T + C - 1) / C;
+  const int lo = c * L, hi = min(T, lo + L);
+  const size_t N = (size_t)n;
+  float dl[LC], v[LC];
+  unsigned live_bits = 0;        // bit k: step lo + k is not an episode end
+  float a = 0.0f, p = 1.0f;
+  const bool live = i < n && lo < hi;
+  if (live) {
+    float r[LC];
+    unsigned char d[LC];
+#pragma unroll
+    for (int k = 0; k < LC; ++k) {
+      if (lo + k < hi) {
+        const size_t o = (size_t)(lo + k) * N + i;
+        r[k] = __ldg(rew + o);
+        v[k] = __ldg(value + o);
+        d[k] = __ldg(done + o);
+      }
+    }
+    float v_next = hi == T ? __ldg(last_value + i) : __ldg(value + (size_t)hi * N + i);
+#pragma unroll
+    for (int k = LC - 1; k >= 0; --k) {
+      if (lo + k < hi) {
+        const float nt = d[k] ? 0.0f : 1.0f;
+        live_bits |= d[k] ? 0u : 1u << k;
+        dl[k] = fmaf(gamma * nt, v_next, r[k]) - v[k];
+        a = fmaf(gl * nt, a, dl[k]);
+        p *= gl * nt;
+        v_next = v[k];
+      }
+    }
+  }
+  sA[c][lane] = a;      // an empty chunk is the identity (0, 1)
+  sP[c][lane] = p;
+  __syncthreads();
+  if (!live) return;
+  a = 0.0f;
+  for (int c2 = C - 1; c2 > c; --c2) a = fmaf(sP[c2][lane], a, sA[c2][lane]);
+#pragma unroll
+  for (int k = LC - 1; k >= 0; --k) {
+    if (lo + k < hi) {
+      a = fmaf((live_bits >> k & 1u) ? gl : 0.0f, a, dl[k]);
+      const size_t o = (size_t)(lo + k) * N + i;
+      adv[o] = a;
+      ret[o] = a + v[k];
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, const float* value,
                        const float* last_value, float gamma, float lam, float* adv, float* ret,
                        cudaStream_t s) {
-  k_gae<<<(n + 255) / 256, 256, 0, s>>>(n, T, rew, done, value, last_value, gamma, gamma * lam,
-                                        adv, ret);
+  const float gl = gamma * lam;
+  const unsigned nb = (unsigned)((n + 31) / 32);
+#define AUV_GAE_CHUNKED(C, LC) \
+  k_gae_chunked<C, LC><<<nb, 32 * C, 0, s>>>(n, T, rew, done, value, last_value, gamma, gl, adv, ret)
+  // 8-step chunks up to T = 128 (C <= 16), 16-step ones up to T = 512
+  if (T > 8 && T <= 512) {
+    if (T <= 16) AUV_GAE_CHUNKED(2, 8);
+    else if (T <= 32) AUV_GAE_CHUNKED(4, 8);
+    else if (T <= 64) AUV_GAE_CHUNKED(8, 8);
+    else if (T <= 128) AUV_GAE_CHUNKED(16, 8);
+    else if (T <= 256) AUV_GAE_CHUNKED(16, 16);
+    else AUV_GAE_CHUNKED(32, 16);
+#undef AUV_GAE_CHUNKED
+    return cudaGetLastError();
+  }
+  k_gae<<<(n + 255) / 256, 256, 0, s>>>(n, T, rew, done, value, last_value, gamma, gl, adv, ret);
   return cudaGetLastError();
 }
 

@@ -1,7 +1,9 @@
 """GPU parity of the PPO learner's advantage estimation (env_gae) against the
 oracle's plain recursion: random trajectories with episode ends at every
-step length, block remainders of the kernel's 16-step loads (T = 1, 37,
-128), a real rollout's rewards, dones and values, and the argument checks."""
+step length; the serial kernel (T <= 8 and T > 512) and each shape of the
+chunked one (2 to 32 chunks of at most 8 or 16 steps, ragged last chunks,
+an empty trailing chunk at T = 129, env counts off the 32-env block);
+a real rollout's rewards, dones and values; and the argument checks."""
 import numpy as np
 import pytest
 
@@ -24,7 +26,11 @@ def _random_traj(seed, T, n, p_done=0.05):
 
 @pytest.mark.parametrize("T,n,gamma,lam", [(128, 65536, 0.99, 0.95), (37, 999, 0.9, 0.8),
                                            (1, 300, 0.99, 0.95), (64, 4096, 1.0, 1.0),
-                                           (20, 500, 0.99, 0.0)])
+                                           (20, 500, 0.99, 0.0), (16, 77, 0.99, 0.95),
+                                           (8, 70, 0.99, 0.95), (9, 50, 0.99, 0.95),
+                                           (17, 33, 0.99, 0.95), (129, 1000, 0.99, 0.95),
+                                           (255, 65, 0.97, 0.9), (512, 96, 0.99, 0.95),
+                                           (600, 40, 0.99, 0.95)])
 def test_gae_matches_oracle(T, n, gamma, lam):
     torch = need_gpu()
     from oracle import ppo_oracle as P
