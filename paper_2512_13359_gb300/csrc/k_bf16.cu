@@ -200,7 +200,10 @@ __device__ __forceinline__ void write_obs_row(uint8_t* tile, int r, const float 
 
 // 32 accumulator columns + bias -> tanh -> 16 bf16 pairs.  The bias is added
 // two columns per instruction (packed fp32 add, round to nearest: the same
-// sums as scalar adds).
+// sums as scalar adds).  tanh runs on the fp32 sums (tanh.approx.f32, one
+// instruction per value) and the results are rounded to a bf16 pair: three
+// instructions per pair, where the packed bf16x2 tanh costs a pack plus
+// three (two multi-function-unit operations and a merge) on sm_103.
 __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const float* bias,
                                             uint32_t (&out)[16]) {
 #pragma unroll
@@ -210,8 +213,8 @@ __device__ __forceinline__ void bias_tanh32(const uint32_t (&acc)[32], const flo
                                  make_float2(b.x, b.y));
     const float2 s1 = __fadd2_rn(make_float2(__uint_as_float(acc[2 * j + 2]), __uint_as_float(acc[2 * j + 3])),
                                  make_float2(b.z, b.w));
-    out[j] = tc::tanh_bf16x2(tc::pack_bf16x2(s0.x, s0.y));
-    out[j + 1] = tc::tanh_bf16x2(tc::pack_bf16x2(s1.x, s1.y));
+    out[j] = tc::pack_bf16x2(tc::tanh_f32(s0.x), tc::tanh_f32(s0.y));
+    out[j + 1] = tc::pack_bf16x2(tc::tanh_f32(s1.x), tc::tanh_f32(s1.y));
   }
 }
 

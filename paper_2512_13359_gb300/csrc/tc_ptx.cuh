@@ -225,9 +225,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
-__device__ __forceinline__ uint32_t tanh_bf16x2(uint32_t x) {
-  uint32_t r;
-  asm("tanh.approx.bf16x2 %0, %1;" : "=r"(r) : "r"(x));
+// tanh, hardware approximation (relative error about 2^-11).
+__device__ __forceinline__ float tanh_f32(float x) {
+  float r;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
   return r;
 }
 

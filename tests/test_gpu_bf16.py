@@ -2,12 +2,15 @@
 oracle's bf16 emulation (bf16 weights, inputs and hidden activations, exact
 accumulation, fp32 biases, exact tanh).
 
-Tolerances: the kernel evaluates tanh with the hardware bf16 tanh unit on the
-bf16-rounded pre-activation, so a hidden unit may differ from the oracle's
-correctly rounded value by up to two bf16 ulps (2^-7 relative); with
-N(0, 1/fan_in) weights these independent errors add in quadrature through
-the 256-wide layers.  BF16_HEAD_TOL bounds the resulting network-output error;
-every test reports the measured maximum next to it."""
+Tolerances: the kernel adds the fp32 bias to the fp32 accumulator, applies
+the hardware fp32 tanh (relative error about 2^-11) and rounds to bf16, so a
+hidden unit is the oracle's correctly rounded value or a neighbour of it
+when the exact value lies within 2^-11 of a rounding boundary; the inputs
+of each layer are the same bf16 values up to those flips and the
+accumulation order.  With N(0, 1/fan_in) weights these independent errors
+add in quadrature through the 256-wide layers to about 2e-3 on outputs of
+order one; BF16_HEAD_TOL (1e-2) bounds them with a margin of five.  Every
+test reports the measured maximum next to it."""
 import numpy as np
 import pytest
 
@@ -16,8 +19,8 @@ from parity_util import STATE_TOL, assert_close, make_env, need_gpu, oracle_batc
 
 pytestmark = pytest.mark.gpu
 
-BF16_HEAD_TOL = 3e-2      # absolute, network outputs of order 1
-BF16_VALUE_TOL = 3e-2
+BF16_HEAD_TOL = 1e-2      # absolute, network outputs of order 1
+BF16_VALUE_TOL = 1e-2
 
 
 def _report(name, err, tol):
@@ -60,6 +63,31 @@ def test_bf16_value_over_trajectory_layout(oracle):
         idx = np.r_[0, 1, 500, 999]
         ref = oracle.mlp(vw, 18, 256, 1, True, obs[t][:, idx].T.astype(np.float64))[:, 0]
         assert np.abs(g[t, idx] - ref).max() <= BF16_VALUE_TOL
+
+
+@pytest.mark.parametrize("name", ["ppo_65536", "paper_4096"])
+def test_bf16_value_many_tiles_per_group(oracle, name):
+    """env_value over a trajectory of 3,909 row tiles: four groups per CTA,
+    each serving 6 or 7 tiles in turn through the shared accumulators;
+    ragged N (5,003) and both observation widths (18 and 12)."""
+    torch = need_gpu()
+    n, T = 5003, 100
+    w = W.workload(name, n_envs=n)
+    d = W.obs_dim(w)
+    env = make_env(w, bias_std=0.1)
+    obs = W.random_observations(5, T * n, d).reshape(T, n, d).transpose(0, 2, 1).copy()
+    val = torch.full((T, n), float("nan"), device="cuda")
+    env.value(torch.from_numpy(obs).cuda(), val)
+    assert env.status().code == 0
+    g = to_np(val)
+    assert np.isfinite(g).all()
+    vw = W.value_weights(w, 0.1)
+    rng = np.random.default_rng(7)
+    for t in (0, 1, 37, 98, 99):
+        idx = np.unique(np.r_[0, 127, 128, n - 1, rng.integers(0, n, 60)])
+        ref = oracle.mlp(vw, d, 256, 1, True, obs[t][:, idx].T.astype(np.float64))[:, 0]
+        err = np.abs(g[t, idx] - ref).max()
+        assert err <= BF16_VALUE_TOL, f"t={t}: {err:.3e}"
 
 
 @pytest.mark.parametrize("n,T", [(65536, 128), (1048576, 4), (1000, 20), (300, 9)])
