@@ -12,8 +12,10 @@
 // integrate their environments.
 //
 // Per 128-row tile and control step:
-//   layer 1: A = observation tile (smem, K = 32 with 18 used), 4 N-chunks of 64
-//   epilogue: + b1, tanh, bf16 -> h1 written back to tensor memory
+//   layer 1: A = observation tile (smem, K = 32: the observation, zeros, and
+//            ones in columns 30 and 31, which carry b1 as a bf16 hi + lo pair
+//            in W1's columns 30 and 31), 4 N-chunks of 64
+//   epilogue: tanh, bf16 -> h1 written back to tensor memory
 //   layer 2: A = h1 from tensor memory (K = 256), 4 N-chunks of 64
 //   epilogue: + b2, tanh, bf16 -> h2 chunk in smem (policy), or the value
 //             head's dot product on CUDA cores (value)
@@ -39,9 +41,11 @@ constexpr int kChunk = 64;
 constexpr int kNChunks = kH / kChunk;
 constexpr int kHeadOut = 16;
 
-// Packed image (bytes).  W1: 256 rows x 64 B (K = 32), 64-byte swizzle.
+// Packed image (bytes).  W1: 256 rows x 64 B (K = 32: the input weights, zeros,
+// then b1 split into bf16 hi and lo parts in columns 30 and 31), 64-byte swizzle.
 // W2: 4 K-atoms x 256 rows x 128 B, 128-byte swizzle.  W3: 4 K-atoms x 16
-// rows x 128 B.  Then fp32 b1[256], b2[256] and either b3[16] (policy) or
+// rows x 128 B.  Then fp32 b1[256] (layer 1 takes its bias through W1's
+// columns 30 and 31 instead), b2[256] and either b3[16] (policy) or
 // w3[256] (bf16-rounded) and b3[1] (value).
 constexpr uint32_t kW1Bytes = kH * 64;
 constexpr uint32_t kW2Bytes = 4 * kH * 128;
@@ -80,6 +84,10 @@ __device__ __forceinline__ uint16_t bf16_bits(float x) {
   return (uint16_t)(tc::pack_bf16x2(x, 0.0f) & 0xFFFFu);
 }
 
+// Column of W1 (and of the observation tile) holding b1's bf16 high part; the
+// low part follows.  Above every network input width (<= 18).
+constexpr int kBiasCol = 30;
+
 // One thread per 16-byte piece of the W1/W2/W3 regions, then the vectors.
 // in_dim: network input width (18 or 12, <= 32); out_dim: 1 (value) or the
 // policy head width (<= 16; head rows out_dim..15 are packed as zeros).
@@ -98,9 +106,12 @@ __global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
   uint32_t off;
   if (piece < n_w1) {
     const int n = piece >> 2, p = piece & 3, q = p ^ ((n >> 1) & 3);
+    const uint16_t b_hi = bf16_bits(b1[n]);
+    const uint16_t b_lo = bf16_bits(b1[n] - __uint_as_float((uint32_t)b_hi << 16));
     for (int e = 0; e < 8; ++e) {
       const int k = 8 * q + e;
-      v[e] = k < in_dim ? bf16_bits(W1[n * in_dim + k]) : (uint16_t)0;
+      v[e] = k < in_dim ? bf16_bits(W1[n * in_dim + k])
+                        : (k == kBiasCol ? b_hi : (k == kBiasCol + 1 ? b_lo : (uint16_t)0));
     }
     off = kOffW1 + n * 64 + p * 16;
   } else if (piece < n_w1 + n_w2) {
@@ -181,21 +192,32 @@ struct Engine {
 };
 
 // Row r of the observation tile (bf16, K = 32, 64-byte swizzle): 4 pieces of
-// 16 bytes, piece q at position q ^ ((r >> 1) & 3).  Features NOBS..31 are zero.
+// 16 bytes, piece q at position q ^ ((r >> 1) & 3).  Features NOBS..29 are
+// zero, 30 and 31 one (the bias columns).
 template <int NOBS>
 __device__ __forceinline__ void write_obs_row(uint8_t* tile, int r, const float o[NOBS]) {
-  static_assert(NOBS % 2 == 0 && NOBS <= 32, "observation width");
+  static_assert(NOBS % 2 == 0 && NOBS <= kBiasCol, "observation width");
   uint32_t w[16];
 #pragma unroll
   for (int j = 0; j < NOBS / 2; ++j) w[j] = tc::pack_bf16x2(o[2 * j], o[2 * j + 1]);
 #pragma unroll
-  for (int j = NOBS / 2; j < 16; ++j) w[j] = 0u;
+  for (int j = NOBS / 2; j < 15; ++j) w[j] = 0u;
+  static_assert(kBiasCol == 30, "bias columns are the last word of the row");
+  w[15] = tc::pack_bf16x2(1.0f, 1.0f);
   const int sw = (r >> 1) & 3;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint4 v = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
     *reinterpret_cast<uint4*>(tile + r * 64 + ((q ^ sw) << 4)) = v;
   }
+}
+
+// 32 accumulator columns (bias included) -> tanh -> 16 bf16 pairs.
+__device__ __forceinline__ void tanh32(const uint32_t (&acc)[32], uint32_t (&out)[16]) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j)
+    out[j] = tc::pack_bf16x2(tc::tanh_f32(__uint_as_float(acc[2 * j])),
+                             tc::tanh_f32(__uint_as_float(acc[2 * j + 1])));
 }
 
 // 32 accumulator columns + bias -> tanh -> 16 bf16 pairs.  The bias is added
@@ -462,7 +484,6 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     uint8_t* obs_tile = smem + E::kOffObs + g * kObsTileBytes;
     uint8_t* h2_tiles = smem + E::kOffH2;
-    const float* b1 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB1P : kOffB1V));
     const float* b2 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB2P : kOffB2V));
     // Barrier phases need no counters: per group-step a group waits on its
     // full_x barrier once per chunk (4 times), on full_y and full_z twice
@@ -486,14 +507,14 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::tc_fence_before();
             tc::mbar_arrive(&bar->empty_x);
           }
-          bias_tanh32(acc, b1 + c * kChunk + 32 * half, hv);
+          tanh32(acc, hv);
           tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
         }
       }
       tc::tmem_st_wait();
       tc::tc_fence_before();
       tc::mbar_arrive(&bar->h1_full[slot]);
-      float vsum = 0.0f;
+      float2 vsum = make_float2(0.0f, 0.0f);   // value head: even and odd columns
       const float* w3v = reinterpret_cast<const float*>(smem + kOffW3V);
       for (int c = 0; c < kNChunks; ++c) {       // layer 2 (Y / Z)
         const bool odd = c & 1;
@@ -527,10 +548,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
                   make_uint4(hv[4 * q], hv[4 * q + 1], hv[4 * q + 2], hv[4 * q + 3]);
             }
           } else {
-            const float* w = w3v + c * kChunk + 32 * half;
+            const float4* w = reinterpret_cast<const float4*>(w3v + c * kChunk + 32 * half);
 #pragma unroll
-            for (int j = 0; j < 16; ++j)
-              vsum = fmaf(tc::bf16lo(hv[j]), w[2 * j], fmaf(tc::bf16hi(hv[j]), w[2 * j + 1], vsum));
+            for (int j = 0; j < 16; j += 2) {
+              const float4 wv = w[j >> 1];
+              vsum = __ffma2_rn(make_float2(tc::bf16lo(hv[j]), tc::bf16hi(hv[j])),
+                                make_float2(wv.x, wv.y), vsum);
+              vsum = __ffma2_rn(make_float2(tc::bf16lo(hv[j + 1]), tc::bf16hi(hv[j + 1])),
+                                make_float2(wv.z, wv.w), vsum);
+            }
           }
         }
         if (kPolicy) {
@@ -539,7 +565,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         }
       }
       if (!kPolicy) {
-        head[0] = vsum + *reinterpret_cast<const float*>(smem + kOffB3V);
+        head[0] = (vsum.x + vsum.y) + *reinterpret_cast<const float*>(smem + kOffB3V);
         return true;
       }
       if (!tc::mbar_wait(&bar->acc3_full[g], (uint32_t)it & 1u, abort, kWaitLimitNs)) return false;
