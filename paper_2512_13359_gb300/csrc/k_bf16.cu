@@ -155,7 +155,9 @@ __global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
 // -------------------------------------------------------------------------
 struct Barriers {
   uint64_t obs_full[4];     // group g's observation tile written (128 arrivals)
-  uint64_t full_x[4];       // layer-1 chunk of group g in X (MMA commit)
+  uint64_t full_x[4];       // layer-1 chunk 2 or 3 of group g in X (MMA commit)
+  uint64_t full_l1a[4];     // layer-1 chunk 0 of group g in its h1 slot, columns 0..63
+  uint64_t full_l1b[4];     // layer-1 chunk 1 of group g in its h1 slot, columns 64..127
   uint64_t full_y[4];       // layer-2 even chunk of group g in Y
   uint64_t full_z[4];       // layer-2 odd chunk of group g in Z
   uint64_t acc3_full[4];    // head accumulator of group g complete
@@ -306,6 +308,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     for (int g = 0; g < G; ++g) {
       tc::mbar_init(&bar->obs_full[g], kRows);
       tc::mbar_init(&bar->full_x[g], 1);
+      tc::mbar_init(&bar->full_l1a[g], 1);
+      tc::mbar_init(&bar->full_l1b[g], 1);
       tc::mbar_init(&bar->full_y[g], 1);
       tc::mbar_init(&bar->full_z[g], 1);
       tc::mbar_init(&bar->acc3_full[g], 1);
@@ -457,16 +461,24 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           ok = tc::mbar_wait(&bar->obs_full[g], (p_obs >> g) & 1u, abort, kWaitLimitNs);
           p_obs ^= 1u << g;
           const uint32_t obs_s = s_base + E::kOffObs + g * kObsTileBytes;
+          // Chunks 0 and 1 accumulate in the step's own h1 slot (free since
+          // h1_free; the epilogue overwrites it with the bf16 h1 only where
+          // it has read the accumulator), chunks 2 and 3 in X.  So three
+          // chunks start at once and only chunk 3 waits for X to drain.
           for (int c = 0; c < kNChunks && ok; ++c) {
-            ok = tc::mbar_wait(&bar->empty_x, (u_x & 1u) ^ 1u, abort, kWaitLimitNs);
-            ++u_x;
-            if (!ok) break;
+            uint32_t d = tmem + kColH1 + s1 * 128 + c * kChunk;
+            if (c >= 2) {
+              ok = tc::mbar_wait(&bar->empty_x, (u_x & 1u) ^ 1u, abort, kWaitLimitNs);
+              ++u_x;
+              if (!ok) break;
+              d = tmem + kColX;
+            }
             tc::tc_fence_after();
             const uint64_t a0 = tc::smem_desc(obs_s, 512, 4);
             const uint64_t b0 = tc::smem_desc(s_base + kOffW1 + c * kChunk * 64, 512, 4);
-            tc::mma_ss(tmem + kColX, a0, b0, kI64, 0u);
-            tc::mma_ss(tmem + kColX, a0 + 2, b0 + 2, kI64, 1u);
-            tc::mma_commit(&bar->full_x[g]);
+            tc::mma_ss(d, a0, b0, kI64, 0u);
+            tc::mma_ss(d, a0 + 2, b0 + 2, kI64, 1u);
+            tc::mma_commit(c == 0 ? &bar->full_l1a[g] : (c == 1 ? &bar->full_l1b[g] : &bar->full_x[g]));
           }
           advance(it, g);
         }
@@ -486,8 +498,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     uint8_t* h2_tiles = smem + E::kOffH2;
     const float* b2 = reinterpret_cast<const float*>(smem + (kPolicy ? kOffB2P : kOffB2V));
     // Barrier phases need no counters: per group-step a group waits on its
-    // full_x barrier once per chunk (4 times), on full_y and full_z twice
-    // each and on acc3_full once, so the phase parities are c & 1,
+    // full_x, full_y and full_z barriers twice each and on full_l1a,
+    // full_l1b and acc3_full once, so the phase parities are c & 1,
     // (c >> 1) & 1 and the parity of the group's own step count.
     bool ok = true;
 
@@ -495,15 +507,21 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     // head dot product in head[0], policy mode the 16 head outputs.
     auto run_network = [&](int k, int it, float* head) -> bool {
       const int slot = k & 1;
-      for (int c = 0; c < kNChunks; ++c) {       // layer 1 (X) -> h1 slot
-        if (!tc::mbar_wait(&bar->full_x[g], (uint32_t)c & 1u, abort, kWaitLimitNs)) return false;
+      // layer 1 -> h1 slot.  Chunk c's bf16 pairs go to slot columns
+      // 32c..32c+31, which held accumulator columns this thread has already
+      // read (chunk 0's second half for c = 1, chunk 1's for c = 2, 3).
+      for (int c = 0; c < kNChunks; ++c) {
+        uint64_t* full = c == 0 ? &bar->full_l1a[g] : (c == 1 ? &bar->full_l1b[g] : &bar->full_x[g]);
+        if (!tc::mbar_wait(full, c < 2 ? (uint32_t)it & 1u : (uint32_t)c & 1u, abort, kWaitLimitNs))
+          return false;
         tc::tc_fence_after();
+        const uint32_t src = c < 2 ? kColH1 + slot * 128 + c * kChunk : kColX;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           uint32_t acc[32], hv[16];
-          tc::tmem_ld32(lane_addr + kColX + 32 * half, acc);
+          tc::tmem_ld32(lane_addr + src + 32 * half, acc);
           tc::tmem_ld_wait(acc);
-          if (half == 1) {
+          if (half == 1 && c >= 2) {
             tc::tc_fence_before();
             tc::mbar_arrive(&bar->empty_x);
           }
