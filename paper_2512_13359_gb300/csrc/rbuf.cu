@@ -101,32 +101,94 @@ __global__ void __launch_bounds__(256) k_rb_insert(int T, int N, int D, int A,
   }
 }
 
-__global__ void __launch_bounds__(256) k_rb_sample(int B, int D, int A, uint32_t size,
-                                                   uint32_t k0, uint32_t k1, uint32_t d0,
-                                                   uint32_t d1, const float* __restrict__ s_obs,
-                                                   const float* __restrict__ s_act,
-                                                   const float* __restrict__ s_rew,
-                                                   const float* __restrict__ s_next,
-                                                   const uint8_t* __restrict__ s_done,
-                                                   float* __restrict__ obs, float* __restrict__ act,
-                                                   float* __restrict__ rew, float* __restrict__ next,
-                                                   uint8_t* __restrict__ done,
-                                                   uint32_t* __restrict__ idx_out) {
-  // 8 samples per block of 256 threads: one warp per sample
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * 8 + w;
-  if (b >= B) return;
-  const uint4 r = philox10((uint32_t)b, 0x52420000u, d0, d1, k0, k1);
-  const uint64_t s = ((uint64_t)r.x * (uint64_t)size) >> 32;
-  for (int k = lane; k < D; k += 32) {
-    obs[(size_t)b * D + k] = __ldg(s_obs + s * D + k);
-    next[(size_t)b * D + k] = __ldg(s_next + s * D + k);
+// 64 samples per block of 256 threads.  One thread per sample draws its slot
+// (Philox at counter (b, 0x52420000, draw), key = seed; slot = the word's
+// multiply-high with size); then the block gathers the observation rows as
+// flat (sample, column) elements, four per thread in flight, reading each
+// sampled row contiguously and writing the output sample-major and
+// coalesced, the actions likewise, and the scalar fields with the first
+// batch of row loads.
+constexpr int kSampPerBlock = 64;
+constexpr int kSampThreads = 256;
+
+__global__ void __launch_bounds__(kSampThreads) k_rb_sample(int B, int D, int A, uint32_t size,
+                                                           uint32_t k0, uint32_t k1, uint32_t d0,
+                                                           uint32_t d1,
+                                                           const float* __restrict__ s_obs,
+                                                           const float* __restrict__ s_act,
+                                                           const float* __restrict__ s_rew,
+                                                           const float* __restrict__ s_next,
+                                                           const uint8_t* __restrict__ s_done,
+                                                           float* __restrict__ obs,
+                                                           float* __restrict__ act,
+                                                           float* __restrict__ rew,
+                                                           float* __restrict__ next,
+                                                           uint8_t* __restrict__ done,
+                                                           uint32_t* __restrict__ idx_out) {
+  __shared__ uint32_t slot[kSampPerBlock];
+  const int b0 = blockIdx.x * kSampPerBlock;
+  const int nb = min(kSampPerBlock, B - b0);
+  const int tid = threadIdx.x;
+  if (tid < nb) {
+    const int b = b0 + tid;
+    const uint4 r = philox10((uint32_t)b, 0x52420000u, d0, d1, k0, k1);
+    const uint32_t sl = (uint32_t)(((uint64_t)r.x * (uint64_t)size) >> 32);
+    slot[tid] = sl;
+    if (idx_out) idx_out[b] = sl;
   }
-  for (int k = lane; k < A; k += 32) act[(size_t)b * A + k] = __ldg(s_act + s * A + k);
-  if (lane == 0) {
-    rew[b] = __ldg(s_rew + s);
-    done[b] = __ldg(s_done + s);
-    if (idx_out) idx_out[b] = (uint32_t)s;
+  __syncthreads();
+  float r_v = 0.0f;
+  uint8_t d_v = 0;
+  if (tid < nb) {
+    const uint32_t sl = slot[tid];
+    r_v = __ldg(s_rew + sl);
+    d_v = __ldg(s_done + sl);
+  }
+  const int nD = nb * D;
+  float* obs_b = obs + (size_t)b0 * D;
+  float* next_b = next + (size_t)b0 * D;
+  for (int e0 = tid; e0 < nD; e0 += 4 * kSampThreads) {
+    float vo[4], vn[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kSampThreads;
+      if (e < nD) {
+        const int j = e / D;
+        const size_t src = (size_t)slot[j] * D + (e - j * D);
+        vo[u] = __ldg(s_obs + src);
+        vn[u] = __ldg(s_next + src);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kSampThreads;
+      if (e < nD) {
+        obs_b[e] = vo[u];
+        next_b[e] = vn[u];
+      }
+    }
+  }
+  if (tid < nb) {
+    rew[b0 + tid] = r_v;
+    done[b0 + tid] = d_v;
+  }
+  const int nA = nb * A;
+  float* act_b = act + (size_t)b0 * A;
+  for (int e0 = tid; e0 < nA; e0 += 4 * kSampThreads) {
+    float va[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kSampThreads;
+      if (e < nA) {
+        const int j = e / A;
+        va[u] = __ldg(s_act + (size_t)slot[j] * A + (e - j * A));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kSampThreads;
+      if (e < nA) act_b[e] = va[u];
+    }
   }
 }
 
@@ -334,7 +396,8 @@ int rbuf_sample(auv_rbuf* r, uint32_t B, uint64_t seed, uint64_t draw, float* ob
       (rc = need_dev(r, done, "done", 1)))
     return rc;
   if (idx && (rc = need_dev(r, idx, "idx", 4))) return rc;
-  auv::k_rb_sample<<<(B + 7) / 8, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+  auv::k_rb_sample<<<(B + auv::kSampPerBlock - 1) / auv::kSampPerBlock, auv::kSampThreads, 0,
+                     static_cast<cudaStream_t>(stream)>>>(
       (int)B, (int)r->D, (int)r->A, (uint32_t)r->size, (uint32_t)seed, (uint32_t)(seed >> 32),
       (uint32_t)draw, (uint32_t)(draw >> 32), r->obs, r->act, r->rew, r->next, r->done, obs, act,
       rew, next_obs, done, idx);

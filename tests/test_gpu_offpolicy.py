@@ -44,11 +44,16 @@ def _traj(rng, T, D, A, N):
             rng.normal(size=(D, N)).astype(np.float32))
 
 
-def test_replay_buffer_matches_oracle_ring():
+@pytest.mark.parametrize("D,A,B", [(18, 8, 4099), (12, 6, 1), (12, 6, 63), (37, 5, 64),
+                                   (37, 5, 4099)])
+def test_replay_buffer_matches_oracle_ring(D, A, B):
+    """Inserts that wrap a 1,000-slot ring, then samples checked field by
+    field: the Fossen and paper widths and an odd width, batches of one, a
+    partial and a whole 64-sample block, and a ragged 4,099."""
     torch = need_gpu()
     from oracle import offpolicy_oracle as F
     from paper_2512_13359_gb300 import auvenv
-    D, A, C = 18, 8, 1000
+    C = 1000
     rb = auvenv.ReplayBuffer(D, A, C)
     ref = F.ReplayBuffer(D, A, C)
     rng = np.random.default_rng(1)
@@ -59,8 +64,8 @@ def test_replay_buffer_matches_oracle_ring():
         ref.insert(obs, act, rew, done, last)
         assert rb.size == (ref.size, ref.head)
     for draw in range(3):
-        out = rb.sample(4099, seed=77, draw=draw, with_idx=True)
-        r = ref.sample(77, draw, 4099)
+        out = rb.sample(B, seed=77, draw=draw, with_idx=True)
+        r = ref.sample(77, draw, B)
         assert np.array_equal(to_np(out["idx"]).view(np.uint32), r["idx"].astype(np.uint32))
         for k in ("obs", "act", "rew", "next_obs", "done"):
             assert np.array_equal(to_np(out[k]), r[k]), k
