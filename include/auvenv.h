@@ -401,6 +401,12 @@ int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const fl
  * L = vf_coef mean (V - ret)^2 / 2 (the critic regression of SHAC, whose
  * TD(lambda) targets are env_gae's returns); the policy is neither run nor
  * changed, and batch.act, .logp, .adv may be NULL. */
+#define AUV_PPO_GEMM_FORWARD 2u /* flags: in bf16 mode, run the forward pass
+ * through cuBLAS GEMMs and tanh passes.  Without it a bf16 learner with
+ * hidden == 256, obs_dim <= 18 runs both networks' forward passes on the
+ * tcgen05 engine of env_rollout (weights packed from the fp32 master copy
+ * every step; tanh on the fp32 pre-activation, rounded to bf16), which
+ * writes H1, H2 and the heads for the cuBLAS backward. */
 #define AUV_PPO_STATS 8   /* floats in a statistics record:                       */
 /* [0] surrogate (policy) loss, [1] value loss (mean (V - ret)^2 / 2),
  * [2] entropy, [3] approx. KL mean(logp_old - logp), [4] clip fraction
@@ -416,7 +422,7 @@ typedef struct auv_ppo_config {
   uint32_t minibatch;     /* B samples per gradient step, 2 .. 2^22            */
   uint32_t precision;     /* AUV_PPO_FP32 | AUV_PPO_TF32 | AUV_PPO_BF16        */
   uint32_t norm_adv;      /* 1: normalise advantages per minibatch, 0: not     */
-  uint32_t flags;         /* AUV_PPO_VALUE_ONLY or 0                           */
+  uint32_t flags;         /* AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_FORWARD, or 0   */
   uint64_t seed;          /* key of the minibatch permutations                 */
   float clip_eps;         /* > 0                                               */
   float vf_coef, ent_coef;            /* finite                                */
@@ -487,6 +493,14 @@ int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream);
  */
 int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t n_minibatches,
                float* stats, void* stream);
+
+/* ppo_status: synchronise `stream`, copy the learner's device status block
+ * to *out and return out->code (the auv_status fields as for env_status):
+ * AUV_ERR_TIMEOUT if a tensor-core engine launch of a gradient step gave up
+ * on a bounded wait (the update's results are then invalid), AUV_OK
+ * otherwise.  ppo_clear_status zeroes it (asynchronously on stream). */
+int ppo_status(auv_ppo* p, auv_status* out, void* stream);
+int ppo_clear_status(auv_ppo* p, void* stream);
 
 /* ppo_export_weights: write both networks, in the env_set_weights layout,
  * to device memory (asynchronous on `stream`) -- e.g. straight into the

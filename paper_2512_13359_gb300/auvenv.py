@@ -32,6 +32,7 @@ AUV_PPO_TF32 = 1
 AUV_PPO_BF16 = 2
 AUV_PPO_STATS = 8
 AUV_PPO_VALUE_ONLY = 1
+AUV_PPO_GEMM_FORWARD = 2
 PPO_PRECISION = {"fp32": AUV_PPO_FP32, "tf32": AUV_PPO_TF32, "bf16": AUV_PPO_BF16}
 PPO_STAT_NAMES = ("pg_loss", "v_loss", "entropy", "approx_kl", "clip_frac", "grad_norm", "loss",
                   "steps")
@@ -45,7 +46,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "rbuf_size", "rbuf_insert", "rbuf_sample",
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
-            "ppo_update", "ppo_export_weights")
+            "ppo_update", "ppo_export_weights", "ppo_status", "ppo_clear_status")
 
 
 class LibraryMissing(RuntimeError):
@@ -180,6 +181,8 @@ def lib(path: str | None = None):
     L.ppo_grads.argtypes = [P, C.POINTER(PpoBatch), U64, U32, P, P, P]
     L.ppo_apply.argtypes = [P, P, P, P]
     L.ppo_update.argtypes = [P, C.POINTER(PpoBatch), U32, U32, P, P]
+    L.ppo_status.argtypes = [P, C.POINTER(AuvStatus), P]
+    L.ppo_clear_status.argtypes = [P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
     L.env_last_error.restype = C.c_char_p
@@ -423,7 +426,8 @@ def make_ppo_config(obs_dim: int, act_dim: int, hidden: int, minibatch: int,
     c.obs_dim, c.act_dim, c.hidden, c.minibatch = obs_dim, act_dim, hidden, minibatch
     c.precision = PPO_PRECISION[precision] if isinstance(precision, str) else int(precision)
     c.norm_adv = 1 if h.pop("norm_adv") else 0
-    c.flags = AUV_PPO_VALUE_ONLY if h.pop("value_only", False) else 0
+    c.flags = ((AUV_PPO_VALUE_ONLY if h.pop("value_only", False) else 0)
+               | (AUV_PPO_GEMM_FORWARD if h.pop("gemm_forward", False) else 0))
     c.seed = seed
     for k, v in h.items():
         setattr(c, k, float(v))
@@ -523,6 +527,16 @@ class Learner:
         b = self._batch(traj)
         self._check(lib().ppo_update(self.h, C.byref(b), epochs, n_minibatches, _ptr(stats),
                                      _stream(stream)))
+
+    def status(self, stream=None) -> AuvStatus:
+        """Synchronise and read the device status block (code 0: no engine
+        wait gave up)."""
+        s = AuvStatus()
+        lib().ppo_status(self.h, C.byref(s), _stream(stream))
+        return s
+
+    def clear_status(self, stream=None):
+        self._check(lib().ppo_clear_status(self.h, _stream(stream)))
 
 
 class ReplayBuffer:

@@ -15,6 +15,21 @@ size_t bf16_value_image_bytes();
 cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* wv_f32,
                              void* wp_packed, void* wv_packed, cudaStream_t s);
 
+// The same from explicit widths: network input in_dim (<= 18), policy head
+// policy_out (<= 16); either weight pointer may be NULL.
+cudaError_t launch_pack_bf16_dims(int in_dim, int policy_out, const float* wp_f32,
+                                  const float* wv_f32, void* wp_packed, void* wv_packed,
+                                  cudaStream_t s);
+
+// Learner forward of one network (policy: out_dim <= 16 head outputs; value:
+// one) on `rows` bf16 input rows x[r][ldx] (ldx a multiple of 8, > in_dim):
+// the bf16 hidden activations to h1, h2 ([rows][ldh], columns 0..255; ldh a
+// multiple of 8) and the head to out[r][ldo], fp32.
+cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_dim, int out_dim,
+                                      const uint16_t* x, int ldx, size_t rows, uint16_t* h1,
+                                      uint16_t* h2, int ldh, float* out, int ldo, Status* st,
+                                      cudaStream_t s);
+
 // Fused rollout with the policy network on tcgen05.
 cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp_packed,
                                 const Traj& tr, int T, uint64_t t_g0, Status* st, cudaStream_t s);

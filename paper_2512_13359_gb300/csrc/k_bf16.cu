@@ -179,7 +179,21 @@ struct RowIO {            // row modes: obs element (r, k) at ((r / ns) * obs_di
   float* out;             // head[r][out_dim] (policy) or value[r] (value)
   int obs_dim;            // 18 (Fossen model) or 12 (paper model)
   int out_dim;            // policy head width written per row
+  // learner rows (zero when unused)
+  const uint16_t* xb;     // bf16 inputs xb[r * ldx + k] in place of obs
+  int ldx;
+  uint16_t* h1;           // bf16 hidden activations h1[r * ldh + j], j < 256
+  uint16_t* h2;
+  int ldh;
+  int ldo;                // head row stride (0: out_dim for the policy, 1 for the value)
 };
+
+// 32 bf16 values (16 pairs) to 64 bytes at p (16-byte aligned).
+__device__ __forceinline__ void store_bf16x32(uint16_t* p, const uint32_t (&v)[16]) {
+  uint4* q = reinterpret_cast<uint4*>(p);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) q[j] = make_uint4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+}
 
 template <int G, int MODE>
 struct Engine {
@@ -504,8 +518,9 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     bool ok = true;
 
     // Layer 1-3 epilogues of this group's step k; value mode returns the
-    // head dot product in head[0], policy mode the 16 head outputs.
-    auto run_network = [&](int k, int it, float* head) -> bool {
+    // head dot product in head[0], policy mode the 16 head outputs.  With
+    // h1r / h2r set, the row's bf16 hidden activations are stored there too.
+    auto run_network = [&](int k, int it, float* head, uint16_t* h1r, uint16_t* h2r) -> bool {
       const int slot = k & 1;
       // layer 1 -> h1 slot.  Chunk c's bf16 pairs go to slot columns
       // 32c..32c+31, which held accumulator columns this thread has already
@@ -527,6 +542,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           }
           tanh32(acc, hv);
           tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
+          if (h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv);
         }
       }
       tc::tmem_st_wait();
@@ -552,6 +568,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::mbar_arrive(odd ? &bar->empty_z : &bar->empty_y);
           }
           bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
+          if (h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv);
           if (kPolicy) {
             // Write j = 2k + (c >> 1) of h2 buffer c & 1 reuses it after
             // layer 3 has consumed write j - 1 (completion j - 1 of h2_empty).
@@ -631,7 +648,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         float head[kHeadOut];
         __syncwarp();
         // every group with work runs T steps: the step index is t * n_act + g
-        if (!(ok = run_network(t * n_act + g, t, head))) break;
+        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr))) break;
         __syncwarp();
         if (active) {
           // The episode parameters are not held in registers across the
@@ -698,7 +715,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(t * n_act + g, t, head))) break;
+        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr))) break;
         __syncwarp();
         if (active) {
           const uint32_t id = M.id_base + (uint32_t)i;
@@ -734,7 +751,24 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         const size_t r = (size_t)(slot0 + g + it * n_slots) * kRows + row;
         const bool active = r < io.rows;
         float o[kObs];
-        if (active) {
+        if (active && io.xb) {
+          // bf16 row, 16-byte pieces (ldx >= obs_dim + 1, a multiple of 8)
+          const uint4* x = reinterpret_cast<const uint4*>(io.xb + r * (size_t)io.ldx);
+#pragma unroll
+          for (int q = 0; q < (kObs + 7) / 8; ++q) {
+            uint4 u = make_uint4(0u, 0u, 0u, 0u);
+            if (8 * q < io.obs_dim) u = __ldg(x + q);
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const int k = 8 * q + j;
+              if (k < kObs) {
+                const float v = (j & 1) ? tc::bf16hi(w4[j >> 1]) : tc::bf16lo(w4[j >> 1]);
+                o[k] = k < io.obs_dim ? v : 0.0f;
+              }
+            }
+          }
+        } else if (active) {
           const size_t ns = (size_t)io.ns;
           const size_t base = (r / ns) * (size_t)io.obs_dim * ns + r % ns;
 #pragma unroll
@@ -749,15 +783,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(step_index<G>(it, g, iters), it, head))) break;
+        uint16_t* h1r = active && io.h1 ? io.h1 + r * (size_t)io.ldh : nullptr;
+        uint16_t* h2r = active && io.h2 ? io.h2 + r * (size_t)io.ldh : nullptr;
+        if (!(ok = run_network(step_index<G>(it, g, iters), it, head, h1r, h2r))) break;
         __syncwarp();
         if (active) {
           if (MODE == kValueRows) {
-            io.out[r] = head[0];
+            io.out[r * (size_t)(io.ldo ? io.ldo : 1)] = head[0];
           } else {
+            const size_t ldo = (size_t)(io.ldo ? io.ldo : io.out_dim);
 #pragma unroll
             for (int k = 0; k < kHeadOut; ++k)
-              if (k < io.out_dim) io.out[r * io.out_dim + k] = head[k];
+              if (k < io.out_dim) io.out[r * ldo + k] = head[k];
           }
         }
       }
@@ -851,11 +888,20 @@ size_t bf16_value_image_bytes() { return kValueImage; }
 
 cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* wv_f32,
                              void* wp_packed, void* wv_packed, cudaStream_t s) {
-  const int in_dim = M.model == 1 ? 12 : kObs;
+  return launch_pack_bf16_dims(M.model == 1 ? 12 : kObs, M.policy_out, wp_f32, wv_f32, wp_packed,
+                               wv_packed, s);
+}
+
+cudaError_t launch_pack_bf16_dims(int in_dim, int policy_out, const float* wp_f32,
+                                  const float* wv_f32, void* wp_packed, void* wv_packed,
+                                  cudaStream_t s) {
   const int pol_pieces = kH * 4 + 4 * kH * 8 + 4 * kHeadOut * 8 + 2 * kH + kHeadOut;
-  k_pack<<<(pol_pieces + 255) / 256, 256, 0, s>>>(wp_f32, in_dim, M.policy_out,
-                                                  static_cast<uint8_t*>(wp_packed));
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = cudaSuccess;
+  if (wp_f32) {
+    k_pack<<<(pol_pieces + 255) / 256, 256, 0, s>>>(wp_f32, in_dim, policy_out,
+                                                    static_cast<uint8_t*>(wp_packed));
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess || !wv_f32) return e;
   const int val_pieces = kH * 4 + 4 * kH * 8 + 3 * kH + 1;
   k_pack<<<(val_pieces + 255) / 256, 256, 0, s>>>(wv_f32, in_dim, 1,
@@ -869,7 +915,7 @@ cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp
   const int G = pick_groups(tiles);
   const int grid = (int)((tiles + G - 1) / G);
   const uint8_t* img = static_cast<const uint8_t*>(wp_packed);
-  const RowIO io = {nullptr, 0, 1, nullptr, 0, 0};
+  const RowIO io = {nullptr, 0, 1, nullptr, 0, 0, nullptr, 0, nullptr, nullptr, 0, 0};
   if (M.model == 1) {
     switch (G) {
       case 4: return launch_engine<4, kRollout, 1>(grid, M, B, img, tr, T, t_g0, io, st, s);
@@ -904,8 +950,20 @@ cudaError_t launch_value_bf16(const Model& M, const void* wv_packed, const float
                               const float* obs, size_t rows, int n, float* value, Status* st,
                               cudaStream_t s) {
   (void)wv_f32;
-  const RowIO io = {obs, rows, n, value, M.model == 1 ? 12 : kObs, 1};
+  const RowIO io = {obs, rows, n, value, M.model == 1 ? 12 : kObs, 1,
+                    nullptr, 0, nullptr, nullptr, 0, 0};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), io, st, s);
+}
+
+cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_dim, int out_dim,
+                                      const uint16_t* x, int ldx, size_t rows, uint16_t* h1,
+                                      uint16_t* h2, int ldh, float* out, int ldo, Status* st,
+                                      cudaStream_t s) {
+  const Model M{};
+  const RowIO io = {nullptr, rows, 1, out, in_dim, policy ? out_dim : 1, x, ldx, h1, h2, ldh, ldo};
+  const uint8_t* img = static_cast<const uint8_t*>(packed);
+  return policy ? launch_rows<kPolicyRows>(M, img, io, st, s)
+                : launch_rows<kValueRows>(M, img, io, st, s);
 }
 
 cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const void* wv_packed,
@@ -913,10 +971,10 @@ cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const voi
                                 float* value, Status* st, cudaStream_t s) {
   (void)wv_f32;
   const int od = M.model == 1 ? 12 : kObs;
-  const RowIO io = {obs, (size_t)n, 1, head, od, M.policy_out};
+  const RowIO io = {obs, (size_t)n, 1, head, od, M.policy_out, nullptr, 0, nullptr, nullptr, 0, 0};
   cudaError_t e = launch_rows<kPolicyRows>(M, static_cast<const uint8_t*>(wp_packed), io, st, s);
   if (e != cudaSuccess || !value) return e;
-  const RowIO iov = {obs, (size_t)n, 1, value, od, 1};
+  const RowIO iov = {obs, (size_t)n, 1, value, od, 1, nullptr, 0, nullptr, nullptr, 0, 0};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), iov, st, s);
 }
 

@@ -23,10 +23,15 @@
 #include <cstring>
 #include <new>
 
+#include <climits>
+
+#include "auv_bf16.h"
+#include "auv_device.cuh"
 #include "auv_kernels.h"
 #include "auvenv.h"
 
 namespace ppo = auv::ppo;
+using auv::Status;
 
 struct auv_ppo {
   auv_ppo_config cfg;
@@ -52,6 +57,12 @@ struct auv_ppo {
   float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
   ppo::StepCtl* ctl;          // device: per-step variables
   void* blas_ws;
+  // bf16 forward on the tensor-core engine: packed images of both networks,
+  // rebuilt from w every step, a flat staging copy and a status block
+  bool eng = false;
+  void *img_p = nullptr, *img_v = nullptr;
+  float* flat_eng = nullptr;
+  Status* st = nullptr;
   uint64_t t, epoch;
   // One gradient step captured as a CUDA graph for ppo_update, replayed on a
   // private stream; valid for the batch it was captured with.
@@ -126,7 +137,8 @@ int validate(const auv_ppo_config* c) {
     return fail(nullptr, AUV_ERR_INVALID, "minibatch outside [2, 2^22]");
   if (c->precision > AUV_PPO_BF16) return fail(nullptr, AUV_ERR_INVALID, "unknown precision %u", c->precision);
   if (c->norm_adv > 1) return fail(nullptr, AUV_ERR_INVALID, "norm_adv must be 0 or 1");
-  if (c->flags & ~AUV_PPO_VALUE_ONLY) return fail(nullptr, AUV_ERR_INVALID, "unknown flags %#x", c->flags);
+  if (c->flags & ~(AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_FORWARD))
+    return fail(nullptr, AUV_ERR_INVALID, "unknown flags %#x", c->flags);
   if (!(std::isfinite(c->clip_eps) && c->clip_eps > 0.0f))
     return fail(nullptr, AUV_ERR_INVALID, "clip_eps must be finite and > 0");
   if (!std::isfinite(c->vf_coef) || !std::isfinite(c->ent_coef) || std::isnan(c->max_grad_norm) ||
@@ -263,6 +275,9 @@ int set_ctl(auv_ppo* p, uint64_t epoch0, uint32_t n_mb, uint32_t step, uint64_t 
   return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "step control");
 }
 
+int convert(auv_ppo* p, float* flat_pol, float* flat_val, float* aug, bool to_aug,
+            cudaStream_t s);
+
 int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
   const ppo::Dims& d = p->d;
   const uint32_t m = b->T * b->N;
@@ -270,7 +285,24 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
                                      b->adv, b->ret, b->N, p->smp, p->X, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "gather");
   int rc;
-  if ((!d.value_only && (rc = forward(p, 0, s))) || (rc = forward(p, 1, s))) return rc;
+  if (p->eng) {
+    // Both networks on the tensor-core engine: flat fp32 weights, packed bf16
+    // images, then one launch per network writing H1, H2 and the head.
+    if ((rc = convert(p, p->flat_eng, p->flat_eng + p->n_flat[0], p->w, false, s))) return rc;
+    if ((e = auv::launch_pack_bf16_dims(d.D, p->out[0], d.value_only ? nullptr : p->flat_eng,
+                                   p->flat_eng + p->n_flat[0], p->img_p, p->img_v, s)))
+      return cuda_fail(p, e, "pack engine weights");
+    for (int net = d.value_only ? 1 : 0; net < 2; ++net) {
+      if ((e = auv::launch_learn_forward_bf16(net == 0, net ? p->img_v : p->img_p, d.D, p->out[net],
+                                         static_cast<const uint16_t*>(p->X), d.Dp, (size_t)d.B,
+                                         static_cast<uint16_t*>(p->h1[net]),
+                                         static_cast<uint16_t*>(p->h2[net]), d.Hp, p->y[net],
+                                         ld_head(p, net), p->st, s)))
+        return cuda_fail(p, e, "engine forward");
+    }
+  } else if ((!d.value_only && (rc = forward(p, 0, s))) || (rc = forward(p, 1, s))) {
+    return rc;
+  }
   const ppo::LossHp hp = loss_hp(p);
   if ((e = ppo::launch_head(d, hp, p->y[0], p->y[1], p->smp, p->g_y, p->g_v, p->head_part, s)))
     return cuda_fail(p, e, "loss head");
@@ -407,6 +439,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     p->n_aug[k] = ppo::aug_count(d.D, d.Dp, d.H, d.Hp, p->out[k]);
   }
   p->n_aug_all = p->n_aug[0] + p->n_aug[1];
+  // the engine's networks: hidden 256, input <= 18, head <= 16 (2A <= 16)
+  p->eng = p->bf16 && d.H == 256 && d.D <= auv::kObs && !(cfg->flags & AUV_PPO_GEMM_FORWARD);
   p->ctype = cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
   // one allocation, 256-byte aligned pieces
   const size_t B = (size_t)d.B, nb = (B + 255) / 256;
@@ -426,7 +460,11 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_gv = take(B * d.ld_val * es), o_hp = take(nb * 5 * 4),
                o_np = take(ppo::kNormBlocks * 4), o_mb = take(AUV_PPO_STATS * 4),
                o_acc = take(AUV_PPO_STATS * 4), o_ctl = take(sizeof(ppo::StepCtl)),
-               o_ws = take(kBlasWorkspace);
+               o_ws = take(kBlasWorkspace),
+               o_ip = take(p->eng ? auv::bf16_policy_image_bytes() : 0),
+               o_iv = take(p->eng ? auv::bf16_value_image_bytes() : 0),
+               o_fe = take(p->eng ? (p->n_flat[0] + p->n_flat[1]) * 4 : 0),
+               o_st = take(sizeof(Status));
   size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
   for (int k = 0; k < 2; ++k) {
     o_h1[k] = take(B * d.Hp * es);
@@ -460,6 +498,12 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   p->acc = reinterpret_cast<float*>(base + o_acc);
   p->ctl = reinterpret_cast<ppo::StepCtl*>(base + o_ctl);
   p->blas_ws = base + o_ws;
+  if (p->eng) {
+    p->img_p = base + o_ip;
+    p->img_v = base + o_iv;
+    p->flat_eng = reinterpret_cast<float*>(base + o_fe);
+  }
+  p->st = reinterpret_cast<Status*>(base + o_st);
   for (int k = 0; k < 2; ++k) {
     p->h1[k] = base + o_h1[k];
     p->h2[k] = base + o_h2[k];
@@ -467,6 +511,10 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     p->y[k] = reinterpret_cast<float*>(base + o_y[k]);
   }
   e = cudaMemset(p->mem, 0, off);
+  if (e == cudaSuccess) {
+    const Status s0 = {0, 0, INT32_MAX, 0};
+    e = cudaMemcpy(p->st, &s0, sizeof(s0), cudaMemcpyHostToDevice);
+  }
   for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
     e = ppo::launch_fill_ones(p->bf16, p->h1[k], d.Hp, d.H, d.B, 0);
     if (e == cudaSuccess) e = ppo::launch_fill_ones(p->bf16, p->h2[k], d.Hp, d.H, d.B, 0);
@@ -617,6 +665,33 @@ int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream) {
     if (e != cudaSuccess) return cuda_fail(p, e, "copy gradient norm");
   }
   return AUV_OK;
+}
+
+int ppo_status(auv_ppo* p, auv_status* out, void* stream) {
+  if (!p || !out) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Status h;
+  cudaError_t e = cudaMemcpyAsync(&h, p->st, sizeof(h), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(p, e, "read status");
+  out->code = h.code;
+  out->nan_flag = h.nan_flag;
+  out->first_nan_env = h.first_nan_env == INT32_MAX ? -1 : h.first_nan_env;
+  out->timeouts = h.timeouts;
+  if (h.code != 0) fail(p, h.code, "device status %d (timeouts %d)", h.code, h.timeouts);
+  return h.code;
+}
+
+int ppo_clear_status(auv_ppo* p, void* stream) {
+  if (!p) return AUV_ERR_INVALID;
+  int rc = check_device(p);
+  if (rc) return rc;
+  static const Status s0 = {0, 0, INT32_MAX, 0};
+  cudaError_t e = cudaMemcpyAsync(p->st, &s0, sizeof(s0), cudaMemcpyHostToDevice,
+                                  static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "clear status");
 }
 
 int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t n_minibatches,

@@ -140,7 +140,7 @@ def test_ppo_config_struct_size_matches_header(auvlib):
 @pytest.mark.parametrize("field,value,msg", [
     ("obs_dim", 0, b"obs_dim"), ("obs_dim", 65, b"obs_dim"), ("act_dim", 9, b"act_dim"),
     ("hidden", 100, b"hidden"), ("hidden", 2048, b"hidden"), ("minibatch", 1, b"minibatch"),
-    ("precision", 3, b"precision"), ("norm_adv", 2, b"norm_adv"), ("flags", 2, b"flags"),
+    ("precision", 3, b"precision"), ("norm_adv", 2, b"norm_adv"), ("flags", 4, b"flags"),
     ("clip_eps", 0.0, b"clip_eps"), ("clip_eps", float("nan"), b"clip_eps"),
     ("vf_coef", float("inf"), b"finite"), ("max_grad_norm", float("nan"), b"finite"),
     ("lr", -1e-3, b"lr"), ("adam_beta1", 1.0, b"betas"), ("adam_beta2", -0.1, b"betas"),

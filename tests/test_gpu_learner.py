@@ -362,3 +362,84 @@ def test_value_only_learner_matches_oracle():
     L.update(dev, 2, 2)
     gp, gv = L.get_weights()
     assert np.array_equal(gp, pw) and not np.array_equal(gv, vw)
+
+
+def _grad_err(gpu, ref, n_pol):
+    return [np.abs(gpu[sl] - ref[sl]).max() / np.abs(ref[sl]).max()
+            for sl in (slice(0, n_pol), slice(n_pol, None))]
+
+
+@pytest.mark.parametrize("D,A,B,seed,calibrated", [(18, 8, 16384, 3, True),
+                                                   (18, 8, 1000, 3, False),
+                                                   (12, 6, 4096, 31, False)])
+def test_bf16_engine_forward(D, A, B, seed, calibrated):
+    """bf16 learners with hidden 256 run the forward pass on the tcgen05
+    engine (H1, H2 and the heads written for the cuBLAS backward): its
+    gradient and loss record against the oracle at a whole-tile and a ragged
+    minibatch and at the paper model's widths, and its error against that of
+    the same learner with the forward through cuBLAS GEMMs
+    (AUV_PPO_GEMM_FORWARD, which rounds the pre-activations to bf16 before
+    tanh); the status block stays clear.  Both paths are held to the
+    tolerance on the calibrated case (that of the tensor-core test above);
+    on other draws the bf16 policy error of the GEMM path reaches 5e-2, so
+    there the engine is held to twice the tolerance (a broken forward is
+    off by order one) and to no more than the GEMM path's error."""
+    torch = need_gpu()
+    from oracle import ppo_oracle as P
+    H, T, N = 256, 4, 8192
+    hp = dict(HP, **COHERENT)
+    pw, vw = _weights(D, H, A, seed=seed)
+    traj = _on_rollout_policy(_traj(seed + 2, T, N, D, A), pw, D, H, A)
+    traj["adv"] = (1.0 + 0.1 * np.random.default_rng(seed + 3).normal(size=(T, N))).astype(np.float32)
+    dtraj = _dev(torch, traj)
+    grads, stats = {}, {}
+    parts, g_ref = P.Learner(pw, vw, (D, H, A), hp, seed=7).grads(traj, 1, 0, B)
+    for gemm in (True, False):
+        L = _learner(D, A, H, B, "bf16", gemm_forward=gemm, **hp)
+        L.set_weights(pw, vw)
+        grad = torch.empty(L.n_policy + L.n_value, device="cuda")
+        st = torch.empty(8, device="cuda")
+        L.grads(dtraj, 1, 0, grad=grad, stats=st)
+        assert L.status().code == 0
+        grads[gemm], stats[gemm] = to_np(grad), to_np(st)
+    e_eng = _grad_err(grads[False], g_ref, L.n_policy)
+    e_gemm = _grad_err(grads[True], g_ref, L.n_policy)
+    print(f"[bf16 forward D={D} B={B}] policy / value error: engine {e_eng[0]:.3e} / "
+          f"{e_eng[1]:.3e}, gemm {e_gemm[0]:.3e} / {e_gemm[1]:.3e} (tol {GRAD_TOL['bf16']})")
+    tol = GRAD_TOL["bf16"] * (1 if calibrated else 2)
+    _check_grad(grads[False], g_ref, L.n_policy, tol, "bf16 engine forward")
+    _check_stats(stats[False], parts, STAT_TOL["bf16"], B)
+    for k in range(2):
+        assert e_eng[k] <= 1.2 * e_gemm[k] + 2e-3, (k, e_eng[k], e_gemm[k])
+    if calibrated:
+        _check_grad(grads[True], g_ref, L.n_policy, GRAD_TOL["bf16"], "bf16 gemm forward")
+        _check_stats(stats[True], parts, STAT_TOL["bf16"], B)
+
+
+def test_bf16_engine_update_repacks_every_step():
+    """A captured multi-step update at a large learning rate: the engine
+    path's weights follow the GEMM path's step by step (the packed images
+    are rebuilt from the updated weights inside every replayed step; stale
+    images would leave the two apart by the size of the updates)."""
+    torch = need_gpu()
+    D, A, H, T, N, B = 18, 8, 256, 4, 4096, 4096
+    hp = dict(HP, **COHERENT, lr=3e-3, max_grad_norm=0.0)
+    pw, vw = _weights(D, H, A, seed=41)
+    traj = _on_rollout_policy(_traj(42, T, N, D, A), pw, D, H, A)
+    traj["adv"] = (1.0 + 0.1 * np.random.default_rng(43).normal(size=(T, N))).astype(np.float32)
+    dtraj = _dev(torch, traj)
+    out = {}
+    for gemm in (False, True):
+        L = _learner(D, A, H, B, "bf16", gemm_forward=gemm, **hp)
+        L.set_weights(pw, vw)
+        L.update(dtraj, 2, 4)
+        assert L.status().code == 0
+        out[gemm] = L.get_weights()
+    # Adam turns small gradient differences into whole steps on components
+    # whose gradient is near zero, so the paths are compared in norm.
+    for k, (a, b) in enumerate(zip(out[False], out[True])):
+        base = (pw, vw)[k]
+        moved = np.linalg.norm(b - base)
+        diff = np.linalg.norm(a - b)
+        print(f"[engine update] net {k}: |move| {moved:.3e}, |engine - gemm| {diff:.3e}")
+        assert moved > 0.1 and diff <= 0.2 * moved
