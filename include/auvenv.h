@@ -401,12 +401,14 @@ int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const fl
  * L = vf_coef mean (V - ret)^2 / 2 (the critic regression of SHAC, whose
  * TD(lambda) targets are env_gae's returns); the policy is neither run nor
  * changed, and batch.act, .logp, .adv may be NULL. */
-#define AUV_PPO_GEMM_FORWARD 2u /* flags: in bf16 mode, run the forward pass
- * through cuBLAS GEMMs and tanh passes.  Without it a bf16 learner with
- * hidden == 256, obs_dim <= 18 runs both networks' forward passes on the
- * tcgen05 engine of env_rollout (weights packed from the fp32 master copy
- * every step; tanh on the fp32 pre-activation, rounded to bf16), which
- * writes H1, H2 and the heads for the cuBLAS backward. */
+#define AUV_PPO_GEMM_PATH 2u /* flags: in bf16 mode, run the forward pass and
+ * the input gradients through cuBLAS GEMMs and tanh passes.  Without it a
+ * bf16 learner with hidden == 256, obs_dim <= 18 runs both networks' forward
+ * passes and their backward-data (dL/dZ2, dL/dZ1 with the tanh derivatives)
+ * on the tcgen05 engine of env_rollout (weights, and their transposes,
+ * packed from the fp32 master copy every step; tanh on the fp32
+ * pre-activation, each product rounded to bf16 once); the weight gradients
+ * stay cuBLAS GEMMs. */
 #define AUV_PPO_STATS 8   /* floats in a statistics record:                       */
 /* [0] surrogate (policy) loss, [1] value loss (mean (V - ret)^2 / 2),
  * [2] entropy, [3] approx. KL mean(logp_old - logp), [4] clip fraction
@@ -422,7 +424,7 @@ typedef struct auv_ppo_config {
   uint32_t minibatch;     /* B samples per gradient step, 2 .. 2^22            */
   uint32_t precision;     /* AUV_PPO_FP32 | AUV_PPO_TF32 | AUV_PPO_BF16        */
   uint32_t norm_adv;      /* 1: normalise advantages per minibatch, 0: not     */
-  uint32_t flags;         /* AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_FORWARD, or 0   */
+  uint32_t flags;         /* AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_PATH, or 0      */
   uint64_t seed;          /* key of the minibatch permutations                 */
   float clip_eps;         /* > 0                                               */
   float vf_coef, ent_coef;            /* finite                                */

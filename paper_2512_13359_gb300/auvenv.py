@@ -32,7 +32,7 @@ AUV_PPO_TF32 = 1
 AUV_PPO_BF16 = 2
 AUV_PPO_STATS = 8
 AUV_PPO_VALUE_ONLY = 1
-AUV_PPO_GEMM_FORWARD = 2
+AUV_PPO_GEMM_PATH = 2
 PPO_PRECISION = {"fp32": AUV_PPO_FP32, "tf32": AUV_PPO_TF32, "bf16": AUV_PPO_BF16}
 PPO_STAT_NAMES = ("pg_loss", "v_loss", "entropy", "approx_kl", "clip_frac", "grad_norm", "loss",
                   "steps")
@@ -427,7 +427,7 @@ def make_ppo_config(obs_dim: int, act_dim: int, hidden: int, minibatch: int,
     c.precision = PPO_PRECISION[precision] if isinstance(precision, str) else int(precision)
     c.norm_adv = 1 if h.pop("norm_adv") else 0
     c.flags = ((AUV_PPO_VALUE_ONLY if h.pop("value_only", False) else 0)
-               | (AUV_PPO_GEMM_FORWARD if h.pop("gemm_forward", False) else 0))
+               | (AUV_PPO_GEMM_PATH if h.pop("gemm_path", False) else 0))
     c.seed = seed
     for k, v in h.items():
         setattr(c, k, float(v))

@@ -30,6 +30,21 @@ cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_di
                                       uint16_t* h2, int ldh, float* out, int ldo, Status* st,
                                       cudaStream_t s);
 
+// Learner backward-data of one network on the same engine, from the packed
+// transposed weights (launch_pack_back_bf16: W3^T and W2^T of the flat fp32
+// weights; in_dim the network input width, out_dim its head width <= 16):
+// gz2 = (W3^T gy) (1 - h2^2) and gz1 = (W2^T gz2) (1 - h1^2), bf16, for
+// `rows` rows (gy [rows][ldy], h1, h2 [rows][ldh], gz2 [rows][ldz2],
+// gz1 [rows][ldz1]; strides multiples of 8, ldy >= 8 ceil(out_dim / 8)).
+// gz1 may be h2 itself: each row is read before it is written, by one thread.
+size_t bf16_back_image_bytes();
+cudaError_t launch_pack_back_bf16(int in_dim, int out_dim, const float* w_f32, void* packed,
+                                  cudaStream_t s);
+cudaError_t launch_learn_backward_bf16(const void* packed, int out_dim, const uint16_t* gy, int ldy,
+                                       size_t rows, const uint16_t* h2, const uint16_t* h1, int ldh,
+                                       uint16_t* gz2, int ldz2, uint16_t* gz1, int ldz1, Status* st,
+                                       cudaStream_t s);
+
 // Fused rollout with the policy network on tcgen05.
 cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp_packed,
                                 const Traj& tr, int T, uint64_t t_g0, Status* st, cudaStream_t s);

@@ -75,7 +75,22 @@ constexpr uint32_t kColA3 = 448;    // two head accumulators of 16 columns
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per wait
 
-enum Mode { kRollout = 0, kPolicyRows = 1, kValueRows = 2 };
+// Learner modes (compile-time, so that the plain row modes carry none of
+// their code): kLearnPolicy / kLearnValue read bf16 input rows and also store
+// H1 and H2; kBackRows is the backward-data pass, the engine's two layers on
+// transposed weights (see k_pack_back).
+enum Mode {
+  kRollout = 0,
+  kPolicyRows = 1,
+  kValueRows = 2,
+  kBackRows = 3,
+  kLearnPolicy = 4,
+  kLearnValue = 5
+};
+
+// Backward image: the W1 slot holds W3^T (rows n < 256, K columns k < out:
+// W3[k][n], the rest zero), the W2 slot W2^T (row n, column k: W2[k][n]).
+constexpr uint32_t kBackImage = kOffW2 + kW2Bytes;
 
 // -------------------------------------------------------------------------
 // weight packing
@@ -150,6 +165,40 @@ __global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
   *reinterpret_cast<uint4*>(img + off) = pk;
 }
 
+// Backward image of one network from its flat fp32 weights (the layout of
+// k_pack): one thread per 16-byte piece of the W1 slot (W3^T, K = 32 with the
+// columns from out_dim up zero) and of the W2 slot (W2^T).
+__global__ void k_pack_back(const float* __restrict__ w, int in_dim, int out_dim,
+                            uint8_t* __restrict__ img) {
+  const float* W2 = w + kH * in_dim + kH;
+  const float* W3 = W2 + kH * kH + kH;
+  const int n_w1 = kH * 4, n_w2 = 4 * kH * 8;
+  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
+  uint16_t v[8];
+  uint32_t off;
+  if (piece < n_w1) {
+    const int n = piece >> 2, p = piece & 3, q = p ^ ((n >> 1) & 3);
+    for (int e = 0; e < 8; ++e) {
+      const int k = 8 * q + e;
+      v[e] = k < out_dim ? bf16_bits(W3[k * kH + n]) : (uint16_t)0;
+    }
+    off = kOffW1 + n * 64 + p * 16;
+  } else if (piece < n_w1 + n_w2) {
+    const int id = piece - n_w1;
+    const int a = id / (kH * 8), n = (id / 8) % kH, p = id & 7, q = p ^ (n & 7);
+    for (int e = 0; e < 8; ++e) v[e] = bf16_bits(W2[(64 * a + 8 * q + e) * kH + n]);
+    off = kOffW2 + a * (kH * 128) + n * 128 + p * 16;
+  } else {
+    return;
+  }
+  uint4 pk;
+  pk.x = v[0] | ((uint32_t)v[1] << 16);
+  pk.y = v[2] | ((uint32_t)v[3] << 16);
+  pk.z = v[4] | ((uint32_t)v[5] << 16);
+  pk.w = v[6] | ((uint32_t)v[7] << 16);
+  *reinterpret_cast<uint4*>(img + off) = pk;
+}
+
 // -------------------------------------------------------------------------
 // engine
 // -------------------------------------------------------------------------
@@ -168,6 +217,7 @@ struct Barriers {
   uint64_t h1_free[2];      // layer-2 MMAs reading an h1 slot completed (commit)
   uint64_t h2_empty[2];     // layer-3 MMAs reading an h2 buffer completed (commit)
   uint64_t drain, drain1, drain2;
+  uint64_t img_full;        // the weight image landed (bulk copies, transaction count)
   uint32_t tmem_base;
   int abort;
 };
@@ -183,10 +233,35 @@ struct RowIO {            // row modes: obs element (r, k) at ((r / ns) * obs_di
   const uint16_t* xb;     // bf16 inputs xb[r * ldx + k] in place of obs
   int ldx;
   uint16_t* h1;           // bf16 hidden activations h1[r * ldh + j], j < 256
-  uint16_t* h2;
+  uint16_t* h2;           // (backward mode: dL/dZ2 and dL/dZ1)
   int ldh;
   int ldo;                // head row stride (0: out_dim for the policy, 1 for the value)
+  // backward mode: the forward's H2 and H1 rows a1[r * lda + j], a2[r * lda + j]
+  // and the row stride of the second output (0: ldh)
+  const uint16_t* a1;
+  const uint16_t* a2;
+  int lda;
+  int ldh2;
 };
+
+// 32 accumulator columns times tanh' from the forward's bf16 activations at
+// h (16-byte aligned): g (1 - h^2), rounded to 16 bf16 pairs.
+__device__ __forceinline__ void dtanh32(const uint32_t (&acc)[32], const uint16_t* h,
+                                        uint32_t (&out)[16]) {
+  const uint4* q = reinterpret_cast<const uint4*>(h);
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const uint4 u = __ldg(q + p);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = 4 * p + e;
+      const float lo = tc::bf16lo(w[e]), hi = tc::bf16hi(w[e]);
+      out[j] = tc::pack_bf16x2(__uint_as_float(acc[2 * j]) * fmaf(-lo, lo, 1.0f),
+                               __uint_as_float(acc[2 * j + 1]) * fmaf(-hi, hi, 1.0f));
+    }
+  }
+}
 
 // 32 bf16 values (16 pairs) to 64 bytes at p (16-byte aligned).
 __device__ __forceinline__ void store_bf16x32(uint16_t* p, const uint32_t (&v)[16]) {
@@ -197,8 +272,11 @@ __device__ __forceinline__ void store_bf16x32(uint16_t* p, const uint32_t (&v)[1
 
 template <int G, int MODE>
 struct Engine {
-  static constexpr bool kPolicy = MODE != kValueRows;
-  static constexpr uint32_t kImage = kPolicy ? kPolicyImage : kValueImage;
+  static constexpr bool kPolicy =
+      MODE == kRollout || MODE == kPolicyRows || MODE == kLearnPolicy;
+  static constexpr bool kBack = MODE == kBackRows;
+  static constexpr bool kLearn = MODE >= kBackRows;
+  static constexpr uint32_t kImage = kPolicy ? kPolicyImage : (kBack ? kBackImage : kValueImage);
   static constexpr uint32_t kImageAl = (kImage + 1023u) & ~1023u;
   static constexpr uint32_t kOffObs = kImageAl;
   static constexpr uint32_t kOffH2 = kOffObs + G * kObsTileBytes;
@@ -341,15 +419,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     tc::mbar_init(&bar->drain, 1);
     tc::mbar_init(&bar->drain1, 1);
     tc::mbar_init(&bar->drain2, 1);
+    tc::mbar_init(&bar->img_full, 1);
     bar->abort = 0;
     tc::mbar_fence_init();
+    // the weight image in a few bulk copies (16-byte multiples; the image
+    // and the shared-memory base are 1024-byte aligned)
+    static_assert(E::kImage % 16 == 0, "image size");
+    constexpr uint32_t kPiece = 32768;
+    tc::mbar_arrive_expect_tx(&bar->img_full, E::kImage);
+    for (uint32_t o = 0; o < E::kImage; o += kPiece)
+      tc::bulk_g2s(smem + o, image + o, E::kImage - o < kPiece ? E::kImage - o : kPiece,
+                   &bar->img_full);
   }
-  {
-    const uint4* src = reinterpret_cast<const uint4*>(image);
-    uint4* dst = reinterpret_cast<uint4*>(smem);
-    for (uint32_t i = tid; i < E::kImage / 16; i += blockDim.x) dst[i] = __ldg(src + i);
-  }
-  tc::fence_async_smem();
   if (warp == 4 * G) {
     tc::tmem_alloc(&bar->tmem_base, kTmemCols);
     tc::tmem_relinquish();
@@ -359,6 +440,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
   tc::tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
   const uint32_t s_base = tc::smem_u32(smem);
+  // every role reads the weights (MMA operands, biases): wait for the image
+  const bool img_ok = tc::mbar_wait(&bar->img_full, 0, abort, kWaitLimitNs);
 
   // ---- work assignment ----
   const int n_tiles = MODE == kRollout ? (M.n + kRows - 1) / kRows
@@ -371,6 +454,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     const int s = slot0 + g;
     iters[g] = MODE == kRollout ? (s < n_tiles ? T : 0)
                                 : (s < n_tiles ? (n_tiles - s - 1) / n_slots + 1 : 0);
+    if (!img_ok) iters[g] = 0;   // the wait gave up: no work, the status latches it
   }
 
   if (is_mma_warp) {
@@ -520,7 +604,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     // Layer 1-3 epilogues of this group's step k; value mode returns the
     // head dot product in head[0], policy mode the 16 head outputs.  With
     // h1r / h2r set, the row's bf16 hidden activations are stored there too.
-    auto run_network = [&](int k, int it, float* head, uint16_t* h1r, uint16_t* h2r) -> bool {
+    auto run_network = [&](int k, int it, float* head, uint16_t* h1r, uint16_t* h2r,
+                           const uint16_t* a1r, const uint16_t* a2r) -> bool {
       const int slot = k & 1;
       // layer 1 -> h1 slot.  Chunk c's bf16 pairs go to slot columns
       // 32c..32c+31, which held accumulator columns this thread has already
@@ -540,9 +625,10 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::tc_fence_before();
             tc::mbar_arrive(&bar->empty_x);
           }
-          tanh32(acc, hv);
+          if constexpr (E::kBack) dtanh32(acc, a1r + c * kChunk + 32 * half, hv);
+          else tanh32(acc, hv);
           tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
-          if (h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv);
+          if (E::kLearn && h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv);
         }
       }
       tc::tmem_st_wait();
@@ -567,9 +653,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::tc_fence_before();
             tc::mbar_arrive(odd ? &bar->empty_z : &bar->empty_y);
           }
-          bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
-          if (h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv);
-          if (kPolicy) {
+          if constexpr (E::kBack) dtanh32(acc, a2r + c * kChunk + 32 * half, hv);
+          else bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
+          if (E::kLearn && h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv);
+          if constexpr (E::kBack) {
+            // backward: dL/dZ1 goes to global memory only
+          } else if (kPolicy) {
             // Write j = 2k + (c >> 1) of h2 buffer c & 1 reuses it after
             // layer 3 has consumed write j - 1 (completion j - 1 of h2_empty).
             const int j = 2 * k + (c >> 1);
@@ -599,6 +688,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           tc::mbar_arrive(&bar->h2_full[c & 1]);
         }
       }
+      if constexpr (E::kBack) return true;
       if (!kPolicy) {
         head[0] = (vsum.x + vsum.y) + *reinterpret_cast<const float*>(smem + kOffB3V);
         return true;
@@ -648,7 +738,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         float head[kHeadOut];
         __syncwarp();
         // every group with work runs T steps: the step index is t * n_act + g
-        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr))) break;
+        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr, nullptr, nullptr))) break;
         __syncwarp();
         if (active) {
           // The episode parameters are not held in registers across the
@@ -715,7 +805,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr))) break;
+        if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr, nullptr, nullptr))) break;
         __syncwarp();
         if (active) {
           const uint32_t id = M.id_base + (uint32_t)i;
@@ -751,8 +841,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         const size_t r = (size_t)(slot0 + g + it * n_slots) * kRows + row;
         const bool active = r < io.rows;
         float o[kObs];
-        if (active && io.xb) {
-          // bf16 row, 16-byte pieces (ldx >= obs_dim + 1, a multiple of 8)
+        if (E::kLearn && active) {
+          // bf16 row, 16-byte pieces (ldx a multiple of 8, >= obs_dim)
           const uint4* x = reinterpret_cast<const uint4*>(io.xb + r * (size_t)io.ldx);
 #pragma unroll
           for (int q = 0; q < (kObs + 7) / 8; ++q) {
@@ -783,12 +873,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
         __syncwarp();
-        uint16_t* h1r = active && io.h1 ? io.h1 + r * (size_t)io.ldh : nullptr;
-        uint16_t* h2r = active && io.h2 ? io.h2 + r * (size_t)io.ldh : nullptr;
-        if (!(ok = run_network(step_index<G>(it, g, iters), it, head, h1r, h2r))) break;
+        uint16_t* h1r = E::kLearn && active && io.h1 ? io.h1 + r * (size_t)io.ldh : nullptr;
+        uint16_t* h2r = E::kLearn && active && io.h2
+                            ? io.h2 + r * (size_t)(io.ldh2 ? io.ldh2 : io.ldh)
+                            : nullptr;
+        // backward mode: inactive rows read row 0's activations (results unused)
+        const size_t ra = active ? r : 0;
+        const uint16_t* a1r = E::kBack ? io.a1 + ra * (size_t)io.lda : nullptr;
+        const uint16_t* a2r = E::kBack ? io.a2 + ra * (size_t)io.lda : nullptr;
+        if (!(ok = run_network(step_index<G>(it, g, iters), it, head, h1r, h2r, a1r, a2r))) break;
         __syncwarp();
-        if (active) {
-          if (MODE == kValueRows) {
+        if (active && !E::kBack) {
+          if (!E::kPolicy) {
             io.out[r * (size_t)(io.ldo ? io.ldo : 1)] = head[0];
           } else {
             const size_t ldo = (size_t)(io.ldo ? io.ldo : io.out_dim);
@@ -885,6 +981,15 @@ cudaError_t launch_wait_selftest(Status* st, uint64_t limit_ns, cudaStream_t s) 
 
 size_t bf16_policy_image_bytes() { return kPolicyImage; }
 size_t bf16_value_image_bytes() { return kValueImage; }
+size_t bf16_back_image_bytes() { return kBackImage; }
+
+cudaError_t launch_pack_back_bf16(int in_dim, int out_dim, const float* w_f32, void* packed,
+                                  cudaStream_t s) {
+  const int pieces = kH * 4 + 4 * kH * 8;
+  k_pack_back<<<(pieces + 255) / 256, 256, 0, s>>>(w_f32, in_dim, out_dim,
+                                                   static_cast<uint8_t*>(packed));
+  return cudaGetLastError();
+}
 
 cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* wv_f32,
                              void* wp_packed, void* wv_packed, cudaStream_t s) {
@@ -915,7 +1020,8 @@ cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp
   const int G = pick_groups(tiles);
   const int grid = (int)((tiles + G - 1) / G);
   const uint8_t* img = static_cast<const uint8_t*>(wp_packed);
-  const RowIO io = {nullptr, 0, 1, nullptr, 0, 0, nullptr, 0, nullptr, nullptr, 0, 0};
+  const RowIO io = {nullptr, 0,       1, nullptr, 0, 0, nullptr, 0,
+                    nullptr, nullptr, 0, 0, nullptr, nullptr, 0, 0};
   if (M.model == 1) {
     switch (G) {
       case 4: return launch_engine<4, kRollout, 1>(grid, M, B, img, tr, T, t_g0, io, st, s);
@@ -951,7 +1057,7 @@ cudaError_t launch_value_bf16(const Model& M, const void* wv_packed, const float
                               cudaStream_t s) {
   (void)wv_f32;
   const RowIO io = {obs, rows, n, value, M.model == 1 ? 12 : kObs, 1,
-                    nullptr, 0, nullptr, nullptr, 0, 0};
+                    nullptr, 0, nullptr, nullptr, 0, 0, nullptr, nullptr, 0, 0};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), io, st, s);
 }
 
@@ -960,10 +1066,21 @@ cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_di
                                       uint16_t* h2, int ldh, float* out, int ldo, Status* st,
                                       cudaStream_t s) {
   const Model M{};
-  const RowIO io = {nullptr, rows, 1, out, in_dim, policy ? out_dim : 1, x, ldx, h1, h2, ldh, ldo};
+  const RowIO io = {nullptr, rows, 1,   out,     in_dim,  policy ? out_dim : 1, x, ldx, h1, h2,
+                    ldh,     ldo,  nullptr, nullptr, 0, 0};
   const uint8_t* img = static_cast<const uint8_t*>(packed);
-  return policy ? launch_rows<kPolicyRows>(M, img, io, st, s)
-                : launch_rows<kValueRows>(M, img, io, st, s);
+  return policy ? launch_rows<kLearnPolicy>(M, img, io, st, s)
+                : launch_rows<kLearnValue>(M, img, io, st, s);
+}
+
+cudaError_t launch_learn_backward_bf16(const void* packed, int out_dim, const uint16_t* gy, int ldy,
+                                       size_t rows, const uint16_t* h2, const uint16_t* h1, int ldh,
+                                       uint16_t* gz2, int ldz2, uint16_t* gz1, int ldz1, Status* st,
+                                       cudaStream_t s) {
+  const Model M{};
+  const RowIO io = {nullptr, rows, 1,  nullptr, out_dim, 1,  gy, ldy, gz2, gz1,
+                    ldz2,    0,    h2, h1,      ldh,     ldz1};
+  return launch_rows<kBackRows>(M, static_cast<const uint8_t*>(packed), io, st, s);
 }
 
 cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const void* wv_packed,
@@ -971,10 +1088,12 @@ cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const voi
                                 float* value, Status* st, cudaStream_t s) {
   (void)wv_f32;
   const int od = M.model == 1 ? 12 : kObs;
-  const RowIO io = {obs, (size_t)n, 1, head, od, M.policy_out, nullptr, 0, nullptr, nullptr, 0, 0};
+  const RowIO io = {obs, (size_t)n, 1, head, od, M.policy_out, nullptr, 0,
+                    nullptr, nullptr, 0, 0, nullptr, nullptr, 0, 0};
   cudaError_t e = launch_rows<kPolicyRows>(M, static_cast<const uint8_t*>(wp_packed), io, st, s);
   if (e != cudaSuccess || !value) return e;
-  const RowIO iov = {obs, (size_t)n, 1, value, od, 1, nullptr, 0, nullptr, nullptr, 0, 0};
+  const RowIO iov = {obs, (size_t)n, 1, value, od, 1, nullptr, 0,
+                     nullptr, nullptr, 0, 0, nullptr, nullptr, 0, 0};
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), iov, st, s);
 }
 

@@ -57,10 +57,11 @@ struct auv_ppo {
   float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
   ppo::StepCtl* ctl;          // device: per-step variables
   void* blas_ws;
-  // bf16 forward on the tensor-core engine: packed images of both networks,
-  // rebuilt from w every step, a flat staging copy and a status block
+  // bf16 forward and backward-data on the tensor-core engine: packed images
+  // of both networks (forward, and transposed for the backward), rebuilt
+  // from w every step, a flat staging copy and a status block
   bool eng = false;
-  void *img_p = nullptr, *img_v = nullptr;
+  void *img_p = nullptr, *img_v = nullptr, *img_bp = nullptr, *img_bv = nullptr;
   float* flat_eng = nullptr;
   Status* st = nullptr;
   uint64_t t, epoch;
@@ -137,7 +138,7 @@ int validate(const auv_ppo_config* c) {
     return fail(nullptr, AUV_ERR_INVALID, "minibatch outside [2, 2^22]");
   if (c->precision > AUV_PPO_BF16) return fail(nullptr, AUV_ERR_INVALID, "unknown precision %u", c->precision);
   if (c->norm_adv > 1) return fail(nullptr, AUV_ERR_INVALID, "norm_adv must be 0 or 1");
-  if (c->flags & ~(AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_FORWARD))
+  if (c->flags & ~(AUV_PPO_VALUE_ONLY | AUV_PPO_GEMM_PATH))
     return fail(nullptr, AUV_ERR_INVALID, "unknown flags %#x", c->flags);
   if (!(std::isfinite(c->clip_eps) && c->clip_eps > 0.0f))
     return fail(nullptr, AUV_ERR_INVALID, "clip_eps must be finite and > 0");
@@ -249,6 +250,22 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
   if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, out, d.B, p->h2[net], d.Hp, gy, ldy, g3, d.Hp,
                  true)))
     return blas_fail(p, bs, "gradient W3");
+  if (p->eng) {
+    // gZ2 and gZ1 (into the dead H2) on the tensor-core engine, then the
+    // weight gradients of layers 2 and 1
+    if ((e = auv::launch_learn_backward_bf16(
+             net ? p->img_bv : p->img_bp, out, static_cast<const uint16_t*>(gy), ldy, (size_t)d.B,
+             static_cast<const uint16_t*>(p->h2[net]), static_cast<const uint16_t*>(p->h1[net]), d.Hp,
+             static_cast<uint16_t*>(gz2), d.H, static_cast<uint16_t*>(gz1), d.Hp, p->st, s)))
+      return cuda_fail(p, e, "engine backward");
+    if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+                   true)))
+      return blas_fail(p, bs, "gradient W2");
+    if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+                   true)))
+      return blas_fail(p, bs, "gradient W1");
+    return AUV_OK;
+  }
   if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, out, w3, d.Hp, gy, ldy, gz2, d.H, false)))
     return blas_fail(p, bs, "gradient H2");
   if ((e = ppo::launch_tanh_bwd(p->bf16, gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
@@ -290,8 +307,12 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
     // images, then one launch per network writing H1, H2 and the head.
     if ((rc = convert(p, p->flat_eng, p->flat_eng + p->n_flat[0], p->w, false, s))) return rc;
     if ((e = auv::launch_pack_bf16_dims(d.D, p->out[0], d.value_only ? nullptr : p->flat_eng,
-                                   p->flat_eng + p->n_flat[0], p->img_p, p->img_v, s)))
+                                        p->flat_eng + p->n_flat[0], p->img_p, p->img_v, s)))
       return cuda_fail(p, e, "pack engine weights");
+    for (int net = d.value_only ? 1 : 0; net < 2; ++net)
+      if ((e = auv::launch_pack_back_bf16(d.D, p->out[net], p->flat_eng + (net ? p->n_flat[0] : 0),
+                                          net ? p->img_bv : p->img_bp, s)))
+        return cuda_fail(p, e, "pack engine backward weights");
     for (int net = d.value_only ? 1 : 0; net < 2; ++net) {
       if ((e = auv::launch_learn_forward_bf16(net == 0, net ? p->img_v : p->img_p, d.D, p->out[net],
                                          static_cast<const uint16_t*>(p->X), d.Dp, (size_t)d.B,
@@ -440,7 +461,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   }
   p->n_aug_all = p->n_aug[0] + p->n_aug[1];
   // the engine's networks: hidden 256, input <= 18, head <= 16 (2A <= 16)
-  p->eng = p->bf16 && d.H == 256 && d.D <= auv::kObs && !(cfg->flags & AUV_PPO_GEMM_FORWARD);
+  p->eng = p->bf16 && d.H == 256 && d.D <= auv::kObs && !(cfg->flags & AUV_PPO_GEMM_PATH);
   p->ctype = cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
   // one allocation, 256-byte aligned pieces
   const size_t B = (size_t)d.B, nb = (B + 255) / 256;
@@ -463,6 +484,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_ws = take(kBlasWorkspace),
                o_ip = take(p->eng ? auv::bf16_policy_image_bytes() : 0),
                o_iv = take(p->eng ? auv::bf16_value_image_bytes() : 0),
+               o_ibp = take(p->eng ? auv::bf16_back_image_bytes() : 0),
+               o_ibv = take(p->eng ? auv::bf16_back_image_bytes() : 0),
                o_fe = take(p->eng ? (p->n_flat[0] + p->n_flat[1]) * 4 : 0),
                o_st = take(sizeof(Status));
   size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
@@ -501,6 +524,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   if (p->eng) {
     p->img_p = base + o_ip;
     p->img_v = base + o_iv;
+    p->img_bp = base + o_ibp;
+    p->img_bv = base + o_ibv;
     p->flat_eng = reinterpret_cast<float*>(base + o_fe);
   }
   p->st = reinterpret_cast<Status*>(base + o_st);

@@ -373,13 +373,13 @@ def _grad_err(gpu, ref, n_pol):
                                                    (18, 8, 1000, 3, False),
                                                    (12, 6, 4096, 31, False)])
 def test_bf16_engine_forward(D, A, B, seed, calibrated):
-    """bf16 learners with hidden 256 run the forward pass on the tcgen05
-    engine (H1, H2 and the heads written for the cuBLAS backward): its
-    gradient and loss record against the oracle at a whole-tile and a ragged
-    minibatch and at the paper model's widths, and its error against that of
-    the same learner with the forward through cuBLAS GEMMs
-    (AUV_PPO_GEMM_FORWARD, which rounds the pre-activations to bf16 before
-    tanh); the status block stays clear.  Both paths are held to the
+    """bf16 learners with hidden 256 run the forward pass and the
+    backward-data (gZ2, gZ1) on the tcgen05 engine, the weight gradients on
+    cuBLAS: its gradient and loss record against the oracle at a whole-tile
+    and a ragged minibatch and at the paper model's widths, and its error
+    against that of the same learner with those products through cuBLAS GEMMs
+    and tanh passes (AUV_PPO_GEMM_PATH, which rounds each product to bf16
+    before its tanh or tanh'); the status block stays clear.  Both paths are held to the
     tolerance on the calibrated case (that of the tensor-core test above);
     on other draws the bf16 policy error of the GEMM path reaches 5e-2, so
     there the engine is held to twice the tolerance (a broken forward is
@@ -395,7 +395,7 @@ def test_bf16_engine_forward(D, A, B, seed, calibrated):
     grads, stats = {}, {}
     parts, g_ref = P.Learner(pw, vw, (D, H, A), hp, seed=7).grads(traj, 1, 0, B)
     for gemm in (True, False):
-        L = _learner(D, A, H, B, "bf16", gemm_forward=gemm, **hp)
+        L = _learner(D, A, H, B, "bf16", gemm_path=gemm, **hp)
         L.set_weights(pw, vw)
         grad = torch.empty(L.n_policy + L.n_value, device="cuda")
         st = torch.empty(8, device="cuda")
@@ -418,9 +418,10 @@ def test_bf16_engine_forward(D, A, B, seed, calibrated):
 
 def test_bf16_engine_update_repacks_every_step():
     """A captured multi-step update at a large learning rate: the engine
-    path's weights follow the GEMM path's step by step (the packed images
-    are rebuilt from the updated weights inside every replayed step; stale
-    images would leave the two apart by the size of the updates)."""
+    path's weights follow the GEMM path's step by step (the packed forward
+    and transposed images are rebuilt from the updated weights inside every
+    replayed step; stale images would leave the two apart by the size of the
+    updates)."""
     torch = need_gpu()
     D, A, H, T, N, B = 18, 8, 256, 4, 4096, 4096
     hp = dict(HP, **COHERENT, lr=3e-3, max_grad_norm=0.0)
@@ -430,7 +431,7 @@ def test_bf16_engine_update_repacks_every_step():
     dtraj = _dev(torch, traj)
     out = {}
     for gemm in (False, True):
-        L = _learner(D, A, H, B, "bf16", gemm_forward=gemm, **hp)
+        L = _learner(D, A, H, B, "bf16", gemm_path=gemm, **hp)
         L.set_weights(pw, vw)
         L.update(dtraj, 2, 4)
         assert L.status().code == 0
