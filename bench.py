@@ -355,8 +355,8 @@ def run_gae(args):
 # dram__bytes_write.sum, 1 pass, `bench.py --steps 1 --warmup 1 --no-e2e
 # --no-cpu-baseline --no-clocks`; profiles/k_engine_ppo_65536_T128_dram.md),
 # valid while the engine's sources hash to ENGINE_SRC_HASH.
-ROLLOUT_TRAFFIC_65536x128 = 10_751_232 + 902_867_200
-ENGINE_SRC_HASH = "77b2dd7b197aa46c"
+ROLLOUT_TRAFFIC_65536x128 = 10_783_232 + 902_189_056
+ENGINE_SRC_HASH = "a1bca85a644c154e"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 
