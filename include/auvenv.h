@@ -491,7 +491,13 @@ int ppo_apply(auv_ppo* p, const float* grad, float* stats, void* stream);
  * PPO update of one rollout; needs n_minibatches * B <= T * N.  stats, if not
  * NULL, receives the record averaged over the steps.  Asynchronous on
  * `stream`; the weights (ppo_get_weights, or the pointers of ppo_weights) are
- * the updated ones once it completes.
+ * the updated ones once it completes.  Each call first copies the batch into
+ * a sample-major buffer (T * N rows of round8(obs_dim + act_dim + 3) floats,
+ * one coalesced pass) from which every step gathers its minibatch; the
+ * learner allocates that buffer the first time it sees a batch of more rows
+ * than the last (the one allocation after ppo_create) and frees it in
+ * ppo_destroy.  If the allocation fails the steps gather from the batch's
+ * own arrays.
  */
 int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t n_minibatches,
                float* stats, void* stream);

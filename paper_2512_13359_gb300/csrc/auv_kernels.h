@@ -177,6 +177,15 @@ cudaError_t launch_gather(const Dims& d, const PermKey& k, const StepCtl* ctl, c
                           cudaStream_t s);
 cudaError_t launch_step_advance(StepCtl* ctl, cudaStream_t s);
 cudaError_t launch_tanh_fwd(bool bf16, void* h, int ld, int B, int H, cudaStream_t s);
+// Sample-major copy of a batch for the gather: rows of sample_row_floats(D, A)
+// floats (obs, act, logp, adv, ret, zero padding), row r = t N + i; act,
+// logp and adv may be NULL (value-only).  D + A + 3 <= 80.
+int sample_row_floats(int D, int A);
+cudaError_t launch_transpose_batch(int D, int A, uint32_t T, uint32_t N, const float* obs,
+                                   const float* act, const float* logp, const float* adv,
+                                   const float* ret, float* dst, cudaStream_t s);
+cudaError_t launch_gather_sm(const Dims& d, const PermKey& k, const StepCtl* ctl,
+                             const float* rows, const Sample& out, void* X, cudaStream_t s);
 cudaError_t launch_tanh_bwd(bool bf16, void* g, int ldg, const void* h, int ldh, int B, int H,
                             cudaStream_t s);
 // y [B][ld_pol], v [B][ld_val] fp32 head outputs; g_y, g_v the same shapes.

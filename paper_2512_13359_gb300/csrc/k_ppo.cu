@@ -274,6 +274,97 @@ __global__ void __launch_bounds__(kT) k_gather(Dims d, PermKey key, const StepCt
   }
 }
 
+// Sample-major copy of a batch: row r = t N + i holds, in Ws floats (Ws a
+// multiple of 8), obs[t][0..D), act[t][0..A), logp, adv, ret of (t, i), the
+// rest zero.  A block transposes 32 consecutive envs of one step through
+// shared memory: coalesced feature-major reads, one contiguous row-block
+// write.  Absent arrays (value-only batches) read as zero.
+constexpr int kSmRows = 32;
+constexpr int kSmMaxW = 80;   // round8(64 + 8 + 3)
+
+__global__ void __launch_bounds__(256) k_transpose_batch(int D, int A, int Ws, uint32_t N,
+                                                         const float* __restrict__ obs,
+                                                         const float* __restrict__ act,
+                                                         const float* __restrict__ logp,
+                                                         const float* __restrict__ adv,
+                                                         const float* __restrict__ ret,
+                                                         float* __restrict__ dst) {
+  __shared__ float tile[kSmRows][kSmMaxW + 1];
+  const uint32_t blocks_per_t = (N + kSmRows - 1) / kSmRows;
+  const size_t t = blockIdx.x / blocks_per_t;
+  const uint32_t i0 = (blockIdx.x % blocks_per_t) * kSmRows;
+  const int F = D + A + 3;
+  const size_t n = N;
+  for (int e = threadIdx.x; e < F * kSmRows; e += blockDim.x) {
+    const int f = e / kSmRows, row = e % kSmRows;
+    const uint32_t i = i0 + row;
+    float v = 0.0f;
+    if (i < N) {
+      if (f < D) v = __ldg(obs + (t * D + f) * n + i);
+      else if (f < D + A) v = act ? __ldg(act + (t * A + (f - D)) * n + i) : 0.0f;
+      else if (f == D + A) v = logp ? __ldg(logp + t * n + i) : 0.0f;
+      else if (f == D + A + 1) v = adv ? __ldg(adv + t * n + i) : 0.0f;
+      else v = __ldg(ret + t * n + i);
+    }
+    tile[row][f] = v;
+  }
+  __syncthreads();
+  const uint32_t rows = N - i0 < (uint32_t)kSmRows ? N - i0 : (uint32_t)kSmRows;
+  float* out = dst + (t * n + i0) * Ws;
+  for (int e = threadIdx.x; e < (int)rows * Ws; e += blockDim.x) {
+    const int row = e / Ws, col = e - row * Ws;
+    out[e] = col < F ? tile[row][col] : 0.0f;
+  }
+}
+
+// k_gather from the sample-major copy: one row of Ws floats per sample, read
+// in 16-byte pieces.
+template <typename TX>
+__global__ void __launch_bounds__(kT) k_gather_sm(Dims d, PermKey key, const StepCtl* ctl,
+                                                  const float* __restrict__ rows, int Ws,
+                                                  Sample out, TX* __restrict__ X) {
+  __shared__ double sh[2 * (kT / 32)];
+  const int b = blockIdx.x * kT + threadIdx.x;
+  const unsigned long long epoch = ctl->epoch0 + ctl->step / ctl->n_mb;
+  const uint32_t start = (ctl->step % ctl->n_mb) * (uint32_t)d.B;
+  key.e0 = (uint32_t)epoch;
+  key.e1 = (uint32_t)(epoch >> 32);
+  double s[2] = {0.0, 0.0};
+  if (b < d.B) {
+    const uint32_t r = perm_index(start + (uint32_t)b, key);
+    const float4* src = reinterpret_cast<const float4*>(rows + (size_t)r * Ws);
+    TX* x = X + (size_t)b * d.Dp;
+    const int F = d.D + d.A + 3;
+    float lp = 0.0f, a = 0.0f;
+    for (int q = 0; q < (F + 3) / 4; ++q) {
+      const float4 v4 = __ldg(src + q);
+      const float v[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int k = 4 * q + j;
+        if (k < d.D) st_act(x + k, v[j]);
+        else if (k < d.D + d.A) { if (!d.value_only) out.act[(size_t)b * d.A + (k - d.D)] = v[j]; }
+        else if (k == d.D + d.A) lp = v[j];
+        else if (k == d.D + d.A + 1) a = v[j];
+        else if (k == d.D + d.A + 2) out.ret[b] = v[j];
+      }
+    }
+    st_act(x + d.D, 1.0f);
+    for (int k = d.D + 1; k < d.Dp; ++k) st_act(x + k, 0.0f);
+    if (!d.value_only) {
+      out.logp[b] = lp;
+      out.adv[b] = a;
+      s[0] = a;
+      s[1] = (double)a * a;
+    }
+  }
+  block_sum<2>(s, sh);
+  if (threadIdx.x == 0) {
+    out.adv_part[2 * blockIdx.x] = s[0];
+    out.adv_part[2 * blockIdx.x + 1] = s[1];
+  }
+}
+
 __global__ void __launch_bounds__(kT) k_tanh_fwd(float* __restrict__ h, int ld, int B, int H4) {
   const size_t n = (size_t)B * H4;
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
@@ -573,6 +664,30 @@ cudaError_t launch_gather(const Dims& d, const PermKey& k, const StepCtl* ctl, c
   else
     k_gather<<<nb, kT, 0, s>>>(d, k, ctl, obs, act, logp, adv, ret, N, out,
                                static_cast<float*>(X));
+  return cudaGetLastError();
+}
+
+int sample_row_floats(int D, int A) { return (D + A + 3 + 7) & ~7; }
+
+cudaError_t launch_transpose_batch(int D, int A, uint32_t T, uint32_t N, const float* obs,
+                                   const float* act, const float* logp, const float* adv,
+                                   const float* ret, float* dst, cudaStream_t s) {
+  const int Ws = sample_row_floats(D, A);
+  if (Ws > kSmMaxW) return cudaErrorInvalidValue;
+  const size_t blocks = (size_t)T * ((N + kSmRows - 1) / kSmRows);
+  if (blocks == 0 || blocks > 0x7fffffffu) return cudaErrorInvalidValue;
+  k_transpose_batch<<<(unsigned)blocks, 256, 0, s>>>(D, A, Ws, N, obs, act, logp, adv, ret, dst);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_sm(const Dims& d, const PermKey& k, const StepCtl* ctl,
+                             const float* rows, const Sample& out, void* X, cudaStream_t s) {
+  const unsigned nb = (d.B + kT - 1) / kT;
+  const int Ws = sample_row_floats(d.D, d.A);
+  if (d.bf16)
+    k_gather_sm<<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, static_cast<__nv_bfloat16*>(X));
+  else
+    k_gather_sm<<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, static_cast<float*>(X));
   return cudaGetLastError();
 }
 

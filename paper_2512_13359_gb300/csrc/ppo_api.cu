@@ -14,7 +14,10 @@
 // weight copy, a flat staging vector, the gathered minibatch, and per
 // network the activations H1, H2 [B][Hp] (constant 1 at column H), the
 // backward buffer G [B][H] and the head output Y [B][ld].  Everything a step
-// touches is resident; no call after ppo_create allocates.
+// touches is resident.  ppo_update adds one separate allocation: a
+// sample-major copy of its batch (rows of round8(D + A + 3) floats), made
+// once per call, from which every step gathers its minibatch; it grows when a
+// larger batch arrives and lives until ppo_destroy.
 #include <cublas_v2.h>
 
 #include <cmath>
@@ -64,6 +67,12 @@ struct auv_ppo {
   void *img_p = nullptr, *img_v = nullptr, *img_bp = nullptr, *img_bv = nullptr;
   float* flat_eng = nullptr;
   Status* st = nullptr;
+  // sample-major copy of the batch of the current ppo_update (use_sm while
+  // that update's steps are enqueued); the step graph records which copy
+  float* sm_buf = nullptr;
+  size_t sm_rows = 0;
+  bool use_sm = false;
+  const float* graph_sm = nullptr;
   uint64_t t, epoch;
   // One gradient step captured as a CUDA graph for ppo_update, replayed on a
   // private stream; valid for the batch it was captured with.
@@ -298,8 +307,10 @@ int convert(auv_ppo* p, float* flat_pol, float* flat_val, float* aug, bool to_au
 int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
   const ppo::Dims& d = p->d;
   const uint32_t m = b->T * b->N;
-  cudaError_t e = ppo::launch_gather(d, perm_key(p, m, 0), p->ctl, b->obs, b->act, b->logp,
-                                     b->adv, b->ret, b->N, p->smp, p->X, s);
+  cudaError_t e =
+      p->use_sm ? ppo::launch_gather_sm(d, perm_key(p, m, 0), p->ctl, p->sm_buf, p->smp, p->X, s)
+                : ppo::launch_gather(d, perm_key(p, m, 0), p->ctl, b->obs, b->act, b->logp, b->adv,
+                                     b->ret, b->N, p->smp, p->X, s);
   if (e != cudaSuccess) return cuda_fail(p, e, "gather");
   int rc;
   if (p->eng) {
@@ -384,6 +395,7 @@ bool capture_step(auv_ppo* p, const auv_ppo_batch* b) {
     return false;
   }
   p->graph_batch = *b;
+  p->graph_sm = p->use_sm ? p->sm_buf : nullptr;
   return true;
 }
 
@@ -574,6 +586,7 @@ int ppo_destroy(auv_ppo* p) {
   if (p->ev_out) cudaEventDestroy(p->ev_out);
   if (p->gstream) cudaStreamDestroy(p->gstream);
   cublasDestroy(p->blas);
+  if (p->sm_buf) cudaFree(p->sm_buf);
   cudaFree(p->mem);
   if (prev >= 0) cudaSetDevice(prev);
   delete p;
@@ -731,8 +744,28 @@ int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t
   if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const uint64_t steps = (uint64_t)epochs * n_minibatches;
+  // The sample-major copy: grown when a larger batch arrives (cudaFree waits
+  // for the work that may still read the old one); without it the steps
+  // gather from the batch's own arrays.
+  const size_t rows = (size_t)batch->T * batch->N;
+  const int ws = ppo::sample_row_floats(p->d.D, p->d.A);
+  if (p->sm_rows < rows) {
+    if (p->sm_buf) cudaFree(p->sm_buf);
+    p->sm_buf = nullptr;
+    p->sm_rows = 0;
+    if (cudaMalloc(&p->sm_buf, rows * ws * sizeof(float)) == cudaSuccess) p->sm_rows = rows;
+    else p->sm_buf = nullptr;
+    cudaGetLastError();
+  }
+  p->use_sm = p->sm_buf != nullptr;
+  struct SmScope {   // the copy serves this update's steps only (ppo_grads gathers directly)
+    auv_ppo* q;
+    ~SmScope() { q->use_sm = false; }
+  } sm_scope{p};
   // replay the captured step on the private stream when it can be had
-  if (!p->graph_failed && (!p->step_graph || !same_batch(p->graph_batch, *batch)) &&
+  if (!p->graph_failed &&
+      (!p->step_graph || !same_batch(p->graph_batch, *batch) ||
+       p->graph_sm != (p->use_sm ? p->sm_buf : nullptr)) &&
       !capture_step(p, batch))
     p->graph_failed = true;
   const bool graph = p->step_graph != nullptr && !p->graph_failed;
@@ -749,6 +782,12 @@ int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t
   if ((rc = set_ctl(p, p->epoch, n_minibatches, 0, p->t, r))) return rc;
   if ((e = cudaMemsetAsync(p->acc, 0, AUV_PPO_STATS * 4, r)))
     return cuda_fail(p, e, "clear statistics");
+  if (p->use_sm && (e = ppo::launch_transpose_batch(p->d.D, p->d.A, batch->T, batch->N, batch->obs,
+                                                     p->d.value_only ? nullptr : batch->act,
+                                                     p->d.value_only ? nullptr : batch->logp,
+                                                     p->d.value_only ? nullptr : batch->adv,
+                                                     batch->ret, p->sm_buf, r)))
+    return cuda_fail(p, e, "sample-major batch copy");
   for (uint64_t k = 0; k < steps; ++k) {
     if (graph) {
       if ((e = cudaGraphLaunch(p->step_graph, r))) return cuda_fail(p, e, "launch step graph");
