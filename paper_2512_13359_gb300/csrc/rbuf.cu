@@ -61,19 +61,29 @@ __global__ void __launch_bounds__(256) k_rb_insert(int T, int N, int D, int A,
     const int i0 = (blockIdx.x * kTilesPerBlock + tile) * kTile;
     if (i0 >= N) break;
     const int i = i0 + lane;
-    // load: feature f of env i (coalesced along envs)
-    for (int f = row0; f < F; f += rows) {
-      float v = 0.0f;
-      if (i < N) {
-        if (f < D) v = __ldg(obs + ((size_t)t * D + f) * n + i);
-        else if (f < D + A) v = __ldg(act + ((size_t)t * A + (f - D)) * n + i);
-        else {
-          const int k = f - D - A;
-          v = (t + 1 < T) ? __ldg(obs + ((size_t)(t + 1) * D + k) * n + i)
-                          : __ldg(last_obs + (size_t)k * n + i);
+    // load: feature f of env i (coalesced along envs), eight features per
+    // thread in flight before any is stored
+    for (int f0 = row0; f0 < F; f0 += 8 * rows) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int f = f0 + u * rows;
+        v[u] = 0.0f;
+        if (i < N && f < F) {
+          if (f < D) v[u] = __ldg(obs + ((size_t)t * D + f) * n + i);
+          else if (f < D + A) v[u] = __ldg(act + ((size_t)t * A + (f - D)) * n + i);
+          else {
+            const int k = f - D - A;
+            v[u] = (t + 1 < T) ? __ldg(obs + ((size_t)(t + 1) * D + k) * n + i)
+                               : __ldg(last_obs + (size_t)k * n + i);
+          }
         }
       }
-      sm[f * (kTile + 1) + lane] = v;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int f = f0 + u * rows;
+        if (f < F) sm[f * (kTile + 1) + lane] = v[u];
+      }
     }
     __syncthreads();
     const int cnt = min(kTile, N - i0);
