@@ -71,6 +71,8 @@ def parse():
                     help="time the inverse thruster allocation over the envs")
     ap.add_argument("--gae", action="store_true",
                     help="advantage estimation (env_gae) over one rollout, HBM roofline")
+    ap.add_argument("--probes", action="store_true",
+                    help="roofline probes: FFMA chain, tanh.approx.f32 chain, cuBLAS tf32/bf16 GEMM")
     ap.add_argument("--sweep", action="store_true",
                     help="batch-size sweep 1,024 .. 1,048,576 envs x 256 steps (one line per size)")
     return ap.parse_args()
@@ -286,6 +288,69 @@ def run_replay(args):
                      "unit": "TFLOP/s", "frac": achieved / fp32_peak, "traffic": None,
                      "peak_source": f"FP32 pipe 2*128*{n_sm} SMs*{sm_mhz:.0f} MHz"},
         "gpu_launches": args.steps, "clocks": clock_info,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_probes(args):
+    """The roofline denominators measured with the library's probes: the FP32
+    pipe (FFMA chains at full occupancy) against 2 x 128 x SMs x clock, the
+    multi-function unit (tanh.approx.f32 chains), and the tensor pipe for
+    tf32 and bf16 operands (one 8192^3 cuBLAS GEMM each)."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv, build
+    build.build()
+    torch.cuda.init()
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    blocks, threads = sms * 8, 256
+    sink = torch.zeros(blocks * threads, device="cuda")
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            work = fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append((e0.elapsed_time(e1) * 1e-3, work))
+        ts.sort()
+        t, work = ts[len(ts) // 2]
+        return work / t
+
+    clocks = ClockSampler(0) if not args.no_clocks else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ffma = timed(lambda: auvenv.probe_ffma(blocks, threads, 20000, sink), max(args.steps, 5))
+    tanh = timed(lambda: auvenv.probe_tanh(blocks, threads, 4000, sink), max(args.steps, 5))
+    n = 8192
+    g = torch.Generator(device="cuda").manual_seed(0)
+    a32 = torch.randn(n, n, device="cuda", generator=g)
+    b32 = torch.randn(n, n, device="cuda", generator=g)
+    c32 = torch.empty(n, n, device="cuda")
+    tf32 = timed(lambda: auvenv.probe_gemm("tf32", a32, b32, c32), max(args.steps, 5))
+    a16, b16 = a32.to(torch.bfloat16), b32.to(torch.bfloat16)
+    bf16 = timed(lambda: auvenv.probe_gemm("bf16", a16, b16, c32), max(args.steps, 5))
+    torch.cuda.synchronize()
+    clock_info = clocks.stop() if clocks else None
+    peaks, src = load_peaks()
+    mhz = (clock_info or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+    derived = 2 * 128 * sms * mhz * 1e6
+    line = {
+        "metric": "roofline probes", "n_gpus": 1, "steps": max(args.steps, 5), "data": "synthetic",
+        "probes": {
+            "fp32_ffma_tflops": ffma / 1e12, "fp32_derived_tflops": derived / 1e12,
+            "fp32_ffma_frac_of_derived": ffma / derived,
+            "mufu_tanh_gops": tanh / 1e9,
+            "mufu_tanh_per_clk_per_sm": tanh / (sms * mhz * 1e6),
+            "tf32_gemm_tflops": tf32 / 1e12, "bf16_gemm_tflops": bf16 / 1e12,
+            "bf16_peak_measured_tflops": peaks.get("bf16_tflops"),
+            "tf32_over_bf16": tf32 / bf16, "nominal_tf32_over_bf16": 1.1 / 2.25,
+            "gemm_n": n, "sms": sms, "sm_mhz_used": mhz, "peaks_source": src},
+        "clocks": clock_info,
     }
     print(json.dumps(line), flush=True)
 
@@ -717,6 +782,9 @@ def main():
         return
     if args.gae:
         run_gae(args)
+        return
+    if args.probes:
+        run_probes(args)
         return
     if args.sweep:
         base_steps = args.steps

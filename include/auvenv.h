@@ -651,6 +651,26 @@ int env_clear_status(auv_env* env, void* stream);
  */
 int env_selftest_wait_timeout(auv_env* env, uint32_t limit_us, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Roofline probes (measurement helpers, not on any hot path).  Each enqueues
+ * work of a known operation count on `stream`; the caller times it.
+ *
+ * auv_probe_ffma: blocks x threads threads, each running `iters` rounds of 8
+ *   independent dependent FMAs: 16 * iters flop per thread (the FP32 pipe).
+ * auv_probe_tanh: the same shape with tanh.approx.f32: 8 * iters operations
+ *   per thread (the multi-function unit).
+ *   blocks in [1, 65535], threads a multiple of 32 in [32, 1024], iters >= 1;
+ *   sink: device memory of blocks * threads floats (written only to keep the
+ *   work from being removed).
+ * auv_probe_gemm: one n x n x n cuBLAS GEMM, C = A B (column-major, fp32 C),
+ *   with A, B fp32 and tf32 tensor-core math (AUV_PPO_TF32) or bf16 operands
+ *   (AUV_PPO_BF16): 2 n^3 flop.  n a multiple of 16.
+ * Return AUV_OK, AUV_ERR_INVALID on bad arguments or AUV_ERR_CUDA.
+ * --------------------------------------------------------------------------- */
+int auv_probe_ffma(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream);
+int auv_probe_tanh(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream);
+int auv_probe_gemm(uint32_t precision, int n, const void* a, const void* b, void* c, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

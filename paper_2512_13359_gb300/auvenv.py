@@ -46,7 +46,8 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "rbuf_size", "rbuf_insert", "rbuf_sample",
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
-            "ppo_update", "ppo_export_weights", "ppo_status", "ppo_clear_status")
+            "ppo_update", "ppo_export_weights", "ppo_status", "ppo_clear_status",
+            "auv_probe_ffma", "auv_probe_tanh", "auv_probe_gemm")
 
 
 class LibraryMissing(RuntimeError):
@@ -182,6 +183,9 @@ def lib(path: str | None = None):
     L.ppo_apply.argtypes = [P, P, P, P]
     L.ppo_update.argtypes = [P, C.POINTER(PpoBatch), U32, U32, P, P]
     L.ppo_status.argtypes = [P, C.POINTER(AuvStatus), P]
+    L.auv_probe_ffma.argtypes = [U32, U32, U32, P, P]
+    L.auv_probe_tanh.argtypes = [U32, U32, U32, P, P]
+    L.auv_probe_gemm.argtypes = [U32, I, P, P, P, P]
     L.ppo_clear_status.argtypes = [P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
@@ -537,6 +541,31 @@ class Learner:
 
     def clear_status(self, stream=None):
         self._check(lib().ppo_clear_status(self.h, _stream(stream)))
+
+
+def _probe_check(rc, what):
+    if rc != AUV_OK:
+        raise AuvError(rc, f"{what} failed")
+
+
+def probe_ffma(blocks: int, threads: int, iters: int, sink, stream=None) -> int:
+    """Enqueue the FFMA-chain probe; returns its flop count (16 per thread-iteration)."""
+    _probe_check(lib().auv_probe_ffma(blocks, threads, iters, _ptr(sink), _stream(stream)), "ffma probe")
+    return 16 * blocks * threads * iters
+
+
+def probe_tanh(blocks: int, threads: int, iters: int, sink, stream=None) -> int:
+    """Enqueue the tanh.approx.f32 probe; returns its operation count."""
+    _probe_check(lib().auv_probe_tanh(blocks, threads, iters, _ptr(sink), _stream(stream)), "tanh probe")
+    return 8 * blocks * threads * iters
+
+
+def probe_gemm(precision: str, a, b, c, stream=None) -> int:
+    """Enqueue one n x n x n cuBLAS GEMM (tf32 on fp32 operands, or bf16); returns 2 n^3."""
+    n = int(a.shape[0])
+    _probe_check(lib().auv_probe_gemm(PPO_PRECISION[precision], n, _ptr(a), _ptr(b), _ptr(c),
+                                      _stream(stream)), "gemm probe")
+    return 2 * n ** 3
 
 
 class ReplayBuffer:
