@@ -190,6 +190,58 @@ def oracle_sample_rate(w, T, target_s, max_envs=4096):
         n = min(max_envs, max(n * 2, int(n * target_s / max(dt, 1e-3)) + 1))
 
 
+def _oracle_worker(w, jobs, results):
+    """Worker process of OraclePool: runs the oracle rollout of env ids
+    [lo, lo + n) for each job (lo, n, T) and reports its seconds."""
+    m, Batch, reset, rollout = oracle_api(w)
+    pw = W.policy_weights(w)
+    vw = W.value_weights(w) if w["has_value"] else None
+    while True:
+        job = jobs.get()
+        if job is None:
+            return
+        lo, n, T = job
+        b = Batch(np.arange(lo, lo + n))
+        reset(m, b)
+        t0 = time.perf_counter()
+        rollout(m, b, pw, vw, 0, T)
+        results.put(time.perf_counter() - t0)
+
+
+class OraclePool:
+    """The unchanged oracle on every host core: one spawned process per core
+    (spawn, so that no process inherits a CUDA context), each on its own
+    range of env ids.  run(n, T) rolls n envs per process over T steps and
+    returns the wall seconds of the whole batch."""
+
+    def __init__(self, w, cores=None):
+        import multiprocessing as mp
+        from oracle import oracle as O
+        O.build()
+        self.cores = cores or len(os.sched_getaffinity(0))
+        ctx = mp.get_context("spawn")
+        self.jobs, self.results = ctx.Queue(), ctx.Queue()
+        self.procs = [ctx.Process(target=_oracle_worker, args=(w, self.jobs, self.results),
+                                  daemon=True) for _ in range(self.cores)]
+        for p in self.procs:
+            p.start()
+        self.run(1, 1)      # every worker has loaded the oracle
+
+    def run(self, n, T):
+        t0 = time.perf_counter()
+        for k in range(self.cores):
+            self.jobs.put((k * n, n, T))
+        for _ in range(self.cores):
+            self.results.get()
+        return time.perf_counter() - t0
+
+    def close(self):
+        for _ in self.procs:
+            self.jobs.put(None)
+        for p in self.procs:
+            p.join(timeout=10)
+
+
 def run_reference(args, w):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -197,24 +249,20 @@ def run_reference(args, w):
     from oracle import oracle as O
     O.build()
     T = w["steps"]
-    m, Batch, reset, rollout = oracle_api(w)
-    pw = W.policy_weights(w)
-    vw = W.value_weights(w) if w["has_value"] else None
-    # size one bench step so that K + W steps take about a minute in total
+    # size one bench step so that K + W steps take about a minute in total;
+    # each step rolls n envs on every host core (disjoint env-id ranges)
     rate, _, _ = oracle_sample_rate(w, T, 2.0)
     per_step_s = max(1.0, 60.0 / max(1, args.steps + args.warmup))
     n = max(1, int(rate * per_step_s / T))
-    times = []
-    for s in range(args.warmup + args.steps):
-        b = Batch(np.arange(n))
-        reset(m, b)
-        t0 = time.perf_counter()
-        rollout(m, b, pw, vw, 0, T)
-        if s >= args.warmup:
-            times.append(time.perf_counter() - t0)
+    pool = OraclePool(w)
+    try:
+        times = [pool.run(n, T) for _ in range(args.warmup + args.steps)][args.warmup:]
+    finally:
+        pool.close()
     sec = sum(times) / len(times)
-    value = n * T / sec
-    sample = f"{n} envs x {T} steps of {w['name']} per step (env ids 0..{n - 1})"
+    value = pool.cores * n * T / sec
+    sample = (f"{n} envs x {T} steps of {w['name']} per process per step, {pool.cores} "
+              f"processes on disjoint env ids (0..{pool.cores * n - 1})")
     line = {
         "impl": "reference", "metric": "env-steps/s (physics+policy+reward)", "value": value,
         "unit": "env-steps/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -222,8 +270,8 @@ def run_reference(args, w):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w["name"], "n_envs": w["n_envs"], "rollout_steps": T,
                    "substeps": w["substeps"], "mlp": w["mlp"], "sample_envs": n},
-        "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": pool.cores,
+                         "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "env-steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -951,8 +999,17 @@ def run(args):
         from oracle import oracle as O
         O.build()
         rate, n_s, dt = oracle_sample_rate(w, T, args.cpu_seconds)
-        cpu = {"value": rate, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
-               "sample": f"{n_s} envs x {T} steps of {w['name']} ({dt:.1f} s, one thread)"}
+        # then the same sample on every host core at once (disjoint env ids)
+        pool = OraclePool(w)
+        try:
+            wall = pool.run(n_s, T)
+        finally:
+            pool.close()
+        cpu = {"value": pool.cores * n_s * T / wall, "unit": "env-steps/s", "cores": pool.cores,
+               "kind": "oracle", "one_core": rate,
+               "sample": (f"{n_s} envs x {T} steps of {w['name']} per process, {pool.cores} "
+                          f"processes ({wall:.1f} s wall); one thread alone {rate:.0f} "
+                          f"env-steps/s ({dt:.1f} s)")}
 
     launches_per_step = 1 + (1 if value is not None else 0)
     line = {
