@@ -362,11 +362,21 @@ __global__ void __launch_bounds__(kAdjThreads, 4) k_adjoint(
   Env e;
   load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   uint64_t ends = 0;
+  // Step t + 1's actions are loaded while step t integrates (and step t - 1's
+  // while the reverse sweep differentiates step t).
+  float a_next[kAct];
+#pragma unroll
+  for (int k = 0; k < kAct; ++k) a_next[k] = T > 0 ? __ldg(act + (size_t)k * n + i) : 0.0f;
   for (int t = 0; t < T; ++t) {
     save_step(scratch + (size_t)t * kScratchF * n, n, i, e);
     float a[kAct];
 #pragma unroll
-    for (int k = 0; k < kAct; ++k) a[k] = __ldg(act + ((size_t)t * kAct + k) * n + i);
+    for (int k = 0; k < kAct; ++k) a[k] = a_next[k];
+    if (t + 1 < T) {
+#pragma unroll
+      for (int k = 0; k < kAct; ++k)
+        a_next[k] = __ldg(act + ((size_t)(t + 1) * kAct + k) * n + i);
+    }
     bool d;
     const float r = physics_step(M, id, e, a, &d);
     if (d) ends |= 1ull << t;
@@ -382,6 +392,9 @@ __global__ void __launch_bounds__(kAdjThreads, 4) k_adjoint(
     else lx.nu[k - 7] = v;
   }
   X xs[8];
+#pragma unroll
+  for (int k = 0; k < kAct; ++k)
+    a_next[k] = T > 0 ? __ldg(act + ((size_t)(T - 1) * kAct + k) * n + i) : 0.0f;
   for (int t = T - 1; t >= 0; --t) {
     if ((ends >> t) & 1ull) {
 #pragma unroll
@@ -395,7 +408,11 @@ __global__ void __launch_bounds__(kAdjThreads, 4) k_adjoint(
     load_step(M, scratch + (size_t)t * kScratchF * n, n, i, es);
     float a[kAct], a_c[kAct], tau[6], nup[6];
 #pragma unroll
-    for (int k = 0; k < kAct; ++k) a[k] = __ldg(act + ((size_t)t * kAct + k) * n + i);
+    for (int k = 0; k < kAct; ++k) a[k] = a_next[k];
+    if (t > 0) {
+#pragma unroll
+      for (int k = 0; k < kAct; ++k) a_next[k] = __ldg(act + ((size_t)(t - 1) * kAct + k) * n + i);
+    }
     allocate(M, a, a_c, tau);
 #pragma unroll
     for (int k = 0; k < 6; ++k) nup[k] = es.nu[k];
@@ -886,11 +903,21 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
   paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   for (int r = 13; r < paper::kStateF; ++r) hsc[r * n + i] = B.state[r * n + i];
   uint64_t ends = 0;
+  // Step t + 1's actions are loaded while step t integrates (and step t - 1's
+  // while the reverse sweep differentiates step t).
+  float a_next[paper::kAct];
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k) a_next[k] = T > 0 ? __ldg(act + (size_t)k * n + i) : 0.0f;
   for (int t = 0; t < T; ++t) {
     paper_save_step(M, e, hsc, scratch + (size_t)t * kPScratchF * n, n, i);
     float a[paper::kAct];
 #pragma unroll
-    for (int k = 0; k < paper::kAct; ++k) a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
+    for (int k = 0; k < paper::kAct; ++k) a[k] = a_next[k];
+    if (t + 1 < T) {
+#pragma unroll
+      for (int k = 0; k < paper::kAct; ++k)
+        a_next[k] = __ldg(act + ((size_t)(t + 1) * paper::kAct + k) * n + i);
+    }
     bool d;
     const float r = paper::physics_step(M, id, e, a, hsc, i, &d);
     if (d) ends |= 1ull << t;
@@ -909,6 +936,9 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
   for (int j = 0; j < paper::kHist; ++j)
 #pragma unroll
     for (int k = 0; k < 6; ++k) lh[j][k] = lam_T ? __ldg(lam_T + (13 + 6 * j + k) * n + i) : 0.0f;
+#pragma unroll
+  for (int k = 0; k < paper::kAct; ++k)
+    a_next[k] = T > 0 ? __ldg(act + ((size_t)(T - 1) * paper::kAct + k) * n + i) : 0.0f;
   for (int t = T - 1; t >= 0; --t) {
     if ((ends >> t) & 1ull) {
 #pragma unroll
@@ -923,7 +953,12 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
     }
     float a[paper::kAct], la[paper::kAct];
 #pragma unroll
-    for (int k = 0; k < paper::kAct; ++k) a[k] = __ldg(act + ((size_t)t * paper::kAct + k) * n + i);
+    for (int k = 0; k < paper::kAct; ++k) a[k] = a_next[k];
+    if (t > 0) {
+#pragma unroll
+      for (int k = 0; k < paper::kAct; ++k)
+        a_next[k] = __ldg(act + ((size_t)(t - 1) * paper::kAct + k) * n + i);
+    }
     paper_step_vjp(M, scratch + (size_t)t * kPScratchF * n, n, i, a, __ldg(coef + t), lx, lh, la);
 #pragma unroll
     for (int k = 0; k < paper::kAct; ++k)

@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(256) k_reset(const Model M, Buffers B, const u
 // ---------------------------------------------------------------------------
 // Action replay: T control steps with given actions act[T][8][N].
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(128) k_replay(const Model M, Buffers B,
+__global__ void __launch_bounds__(128, 4) k_replay(const Model M, Buffers B,
                                                 const float* __restrict__ act, int T,
                                                 float* __restrict__ rew, uint8_t* __restrict__ done,
                                                 float* __restrict__ trace, Status* st) {
@@ -35,10 +35,20 @@ __global__ void __launch_bounds__(128) k_replay(const Model M, Buffers B,
   Env e;
   load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   bool bad = false;
+  // Step t + 1's actions are loaded while step t integrates, so their DRAM
+  // latency is hidden behind a step of arithmetic.
+  float a_next[kAct];
+#pragma unroll
+  for (int k = 0; k < kAct; ++k) a_next[k] = T > 0 ? __ldg(act + (size_t)k * n + i) : 0.0f;
   for (int t = 0; t < T; ++t) {
     float a[kAct];
 #pragma unroll
-    for (int k = 0; k < kAct; ++k) a[k] = __ldg(act + ((size_t)t * kAct + k) * n + i);
+    for (int k = 0; k < kAct; ++k) a[k] = a_next[k];
+    if (t + 1 < T) {
+#pragma unroll
+      for (int k = 0; k < kAct; ++k)
+        a_next[k] = __ldg(act + ((size_t)(t + 1) * kAct + k) * n + i);
+    }
     bool d;
     const float r = physics_step(M, M.id_base + (uint32_t)i, e, a, &d);
     rew[(size_t)t * n + i] = r;

@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(256) k_paper_reset(const Model M, Buffers B,
   paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
 }
 
-__global__ void __launch_bounds__(128) k_paper_replay(const Model M, Buffers B,
+__global__ void __launch_bounds__(128, 4) k_paper_replay(const Model M, Buffers B,
                                                       const float* __restrict__ act, int T,
                                                       float* __restrict__ rew,
                                                       uint8_t* __restrict__ done, float* trace,
@@ -36,10 +36,20 @@ __global__ void __launch_bounds__(128) k_paper_replay(const Model M, Buffers B,
   paper::Env e;
   paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   bool bad = false;
+  // Step t + 1's actions are loaded while step t integrates, so their DRAM
+  // latency is hidden behind a step of arithmetic.
+  float a_next[kAct];
+#pragma unroll
+  for (int k = 0; k < kAct; ++k) a_next[k] = T > 0 ? __ldg(act + (size_t)k * n + i) : 0.0f;
   for (int t = 0; t < T; ++t) {
     float a[kAct];
 #pragma unroll
-    for (int k = 0; k < kAct; ++k) a[k] = __ldg(act + ((size_t)t * kAct + k) * n + i);
+    for (int k = 0; k < kAct; ++k) a[k] = a_next[k];
+    if (t + 1 < T) {
+#pragma unroll
+      for (int k = 0; k < kAct; ++k)
+        a_next[k] = __ldg(act + ((size_t)(t + 1) * kAct + k) * n + i);
+    }
     bool d;
     const float r = paper::physics_step(M, M.id_base + (uint32_t)i, e, a, B.state, i, &d);
     rew[(size_t)t * n + i] = r;
