@@ -261,7 +261,7 @@ int env_reset(auv_env* env, const uint8_t* mask, void* stream);
  * In AUV_MLP_BF16 mode traj.value (if given) comes from a value-network pass
  * over traj.obs after the steps, so traj.obs is required with it.
  * Host arrays (T >= 2): the steps run in segments into two device staging
- * buffers (allocated on the first such call, about 2 x 128 MiB, kept until
+ * buffers (allocated on the first such call, about 2 x 64 MiB, kept until
  * env_destroy); each finished segment is copied to the host arrays on a
  * copy stream of the env while the next segment computes.  `stream` waits
  * for the last copy, so its completion still means every array is written.

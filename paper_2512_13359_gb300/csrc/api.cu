@@ -486,9 +486,9 @@ int rollout_staged(auv_env* env, int T, const auv_traj* traj, Traj mapped,
   size_t step_bytes = 0;
   for (int k = 0; k < kTrajArrays; ++k)
     if (host[k]) step_bytes += row[k];
-  // about 128 MiB per segment buffer: a power of two of steps in [4, T]
+  // about 64 MiB per segment buffer: a power of two of steps in [4, T]
   int seg = 4;
-  while (seg < T && (size_t)(2 * seg) * step_bytes <= ((size_t)1 << 27)) seg *= 2;
+  while (seg < T && (size_t)(2 * seg) * step_bytes <= ((size_t)1 << 26)) seg *= 2;
   if (seg > T) seg = T;
   size_t off[kTrajArrays], half = 0;
   for (int k = 0; k < kTrajArrays; ++k) {
