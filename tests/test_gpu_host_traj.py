@@ -37,8 +37,9 @@ def _run(w, T, placement, calls=2):
 
 @pytest.mark.parametrize("n,T", [(65536, 37), (1000, 9)])
 def test_host_trajectory_matches_device(n, T):
-    """65,536 envs x 37 steps runs as segments of 16, 16, 5 (both staging
-    buffers, then reuse); 1,000 envs x 9 steps is a single segment."""
+    """65,536 envs x 37 steps runs as segments of 8, 8, 8, 8, 5 (each staging
+    buffer used three or two times); 1,000 envs x 9 steps is a single
+    segment."""
     need_gpu()
     w = W.workload("ppo_65536", n_envs=n)
     dev_out, dev_state = _run(w, T, {k: "device" for k in KEYS})
