@@ -281,3 +281,42 @@ def test_rollout_log_probability_and_dones(oracle):
             lp = np.sum(norm.logpdf(a, loc=mu[i], scale=np.exp(ls)))
             assert out["logp"][t, i] == pytest.approx(lp, rel=1e-12)
     assert np.array_equal(out["done"][:, 0], [(t + 1) % L == 0 for t in range(T)])
+
+
+def _golden_setup():
+    import os
+    vals = {}
+    with open(os.path.join(os.path.dirname(__file__), "golden", "paper_setup.txt")) as f:
+        for line in f:
+            line = line.split("#", 1)[0].split()
+            if line:
+                vals[line[0]] = float(line[1])
+    return vals
+
+
+def test_golden_paper_setup(oracle):
+    """The task constants the paper prints (golden/paper_setup.txt, each line
+    cited: §IV-A, §IV-B1, §IV-B2, §V-A1) against the 4,096-env paper workload
+    and the oracle's reset draws for it: observation and action widths, the
+    action bound, env count, episode length, and references within [-2, 2] m
+    and [-60, 60] degrees per axis, each range used in full."""
+    from scipy.spatial.transform import Rotation
+    g = _golden_setup()
+    w = W.workload("paper_4096")
+    assert W.obs_dim(w) == g["obs_dim"] and W.act_dim(w) == g["act_dim"]
+    assert w["n_envs"] == g["n_envs"] and w["episode_len"] == g["episode_len"]
+    m = oracle.paper_model(w)
+    bound = g["action_bound"]
+    a_c, tau = oracle.paper_wrench(m, np.array([3.0, -3.0, 0.5, 3.0, -3.0, -0.5]))
+    assert np.array_equal(a_c, [bound, -bound, 0.5, bound, -bound, -0.5])
+    assert np.allclose(tau[[0, 3]], [w["f_max"], w["tau_max"]], rtol=1e-15)
+    b = oracle.PaperBatch(np.arange(int(g["n_envs"])))
+    oracle.paper_reset(m, b)
+    pd = b.params[0:3]
+    assert np.all(np.abs(pd) <= g["goal_pos_range_m"])
+    assert np.all(np.abs(pd).max(axis=1) > 0.99 * g["goal_pos_range_m"])
+    qd = b.params[3:7]
+    yaw_pitch_roll = Rotation.from_quat(np.stack([qd[1], qd[2], qd[3], qd[0]], axis=1)).as_euler(
+        "ZYX", degrees=True)
+    assert np.all(np.abs(yaw_pitch_roll) <= g["goal_att_range_deg"] + 1e-4)
+    assert np.all(np.abs(yaw_pitch_roll).max(axis=0) > 0.99 * g["goal_att_range_deg"])
