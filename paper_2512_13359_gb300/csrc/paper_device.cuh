@@ -187,12 +187,20 @@ __device__ __forceinline__ float reward(const Model& M, const Env& e, const floa
   }
   const int n = M.n;
   const float inv_k = 1.0f / (float)M.mavg_len;
+  // Slots in ascending order for each component, as a loop over the
+  // compile-time slot count: every slot's loads can be in flight at once.
+  float sum[kAct] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+  for (int j = 0; j < kHist; ++j) {
+    if (j < M.mavg_len) {
+#pragma unroll
+      for (int k = 0; k < kAct; ++k) sum[k] += __ldcg(st + (13 + 6 * j + k) * n + i);
+    }
+  }
   float r_mavg = 0.0f;
 #pragma unroll
   for (int k = 0; k < kAct; ++k) {
-    float sum = 0.0f;
-    for (int j = 0; j < M.mavg_len; ++j) sum += __ldcg(st + (13 + 6 * j + k) * n + i);
-    const float d = a_c[k] - sum * inv_k;
+    const float d = a_c[k] - sum[k] * inv_k;
     r_mavg = fmaf(d, d, r_mavg);
   }
   return -M.w_pos * r_pos - M.w_att * r_att - M.w_act * r_act - M.w_vel * r_vel -
