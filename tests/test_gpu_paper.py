@@ -146,14 +146,16 @@ def test_paper_bf16_forward(oracle, n):
     assert eh <= BF16_TOL and ev <= BF16_TOL
 
 
-def test_paper_bf16_rollout(oracle):
+@pytest.mark.parametrize("T", [48, 512])
+def test_paper_bf16_rollout(oracle, T):
     """The paper workload's tensor-core rollout over one whole episode
-    (T = episode_len): step-0 observations to 1e-5, actions and log-probs
-    within the bf16 head tolerance, dones exact, values against the oracle's
-    bf16 value network, and the final state equal bit for bit to the next
-    episode's reset draw (history cleared)."""
+    (T = episode_len; 512 is the paper's episode and the benchmark's launch
+    of 4,096 envs x 512 steps): step-0 observations to 1e-5, actions and
+    log-probs within the bf16 head tolerance, dones exact, values against
+    the oracle's bf16 value network, and the final state equal bit for bit
+    to the next episode's reset draw (history cleared)."""
     torch = need_gpu()
-    n, T = 4096, 48
+    n = 4096
     w = W.workload("paper_4096", n_envs=n, episode_len=T)
     env = make_env(w)
     env.reset()
