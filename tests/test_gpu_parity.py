@@ -146,7 +146,7 @@ def _replay_compare(oracle, w, T, sample_ids, act_scale=0.7):
     ("fp32_4096", 4096, 200, 500),
     ("dr_16384", 16384, 150, 500),
     ("dr_16384", 999, 120, 37),          # ragged N, auto-resets inside the horizon
-    ("ppo_65536", 65536, 60, 500),
+    ("ppo_65536", 65536, 128, 500),      # the benchmark's launch: 65,536 envs x 128 steps
 ])
 def test_action_replay_parity(oracle, name, n, T, L):
     w = W.workload(name, n_envs=n, episode_len=L)
