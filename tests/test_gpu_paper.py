@@ -86,6 +86,35 @@ def test_paper_replay_against_oracle(oracle, n, T, L, K):
     assert np.array_equal(u32(env.episode), b.episode)
 
 
+def test_paper_replay_full_episode_sampled(oracle):
+    """The physics-only launch the benchmark times on the paper workload:
+    4,096 envs x 512 steps (one whole episode, K = 4, gravity randomised),
+    40 sampled envs against the oracle step by step (trace with history
+    rows, reward); dones bit-exact, the last step's state the next reset."""
+    torch = need_gpu()
+    w = W.workload("paper_4096")
+    n, T = int(w["n_envs"]), int(w["steps"])
+    env = make_env(w, policy=False)
+    env.reset()
+    m = oracle.paper_model(w)
+    ids = np.unique(np.r_[0, n - 1, np.random.default_rng(11).integers(0, n, 38)])
+    b = oracle.PaperBatch(ids)
+    oracle.paper_reset(m, b)
+    acts = W.replay_actions(3, T, n, scale=0.8, act=6)
+    rew = torch.empty((T, n), device="cuda")
+    done = torch.empty((T, n), dtype=torch.uint8, device="cuda")
+    trace = torch.empty((T, W.PAPER_STATE_FIELDS, n), device="cuda")
+    env.step_actions(torch.from_numpy(acts).cuda(), rew, done, trace)
+    assert env.status().code == 0
+    r_rew, r_done, r_tr = oracle.paper_replay(m, b, np.ascontiguousarray(acts[:, :, ids]),
+                                              trace=True)
+    g_done = to_np(done)[:, ids]
+    assert np.array_equal(g_done, r_done) and np.all(g_done[-1] == 1) and g_done[:-1].sum() == 0
+    assert_close(to_np(rew)[:, ids], r_rew, STATE_TOL * 10, what="reward")
+    assert_close(to_np(trace)[:, :, ids], r_tr, STATE_TOL, what="state trace")
+    assert_close(to_np(env.state)[:, ids], b.state, STATE_TOL, what="final state")
+
+
 @pytest.mark.parametrize("hidden,policy_out,has_value", [(64, 6, 0), (256, 12, 1)])
 def test_paper_fp32_rollout_against_oracle(oracle, hidden, policy_out, has_value):
     torch = need_gpu()
