@@ -319,7 +319,27 @@ __global__ void __launch_bounds__(256) k_transpose_batch(int D, int A, int Ws, u
 
 // k_gather from the sample-major copy: one row of Ws floats per sample, read
 // in 16-byte pieces.
-template <typename TX>
+// Eight consecutive X values as 16-byte stores (X rows are multiples of 8
+// elements, so every chunk starts on a 16-byte boundary).
+__device__ __forceinline__ void st_act8(__nv_bfloat16* p, const float v[8]) {
+  uint4 q;
+  __nv_bfloat162 h0 = __floats2bfloat162_rn(v[0], v[1]), h1 = __floats2bfloat162_rn(v[2], v[3]);
+  __nv_bfloat162 h2 = __floats2bfloat162_rn(v[4], v[5]), h3 = __floats2bfloat162_rn(v[6], v[7]);
+  memcpy(&q.x, &h0, 4);
+  memcpy(&q.y, &h1, 4);
+  memcpy(&q.z, &h2, 4);
+  memcpy(&q.w, &h3, 4);
+  *reinterpret_cast<uint4*>(p) = q;
+}
+__device__ __forceinline__ void st_act8(float* p, const float v[8]) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+// One sample per thread: its whole row (Ws <= W floats) is loaded at once
+// and X is written in chunks of eight with vector stores; W is a
+// compile-time bound on the row, so the row lives in registers.
+template <typename TX, int W>
 __global__ void __launch_bounds__(kT) k_gather_sm(Dims d, PermKey key, const StepCtl* ctl,
                                                   const float* __restrict__ rows, int Ws,
                                                   Sample out, TX* __restrict__ X) {
@@ -333,24 +353,37 @@ __global__ void __launch_bounds__(kT) k_gather_sm(Dims d, PermKey key, const Ste
   if (b < d.B) {
     const uint32_t r = perm_index(start + (uint32_t)b, key);
     const float4* src = reinterpret_cast<const float4*>(rows + (size_t)r * Ws);
-    TX* x = X + (size_t)b * d.Dp;
-    const int F = d.D + d.A + 3;
-    float lp = 0.0f, a = 0.0f;
-    for (int q = 0; q < (F + 3) / 4; ++q) {
-      const float4 v4 = __ldg(src + q);
-      const float v[4] = {v4.x, v4.y, v4.z, v4.w};
+    float v[W];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int k = 4 * q + j;
-        if (k < d.D) st_act(x + k, v[j]);
-        else if (k < d.D + d.A) { if (!d.value_only) out.act[(size_t)b * d.A + (k - d.D)] = v[j]; }
-        else if (k == d.D + d.A) lp = v[j];
-        else if (k == d.D + d.A + 1) a = v[j];
-        else if (k == d.D + d.A + 2) out.ret[b] = v[j];
+    for (int q = 0; q < W / 4; ++q) {
+      float4 t = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      if (4 * q < Ws) t = __ldg(src + q);
+      v[4 * q] = t.x;
+      v[4 * q + 1] = t.y;
+      v[4 * q + 2] = t.z;
+      v[4 * q + 3] = t.w;
+    }
+    TX* x = X + (size_t)b * d.Dp;
+#pragma unroll
+    for (int c = 0; c < W / 8; ++c) {
+      if (8 * c < d.Dp) {
+        float x8[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int k = 8 * c + j;
+          x8[j] = k < d.D ? v[k] : (k == d.D ? 1.0f : 0.0f);
+        }
+        st_act8(x + 8 * c, x8);
       }
     }
-    st_act(x + d.D, 1.0f);
-    for (int k = d.D + 1; k < d.Dp; ++k) st_act(x + k, 0.0f);
+    // the fields after the observation sit at run-time offsets: read them
+    // from the row again (its sectors are in L1 from the loads above), so
+    // that v stays in registers
+    const float* f = rows + (size_t)r * Ws + d.D;
+    if (!d.value_only)
+      for (int j = 0; j < d.A; ++j) out.act[(size_t)b * d.A + j] = __ldg(f + j);
+    const float lp = __ldg(f + d.A), a = __ldg(f + d.A + 1);
+    out.ret[b] = __ldg(f + d.A + 2);
     if (!d.value_only) {
       out.logp[b] = lp;
       out.adv[b] = a;
@@ -684,10 +717,18 @@ cudaError_t launch_gather_sm(const Dims& d, const PermKey& k, const StepCtl* ctl
                              const float* rows, const Sample& out, void* X, cudaStream_t s) {
   const unsigned nb = (d.B + kT - 1) / kT;
   const int Ws = sample_row_floats(d.D, d.A);
-  if (d.bf16)
-    k_gather_sm<<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, static_cast<__nv_bfloat16*>(X));
-  else
-    k_gather_sm<<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, static_cast<float*>(X));
+  if (Ws > kSmMaxW || d.Dp > Ws || d.Dp % 8 != 0 || reinterpret_cast<uintptr_t>(X) % 16 != 0 ||
+      reinterpret_cast<uintptr_t>(rows) % 16 != 0)
+    return cudaErrorInvalidValue;
+  if (d.bf16) {
+    __nv_bfloat16* xb = static_cast<__nv_bfloat16*>(X);
+    if (Ws <= 32) k_gather_sm<__nv_bfloat16, 32><<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, xb);
+    else k_gather_sm<__nv_bfloat16, kSmMaxW><<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, xb);
+  } else {
+    float* xf = static_cast<float*>(X);
+    if (Ws <= 32) k_gather_sm<float, 32><<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, xf);
+    else k_gather_sm<float, kSmMaxW><<<nb, kT, 0, s>>>(d, k, ctl, rows, Ws, out, xf);
+  }
   return cudaGetLastError();
 }
 
