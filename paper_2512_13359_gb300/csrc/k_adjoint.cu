@@ -888,7 +888,7 @@ __device__ void paper_step_vjp(const Model& M, const float* sc, size_t n, int i,
     if (!(a[k] >= -1.0f && a[k] <= 1.0f)) la[k] = 0.0f;
 }
 
-__global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
+__global__ void __launch_bounds__(kAdjThreads, 4) k_paper_adjoint(
     const Model M, Buffers B, const float* __restrict__ act, int T,
     const float* __restrict__ coef, const float* __restrict__ lam_T, float* __restrict__ g_act,
     float* __restrict__ lam_0, float* __restrict__ rew, uint8_t* __restrict__ done,
@@ -919,7 +919,7 @@ __global__ void __launch_bounds__(kAdjThreads) k_paper_adjoint(
         a_next[k] = __ldg(act + ((size_t)(t + 1) * paper::kAct + k) * n + i);
     }
     bool d;
-    const float r = paper::physics_step(M, id, e, a, hsc, i, &d);
+    const float r = paper::physics_step(M, id, e, a, paper::hist_rows(hsc, (int)n, i), &d);
     if (d) ends |= 1ull << t;
     if (rew) rew[(size_t)t * n + i] = r;
     if (done) done[(size_t)t * n + i] = d ? 1 : 0;
@@ -1042,7 +1042,7 @@ __global__ void __launch_bounds__(kAdjThreads) k_shac_step_paper(const Model M, 
   action_noise(id, M.seed, t_g, eps);
   paper_shac_action(M, Y + (size_t)i * ldy, eps, a, sig, in);
   bool d;
-  const float r = paper::physics_step(M, id, e, a, B.state, i, &d);
+  const float r = paper::physics_step(M, id, e, a, paper::hist_rows(B.state, M.n, i), &d);
   if (!paper::env_finite(e)) flag_nan(st, i);
   paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   rew[i] = r;

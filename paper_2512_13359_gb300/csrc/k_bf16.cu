@@ -825,7 +825,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           }
           if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
           bool d;
-          const float r = paper::physics_step(M, id, e, a, B.state, i, &d);
+          const float r =
+              paper::physics_step(M, id, e, a, paper::hist_rows(B.state, M.n, i), &d);
           if (tr.rew) tr.rew[(size_t)t * n + i] = r;
           if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
           bad |= !paper::env_finite(e);

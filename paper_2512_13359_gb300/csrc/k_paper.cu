@@ -21,18 +21,26 @@ __global__ void __launch_bounds__(256) k_paper_reset(const Model M, Buffers B,
   if (mask && !mask[i]) return;
   paper::Env e;
   e.ep = B.episode[i];
-  paper::reset_env(M, M.id_base + (uint32_t)i, e, B.state, i);
+  paper::reset_env(M, M.id_base + (uint32_t)i, e, paper::hist_rows(B.state, M.n, i));
   paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
 }
 
-__global__ void __launch_bounds__(128, 4) k_paper_replay(const Model M, Buffers B,
+constexpr int kReplayThreads = 128;
+
+__global__ void __launch_bounds__(kReplayThreads, 4) k_paper_replay(const Model M, Buffers B,
                                                       const float* __restrict__ act, int T,
                                                       float* __restrict__ rew,
                                                       uint8_t* __restrict__ done, float* trace,
                                                       Status* st) {
+  // The action history lives in shared memory for the whole launch (one
+  // column per thread, copied in and out once): its reads every step are
+  // shared-memory loads instead of L2 round trips.
+  __shared__ float hist[6 * paper::kHist * kReplayThreads];
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= M.n) return;
   const size_t n = (size_t)M.n;
+  const paper::HistS h{hist + threadIdx.x, kReplayThreads};
+  for (int r = 0; r < 6 * paper::kHist; ++r) h.st(r, B.state[(13 + r) * n + i]);
   paper::Env e;
   paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
   bool bad = false;
@@ -51,14 +59,15 @@ __global__ void __launch_bounds__(128, 4) k_paper_replay(const Model M, Buffers 
         a_next[k] = __ldg(act + ((size_t)(t + 1) * kAct + k) * n + i);
     }
     bool d;
-    const float r = paper::physics_step(M, M.id_base + (uint32_t)i, e, a, B.state, i, &d);
+    const float r = paper::physics_step(M, M.id_base + (uint32_t)i, e, a, h, &d);
     rew[(size_t)t * n + i] = r;
     done[(size_t)t * n + i] = d ? 1 : 0;
-    if (trace) paper::trace_state(M, B.state, trace + (size_t)t * paper::kStateF * n, i, e);
+    if (trace) paper::trace_state(M, h, trace + (size_t)t * paper::kStateF * n, i, e);
     bad |= !paper::env_finite(e);
   }
   if (bad) flag_nan(st, i);
   paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  for (int r = 0; r < 6 * paper::kHist; ++r) B.state[(13 + r) * n + i] = h.ld(r);
 }
 
 __global__ void __launch_bounds__(256) k_paper_observe(const Model M, Buffers B,
@@ -125,7 +134,8 @@ __global__ void __launch_bounds__(kTile) k_paper_rollout_fp32(const Model M, Buf
     }
     if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
     bool d;
-    const float r = paper::physics_step(M, M.id_base + (uint32_t)i, e, a, B.state, i, &d);
+    const float r = paper::physics_step(M, M.id_base + (uint32_t)i, e, a,
+                                        paper::hist_rows(B.state, M.n, i), &d);
     if (tr.rew) tr.rew[(size_t)t * n + i] = r;
     if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
     bad |= !paper::env_finite(e);
@@ -160,7 +170,8 @@ cudaError_t launch_paper_reset(const Model& M, const Buffers& B, const uint8_t* 
 cudaError_t launch_paper_replay(const Model& M, const Buffers& B, const float* act, int T,
                                 float* rew, uint8_t* done, float* trace, Status* st,
                                 cudaStream_t s) {
-  k_paper_replay<<<blocks_for(M.n, 128), 128, 0, s>>>(M, B, act, T, rew, done, trace, st);
+  k_paper_replay<<<blocks_for(M.n, kReplayThreads), kReplayThreads, 0, s>>>(M, B, act, T, rew,
+                                                                             done, trace, st);
   return cudaGetLastError();
 }
 

@@ -37,6 +37,25 @@ struct Env {
   uint32_t ep;
 };
 
+// The K-slot action history of one env, entry r = 6 j + k (slot j,
+// component k).  HistG: the state rows 13.. of [kStateF][n] in global memory,
+// read past L1; HistS: a copy in shared memory, one column per thread.
+struct HistG {
+  float* p;
+  int s;   // r * s < 48 n fits an int for every env count the state array allows
+  __device__ __forceinline__ float ld(int r) const { return __ldcg(p + r * s); }
+  __device__ __forceinline__ void st(int r, float v) const { p[r * s] = v; }
+};
+struct HistS {
+  float* p;
+  int s;
+  __device__ __forceinline__ float ld(int r) const { return p[r * s]; }
+  __device__ __forceinline__ void st(int r, float v) const { p[r * s] = v; }
+};
+__device__ __forceinline__ HistG hist_rows(float* st, int n, int i) {
+  return HistG{st + 13 * (size_t)n + i, n};
+}
+
 __device__ __forceinline__ void load_env(const Model& M, const float* st, const float* pr,
                                          const int* t_ep, const uint32_t* ep, int i, Env& e) {
   const int n = M.n;
@@ -81,17 +100,19 @@ __device__ __forceinline__ void store_env(const Model& M, float* st, float* pr, 
 
 // Full state of env i to a trace slice (rows 0..12 from registers, the
 // history rows copied from the state array).
-__device__ __forceinline__ void trace_state(const Model& M, const float* st, float* tr, int i,
+template <class Hist>
+__device__ __forceinline__ void trace_state(const Model& M, const Hist& h, float* tr, int i,
                                             const Env& e) {
   const int n = M.n;
   store_state(M, tr, i, e);
-  for (int r = 13; r < kStateF; ++r) tr[r * n + i] = __ldcg(st + r * n + i);
+  for (int r = 0; r < 6 * kHist; ++r) tr[(13 + r) * n + i] = h.ld(r);
 }
 
 // New episode (counter (episode, 0, 1, block 0..3) of the reset stream):
 // goal position, goal roll/pitch/yaw, effective-gravity offset, initial
 // position, initial roll/pitch/yaw; velocities and history zeroed.
-__device__ __forceinline__ void reset_env(const Model& M, uint32_t id, Env& e, float* st, int i) {
+template <class Hist>
+__device__ __forceinline__ void reset_env(const Model& M, uint32_t id, Env& e, const Hist& h) {
   uint32_t w[16];
 #pragma unroll
   for (int b = 0; b < 4; ++b) {
@@ -113,8 +134,7 @@ __device__ __forceinline__ void reset_env(const Model& M, uint32_t id, Env& e, f
   e.g = M.dr_enable ? __fadd_rn(M.g_eff0, sym_draw(u[6], M.dr_grav)) : M.g_eff0;
 #pragma unroll
   for (int k = 0; k < 6; ++k) e.nu[k] = 0.0f;
-  const int n = M.n;
-  for (int r = 13; r < kStateF; ++r) st[r * n + i] = 0.0f;
+  for (int r = 0; r < 6 * kHist; ++r) h.st(r, 0.0f);
   e.t_ep = 0;
   e.ep += 1u;
 }
@@ -172,8 +192,9 @@ __device__ __forceinline__ void observe(const Env& e, float o[kObs]) {
 
 // Reward on the post-step state; the history mean is over the K slots as
 // they stand before this step's action is entered.
+template <class Hist>
 __device__ __forceinline__ float reward(const Model& M, const Env& e, const float a_c[kAct],
-                                        const float* st, int i) {
+                                        const Hist& h) {
   float o[kObs];
   observe(e, o);
   float r_pos = 0.0f, r_att = 0.0f, r_act = 0.0f, r_vel = 0.0f;
@@ -185,7 +206,6 @@ __device__ __forceinline__ float reward(const Model& M, const Env& e, const floa
     r_act = fmaf(a_c[3 + k], a_c[3 + k], r_act);
     r_vel = fmaf(e.nu[3 + k], e.nu[3 + k], r_vel);
   }
-  const int n = M.n;
   const float inv_k = 1.0f / (float)M.mavg_len;
   // Slots in ascending order for each component, as a loop over the
   // compile-time slot count: every slot's loads can be in flight at once.
@@ -194,7 +214,7 @@ __device__ __forceinline__ float reward(const Model& M, const Env& e, const floa
   for (int j = 0; j < kHist; ++j) {
     if (j < M.mavg_len) {
 #pragma unroll
-      for (int k = 0; k < kAct; ++k) sum[k] += __ldcg(st + (13 + 6 * j + k) * n + i);
+      for (int k = 0; k < kAct; ++k) sum[k] += h.ld(6 * j + k);
     }
   }
   float r_mavg = 0.0f;
@@ -221,9 +241,9 @@ __device__ __forceinline__ bool env_finite(const Env& e) {
 // One control step with action a: Eq. (1) wrench, substeps, reward, history
 // entry (slot t_ep mod K), episode bookkeeping and auto-reset.  st is the
 // state array holding this env's history rows.
+template <class Hist>
 __device__ __forceinline__ float physics_step(const Model& M, uint32_t id, Env& e,
-                                              const float a[kAct], float* st, int i,
-                                              bool* done) {
+                                              const float a[kAct], const Hist& h, bool* done) {
   float a_c[kAct], tau[6];
 #pragma unroll
   for (int k = 0; k < kAct; ++k) a_c[k] = fminf(fmaxf(a[k], -1.0f), 1.0f);
@@ -233,14 +253,13 @@ __device__ __forceinline__ float physics_step(const Model& M, uint32_t id, Env& 
     tau[3 + k] = M.tau_max * a_c[3 + k];
   }
   for (int s = 0; s < M.substeps; ++s) substep(M, e, tau);
-  const float r = reward(M, e, a_c, st, i);
+  const float r = reward(M, e, a_c, h);
   const int slot = e.t_ep % M.mavg_len;
-  const int n = M.n;
 #pragma unroll
-  for (int k = 0; k < kAct; ++k) st[(13 + 6 * slot + k) * n + i] = a_c[k];
+  for (int k = 0; k < kAct; ++k) h.st(6 * slot + k, a_c[k]);
   e.t_ep += 1;
   *done = (e.t_ep == M.episode_len);
-  if (*done) reset_env(M, id, e, st, i);
+  if (*done) reset_env(M, id, e, h);
   return r;
 }
 
