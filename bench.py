@@ -469,7 +469,7 @@ def run_gae(args):
 # --no-cpu-baseline --no-clocks`; profiles/k_engine_ppo_65536_T128_dram.md),
 # valid while the engine's sources hash to ENGINE_SRC_HASH.
 ROLLOUT_TRAFFIC_65536x128 = 10_783_232 + 902_189_056
-ENGINE_SRC_HASH = "a1bca85a644c154e"
+ENGINE_SRC_HASH = "7832b756ffc66fe2"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 
