@@ -52,7 +52,7 @@
 extern "C" {
 #endif
 
-#define AUV_ABI_VERSION 2
+#define AUV_ABI_VERSION 3
 
 /* status codes */
 #define AUV_OK 0
@@ -324,23 +324,30 @@ int env_draw_words(auv_env* env, uint32_t stream_id, uint64_t index, int n_block
  * library convenience.
  *  - No handle and no allocation: the packed weights and a status word live
  *    in one static device array of 312.25 KiB that every GPU loading this
- *    library holds until the process exits.  The first call on a device looks
- *    up that array's address (once per device); make it before any stream
- *    capture.
+ *    library holds until the process exits.
+ *  - The first call on a device is a warm-up: it looks up that array's
+ *    address (once per device), and under the CUDA runtime's lazy module
+ *    loading (the default) it is also the call that loads the array's module
+ *    and the kernels, which may take device memory and synchronise.  Make
+ *    it before the period in which nothing may allocate, and before any
+ *    stream capture; later calls allocate nothing.
  *  - hidden must be 256 and policy_out 16 (the built tensor-core shape);
  *    larger values return AUV_ERR_SIZE (the packed weights would not fit
  *    the array), other values AUV_ERR_UNSUPPORTED.
  *  - policy[, value_w]: fp32 weights in the env_set_weights layout; obs[n][18]
  *    (row-major); outputs head[n][policy_out] and, iff value_w is given,
- *    value[n].  All device memory, 16-byte aligned; n >= 1.
+ *    value[n].  All device memory of the current device, 16-byte aligned;
+ *    n >= 1.  Pointers to another GPU's memory return AUV_ERR_SIZE.
+ *  - status_out (device memory of the current device, or NULL): receives the
+ *    call's status block (code AUV_ERR_TIMEOUT and timeouts > 0 if a device
+ *    wait gave up), copied on `stream` after the kernels.
  *  - Every call on a device shares the array and leaves its contents there:
  *    calls that overlap on the GPU (other streams, other host threads) race
- *    on it and must be serialised by the caller.  Device-side wait timeouts
- *    are not reported by this entry point.
+ *    on it and must be serialised by the caller.
  */
 int env_policy_forward_noalloc(int hidden, int policy_out, const float* policy,
                                const float* value_w, const float* obs, int n, float* head,
-                               float* value, void* stream);
+                               float* value, auv_status* status_out, void* stream);
 
 /*
  * env_gae: generalised advantage estimation over a rollout's trajectory --
@@ -633,6 +640,49 @@ int rbuf_sample(auv_rbuf* r, uint32_t B, uint64_t seed, uint64_t draw, float* ob
 /* Global step counter (action-noise stream index) get/set, for checkpoints. */
 int env_get_step(const auv_env* env, uint64_t* t_g);
 int env_set_step(auv_env* env, uint64_t t_g);
+
+/*
+ * Snapshot of a batch for checkpoint and resume: everything that determines
+ * the envs' future steps besides the configuration and the network weights.
+ * Per env that is the dynamic state of the vehicle (the body pose and
+ * velocities of §IV-B; the paper model adds the action history read by the
+ * moving-average term of Eq. 7), the episode's randomised parameters (goal
+ * of §V-A1, domain randomisation of §IV-C), the control steps taken in the
+ * episode and the index of the next episode's reset draw; for the batch the
+ * global step t_g that keys the action noise.  The arrays are caller-owned,
+ * in the layout of auv_buffers (row counts from env_layout), device or host
+ * memory (page-locked host memory keeps the copies asynchronous).
+ */
+typedef struct auv_snapshot {
+  uint32_t struct_size;   /* sizeof(auv_snapshot): version guard            */
+  uint32_t model;         /* AUV_MODEL_* of the env the snapshot came from  */
+  uint32_t n_envs;        /* N                                              */
+  uint32_t state_fields;  /* rows of state                                  */
+  uint32_t param_fields;  /* rows of params                                 */
+  uint32_t reserved;      /* 0                                              */
+  uint64_t t_g;           /* global step (action-noise stream index)        */
+  float* state;           /* [state_fields][N]                              */
+  float* params;          /* [param_fields][N]                              */
+  int32_t* t_ep;          /* [N]                                            */
+  uint32_t* episode;      /* [N]                                            */
+} auv_snapshot;
+
+/*
+ * env_get_state: copy the env's state, params, t_ep and episode arrays into
+ * the snapshot's arrays (4-byte aligned, non-NULL) and fill its model,
+ * n_envs, field counts and t_g.  The copies are enqueued on `stream` after
+ * the work already there; t_g is the counter as of the call (it counts the
+ * steps of every rollout enqueued before it).  The snapshot is complete when
+ * `stream` has reached this point.
+ * env_set_state: the reverse, into an env of the same model and n_envs:
+ * copies the snapshot's arrays into the env's buffers on `stream` and sets
+ * t_g.  Continuing from it reproduces, bit for bit, the steps the source env
+ * would have taken next (same configuration and weights).
+ * Errors: AUV_ERR_INVALID (NULL, struct_size, model, n_envs or field counts
+ * that do not match the env), AUV_ERR_SIZE (misaligned array), AUV_ERR_CUDA.
+ */
+int env_get_state(auv_env* env, auv_snapshot* snap, void* stream);
+int env_set_state(auv_env* env, const auv_snapshot* snap, void* stream);
 
 /*
  * env_status: synchronise `stream`, copy the device status block to *out and

@@ -1581,6 +1581,63 @@ void oracle_paper_rollout(const PaperModel* m, int precision, const float* pol_w
                                act, logp, value, rew, done);
 }
 
+// The Gaussian policy's draw for given observations, in double: head =
+// network(obs) (bf16 emulation when the model says so), log sigma = the
+// clamped head or the fixed vector (A6), eps = the first n_act normals of the
+// action-noise stream at global step t_g, a = mu + exp(log sigma) eps and
+// log pi(a) = sum(-eps^2/2 - log sigma - log(2 pi)/2), as one step of the
+// rollout computes them.  obs[n][obs_dim] row-major; act[n][n_act], logp[n].
+void oracle_policy_act(const OracleModel* m, const float* pol_w, int n,
+                       const uint32_t* env_ids, uint64_t t_g, const double* obs, double* act,
+                       double* logp) {
+  const double half_log_2pi = 0.91893853320467274178032973640562;
+  for (int i = 0; i < n; ++i) {
+    double mu[kAct], logstd[kAct];
+    policy_head<double>(*m, pol_w, obs + (size_t)i * kObs, mu, logstd);
+    uint32_t w[8];
+    draw_words(env_ids[i], m->seed, t_g, 0u, 2, w);
+    float u[8];
+    for (int k = 0; k < 8; ++k) u[k] = word_to_uniform(w[k]);
+    double eps[8];
+    box_muller8(u, eps);
+    double lp = 0;
+    for (int k = 0; k < kAct; ++k) {
+      act[(size_t)i * kAct + k] = mu[k] + std::exp(logstd[k]) * eps[k];
+      lp += -0.5 * eps[k] * eps[k] - logstd[k] - half_log_2pi;
+    }
+    logp[i] = lp;
+  }
+}
+
+void oracle_paper_policy_act(const PaperModel* m, const float* pol_w, int n,
+                             const uint32_t* env_ids, uint64_t t_g, const double* obs,
+                             double* act, double* logp) {
+  const double half_log_2pi = 0.91893853320467274178032973640562;
+  for (int i = 0; i < n; ++i) {
+    double out[12];
+    mlp_forward<double>(pol_w, kPObs, m->hidden, m->policy_out, m->mlp_bf16 != 0,
+                        obs + (size_t)i * kPObs, out);
+    uint32_t w[8];
+    draw_words(env_ids[i], m->seed, t_g, 0u, 2, w);
+    float u[8];
+    for (int k = 0; k < 8; ++k) u[k] = word_to_uniform(w[k]);
+    double eps[8];
+    box_muller8(u, eps);
+    double lp = 0;
+    for (int k = 0; k < kPAct; ++k) {
+      double ls = (double)m->logstd_fixed[k];
+      if (m->policy_out == 12) {
+        ls = out[kPAct + k];
+        ls = ls < (double)m->logstd_min ? (double)m->logstd_min : ls;
+        ls = ls > (double)m->logstd_max ? (double)m->logstd_max : ls;
+      }
+      act[(size_t)i * kPAct + k] = out[k] + std::exp(ls) * eps[k];
+      lp += -0.5 * eps[k] * eps[k] - ls - half_log_2pi;
+    }
+    logp[i] = lp;
+  }
+}
+
 // Observation of one env (SoA with n = 1).
 void oracle_paper_observe(const double* st, const double* pr, double* obs) {
   int32_t t = 0;

@@ -40,6 +40,7 @@ PPO_STAT_NAMES = ("pg_loss", "v_loss", "entropy", "approx_kl", "clip_frac", "gra
 EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "env_set_weights",
             "env_reset", "env_rollout", "env_value", "env_step", "env_step_actions", "env_observe",
             "env_policy_forward", "env_draw_words", "env_get_step", "env_set_step",
+            "env_get_state", "env_set_state",
             "env_status", "env_clear_status", "env_selftest_wait_timeout",
             "env_policy_forward_noalloc", "env_layout", "env_gae", "env_adjoint",
             "env_inverse_allocate", "env_shac_window", "rbuf_create", "rbuf_destroy", "rbuf_last_error",
@@ -115,6 +116,13 @@ class PpoBatch(C.Structure):
                 ("adv", C.c_void_p), ("ret", C.c_void_p), ("T", C.c_uint32), ("N", C.c_uint32)]
 
 
+class AuvSnapshot(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("model", C.c_uint32), ("n_envs", C.c_uint32),
+                ("state_fields", C.c_uint32), ("param_fields", C.c_uint32),
+                ("reserved", C.c_uint32), ("t_g", C.c_uint64), ("state", C.c_void_p),
+                ("params", C.c_void_p), ("t_ep", C.c_void_p), ("episode", C.c_void_p)]
+
+
 class AuvStatus(C.Structure):
     _fields_ = [("code", C.c_int32), ("nan_flag", C.c_int32), ("first_nan_env", C.c_int32),
                 ("timeouts", C.c_int32)]
@@ -152,10 +160,12 @@ def lib(path: str | None = None):
     L.env_draw_words.argtypes = [P, C.c_uint32, C.c_uint64, I, P, P]
     L.env_get_step.argtypes = [P, C.POINTER(C.c_uint64)]
     L.env_set_step.argtypes = [P, C.c_uint64]
+    L.env_get_state.argtypes = [P, C.POINTER(AuvSnapshot), P]
+    L.env_set_state.argtypes = [P, C.POINTER(AuvSnapshot), P]
     L.env_status.argtypes = [P, C.POINTER(AuvStatus), P]
     L.env_clear_status.argtypes = [P, P]
     L.env_selftest_wait_timeout.argtypes = [P, C.c_uint32, P]
-    L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P]
+    L.env_policy_forward_noalloc.argtypes = [I, I, P, P, P, I, P, P, P, P]
     L.env_layout.argtypes = [C.c_uint32, C.POINTER(AuvLayout)]
     L.env_gae.argtypes = [P, I, P, P, P, P, C.c_float, C.c_float, P, P, P]
     L.env_adjoint.argtypes = [P, I, P, P, P, P, P, P, P, P]
@@ -391,6 +401,25 @@ class Env:
         s = AuvStatus()
         lib().env_status(self.h, C.byref(s), _stream(stream))
         return s
+
+    def get_state(self, snap: dict, stream=None) -> int:
+        """env_get_state into snap's tensors (keys state, params, t_ep,
+        episode; device or host).  Returns the snapshot's t_g."""
+        sn = AuvSnapshot(C.sizeof(AuvSnapshot), 0, 0, 0, 0, 0, 0,
+                         *(snap[k].data_ptr() for k in ("state", "params", "t_ep", "episode")))
+        self._check(lib().env_get_state(self.h, C.byref(sn), _stream(stream)))
+        snap["t_g"] = int(sn.t_g)
+        return int(sn.t_g)
+
+    def set_state(self, snap: dict, stream=None):
+        """env_set_state from snap's tensors and t_g (as get_state filled it)."""
+        lay = AuvLayout()
+        lib().env_layout(self.cfg.model, C.byref(lay))
+        sn = AuvSnapshot(C.sizeof(AuvSnapshot), snap.get("model", self.cfg.model),
+                         snap.get("n_envs", self.n), snap.get("state_fields", lay.state_fields),
+                         snap.get("param_fields", lay.param_fields), 0, int(snap["t_g"]),
+                         *(snap[k].data_ptr() for k in ("state", "params", "t_ep", "episode")))
+        self._check(lib().env_set_state(self.h, C.byref(sn), _stream(stream)))
 
     def selftest_wait_timeout(self, limit_us: int, stream=None):
         self._check(lib().env_selftest_wait_timeout(self.h, int(limit_us), _stream(stream)))

@@ -304,6 +304,44 @@ int check_device(auv_env* env) {
   return AUV_OK;
 }
 
+// Checkpoint and resume: the caller's batch arrays plus the global step.
+int snapshot_arrays(auv_env* env, const auv_snapshot* snap, bool check_header) {
+  if (!env || !snap) return AUV_ERR_INVALID;
+  if (snap->struct_size != sizeof(auv_snapshot))
+    return fail(env, AUV_ERR_INVALID, "snapshot struct_size %u != sizeof(auv_snapshot) %zu",
+                snap->struct_size, sizeof(auv_snapshot));
+  if (!snap->state || !snap->params || !snap->t_ep || !snap->episode)
+    return fail(env, AUV_ERR_INVALID, "snapshot array is NULL");
+  const void* arr[4] = {snap->state, snap->params, snap->t_ep, snap->episode};
+  for (const void* p : arr)
+    if (reinterpret_cast<uintptr_t>(p) % 4)
+      return fail(env, AUV_ERR_SIZE, "snapshot array is not 4-byte aligned");
+  if (check_header) {
+    auv_layout lay;
+    env_layout(env->cfg.model, &lay);
+    if (snap->model != env->cfg.model || snap->n_envs != env->cfg.n_envs ||
+        snap->state_fields != lay.state_fields || snap->param_fields != lay.param_fields)
+      return fail(env, AUV_ERR_INVALID,
+                  "snapshot (model %u, %u envs, %u/%u fields) does not match the env "
+                  "(model %u, %u envs, %u/%u fields)",
+                  snap->model, snap->n_envs, snap->state_fields, snap->param_fields,
+                  env->cfg.model, env->cfg.n_envs, lay.state_fields, lay.param_fields);
+  }
+  return AUV_OK;
+}
+
+int copy_batch(auv_env* env, void* const dst[4], const void* const src[4], cudaStream_t s) {
+  auv_layout lay;
+  env_layout(env->cfg.model, &lay);
+  const size_t n = env->cfg.n_envs;
+  const size_t bytes[4] = {lay.state_fields * n * sizeof(float), lay.param_fields * n * sizeof(float),
+                           n * sizeof(int32_t), n * sizeof(uint32_t)};
+  for (int k = 0; k < 4; ++k) {
+    cudaError_t e = cudaMemcpyAsync(dst[k], src[k], bytes[k], cudaMemcpyDefault, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "snapshot copy");
+  }
+  return AUV_OK;
+}
 }  // namespace
 
 extern "C" {
@@ -859,6 +897,35 @@ int env_get_step(const auv_env* env, uint64_t* t_g) {
 int env_set_step(auv_env* env, uint64_t t_g) {
   if (!env) return AUV_ERR_INVALID;
   env->t_g = t_g;
+  return AUV_OK;
+}
+
+int env_get_state(auv_env* env, auv_snapshot* snap, void* stream) {
+  int rc = snapshot_arrays(env, snap, false);
+  if (rc) return rc;
+  if ((rc = check_device(env))) return rc;
+  auv_layout lay;
+  env_layout(env->cfg.model, &lay);
+  snap->model = env->cfg.model;
+  snap->n_envs = env->cfg.n_envs;
+  snap->state_fields = lay.state_fields;
+  snap->param_fields = lay.param_fields;
+  snap->reserved = 0;
+  snap->t_g = env->t_g;
+  void* const dst[4] = {snap->state, snap->params, snap->t_ep, snap->episode};
+  const void* const src[4] = {env->buf.state, env->buf.params, env->buf.t_ep, env->buf.episode};
+  return copy_batch(env, dst, src, static_cast<cudaStream_t>(stream));
+}
+
+int env_set_state(auv_env* env, const auv_snapshot* snap, void* stream) {
+  int rc = snapshot_arrays(env, snap, true);
+  if (rc) return rc;
+  if ((rc = check_device(env))) return rc;
+  void* const dst[4] = {env->buf.state, env->buf.params, env->buf.t_ep, env->buf.episode};
+  const void* const src[4] = {snap->state, snap->params, snap->t_ep, snap->episode};
+  rc = copy_batch(env, dst, src, static_cast<cudaStream_t>(stream));
+  if (rc) return rc;
+  env->t_g = snap->t_g;
   return AUV_OK;
 }
 

@@ -25,6 +25,7 @@
 // Tensor-memory columns: h1 slots 0..127 and 128..255 (bf16 pairs), layer-1
 // accumulator X 256..319, layer-2 accumulators Y 320..383 and Z 384..447,
 // head accumulators 448..463 and 464..479.
+#include <atomic>
 #include <climits>
 
 #include "auv_bf16.h"
@@ -910,15 +911,25 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
   }
 }
 
+// SM count of the current device, looked up once per device (the grids are
+// sized per launch for the device the launch goes to).
 int sm_count() {
-  static int cached = 0;
-  if (!cached) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&cached, cudaDevAttrMultiProcessorCount, dev);
-    if (cached <= 0) cached = 1;
+  constexpr int kMaxDev = 64;
+  static std::atomic<int> cached[kMaxDev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) {
+    cudaGetLastError();
+    dev = 0;
   }
-  return cached;
+  int v = dev < kMaxDev ? cached[dev].load(std::memory_order_relaxed) : 0;
+  if (v <= 0) {
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
+      cudaGetLastError();
+      v = 1;
+    }
+    if (dev < kMaxDev) cached[dev].store(v, std::memory_order_relaxed);
+  }
+  return v;
 }
 
 template <int G, int MODE, int SIM = 0>

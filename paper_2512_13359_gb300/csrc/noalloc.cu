@@ -8,8 +8,15 @@
 // forbids any other allocator once it has started, is another.  This entry
 // point serves both.  It needs no env handle, and its working memory (the
 // packed bf16 weight images and a status word) is one file-scope device
-// array that is reserved when the library's GPU code is loaded and held until
-// the process exits.
+// array, held by every GPU that loads it until the process exits.
+//
+// When the array and the kernels become resident depends on the CUDA
+// runtime's module loading: with lazy loading (the default since CUDA 12.2)
+// the module that holds the array is loaded by the first call on a device,
+// and each kernel by its first launch, and that loading may itself take
+// device memory and synchronise.  The first call on a device is therefore a
+// warm-up: make it before the period in which nothing may allocate (and
+// before any stream capture).  Later calls allocate nothing.
 #include <climits>
 #include <cstdint>
 #include <mutex>
@@ -51,20 +58,30 @@ int scratch_address(unsigned char** out) {
   return AUV_OK;
 }
 
+// Device memory of the current device (or managed memory).  A buffer on
+// another GPU is rejected: the kernels would read or write it over the
+// interconnect, or fault where peer access is off.
 bool is_device_ptr(const void* p) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();
     return false;
   }
-  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+  if (a.type == cudaMemoryTypeManaged) return true;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice && a.device == dev;
 }
 
 }  // namespace
 
 extern "C" int env_policy_forward_noalloc(int hidden, int policy_out, const float* policy,
                                           const float* value_w, const float* obs, int n,
-                                          float* head, float* value, void* stream) {
+                                          float* head, float* value, auv_status* status_out,
+                                          void* stream) {
   // Shapes: the packed images of larger networks would not fit the array.
   if (hidden > 256 || policy_out > 16) return AUV_ERR_SIZE;
   if (hidden != 256 || policy_out != 16) return AUV_ERR_UNSUPPORTED;
@@ -78,11 +95,14 @@ extern "C" int env_policy_forward_noalloc(int hidden, int policy_out, const floa
     if (!p) continue;
     if (reinterpret_cast<uintptr_t>(p) % 16 || !is_device_ptr(p)) return AUV_ERR_SIZE;
   }
+  if (status_out && (reinterpret_cast<uintptr_t>(status_out) % 4 || !is_device_ptr(status_out)))
+    return AUV_ERR_SIZE;
   unsigned char* base = nullptr;
   int rc = scratch_address(&base);
   if (rc) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   auv::Status* status = reinterpret_cast<auv::Status*>(base);
+  static_assert(sizeof(auv::Status) == sizeof(auv_status), "status block layout");
   void* pol_img = base + kStatusBytes;
   void* val_img = base + kStatusBytes + kPolicyRegion;
   // The array keeps the previous call's contents: reset the status word; the
@@ -94,5 +114,11 @@ extern "C" int env_policy_forward_noalloc(int hidden, int policy_out, const floa
   cudaError_t e = auv::launch_pack_bf16(M0, policy, value_w, pol_img, val_img, s);
   if (e != cudaSuccess) return AUV_ERR_CUDA;
   e = auv::launch_forward_bf16(M0, pol_img, val_img, nullptr, obs, n, head, value, status, s);
-  return e == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
+  if (e != cudaSuccess) return AUV_ERR_CUDA;
+  // The call's status word (a wait that gave up) for the caller, copied on
+  // the stream after the kernels.
+  if (status_out && cudaMemcpyAsync(status_out, status, sizeof(auv_status),
+                                    cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return AUV_ERR_CUDA;
+  return AUV_OK;
 }

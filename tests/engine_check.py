@@ -1,0 +1,135 @@
+"""Every-step check of a tensor-core (bf16) rollout against the oracle.
+
+The fused rollout kernel computes, per env and control step, the
+observation, the bf16 policy network, the Gaussian draw, the physics
+substeps, the reward and the done flag, and writes all of them to the
+trajectory.  This module checks every step of such a trajectory for a set of
+sampled envs:
+
+- physics: the oracle replays the kernel's own actions act[t] from the same
+  reset draw (action replay, so the comparison does not depend on the bf16
+  network's rounding): obs[t] of the oracle's state against the kernel's at
+  the fp32 tolerance, rew[t] per step, dones bit-exact, reward sums over
+  100-step windows, and the final state and counters;
+- network and draw: at every t the oracle's bf16 network on the kernel's
+  own obs[t], the oracle's log-std clamp and the oracle's normals of global
+  step t_g0 + t give a and log pi (oracle.policy_act), and the oracle's
+  bf16 value network gives V; the kernel's act, logp and value must agree
+  within the bf16 tolerance.
+
+Tolerances.  bf16 network outputs carry at most BF16_TOL (1e-2) absolute
+error (measured about 2e-3).  a = mu + sigma eps inherits the error of mu
+and sigma eps times that of the log-std, so |da| <= BF16_TOL (1 + sigma
+|eps|), with sigma |eps| = |a - mu| taken from the oracle.  log pi sums the
+log-std of every action component: |dlogp| <= act_dim * BF16_TOL.  The
+kernel's normals use the hardware log and sine (absolute error about 1e-6),
+far inside these bounds.
+
+Test infrastructure: used by tests/ and __graft_entry__.smoke() only.
+"""
+import numpy as np
+
+from paper_2512_13359_gb300 import workloads as W
+
+STATE_TOL = 1e-5          # per-step state and observation, fp32 vs double
+REWARD_TOL = 1e-4         # per-step reward (floor 1), and 100-step sums
+BF16_TOL = 1e-2           # bf16 network outputs (absolute)
+
+
+def _rel(gpu, ref, floor=1.0):
+    return np.abs(np.asarray(gpu, np.float64) - ref) / np.maximum(np.abs(ref), floor)
+
+
+def _check(cond, msg):
+    if not cond:
+        raise AssertionError(msg)
+
+
+def sample_ids(n, k=40, seed=5):
+    """k or more env ids of [0, n): both ends, the first tile boundary and
+    random ids."""
+    fixed = [0, 1, 127, 128, n - 2, n - 1]
+    rnd = np.random.default_rng(seed).integers(0, n, k)
+    ids = np.unique(np.clip(np.r_[fixed, rnd], 0, n - 1))
+    return ids.astype(np.int64)
+
+
+def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None):
+    """Check the trajectory `traj` (dict of torch tensors or numpy arrays
+    with the env's [T][K][N] layout) of a rollout of workload `w` that
+    started from the first reset draw at global step t_g0.  final_state:
+    optional (state, params, t_ep, episode) arrays of the env after the
+    rollout.  Returns the measured maxima."""
+    paper = W.is_paper(w)
+    n_all = int(w["n_envs"])
+    ids = np.asarray(ids, dtype=np.int64)
+    k = len(ids)
+    d, na = W.obs_dim(w), W.act_dim(w)
+
+    def take(key):
+        v = traj[key]
+        if hasattr(v, "detach"):
+            import torch
+            return v.detach().index_select(-1, torch.as_tensor(ids, device=v.device)).cpu().numpy()
+        return np.asarray(v)[..., ids]
+
+    g = {key: take(key) for key in traj}
+    _check(g["obs"].shape == (T, d, k), f"obs shape {g['obs'].shape}")
+    m = oracle.paper_model(w) if paper else oracle.model(w)
+    b = oracle.PaperBatch(ids) if paper else oracle.Batch(ids)
+    (oracle.paper_reset if paper else oracle.reset)(m, b)
+    pw = W.policy_weights(w)
+    vw = W.value_weights(w) if w["has_value"] else None
+    act_fn = oracle.paper_policy_act if paper else oracle.policy_act
+    replay = oracle.paper_replay if paper else oracle.replay
+    H = int(w["hidden"])
+    po = int(w["policy_out"])
+    worst = dict(obs=0.0, rew=0.0, act=0.0, logp=0.0, value=0.0)
+    rew_ref = np.zeros((T, k))
+    for t in range(T):
+        if paper:
+            ref_obs = np.stack([oracle.paper_observe(b.state[:, j], b.params[:, j])
+                                for j in range(k)], axis=1)
+        else:
+            ref_obs = np.stack([oracle.observe(b.state[:, j], b.params[:, j])[0]
+                                for j in range(k)], axis=1)
+        e = _rel(g["obs"][t], ref_obs)
+        worst["obs"] = max(worst["obs"], e.max())
+        _check(e.max() <= STATE_TOL, f"obs[{t}]: rel err {e.max():.3e}")
+        o = g["obs"][t].T.astype(np.float64)
+        a_ref, lp_ref = act_fn(m, pw, ids.astype(np.uint32), t_g0 + t, o)
+        mu = oracle.mlp(pw, d, H, po, True, o)[:, :na]
+        da = np.abs(g["act"][t].T - a_ref)
+        bound = BF16_TOL * (1.0 + np.abs(a_ref - mu))
+        worst["act"] = max(worst["act"], (da / (1.0 + np.abs(a_ref - mu))).max())
+        _check(np.all(da <= bound), f"act[{t}]: max excess {(da - bound).max():.3e}")
+        dl = np.abs(g["logp"][t] - lp_ref)
+        worst["logp"] = max(worst["logp"], dl.max())
+        _check(dl.max() <= na * BF16_TOL, f"logp[{t}]: {dl.max():.3e}")
+        if vw is not None and "value" in g:
+            v_ref = oracle.mlp(vw, d, H, 1, True, o)[:, 0]
+            dv = np.abs(g["value"][t] - v_ref).max()
+            worst["value"] = max(worst["value"], dv)
+            _check(dv <= BF16_TOL, f"value[{t}]: {dv:.3e}")
+        r, dn, _ = replay(m, b, np.ascontiguousarray(g["act"][t:t + 1], dtype=np.float32))
+        _check(np.array_equal(g["done"][t], dn[0]), f"done[{t}] differs")
+        e = _rel(g["rew"][t], r[0])
+        worst["rew"] = max(worst["rew"], e.max())
+        _check(e.max() <= REWARD_TOL, f"rew[{t}]: rel err {e.max():.3e}")
+        rew_ref[t] = r[0]
+    for t0 in range(0, T, 100):
+        s_g = g["rew"][t0:t0 + 100].astype(np.float64).sum(axis=0)
+        s_r = rew_ref[t0:t0 + 100].sum(axis=0)
+        e = _rel(s_g, s_r)
+        _check(e.max() <= REWARD_TOL, f"reward sum from step {t0}: rel err {e.max():.3e}")
+    if final_state is not None:
+        st, pr, t_ep, ep = final_state
+        e = _rel(np.asarray(st)[:, ids], b.state)
+        worst["state"] = e.max()
+        _check(e.max() <= STATE_TOL, f"final state: rel err {e.max():.3e}")
+        _check(np.array_equal(np.asarray(pr)[:, ids].astype(np.float32),
+                              b.params.astype(np.float32)), "final params differ")
+        _check(np.array_equal(np.asarray(t_ep)[ids], b.t_ep), "t_ep differs")
+        _check(np.array_equal(np.asarray(ep).view(np.uint32)[ids], b.episode), "episode differs")
+    _check(n_all >= int(ids.max()) + 1, "sampled id out of range")
+    return worst

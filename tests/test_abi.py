@@ -44,7 +44,7 @@ def test_library_exports_every_declared_symbol(auvlib):
     assert not missing, missing
     for n in names:
         assert hasattr(auvlib, n)
-    assert auvlib.env_abi_version() == 2
+    assert auvlib.env_abi_version() == 3
 
 
 def test_config_struct_size_matches_header(auvlib):

@@ -278,6 +278,58 @@ def test_checkpoint_resume_in_a_new_env(oracle):
     assert b.t_g == a.t_g == 55
 
 
+@pytest.mark.parametrize("name,host", [("dr_16384", True), ("paper_4096", False)])
+def test_snapshot_get_set_state(oracle, name, host):
+    """env_get_state / env_set_state: a snapshot (state, params, t_ep,
+    episode and the global step) taken mid-episode into page-locked host or
+    device arrays, restored into a fresh env, continues bit for bit (the
+    trajectory of the next launch, including resets inside it, and the final
+    arrays); snapshots that do not fit the env are rejected."""
+    torch = need_gpu()
+    from paper_2512_13359_gb300 import auvenv
+    n = 1000
+    w = W.workload(name, n_envs=n, episode_len=17)
+    a = make_env(w)
+    a.reset()
+    a.rollout(25, a.alloc_traj(25))
+    snap = {k: (torch.empty(getattr(a, k).shape, dtype=getattr(a, k).dtype, pin_memory=True)
+                if host else torch.empty_like(getattr(a, k)))
+            for k in ("state", "params", "t_ep", "episode")}
+    t_g = a.get_state(snap)
+    torch.cuda.synchronize()
+    assert t_g == 25 and snap["t_g"] == 25
+    for k in ("state", "params", "t_ep", "episode"):
+        assert torch.equal(snap[k].cuda(), getattr(a, k)), k
+    b = make_env(w)
+    b.set_state(snap)
+    assert b.t_g == 25
+    ta, tb = a.alloc_traj(30), b.alloc_traj(30)
+    a.rollout(30, ta)
+    b.rollout(30, tb)
+    for k in ta:
+        assert torch.equal(ta[k], tb[k]), k
+    for k in ("state", "params", "t_ep", "episode"):
+        assert torch.equal(getattr(a, k), getattr(b, k)), k
+    # snapshots of another batch size or model, a bad header, a misaligned array
+    c = make_env(dict(w, n_envs=n - 1))
+    with pytest.raises(auvenv.AuvError) as e:
+        c.set_state(snap)
+    assert e.value.code == auvenv.AUV_ERR_INVALID
+    other = W.workload("tiny_64" if W.is_paper(w) else "paper_tiny", n_envs=n)
+    d = make_env(other, policy=False)
+    with pytest.raises(auvenv.AuvError) as e:
+        d.set_state(dict(snap, model=a.cfg.model))
+    assert e.value.code == auvenv.AUV_ERR_INVALID
+    with pytest.raises(auvenv.AuvError) as e:
+        b.set_state(dict(snap, n_envs=n + 1))
+    assert e.value.code == auvenv.AUV_ERR_INVALID
+    raw = torch.empty(snap["t_ep"].numel() + 1, dtype=torch.int32, device="cuda")
+    bad = dict(snap, t_ep=raw.view(torch.uint8)[1:])   # one byte past a 4-byte boundary
+    with pytest.raises(auvenv.AuvError) as e:
+        b.get_state(bad)
+    assert e.value.code == auvenv.AUV_ERR_SIZE
+
+
 def test_nan_state_is_reported(oracle):
     torch = need_gpu()
     w = W.workload("tiny_64", n_envs=300)

@@ -287,3 +287,51 @@ def test_rollout_matches_replay_of_its_own_actions(oracle):
     assert np.array_equal(done, out["done"])
     assert np.allclose(rew, out["rew"], atol=1e-5)
     assert np.allclose(b1.state, b2.state, atol=1e-5)
+
+
+@pytest.mark.parametrize("model", ["fossen", "paper"])
+def test_logstd_clamp_pinned_beyond_both_bounds(oracle, model):
+    """The log-std clamp of the policy head (A6: [-5, 2]).  The head's
+    log-std rows are made constant by zero weights and biases of +50, -50,
+    0.3 and -0.7: the clamp must give sigma = e^2, e^-5, e^0.3 and e^-0.7.
+    Both the draw a - mu = sigma eps (normals pinned against cuRAND's words
+    and Box-Muller's moments elsewhere) and the log-density, against
+    scipy's normal logpdf at that sigma, are checked; a missing clamp
+    (sigma = e^50), swapped bounds (every sigma = e^-5 or e^2) or a dropped
+    term of the density fails.  The rollout's first step agrees with the
+    same draw."""
+    stats = pytest.importorskip("scipy.stats")
+    paper = model == "paper"
+    w = W.workload("paper_4096" if paper else "ppo_65536", n_envs=6)
+    na = W.act_dim(w)
+    d = W.obs_dim(w)
+    pw = W.policy_weights(w, 0.1).astype(np.float32).copy()
+    H = w["hidden"]
+    o3 = H * d + H + H * H + H          # start of W3 [2 na][H]
+    heads = np.array([50.0, -50.0, 0.3, -0.7, 50.0, -50.0, 0.3, -0.7][:na], dtype=np.float32)
+    pw[o3 + na * H:o3 + 2 * na * H] = 0.0
+    pw[o3 + 2 * na * H + na:o3 + 2 * na * H + 2 * na] = heads
+    # the fp32 biases are the head's exact outputs (zero weights)
+    sig = np.exp(np.clip(heads.astype(np.float64), -5.0, 2.0))
+    assert np.allclose(np.log(sig), [2.0, -5.0, 0.3, -0.7, 2.0, -5.0, 0.3, -0.7][:na],
+                       atol=1e-7)
+    ids = np.array([0, 3, 17, 4095, 65535, 123456])
+    obs = W.random_observations(9, len(ids), d)
+    t_g = 77
+    m = oracle.paper_model(w) if paper else oracle.model(w)
+    act_fn = oracle.paper_policy_act if paper else oracle.policy_act
+    act, logp = act_fn(m, pw, ids, t_g, obs.astype(np.float64))
+    mu = oracle.mlp(pw, d, H, 2 * na, True, obs.astype(np.float64))[:, :na]
+    for i, e in enumerate(ids):
+        eps = oracle.normals(int(e), int(w["seed"]), t_g)[:na]
+        assert np.allclose(act[i] - mu[i], sig * eps, rtol=1e-12, atol=1e-12)
+        lp = stats.norm.logpdf(act[i], loc=mu[i], scale=sig).sum()
+        assert math.isclose(logp[i], lp, rel_tol=1e-10, abs_tol=1e-9)
+    # the rollout's step 0 takes the same draw from its own observation
+    b = oracle.PaperBatch(ids) if paper else oracle.Batch(ids)
+    (oracle.paper_reset if paper else oracle.reset)(m, b)
+    roll = oracle.paper_rollout if paper else oracle.rollout
+    out = roll(m, b, pw, None, t_g, 1, want=("obs", "act", "logp"))
+    a0, lp0 = act_fn(m, pw, ids, t_g, out["obs"][0].T)
+    assert np.allclose(out["act"][0].T, a0, rtol=1e-12, atol=1e-12)
+    assert np.allclose(out["logp"][0], lp0, rtol=1e-12, atol=1e-12)
