@@ -1586,10 +1586,11 @@ void oracle_paper_rollout(const PaperModel* m, int precision, const float* pol_w
 // clamped head or the fixed vector (A6), eps = the first n_act normals of the
 // action-noise stream at global step t_g, a = mu + exp(log sigma) eps and
 // log pi(a) = sum(-eps^2/2 - log sigma - log(2 pi)/2), as one step of the
-// rollout computes them.  obs[n][obs_dim] row-major; act[n][n_act], logp[n].
+// rollout computes them.  obs[n][obs_dim] row-major; act[n][n_act], logp[n]
+// and, if mu is not NULL, the mean mu[n][n_act].
 void oracle_policy_act(const OracleModel* m, const float* pol_w, int n,
                        const uint32_t* env_ids, uint64_t t_g, const double* obs, double* act,
-                       double* logp) {
+                       double* logp, double* mu_out) {
   const double half_log_2pi = 0.91893853320467274178032973640562;
   for (int i = 0; i < n; ++i) {
     double mu[kAct], logstd[kAct];
@@ -1604,6 +1605,7 @@ void oracle_policy_act(const OracleModel* m, const float* pol_w, int n,
     for (int k = 0; k < kAct; ++k) {
       act[(size_t)i * kAct + k] = mu[k] + std::exp(logstd[k]) * eps[k];
       lp += -0.5 * eps[k] * eps[k] - logstd[k] - half_log_2pi;
+      if (mu_out) mu_out[(size_t)i * kAct + k] = mu[k];
     }
     logp[i] = lp;
   }
@@ -1611,7 +1613,7 @@ void oracle_policy_act(const OracleModel* m, const float* pol_w, int n,
 
 void oracle_paper_policy_act(const PaperModel* m, const float* pol_w, int n,
                              const uint32_t* env_ids, uint64_t t_g, const double* obs,
-                             double* act, double* logp) {
+                             double* act, double* logp, double* mu_out) {
   const double half_log_2pi = 0.91893853320467274178032973640562;
   for (int i = 0; i < n; ++i) {
     double out[12];
@@ -1633,6 +1635,7 @@ void oracle_paper_policy_act(const PaperModel* m, const float* pol_w, int n,
       }
       act[(size_t)i * kPAct + k] = out[k] + std::exp(ls) * eps[k];
       lp += -0.5 * eps[k] * eps[k] - ls - half_log_2pi;
+      if (mu_out) mu_out[(size_t)i * kPAct + k] = out[k];
     }
     logp[i] = lp;
   }

@@ -79,7 +79,7 @@ def lib():
         _lib.oracle_rollout.argtypes = [P, C.c_int, P, P, C.c_int, P, P, P, P, P, C.c_uint64,
                                         C.c_int, P, P, P, P, P, P]
         _lib.oracle_mlp.argtypes = [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, P]
-        _lib.oracle_policy_act.argtypes = [P, P, C.c_int, P, C.c_uint64, P, P, P]
+        _lib.oracle_policy_act.argtypes = [P, P, C.c_int, P, C.c_uint64, P, P, P, P]
         _lib.oracle_observe.argtypes = [P, P, P, P]
         _lib.oracle_reward.argtypes = [P, P, P, P]
         _lib.oracle_reward.restype = C.c_double
@@ -244,19 +244,22 @@ def mlp(weights: np.ndarray, in_dim: int, hidden: int, out_dim: int, bf16: bool,
     return out
 
 
-def policy_act(m: OracleModel, pol_w, env_ids, t_g: int, obs: np.ndarray):
+def policy_act(m: OracleModel, pol_w, env_ids, t_g: int, obs: np.ndarray, with_mu=False):
     """One policy draw per row of obs[n][18] (env ids env_ids, global step
     t_g): the network head, the clamped (or fixed) log-std, the step's
-    normals, a = mu + sigma eps and log pi(a).  Returns (act[n][8], logp[n])."""
+    normals, a = mu + sigma eps and log pi(a).  Returns (act[n][8], logp[n])
+    and, with with_mu, the mean mu[n][8] as a third array."""
     ids = np.ascontiguousarray(env_ids, dtype=np.uint32)
     x = np.ascontiguousarray(obs, dtype=np.float64)
     n = len(ids)
     assert x.shape == (n, 18)
     act = np.zeros((n, 8))
     logp = np.zeros(n)
+    mu = np.zeros((n, 8)) if with_mu else None
     pw = np.ascontiguousarray(pol_w, dtype=np.float32)
-    lib().oracle_policy_act(C.byref(m), _p(pw), n, _p(ids), int(t_g), _p(x), _p(act), _p(logp))
-    return act, logp
+    lib().oracle_policy_act(C.byref(m), _p(pw), n, _p(ids), int(t_g), _p(x), _p(act), _p(logp),
+                            _p(mu))
+    return (act, logp, mu) if with_mu else (act, logp)
 
 
 def philox(key0: int, key1: int, ctr) -> np.ndarray:
@@ -382,7 +385,7 @@ def _paper_lib():
         L.oracle_paper_rollout.argtypes = [P, C.c_int, P, P, C.c_int, P, P, P, P, P,
                                            C.c_uint64, C.c_int, P, P, P, P, P, P]
         L.oracle_paper_observe.argtypes = [P, P, P]
-        L.oracle_paper_policy_act.argtypes = [P, P, C.c_int, P, C.c_uint64, P, P, P]
+        L.oracle_paper_policy_act.argtypes = [P, P, C.c_int, P, C.c_uint64, P, P, P, P]
         L.oracle_paper_reward.argtypes = [P, P, P, P]
         L.oracle_paper_reward.restype = C.c_double
         L.oracle_paper_wrench.argtypes = [P, P, P, P]
@@ -537,18 +540,20 @@ def paper_rollout(m: PaperModel, batch: PaperBatch, pol_w, val_w, t_g0: int, T: 
     return {k: v for k, v in out.items() if v is not None}
 
 
-def paper_policy_act(m: PaperModel, pol_w, env_ids, t_g: int, obs: np.ndarray):
-    """The paper model's policy draw per row of obs[n][12]: (act[n][6], logp[n])."""
+def paper_policy_act(m: PaperModel, pol_w, env_ids, t_g: int, obs: np.ndarray, with_mu=False):
+    """The paper model's policy draw per row of obs[n][12]: (act[n][6],
+    logp[n]) and, with with_mu, the mean mu[n][6]."""
     ids = np.ascontiguousarray(env_ids, dtype=np.uint32)
     x = np.ascontiguousarray(obs, dtype=np.float64)
     n = len(ids)
     assert x.shape == (n, PAPER_OBS)
     act = np.zeros((n, PAPER_ACT))
     logp = np.zeros(n)
+    mu = np.zeros((n, PAPER_ACT)) if with_mu else None
     pw = np.ascontiguousarray(pol_w, dtype=np.float32)
     _paper_lib().oracle_paper_policy_act(C.byref(m), _p(pw), n, _p(ids), int(t_g), _p(x),
-                                         _p(act), _p(logp))
-    return act, logp
+                                         _p(act), _p(logp), _p(mu))
+    return (act, logp, mu) if with_mu else (act, logp)
 
 
 def paper_single_env(state: dict, params: dict):

@@ -408,11 +408,13 @@ class Env:
         sn = AuvSnapshot(C.sizeof(AuvSnapshot), 0, 0, 0, 0, 0, 0,
                          *(snap[k].data_ptr() for k in ("state", "params", "t_ep", "episode")))
         self._check(lib().env_get_state(self.h, C.byref(sn), _stream(stream)))
-        snap["t_g"] = int(sn.t_g)
+        snap.update(t_g=int(sn.t_g), model=int(sn.model), n_envs=int(sn.n_envs),
+                    state_fields=int(sn.state_fields), param_fields=int(sn.param_fields))
         return int(sn.t_g)
 
     def set_state(self, snap: dict, stream=None):
-        """env_set_state from snap's tensors and t_g (as get_state filled it)."""
+        """env_set_state from snap's tensors, t_g and header fields (model,
+        n_envs, field counts; as get_state filled them, else this env's)."""
         lay = AuvLayout()
         lib().env_layout(self.cfg.model, C.byref(lay))
         sn = AuvSnapshot(C.sizeof(AuvSnapshot), snap.get("model", self.cfg.model),

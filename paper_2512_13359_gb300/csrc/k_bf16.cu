@@ -611,6 +611,12 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       // layer 1 -> h1 slot.  Chunk c's bf16 pairs go to slot columns
       // 32c..32c+31, which held accumulator columns this thread has already
       // read (chunk 0's second half for c = 1, chunk 1's for c = 2, 3).
+      // The Fossen rollout keeps this loop rolled: its hot loop (network
+      // epilogues, sampling, physics) otherwise outgrows the SM's instruction
+      // cache, and with every SM busy the misses cost more than the loop
+      // (2.52 -> 2.19 ms at 152 CTAs, 2.02 -> 1.95 ms at 128).  The paper
+      // model and the row modes run faster unrolled.
+#pragma unroll(MODE == kRollout && SIM == 0 ? 1 : 4)
       for (int c = 0; c < kNChunks; ++c) {
         uint64_t* full = c == 0 ? &bar->full_l1a[g] : (c == 1 ? &bar->full_l1b[g] : &bar->full_x[g]);
         if (!tc::mbar_wait(full, c < 2 ? (uint32_t)it & 1u : (uint32_t)c & 1u, abort, kWaitLimitNs))

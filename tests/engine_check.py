@@ -10,7 +10,13 @@ sampled envs:
   reset draw (action replay, so the comparison does not depend on the bf16
   network's rounding): obs[t] of the oracle's state against the kernel's at
   the fp32 tolerance, rew[t] per step, dones bit-exact, reward sums over
-  100-step windows, and the final state and counters;
+  100-step windows, and the final state and counters.  Over a long launch
+  the fp32 trajectory drifts from the double one by accumulated rounding
+  (about 1e-5 relative after some 400 steps of the paper model); for such
+  launches the caller passes the kernel's own state at window starts
+  (`resync`, from the same rollout run in windows, which is bit-identical),
+  and the oracle restarts from it, so each window is held to the fp32
+  tolerance from a common state;
 - network and draw: at every t the oracle's bf16 network on the kernel's
   own obs[t], the oracle's log-std clamp and the oracle's normals of global
   step t_g0 + t give a and log pi (oracle.policy_act), and the oracle's
@@ -54,12 +60,14 @@ def sample_ids(n, k=40, seed=5):
     return ids.astype(np.int64)
 
 
-def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None):
+def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None, resync=None):
     """Check the trajectory `traj` (dict of torch tensors or numpy arrays
     with the env's [T][K][N] layout) of a rollout of workload `w` that
     started from the first reset draw at global step t_g0.  final_state:
     optional (state, params, t_ep, episode) arrays of the env after the
-    rollout.  Returns the measured maxima."""
+    rollout.  resync: optional {t: (state, params, t_ep, episode)} of the
+    kernel's batch before step t; the oracle continues from it.  Returns the
+    measured maxima."""
     paper = W.is_paper(w)
     n_all = int(w["n_envs"])
     ids = np.asarray(ids, dtype=np.int64)
@@ -83,10 +91,15 @@ def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None):
     act_fn = oracle.paper_policy_act if paper else oracle.policy_act
     replay = oracle.paper_replay if paper else oracle.replay
     H = int(w["hidden"])
-    po = int(w["policy_out"])
     worst = dict(obs=0.0, rew=0.0, act=0.0, logp=0.0, value=0.0)
     rew_ref = np.zeros((T, k))
     for t in range(T):
+        if resync and t in resync:
+            st, pr, t_ep, ep = (np.asarray(x) for x in resync[t])
+            b.state[:] = st[:, ids]
+            b.params[:] = pr[:, ids]
+            b.t_ep[:] = t_ep[ids]
+            b.episode[:] = ep.view(np.uint32)[ids]
         if paper:
             ref_obs = np.stack([oracle.paper_observe(b.state[:, j], b.params[:, j])
                                 for j in range(k)], axis=1)
@@ -97,8 +110,7 @@ def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None):
         worst["obs"] = max(worst["obs"], e.max())
         _check(e.max() <= STATE_TOL, f"obs[{t}]: rel err {e.max():.3e}")
         o = g["obs"][t].T.astype(np.float64)
-        a_ref, lp_ref = act_fn(m, pw, ids.astype(np.uint32), t_g0 + t, o)
-        mu = oracle.mlp(pw, d, H, po, True, o)[:, :na]
+        a_ref, lp_ref, mu = act_fn(m, pw, ids.astype(np.uint32), t_g0 + t, o, with_mu=True)
         da = np.abs(g["act"][t].T - a_ref)
         bound = BF16_TOL * (1.0 + np.abs(a_ref - mu))
         worst["act"] = max(worst["act"], (da / (1.0 + np.abs(a_ref - mu))).max())
