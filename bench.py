@@ -481,11 +481,12 @@ def run_gae(args):
 
 # DRAM bytes (read + write) of one rollout launch of the 65,536-env x
 # 128-step workload, from one ncu capture (dram__bytes_read.sum +
-# dram__bytes_write.sum, 1 pass, `bench.py --steps 1 --warmup 1 --no-e2e
-# --no-cpu-baseline --no-clocks`; profiles/k_engine_ppo_65536_T128_dram.md),
-# valid while the engine's sources hash to ENGINE_SRC_HASH.
-ROLLOUT_TRAFFIC_65536x128 = 10_783_232 + 902_189_056
-ENGINE_SRC_HASH = "7832b756ffc66fe2"
+# dram__bytes_write.sum, 1 pass, the first timed rollout of `bench.py
+# --steps 2 --warmup 1 --no-e2e --no-cpu-baseline --no-replay --no-clocks`;
+# profiles/k_engine_ppo_65536_T128_dram.md), valid while the engine's sources
+# hash to ENGINE_SRC_HASH.
+ROLLOUT_TRAFFIC_65536x128 = 10_482_176 + 900_390_144
+ENGINE_SRC_HASH = "e5a53d13eb31f1f0"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 
