@@ -702,6 +702,33 @@ int env_clear_status(auv_env* env, void* stream);
 int env_selftest_wait_timeout(auv_env* env, uint32_t limit_us, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * The learners' dense product (the contractions of the PPO update and of the
+ * SHAC window, paper §III-A), on its own:
+ *
+ *   C[M][N] = beta * C + sum_{k < K} A(m, k) B(n, k)
+ *
+ * A(m, k) is A[m * lda + k] (a_mn = 0: rows are the M index, K contiguous)
+ * or A[k * lda + m] (a_mn = 1: a sample-major array read along its samples,
+ * as in a weight gradient); B(n, k) likewise with ldb, b_mn.  C is row-major
+ * with ldc >= N, fp32, or bf16 with c_bf16 = 1 (bf16 precision only; rounded
+ * to nearest even).  precision: AUV_PPO_BF16 (bf16 A and B, tcgen05
+ * kind::f16), AUV_PPO_TF32 (fp32 A and B read as tf32, tcgen05 kind::tf32)
+ * or AUV_PPO_FP32 (fp32 on CUDA cores); accumulation is fp32.  Tensor-core
+ * precisions need A, B 16-byte aligned and lda, ldb times the element size a
+ * multiple of 16 bytes (else AUV_ERR_SIZE).  workspace (device, or NULL):
+ * room for the fp32 partials of a contraction split over CTAs, at least
+ * auv_gemm_workspace_bytes(M, N, K) bytes for the split to be used;
+ * partials are added in a fixed order, so results are reproducible.
+ * status: a device auv_status the kernels latch AUV_ERR_TIMEOUT into if a
+ * bounded wait gives up.  Asynchronous on stream.  Returns AUV_OK,
+ * AUV_ERR_INVALID, AUV_ERR_SIZE or AUV_ERR_CUDA.
+ * --------------------------------------------------------------------------- */
+size_t auv_gemm_workspace_bytes(int M, int N, int K);
+int auv_gemm(uint32_t precision, int M, int N, int K, const void* A, int lda, int a_mn,
+             const void* B, int ldb, int b_mn, void* C, int ldc, int c_bf16, float beta,
+             void* workspace, size_t workspace_bytes, auv_status* status, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Roofline probes (measurement helpers, not on any hot path).  Each enqueues
  * work of a known operation count on `stream`; the caller times it.
  *

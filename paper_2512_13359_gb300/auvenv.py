@@ -48,6 +48,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "ppo_create", "ppo_destroy", "ppo_last_error", "ppo_param_counts", "ppo_set_weights",
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
             "ppo_update", "ppo_export_weights", "ppo_status", "ppo_clear_status",
+            "auv_gemm", "auv_gemm_workspace_bytes",
             "auv_probe_ffma", "auv_probe_tanh", "auv_probe_gemm")
 
 
@@ -196,6 +197,10 @@ def lib(path: str | None = None):
     L.auv_probe_ffma.argtypes = [U32, U32, U32, P, P]
     L.auv_probe_tanh.argtypes = [U32, U32, U32, P, P]
     L.auv_probe_gemm.argtypes = [U32, I, P, P, P, P]
+    L.auv_gemm_workspace_bytes.argtypes = [I, I, I]
+    L.auv_gemm_workspace_bytes.restype = C.c_size_t
+    L.auv_gemm.argtypes = [U32, I, I, I, P, I, I, P, I, I, P, I, I, C.c_float, P, C.c_size_t, P,
+                           P]
     L.ppo_clear_status.argtypes = [P, P]
     for name in EXPORTED:
         getattr(L, name).restype = getattr(L, name).restype or I
@@ -651,3 +656,25 @@ class ReplayBuffer:
                                       _ptr(out["rew"]), _ptr(out["next_obs"]), _ptr(out["done"]),
                                       _ptr(out.get("idx")), _stream(stream)))
         return out
+
+
+def gemm(precision: str, M: int, N: int, K: int, A, lda: int, a_mn: bool, B, ldb: int,
+         b_mn: bool, Cout, ldc: int, beta: float = 0.0, workspace=None, status=None,
+         stream=None):
+    """auv_gemm on torch device tensors: Cout[M][N] = beta Cout + A B^T with
+    A(m, k) = A[m*lda + k] (a_mn False) or A[k*lda + m] (a_mn True), B
+    likewise.  precision 'bf16' | 'tf32' | 'fp32'; Cout fp32 or bf16.
+    status: int32 device tensor of 4 (allocated if None).  Returns status."""
+    import torch
+    if status is None:
+        status = torch.zeros(4, dtype=torch.int32, device=Cout.device)
+    ws_ptr = C.c_void_p(workspace.data_ptr()) if workspace is not None else None
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = lib().auv_gemm(PPO_PRECISION[precision], M, N, K, C.c_void_p(A.data_ptr()), lda,
+                        int(a_mn), C.c_void_p(B.data_ptr()), ldb, int(b_mn),
+                        C.c_void_p(Cout.data_ptr()), ldc, int(Cout.dtype == torch.bfloat16),
+                        float(beta), ws_ptr, ws_bytes, C.c_void_p(status.data_ptr()),
+                        _stream(stream))
+    if rc != AUV_OK:
+        raise AuvError(rc, "auv_gemm")
+    return status

@@ -22,7 +22,7 @@ def auvlib():
 def header_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\**\s*((?:env|ppo|rbuf|auv_probe)_\w+)\s*\(", text,
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\**\s*((?:env|ppo|rbuf|auv_probe)_\w+|auv_gemm\w*)\s*\(", text,
                                  flags=re.M)))
 
 
