@@ -409,13 +409,14 @@ int env_gae(auv_env* env, int T, const float* rew, const uint8_t* done, const fl
  * TD(lambda) targets are env_gae's returns); the policy is neither run nor
  * changed, and batch.act, .logp, .adv may be NULL. */
 #define AUV_PPO_GEMM_PATH 2u /* flags: in bf16 mode, run the forward pass and
- * the input gradients through cuBLAS GEMMs and tanh passes.  Without it a
- * bf16 learner with hidden == 256, obs_dim <= 18 runs both networks' forward
- * passes and their backward-data (dL/dZ2, dL/dZ1 with the tanh derivatives)
- * on the tcgen05 engine of env_rollout (weights, and their transposes,
- * packed from the fp32 master copy every step; tanh on the fp32
- * pre-activation, each product rounded to bf16 once); the weight gradients
- * stay cuBLAS GEMMs. */
+ * the input gradients as separate GEMMs (auv_gemm) and tanh passes.  Without
+ * it a bf16 learner with hidden == 256, obs_dim <= 18 runs both networks'
+ * forward passes and their backward-data (dL/dZ2, dL/dZ1 with the tanh
+ * derivatives) on the tcgen05 engine of env_rollout (weights, and their
+ * transposes, packed from the fp32 master copy every step; tanh on the fp32
+ * pre-activation, each product rounded to bf16 once).  The weight gradients
+ * are tcgen05 GEMMs over the minibatch (auv_gemm) in every mode.  All
+ * products of every precision run in the library's own kernels. */
 #define AUV_PPO_STATS 8   /* floats in a statistics record:                       */
 /* [0] surrogate (policy) loss, [1] value loss (mean (V - ret)^2 / 2),
  * [2] entropy, [3] approx. KL mean(logp_old - logp), [4] clip fraction

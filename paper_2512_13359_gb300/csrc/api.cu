@@ -8,7 +8,6 @@
 #include <cstring>
 #include <new>
 
-#include <cublas_v2.h>
 
 #include "auv_kernels.h"
 #include "auv_bf16.h"
@@ -49,12 +48,11 @@ struct auv_env {
   // Inverse allocation (env_inverse_allocate): made on first use.
   bool inv_ready = false;
   auv::InvAlloc inv;
-  // SHAC windows (env_shac_window): workspace for the last (N, T, H) and a
-  // cuBLAS handle, made on first use.
+  // SHAC windows (env_shac_window): workspace for the last (N, T, H), made on
+  // first use.
   char* shac_ws = nullptr;
   size_t shac_ws_bytes = 0;
   int shac_T = 0;
-  cublasHandle_t blas = nullptr;
 };
 
 namespace {
@@ -429,7 +427,6 @@ int env_destroy(auv_env* env) {
   if (env->stage) cudaFree(env->stage);
   if (env->adj_scratch) cudaFree(env->adj_scratch);
   if (env->shac_ws) cudaFree(env->shac_ws);
-  if (env->blas) cublasDestroy(env->blas);
   for (int b = 0; b < 2; ++b) {
     if (env->seg_done[b]) cudaEventDestroy(env->seg_done[b]);
     if (env->copy_done[b]) cudaEventDestroy(env->copy_done[b]);
@@ -784,13 +781,6 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
     return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const auv::shac::Layout L = auv::shac::layout(env->model.n, T, H, is_paper(&env->cfg));
-  if (!env->blas) {
-    cublasStatus_t bs = cublasCreate(&env->blas);
-    if (bs != CUBLAS_STATUS_SUCCESS) {
-      env->blas = nullptr;
-      return fail(env, AUV_ERR_CUDA, "cuBLAS handle: status %d", (int)bs);
-    }
-  }
   if (L.bytes > env->shac_ws_bytes || T != env->shac_T) {
     if (L.bytes > env->shac_ws_bytes) {
       if (env->shac_ws) {
@@ -810,7 +800,7 @@ int env_shac_window(auv_env* env, const float* policy, const float* value, int T
     if (e != cudaSuccess) return cuda_fail(env, e, "initialise SHAC workspace");
     env->shac_T = T;
   }
-  rc = auv::shac::run_window(env->blas, env->model, env->buf, env->status, L, env->shac_ws,
+  rc = auv::shac::run_window(env->model, env->buf, env->status, L, env->shac_ws,
                              env->t_g, policy, value, coef, coef_V, precision == AUV_PPO_TF32,
                              grad, static_cast<float*>(J),
                              obs_out, static_cast<float*>(rew), static_cast<uint8_t*>(done), s,

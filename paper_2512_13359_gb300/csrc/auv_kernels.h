@@ -72,14 +72,14 @@ struct Layout {
   int D, out, S;     // network input, policy head width, adjoint rows (model)
   size_t n_aug_p, n_aug_v;
   size_t o_X, o_H1, o_H2, o_Y, o_G, o_GX, o_gY, o_lam, o_done, o_rew, o_VH1, o_VH2, o_V, o_gYv,
-      o_wp, o_wv, o_gp, o_sc, bytes;
+      o_wp, o_wv, o_gp, o_sc, o_gws, gws_bytes, bytes;
 };
 // paper: the paper model (input 12, head 12, 61 adjoint rows), else Fossen
 // (18, 16, 13).
 Layout layout(int n, int T, int H, bool paper);
 cudaError_t init(const Layout& L, char* base, cudaStream_t s);
-// blas: a cublasHandle_t.  Returns AUV_OK or an AUV_ERR_* code with err set.
-int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
+// Returns AUV_OK or an AUV_ERR_* code with err set.
+int run_window(const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
                const float* coef, float coef_V, bool tf32, float* grad, float* J,
                float* obs_out, float* rew_out, uint8_t* done_out, cudaStream_t s, char* err);

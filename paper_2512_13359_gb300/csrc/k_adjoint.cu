@@ -451,7 +451,7 @@ __global__ void __launch_bounds__(kAdjThreads, 4) k_adjoint(
 
 // ---------------------------------------------------------------------------
 // SHAC in closed loop: the window's steps one at a time, with the policy
-// network's products done outside (cuBLAS) between these kernels.
+// network's products done outside (k_gemm.cu) between these kernels.
 // ---------------------------------------------------------------------------
 
 // dJ/d(state) += (d obs / d state)^T lo for the observation of auv_device.cuh.

@@ -102,6 +102,7 @@ struct TcArgs {
   float* ws;              // split partials, or null (write C directly)
   int n_pad, m_pad;
   Status* st;
+  int vec;                // C base and ldc allow 16-byte row segments
 };
 
 template <bool TF32, bool A_MN, bool B_MN, int BN>
@@ -241,6 +242,28 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
             dst[q] = make_float4(__uint_as_float(acc[4 * q]), __uint_as_float(acc[4 * q + 1]),
                                  __uint_as_float(acc[4 * q + 2]), __uint_as_float(acc[4 * q + 3]));
         }
+      } else if (row < args.M && args.beta == 0.0f && nb + 32 <= args.N && args.vec) {
+        // whole 32-column segment, 16-byte aligned rows: vector stores
+        if (args.c_bf16) {
+          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(args.C) +
+                                                (size_t)row * args.ldc + nb);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              w[e] = tc::pack_bf16x2(__uint_as_float(acc[8 * q + 2 * e]),
+                                     __uint_as_float(acc[8 * q + 2 * e + 1]));
+            dst[q] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        } else {
+          float4* dst = reinterpret_cast<float4*>(static_cast<float*>(args.C) +
+                                                  (size_t)row * args.ldc + nb);
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            dst[q] = make_float4(__uint_as_float(acc[4 * q]), __uint_as_float(acc[4 * q + 1]),
+                                 __uint_as_float(acc[4 * q + 2]), __uint_as_float(acc[4 * q + 3]));
+        }
       } else if (row < args.M) {
         if (args.c_bf16) {
           uint16_t* crow = static_cast<uint16_t*>(args.C) + (size_t)row * args.ldc;
@@ -339,21 +362,52 @@ k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const flo
   }
 }
 
-// C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output.
+// C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output; four
+// consecutive columns per thread (n_pad is a multiple of 64), the split loop
+// unrolled so that several partial loads are in flight.
 __global__ void k_reduce(int M, int N, int splits, const float* __restrict__ ws, int m_pad,
                          int n_pad, void* C, int ldc, int c_bf16, float beta) {
+  const int nq = (N + 3) >> 2;
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (size_t)M * N) return;
-  const int m = (int)(idx / N), n = (int)(idx % N);
-  float v = 0.0f;
-  for (int z = 0; z < splits; ++z) v += ws[((size_t)z * m_pad + m) * n_pad + n];
-  if (c_bf16) {
-    uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
-    if (beta != 0.0f) v = fmaf(beta, __uint_as_float((uint32_t)*c << 16), v);
-    *c = (uint16_t)(tc::pack_bf16x2(v, 0.0f) & 0xFFFFu);
-  } else {
-    float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
-    *c = beta != 0.0f ? fmaf(beta, *c, v) : v;
+  if (idx >= (size_t)M * nq) return;
+  const int m = (int)(idx / nq), n0 = 4 * (int)(idx % nq);
+  const size_t zs = (size_t)m_pad * n_pad;
+  const float4* src = reinterpret_cast<const float4*>(ws + (size_t)m * n_pad + n0);
+  float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  int z = 0;
+  for (; z + 4 <= splits; z += 4) {
+    float4 p[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) p[q] = __ldg(src + (z + q) * (zs >> 2));
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      v.x += p[q].x;
+      v.y += p[q].y;
+      v.z += p[q].z;
+      v.w += p[q].w;
+    }
+  }
+  for (; z < splits; ++z) {
+    const float4 p = __ldg(src + z * (zs >> 2));
+    v.x += p.x;
+    v.y += p.y;
+    v.z += p.z;
+    v.w += p.w;
+  }
+  const float r[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int n = n0 + q;
+    if (n >= N) break;
+    float x = r[q];
+    if (c_bf16) {
+      uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
+      if (beta != 0.0f) x = fmaf(beta, __uint_as_float((uint32_t)*c << 16), x);
+      *c = (uint16_t)(tc::pack_bf16x2(x, 0.0f) & 0xFFFFu);
+    } else {
+      float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
+      *c = beta != 0.0f ? fmaf(beta, *c, x) : x;
+    }
   }
 }
 
@@ -410,7 +464,9 @@ bool make_map(CUtensorMap* map, bool tf32, const void* ptr, uint64_t inner, uint
   const cuuint64_t strides[1] = {(cuuint64_t)ld * es};
   const cuuint32_t box[2] = {(cuuint32_t)(128 / es), box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  return fn(map, tf32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+  // tf32: the copy rounds each fp32 element to tf32 (nearest), as a tf32
+  // GEMM rounds its operands, instead of the MMA dropping the low bits
+  return fn(map, tf32 ? CU_TENSOR_MAP_DATA_TYPE_TFLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
             const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -562,7 +618,9 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
     const bool ok_b = B.mn_major ? make_map(&mb, tf32, B.ptr, N, K, B.ld, bk)
                                  : make_map(&mb, tf32, B.ptr, K, N, B.ld, P.bn);
     if (!ok_a || !ok_b) return cudaErrorInvalidValue;
-    TcArgs a = {M, N, K, P.per_split, C, ldc, c_bf16 ? 1 : 0, beta, part, P.n_pad, P.m_pad, st};
+    const int ces = c_bf16 ? 2 : 4;
+    const int vec = (reinterpret_cast<uintptr_t>(C) % 16 == 0 && ((size_t)ldc * ces) % 16 == 0) ? 1 : 0;
+    TcArgs a = {M, N, K, P.per_split, C, ldc, c_bf16 ? 1 : 0, beta, part, P.n_pad, P.m_pad, st, vec};
     if (tf32)
       e = P.bn == 256 ? dispatch_major<true, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)
                       : dispatch_major<true, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
@@ -571,7 +629,7 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
                       : dispatch_major<false, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
   }
   if (e != cudaSuccess || !part) return e;
-  const size_t n = (size_t)M * N;
+  const size_t n = (size_t)M * ((N + 3) / 4);
   k_reduce<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(M, N, P.splits, part, P.m_pad, P.n_pad, C,
                                                        ldc, c_bf16 ? 1 : 0, beta);
   return cudaGetLastError();

@@ -155,7 +155,7 @@ cudaError_t launch_gae(int n, int T, const float* rew, const uint8_t* done, cons
 
 // ---------------------------------------------------------------------------
 // PPO minibatch update (Schulman et al. 2017).  The GEMMs of the two MLPs run
-// in cuBLAS (the host side); these kernels do everything around them: the
+// in k_gemm.cu and the tcgen05 engine; these kernels do everything around them: the
 // epoch permutation and minibatch gather, tanh forward and backward, the
 // per-sample loss and its gradient at the heads, the minibatch statistics,
 // the global gradient norm and Adam, and the weight-layout conversion.

@@ -1,8 +1,10 @@
 // ppo_api.cu -- the PPO learner's extern "C" entry points (include/auvenv.h):
 // validation, the learner's device memory, and the sequence of one gradient
 // step: gather -> forward GEMMs + tanh -> loss head -> backward GEMMs + tanh'
-// -> (gradient norm, Adam).  The dense products are plain GEMMs and run in
-// cuBLAS; every other step runs in the kernels of k_ppo.cu.  Precision modes:
+// -> (gradient norm, Adam).  The dense products run in the library's GEMM
+// (k_gemm.cu) and, in bf16 mode, the forward and backward-data passes on the
+// tensor-core engine (k_bf16.cu); every other step runs in the kernels of
+// k_ppo.cu.  Precision modes:
 //   fp32  fp32 activations, fp32 GEMMs on the CUDA cores;
 //   tf32  fp32 activations, tensor-core GEMMs with tf32 operands;
 //   bf16  bf16 activations, backward signals and weight copy (the GEMM
@@ -18,8 +20,8 @@
 // sample-major copy of its batch (rows of round8(D + A + 3) floats), made
 // once per call, from which every step gathers its minibatch; it grows when a
 // larger batch arrives and lives until ppo_destroy.
-#include <cublas_v2.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -30,6 +32,7 @@
 
 #include "auv_bf16.h"
 #include "auv_device.cuh"
+#include "auv_gemm.h"
 #include "auv_kernels.h"
 #include "auvenv.h"
 
@@ -39,14 +42,11 @@ using auv::Status;
 struct auv_ppo {
   auv_ppo_config cfg;
   int device;
-  cublasHandle_t blas;
-  cublasComputeType_t ctype;
   ppo::Dims d;
   int out[2];                 // head widths: 2A (policy), 1 (value)
   size_t n_flat[2], n_aug[2], n_aug_all;
   char* mem;
   bool bf16;
-  cudaDataType_t act_t;       // storage type of X, H1, H2, G, dL/d(head)
   size_t esz;                 // its size in bytes
   float *w, *g, *m, *v;       // augmented [policy | value]
   void* wb;                   // bf16 copy of w (bf16 mode)
@@ -59,7 +59,8 @@ struct auv_ppo {
   float *head_part, *norm_part;
   float *mb, *acc;            // statistics records (AUV_PPO_STATS floats)
   ppo::StepCtl* ctl;          // device: per-step variables
-  void* blas_ws;
+  float* gws;                 // GEMM workspace: split-K partials, tf32 transposes
+  size_t gws_bytes;
   // bf16 forward and backward-data on the tensor-core engine: packed images
   // of both networks (forward, and transposed for the backward), rebuilt
   // from w every step, a flat staging copy and a status block
@@ -86,7 +87,6 @@ struct auv_ppo {
 
 namespace {
 
-constexpr size_t kBlasWorkspace = 32u << 20;
 thread_local char g_err[256] = "";
 
 int fail(auv_ppo* p, int code, const char* fmt, ...) {
@@ -102,9 +102,6 @@ int cuda_fail(auv_ppo* p, cudaError_t e, const char* what) {
   return fail(p, AUV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-int blas_fail(auv_ppo* p, cublasStatus_t e, const char* what) {
-  return fail(p, AUV_ERR_CUDA, "%s: cuBLAS status %d", what, (int)e);
-}
 
 int round8(int x) { return (x + 7) & ~7; }
 
@@ -197,13 +194,29 @@ ppo::LossHp loss_hp(const auv_ppo* p) {
   return {c.clip_eps, c.vf_coef, c.ent_coef, c.logstd_min, c.logstd_max, (int)c.norm_adv};
 }
 
-// C = op(A) op(B) with A, B in the activation type; C in that type too
-// (c32 = false) or fp32 (c32 = true).
-cublasStatus_t gemm(auv_ppo* p, cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
-                    const void* A, int lda, const void* B, int ldb, void* C, int ldc, bool c32) {
-  const float one = 1.0f, zero = 0.0f;
-  return cublasGemmEx(p->blas, ta, tb, m, n, k, &one, A, p->act_t, lda, B, p->act_t, ldb, &zero, C,
-                      c32 ? CUDA_R_32F : p->act_t, ldc, p->ctype, CUBLAS_GEMM_DEFAULT);
+// C = op(A) op(B) in column-major terms (ta / tb: the operand is
+// transposed), A and B in the activation type, C in that type too (c32 =
+// false) or fp32 (c32 = true): the library's GEMM (k_gemm.cu) on the
+// row-major product C'[n][m] = sum_k opB(k, n) opA(m, k), whose first
+// operand is B (K-major unless transposed) and second A (K-major when
+// transposed).
+cudaError_t gemm(auv_ppo* p, bool ta, bool tb, int m, int n, int k, const void* A, int lda,
+                 const void* B, int ldb, void* C, int ldc, bool c32, cudaStream_t s) {
+  const auv::gemm::Operand a = {B, ldb, tb}, b = {A, lda, !ta};
+  return auv::gemm::launch(static_cast<auv::gemm::Prec>(p->cfg.precision), n, m, k, a, b, C, ldc,
+                           p->bf16 && !c32, 0.0f, p->gws, p->gws_bytes, p->st, s);
+}
+
+// Workspace of every product the learner runs (both networks).
+size_t gemm_workspace(const ppo::Dims& d, const int out[2]) {
+  size_t b = 0;
+  for (int k = 0; k < 2; ++k) {
+    const int o = out[k];
+    const int shapes[8][3] = {{d.B, d.H, d.Dp}, {d.B, d.H, d.Hp}, {d.B, o, d.Hp}, {o, d.Hp, d.B},
+                              {d.B, d.H, o},    {d.H, d.Hp, d.B}, {d.B, d.H, d.H}, {d.H, d.Dp, d.B}};
+    for (const auto& sh : shapes) b = std::max(b, auv::gemm::workspace_bytes(sh[0], sh[1], sh[2]));
+  }
+  return b;
 }
 
 size_t net_offset(const auv_ppo* p, int net) { return net ? p->n_aug[0] : 0; }
@@ -217,7 +230,7 @@ const char* weights_for_gemm(const auv_ppo* p, int net) {
 
 int ld_head(const auv_ppo* p, int net) { return net ? p->d.ld_val : p->d.ld_pol; }
 
-// Column-major view (cuBLAS): a sample-major [B][ld] array is an ld x B
+// Column-major view (the gemm() arguments): a sample-major [B][ld] array is an ld x B
 // matrix; a row-major weight [out][in_p] is an in_p x out matrix.
 //   Z1 = W1a^T X,  Z2 = W2a^T H1,  Y = W3a^T H2           (forward)
 //   gW3a = H2 gY^T, gH2 = W3 gY, gW2a = H1 gZ2^T, gH1 = W2 gZ2, gW1a = X gZ1^T
@@ -226,21 +239,20 @@ int forward(auv_ppo* p, int net, cudaStream_t s) {
   const size_t es = p->esz;
   const char* w = weights_for_gemm(p, net);
   const char *w1 = w, *w2 = w + (size_t)d.H * d.Dp * es, *w3 = w2 + (size_t)d.H * d.Hp * es;
-  cublasStatus_t bs;
   cudaError_t e;
-  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Dp, w1, d.Dp, p->X, d.Dp, p->h1[net],
-                 d.Hp, false)))
-    return blas_fail(p, bs, "forward layer 1");
+  if ((e = gemm(p, true, false, d.H, d.B, d.Dp, w1, d.Dp, p->X, d.Dp, p->h1[net],
+                 d.Hp, false, s)))
+    return cuda_fail(p, e, "forward layer 1");
   if ((e = ppo::launch_tanh_fwd(p->bf16, p->h1[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh 1");
-  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp,
-                 p->h2[net], d.Hp, false)))
-    return blas_fail(p, bs, "forward layer 2");
+  if ((e = gemm(p, true, false, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp,
+                 p->h2[net], d.Hp, false, s)))
+    return cuda_fail(p, e, "forward layer 2");
   if ((e = ppo::launch_tanh_fwd(p->bf16, p->h2[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh 2");
-  if ((bs = gemm(p, CUBLAS_OP_T, CUBLAS_OP_N, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Hp,
-                 p->y[net], ld_head(p, net), true)))
-    return blas_fail(p, bs, "forward layer 3");
+  if ((e = gemm(p, true, false, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Hp,
+                 p->y[net], ld_head(p, net), true, s)))
+    return cuda_fail(p, e, "forward layer 3");
   return AUV_OK;
 }
 
@@ -254,11 +266,10 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
   float *g1 = g, *g2 = g + (size_t)d.H * d.Dp, *g3 = g2 + (size_t)d.H * d.Hp;
   void* gz2 = p->gb[net];
   void* gz1 = p->h2[net];       // H2 is dead once gZ2 exists
-  cublasStatus_t bs;
   cudaError_t e;
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, out, d.B, p->h2[net], d.Hp, gy, ldy, g3, d.Hp,
-                 true)))
-    return blas_fail(p, bs, "gradient W3");
+  if ((e = gemm(p, false, true, d.Hp, out, d.B, p->h2[net], d.Hp, gy, ldy, g3, d.Hp,
+                 true, s)))
+    return cuda_fail(p, e, "gradient W3");
   if (p->eng) {
     // gZ2 and gZ1 (into the dead H2) on the tensor-core engine, then the
     // weight gradients of layers 2 and 1
@@ -267,28 +278,28 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
              static_cast<const uint16_t*>(p->h2[net]), static_cast<const uint16_t*>(p->h1[net]), d.Hp,
              static_cast<uint16_t*>(gz2), d.H, static_cast<uint16_t*>(gz1), d.Hp, p->st, s)))
       return cuda_fail(p, e, "engine backward");
-    if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
-                   true)))
-      return blas_fail(p, bs, "gradient W2");
-    if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
-                   true)))
-      return blas_fail(p, bs, "gradient W1");
+    if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+                   true, s)))
+      return cuda_fail(p, e, "gradient W2");
+    if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+                   true, s)))
+      return cuda_fail(p, e, "gradient W1");
     return AUV_OK;
   }
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, out, w3, d.Hp, gy, ldy, gz2, d.H, false)))
-    return blas_fail(p, bs, "gradient H2");
+  if ((e = gemm(p, false, false, d.H, d.B, out, w3, d.Hp, gy, ldy, gz2, d.H, false, s)))
+    return cuda_fail(p, e, "gradient H2");
   if ((e = ppo::launch_tanh_bwd(p->bf16, gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 2");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
-                 true)))
-    return blas_fail(p, bs, "gradient W2");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_N, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp, false)))
-    return blas_fail(p, bs, "gradient H1");
+  if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+                 true, s)))
+    return cuda_fail(p, e, "gradient W2");
+  if ((e = gemm(p, false, false, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp, false, s)))
+    return cuda_fail(p, e, "gradient H1");
   if ((e = ppo::launch_tanh_bwd(p->bf16, gz1, d.Hp, p->h1[net], d.Hp, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 1");
-  if ((bs = gemm(p, CUBLAS_OP_N, CUBLAS_OP_T, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
-                 true)))
-    return blas_fail(p, bs, "gradient W1");
+  if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+                 true, s)))
+    return cuda_fail(p, e, "gradient W1");
   return AUV_OK;
 }
 
@@ -378,7 +389,6 @@ bool capture_step(auv_ppo* p, const auv_ppo_batch* b) {
        cudaEventCreateWithFlags(&p->ev_in, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&p->ev_out, cudaEventDisableTiming) != cudaSuccess))
     return false;
-  if (cublasSetStream(p->blas, p->gstream) != CUBLAS_STATUS_SUCCESS) return false;
   if (cudaStreamBeginCapture(p->gstream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
     return false;
   const bool ok = grads_impl(p, b, p->acc, p->gstream) == AUV_OK &&
@@ -462,7 +472,6 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   d.bf16 = cfg->precision == AUV_PPO_BF16;
   d.value_only = (cfg->flags & AUV_PPO_VALUE_ONLY) ? 1 : 0;
   p->bf16 = d.bf16 != 0;
-  p->act_t = p->bf16 ? CUDA_R_16BF : CUDA_R_32F;
   p->esz = p->bf16 ? 2 : 4;
   p->out[0] = 2 * d.A;
   p->out[1] = 1;
@@ -474,7 +483,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   p->n_aug_all = p->n_aug[0] + p->n_aug[1];
   // the engine's networks: hidden 256, input <= 18, head <= 16 (2A <= 16)
   p->eng = p->bf16 && d.H == 256 && d.D <= auv::kObs && !(cfg->flags & AUV_PPO_GEMM_PATH);
-  p->ctype = cfg->precision == AUV_PPO_TF32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
+  const size_t gws_bytes = gemm_workspace(d, p->out);
   // one allocation, 256-byte aligned pieces
   const size_t B = (size_t)d.B, nb = (B + 255) / 256;
   size_t off = 0;
@@ -493,7 +502,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_gv = take(B * d.ld_val * es), o_hp = take(nb * 5 * 4),
                o_np = take(ppo::kNormBlocks * 4), o_mb = take(AUV_PPO_STATS * 4),
                o_acc = take(AUV_PPO_STATS * 4), o_ctl = take(sizeof(ppo::StepCtl)),
-               o_ws = take(kBlasWorkspace),
+               o_ws = take(gws_bytes),
                o_ip = take(p->eng ? auv::bf16_policy_image_bytes() : 0),
                o_iv = take(p->eng ? auv::bf16_value_image_bytes() : 0),
                o_ibp = take(p->eng ? auv::bf16_back_image_bytes() : 0),
@@ -532,7 +541,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   p->mb = reinterpret_cast<float*>(base + o_mb);
   p->acc = reinterpret_cast<float*>(base + o_acc);
   p->ctl = reinterpret_cast<ppo::StepCtl*>(base + o_ctl);
-  p->blas_ws = base + o_ws;
+  p->gws = reinterpret_cast<float*>(base + o_ws);
+  p->gws_bytes = gws_bytes;
   if (p->eng) {
     p->img_p = base + o_ip;
     p->img_v = base + o_iv;
@@ -562,15 +572,6 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     delete p;
     return cuda_fail(nullptr, e, "initialise learner memory");
   }
-  cublasStatus_t bs = cublasCreate(&p->blas);
-  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetWorkspace(p->blas, p->blas_ws, kBlasWorkspace);
-  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetMathMode(p->blas, CUBLAS_DEFAULT_MATH);
-  if (bs != CUBLAS_STATUS_SUCCESS) {
-    if (p->blas) cublasDestroy(p->blas);
-    cudaFree(p->mem);
-    delete p;
-    return blas_fail(nullptr, bs, "cuBLAS handle");
-  }
   *out = p;
   return AUV_OK;
 }
@@ -585,7 +586,6 @@ int ppo_destroy(auv_ppo* p) {
   if (p->ev_in) cudaEventDestroy(p->ev_in);
   if (p->ev_out) cudaEventDestroy(p->ev_out);
   if (p->gstream) cudaStreamDestroy(p->gstream);
-  cublasDestroy(p->blas);
   if (p->sm_buf) cudaFree(p->sm_buf);
   cudaFree(p->mem);
   if (prev >= 0) cudaSetDevice(prev);
@@ -670,8 +670,6 @@ int ppo_grads(auv_ppo* p, const auv_ppo_batch* batch, uint64_t epoch, uint32_t m
   if (grad && (rc = check_dev(p, grad, "grad"))) return rc;
   if (stats && (rc = check_dev(p, stats, "stats"))) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cublasStatus_t bs = cublasSetStream(p->blas, s);
-  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
   if ((rc = set_ctl(p, epoch, 1u << 31, minibatch, p->t, s))) return rc;
   if ((rc = grads_impl(p, batch, nullptr, s))) return rc;
   if (grad && (rc = convert(p, grad, grad + p->n_flat[0], p->g, false, s))) return rc;
@@ -775,9 +773,6 @@ int ppo_update(auv_ppo* p, const auv_ppo_batch* batch, uint32_t epochs, uint32_t
     if ((e = cudaEventRecord(p->ev_in, s)) || (e = cudaStreamWaitEvent(p->gstream, p->ev_in, 0)))
       return cuda_fail(p, e, "order update after caller");
     r = p->gstream;
-  } else {
-    cublasStatus_t bs = cublasSetStream(p->blas, s);
-    if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(p, bs, "cublasSetStream");
   }
   if ((rc = set_ctl(p, p->epoch, n_minibatches, 0, p->t, r))) return rc;
   if ((e = cudaMemsetAsync(p->acc, 0, AUV_PPO_STATS * 4, r)))

@@ -8,18 +8,19 @@
 //
 // Per step the per-env work (observation, action, physics and their VJPs)
 // runs in the k_shac_* kernels of k_adjoint.cu; the policy network's dense
-// products run in cuBLAS (fp32 compute) on the augmented layout of the PPO
-// learner (a constant-1 input column carries each bias).  Forward: for each
+// products run in the library's GEMM (k_gemm.cu: tcgen05 with tf32 operands,
+// or fp32 on the CUDA cores) on the augmented layout of the PPO learner (a
+// constant-1 input column carries each bias).  Forward: for each
 // step, observation -> policy GEMMs (activations kept for every step) ->
 // action and physics (the env advances).  Backward, t = T-1 .. 0: physics
 // VJP of step t (the state adjoint lam and the head gradient), the policy's
 // backward (weight gradients accumulated over steps, input gradient), then
 // the observation VJP into lam.  The terminal critic seeds lam with
 // coef_V dV(o(x_T))/dx_T through the value network's input gradient.
-#include <cublas_v2.h>
-
+#include <algorithm>
 #include <cstdio>
 
+#include "auv_gemm.h"
 #include "auv_kernels.h"
 #include "auvenv.h"
 #include "paper_device.cuh"
@@ -31,15 +32,20 @@ namespace {
 
 int round8(int x) { return (x + 7) & ~7; }
 
+// C = op(A) op(B) (+ beta C) in column-major terms (ta / tb: the operand is
+// transposed), fp32 operands and result: the row-major product
+// C'[n][m] = sum_k opB(k, n) opA(m, k) on the library's GEMM.
 struct Gemm {
-  cublasHandle_t h;
-  cublasComputeType_t ct;
-  cublasStatus_t operator()(cublasOperation_t ta, cublasOperation_t tb, int m, int n, int k,
-                            const float* A, int lda, const float* B, int ldb, float* C, int ldc,
-                            float beta = 0.0f) const {
-    const float one = 1.0f;
-    return cublasGemmEx(h, ta, tb, m, n, k, &one, A, CUDA_R_32F, lda, B, CUDA_R_32F, ldb, &beta,
-                        C, CUDA_R_32F, ldc, ct, CUBLAS_GEMM_DEFAULT);
+  bool tf32;
+  float* ws;
+  size_t ws_bytes;
+  Status* st;
+  cudaStream_t s;
+  cudaError_t operator()(bool ta, bool tb, int m, int n, int k, const float* A, int lda,
+                         const float* B, int ldb, float* C, int ldc, float beta = 0.0f) const {
+    const gemm::Operand a = {B, ldb, tb}, b = {A, lda, !ta};
+    return gemm::launch(tf32 ? gemm::kTf32 : gemm::kFp32, n, m, k, a, b, C, ldc, false, beta, ws,
+                        ws_bytes, st, s);
   }
 };
 
@@ -85,6 +91,15 @@ Layout layout(int n, int T, int H, bool paper) {
   L.o_wv = take(L.n_aug_v * 4);
   L.o_gp = take(L.n_aug_p * 4);
   L.o_sc = take(adjoint_scratch_floats(n, T) * 4);
+  // the GEMM workspace of the largest product (policy and value networks)
+  size_t gws = 0;
+  for (int o : {L.out, 1}) {
+    const int shapes[9][3] = {{n, H, L.Dp}, {n, H, L.Hp}, {n, o, L.Hp},   {o, L.Hp, n},    {n, H, o},
+                              {H, L.Hp, n}, {n, H, H},    {H, L.Dp, n}, {n, L.Dp, H}};
+    for (const auto& sh : shapes) gws = std::max(gws, gemm::workspace_bytes(sh[0], sh[1], sh[2]));
+  }
+  L.o_gws = take(gws);
+  L.gws_bytes = gws;
   L.bytes = off;
   return L;
 }
@@ -103,7 +118,7 @@ cudaError_t init(const Layout& L, char* base, cudaStream_t s) {
   return e;
 }
 
-int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const Layout& L,
+int run_window(const Model& M, const Buffers& B, Status* st, const Layout& L,
                char* base, uint64_t t_g0, const float* policy, const float* value,
                const float* coef, float coef_V, bool tf32, float* grad, float* J,
                float* obs_out, float* rew_out, uint8_t* done_out, cudaStream_t s, char* err) {
@@ -124,20 +139,13 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   float *g1 = gp, *g2 = gp + (size_t)H * Dp, *g3 = g2 + (size_t)H * Hp;
   const float *v1 = wv, *v2 = wv + (size_t)H * Dp, *v3 = v2 + (size_t)H * Hp;
 
-  cublasHandle_t h = static_cast<cublasHandle_t>(blas);
-  Gemm gemm{h, tf32 ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F};
-  cublasStatus_t bs = cublasSetStream(h, s);
+  const Gemm gemm{tf32, F(L.o_gws), L.gws_bytes, st, s};
   cudaError_t e = cudaSuccess;
   auto cfail = [&](cudaError_t x, const char* what) {
     snprintf(err, 256, "%s: %s", what, cudaGetErrorString(x));
     return AUV_ERR_CUDA;
   };
-  auto bfail = [&](cublasStatus_t x, const char* what) {
-    snprintf(err, 256, "%s: cuBLAS status %d", what, (int)x);
-    return AUV_ERR_CUDA;
-  };
-  if (bs) return bfail(bs, "cublasSetStream");
-  const auto T_ = CUBLAS_OP_T, N_ = CUBLAS_OP_N;
+  const bool T_ = true, N_ = false;
 
   // weights into the augmented layout; gradient accumulator to zero
   const int D = L.D, out = L.out;
@@ -151,12 +159,12 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   // ---- forward ----
   for (int t = 0; t < T; ++t) {
     if ((e = launch_obs(M, B, SCs(t), Xs(t), Dp, obs_out, t, s))) return cfail(e, "observation");
-    if ((bs = gemm(T_, N_, H, n, Dp, w1, Dp, Xs(t), Dp, H1s(t), Hp))) return bfail(bs, "policy 1");
+    if ((e = gemm(T_, N_, H, n, Dp, w1, Dp, Xs(t), Dp, H1s(t), Hp))) return cfail(e, "policy 1");
     if ((e = ppo::launch_tanh_fwd(false, H1s(t), Hp, n, H, s))) return cfail(e, "tanh");
-    if ((bs = gemm(T_, N_, H, n, Hp, w2, Hp, H1s(t), Hp, H2s(t), Hp))) return bfail(bs, "policy 2");
+    if ((e = gemm(T_, N_, H, n, Hp, w2, Hp, H1s(t), Hp, H2s(t), Hp))) return cfail(e, "policy 2");
     if ((e = ppo::launch_tanh_fwd(false, H2s(t), Hp, n, H, s))) return cfail(e, "tanh");
-    if ((bs = gemm(T_, N_, out, n, Hp, w3, Hp, H2s(t), Hp, Ys(t), kLdy)))
-      return bfail(bs, "policy 3");
+    if ((e = gemm(T_, N_, out, n, Hp, w3, Hp, H2s(t), Hp, Ys(t), kLdy)))
+      return cfail(e, "policy 3");
     if ((e = launch_step(M, B, Ys(t), kLdy, t_g0 + (uint64_t)t, rew + (size_t)t * N,
                          done + (size_t)t * N, st, s)))
       return cfail(e, "step");
@@ -165,17 +173,17 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
   // ---- terminal critic: lam = coef_V dV(o(x_T))/dx_T ----
   if (value) {
     if ((e = launch_obs(M, B, nullptr, Xs(T), Dp, nullptr, 0, s))) return cfail(e, "observation");
-    if ((bs = gemm(T_, N_, H, n, Dp, v1, Dp, Xs(T), Dp, VH1, Hp))) return bfail(bs, "value 1");
+    if ((e = gemm(T_, N_, H, n, Dp, v1, Dp, Xs(T), Dp, VH1, Hp))) return cfail(e, "value 1");
     if ((e = ppo::launch_tanh_fwd(false, VH1, Hp, n, H, s))) return cfail(e, "tanh");
-    if ((bs = gemm(T_, N_, H, n, Hp, v2, Hp, VH1, Hp, VH2, Hp))) return bfail(bs, "value 2");
+    if ((e = gemm(T_, N_, H, n, Hp, v2, Hp, VH1, Hp, VH2, Hp))) return cfail(e, "value 2");
     if ((e = ppo::launch_tanh_fwd(false, VH2, Hp, n, H, s))) return cfail(e, "tanh");
-    if ((bs = gemm(T_, N_, 1, n, Hp, v3, Hp, VH2, Hp, V, kLdv))) return bfail(bs, "value 3");
+    if ((e = gemm(T_, N_, 1, n, Hp, v3, Hp, VH2, Hp, V, kLdv))) return cfail(e, "value 3");
     if ((e = launch_fill_col(n, gYv, kLdv, coef_V, s))) return cfail(e, "critic seed");
-    if ((bs = gemm(N_, N_, H, n, 1, v3, Hp, gYv, kLdv, G, H))) return bfail(bs, "value dH2");
+    if ((e = gemm(N_, N_, H, n, 1, v3, Hp, gYv, kLdv, G, H))) return cfail(e, "value dH2");
     if ((e = ppo::launch_tanh_bwd(false, G, H, VH2, Hp, n, H, s))) return cfail(e, "tanh'");
-    if ((bs = gemm(N_, N_, H, n, H, v2, Hp, G, H, VH2, Hp))) return bfail(bs, "value dH1");
+    if ((e = gemm(N_, N_, H, n, H, v2, Hp, G, H, VH2, Hp))) return cfail(e, "value dH1");
     if ((e = ppo::launch_tanh_bwd(false, VH2, Hp, VH1, Hp, n, H, s))) return cfail(e, "tanh'");
-    if ((bs = gemm(N_, N_, Dp, n, H, v1, Dp, VH2, Hp, GX, Dp))) return bfail(bs, "value dX");
+    if ((e = gemm(N_, N_, Dp, n, H, v1, Dp, VH2, Hp, GX, Dp))) return cfail(e, "value dX");
     if ((e = launch_obs_vjp(M, B, nullptr, GX, Dp, lam, s))) return cfail(e, "observation VJP");
   }
   if (J && (e = launch_objective(n, T, rew, coef, value ? V : nullptr, kLdv, coef_V, J, s)))
@@ -185,16 +193,16 @@ int run_window(void* blas, const Model& M, const Buffers& B, Status* st, const L
     if ((e = launch_bwd(M, SCs(t), Ys(t), kLdy, done + (size_t)t * N, t_g0 + (uint64_t)t,
                         coef + t, lam, gY, s)))
       return cfail(e, "step VJP");
-    if ((bs = gemm(N_, T_, Hp, out, n, H2s(t), Hp, gY, kLdy, g3, Hp, 1.0f)))
-      return bfail(bs, "dW3");
-    if ((bs = gemm(N_, N_, H, n, out, w3, Hp, gY, kLdy, G, H))) return bfail(bs, "dH2");
+    if ((e = gemm(N_, T_, Hp, out, n, H2s(t), Hp, gY, kLdy, g3, Hp, 1.0f)))
+      return cfail(e, "dW3");
+    if ((e = gemm(N_, N_, H, n, out, w3, Hp, gY, kLdy, G, H))) return cfail(e, "dH2");
     if ((e = ppo::launch_tanh_bwd(false, G, H, H2s(t), Hp, n, H, s))) return cfail(e, "tanh'");
-    if ((bs = gemm(N_, T_, Hp, H, n, H1s(t), Hp, G, H, g2, Hp, 1.0f))) return bfail(bs, "dW2");
-    if ((bs = gemm(N_, N_, H, n, H, w2, Hp, G, H, H2s(t), Hp))) return bfail(bs, "dH1");
+    if ((e = gemm(N_, T_, Hp, H, n, H1s(t), Hp, G, H, g2, Hp, 1.0f))) return cfail(e, "dW2");
+    if ((e = gemm(N_, N_, H, n, H, w2, Hp, G, H, H2s(t), Hp))) return cfail(e, "dH1");
     if ((e = ppo::launch_tanh_bwd(false, H2s(t), Hp, H1s(t), Hp, n, H, s)))
       return cfail(e, "tanh'");
-    if ((bs = gemm(N_, T_, Dp, H, n, Xs(t), Dp, H2s(t), Hp, g1, Dp, 1.0f))) return bfail(bs, "dW1");
-    if ((bs = gemm(N_, N_, Dp, n, H, w1, Dp, H2s(t), Hp, GX, Dp))) return bfail(bs, "dX");
+    if ((e = gemm(N_, T_, Dp, H, n, Xs(t), Dp, H2s(t), Hp, g1, Dp, 1.0f))) return cfail(e, "dW1");
+    if ((e = gemm(N_, N_, Dp, n, H, w1, Dp, H2s(t), Hp, GX, Dp))) return cfail(e, "dX");
     if ((e = launch_obs_vjp(M, B, SCs(t), GX, Dp, lam, s))) return cfail(e, "observation VJP");
   }
   if ((e = ppo::launch_convert(grad, gp, D, Dp, H, Hp, out, false, s)))
