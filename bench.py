@@ -45,10 +45,12 @@ def parse():
     ap.add_argument("--workload", default="ppo_65536")
     ap.add_argument("--n-envs", type=int, default=None)
     ap.add_argument("--rollout-steps", type=int, default=None)
-    ap.add_argument("--mlp", default=None, choices=[None, "fp32", "bf16"])
+    ap.add_argument("--mlp", default=None, choices=[None, "fp32", "bf16", "tf32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the fp32 workloads' rollouts of the default line")
     ap.add_argument("--no-replay", action="store_true",
                     help="skip the physics-only measurement of the default line")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -326,6 +328,70 @@ def measure_replay(w, steps, warmup, clocks_on=True, device=0):
     achieved = n * T * dyn_flops_per_env_step(w) / (step_ms * 1e-3) / 1e12
     src = f"FP32 pipe 2*128*{n_sm} SMs*{sm_mhz:.0f} MHz (derived)"
     return step_ms, n * T, achieved, fp32_peak, src, clock_info
+
+
+# The fp32 workloads (BASELINE's first three): 64 envs x 200 steps with the
+# 18-64-64-8 network on CUDA cores (hidden 64 is far below a tensor-core
+# tile), and 4,096 / 16,384 envs x 1,000 steps with the 18-256-256-8 network
+# on the tensor cores in tf32 (kind::tf32); trajectories of rewards and dones.
+CONFIG_LINES = (("tiny_64", "fp32"), ("fp32_4096", "tf32"), ("dr_16384", "tf32"))
+
+
+def dyn_flops(w):
+    """Physics flops per env-step for the workload's substep count (the
+    counts behind DYN_FLOPS_PER_ENV_STEP)."""
+    if W.is_paper(w):
+        return PAPER_DYN_FLOPS_PER_ENV_STEP
+    return 141 + 144 + 378 * int(w["substeps"]) + 93 + 72
+
+
+def measure_config(name, mlp, reps, device=0):
+    """Time whole rollouts of one fp32 workload (T = its step count, rewards
+    and dones written), L2 flushed before each; returns a result dict."""
+    import torch
+    from paper_2512_13359_gb300 import auvenv
+    w = W.workload(name, mlp=mlp)
+    n, T = int(w["n_envs"]), int(w["steps"])
+    env = auvenv.Env(w)
+    env.set_weights(W.policy_weights(w))
+    env.reset()
+    traj = env.alloc_traj(T, keys=("rew", "done"))
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    env.rollout(T, traj)
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(reps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        env.rollout(T, traj)
+        e1.record(stream)
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    if env.status().code != 0:
+        raise RuntimeError(f"device status after the {name} rollouts")
+    env.close()
+    t_ms = sum(a.elapsed_time(b) for a, b in ms) / len(ms)
+    rate = n * T / (t_ms * 1e-3)
+    peaks, src = load_peaks()
+    pol = mlp_flops(W.obs_dim(w), w["hidden"], w["policy_out"])
+    if mlp == "tf32":
+        peak = peaks["bf16_tflops"] * 1.1 / 2.25
+        roof = {"bound": "tensor", "kernel": "k_rollout_tf32", "achieved": rate * pol / 1e12,
+                "peak": peak, "unit": "TFLOP/s", "frac": rate * pol / 1e12 / peak,
+                "peak_source": f"bf16 burst, {src}, x tf32/bf16 nominal 1.1/2.25"}
+    else:
+        n_sm = torch.cuda.get_device_properties(device).multi_processor_count
+        peak = 2 * 128 * n_sm * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = rate * (pol + dyn_flops(w)) / 1e12
+        roof = {"bound": "alu", "kernel": "k_rollout_fp32", "achieved": ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": ach / peak,
+                "peak_source": f"FP32 pipe 2*128*{n_sm} SMs*max clock (derived)"}
+    return {"workload": name, "mlp": mlp, "n_envs": n, "steps": T, "substeps": w["substeps"],
+            "value": rate, "unit": "env-steps/s", "ms_per_rollout": t_ms, "reps": reps,
+            "flops_per_env_step": pol + dyn_flops(w), "roofline": roof,
+            "trajectory": ["rew", "done"], "l2": "flushed before each rollout"}
 
 
 def run_replay(args):
@@ -856,7 +922,7 @@ def main():
         for n in W.SWEEP_SIZES:
             a = argparse.Namespace(**vars(args))
             a.workload, a.n_envs, a.rollout_steps, a.sweep = "sweep", n, None, False
-            a.no_e2e, a.no_cpu_baseline, a.no_replay = True, True, True
+            a.no_e2e, a.no_cpu_baseline, a.no_replay, a.no_configs = True, True, True, True
             a.steps = max(3, min(base_steps, int(2e8 // (n * 256)) + 3))
             run(a)
         return
@@ -1001,6 +1067,12 @@ def run(args):
                 "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
                 "traffic": rollout_traffic(w, n, T) if kern == "rollout_bf16" else None,
                 "peak_source": f"bf16 burst, {peak_src}"}
+    elif w["mlp"] == "tf32":
+        peak = peaks["bf16_tflops"] * 1.1 / 2.25
+        achieved = n * T * pol_fl / (roll_avg * 1e-3) / 1e12
+        roof = {"bound": "tensor", "kernel": "rollout_tf32", "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "peak_source": f"bf16 burst, {peak_src}, x tf32/bf16 nominal 1.1/2.25"}
     else:
         kern, dur = "rollout_fp32", roll_avg
         flops = n * T * (pol_fl + val_fl + dyn_flops_per_env_step(w))
@@ -1043,12 +1115,17 @@ def run(args):
                    "frac": r_ach / r_peak, "flops_per_env_step": dyn_flops_per_env_step(w),
                    "peak_source": r_src, "sm_mhz": (r_clk or {}).get("sm_mhz")}
 
+    # the fp32 workloads (one whole rollout each, timed after the timed region)
+    configs = None
+    if not args.no_configs and world == 1:
+        configs = [measure_config(nm, mlp, 3, local) for nm, mlp in CONFIG_LINES]
+
     launches_per_step = 1 + (1 if value is not None else 0)
     line = {
         "metric": "env-steps/s (physics+policy+reward)", "value": value_rate,
         "unit": "env-steps/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16" if w["mlp"] == "bf16" else "f32",
+        "vs_baseline": None, "dtype": {"bf16": "bf16", "tf32": "tf32"}.get(w["mlp"], "f32"),
         "data": "synthetic",
         "config": {"workload": w["name"], "n_envs_per_gpu": n, "rollout_steps": T,
                    "substeps": w["substeps"], "mlp": w["mlp"], "hidden": w["hidden"],
@@ -1056,6 +1133,7 @@ def run(args):
                    "l2": "flushed between timed steps (2 x L2 buffer written)",
                    "rollout_ms": roll_avg, "value_ms": val_avg},
         "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "physics_only": physics,
+        "fp32_workloads": configs,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clock_info,
     }

@@ -66,6 +66,11 @@ extern "C" {
 /* network arithmetic */
 #define AUV_MLP_FP32 0   /* fp32 operands and accumulation on CUDA cores        */
 #define AUV_MLP_BF16 1   /* bf16 weights/activations, fp32 accumulation, tcgen05 */
+#define AUV_MLP_TF32 2   /* fp32 networks with tf32 operands (rounded to nearest),
+                            fp32 accumulation, tcgen05 kind::tf32: Fossen model,
+                            hidden 256, policy_out 8 or 16, no value network;
+                            env_rollout only (env_value and env_policy_forward
+                            return AUV_ERR_UNSUPPORTED) */
 
 /* environment models */
 #define AUV_MODEL_FOSSEN 0
@@ -127,7 +132,7 @@ typedef struct auv_config {
   float dr_cob_range;     /* r_b ~ U[-r, r] per axis [m]                     */
   uint32_t hidden;        /* hidden width H of both networks                 */
   uint32_t policy_out;    /* 8: mean only (fixed log-std); 16: mean + log-std */
-  uint32_t mlp_mode;      /* AUV_MLP_FP32 or AUV_MLP_BF16                    */
+  uint32_t mlp_mode;      /* AUV_MLP_FP32, AUV_MLP_BF16 or AUV_MLP_TF32      */
   uint32_t has_value;     /* 1: value network present                        */
   float logstd_fixed[8];  /* log-std used when policy_out == 8               */
   float logstd_min, logstd_max;     /* clamp of the log-std head             */

@@ -25,6 +25,7 @@ AUV_ERR_NAN = -5
 AUV_ERR_UNSUPPORTED = -6
 AUV_MLP_FP32 = 0
 AUV_MLP_BF16 = 1
+AUV_MLP_TF32 = 2
 AUV_MODEL_FOSSEN = 0
 AUV_MODEL_PAPER = 1
 AUV_PPO_FP32 = 0
@@ -235,7 +236,7 @@ def make_config(w: dict) -> AuvConfig:
         setattr(c, k, float(w[k]))
     c.hidden = int(w["hidden"])
     c.policy_out = int(w["policy_out"])
-    c.mlp_mode = AUV_MLP_BF16 if w["mlp"] == "bf16" else AUV_MLP_FP32
+    c.mlp_mode = {"bf16": AUV_MLP_BF16, "tf32": AUV_MLP_TF32}.get(w["mlp"], AUV_MLP_FP32)
     c.has_value = int(w["has_value"])
     ls = [float(x) for x in w["logstd_fixed"]]
     c.logstd_fixed[:] = ls + [0.0] * (8 - len(ls))

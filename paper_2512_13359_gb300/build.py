@@ -16,7 +16,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libauvenv.so")
 SOURCES = ["api.cu", "ppo_api.cu", "rbuf.cu", "shac.cu", "k_env.cu", "k_paper.cu", "k_ppo.cu",
-           "k_adjoint.cu", "k_bf16.cu", "k_gemm.cu", "noalloc.cu", "probes.cu"]
+           "k_adjoint.cu", "k_bf16.cu", "k_gemm.cu", "k_tf32.cu", "noalloc.cu", "probes.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I", CSRC, "-I", INCLUDE]

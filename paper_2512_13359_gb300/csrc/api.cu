@@ -128,7 +128,7 @@ int map_output(auv_env* env, void* p, const char* name, size_t align, void** dev
 int validate_networks(const auv_config* c, uint32_t out_mean) {
   if (c->policy_out != out_mean && c->policy_out != 2 * out_mean)
     return fail(nullptr, AUV_ERR_INVALID, "policy_out must be %u or %u", out_mean, 2 * out_mean);
-  if (c->mlp_mode != AUV_MLP_FP32 && c->mlp_mode != AUV_MLP_BF16)
+  if (c->mlp_mode != AUV_MLP_FP32 && c->mlp_mode != AUV_MLP_BF16 && c->mlp_mode != AUV_MLP_TF32)
     return fail(nullptr, AUV_ERR_INVALID, "unknown mlp_mode %u", c->mlp_mode);
   if (c->has_value > 1) return fail(nullptr, AUV_ERR_INVALID, "has_value must be 0 or 1");
   if (!(c->logstd_min <= c->logstd_max) || !std::isfinite(c->logstd_min) ||
@@ -139,6 +139,10 @@ int validate_networks(const auv_config* c, uint32_t out_mean) {
       return fail(nullptr, AUV_ERR_INVALID, "logstd_fixed not finite");
   if (c->mlp_mode == AUV_MLP_FP32 && c->hidden != 64 && c->hidden != 256)
     return fail(nullptr, AUV_ERR_UNSUPPORTED, "fp32 networks are built for hidden 64 or 256");
+  if (c->mlp_mode == AUV_MLP_TF32 &&
+      (c->model != AUV_MODEL_FOSSEN || c->hidden != 256 || c->has_value))
+    return fail(nullptr, AUV_ERR_UNSUPPORTED,
+                "tf32 networks are built for the Fossen model, hidden 256, no value network");
   if (c->mlp_mode == AUV_MLP_BF16 && (c->hidden != 256 || c->policy_out != 2 * out_mean))
     return fail(nullptr, AUV_ERR_UNSUPPORTED,
                 "bf16 networks are built for hidden 256 with the mean + log-std head");
@@ -396,6 +400,9 @@ int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
     off += ((auv::bf16_policy_image_bytes() + 1023) / 1024) * 1024;
     val_pk_off = off;
     off += ((auv::bf16_value_image_bytes() + 1023) / 1024) * 1024;
+  } else if (cfg->mlp_mode == AUV_MLP_TF32) {
+    pol_pk_off = off;
+    off += ((auv::tf32_policy_image_bytes() + 1023) / 1024) * 1024;
   }
   cudaError_t e = cudaMalloc(&env->workspace, off);
   if (e != cudaSuccess) {
@@ -408,6 +415,8 @@ int env_create(const auv_config* cfg, const auv_buffers* buf, auv_env** out) {
   if (cfg->mlp_mode == AUV_MLP_BF16) {
     env->w_policy_packed = env->workspace + pol_pk_off;
     env->w_value_packed = env->workspace + val_pk_off;
+  } else if (cfg->mlp_mode == AUV_MLP_TF32) {
+    env->w_policy_packed = env->workspace + pol_pk_off;
   }
   Status s0 = {0, 0, INT_MAX, 0};
   e = cudaMemcpy(env->status, &s0, sizeof(s0), cudaMemcpyHostToDevice);
@@ -456,6 +465,9 @@ int env_set_weights(auv_env* env, const float* policy, const float* value, void*
     e = auv::launch_pack_bf16(env->model, env->w_policy_f32, env->w_value_f32,
                               env->w_policy_packed, env->w_value_packed, s);
     if (e != cudaSuccess) return cuda_fail(env, e, "pack bf16 weights");
+  } else if (env->cfg.mlp_mode == AUV_MLP_TF32) {
+    e = auv::launch_pack_tf32(env->model, env->w_policy_f32, env->w_policy_packed, s);
+    if (e != cudaSuccess) return cuda_fail(env, e, "pack tf32 weights");
   }
   // host sources are read before return
   void* d = nullptr;
@@ -490,6 +502,9 @@ cudaError_t launch_rollout_any(auv_env* env, const Traj& tr, int T, uint64_t t_g
                                                 env->w_value_f32, tr, T, t_g0, env->status, s)
                : auv::launch_rollout_fp32(env->model, env->buf, env->w_policy_f32,
                                           env->w_value_f32, tr, T, t_g0, env->status, s);
+  if (env->cfg.mlp_mode == AUV_MLP_TF32)
+    return auv::launch_rollout_tf32(env->model, env->buf, env->w_policy_packed, tr, T, t_g0,
+                                    env->status, s);
   cudaError_t e = auv::launch_rollout_bf16(env->model, env->buf, env->w_policy_packed, tr, T,
                                            t_g0, env->status, s);
   if (e != cudaSuccess || !tr.value) return e;
@@ -643,6 +658,8 @@ int env_value(auv_env* env, const float* obs, int T, float* value, void* stream)
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t rows = (size_t)T * env->model.n;
   cudaError_t e;
+  if (env->cfg.mlp_mode == AUV_MLP_TF32)
+    return fail(env, AUV_ERR_UNSUPPORTED, "tf32 mode has no value network");
   if (env->cfg.mlp_mode == AUV_MLP_FP32)
     e = auv::launch_value_fp32(env->model, env->w_value_f32, static_cast<const float*>(o), rows,
                                env->model.n, static_cast<float*>(v), s);
@@ -857,6 +874,8 @@ int env_policy_forward(auv_env* env, const float* obs, int n, float* head, float
   if (value && (rc = check_device_buffer(env, value, "value", 4))) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
+  if (env->cfg.mlp_mode == AUV_MLP_TF32)
+    return fail(env, AUV_ERR_UNSUPPORTED, "tf32 mode evaluates the policy inside env_rollout only");
   if (env->cfg.mlp_mode == AUV_MLP_FP32)
     e = auv::launch_forward_fp32(env->model, env->w_policy_f32, env->w_value_f32, obs, n, head,
                                  value, s);

@@ -46,6 +46,13 @@ cudaError_t launch_learn_backward_bf16(const void* packed, int out_dim, const ui
                                        cudaStream_t s);
 
 // Fused rollout with the policy network on tcgen05.
+// tf32 tensor-core rollout (k_tf32.cu): Fossen model, hidden 256, policy head
+// 8 or 16, no value network; packed image from the fp32 policy weights.
+size_t tf32_policy_image_bytes();
+cudaError_t launch_pack_tf32(const Model& M, const float* wp_f32, void* packed, cudaStream_t s);
+cudaError_t launch_rollout_tf32(const Model& M, const Buffers& B, const void* packed,
+                                const Traj& tr, int T, uint64_t t_g0, Status* st, cudaStream_t s);
+
 cudaError_t launch_rollout_bf16(const Model& M, const Buffers& B, const void* wp_packed,
                                 const Traj& tr, int T, uint64_t t_g0, Status* st, cudaStream_t s);
 

@@ -60,14 +60,17 @@ def sample_ids(n, k=40, seed=5):
     return ids.astype(np.int64)
 
 
-def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None, resync=None):
+def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None, resync=None,
+                         net_tol=BF16_TOL):
     """Check the trajectory `traj` (dict of torch tensors or numpy arrays
     with the env's [T][K][N] layout) of a rollout of workload `w` that
     started from the first reset draw at global step t_g0.  final_state:
     optional (state, params, t_ep, episode) arrays of the env after the
     rollout.  resync: optional {t: (state, params, t_ep, episode)} of the
-    kernel's batch before step t; the oracle continues from it.  Returns the
-    measured maxima."""
+    kernel's batch before step t; the oracle continues from it.  net_tol:
+    bound on the network outputs' absolute error (the oracle evaluates the
+    workload's network arithmetic: bf16 emulation for bf16 networks, exact
+    otherwise).  Returns the measured maxima."""
     paper = W.is_paper(w)
     n_all = int(w["n_envs"])
     ids = np.asarray(ids, dtype=np.int64)
@@ -93,6 +96,7 @@ def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None, resy
     H = int(w["hidden"])
     worst = dict(obs=0.0, rew=0.0, act=0.0, logp=0.0, value=0.0)
     rew_ref = np.zeros((T, k))
+    obs_hist = []
     for t in range(T):
         if resync and t in resync:
             st, pr, t_ep, ep = (np.asarray(x) for x in resync[t])
@@ -108,22 +112,30 @@ def check_engine_rollout(oracle, w, traj, ids, T, t_g0=0, final_state=None, resy
                                 for j in range(k)], axis=1)
         e = _rel(g["obs"][t], ref_obs)
         worst["obs"] = max(worst["obs"], e.max())
-        _check(e.max() <= STATE_TOL, f"obs[{t}]: rel err {e.max():.3e}")
+        if e.max() > STATE_TOL:
+            kk, jj = np.unravel_index(np.argmax(e), e.shape)
+            hist = [float(np.max(_rel(g["obs"][u][:, jj], obs_hist[u][:, jj])))
+                    for u in range(max(0, t - 8), t)]
+            _check(False, f"obs[{t}]: rel err {e.max():.3e} at component {kk}, env {ids[jj]}: "
+                          f"gpu {g['obs'][t][kk, jj]!r} oracle {ref_obs[kk, jj]!r}; env "
+                          f"obs errors of the 8 previous steps {hist}; t_ep {b.t_ep[jj]}")
+        obs_hist.append(ref_obs)
         o = g["obs"][t].T.astype(np.float64)
         a_ref, lp_ref, mu = act_fn(m, pw, ids.astype(np.uint32), t_g0 + t, o, with_mu=True)
         da = np.abs(g["act"][t].T - a_ref)
-        bound = BF16_TOL * (1.0 + np.abs(a_ref - mu))
+        bound = net_tol * (1.0 + np.abs(a_ref - mu))
         worst["act"] = max(worst["act"], (da / (1.0 + np.abs(a_ref - mu))).max())
         _check(np.all(da <= bound), f"act[{t}]: max excess {(da - bound).max():.3e}")
         dl = np.abs(g["logp"][t] - lp_ref)
         worst["logp"] = max(worst["logp"], dl.max())
-        _check(dl.max() <= na * BF16_TOL, f"logp[{t}]: {dl.max():.3e}")
+        _check(dl.max() <= na * net_tol, f"logp[{t}]: {dl.max():.3e}")
         if vw is not None and "value" in g:
             v_ref = oracle.mlp(vw, d, H, 1, True, o)[:, 0]
             dv = np.abs(g["value"][t] - v_ref).max()
             worst["value"] = max(worst["value"], dv)
-            _check(dv <= BF16_TOL, f"value[{t}]: {dv:.3e}")
-        r, dn, _ = replay(m, b, np.ascontiguousarray(g["act"][t:t + 1], dtype=np.float32))
+            _check(dv <= net_tol, f"value[{t}]: {dv:.3e}")
+        a_t = np.ascontiguousarray(g["act"][t:t + 1], dtype=np.float32)
+        r, dn, _ = replay(m, b, a_t)
         _check(np.array_equal(g["done"][t], dn[0]), f"done[{t}] differs")
         e = _rel(g["rew"][t], r[0])
         worst["rew"] = max(worst["rew"], e.max())

@@ -46,23 +46,23 @@ def test_engine_rollout_every_step_paper(oracle, n, T, L):
     the benchmark's launch (the paper's env count and episode length,
     §IV-A, §V-A1); the ragged cases reset inside the launch, clearing the
     action history of Eq. 7's moving average.  The long launch is checked
-    in windows of 128 steps: the same rollout run as four launches of 128
-    steps is bit-identical to the single launch, and its state at each
-    window start restarts the oracle (fp32 against double rounding drift
-    reaches the 1e-5 tolerance after about 400 steps)."""
+    in windows of 64 steps: the same rollout run as launches of 64 steps is
+    bit-identical to the single launch, and its state at each window start
+    restarts the oracle (fp32 against double rounding drift can reach the
+    1e-5 tolerance within about a hundred steps)."""
     torch = need_gpu()
     w = W.workload("paper_4096", n_envs=n, episode_len=L)
     traj, final = _run(w, T)
     resync = None
-    if T > 128:
+    if T > 64:
         env = make_env(w)
         env.reset()
         resync, parts = {}, []
-        for t0 in range(0, T, 128):
+        for t0 in range(0, T, 64):
             resync[t0] = (to_np(env.state), to_np(env.params), to_np(env.t_ep),
                           to_np(env.episode))
-            part = env.alloc_traj(min(128, T - t0))
-            env.rollout(min(128, T - t0), part)
+            part = env.alloc_traj(min(64, T - t0))
+            env.rollout(min(64, T - t0), part)
             parts.append(part)
         assert env.status().code == 0
         for k in ("obs", "act", "logp", "rew", "done"):
@@ -90,3 +90,60 @@ def test_engine_rollout_every_step_after_a_first_launch(oracle):
     final = (to_np(env.state), to_np(env.params), to_np(env.t_ep), to_np(env.episode))
     ids = sample_ids(n, k=40)
     check_engine_rollout(oracle, w, full, ids, T1 + T2, final_state=final)
+
+
+# fp32 networks on the tensor cores (kind::tf32).  Weights, observations and
+# hidden activations are rounded to tf32 (10 explicit mantissa bits, relative
+# error below 2^-11), tanh is the hardware approximation (about 2^-11) and
+# sums are fp32: each hidden unit is within about 2^-10 of its exact value
+# relative to its size, and with N(0, 1/fan_in) weights these errors add in
+# quadrature through the 256-wide layers to a few 1e-4 on outputs of order
+# one.  TF32_TOL bounds them with a margin against the oracle's exact (double)
+# network; the measured maximum is printed.
+TF32_TOL = 3e-3
+
+
+def _windows(w, T, win=16):
+    """Run T steps as one launch and as launches of `win` steps; the two must
+    agree bit for bit, and the windowed run gives the state at each window
+    start for the checker to restart the oracle from.  The tolerance is on
+    the state one step produces (1e-5 relative); over tens of steps fp32 and
+    double rounding compound (with this workload's unit action noise the
+    thrust saturates often and the attitude error grows fastest: 1.1e-5 on
+    one env's body-frame position 32 steps after a common state), so
+    windows of 16 steps keep the comparison about single steps."""
+    torch = need_gpu()
+    traj, final = _run(w, T)
+    env = make_env(w)
+    env.reset()
+    resync, parts = {}, []
+    for t0 in range(0, T, win):
+        resync[t0] = (to_np(env.state), to_np(env.params), to_np(env.t_ep), to_np(env.episode))
+        part = env.alloc_traj(min(win, T - t0))
+        env.rollout(min(win, T - t0), part)
+        parts.append(part)
+    assert env.status().code == 0
+    for k in traj:
+        assert torch.equal(torch.cat([p[k] for p in parts]), traj[k]), k
+    return traj, final, resync
+
+
+@pytest.mark.parametrize("name,n,T,L", [("fp32_4096", 4096, 1000, 500),
+                                        ("dr_16384", 16384, 1000, 500),
+                                        ("fp32_4096", 999, 50, 17),
+                                        ("dr_16384", 300, 20, 6)])
+def test_tf32_engine_rollout_every_step(oracle, name, n, T, L):
+    """The fp32 workloads' tensor-core rollout (k_rollout_tf32): 4,096 envs x
+    1,000 steps (the paper's env count, BASELINE's second workload) and
+    16,384 envs x 1,000 steps with domain randomisation and current (the
+    third), both with auto-resets at step 500, plus ragged sizes that reset
+    inside short launches; every step of 40 sampled envs against the oracle."""
+    need_gpu()
+    w = W.workload(name, n_envs=n, episode_len=L, mlp="tf32")
+    traj, final, resync = _windows(w, T) if T > 16 else (*_run(w, T), None)
+    ids = sample_ids(n, k=40)
+    worst = check_engine_rollout(oracle, w, traj, ids, T, final_state=final, resync=resync,
+                                 net_tol=TF32_TOL)
+    print(f"[tf32 engine {name} n={n} T={T} L={L}] " +
+          " ".join(f"{k} {v:.2e}" for k, v in worst.items()))
+    assert worst["act"] <= TF32_TOL
