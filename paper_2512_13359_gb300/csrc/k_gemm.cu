@@ -362,52 +362,33 @@ k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const flo
   }
 }
 
-// C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output; four
-// consecutive columns per thread (n_pad is a multiple of 64), the split loop
-// unrolled so that several partial loads are in flight.
+// C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output; one element
+// per thread (tens of thousands of threads for a weight gradient), the split
+// loop unrolled by four so that four partial loads are in flight.
 __global__ void k_reduce(int M, int N, int splits, const float* __restrict__ ws, int m_pad,
                          int n_pad, void* C, int ldc, int c_bf16, float beta) {
-  const int nq = (N + 3) >> 2;
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (size_t)M * nq) return;
-  const int m = (int)(idx / nq), n0 = 4 * (int)(idx % nq);
+  if (idx >= (size_t)M * N) return;
+  const int m = (int)(idx / N), n = (int)(idx % N);
   const size_t zs = (size_t)m_pad * n_pad;
-  const float4* src = reinterpret_cast<const float4*>(ws + (size_t)m * n_pad + n0);
-  float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  const float* src = ws + (size_t)m * n_pad + n;
+  float v = 0.0f;
   int z = 0;
   for (; z + 4 <= splits; z += 4) {
-    float4 p[4];
+    float p[4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) p[q] = __ldg(src + (z + q) * (zs >> 2));
+    for (int q = 0; q < 4; ++q) p[q] = __ldg(src + (size_t)(z + q) * zs);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      v.x += p[q].x;
-      v.y += p[q].y;
-      v.z += p[q].z;
-      v.w += p[q].w;
-    }
+    for (int q = 0; q < 4; ++q) v += p[q];
   }
-  for (; z < splits; ++z) {
-    const float4 p = __ldg(src + z * (zs >> 2));
-    v.x += p.x;
-    v.y += p.y;
-    v.z += p.z;
-    v.w += p.w;
-  }
-  const float r[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int n = n0 + q;
-    if (n >= N) break;
-    float x = r[q];
-    if (c_bf16) {
-      uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
-      if (beta != 0.0f) x = fmaf(beta, __uint_as_float((uint32_t)*c << 16), x);
-      *c = (uint16_t)(tc::pack_bf16x2(x, 0.0f) & 0xFFFFu);
-    } else {
-      float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
-      *c = beta != 0.0f ? fmaf(beta, *c, x) : x;
-    }
+  for (; z < splits; ++z) v += __ldg(src + (size_t)z * zs);
+  if (c_bf16) {
+    uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
+    if (beta != 0.0f) v = fmaf(beta, __uint_as_float((uint32_t)*c << 16), v);
+    *c = (uint16_t)(tc::pack_bf16x2(v, 0.0f) & 0xFFFFu);
+  } else {
+    float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
+    *c = beta != 0.0f ? fmaf(beta, *c, v) : v;
   }
 }
 
@@ -629,7 +610,7 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
                       : dispatch_major<false, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
   }
   if (e != cudaSuccess || !part) return e;
-  const size_t n = (size_t)M * ((N + 3) / 4);
+  const size_t n = (size_t)M * N;
   k_reduce<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(M, N, P.splits, part, P.m_pad, P.n_pad, C,
                                                        ldc, c_bf16 ? 1 : 0, beta);
   return cudaGetLastError();
