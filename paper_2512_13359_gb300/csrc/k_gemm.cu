@@ -40,7 +40,7 @@ namespace auv {
 namespace gemm {
 namespace {
 
-constexpr int kStages = 4;
+constexpr int kMaxStages = 4;
 constexpr int kBM = 128;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
@@ -105,20 +105,26 @@ struct TcArgs {
   int vec;                // C base and ldc allow 16-byte row segments
 };
 
+// BN = 320 (for N in (256, 320]: the weight gradients' 264 augmented
+// columns) is one N = 256 and one N = 64 MMA per K-step, in a three-stage
+// ring; the other widths are one MMA in a four-stage ring.
 template <bool TF32, bool A_MN, bool B_MN, int BN>
 struct Tile {
   static constexpr int kEs = TF32 ? 4 : 2;
   static constexpr int kBK = 128 / kEs;                 // K elements per stage
+  static constexpr int kStages = BN > 256 ? 3 : 4;
   static constexpr uint32_t kABytes = kBM * 128;        // 128 rows (or BK K-rows x 128 B x 128/E)
   static constexpr uint32_t kBBytes = BN * 128;
   static constexpr uint32_t kStage = kABytes + kBBytes;
   static constexpr uint32_t kSmem = kStages * kStage + 256 + 1024;
   static constexpr int kElemsPer128 = 128 / kEs;        // M/N elements per MN-major box
+  static constexpr int kBoxRows = BN > 256 ? 64 : BN;   // K-major B: rows per TMA box
+  static constexpr uint32_t kTmemCols = BN > 256 ? 512 : BN;
 };
 
 struct Bars {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[kMaxStages];
+  uint64_t empty[kMaxStages];
   uint64_t acc_full;
   uint32_t tmem_base;
   int abort;
@@ -134,6 +140,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023u) & ~(uintptr_t)1023u);
+  constexpr int kStages = TL::kStages;
   Bars* bar = reinterpret_cast<Bars*>(smem + kStages * TL::kStage);
   volatile int* abort = &bar->abort;
   const int tid = threadIdx.x, warp = tid >> 5;
@@ -153,7 +160,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     tc::mbar_fence_init();
   }
   if (warp == 5) {
-    tc::tmem_alloc(&bar->tmem_base, BN);
+    tc::tmem_alloc(&bar->tmem_base, TL::kTmemCols);
     tc::tmem_relinquish();
   }
   tc::tc_fence_before();
@@ -186,7 +193,10 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
           for (int j = 0; j < BN / TL::kElemsPer128; ++j)
             tma_load_2d(b_dst + j * (TL::kBK * 128), &map_b, n0 + j * TL::kElemsPer128, k, &bar->full[s]);
         } else {
-          tma_load_2d(b_dst, &map_b, k, n0, &bar->full[s]);
+#pragma unroll
+          for (int j = 0; j < BN / TL::kBoxRows; ++j)
+            tma_load_2d(b_dst + j * (TL::kBoxRows * 128), &map_b, k, n0 + j * TL::kBoxRows,
+                        &bar->full[s]);
         }
       }
     }
@@ -194,7 +204,11 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   } else if (warp == 5) {
     // ---- MMA issue ----
     if ((tid & 31) == 0) {
-      constexpr uint32_t kId = idesc(TF32, A_MN, B_MN, kBM, BN);
+      constexpr uint32_t kId = idesc(TF32, A_MN, B_MN, kBM, BN > 256 ? 256 : BN);
+      constexpr uint32_t kId2 = idesc(TF32, A_MN, B_MN, kBM, BN > 256 ? BN - 256 : 16);
+      // second MMA of a 320-wide tile: B from column 256 (MN-major: the fifth
+      // 128-byte block of bf16; K-major: row 256)
+      constexpr uint32_t kB2 = B_MN ? (256 / TL::kElemsPer128) * (TL::kBK * 128) : 256 * 128;
       constexpr uint32_t kLbo = TL::kBK * 128;          // MN-major: between 128-byte M/N blocks
       constexpr uint32_t kKStepMn = 4096 / TL::kEs;     // MN-major: bytes per 32 bytes of K
       bool ok = true;
@@ -211,6 +225,11 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
           const uint64_t db = B_MN ? desc_sw128(b0 + kk * kKStepMn, kLbo, 1024)
                                    : desc_sw128(b0 + kk * 32, 16, 1024);
           mma<TF32>(tmem, da, db, kId, (c > 0 || kk > 0) ? 1u : 0u);
+          if constexpr (BN > 256) {
+            const uint64_t db2 = B_MN ? desc_sw128(b0 + kB2 + kk * kKStepMn, kLbo, 1024)
+                                      : desc_sw128(b0 + kB2 + kk * 32, 16, 1024);
+            mma<TF32>(tmem + 256, da, db2, kId2, (c > 0 || kk > 0) ? 1u : 0u);
+          }
         }
         tc::mma_commit(&bar->empty[s]);
       }
@@ -300,7 +319,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   }
   if (warp == 5) {
     tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, BN);
+    tc::tmem_dealloc(tmem, TL::kTmemCols);
   }
 }
 
@@ -477,7 +496,12 @@ Plan plan(Prec prec, int M, int N, int K) {
     p.bk = 16;
   } else {
     p.bm = kBM;
-    p.bn = (N > 128 && N <= 256) ? 256 : 128;
+    // 320-wide tiles (one CTA over the weight gradients' 264 augmented
+    // columns: the other operand read once instead of three times) pay when
+    // there are at least two M-tiles; with one, three 128-wide tiles keep more
+    // CTAs per K-range (measured 28.1 against 37.9 us for 256 x 264 x 65,536,
+    // 25.4 against 21.4 us for 16 x 264 x 65,536)
+    p.bn = (N > 128 && N <= 256) ? 256 : ((N > 256 && N <= 320 && M > kBM) ? 320 : 128);
     p.bk = prec == kTf32 ? 32 : 64;
   }
   p.tiles_m = (M + p.bm - 1) / p.bm;
@@ -597,17 +621,19 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
     const bool ok_a = A.mn_major ? make_map(&ma, tf32, A.ptr, M, K, A.ld, bk)
                                  : make_map(&ma, tf32, A.ptr, K, M, A.ld, kBM);
     const bool ok_b = B.mn_major ? make_map(&mb, tf32, B.ptr, N, K, B.ld, bk)
-                                 : make_map(&mb, tf32, B.ptr, K, N, B.ld, P.bn);
+                                 : make_map(&mb, tf32, B.ptr, K, N, B.ld, P.bn > 256 ? 64 : P.bn);
     if (!ok_a || !ok_b) return cudaErrorInvalidValue;
     const int ces = c_bf16 ? 2 : 4;
     const int vec = (reinterpret_cast<uintptr_t>(C) % 16 == 0 && ((size_t)ldc * ces) % 16 == 0) ? 1 : 0;
     TcArgs a = {M, N, K, P.per_split, C, ldc, c_bf16 ? 1 : 0, beta, part, P.n_pad, P.m_pad, st, vec};
     if (tf32)
-      e = P.bn == 256 ? dispatch_major<true, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)
-                      : dispatch_major<true, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
+      e = P.bn == 320   ? dispatch_major<true, 320>(A.mn_major, B.mn_major, P, ma, mb, a, s)
+          : P.bn == 256 ? dispatch_major<true, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)
+                        : dispatch_major<true, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
     else
-      e = P.bn == 256 ? dispatch_major<false, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)
-                      : dispatch_major<false, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
+      e = P.bn == 320   ? dispatch_major<false, 320>(A.mn_major, B.mn_major, P, ma, mb, a, s)
+          : P.bn == 256 ? dispatch_major<false, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)
+                        : dispatch_major<false, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
   }
   if (e != cudaSuccess || !part) return e;
   const size_t n = (size_t)M * N;

@@ -48,12 +48,15 @@ CASES = [
     ("bf16", 16, 264, 5000, True, True, False, 1.0, 0),         # gW3 (out = 16), ragged K
     ("bf16", 256, 24, 9999, True, True, False, 0.0, 0),         # gW1 (Dp = 24)
     ("bf16", 1, 1, 1, False, False, False, 0.0, 7),             # smallest
+    ("bf16", 500, 300, 64, False, False, False, 0.0, 0),        # 320-wide tile, K-major B
+    ("bf16", 300, 290, 3000, True, True, True, 1.0, 0),         # 320-wide tile, bf16 out
     ("tf32", 1000, 256, 24, False, False, False, 0.0, 0),
     ("tf32", 4096, 264, 264, False, False, False, 0.0, 0),
     ("tf32", 1000, 256, 264, False, True, False, 0.0, 0),
     ("tf32", 256, 264, 32768, True, True, False, 1.0, 4),
     ("tf32", 16, 264, 3000, True, True, False, 0.0, 0),
     ("tf32", 3, 5, 7, True, False, False, 0.0, 1),
+    ("tf32", 500, 290, 40, False, False, False, 0.0, 0),        # 320-wide tile
     ("fp32", 1000, 256, 24, False, False, False, 0.0, 0),
     ("fp32", 513, 264, 256, False, True, False, 1.0, 3),
     ("fp32", 256, 264, 20000, True, True, False, 0.0, 0),
