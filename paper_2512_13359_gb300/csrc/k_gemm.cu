@@ -21,7 +21,7 @@
 //    8 K rows form a 1024-byte group (SBO); an MMA's K-step (32 bytes of
 //    K) advances the start address by 4096 / element-size bytes.
 //
-// fp32 operands without tensor cores (the exact mode): a tiled CUDA-core
+// fp32 operands without tensor cores (the exact mode): a register-blocked CUDA-core
 // kernel with the same operand layouts and the same split-K.
 //
 // Split-K: partial tiles go to ws[z][M_pad][N_pad] (fp32); k_reduce adds
@@ -323,54 +323,100 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   }
 }
 
-// fp32 CUDA-core GEMM: 64 x 64 tile of C per CTA, 256 threads with 4 x 4
-// outputs each, K in slices of 16 through shared memory.
-template <bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(256)
+// fp32 CUDA-core GEMM: a BM x 128 tile of C per CTA (BM = 128, or 32 for
+// the few-row weight gradients of the output layers), 256 threads as 16 x 16
+// with BM/16 x 8 outputs each (BM = 128: rows ty*4 .. +3 and 64 + ty*4 .. +3,
+// columns likewise, so shared-memory reads are float4; BM = 32: rows ty*2,
+// ty*2 + 1), K in slices of 8 through double-buffered shared memory that
+// holds both operands M/N-fastest (As[k][m], Bs[k][n]) whichever way they
+// are stored.  Rows are padded by 4 floats: the K-major loads' stores (8 k of
+// 4 rows per warp) then land in 32 distinct banks, and row starts stay
+// 16-byte aligned.
+template <int BM, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(256, 2)
 k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const float* __restrict__ B,
             int ldb, int chunks_per_split, void* C, int ldc, float beta, float* ws, int m_pad,
             int n_pad) {
-  __shared__ float As[16][64 + 4];
-  __shared__ float Bs[16][64 + 4];
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const int m0 = blockIdx.x * 64, n0 = blockIdx.y * 64;
-  const int k_begin = blockIdx.z * chunks_per_split * 16;
-  const int k_end = min(K, k_begin + chunks_per_split * 16);
-  float acc[4][4] = {};
-  for (int kb = k_begin; kb < k_end; kb += 16) {
-    // 64 x 16 elements of each operand, 4 per thread
+  constexpr int RM = BM / 16, QA = BM / 32;
+  __shared__ __align__(16) float As[2][8][BM + 4];
+  __shared__ __align__(16) float Bs[2][8][132];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * 128;
+  const int k_begin = blockIdx.z * chunks_per_split * 8;
+  const int k_end = min(K, k_begin + chunks_per_split * 8);
+  // element e of a ROWS x 8 slice: (row, k) with consecutive threads along
+  // the stored-contiguous index
+  auto coord = [](int e, int rows, bool mn, int& r, int& kk) {
+    if (mn) { kk = e / rows; r = e % rows; } else { r = e >> 3; kk = e & 7; }
+  };
+  auto load = [&](const float* X, int ld, bool mn, int rows, int r0, int R, int kb, float* v, int q_n) {
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const int e = threadIdx.x + 256 * q;
+      if (q >= q_n) break;
       int r, kk;
-      if (A_MN) { kk = e >> 6; r = e & 63; } else { r = e >> 4; kk = e & 15; }
-      const int m = m0 + r, k = kb + kk;
-      As[kk][r] = (m < M && k < k_end) ? (A_MN ? A[(size_t)k * lda + m] : A[(size_t)m * lda + k]) : 0.0f;
-      if (B_MN) { kk = e >> 6; r = e & 63; } else { r = e >> 4; kk = e & 15; }
-      const int n = n0 + r, k2 = kb + kk;
-      Bs[kk][r] = (n < N && k2 < k_end) ? (B_MN ? B[(size_t)k2 * ldb + n] : B[(size_t)n * ldb + k2]) : 0.0f;
+      coord(tid + 256 * q, rows, mn, r, kk);
+      const int rr = r0 + r, k = kb + kk;
+      v[q] = (rr < R && k < k_end) ? (mn ? X[(size_t)k * ld + rr] : X[(size_t)rr * ld + k]) : 0.0f;
+    }
+  };
+  auto store = [&](float* S, int stride, bool mn, int rows, const float* v, int q_n) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (q >= q_n) break;
+      int r, kk;
+      coord(tid + 256 * q, rows, mn, r, kk);
+      S[kk * stride + r] = v[q];
+    }
+  };
+  float acc[RM][8] = {};
+  float va[4], vb[4];
+  int buf = 0;
+  if (k_begin < k_end) {
+    load(A, lda, A_MN, BM, m0, M, k_begin, va, QA);
+    load(B, ldb, B_MN, 128, n0, N, k_begin, vb, 4);
+    store(&As[0][0][0], BM + 4, A_MN, BM, va, QA);
+    store(&Bs[0][0][0], 132, B_MN, 128, vb, 4);
+  }
+  __syncthreads();
+  for (int kb = k_begin; kb < k_end; kb += 8) {
+    const bool more = kb + 8 < k_end;
+    if (more) {                                   // next slice in flight during this one
+      load(A, lda, A_MN, BM, m0, M, kb + 8, va, QA);
+      load(B, ldb, B_MN, 128, n0, N, kb + 8, vb, 4);
+    }
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+      float a[RM];
+      if constexpr (BM == 128) {
+        const float4 a0 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
+        const float4 a1 = *reinterpret_cast<const float4*>(&As[buf][kk][64 + ty * 4]);
+        a[0] = a0.x; a[1] = a0.y; a[2] = a0.z; a[3] = a0.w;
+        a[4] = a1.x; a[5] = a1.y; a[6] = a1.z; a[7] = a1.w;
+      } else {
+        const float2 a0 = *reinterpret_cast<const float2*>(&As[buf][kk][ty * 2]);
+        a[0] = a0.x; a[1] = a0.y;
+      }
+      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][64 + tx * 4]);
+      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int i = 0; i < RM; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    if (more) {
+      store(&As[buf ^ 1][0][0], BM + 4, A_MN, BM, va, QA);
+      store(&Bs[buf ^ 1][0][0], 132, B_MN, 128, vb, 4);
     }
     __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < 16; ++kk) {
-      float a[4], b[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-    }
-    __syncthreads();
+    buf ^= 1;
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int m = m0 + ty * 4 + i;
+  for (int i = 0; i < RM; ++i) {
+    const int m = m0 + (BM == 128 ? (i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4) : ty * 2 + i);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int n = n0 + tx * 4 + j;
+    for (int j = 0; j < 8; ++j) {
+      const int n = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + j - 4);
       if (ws) {
         if (m < m_pad && n < n_pad) ws[((size_t)blockIdx.z * m_pad + m) * n_pad + n] = acc[i][j];
       } else if (m < M && n < N) {
@@ -492,8 +538,9 @@ struct Plan {
 Plan plan(Prec prec, int M, int N, int K) {
   Plan p;
   if (prec == kFp32) {
-    p.bm = p.bn = 64;
-    p.bk = 16;
+    p.bm = M <= 32 ? 32 : 128;
+    p.bn = 128;
+    p.bk = 8;
   } else {
     p.bm = kBM;
     // 320-wide tiles (one CTA over the weight gradients' 264 augmented
@@ -508,7 +555,9 @@ Plan plan(Prec prec, int M, int N, int K) {
   p.tiles_n = (N + p.bn - 1) / p.bn;
   p.chunks = std::max(1, (K + p.bk - 1) / p.bk);
   const int tiles = p.tiles_m * p.tiles_n;
-  const int sms = sm_count_dev();
+  // CTAs wanted: one per SM for the tensor-core kernel, two for the
+  // CUDA-core one (two 256-thread CTAs resident per SM hide its loads)
+  const int sms = sm_count_dev() * (prec == kFp32 ? 2 : 1);
   int want = tiles >= sms / 2 ? 1 : (sms + tiles - 1) / tiles;
   // at least 4 K-chunks per CTA, at most one split per chunk
   want = std::max(1, std::min(want, p.chunks / 4));
@@ -601,13 +650,17 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
     const dim3 grid(P.tiles_m, P.tiles_n, P.splits);
     const float* a = static_cast<const float*>(A.ptr);
     const float* b = static_cast<const float*>(B.ptr);
-#define AUV_FP32_GEMM(AM, BM)                                                                    \
-  k_gemm_fp32<AM, BM><<<grid, 256, 0, s>>>(M, N, K, a, A.ld, b, B.ld, P.per_split, C, ldc, beta, \
-                                           part, P.m_pad, P.n_pad)
-    if (A.mn_major && B.mn_major) AUV_FP32_GEMM(true, true);
-    else if (A.mn_major) AUV_FP32_GEMM(true, false);
-    else if (B.mn_major) AUV_FP32_GEMM(false, true);
-    else AUV_FP32_GEMM(false, false);
+#define AUV_FP32_GEMM(TM, AM, BM)                                                           \
+  k_gemm_fp32<TM, AM, BM><<<grid, 256, 0, s>>>(M, N, K, a, A.ld, b, B.ld, P.per_split, C, ldc, \
+                                               beta, part, P.m_pad, P.n_pad)
+#define AUV_FP32_MAJOR(TM)                                         \
+  if (A.mn_major && B.mn_major) AUV_FP32_GEMM(TM, true, true);     \
+  else if (A.mn_major) AUV_FP32_GEMM(TM, true, false);             \
+  else if (B.mn_major) AUV_FP32_GEMM(TM, false, true);             \
+  else AUV_FP32_GEMM(TM, false, false)
+    if (P.bm == 32) { AUV_FP32_MAJOR(32); }
+    else { AUV_FP32_MAJOR(128); }
+#undef AUV_FP32_MAJOR
 #undef AUV_FP32_GEMM
     e = cudaGetLastError();
   } else {

@@ -61,6 +61,10 @@ CASES = [
     ("fp32", 513, 264, 256, False, True, False, 1.0, 3),
     ("fp32", 256, 264, 20000, True, True, False, 0.0, 0),
     ("fp32", 2, 3, 1, True, True, False, 0.0, 0),
+    ("fp32", 16, 264, 5000, True, True, False, 1.0, 0),         # 32-row tile: gW3
+    ("fp32", 1, 264, 3001, True, True, False, 0.0, 2),          # value head gW3 (out = 1)
+    ("fp32", 32, 130, 77, False, True, False, 0.0, 1),          # 32-row tile, K-major A
+    ("fp32", 33, 129, 40, True, False, False, 1.0, 0),          # just over: 128-row tile
 ]
 
 
