@@ -122,6 +122,8 @@ struct Dims {
   int D, Dp;     // observation width and its padded, augmented row (>= D + 1)
   int A;         // action width; policy head 2A
   int H, Hp;     // hidden width and its augmented row (>= H + 1)
+  int Ha;        // row length of the activation arrays H1, H2 (>= Hp; bf16: a
+                 // multiple of 16, so that rows start on 32-byte boundaries)
   int B;         // minibatch
   int ld_pol;    // row length of the policy head arrays Y, dL/dY (>= 2A)
   int ld_val;    // row length of the value head arrays (>= 1)

@@ -243,16 +243,55 @@ struct RowIO {            // row modes: obs element (r, k) at ((r / ns) * obs_di
   const uint16_t* a2;
   int lda;
   int ldh2;
+  // every learner row (h1, h2, a1, a2; a 16-wide policy head) starts on a
+  // 32-byte boundary: rows move as 32-byte pieces, whole L2 sectors
+  int wide;
 };
 
-// 32 accumulator columns times tanh' from the forward's bf16 activations at
-// h (16-byte aligned): g (1 - h^2), rounded to 16 bf16 pairs.
-__device__ __forceinline__ void dtanh32(const uint32_t (&acc)[32], const uint16_t* h,
-                                        uint32_t (&out)[16]) {
+// Row pieces as whole 32-byte sectors (sm_100 and later: 256-bit loads and
+// stores).  A thread's row piece is otherwise half a sector per access, and
+// the warp's 32 rows make 32 partial-sector requests.
+__device__ __forceinline__ void st_b32x8(void* p, uint32_t a, uint32_t b, uint32_t c, uint32_t d,
+                                         uint32_t e, uint32_t f, uint32_t g, uint32_t h) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(a),
+               "r"(b), "r"(c), "r"(d), "r"(e), "r"(f), "r"(g), "r"(h)
+               : "memory");
+}
+
+__device__ __forceinline__ void ld_b32x8(const void* p, uint4& lo, uint4& hi) {
+  asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(lo.x), "=r"(lo.y), "=r"(lo.z), "=r"(lo.w), "=r"(hi.x), "=r"(hi.y),
+                 "=r"(hi.z), "=r"(hi.w)
+               : "l"(p));
+}
+
+// 32 bf16 values (64 bytes, 16-byte aligned; wide: 32-byte aligned) from
+// global memory.
+__device__ __forceinline__ void ld_bf16x32(const uint16_t* h, uint4 (&u)[4], bool wide = false) {
+  if (wide) {
+    ld_b32x8(h, u[0], u[1]);
+    ld_b32x8(h + 16, u[2], u[3]);
+    return;
+  }
   const uint4* q = reinterpret_cast<const uint4*>(h);
 #pragma unroll
+  for (int p = 0; p < 4; ++p) u[p] = __ldg(q + p);
+}
+
+// Ask for the 128-byte lines of a row of `bytes` bytes to be brought into L2.
+__device__ __forceinline__ void prefetch_row_l2(const void* p, int bytes) {
+  const char* c = static_cast<const char*>(p);
+  for (int o = 0; o < bytes; o += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(c + o));
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(c + bytes - 1));
+}
+
+// 32 accumulator columns times tanh' from the forward's bf16 activations h
+// (32 values): g (1 - h^2), rounded to 16 bf16 pairs.
+__device__ __forceinline__ void dtanh32(const uint32_t (&acc)[32], const uint4 (&hv)[4],
+                                        uint32_t (&out)[16]) {
+#pragma unroll
   for (int p = 0; p < 4; ++p) {
-    const uint4 u = __ldg(q + p);
+    const uint4 u = hv[p];
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -264,8 +303,23 @@ __device__ __forceinline__ void dtanh32(const uint32_t (&acc)[32], const uint16_
   }
 }
 
-// 32 bf16 values (16 pairs) to 64 bytes at p (16-byte aligned).
-__device__ __forceinline__ void store_bf16x32(uint16_t* p, const uint32_t (&v)[16]) {
+// The same, reading the activations at h (16-byte aligned) when needed.
+__device__ __forceinline__ void dtanh32(const uint32_t (&acc)[32], const uint16_t* h,
+                                        uint32_t (&out)[16]) {
+  uint4 u[4];
+  ld_bf16x32(h, u);
+  dtanh32(acc, u, out);
+}
+
+// 32 bf16 values (16 pairs) to 64 bytes at p (16-byte aligned; wide:
+// 32-byte aligned).
+__device__ __forceinline__ void store_bf16x32(uint16_t* p, const uint32_t (&v)[16],
+                                              bool wide = false) {
+  if (wide) {
+    st_b32x8(p, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7]);
+    st_b32x8(p + 16, v[8], v[9], v[10], v[11], v[12], v[13], v[14], v[15]);
+    return;
+  }
   uint4* q = reinterpret_cast<uint4*>(p);
 #pragma unroll
   for (int j = 0; j < 4; ++j) q[j] = make_uint4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
@@ -608,6 +662,17 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     auto run_network = [&](int k, int it, float* head, uint16_t* h1r, uint16_t* h2r,
                            const uint16_t* a1r, const uint16_t* a2r) -> bool {
       const int slot = k & 1;
+      // Backward with at most two groups (registers to spare): the forward
+      // activations tanh' needs are loaded one chunk ahead of their use, so
+      // that their memory latency overlaps the tensor-core work instead of
+      // sitting between an accumulator read and its epilogue.
+      constexpr bool kPreA = E::kBack && G <= 2;
+      uint4 pa[2][4];
+      const bool wide = io.wide != 0;
+      if constexpr (kPreA) {
+        ld_bf16x32(a1r, pa[0], wide);
+        ld_bf16x32(a1r + 32, pa[1], wide);
+      }
       // layer 1 -> h1 slot.  Chunk c's bf16 pairs go to slot columns
       // 32c..32c+31, which held accumulator columns this thread has already
       // read (chunk 0's second half for c = 1, chunk 1's for c = 2, 3).
@@ -632,10 +697,21 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::tc_fence_before();
             tc::mbar_arrive(&bar->empty_x);
           }
-          if constexpr (E::kBack) dtanh32(acc, a1r + c * kChunk + 32 * half, hv);
-          else tanh32(acc, hv);
+          if constexpr (kPreA) {
+            uint4 cur[4];
+#pragma unroll
+            for (int p = 0; p < 4; ++p) cur[p] = pa[half][p];
+            // next: this half of chunk c + 1, or of layer 2's chunk 0
+            ld_bf16x32(c + 1 < kNChunks ? a1r + (c + 1) * kChunk + 32 * half : a2r + 32 * half,
+                       pa[half], wide);
+            dtanh32(acc, cur, hv);
+          } else if constexpr (E::kBack) {
+            dtanh32(acc, a1r + c * kChunk + 32 * half, hv);
+          } else {
+            tanh32(acc, hv);
+          }
           tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
-          if (E::kLearn && h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv);
+          if (E::kLearn && h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv, wide);
         }
       }
       tc::tmem_st_wait();
@@ -660,9 +736,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             tc::tc_fence_before();
             tc::mbar_arrive(odd ? &bar->empty_z : &bar->empty_y);
           }
-          if constexpr (E::kBack) dtanh32(acc, a2r + c * kChunk + 32 * half, hv);
-          else bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
-          if (E::kLearn && h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv);
+          if constexpr (kPreA) {
+            uint4 cur[4];
+#pragma unroll
+            for (int p = 0; p < 4; ++p) cur[p] = pa[half][p];
+            if (c + 1 < kNChunks) ld_bf16x32(a2r + (c + 1) * kChunk + 32 * half, pa[half], wide);
+            dtanh32(acc, cur, hv);
+          } else if constexpr (E::kBack) {
+            dtanh32(acc, a2r + c * kChunk + 32 * half, hv);
+          } else {
+            bias_tanh32(acc, b2 + c * kChunk + 32 * half, hv);
+          }
+          if (E::kLearn && h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv, wide);
           if constexpr (E::kBack) {
             // backward: dL/dZ1 goes to global memory only
           } else if (kPolicy) {
@@ -845,17 +930,44 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
       }
     } else {
+      // Learner modes with at most two groups: the next iteration's input
+      // row is loaded while this one runs (and, backward, the next rows of
+      // forward activations are requested into L2), so no iteration starts
+      // with a wait on memory.
+      constexpr bool kPreX = E::kLearn && G <= 2;
+      constexpr int kXq = (kObs + 7) / 8;
+      auto load_x = [&](size_t rr, uint4 (&u)[kXq]) {
+        const uint4* x = reinterpret_cast<const uint4*>(io.xb + rr * (size_t)io.ldx);
+#pragma unroll
+        for (int q = 0; q < kXq; ++q)
+          u[q] = (rr < io.rows && 8 * q < io.obs_dim) ? __ldg(x + q) : make_uint4(0u, 0u, 0u, 0u);
+      };
+      uint4 xn[kXq];
+      if constexpr (kPreX) load_x((size_t)(slot0 + g) * kRows + row, xn);
       for (int it = 0; it < my_iters && ok; ++it) {
         const size_t r = (size_t)(slot0 + g + it * n_slots) * kRows + row;
         const bool active = r < io.rows;
         float o[kObs];
+        uint4 xc[kXq];
+        if constexpr (kPreX) {
+          const size_t rn = r + (size_t)n_slots * kRows;
+#pragma unroll
+          for (int q = 0; q < kXq; ++q) xc[q] = xn[q];
+          if (it + 1 < my_iters) {
+            load_x(rn, xn);
+            if (E::kBack && rn < io.rows) {
+              prefetch_row_l2(io.a1 + rn * (size_t)io.lda, 2 * kH);
+              prefetch_row_l2(io.a2 + rn * (size_t)io.lda, 2 * kH);
+            }
+          }
+        } else if (E::kLearn && active) {
+          load_x(r, xc);
+        }
         if (E::kLearn && active) {
           // bf16 row, 16-byte pieces (ldx a multiple of 8, >= obs_dim)
-          const uint4* x = reinterpret_cast<const uint4*>(io.xb + r * (size_t)io.ldx);
 #pragma unroll
-          for (int q = 0; q < (kObs + 7) / 8; ++q) {
-            uint4 u = make_uint4(0u, 0u, 0u, 0u);
-            if (8 * q < io.obs_dim) u = __ldg(x + q);
+          for (int q = 0; q < kXq; ++q) {
+            const uint4 u = xc[q];
             const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
@@ -896,9 +1008,20 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             io.out[r * (size_t)(io.ldo ? io.ldo : 1)] = head[0];
           } else {
             const size_t ldo = (size_t)(io.ldo ? io.ldo : io.out_dim);
+            if (E::kLearn && io.wide && io.out_dim == kHeadOut) {
+              float* o16 = io.out + r * ldo;
+              st_b32x8(o16, __float_as_uint(head[0]), __float_as_uint(head[1]),
+                       __float_as_uint(head[2]), __float_as_uint(head[3]), __float_as_uint(head[4]),
+                       __float_as_uint(head[5]), __float_as_uint(head[6]), __float_as_uint(head[7]));
+              st_b32x8(o16 + 8, __float_as_uint(head[8]), __float_as_uint(head[9]),
+                       __float_as_uint(head[10]), __float_as_uint(head[11]),
+                       __float_as_uint(head[12]), __float_as_uint(head[13]),
+                       __float_as_uint(head[14]), __float_as_uint(head[15]));
+            } else {
 #pragma unroll
-            for (int k = 0; k < kHeadOut; ++k)
-              if (k < io.out_dim) io.out[r * ldo + k] = head[k];
+              for (int k = 0; k < kHeadOut; ++k)
+                if (k < io.out_dim) io.out[r * ldo + k] = head[k];
+            }
           }
         }
       }
@@ -1079,13 +1202,17 @@ cudaError_t launch_value_bf16(const Model& M, const void* wv_packed, const float
   return launch_rows<kValueRows>(M, static_cast<const uint8_t*>(wv_packed), io, st, s);
 }
 
+static bool al32(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 31u) == 0; }
+
 cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_dim, int out_dim,
                                       const uint16_t* x, int ldx, size_t rows, uint16_t* h1,
                                       uint16_t* h2, int ldh, float* out, int ldo, Status* st,
                                       cudaStream_t s) {
   const Model M{};
-  const RowIO io = {nullptr, rows, 1,   out,     in_dim,  policy ? out_dim : 1, x, ldx, h1, h2,
-                    ldh,     ldo,  nullptr, nullptr, 0, 0};
+  RowIO io = {nullptr, rows, 1,   out,     in_dim,  policy ? out_dim : 1, x, ldx, h1, h2,
+              ldh,     ldo,  nullptr, nullptr, 0, 0};
+  io.wide = ldh % 16 == 0 && al32(h1) && al32(h2) &&
+            (!policy || out_dim != kHeadOut || (ldo % 8 == 0 && al32(out)));
   const uint8_t* img = static_cast<const uint8_t*>(packed);
   return policy ? launch_rows<kLearnPolicy>(M, img, io, st, s)
                 : launch_rows<kLearnValue>(M, img, io, st, s);
@@ -1096,8 +1223,10 @@ cudaError_t launch_learn_backward_bf16(const void* packed, int out_dim, const ui
                                        uint16_t* gz2, int ldz2, uint16_t* gz1, int ldz1, Status* st,
                                        cudaStream_t s) {
   const Model M{};
-  const RowIO io = {nullptr, rows, 1,  nullptr, out_dim, 1,  gy, ldy, gz2, gz1,
-                    ldz2,    0,    h2, h1,      ldh,     ldz1};
+  RowIO io = {nullptr, rows, 1,  nullptr, out_dim, 1,  gy, ldy, gz2, gz1,
+              ldz2,    0,    h2, h1,      ldh,     ldz1};
+  io.wide = ldz2 % 16 == 0 && ldz1 % 16 == 0 && ldh % 16 == 0 && al32(gz2) && al32(gz1) &&
+            al32(h2) && al32(h1);
   return launch_rows<kBackRows>(M, static_cast<const uint8_t*>(packed), io, st, s);
 }
 

@@ -428,25 +428,27 @@ k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const flo
 }
 
 // C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output; one element
-// per thread (tens of thousands of threads for a weight gradient), the split
-// loop unrolled by four so that four partial loads are in flight.
+// per thread.  A weight gradient has a few tens of thousands of elements and
+// tens of splits, so the kernel is bound by load latency: each thread issues
+// the loads of 16 partials before it adds them (in z order), so that a split
+// count below 80 costs at most five round trips to memory.
 __global__ void k_reduce(int M, int N, int splits, const float* __restrict__ ws, int m_pad,
                          int n_pad, void* C, int ldc, int c_bf16, float beta) {
+  constexpr int kU = 16;
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (size_t)M * N) return;
   const int m = (int)(idx / N), n = (int)(idx % N);
   const size_t zs = (size_t)m_pad * n_pad;
   const float* src = ws + (size_t)m * n_pad + n;
   float v = 0.0f;
-  int z = 0;
-  for (; z + 4 <= splits; z += 4) {
-    float p[4];
+  for (int z = 0; z < splits; z += kU) {
+    float p[kU];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) p[q] = __ldg(src + (size_t)(z + q) * zs);
+    for (int q = 0; q < kU; ++q) p[q] = z + q < splits ? __ldcs(src + (size_t)(z + q) * zs) : 0.0f;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) v += p[q];
+    for (int q = 0; q < kU; ++q)
+      if (z + q < splits) v += p[q];
   }
-  for (; z < splits; ++z) v += __ldg(src + (size_t)z * zs);
   if (c_bf16) {
     uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
     if (beta != 0.0f) v = fmaf(beta, __uint_as_float((uint32_t)*c << 16), v);

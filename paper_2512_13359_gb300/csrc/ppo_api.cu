@@ -241,16 +241,16 @@ int forward(auv_ppo* p, int net, cudaStream_t s) {
   const char *w1 = w, *w2 = w + (size_t)d.H * d.Dp * es, *w3 = w2 + (size_t)d.H * d.Hp * es;
   cudaError_t e;
   if ((e = gemm(p, true, false, d.H, d.B, d.Dp, w1, d.Dp, p->X, d.Dp, p->h1[net],
-                 d.Hp, false, s)))
+                 d.Ha, false, s)))
     return cuda_fail(p, e, "forward layer 1");
-  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h1[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h1[net], d.Ha, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh 1");
-  if ((e = gemm(p, true, false, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Hp,
-                 p->h2[net], d.Hp, false, s)))
+  if ((e = gemm(p, true, false, d.H, d.B, d.Hp, w2, d.Hp, p->h1[net], d.Ha,
+                 p->h2[net], d.Ha, false, s)))
     return cuda_fail(p, e, "forward layer 2");
-  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h2[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_fwd(p->bf16, p->h2[net], d.Ha, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh 2");
-  if ((e = gemm(p, true, false, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Hp,
+  if ((e = gemm(p, true, false, p->out[net], d.B, d.Hp, w3, d.Hp, p->h2[net], d.Ha,
                  p->y[net], ld_head(p, net), true, s)))
     return cuda_fail(p, e, "forward layer 3");
   return AUV_OK;
@@ -267,7 +267,7 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
   void* gz2 = p->gb[net];
   void* gz1 = p->h2[net];       // H2 is dead once gZ2 exists
   cudaError_t e;
-  if ((e = gemm(p, false, true, d.Hp, out, d.B, p->h2[net], d.Hp, gy, ldy, g3, d.Hp,
+  if ((e = gemm(p, false, true, d.Hp, out, d.B, p->h2[net], d.Ha, gy, ldy, g3, d.Hp,
                  true, s)))
     return cuda_fail(p, e, "gradient W3");
   if (p->eng) {
@@ -275,29 +275,29 @@ int backward(auv_ppo* p, int net, const void* gy, cudaStream_t s) {
     // weight gradients of layers 2 and 1
     if ((e = auv::launch_learn_backward_bf16(
              net ? p->img_bv : p->img_bp, out, static_cast<const uint16_t*>(gy), ldy, (size_t)d.B,
-             static_cast<const uint16_t*>(p->h2[net]), static_cast<const uint16_t*>(p->h1[net]), d.Hp,
-             static_cast<uint16_t*>(gz2), d.H, static_cast<uint16_t*>(gz1), d.Hp, p->st, s)))
+             static_cast<const uint16_t*>(p->h2[net]), static_cast<const uint16_t*>(p->h1[net]), d.Ha,
+             static_cast<uint16_t*>(gz2), d.H, static_cast<uint16_t*>(gz1), d.Ha, p->st, s)))
       return cuda_fail(p, e, "engine backward");
-    if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+    if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Ha, gz2, d.H, g2, d.Hp,
                    true, s)))
       return cuda_fail(p, e, "gradient W2");
-    if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+    if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Ha, g1, d.Dp,
                    true, s)))
       return cuda_fail(p, e, "gradient W1");
     return AUV_OK;
   }
   if ((e = gemm(p, false, false, d.H, d.B, out, w3, d.Hp, gy, ldy, gz2, d.H, false, s)))
     return cuda_fail(p, e, "gradient H2");
-  if ((e = ppo::launch_tanh_bwd(p->bf16, gz2, d.H, p->h2[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_bwd(p->bf16, gz2, d.H, p->h2[net], d.Ha, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 2");
-  if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Hp, gz2, d.H, g2, d.Hp,
+  if ((e = gemm(p, false, true, d.Hp, d.H, d.B, p->h1[net], d.Ha, gz2, d.H, g2, d.Hp,
                  true, s)))
     return cuda_fail(p, e, "gradient W2");
-  if ((e = gemm(p, false, false, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Hp, false, s)))
+  if ((e = gemm(p, false, false, d.H, d.B, d.H, w2, d.Hp, gz2, d.H, gz1, d.Ha, false, s)))
     return cuda_fail(p, e, "gradient H1");
-  if ((e = ppo::launch_tanh_bwd(p->bf16, gz1, d.Hp, p->h1[net], d.Hp, d.B, d.H, s)))
+  if ((e = ppo::launch_tanh_bwd(p->bf16, gz1, d.Ha, p->h1[net], d.Ha, d.B, d.H, s)))
     return cuda_fail(p, e, "tanh' 1");
-  if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Hp, g1, d.Dp,
+  if ((e = gemm(p, false, true, d.Dp, d.H, d.B, p->X, d.Dp, gz1, d.Ha, g1, d.Dp,
                  true, s)))
     return cuda_fail(p, e, "gradient W1");
   return AUV_OK;
@@ -339,7 +339,7 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
       if ((e = auv::launch_learn_forward_bf16(net == 0, net ? p->img_v : p->img_p, d.D, p->out[net],
                                          static_cast<const uint16_t*>(p->X), d.Dp, (size_t)d.B,
                                          static_cast<uint16_t*>(p->h1[net]),
-                                         static_cast<uint16_t*>(p->h2[net]), d.Hp, p->y[net],
+                                         static_cast<uint16_t*>(p->h2[net]), d.Ha, p->y[net],
                                          ld_head(p, net), p->st, s)))
         return cuda_fail(p, e, "engine forward");
     }
@@ -470,6 +470,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
   d.ld_pol = round8(2 * d.A);
   d.ld_val = 8;
   d.bf16 = cfg->precision == AUV_PPO_BF16;
+  d.Ha = d.bf16 ? (d.H + 16) / 16 * 16 : d.Hp;
   d.value_only = (cfg->flags & AUV_PPO_VALUE_ONLY) ? 1 : 0;
   p->bf16 = d.bf16 != 0;
   p->esz = p->bf16 ? 2 : 4;
@@ -511,8 +512,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_st = take(sizeof(Status));
   size_t o_h1[2], o_h2[2], o_gb[2], o_y[2];
   for (int k = 0; k < 2; ++k) {
-    o_h1[k] = take(B * d.Hp * es);
-    o_h2[k] = take(B * d.Hp * es);
+    o_h1[k] = take(B * d.Ha * es);
+    o_h2[k] = take(B * d.Ha * es);
     o_gb[k] = take(B * d.H * es);
     o_y[k] = take(B * (k ? d.ld_val : d.ld_pol) * 4);
   }
@@ -563,8 +564,8 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
     e = cudaMemcpy(p->st, &s0, sizeof(s0), cudaMemcpyHostToDevice);
   }
   for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
-    e = ppo::launch_fill_ones(p->bf16, p->h1[k], d.Hp, d.H, d.B, 0);
-    if (e == cudaSuccess) e = ppo::launch_fill_ones(p->bf16, p->h2[k], d.Hp, d.H, d.B, 0);
+    e = ppo::launch_fill_ones(p->bf16, p->h1[k], d.Ha, d.H, d.B, 0);
+    if (e == cudaSuccess) e = ppo::launch_fill_ones(p->bf16, p->h2[k], d.Ha, d.H, d.B, 0);
   }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
