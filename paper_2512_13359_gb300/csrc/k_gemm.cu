@@ -103,7 +103,17 @@ struct TcArgs {
   int n_pad, m_pad;
   Status* st;
   int vec;                // C base and ldc allow 16-byte row segments
+  int ws_wide;            // ws 32-byte aligned: partial rows as whole 32-byte sectors
 };
+
+// 8 floats to a 32-byte aligned address with one 256-bit store (a whole L2
+// sector; a thread writing its own row otherwise fills half a sector per
+// access).
+__device__ __forceinline__ void st_f32x8(float* p, const uint32_t* v) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]),
+               "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
 
 // BN = 320 (for N in (256, 320]: the weight gradients' 264 augmented
 // columns) is one N = 256 and one N = 64 MMA per K-step, in a three-stage
@@ -253,13 +263,19 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       }
       const int nb = n0 + j * 32;
       if (args.ws) {
-        if (row < args.m_pad) {
-          float4* dst = reinterpret_cast<float4*>(
-              args.ws + ((size_t)blockIdx.z * args.m_pad + row) * args.n_pad + nb);
+        // partials of the rows and 32-column groups the reduction reads
+        if (row < args.M && nb < args.N) {
+          float* dst = args.ws + ((size_t)blockIdx.z * args.m_pad + row) * args.n_pad + nb;
+          if (args.ws_wide) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            dst[q] = make_float4(__uint_as_float(acc[4 * q]), __uint_as_float(acc[4 * q + 1]),
-                                 __uint_as_float(acc[4 * q + 2]), __uint_as_float(acc[4 * q + 3]));
+            for (int q = 0; q < 4; ++q) st_f32x8(dst + 8 * q, acc + 8 * q);
+          } else {
+            float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              d4[q] = make_float4(__uint_as_float(acc[4 * q]), __uint_as_float(acc[4 * q + 1]),
+                                  __uint_as_float(acc[4 * q + 2]), __uint_as_float(acc[4 * q + 3]));
+          }
         }
       } else if (row < args.M && args.beta == 0.0f && nb + 32 <= args.N && args.vec) {
         // whole 32-column segment, 16-byte aligned rows: vector stores
@@ -417,8 +433,8 @@ k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const flo
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int n = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + j - 4);
-      if (ws) {
-        if (m < m_pad && n < n_pad) ws[((size_t)blockIdx.z * m_pad + m) * n_pad + n] = acc[i][j];
+      if (ws) {   // partials of the elements the reduction reads
+        if (m < M && n < N) ws[((size_t)blockIdx.z * m_pad + m) * n_pad + n] = acc[i][j];
       } else if (m < M && n < N) {
         float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
         *c = beta != 0.0f ? fmaf(beta, *c, acc[i][j]) : acc[i][j];
@@ -680,7 +696,9 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
     if (!ok_a || !ok_b) return cudaErrorInvalidValue;
     const int ces = c_bf16 ? 2 : 4;
     const int vec = (reinterpret_cast<uintptr_t>(C) % 16 == 0 && ((size_t)ldc * ces) % 16 == 0) ? 1 : 0;
-    TcArgs a = {M, N, K, P.per_split, C, ldc, c_bf16 ? 1 : 0, beta, part, P.n_pad, P.m_pad, st, vec};
+    const int ws_wide = reinterpret_cast<uintptr_t>(part) % 32 == 0 ? 1 : 0;
+    TcArgs a = {M,     N,      K,       P.per_split, C,  ldc,    c_bf16 ? 1 : 0,
+                beta,  part,   P.n_pad, P.m_pad,     st, vec,    ws_wide};
     if (tf32)
       e = P.bn == 320   ? dispatch_major<true, 320>(A.mn_major, B.mn_major, P, ma, mb, a, s)
           : P.bn == 256 ? dispatch_major<true, 256>(A.mn_major, B.mn_major, P, ma, mb, a, s)

@@ -169,8 +169,6 @@ constexpr int kT = 256;
 constexpr float kHalfLog2Pi = 0.91893853320467274f;
 
 // Activation storage: fp32, or bf16 (round to nearest even) in bf16 mode.
-__device__ __forceinline__ float ld_act(const float* p) { return *p; }
-__device__ __forceinline__ float ld_act(const __nv_bfloat16* p) { return __bfloat162float(*p); }
 __device__ __forceinline__ void st_act(float* p, float x) { *p = x; }
 __device__ __forceinline__ void st_act(__nv_bfloat16* p, float x) { *p = __float2bfloat16_rn(x); }
 
@@ -336,6 +334,59 @@ __device__ __forceinline__ void st_act8(float* p, const float v[8]) {
   reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
 }
 
+// A row of 8 words at p: one 256-bit access (a whole 32-byte L2 sector) when
+// p is 32-byte aligned, else 16-byte pieces or single words.  A thread that
+// writes its own sample's row otherwise covers a fraction of a sector per
+// access, and the warp's 32 rows make 32 partial-sector requests.
+__device__ __forceinline__ void st_row8(void* p, const uint32_t w[8]) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  if (a % 32 == 0) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]),
+                 "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+  } else if (a % 16 == 0) {
+    reinterpret_cast<uint4*>(p)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    reinterpret_cast<uint4*>(p)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) static_cast<uint32_t*>(p)[j] = w[j];
+  }
+}
+
+__device__ __forceinline__ void ld_row8(const void* p, uint32_t w[8]) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  if (a % 32 == 0) {
+    asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]),
+                   "=r"(w[6]), "=r"(w[7])
+                 : "l"(p));
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = __ldg(static_cast<const uint32_t*>(p) + j);
+  }
+}
+
+// 2A head-gradient values of one sample (A = 8) as one row: bf16 pairs in
+// one sector, or fp32 in two.
+__device__ __forceinline__ void st_head16(__nv_bfloat16* p, const float v[16]) {
+  uint32_t w[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+    memcpy(&w[j], &h, 4);
+  }
+  st_row8(p, w);
+}
+__device__ __forceinline__ void st_head16(float* p, const float v[16]) {
+  uint32_t w[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) w[j] = __float_as_uint(v[j]);
+  st_row8(p, w);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) w[j] = __float_as_uint(v[8 + j]);
+  st_row8(p + 8, w);
+}
+
 // One sample per thread: its whole row (Ws <= W floats) is loaded at once
 // and X is written in chunks of eight with vector stores; W is a
 // compile-time bound on the row, so the row lives in registers.
@@ -380,8 +431,14 @@ __global__ void __launch_bounds__(kT) k_gather_sm(Dims d, PermKey key, const Ste
     // from the row again (its sectors are in L1 from the loads above), so
     // that v stays in registers
     const float* f = rows + (size_t)r * Ws + d.D;
-    if (!d.value_only)
+    if (!d.value_only && d.A == 8) {
+      uint32_t w[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = __float_as_uint(__ldg(f + j));
+      st_row8(out.act + (size_t)b * 8, w);
+    } else if (!d.value_only) {
       for (int j = 0; j < d.A; ++j) out.act[(size_t)b * d.A + j] = __ldg(f + j);
+    }
     const float lp = __ldg(f + d.A), a = __ldg(f + d.A + 1);
     out.ret[b] = __ldg(f + d.A + 2);
     if (!d.value_only) {
@@ -502,14 +559,28 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
     float dm[8], iv[8], z2[8];
     bool in[8];
     float lp = -(float)A * kHalfLog2Pi, ent = (float)A * (0.5f + kHalfLog2Pi);
+    // A = 8: the sample's 16 head outputs and 8 actions as whole sectors
+    float yv[16], av[8];
+    if (A == 8) {
+      uint32_t w[8];
+      ld_row8(yb, w);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) yv[j] = __uint_as_float(w[j]);
+      ld_row8(yb + 8, w);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) yv[8 + j] = __uint_as_float(w[j]);
+      ld_row8(ab, w);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) av[j] = __uint_as_float(w[j]);
+    }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       if (k < A) {
-        const float raw = yb[A + k];
+        const float raw = A == 8 ? yv[8 + k] : yb[A + k];
         const float ls = fminf(fmaxf(raw, hp.logstd_min), hp.logstd_max);
         in[k] = raw >= hp.logstd_min && raw <= hp.logstd_max;
         iv[k] = expf(-2.0f * ls);
-        dm[k] = ab[k] - yb[k];
+        dm[k] = A == 8 ? av[k] - yv[k] : ab[k] - yb[k];
         z2[k] = dm[k] * dm[k] * iv[k];
         lp += -0.5f * z2[k] - ls;
         ent += ls;
@@ -521,11 +592,21 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
     const bool unclipped = an > 0.0f ? r <= hi : r >= lo;
     const float g_lp = unclipped ? -an * r * inv_b : 0.0f;
     TG* gy = g_y + (size_t)b * d.ld_pol;
+    if (A == 8) {
+      float gv[16];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      if (k < A) {
-        st_act(gy + k, g_lp * dm[k] * iv[k]);
-        st_act(gy + A + k, in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f);
+      for (int k = 0; k < 8; ++k) {
+        gv[k] = g_lp * dm[k] * iv[k];
+        gv[8 + k] = in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f;
+      }
+      st_head16(gy, gv);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (k < A) {
+          st_act(gy + k, g_lp * dm[k] * iv[k]);
+          st_act(gy + A + k, in[k] ? g_lp * (z2[k] - 1.0f) - hp.ent_coef * inv_b : 0.0f);
+        }
       }
     }
     const float dv = v[(size_t)b * d.ld_val] - smp.ret[b];
