@@ -196,6 +196,7 @@ cudaError_t launch_head(const Dims& d, const LossHp& hp, const float* y, const f
 cudaError_t launch_stats(const Dims& d, const LossHp& hp, const float* part, float* mb,
                          float* acc, cudaStream_t s);
 // wb (bf16 copy of w, may be NULL) is rewritten with the new weights.
+// part: kNormBlocks + 3 floats (norm partials, then the step's scalars).
 cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, float* part,
                         const AdamHp& hp, const StepCtl* ctl, float* mb, float* acc, void* wb,
                         cudaStream_t s);

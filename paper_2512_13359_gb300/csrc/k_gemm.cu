@@ -102,7 +102,7 @@ struct TcArgs {
   float* ws;              // split partials, or null (write C directly)
   int n_pad, m_pad;
   Status* st;
-  int vec;                // C base and ldc allow 16-byte row segments
+  int vec;                // C base and ldc allow 16-byte (1) or 32-byte (2) row segments
   int ws_wide;            // ws 32-byte aligned: partial rows as whole 32-byte sectors
 };
 
@@ -279,18 +279,25 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         }
       } else if (row < args.M && args.beta == 0.0f && nb + 32 <= args.N && args.vec) {
         // whole 32-column segment, 16-byte aligned rows: vector stores
+        // (32-byte aligned rows: whole sectors)
         if (args.c_bf16) {
-          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(args.C) +
-                                                (size_t)row * args.ldc + nb);
+          uint16_t* crow = static_cast<uint16_t*>(args.C) + (size_t)row * args.ldc + nb;
+          uint32_t w[16];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint32_t w[4];
+          for (int e = 0; e < 16; ++e)
+            w[e] = tc::pack_bf16x2(__uint_as_float(acc[2 * e]), __uint_as_float(acc[2 * e + 1]));
+          if (args.vec == 2) {
+            st_f32x8(reinterpret_cast<float*>(crow), w);
+            st_f32x8(reinterpret_cast<float*>(crow + 16), w + 8);
+          } else {
+            uint4* dst = reinterpret_cast<uint4*>(crow);
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              w[e] = tc::pack_bf16x2(__uint_as_float(acc[8 * q + 2 * e]),
-                                     __uint_as_float(acc[8 * q + 2 * e + 1]));
-            dst[q] = make_uint4(w[0], w[1], w[2], w[3]);
+            for (int q = 0; q < 4; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
           }
+        } else if (args.vec == 2) {
+          float* crow = static_cast<float*>(args.C) + (size_t)row * args.ldc + nb;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) st_f32x8(crow + 8 * q, acc + 8 * q);
         } else {
           float4* dst = reinterpret_cast<float4*>(static_cast<float*>(args.C) +
                                                   (size_t)row * args.ldc + nb);
@@ -695,7 +702,9 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
                                  : make_map(&mb, tf32, B.ptr, K, N, B.ld, P.bn > 256 ? 64 : P.bn);
     if (!ok_a || !ok_b) return cudaErrorInvalidValue;
     const int ces = c_bf16 ? 2 : 4;
-    const int vec = (reinterpret_cast<uintptr_t>(C) % 16 == 0 && ((size_t)ldc * ces) % 16 == 0) ? 1 : 0;
+    const int vec = (reinterpret_cast<uintptr_t>(C) % 32 == 0 && ((size_t)ldc * ces) % 32 == 0)
+                        ? 2
+                        : ((reinterpret_cast<uintptr_t>(C) % 16 == 0 && ((size_t)ldc * ces) % 16 == 0) ? 1 : 0);
     const int ws_wide = reinterpret_cast<uintptr_t>(part) % 32 == 0 ? 1 : 0;
     TcArgs a = {M,     N,      K,       P.per_split, C,  ldc,    c_bf16 ? 1 : 0,
                 beta,  part,   P.n_pad, P.m_pad,     st, vec,    ws_wide};

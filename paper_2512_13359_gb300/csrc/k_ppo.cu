@@ -656,34 +656,37 @@ __global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_
   if (threadIdx.x == 0) part[blockIdx.x] = (float)s[0];
 }
 
-// Clip by the global norm (every block reduces the same partials in the
-// same order) and take one Adam step.
-__global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float* __restrict__ g,
-                                             float* __restrict__ m, float* __restrict__ v,
-                                             size_t n, const float* __restrict__ part, AdamHp hp,
-                                             const StepCtl* ctl, float* mb, float* acc,
-                                             __nv_bfloat16* __restrict__ wb) {
+// The clip scale of the global gradient norm and the bias corrections of
+// step t + 1, once per step (one block; the partials summed in index order):
+// part[kNormBlocks + 0, 1, 2] = scale, 1 - b1^(t+1), 1 - b2^(t+1).
+__global__ void __launch_bounds__(kT) k_adam_prep(float* __restrict__ part, AdamHp hp,
+                                                  const StepCtl* ctl, float* mb, float* acc) {
   __shared__ double sh[kT / 32];
-  __shared__ float scale_sh, c1_sh, c2_sh;
   double s[1] = {0.0};
   for (int k = threadIdx.x; k < kNormBlocks; k += kT) s[0] += part[k];
   block_sum<1>(s, sh);
   if (threadIdx.x == 0) {
-    const double norm = sqrt(s[0]);
-    scale_sh = hp.max_norm > 0.0f ? (float)fmin(1.0, hp.max_norm / (norm + 1e-6)) : 1.0f;
-    // bias corrections of step t + 1; beta = 0 keeps the plain moment
-    const double t1 = (double)(ctl->t + 1ull);
-    const double c1 = 1.0 - pow((double)hp.b1, t1), c2 = 1.0 - pow((double)hp.b2, t1);
-    c1_sh = c1 > 0.0 ? (float)c1 : 1.0f;
-    c2_sh = c2 > 0.0 ? (float)c2 : 1.0f;
-    if (blockIdx.x == 0) {
-      mb[5] = (float)norm;
-      if (acc) acc[5] += (float)norm;
-    }
+    // fp32 from here: the GPU's fp64 pipe makes a double pow take microseconds
+    const float norm = sqrtf((float)s[0]);
+    part[kNormBlocks] = hp.max_norm > 0.0f ? fminf(1.0f, hp.max_norm / (norm + 1e-6f)) : 1.0f;
+    // 1 - b^t as -expm1(t log b); b = 0 keeps the plain moment
+    const float t1 = (float)(ctl->t + 1ull);
+    const float c1 = hp.b1 > 0.0f ? -expm1f(t1 * logf(hp.b1)) : 1.0f;
+    const float c2 = hp.b2 > 0.0f ? -expm1f(t1 * logf(hp.b2)) : 1.0f;
+    part[kNormBlocks + 1] = c1 > 0.0f ? c1 : 1.0f;
+    part[kNormBlocks + 2] = c2 > 0.0f ? c2 : 1.0f;
+    mb[5] = norm;
+    if (acc) acc[5] += norm;
   }
-  __syncthreads();
-  const float scale = scale_sh;
-  const float c1 = c1_sh, c2 = c2_sh;
+}
+
+// One Adam step on the clipped gradient (scalars from k_adam_prep).
+__global__ void __launch_bounds__(kT) k_adam(float* __restrict__ w, const float* __restrict__ g,
+                                             float* __restrict__ m, float* __restrict__ v,
+                                             size_t n, const float* __restrict__ part, AdamHp hp,
+                                             __nv_bfloat16* __restrict__ wb) {
+  const float scale = part[kNormBlocks];
+  const float c1 = part[kNormBlocks + 1], c2 = part[kNormBlocks + 2];
   const float ib1 = 1.0f - hp.b1, ib2 = 1.0f - hp.b2;
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
     const float gi = g[e] * scale;
@@ -861,8 +864,8 @@ cudaError_t launch_adam(float* w, const float* g, float* m, float* v, size_t n, 
                         const AdamHp& hp, const StepCtl* ctl, float* mb, float* acc, void* wb,
                         cudaStream_t s) {
   k_sumsq<<<kNormBlocks, kT, 0, s>>>(g, n, part);
-  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, ctl, mb, acc,
-                                    static_cast<__nv_bfloat16*>(wb));
+  k_adam_prep<<<1, kT, 0, s>>>(part, hp, ctl, mb, acc);
+  k_adam<<<grid_for(n), kT, 0, s>>>(w, g, m, v, n, part, hp, static_cast<__nv_bfloat16*>(wb));
   return cudaGetLastError();
 }
 

@@ -501,7 +501,7 @@ int ppo_create(const auv_ppo_config* cfg, auv_ppo** out) {
                o_act = take(B * d.A * 4), o_lp = take(B * 4), o_adv = take(B * 4),
                o_ret = take(B * 4), o_ap = take(nb * 2 * 8), o_gy = take(B * d.ld_pol * es),
                o_gv = take(B * d.ld_val * es), o_hp = take(nb * 5 * 4),
-               o_np = take(ppo::kNormBlocks * 4), o_mb = take(AUV_PPO_STATS * 4),
+               o_np = take((ppo::kNormBlocks + 3) * 4), o_mb = take(AUV_PPO_STATS * 4),
                o_acc = take(AUV_PPO_STATS * 4), o_ctl = take(sizeof(ppo::StepCtl)),
                o_ws = take(gws_bytes),
                o_ip = take(p->eng ? auv::bf16_policy_image_bytes() : 0),

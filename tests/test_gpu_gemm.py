@@ -103,6 +103,36 @@ def test_gemm_against_float64(prec, M, N, K, a_mn, b_mn, c_bf16, beta, pad):
     assert torch.equal(Cout[:, N:], C0[:, N:])
 
 
+@pytest.mark.parametrize("prec,M,N,K,c_bf16", [
+    ("bf16", 1000, 256, 24, False), ("bf16", 777, 264, 264, True), ("tf32", 513, 256, 40, False),
+    ("bf16", 300, 290, 64, True)])
+def test_gemm_sector_aligned_output(prec, M, N, K, c_bf16):
+    """C rows on 32-byte boundaries (ldc a multiple of 16): the epilogue's
+    whole-sector stores; the columns past N stay untouched."""
+    torch = need_gpu()
+    from paper_2512_13359_gb300 import auvenv
+    rng = np.random.default_rng(M + N + K)
+    dt = torch.bfloat16 if prec == "bf16" else torch.float32
+    mult = {"bf16": 8, "tf32": 4}[prec]
+    A, lda, a_log = _operand(torch, rng, M, K, False, dt, 0, mult)
+    B, ldb, b_log = _operand(torch, rng, N, K, False, dt, 0, mult)
+    ldc = -(-N // 16) * 16 + 16
+    cdt = torch.bfloat16 if c_bf16 else torch.float32
+    C0 = torch.from_numpy(rng.standard_normal((M, ldc)).astype(np.float32)).cuda().to(cdt)
+    Cout = C0.clone()
+    ws = torch.empty(max(1, auvenv.lib().auv_gemm_workspace_bytes(M, N, K)) // 4 + 1,
+                     dtype=torch.float32, device="cuda")
+    st = auvenv.gemm(prec, M, N, K, A, lda, False, B, ldb, False, Cout, ldc, 0.0, ws)
+    torch.cuda.synchronize()
+    assert st.cpu().tolist() == [0, 0, 0, 0]
+    ref = a_log @ b_log.T
+    scale = np.abs(a_log) @ np.abs(b_log).T
+    got = Cout.float().cpu().numpy().astype(np.float64)[:, :N]
+    tol = TOL[prec] * scale + 1e-30 + (2.0 ** -8 * np.abs(ref) if c_bf16 else 0.0)
+    assert np.all(np.abs(got - ref) <= tol)
+    assert torch.equal(Cout[:, N:], C0[:, N:])
+
+
 def test_gemm_rejects_bad_operands():
     torch = need_gpu()
     from paper_2512_13359_gb300 import auvenv
