@@ -625,15 +625,18 @@ __global__ void __launch_bounds__(kT) k_head(Dims d, LossHp hp, const float* __r
 __global__ void __launch_bounds__(kT) k_stats(int B, int n_part, float vf_coef, float ent_coef,
                                               const float* __restrict__ part, float* mb,
                                               float* acc) {
-  // (value-only steps leave the policy terms of part at 0)
-  __shared__ double sh[5 * (kT / 32)];
-  double s[5] = {0, 0, 0, 0, 0};
+  // (value-only steps leave the policy terms of part at 0).  fp32 sums of the
+  // per-block fp32 partials: the GPU's fp64 pipe made this one-block kernel
+  // take about 10 us, for statistics that are reported, not trained on.
+  __shared__ float sh[5 * (kT / 32)];
+  float s[5] = {0, 0, 0, 0, 0};
   for (int k = threadIdx.x; k < n_part; k += kT)
     for (int j = 0; j < 5; ++j) s[j] += part[5 * k + j];
   block_sum<5>(s, sh);
   if (threadIdx.x == 0) {
     float r[8];
-    for (int j = 0; j < 5; ++j) r[j] = (float)(s[j] / B);
+    const float inv_b = 1.0f / (float)B;
+    for (int j = 0; j < 5; ++j) r[j] = s[j] * inv_b;
     r[5] = 0.0f;
     r[6] = r[0] + vf_coef * r[1] - ent_coef * r[2];
     r[7] = 1.0f;
@@ -646,14 +649,14 @@ __global__ void __launch_bounds__(kT) k_stats(int B, int n_part, float vf_coef, 
 
 __global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_t n,
                                               float* __restrict__ part) {
-  __shared__ double sh[kT / 32];
-  double s[1] = {0.0};
+  __shared__ float sh[kT / 32];
+  float s[1] = {0.0f};
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n; e += (size_t)gridDim.x * kT) {
     const float x = g[e];
-    s[0] += (double)x * x;
+    s[0] = fmaf(x, x, s[0]);
   }
   block_sum<1>(s, sh);
-  if (threadIdx.x == 0) part[blockIdx.x] = (float)s[0];
+  if (threadIdx.x == 0) part[blockIdx.x] = s[0];
 }
 
 // The clip scale of the global gradient norm and the bias corrections of
@@ -661,13 +664,13 @@ __global__ void __launch_bounds__(kT) k_sumsq(const float* __restrict__ g, size_
 // part[kNormBlocks + 0, 1, 2] = scale, 1 - b1^(t+1), 1 - b2^(t+1).
 __global__ void __launch_bounds__(kT) k_adam_prep(float* __restrict__ part, AdamHp hp,
                                                   const StepCtl* ctl, float* mb, float* acc) {
-  __shared__ double sh[kT / 32];
-  double s[1] = {0.0};
+  __shared__ float sh[kT / 32];
+  float s[1] = {0.0f};
   for (int k = threadIdx.x; k < kNormBlocks; k += kT) s[0] += part[k];
   block_sum<1>(s, sh);
   if (threadIdx.x == 0) {
-    // fp32 from here: the GPU's fp64 pipe makes a double pow take microseconds
-    const float norm = sqrtf((float)s[0]);
+    // fp32 throughout: on the GPU's fp64 pipe a double pow takes microseconds
+    const float norm = sqrtf(s[0]);
     part[kNormBlocks] = hp.max_norm > 0.0f ? fminf(1.0f, hp.max_norm / (norm + 1e-6f)) : 1.0f;
     // 1 - b^t as -expm1(t log b); b = 0 keeps the plain moment
     const float t1 = (float)(ctl->t + 1ull);
