@@ -336,7 +336,13 @@ struct Engine {
   static constexpr uint32_t kOffObs = kImageAl;
   static constexpr uint32_t kOffH2 = kOffObs + G * kObsTileBytes;
   static constexpr uint32_t kOffBar = kOffH2 + (kPolicy ? 2 * kH2TileBytes : 0);
-  static constexpr uint32_t kSmem = kOffBar + sizeof(Barriers) + 1024;   // + alignment slack
+  // The paper model's action history in shared memory (one column per
+  // thread, copied in and out once per launch) where it fits: one group.
+  static constexpr bool kHistSmem = MODE == kRollout && G == 1;
+  static constexpr uint32_t kOffHist = (kOffBar + sizeof(Barriers) + 15u) & ~15u;
+  static constexpr uint32_t kHistBytes = kHistSmem ? 6u * paper::kHist * kRows * 4u : 0u;
+  static constexpr uint32_t kSmem = kOffHist + kHistBytes + 1024;   // + alignment slack
+  static_assert(kSmem <= 227u * 1024u, "shared memory per CTA");
   static constexpr int kThreads = G * kRows + 96;
 };
 
@@ -880,6 +886,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       paper::Env e;
       if (active) paper::load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
       bool bad = false;
+      // history rows: global (read past L1), or with one group this thread's
+      // shared-memory column
+      float* const hist_col = reinterpret_cast<float*>(smem + E::kOffHist) + row;
+      if constexpr (E::kHistSmem) {
+        if (active) {
+          const paper::HistG hg = paper::hist_rows(B.state, M.n, i);
+          for (int r = 0; r < 6 * paper::kHist; ++r) hist_col[r * kRows] = hg.ld(r);
+        }
+      }
       for (int t = 0; t < my_iters && ok; ++t) {
         float o[kPO];
         if (active) {
@@ -917,8 +932,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           }
           if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
           bool d;
-          const float r =
-              paper::physics_step(M, id, e, a, paper::hist_rows(B.state, M.n, i), &d);
+          float r;
+          if constexpr (E::kHistSmem)
+            r = paper::physics_step(M, id, e, a, paper::HistS{hist_col, kRows}, &d);
+          else
+            r = paper::physics_step(M, id, e, a, paper::hist_rows(B.state, M.n, i), &d);
           if (tr.rew) tr.rew[(size_t)t * n + i] = r;
           if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
           bad |= !paper::env_finite(e);
@@ -928,6 +946,10 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       if (active) {
         if (bad) flag_nan(st, i);
         paper::store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+        if constexpr (E::kHistSmem) {
+          const paper::HistG hg = paper::hist_rows(B.state, M.n, i);
+          for (int r = 0; r < 6 * paper::kHist; ++r) hg.st(r, hist_col[r * kRows]);
+        }
       }
     } else {
       // Learner modes with at most two groups: the next iteration's input
