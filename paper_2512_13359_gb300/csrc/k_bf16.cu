@@ -911,13 +911,18 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         tc::fence_async_smem();
         tc::mbar_arrive(&bar->obs_full[g]);
         float head[kHeadOut];
+        // The step's normals depend only on (env, seed, step): with one group
+        // per CTA (registers to spare) they are drawn while layer 1 runs
+        // instead of after the network.
+        constexpr bool kEarlyNoise = G == 1;
+        float eps[8];
+        if (kEarlyNoise && active) action_noise_approx(M.id_base + (uint32_t)i, M.seed, t_g0 + (uint64_t)t, eps);
         __syncwarp();
         if (!(ok = run_network(t * n_act + g, t, head, nullptr, nullptr, nullptr, nullptr))) break;
         __syncwarp();
         if (active) {
           const uint32_t id = M.id_base + (uint32_t)i;
-          float eps[8];
-          action_noise_approx(id, M.seed, t_g0 + (uint64_t)t, eps);
+          if (!kEarlyNoise) action_noise_approx(id, M.seed, t_g0 + (uint64_t)t, eps);
           float a[kPA], lp = 0.0f;
 #pragma unroll
           for (int k = 0; k < kPA; ++k) {
