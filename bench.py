@@ -551,8 +551,8 @@ def run_gae(args):
 # --steps 2 --warmup 1 --no-e2e --no-cpu-baseline --no-replay --no-clocks`;
 # profiles/k_engine_ppo_65536_T128_dram.md), valid while the engine's sources
 # hash to ENGINE_SRC_HASH.
-ROLLOUT_TRAFFIC_65536x128 = 10_482_176 + 900_390_144
-ENGINE_SRC_HASH = "e5a53d13eb31f1f0"
+ROLLOUT_TRAFFIC_65536x128 = 10_503_424 + 900_826_624
+ENGINE_SRC_HASH = "6302791373f9144f"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 
