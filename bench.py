@@ -651,7 +651,7 @@ def run_ppo(args):
                    "minibatch": B, "minibatches_per_epoch": n_mb, "epochs": args.epochs,
                    "precision": args.ppo_precision,
                    "l2": "working set per step larger than L2 when B >= 32768"},
-        "roofline": {"bound": bound, "kernel": "whole update (cuBLAS GEMMs + own kernels)",
+        "roofline": {"bound": bound, "kernel": "whole update (the library's GEMMs and learner kernels)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None, "peak_source": psrc,
                      "flops_per_sample": fps},
@@ -882,7 +882,7 @@ def run_shac(args):
         "data": "synthetic (workload resets, seeded random policy and critic)",
         "config": {"workload": w["name"], "n_envs": n, "window": T, "hidden": H, "precision": prec,
                    "l2": "working set per window (activations of every step) larger than L2"},
-        "roofline": {"bound": bound, "kernel": "whole window (cuBLAS GEMMs + own kernels)",
+        "roofline": {"bound": bound, "kernel": "whole window (the library's GEMMs and adjoint kernels)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None, "peak_source": psrc,
                      "flops_per_env_step": fps},
