@@ -9,8 +9,12 @@
 // control step:
 //   observation -> obs tile (smem, 32 fp32 columns, 18 used)
 //   layer 1: D[0, 256) = obs x W1^T          (W1 resident in smem)
-//   epilogue: + b1, tanh, round to tf32, written back in place (tcgen05.st)
-//   layer 2: D[256, 512) = h1 (A from tensor memory) x W2^T, W2 streamed
+//   epilogue: + b1, tanh, round to tf32, written back in place (tcgen05.st),
+//            32 columns at a time, each chunk announced as soon as it is in
+//            tensor memory
+//   layer 2: D[256, 512) = h1 (A from tensor memory) x W2^T, K-slice j
+//            issued once h1's chunk j is written (so it runs while the
+//            epilogue computes the later chunks), W2 streamed
 //            through a four-stage ring of 32 KB K-slices by bulk copies
 //            (256 KB of fp32 W2 does not fit beside the rest; the producer
 //            runs ahead, so the next step's first slices load during the
@@ -53,7 +57,8 @@ constexpr uint32_t kSRing = kSObs + kRows * 128;
 constexpr uint32_t kSBar = kSRing + kRing * kSliceBytes;
 
 struct Bars {
-  uint64_t img_full, obs_full, l1_full, h1_full, l2_full, h2_full, l3_full, drain;
+  uint64_t img_full, obs_full, l1_full, l2_full, h2_full, l3_full, drain;
+  uint64_t h1_part[kSlices];   // h1 columns 32j..32j+31 written (128 arrivals): layer-2 K-slice j may run
   uint64_t w2_full[kRing], w2_empty[kRing];
   uint32_t tmem_base;
   int abort;
@@ -147,9 +152,12 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 }
 
 // Hidden layer epilogue for this thread's row: 256 accumulator columns at
-// col0 -> + bias -> tanh -> tf32, written back in place.
+// col0 -> + bias -> tanh -> tf32, written back in place.  With `part` set,
+// each 32-column chunk is announced as soon as it is in tensor memory
+// (part[c], one arrival per thread), so that the next layer's K-slice c can
+// start while the later chunks are still being computed.
 __device__ __forceinline__ void hidden_epilogue(uint32_t lane_addr, uint32_t col0,
-                                                const float* bias) {
+                                                const float* bias, uint64_t* part = nullptr) {
 #pragma unroll 1
   for (int c = 0; c < kH / 32; ++c) {
     uint32_t acc[32];
@@ -160,6 +168,11 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t lane_addr, uint32_t col
       acc[j] = __float_as_uint(
           to_tf32(tc::tanh_f32(__uint_as_float(acc[j]) + bias[32 * c + j])));
     tmem_st32(lane_addr + col0 + 32 * c, acc);
+    if (part) {
+      tc::tmem_st_wait();
+      tc::tc_fence_before();
+      tc::mbar_arrive(&part[c]);
+    }
   }
   tc::tmem_st_wait();
 }
@@ -195,7 +208,7 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
     tc::mbar_init(&bar->img_full, 1);
     tc::mbar_init(&bar->obs_full, kRows);
     tc::mbar_init(&bar->l1_full, 1);
-    tc::mbar_init(&bar->h1_full, kRows);
+    for (int j = 0; j < kSlices; ++j) tc::mbar_init(&bar->h1_part[j], kRows);
     tc::mbar_init(&bar->l2_full, 1);
     tc::mbar_init(&bar->h2_full, kRows);
     tc::mbar_init(&bar->l3_full, 1);
@@ -254,10 +267,10 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
           mma_ss(tmem, desc(s_base + kSObs + kk * 32), desc(s_base + kSW1 + kk * 32), kI256,
                  kk > 0 ? 1u : 0u);
         tc::mma_commit(&bar->l1_full);
-        if (!(ok = tc::mbar_wait(&bar->h1_full, ph, abort, kWaitLimitNs))) break;
-        tc::tc_fence_after();
+        // layer 2, K-slice by K-slice as the epilogue writes h1's chunks
         for (int j = 0; j < kSlices && ok; ++j) {
           const int g = t * kSlices + j, s = g % kRing;
+          if (!(ok = tc::mbar_wait(&bar->h1_part[j], ph, abort, kWaitLimitNs))) break;
           if (!(ok = tc::mbar_wait(&bar->w2_full[s], (uint32_t)(g / kRing) & 1u, abort,
                                    kWaitLimitNs)))
             break;
@@ -324,9 +337,7 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
       __syncwarp();
       if (!(ok = tc::mbar_wait(&bar->l1_full, ph, abort, kWaitLimitNs))) break;
       tc::tc_fence_after();
-      hidden_epilogue(lane_addr, 0, bias);
-      tc::tc_fence_before();
-      tc::mbar_arrive(&bar->h1_full);
+      hidden_epilogue(lane_addr, 0, bias, bar->h1_part);
       if (!(ok = tc::mbar_wait(&bar->l2_full, ph, abort, kWaitLimitNs))) break;
       tc::tc_fence_after();
       hidden_epilogue(lane_addr, 256, bias + kH);
