@@ -19,8 +19,10 @@
 //            (256 KB of fp32 W2 does not fit beside the rest; the producer
 //            runs ahead, so the next step's first slices load during the
 //            current step's physics)
-//   epilogue: + b2, tanh, tf32, in place
-//   layer 3: D[0, 16) = h2 (tensor memory) x W3^T (resident)
+//   epilogue: + b2, tanh, tf32, in place, each 32-column chunk announced
+//   layer 3: D[0, 16) = h2 (tensor memory) x W3^T (resident), K-slice j
+//            issued once h2's chunk j is written (layer 2 has completed, so
+//            h1's columns are free for its accumulator)
 //   head: + b3 -> Gaussian action, physics substeps, reward, done, reset
 // Every wait is an mbarrier wait bounded by 2 s; a timeout raises the CTA's
 // abort flag and latches AUV_ERR_TIMEOUT in the status block.
@@ -57,8 +59,9 @@ constexpr uint32_t kSRing = kSObs + kRows * 128;
 constexpr uint32_t kSBar = kSRing + kRing * kSliceBytes;
 
 struct Bars {
-  uint64_t img_full, obs_full, l1_full, l2_full, h2_full, l3_full, drain;
+  uint64_t img_full, obs_full, l1_full, l2_full, l3_full, drain;
   uint64_t h1_part[kSlices];   // h1 columns 32j..32j+31 written (128 arrivals): layer-2 K-slice j may run
+  uint64_t h2_part[kSlices];   // h2 columns 256+32j.. written (128 arrivals): layer-3 K-slice j may run
   uint64_t w2_full[kRing], w2_empty[kRing];
   uint32_t tmem_base;
   int abort;
@@ -177,12 +180,10 @@ __device__ __forceinline__ void hidden_epilogue(uint32_t lane_addr, uint32_t col
   tc::tmem_st_wait();
 }
 
-// Gaussian head -> action and log-density (the fp32 path's sampling: the
-// accurate log, sine and exponential).
-__device__ __forceinline__ void sample(const Model& M, uint32_t id, uint64_t t_g,
-                                       const float* head, float a[kAct], float* logp) {
-  float eps[kAct];
-  action_noise(id, M.seed, t_g, eps);
+// Gaussian head and the step's normals -> action and log-density (the fp32
+// path's sampling: the accurate log, sine and exponential).
+__device__ __forceinline__ void sample(const Model& M, const float* head, const float eps[kAct],
+                                       float a[kAct], float* logp) {
   float lp = 0.0f;
 #pragma unroll
   for (int k = 0; k < kAct; ++k) {
@@ -210,7 +211,7 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
     tc::mbar_init(&bar->l1_full, 1);
     for (int j = 0; j < kSlices; ++j) tc::mbar_init(&bar->h1_part[j], kRows);
     tc::mbar_init(&bar->l2_full, 1);
-    tc::mbar_init(&bar->h2_full, kRows);
+    for (int j = 0; j < kSlices; ++j) tc::mbar_init(&bar->h2_part[j], kRows);
     tc::mbar_init(&bar->l3_full, 1);
     tc::mbar_init(&bar->drain, 1);
     for (int s = 0; s < kRing; ++s) {
@@ -262,8 +263,11 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
         const uint32_t ph = (uint32_t)t & 1u;
         if (!(ok = tc::mbar_wait(&bar->obs_full, ph, abort, kWaitLimitNs))) break;
         tc::tc_fence_after();
+        // K = 24 covers the 18 observation columns (the rest of the tile and
+        // of W1 is zero)
+        static_assert(kObs <= 24, "observation width");
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
+        for (int kk = 0; kk < 3; ++kk)
           mma_ss(tmem, desc(s_base + kSObs + kk * 32), desc(s_base + kSW1 + kk * 32), kI256,
                  kk > 0 ? 1u : 0u);
         tc::mma_commit(&bar->l1_full);
@@ -284,14 +288,15 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
         }
         if (!ok) break;
         tc::mma_commit(&bar->l2_full);
-        if (!(ok = tc::mbar_wait(&bar->h2_full, ph, abort, kWaitLimitNs))) break;
-        tc::tc_fence_after();
-        for (int j = 0; j < kSlices; ++j) {
+        for (int j = 0; j < kSlices && ok; ++j) {
+          if (!(ok = tc::mbar_wait(&bar->h2_part[j], ph, abort, kWaitLimitNs))) break;
+          tc::tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             mma_ts(tmem, tmem + 256 + 32 * j + 8 * kk, desc(s_base + kSW3 + j * kW3Slice + kk * 32),
                    kI16, (j > 0 || kk > 0) ? 1u : 0u);
         }
+        if (!ok) break;
         tc::mma_commit(&bar->l3_full);
       }
       tc::mma_commit(&bar->drain);
@@ -338,11 +343,14 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
       if (!(ok = tc::mbar_wait(&bar->l1_full, ph, abort, kWaitLimitNs))) break;
       tc::tc_fence_after();
       hidden_epilogue(lane_addr, 0, bias, bar->h1_part);
+      // The step's normals depend only on (env, seed, step): drawn here,
+      // while layer 2's last MMAs run, instead of after the head.
+      const uint32_t id = M.id_base + (uint32_t)i;
+      float eps[kAct];
+      if (active) action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
       if (!(ok = tc::mbar_wait(&bar->l2_full, ph, abort, kWaitLimitNs))) break;
       tc::tc_fence_after();
-      hidden_epilogue(lane_addr, 256, bias + kH);
-      tc::tc_fence_before();
-      tc::mbar_arrive(&bar->h2_full);
+      hidden_epilogue(lane_addr, 256, bias + kH, bar->h2_part);
       if (!(ok = tc::mbar_wait(&bar->l3_full, ph, abort, kWaitLimitNs))) break;
       tc::tc_fence_after();
       uint32_t o3[16];
@@ -355,8 +363,7 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
 #pragma unroll
         for (int k = 0; k < 16; ++k) head[k] = __uint_as_float(o3[k]) + bias[2 * kH + k];
         float a[kAct], lp;
-        const uint32_t id = M.id_base + (uint32_t)i;
-        sample(M, id, t_g0 + (uint64_t)t, head, a, &lp);
+        sample(M, head, eps, a, &lp);
         if (tr.act) {
 #pragma unroll
           for (int k = 0; k < kAct; ++k) tr.act[((size_t)t * kAct + k) * n + i] = a[k];
