@@ -213,6 +213,7 @@ struct Barriers {
   uint64_t acc3_full[4];    // head accumulator of group g complete
   uint64_t empty_x, empty_y, empty_z;   // accumulator read back (128 arrivals)
   uint64_t h1_full[2];      // h1 slot complete (128 arrivals)
+  uint64_t h1_part[2][4];   // one group per CTA: h1 chunk c of slot s written (128 arrivals)
   uint64_t h2_full[2];      // h2 buffer written (128 arrivals)
   uint64_t acc3_empty[2];   // head slot read back (128 arrivals)
   uint64_t h1_free[2];      // layer-2 MMAs reading an h1 slot completed (commit)
@@ -472,6 +473,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     tc::mbar_init(&bar->empty_z, kRows);
     for (int s = 0; s < 2; ++s) {
       tc::mbar_init(&bar->h1_full[s], kRows);
+      for (int c = 0; c < kNChunks; ++c) tc::mbar_init(&bar->h1_part[s][c], kRows);
       tc::mbar_init(&bar->h2_full[s], kRows);
       tc::mbar_init(&bar->acc3_empty[s], kRows);
       tc::mbar_init(&bar->h1_free[s], 1);
@@ -553,6 +555,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       };
       bool ok = true;
       int it = 0, g = 0;
+      // One group per CTA: no other group's layer 2 fills the tensor pipe
+      // while this group's layer-1 epilogue runs, so layer 2's chunks 0 and
+      // 1 (accumulators Y and Z, both drained by then) are fed K-slice by
+      // K-slice as h1's chunks are written (h1_part), not after all of h1.
+      constexpr bool kProgL2 = G == 1 && MODE == kRollout;
       if (warp == 4 * G) {
         uint32_t u_y = 0, u_z = 0;
         uint32_t p_h1 = 0;   // phase bit of slot s at bit s
@@ -579,11 +586,39 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         };
         for (int k = 0; k < total && ok; ++k) {
           const int s2 = k & 1;
-          ok = tc::mbar_wait(&bar->h1_full[s2], (p_h1 >> s2) & 1u, abort, kWaitLimitNs);
-          p_h1 ^= 1u << s2;
-          if (!ok) break;
-          tc::tc_fence_after();
-          ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          if constexpr (kProgL2) {
+            // chunks 0 and 1 (Y, Z) K-slice by K-slice as h1's chunks land
+            ok = tc::mbar_wait(&bar->empty_y, (u_y & 1u) ^ 1u, abort, kWaitLimitNs) &&
+                 tc::mbar_wait(&bar->empty_z, (u_z & 1u) ^ 1u, abort, kWaitLimitNs);
+            ++u_y;
+            ++u_z;
+            const uint32_t a0 = tmem + kColH1 + s2 * 128;
+            const uint64_t by = tc::smem_desc(s_base + kOffW2, 1024, 2);
+            const uint64_t bz = tc::smem_desc(s_base + kOffW2 + kChunk * 128, 1024, 2);
+            for (int c = 0; c < kNChunks && ok; ++c) {
+              ok = tc::mbar_wait(&bar->h1_part[s2][c], (p_h1 >> s2) & 1u, abort, kWaitLimitNs);
+              if (!ok) break;
+              tc::tc_fence_after();
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const int kk = 4 * c + q;
+                const uint64_t off = (uint64_t)(((kk >> 2) * (kH * 128) + (kk & 3) * 32) >> 4);
+                tc::mma_ts(tmem + kColY, a0 + kk * 8, by + off, kI64, kk > 0 ? 1u : 0u);
+                tc::mma_ts(tmem + kColZ, a0 + kk * 8, bz + off, kI64, kk > 0 ? 1u : 0u);
+              }
+            }
+            p_h1 ^= 1u << s2;
+            if (!ok) break;
+            tc::mma_commit(&bar->full_y[g]);
+            tc::mma_commit(&bar->full_z[g]);
+            ok = issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          } else {
+            ok = tc::mbar_wait(&bar->h1_full[s2], (p_h1 >> s2) & 1u, abort, kWaitLimitNs);
+            p_h1 ^= 1u << s2;
+            if (!ok) break;
+            tc::tc_fence_after();
+            ok = issue_l2(k, g, 0) && issue_l2(k, g, 1) && issue_l2(k, g, 2) && issue_l2(k, g, 3);
+          }
           advance(it, g);
         }
       } else if (warp == 4 * G + 2) {
@@ -719,10 +754,17 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           tc::tmem_st16(lane_addr + kColH1 + slot * 128 + c * 32 + half * 16, hv);
           if (E::kLearn && h1r) store_bf16x32(h1r + c * kChunk + 32 * half, hv, wide);
         }
+        if constexpr (G == 1 && MODE == kRollout) {   // chunk c announced (layer 2 starts on it)
+          tc::tmem_st_wait();
+          tc::tc_fence_before();
+          tc::mbar_arrive(&bar->h1_part[slot][c]);
+        }
       }
-      tc::tmem_st_wait();
-      tc::tc_fence_before();
-      tc::mbar_arrive(&bar->h1_full[slot]);
+      if constexpr (!(G == 1 && MODE == kRollout)) {
+        tc::tmem_st_wait();
+        tc::tc_fence_before();
+        tc::mbar_arrive(&bar->h1_full[slot]);
+      }
       float2 vsum = make_float2(0.0f, 0.0f);   // value head: even and odd columns
       const float* w3v = reinterpret_cast<const float*>(smem + kOffW3V);
       for (int c = 0; c < kNChunks; ++c) {       // layer 2 (Y / Z)
