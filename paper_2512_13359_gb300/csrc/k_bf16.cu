@@ -344,7 +344,16 @@ struct Engine {
   static constexpr uint32_t kHistBytes = kHistSmem ? 6u * paper::kHist * kRows * 4u : 0u;
   static constexpr uint32_t kSmem = kOffHist + kHistBytes + 1024;   // + alignment slack
   static_assert(kSmem <= 227u * 1024u, "shared memory per CTA");
-  static constexpr int kThreads = G * kRows + 96;
+  // One group per CTA in the rollout: a second warpgroup (warps 4-7, the
+  // same tensor-memory lanes) takes the second 32-column half of every
+  // epilogue chunk, so each sub-partition runs two epilogue warps.
+  // With one group a single h1 slot suffices (layer 1 of the next step waits
+  // for this step's physics anyway): h1 stays in slot 0, and layer 1's
+  // chunks 0 and 1 accumulate in slot 1's columns, so the two warpgroups'
+  // packed halves never overwrite accumulator columns the other still reads.
+  static constexpr bool kSplit = MODE == kRollout && G == 1;
+  static constexpr int kGroupWarps = kSplit ? 8 : 4 * G;
+  static constexpr int kThreads = kGroupWarps * 32 + 96;
 };
 
 // Row r of the observation tile (bf16, K = 32, 64-byte swizzle): 4 pieces of
@@ -443,7 +452,7 @@ __device__ __forceinline__ int step_index(int it, int g, const int (&iters)[G]) 
 // SIM selects the environment model of the fused rollout (0: Fossen,
 // 1: the paper model); the row modes ignore it.
 template <int G, int MODE, int SIM>
-__global__ void __launch_bounds__(G * 128 + 96) __maxnreg__(G == 4 ? 96 : 168)
+__global__ void __launch_bounds__(Engine<G, MODE>::kThreads) __maxnreg__(G == 4 ? 96 : 168)
 k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
          uint64_t t_g0, RowIO io, Status* st) {
   using E = Engine<G, MODE>;
@@ -455,7 +464,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
   volatile int* abort = &bar->abort;
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
-  const bool is_mma_warp = warp >= 4 * G;
+  constexpr int kGW = E::kGroupWarps;   // MMA-issuing warps: kGW (layer 2), kGW + 1, kGW + 2
+  const bool is_mma_warp = warp >= kGW;
 
   // ---- set-up: barriers, weights, tensor memory ----
   if (tid == 0) {
@@ -468,13 +478,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       tc::mbar_init(&bar->full_z[g], 1);
       tc::mbar_init(&bar->acc3_full[g], 1);
     }
-    tc::mbar_init(&bar->empty_x, kRows);
-    tc::mbar_init(&bar->empty_y, kRows);
-    tc::mbar_init(&bar->empty_z, kRows);
+    // epilogue arrivals: 128, or 256 with the split warpgroups
+    constexpr uint32_t kEpi = kRows * (E::kSplit ? 2 : 1);
+    tc::mbar_init(&bar->empty_x, kEpi);
+    tc::mbar_init(&bar->empty_y, kEpi);
+    tc::mbar_init(&bar->empty_z, kEpi);
     for (int s = 0; s < 2; ++s) {
-      tc::mbar_init(&bar->h1_full[s], kRows);
-      for (int c = 0; c < kNChunks; ++c) tc::mbar_init(&bar->h1_part[s][c], kRows);
-      tc::mbar_init(&bar->h2_full[s], kRows);
+      tc::mbar_init(&bar->h1_full[s], kEpi);
+      for (int c = 0; c < kNChunks; ++c) tc::mbar_init(&bar->h1_part[s][c], kEpi);
+      tc::mbar_init(&bar->h2_full[s], kEpi);
       tc::mbar_init(&bar->acc3_empty[s], kRows);
       tc::mbar_init(&bar->h1_free[s], 1);
       tc::mbar_init(&bar->h2_empty[s], 1);
@@ -494,7 +506,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       tc::bulk_g2s(smem + o, image + o, E::kImage - o < kPiece ? E::kImage - o : kPiece,
                    &bar->img_full);
   }
-  if (warp == 4 * G) {
+  if (warp == kGW) {
     tc::tmem_alloc(&bar->tmem_base, kTmemCols);
     tc::tmem_relinquish();
   }
@@ -560,11 +572,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       // 1 (accumulators Y and Z, both drained by then) are fed K-slice by
       // K-slice as h1's chunks are written (h1_part), not after all of h1.
       constexpr bool kProgL2 = G == 1 && MODE == kRollout;
-      if (warp == 4 * G) {
+      if (warp == kGW) {
         uint32_t u_y = 0, u_z = 0;
         uint32_t p_h1 = 0;   // phase bit of slot s at bit s
         auto issue_l2 = [&](int k, int g2, int c) -> bool {
-          const int s2 = k & 1;
+          const int s2 = E::kSplit ? 0 : k & 1;
           const bool odd = c & 1;
           uint32_t& u = odd ? u_z : u_y;
           const bool r = tc::mbar_wait(odd ? &bar->empty_z : &bar->empty_y, (u & 1u) ^ 1u, abort,
@@ -585,7 +597,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           return true;
         };
         for (int k = 0; k < total && ok; ++k) {
-          const int s2 = k & 1;
+          const int s2 = E::kSplit ? 0 : k & 1;
           if constexpr (kProgL2) {
             // chunks 0 and 1 (Y, Z) K-slice by K-slice as h1's chunks land
             ok = tc::mbar_wait(&bar->empty_y, (u_y & 1u) ^ 1u, abort, kWaitLimitNs) &&
@@ -621,7 +633,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           }
           advance(it, g);
         }
-      } else if (warp == 4 * G + 2) {
+      } else if (warp == kGW + 2) {
         // layer 3: A = h2 buffer (c & 1), B = W3 K-slice c, into head slot k & 1
         uint32_t p_h2 = 0, p_a3 = 0;   // phase bit of buffer / slot s at bit s
         for (int k = 0; k < total && ok && kPolicy; ++k) {
@@ -648,7 +660,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
       } else {
         uint32_t u_x = 0, p_hf = 0, p_obs = 0;   // phase bits per slot / group
         for (int k = 0; k < total && ok; ++k) {
-          const int s1 = k & 1;
+          const int s1 = E::kSplit ? 0 : k & 1;
           ok = tc::mbar_wait(&bar->h1_free[s1], ((p_hf >> s1) & 1u) ^ 1u, abort, kWaitLimitNs);
           p_hf ^= 1u << s1;
           if (!ok) break;
@@ -660,7 +672,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           // it has read the accumulator), chunks 2 and 3 in X.  So three
           // chunks start at once and only chunk 3 waits for X to drain.
           for (int c = 0; c < kNChunks && ok; ++c) {
-            uint32_t d = tmem + kColH1 + s1 * 128 + c * kChunk;
+            uint32_t d = tmem + kColH1 + (E::kSplit ? 128 : s1 * 128) + c * kChunk;
             if (c >= 2) {
               ok = tc::mbar_wait(&bar->empty_x, (u_x & 1u) ^ 1u, abort, kWaitLimitNs);
               ++u_x;
@@ -678,15 +690,20 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         }
       }
       // drain: every MMA this thread issued has completed before tensor memory is freed
-      uint64_t* drain = warp == 4 * G ? &bar->drain : (warp == 4 * G + 1 ? &bar->drain1 : &bar->drain2);
+      uint64_t* drain = warp == kGW ? &bar->drain : (warp == kGW + 1 ? &bar->drain1 : &bar->drain2);
       tc::mma_commit(drain);
       tc::mbar_wait(drain, 0, abort, kWaitLimitNs);
     }
     __syncwarp();
   } else {
     // =================== groups: epilogues + physics / row I/O ===================
-    const int g = warp >> 2;
+    const int g = E::kSplit ? 0 : warp >> 2;
     const int row = tid & (kRows - 1);
+    // split epilogues: warps 0-3 take the first 32 columns of every chunk
+    // (and the head, sampling and physics), warps 4-7 the second
+    const bool helper = E::kSplit && warp >= 4;
+    const int half_lo = E::kSplit ? (helper ? 1 : 0) : 0;
+    const int half_hi = E::kSplit ? half_lo + 1 : 2;
     const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     uint8_t* obs_tile = smem + E::kOffObs + g * kObsTileBytes;
     uint8_t* h2_tiles = smem + E::kOffH2;
@@ -702,7 +719,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     // h1r / h2r set, the row's bf16 hidden activations are stored there too.
     auto run_network = [&](int k, int it, float* head, uint16_t* h1r, uint16_t* h2r,
                            const uint16_t* a1r, const uint16_t* a2r) -> bool {
-      const int slot = k & 1;
+      const int slot = E::kSplit ? 0 : k & 1;
       // Backward with at most two groups (registers to spare): the forward
       // activations tanh' needs are loaded one chunk ahead of their use, so
       // that their memory latency overlaps the tensor-core work instead of
@@ -728,13 +745,15 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         if (!tc::mbar_wait(full, c < 2 ? (uint32_t)it & 1u : (uint32_t)c & 1u, abort, kWaitLimitNs))
           return false;
         tc::tc_fence_after();
-        const uint32_t src = c < 2 ? kColH1 + slot * 128 + c * kChunk : kColX;
+        const uint32_t src =
+            c < 2 ? kColH1 + (E::kSplit ? 128 : slot * 128) + c * kChunk : kColX;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
+          if (E::kSplit && (half < half_lo || half >= half_hi)) continue;
           uint32_t acc[32], hv[16];
           tc::tmem_ld32(lane_addr + src + 32 * half, acc);
           tc::tmem_ld_wait(acc);
-          if (half == 1 && c >= 2) {
+          if ((E::kSplit || half == 1) && c >= 2) {
             tc::tc_fence_before();
             tc::mbar_arrive(&bar->empty_x);
           }
@@ -777,10 +796,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         uint8_t* h2 = h2_tiles + (c & 1) * kH2TileBytes + row * 128;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
+          if (E::kSplit && (half < half_lo || half >= half_hi)) continue;
           uint32_t acc[32], hv[16];
           tc::tmem_ld32(lane_addr + col + 32 * half, acc);
           tc::tmem_ld_wait(acc);
-          if (half == 1) {
+          if (E::kSplit || half == 1) {
             tc::tc_fence_before();
             tc::mbar_arrive(odd ? &bar->empty_z : &bar->empty_y);
           }
@@ -802,7 +822,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             // Write j = 2k + (c >> 1) of h2 buffer c & 1 reuses it after
             // layer 3 has consumed write j - 1 (completion j - 1 of h2_empty).
             const int j = 2 * k + (c >> 1);
-            if (half == 0 && j > 0 &&
+            if ((E::kSplit || half == 0) && j > 0 &&
                 !tc::mbar_wait(&bar->h2_empty[c & 1], (uint32_t)(j - 1) & 1u, abort, kWaitLimitNs))
               return false;
 #pragma unroll
@@ -833,13 +853,16 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
         head[0] = (vsum.x + vsum.y) + *reinterpret_cast<const float*>(smem + kOffB3V);
         return true;
       }
+      if (helper) return true;   // the head belongs to the first warpgroup
       if (!tc::mbar_wait(&bar->acc3_full[g], (uint32_t)it & 1u, abort, kWaitLimitNs)) return false;
       tc::tc_fence_after();
       uint32_t o3[16];
-      tc::tmem_ld16(lane_addr + kColA3 + slot * 16, o3);
+      // head slot: by group-step parity (layer 3 alternates), also with one
+      // h1 slot
+      tc::tmem_ld16(lane_addr + kColA3 + (k & 1) * 16, o3);
       tc::tmem_ld_wait(o3);
       tc::tc_fence_before();
-      tc::mbar_arrive(&bar->acc3_empty[slot]);
+      tc::mbar_arrive(&bar->acc3_empty[k & 1]);
       const float* b3 = reinterpret_cast<const float*>(smem + kOffB3P);
 #pragma unroll
       for (int j = 0; j < kHeadOut; ++j) head[j] = __uint_as_float(o3[j]) + b3[j];
@@ -849,7 +872,13 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     int my_iters = 0;
 #pragma unroll
     for (int j = 0; j < G; ++j) my_iters = j == g ? iters[j] : my_iters;
-    if constexpr (MODE == kRollout && SIM == 0) {
+    if (helper) {
+      // the second epilogue warpgroup: the networks only, one item per step
+      for (int t = 0; t < my_iters && ok; ++t) {
+        float head[kHeadOut];
+        ok = run_network(t, t, head, nullptr, nullptr, nullptr, nullptr);
+      }
+    } else if constexpr (MODE == kRollout && SIM == 0) {
       int n_act = 0;
 #pragma unroll
       for (int j = 0; j < G; ++j) n_act += iters[j] > 0 ? 1 : 0;
@@ -1103,7 +1132,7 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     atomicAdd(&st->timeouts, 1);
     atomicCAS(&st->code, 0, -4);
   }
-  if (warp == 4 * G) {
+  if (warp == kGW) {
     tc::tc_fence_after();
     tc::tmem_dealloc(tmem, kTmemCols);
   }
