@@ -214,6 +214,7 @@ struct Barriers {
   uint64_t empty_x, empty_y, empty_z;   // accumulator read back (128 arrivals)
   uint64_t h1_full[2];      // h1 slot complete (128 arrivals)
   uint64_t h1_part[2][4];   // one group per CTA: h1 chunk c of slot s written (128 arrivals)
+  uint64_t h2_part[4];      // one group per CTA: h2 chunk c in tensor memory (both warpgroups)
   uint64_t h2_full[2];      // h2 buffer written (128 arrivals)
   uint64_t acc3_empty[2];   // head slot read back (128 arrivals)
   uint64_t h1_free[2];      // layer-2 MMAs reading an h1 slot completed (commit)
@@ -486,6 +487,8 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
     for (int s = 0; s < 2; ++s) {
       tc::mbar_init(&bar->h1_full[s], kEpi);
       for (int c = 0; c < kNChunks; ++c) tc::mbar_init(&bar->h1_part[s][c], kEpi);
+      if (s == 0)
+        for (int c = 0; c < kNChunks; ++c) tc::mbar_init(&bar->h2_part[c], kEpi);
       tc::mbar_init(&bar->h2_full[s], kEpi);
       tc::mbar_init(&bar->acc3_empty[s], kRows);
       tc::mbar_init(&bar->h1_free[s], 1);
@@ -641,6 +644,20 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           ok = tc::mbar_wait(&bar->acc3_empty[s2], ((p_a3 >> s2) & 1u) ^ 1u, abort, kWaitLimitNs);
           p_a3 ^= 1u << s2;
           for (int c = 0; c < kNChunks && ok; ++c) {
+            if constexpr (E::kSplit) {
+              // h2 chunk c in tensor memory (columns 128 + 32c.., packed bf16)
+              ok = tc::mbar_wait(&bar->h2_part[c], (uint32_t)k & 1u, abort, kWaitLimitNs);
+              if (!ok) break;
+              tc::tc_fence_after();
+              const uint32_t a0 = tmem + kColH1 + 128 + c * 32;
+              const uint64_t b0 = tc::smem_desc(s_base + kOffW3 + c * (kHeadOut * 128), 1024, 2);
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc::mma_ts(tmem + kColA3 + s2 * 16, a0 + kk * 8, b0 + (uint64_t)(kk * 2), kI16,
+                           (c > 0 || kk > 0) ? 1u : 0u);
+              if (c == kNChunks - 1) tc::mma_commit(&bar->acc3_full[g]);
+              continue;
+            }
             const int hb = c & 1;
             ok = tc::mbar_wait(&bar->h2_full[hb], (p_h2 >> hb) & 1u, abort, kWaitLimitNs);
             p_h2 ^= 1u << hb;
@@ -818,11 +835,16 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
           if (E::kLearn && h2r) store_bf16x32(h2r + c * kChunk + 32 * half, hv, wide);
           if constexpr (E::kBack) {
             // backward: dL/dZ1 goes to global memory only
+          } else if (E::kSplit) {
+            // one group: h2 stays in tensor memory (columns 128..255, free
+            // once layer 1's epilogue has read its accumulators) as layer 3's
+            // A operand
+            tc::tmem_st16(lane_addr + kColH1 + 128 + c * 32 + half * 16, hv);
           } else if (kPolicy) {
             // Write j = 2k + (c >> 1) of h2 buffer c & 1 reuses it after
             // layer 3 has consumed write j - 1 (completion j - 1 of h2_empty).
             const int j = 2 * k + (c >> 1);
-            if ((E::kSplit || half == 0) && j > 0 &&
+            if (half == 0 && j > 0 &&
                 !tc::mbar_wait(&bar->h2_empty[c & 1], (uint32_t)(j - 1) & 1u, abort, kWaitLimitNs))
               return false;
 #pragma unroll
@@ -843,7 +865,11 @@ k_engine(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, i
             }
           }
         }
-        if (kPolicy) {
+        if constexpr (E::kSplit) {
+          tc::tmem_st_wait();
+          tc::tc_fence_before();
+          tc::mbar_arrive(&bar->h2_part[c]);
+        } else if (kPolicy) {
           tc::fence_async_smem();
           tc::mbar_arrive(&bar->h2_full[c & 1]);
         }
