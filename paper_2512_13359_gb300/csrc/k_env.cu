@@ -148,6 +148,123 @@ __global__ void __launch_bounds__(kTile) k_rollout_fp32(const Model M, Buffers B
   store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
 }
 
+// Small batches (tens to a few thousand envs): the one-thread-per-env kernel
+// above leaves each env's network as one thread's serial chain on a handful
+// of SMs.  Here a team of H threads evaluates each env's networks, thread j
+// computing hidden unit j of both layers and output j of the head, each sum
+// in mlp_fp32's order (the same floats); the team's first thread holds the
+// env's state and runs the sampling and the physics.  H = 64, four envs per
+// 256-thread CTA.
+template <int H, int OUT>
+__global__ void __launch_bounds__(256) k_rollout_fp32_team(const Model M, Buffers B,
+                                                           const float* __restrict__ wp,
+                                                           const float* __restrict__ wv, Traj tr,
+                                                           int T, uint64_t t_g0, Status* st) {
+  static_assert(H >= OUT && 256 % H == 0, "team shape");
+  constexpr int E = 256 / H;
+  __shared__ float s_x[E][kObs];
+  __shared__ float s_h1[E][H];
+  __shared__ float s_h2[E][H];
+  __shared__ float s_out[E][OUT + 1];   // policy head, then the value
+  const int el = threadIdx.x / H, j = threadIdx.x % H;
+  const int i = blockIdx.x * E + el;
+  const bool active = i < M.n, lead = j == 0;
+  const size_t n = (size_t)M.n;
+  // hidden unit j of layer 1 / layer 2 and output o of the head of one
+  // network (row-major weights, mlp_fp32's layout and summation order)
+  auto unit1 = [&](const float* w, int u) {
+    const float* W1 = w;
+    const float* b1 = W1 + H * kObs;
+    float s = __ldg(b1 + u);
+    const float2* row = reinterpret_cast<const float2*>(W1 + u * kObs);
+#pragma unroll
+    for (int i2 = 0; i2 < kObs / 2; ++i2) {
+      const float2 wv2 = __ldg(row + i2);
+      s = fmaf(wv2.x, s_x[el][2 * i2], s);
+      s = fmaf(wv2.y, s_x[el][2 * i2 + 1], s);
+    }
+    s_h1[el][u] = tanhf(s);
+  };
+  auto unit2 = [&](const float* w, int u) {
+    const float* W2 = w + H * kObs + H;
+    const float* b2 = W2 + H * H;
+    float s0 = __ldg(b2 + u), s1 = 0.0f;
+    const float4* row = reinterpret_cast<const float4*>(W2 + (size_t)u * H);
+#pragma unroll 8
+    for (int k4 = 0; k4 < H / 4; ++k4) {
+      const float4 q = __ldg(row + k4);
+      s0 = fmaf(q.x, s_h1[el][4 * k4 + 0], s0);
+      s1 = fmaf(q.y, s_h1[el][4 * k4 + 1], s1);
+      s0 = fmaf(q.z, s_h1[el][4 * k4 + 2], s0);
+      s1 = fmaf(q.w, s_h1[el][4 * k4 + 3], s1);
+    }
+    s_h2[el][u] = tanhf(s0 + s1);
+  };
+  auto head = [&](const float* w, int out_dim, int o) {
+    const float* W3 = w + H * kObs + H + H * H + H;
+    const float* b3 = W3 + out_dim * H;
+    float s = __ldg(b3 + o);
+    for (int u = 0; u < H; ++u) s = fmaf(__ldg(W3 + o * H + u), s_h2[el][u], s);
+    return s;
+  };
+  Env e;
+  if (lead && active) load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  bool bad = false;
+  for (int t = 0; t < T; ++t) {
+    if (lead) {
+      float o[kObs];
+      if (active) {
+        observe(e, o);
+        if (tr.obs) {
+#pragma unroll
+          for (int k = 0; k < kObs; ++k) tr.obs[((size_t)t * kObs + k) * n + i] = o[k];
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < kObs; ++k) o[k] = 0.0f;
+      }
+#pragma unroll
+      for (int k = 0; k < kObs; ++k) s_x[el][k] = o[k];
+    }
+    __syncthreads();
+    unit1(wp, j);
+    __syncthreads();
+    unit2(wp, j);
+    __syncthreads();
+    if (j < OUT) s_out[el][j] = head(wp, OUT, j);
+    if (tr.value) unit1(wv, j);       // the value network's layer 1 (s_h1 is free)
+    __syncthreads();
+    if (tr.value) {
+      unit2(wv, j);
+      __syncthreads();
+      if (j == 0) s_out[el][OUT] = head(wv, 1, 0);
+      __syncthreads();
+    }
+    if (lead && active) {
+      float hd[OUT];
+#pragma unroll
+      for (int k = 0; k < OUT; ++k) hd[k] = s_out[el][k];
+      float a[kAct], lp;
+      sample_action(M, M.id_base + (uint32_t)i, t_g0 + (uint64_t)t, hd, a, &lp);
+      if (tr.value) tr.value[(size_t)t * n + i] = s_out[el][OUT];
+      if (tr.act) {
+#pragma unroll
+        for (int k = 0; k < kAct; ++k) tr.act[((size_t)t * kAct + k) * n + i] = a[k];
+      }
+      if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
+      bool d;
+      const float r = physics_step(M, M.id_base + (uint32_t)i, e, a, &d);
+      if (tr.rew) tr.rew[(size_t)t * n + i] = r;
+      if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
+      bad |= !env_finite(e);
+    }
+  }
+  if (lead && active) {
+    if (bad) flag_nan(st, i);
+    store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+  }
+}
+
 template <int IN, int H, int OUT>
 __global__ void __launch_bounds__(kTile) k_forward_fp32(const float* __restrict__ wp,
                                                         const float* __restrict__ wv,
@@ -218,10 +335,20 @@ cudaError_t launch_draw_words(const Model& M, uint32_t stream_id, uint64_t index
   return cudaGetLastError();
 }
 
+// Batches at most this large run the team kernel (hidden width 64).
+constexpr int kTeamMaxEnvs = 2048;
+
 template <int H, int OUT>
 static cudaError_t rollout_fp32_impl(const Model& M, const Buffers& B, const float* wp,
                                      const float* wv, const Traj& tr, int T, uint64_t t_g0,
                                      Status* st, cudaStream_t s) {
+  if constexpr (H == 64) {
+    if (M.n <= kTeamMaxEnvs) {
+      k_rollout_fp32_team<H, OUT><<<blocks_for(M.n, 256 / H), 256, 0, s>>>(M, B, wp, wv, tr, T,
+                                                                           t_g0, st);
+      return cudaGetLastError();
+    }
+  }
   const size_t smem = (size_t)H * kTile * sizeof(float);
   cudaError_t err = cudaFuncSetAttribute(k_rollout_fp32<H, OUT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
