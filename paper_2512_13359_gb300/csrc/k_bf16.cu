@@ -25,6 +25,13 @@
 // Tensor-memory columns: h1 slots 0..127 and 128..255 (bf16 pairs), layer-1
 // accumulator X 256..319, layer-2 accumulators Y 320..383 and Z 384..447,
 // head accumulators 448..463 and 464..479.
+//
+// One group per CTA (the rollout with fewer tiles than SMs) differs: a
+// second warpgroup takes the second 32-column half of every epilogue chunk;
+// h1 stays in slot 0 while layer 1's chunks 0 and 1 accumulate in slot 1's
+// columns, which then hold h2 (packed, layer 3's A operand from tensor
+// memory); layer 2's chunks 0 and 1 start K-slice by K-slice as h1 is
+// written.
 #include <atomic>
 #include <climits>
 
