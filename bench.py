@@ -552,7 +552,7 @@ def run_gae(args):
 # profiles/k_engine_ppo_65536_T128_dram.md), valid while the engine's sources
 # hash to ENGINE_SRC_HASH.
 ROLLOUT_TRAFFIC_65536x128 = 10_622_976 + 900_608_256
-ENGINE_SRC_HASH = "c913bc987e9eca3a"
+ENGINE_SRC_HASH = "ce6892845323d80d"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 

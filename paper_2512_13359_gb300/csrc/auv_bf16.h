@@ -66,6 +66,9 @@ cudaError_t launch_forward_bf16(const Model& M, const void* wp_packed, const voi
                                 const float* wv_f32, const float* obs, int n, float* head,
                                 float* value, Status* st, cudaStream_t s);
 
+// SM count of the current device (looked up once per device).
+int engine_sm_count();
+
 // Failure-detection self-test (a bounded wait that is made to run out).
 cudaError_t launch_wait_selftest(Status* st, uint64_t limit_ns, cudaStream_t s);
 

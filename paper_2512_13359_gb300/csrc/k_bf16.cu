@@ -1251,6 +1251,8 @@ cudaError_t launch_wait_selftest(Status* st, uint64_t limit_ns, cudaStream_t s) 
   return cudaGetLastError();
 }
 
+int engine_sm_count() { return sm_count(); }
+
 size_t bf16_policy_image_bytes() { return kPolicyImage; }
 size_t bf16_value_image_bytes() { return kValueImage; }
 size_t bf16_back_image_bytes() { return kBackImage; }

@@ -27,6 +27,7 @@
 // Every wait is an mbarrier wait bounded by 2 s; a timeout raises the CTA's
 // abort flag and latches AUV_ERR_TIMEOUT in the status block.
 #include "auv_kernels.h"
+#include "auv_bf16.h"
 #include "tc_ptx.cuh"
 
 namespace auv {
@@ -394,6 +395,254 @@ k_rollout_tf32(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj
   }
 }
 
+// ---------------------------------------------------------------------------
+// Small batches (at most one tile per two SMs): a cluster of two CTAs per
+// tile.  Both CTAs hold W1, W3 and the biases, and each holds its half of W2
+// (rows 128r..128r+127 of every K-slice: 128 KB, resident, no streaming).
+// Both compute the observation, layer 1 and h1 for the same 128 envs; CTA r
+// then computes columns 128r..128r+127 of layer 2, their epilogue and the
+// partial head over them (K-slices 4r..4r+3 of W3), and the two partial
+// heads are exchanged through distributed shared memory and summed in rank
+// order, so both CTAs hold the same head and run the same sampling and
+// physics (identical state); CTA 0 writes the trajectory.  A control step is
+// one tile's serial chain either way; this halves its layer 2 and its
+// layer-2 epilogue.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kPHalf = kSliceBytes / 2;              // one K-slice, 128 rows
+constexpr uint32_t kPSObs = kSObs;
+constexpr uint32_t kPSW2 = kPSObs + kRows * 128;          // 8 half K-slices of W2
+constexpr uint32_t kPSX = kPSW2 + kSlices * kPHalf;       // exchange: [2][128][16] fp32
+constexpr uint32_t kPSBar = kPSX + 2 * kRows * 16 * 4;
+
+struct PairBars {
+  uint64_t img_full, obs_full, l1_full, l2_full, l3_full, drain;
+  uint64_t h1_part[kSlices];   // h1 chunk j written (128 arrivals)
+  uint64_t h2_part[4];         // h2 chunk j of this CTA's half written (128 arrivals)
+  uint64_t xch_full[2];        // the other CTA's partial head in exchange slot s (128 arrivals)
+  uint32_t tmem_base;
+  int abort;
+};
+constexpr uint32_t kPSmem = kPSBar + sizeof(PairBars) + 1024;
+static_assert(kPSmem <= 227u * 1024u, "shared memory per CTA");
+constexpr uint32_t kColHalf = 256;   // this CTA's 128 columns of layer 2, then h2
+constexpr uint32_t kColPart = 384;   // partial head (16 columns)
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(160, 1)
+k_rollout_tf32_pair(const Model M, Buffers B, const uint8_t* __restrict__ image, Traj tr, int T,
+                    uint64_t t_g0, Status* st) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023u) & ~(uintptr_t)1023u);
+  PairBars* bar = reinterpret_cast<PairBars*>(smem + kPSBar);
+  volatile int* abort = &bar->abort;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const uint32_t rank = tc::cluster_rank(), peer = rank ^ 1u;
+
+  if (tid == 0) {
+    tc::mbar_init(&bar->img_full, 1);
+    tc::mbar_init(&bar->obs_full, kRows);
+    tc::mbar_init(&bar->l1_full, 1);
+    tc::mbar_init(&bar->l2_full, 1);
+    tc::mbar_init(&bar->l3_full, 1);
+    tc::mbar_init(&bar->drain, 1);
+    for (int j = 0; j < kSlices; ++j) tc::mbar_init(&bar->h1_part[j], kRows);
+    for (int j = 0; j < 4; ++j) tc::mbar_init(&bar->h2_part[j], kRows);
+    tc::mbar_init(&bar->xch_full[0], kRows);
+    tc::mbar_init(&bar->xch_full[1], kRows);
+    bar->abort = 0;
+    tc::mbar_fence_init();
+    tc::mbar_arrive_expect_tx(&bar->img_full, kH * 128 + kSlices * kW3Slice + (2 * kH + 16) * 4 +
+                                                  kSlices * kPHalf);
+    tc::bulk_g2s(smem + kSW1, image + kOffW1, kH * 128, &bar->img_full);
+    tc::bulk_g2s(smem + kSW3, image + kOffW3, kSlices * kW3Slice, &bar->img_full);
+    tc::bulk_g2s(smem + kSB, image + kOffB, (2 * kH + 16) * 4, &bar->img_full);
+    for (int j = 0; j < kSlices; ++j)
+      tc::bulk_g2s(smem + kPSW2 + j * kPHalf, image + kOffW2 + j * kSliceBytes + rank * kPHalf,
+                   kPHalf, &bar->img_full);
+  }
+  if (warp == 4) {
+    tc::tmem_alloc(&bar->tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::tc_fence_before();
+  // both CTAs' barriers exist before either arrives on the other's
+  tc::cluster_sync();
+  tc::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+  const uint32_t s_base = tc::smem_u32(smem);
+  const bool img_ok = tc::mbar_wait(&bar->img_full, 0, abort, kWaitLimitNs);
+  const int steps = img_ok ? T : 0;
+
+  if (warp == 4) {
+    // ---- MMA issue ----
+    if ((tid & 31) == 0) {
+      constexpr uint32_t kI256 = idesc_tf32(128, 256);
+      constexpr uint32_t kI128 = idesc_tf32(128, 128);
+      constexpr uint32_t kI16 = idesc_tf32(128, 16);
+      bool ok = true;
+      for (int t = 0; t < steps && ok; ++t) {
+        const uint32_t ph = (uint32_t)t & 1u;
+        if (!(ok = tc::mbar_wait(&bar->obs_full, ph, abort, kWaitLimitNs))) break;
+        tc::tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < 3; ++kk)   // K = 24 covers the 18 observation columns
+          mma_ss(tmem, desc(s_base + kPSObs + kk * 32), desc(s_base + kSW1 + kk * 32), kI256,
+                 kk > 0 ? 1u : 0u);
+        tc::mma_commit(&bar->l1_full);
+        // this CTA's half of layer 2, K-slice by K-slice as h1's chunks land
+        for (int j = 0; j < kSlices && ok; ++j) {
+          if (!(ok = tc::mbar_wait(&bar->h1_part[j], ph, abort, kWaitLimitNs))) break;
+          tc::tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_ts(tmem + kColHalf, tmem + 32 * j + 8 * kk,
+                   desc(s_base + kPSW2 + j * kPHalf + kk * 32), kI128, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (!ok) break;
+        tc::mma_commit(&bar->l2_full);
+        // the partial head over this half's h2 chunks (W3 K-slices 4r + j)
+        for (int j = 0; j < 4 && ok; ++j) {
+          if (!(ok = tc::mbar_wait(&bar->h2_part[j], ph, abort, kWaitLimitNs))) break;
+          tc::tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_ts(tmem + kColPart, tmem + kColHalf + 32 * j + 8 * kk,
+                   desc(s_base + kSW3 + (4 * rank + j) * kW3Slice + kk * 32), kI16,
+                   (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (!ok) break;
+        tc::mma_commit(&bar->l3_full);
+      }
+      tc::mma_commit(&bar->drain);
+      tc::mbar_wait(&bar->drain, 0, abort, kWaitLimitNs);
+    }
+    __syncwarp();
+  } else {
+    // ---- env threads (both CTAs; CTA 0 writes the trajectory) ----
+    const int row = tid;
+    const int i = (int)(blockIdx.x >> 1) * kRows + row;
+    const bool active = i < M.n, writer = rank == 0;
+    const size_t n = (size_t)M.n;
+    const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
+    const float* bias = reinterpret_cast<const float*>(smem + kSB);
+    uint8_t* obs_tile = smem + kPSObs;
+    float* xch = reinterpret_cast<float*>(smem + kPSX);
+    Env e;
+    if (active) load_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+    bool bad = false, ok = true;
+    for (int t = 0; t < steps && ok; ++t) {
+      const uint32_t ph = (uint32_t)t & 1u;
+      float o[kObs];
+      if (active) {
+        observe(e, o);
+        if (writer && tr.obs) {
+#pragma unroll
+          for (int k = 0; k < kObs; ++k) tr.obs[((size_t)t * kObs + k) * n + i] = o[k];
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < kObs; ++k) o[k] = 0.0f;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 v;
+        v.x = 4 * q + 0 < kObs ? to_tf32(o[4 * q + 0]) : 0.0f;
+        v.y = 4 * q + 1 < kObs ? to_tf32(o[4 * q + 1]) : 0.0f;
+        v.z = 4 * q + 2 < kObs ? to_tf32(o[4 * q + 2]) : 0.0f;
+        v.w = 4 * q + 3 < kObs ? to_tf32(o[4 * q + 3]) : 0.0f;
+        *reinterpret_cast<float4*>(obs_tile + row * 128 + ((q ^ (row & 7)) << 4)) = v;
+      }
+      tc::fence_async_smem();
+      tc::mbar_arrive(&bar->obs_full);
+      __syncwarp();
+      if (!(ok = tc::mbar_wait(&bar->l1_full, ph, abort, kWaitLimitNs))) break;
+      tc::tc_fence_after();
+      hidden_epilogue(lane_addr, 0, bias, bar->h1_part);
+      const uint32_t id = M.id_base + (uint32_t)i;
+      float eps[kAct];
+      if (active) action_noise(id, M.seed, t_g0 + (uint64_t)t, eps);
+      if (!(ok = tc::mbar_wait(&bar->l2_full, ph, abort, kWaitLimitNs))) break;
+      tc::tc_fence_after();
+      // this CTA's 128 columns of h2: four chunks, each announced to layer 3
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t acc[32];
+        const float* b2 = bias + kH + 128 * rank + 32 * c;
+        tc::tmem_ld32(lane_addr + kColHalf + 32 * c, acc);
+        tc::tmem_ld_wait(acc);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          acc[j] = __float_as_uint(to_tf32(tc::tanh_f32(__uint_as_float(acc[j]) + b2[j])));
+        tmem_st32(lane_addr + kColHalf + 32 * c, acc);
+        tc::tmem_st_wait();
+        tc::tc_fence_before();
+        tc::mbar_arrive(&bar->h2_part[c]);
+      }
+      if (!(ok = tc::mbar_wait(&bar->l3_full, ph, abort, kWaitLimitNs))) break;
+      tc::tc_fence_after();
+      uint32_t p3[16];
+      tc::tmem_ld16(lane_addr + kColPart, p3);
+      tc::tmem_ld_wait(p3);
+      tc::tc_fence_before();
+      // the partial head to the other CTA's exchange slot t & 1, then its
+      // arrival there; then the other CTA's partial from this CTA's slot
+      const uint32_t slot = (uint32_t)t & 1u;
+      const uint32_t xoff = tc::smem_u32(xch + (slot * kRows + row) * 16);
+      const uint32_t xrem = tc::mapa(xoff, peer);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        tc::st_cluster_v4(xrem + 16 * q, __uint_as_float(p3[4 * q]), __uint_as_float(p3[4 * q + 1]),
+                          __uint_as_float(p3[4 * q + 2]), __uint_as_float(p3[4 * q + 3]));
+      tc::mbar_arrive_cluster(tc::mapa(tc::smem_u32(&bar->xch_full[slot]), peer));
+      if (!(ok = tc::mbar_wait_cluster(&bar->xch_full[slot], ((uint32_t)t >> 1) & 1u, abort,
+                                       kWaitLimitNs)))
+        break;
+      __syncwarp();
+      if (active) {
+        const float* other = xch + (slot * kRows + row) * 16;
+        float head[16];
+        // CTA 0's partial plus CTA 1's (the same sum in both CTAs), + b3
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          head[k] = (__uint_as_float(p3[k]) + other[k]) + bias[2 * kH + k];
+        float a[kAct], lp;
+        sample(M, head, eps, a, &lp);
+        if (writer) {
+          if (tr.act) {
+#pragma unroll
+            for (int k = 0; k < kAct; ++k) tr.act[((size_t)t * kAct + k) * n + i] = a[k];
+          }
+          if (tr.logp) tr.logp[(size_t)t * n + i] = lp;
+        }
+        bool d;
+        const float r = physics_step(M, id, e, a, &d);
+        if (writer) {
+          if (tr.rew) tr.rew[(size_t)t * n + i] = r;
+          if (tr.done) tr.done[(size_t)t * n + i] = d ? 1 : 0;
+        }
+        bad |= !env_finite(e);
+      }
+      __syncwarp();
+    }
+    if (active && writer) {
+      if (bad) flag_nan(st, i);
+      store_env(M, B.state, B.params, B.t_ep, B.episode, i, e);
+    }
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (tid == 0 && bar->abort) {
+    atomicAdd(&st->timeouts, 1);
+    atomicCAS(&st->code, 0, -4);
+  }
+  // neither CTA leaves while the other may still write into its shared memory
+  tc::cluster_sync();
+  if (warp == 4) {
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
 }  // namespace
 
 size_t tf32_policy_image_bytes() { return kImage; }
@@ -411,6 +660,15 @@ cudaError_t launch_rollout_tf32(const Model& M, const Buffers& B, const void* pa
                                        (int)kSmem);
   if (e != cudaSuccess) return e;
   const int grid = (M.n + kRows - 1) / kRows;
+  if (2 * grid <= engine_sm_count()) {
+    // at most one tile per two SMs: the two-CTA kernel
+    e = cudaFuncSetAttribute(k_rollout_tf32_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kPSmem);
+    if (e != cudaSuccess) return e;
+    k_rollout_tf32_pair<<<2 * grid, 160, kPSmem, s>>>(M, B, static_cast<const uint8_t*>(packed),
+                                                      tr, T, t_g0, st);
+    return cudaGetLastError();
+  }
   k_rollout_tf32<<<grid, 192, kSmem, s>>>(M, B, static_cast<const uint8_t*>(packed), tr, T, t_g0,
                                           st);
   return cudaGetLastError();
