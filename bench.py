@@ -76,7 +76,8 @@ def parse():
     ap.add_argument("--gae", action="store_true",
                     help="advantage estimation (env_gae) over one rollout, HBM roofline")
     ap.add_argument("--probes", action="store_true",
-                    help="roofline probes: FFMA chain, tanh.approx.f32 chain, cuBLAS tf32/bf16 GEMM")
+                    help="roofline probes: FFMA chain, tanh.approx.f32 and ex2.approx.f32 chains, "
+                         "cuBLAS tf32/bf16 GEMM, tcgen05 MMA cost per instruction by N")
     ap.add_argument("--sweep", action="store_true",
                     help="batch-size sweep 1,024 .. 1,048,576 envs x 256 steps (one line per size)")
     return ap.parse_args()
@@ -425,8 +426,10 @@ def run_replay(args):
 def run_probes(args):
     """The roofline denominators measured with the library's probes: the FP32
     pipe (FFMA chains at full occupancy) against 2 x 128 x SMs x clock, the
-    multi-function unit (tanh.approx.f32 chains), and the tensor pipe for
-    tf32 and bf16 operands (one 8192^3 cuBLAS GEMM each)."""
+    multi-function unit (tanh.approx.f32 and ex2.approx.f32 chains), the
+    tensor pipe for tf32 and bf16 operands (one 8192^3 cuBLAS GEMM each), and
+    the tensor pipe's cost per tcgen05 MMA instruction (M = 128, K = 16,
+    bf16) for each N the engine issues, one CTA per SM, in SM cycles."""
     import torch
     from paper_2512_13359_gb300 import auvenv, build
     build.build()
@@ -456,6 +459,21 @@ def run_probes(args):
         time.sleep(0.3)
     ffma = timed(lambda: auvenv.probe_ffma(blocks, threads, 20000, sink), max(args.steps, 5))
     tanh = timed(lambda: auvenv.probe_tanh(blocks, threads, 4000, sink), max(args.steps, 5))
+    ex2 = timed(lambda: auvenv.probe_ex2(blocks, threads, 4000, sink), max(args.steps, 5))
+    mma = {}
+    mma_iters = 1024
+    cyc = torch.zeros(sms, dtype=torch.int64, device="cuda")
+    for nn in (16, 32, 64, 128, 256):
+        for a_tmem in (False, True):
+            for _ in range(2):
+                auvenv.probe_mma(nn, a_tmem, mma_iters, cyc)
+            torch.cuda.synchronize()
+            c = cyc.cpu()
+            if int((c == 0).sum()):
+                raise RuntimeError("mma probe: a bounded wait gave up")
+            per = float(c.double().median()) / mma_iters
+            mma[f"n{nn}_{'ts' if a_tmem else 'ss'}"] = {
+                "cycles_per_mma": per, "mac_per_clk_per_sm": 128 * nn * 16 / per}
     n = 8192
     g = torch.Generator(device="cuda").manual_seed(0)
     a32 = torch.randn(n, n, device="cuda", generator=g)
@@ -476,6 +494,9 @@ def run_probes(args):
             "fp32_ffma_frac_of_derived": ffma / derived,
             "mufu_tanh_gops": tanh / 1e9,
             "mufu_tanh_per_clk_per_sm": tanh / (sms * mhz * 1e6),
+            "mufu_ex2_gops": ex2 / 1e9,
+            "mufu_ex2_per_clk_per_sm": ex2 / (sms * mhz * 1e6),
+            "tcgen05_mma_m128_k16_bf16": mma,
             "tf32_gemm_tflops": tf32 / 1e12, "bf16_gemm_tflops": bf16 / 1e12,
             "bf16_peak_measured_tflops": peaks.get("bf16_tflops"),
             "tf32_over_bf16": tf32 / bf16, "nominal_tf32_over_bf16": 1.1 / 2.25,

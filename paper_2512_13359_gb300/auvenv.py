@@ -50,7 +50,7 @@ EXPORTED = ("env_abi_version", "env_create", "env_destroy", "env_last_error", "e
             "ppo_get_weights", "ppo_get_state", "ppo_set_state", "ppo_grads", "ppo_apply",
             "ppo_update", "ppo_export_weights", "ppo_status", "ppo_clear_status",
             "auv_gemm", "auv_gemm_workspace_bytes",
-            "auv_probe_ffma", "auv_probe_tanh", "auv_probe_gemm")
+            "auv_probe_ffma", "auv_probe_tanh", "auv_probe_ex2", "auv_probe_mma", "auv_probe_gemm")
 
 
 class LibraryMissing(RuntimeError):
@@ -197,6 +197,8 @@ def lib(path: str | None = None):
     L.ppo_status.argtypes = [P, C.POINTER(AuvStatus), P]
     L.auv_probe_ffma.argtypes = [U32, U32, U32, P, P]
     L.auv_probe_tanh.argtypes = [U32, U32, U32, P, P]
+    L.auv_probe_ex2.argtypes = [U32, U32, U32, P, P]
+    L.auv_probe_mma.argtypes = [I, I, U32, U32, P, P]
     L.auv_probe_gemm.argtypes = [U32, I, P, P, P, P]
     L.auv_gemm_workspace_bytes.argtypes = [I, I, I]
     L.auv_gemm_workspace_bytes.restype = C.c_size_t
@@ -595,6 +597,19 @@ def probe_tanh(blocks: int, threads: int, iters: int, sink, stream=None) -> int:
     """Enqueue the tanh.approx.f32 probe; returns its operation count."""
     _probe_check(lib().auv_probe_tanh(blocks, threads, iters, _ptr(sink), _stream(stream)), "tanh probe")
     return 8 * blocks * threads * iters
+
+
+def probe_ex2(blocks: int, threads: int, iters: int, sink, stream=None) -> int:
+    """Enqueue the ex2.approx.ftz.f32 probe; returns its operation count."""
+    _probe_check(lib().auv_probe_ex2(blocks, threads, iters, _ptr(sink), _stream(stream)), "ex2 probe")
+    return 8 * blocks * threads * iters
+
+
+def probe_mma(n: int, a_tmem: bool, iters: int, cycles, stream=None) -> None:
+    """Enqueue the tcgen05 MMA probe on cycles.numel() CTAs (cycles: uint64
+    device tensor, one SM-cycle span per CTA, 0 where the wait gave up)."""
+    _probe_check(lib().auv_probe_mma(n, 1 if a_tmem else 0, iters, int(cycles.numel()), _ptr(cycles),
+                                     _stream(stream)), "mma probe")
 
 
 def probe_gemm(precision: str, a, b, c, stream=None) -> int:

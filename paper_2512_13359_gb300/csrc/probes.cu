@@ -1,8 +1,11 @@
 // probes.cu -- measurement probes for the roofline denominators: an FFMA
-// chain (the FP32 pipe), a tanh.approx.f32 chain (the multi-function unit)
-// and a cuBLAS GEMM in tf32 or bf16 (the tensor pipe for those operand
-// types).  Each launches work of a known operation count on the caller's
-// stream; the caller times it with events.  Not on any hot path.
+// chain (the FP32 pipe), tanh.approx.f32 and ex2.approx.f32 chains (the
+// multi-function unit), a cuBLAS GEMM in tf32 or bf16 (the tensor pipe for
+// those operand types), and back-to-back tcgen05 MMAs of one shape (the
+// tensor pipe's cost per instruction at the engine's small N).  Each
+// launches work of a known operation count on the caller's stream; the
+// caller times it with events (the MMA probe times itself in cycles).  Not
+// on any hot path.
 #include <cublas_v2.h>
 #include <cuda_runtime.h>
 
@@ -10,8 +13,11 @@
 #include <mutex>
 
 #include "auvenv.h"
+#include "tc_ptx.cuh"
 
 namespace {
+
+namespace tc = auv::tc;
 
 constexpr int kChains = 8;   // independent dependency chains per thread
 
@@ -51,6 +57,106 @@ __global__ void k_probe_tanh(uint32_t iters, float* sink) {
   if (s == 12345.678f) sink[blockIdx.x * blockDim.x + threadIdx.x] = s;
 }
 
+// iters x kChains dependent ex2.approx.ftz.f32 per thread (one operation each).
+__global__ void k_probe_ex2(uint32_t iters, float* sink) {
+  float a[kChains];
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) a[j] = 1e-3f * (threadIdx.x + j);
+  for (uint32_t i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int j = 0; j < kChains; ++j) {
+      float r;
+      asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(a[j]));
+      a[j] = r - 1.0f;
+    }
+  }
+  float s = 0.0f;
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) s += a[j];
+  if (s == 12345.678f) sink[blockIdx.x * blockDim.x + threadIdx.x] = s;
+}
+
+// One elected thread per CTA issues `iters` tcgen05 MMAs of shape M = 128,
+// N, K = 16 (bf16 operands, zero-filled; fp32 accumulator in tensor memory
+// columns 0..N-1) back to back into one accumulator, with B from shared
+// memory (128-byte swizzled K-major rows) and A from shared memory or from
+// tensor memory (columns 256..287), commits once and waits (bounded) for
+// the completion.  cycles[block] = clock64 span from the first issue to the
+// completion, or 0 if the wait gave up.  120 KB of shared memory keep one
+// CTA per SM.
+constexpr uint32_t kMmaSmem = 120u * 1024u;
+template <int N, bool kTs>
+__global__ void __launch_bounds__(128) k_probe_mma(uint32_t iters, unsigned long long* cycles) {
+  extern __shared__ uint8_t mma_smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(mma_smem_raw) + 1023u) & ~(uintptr_t)1023u);
+  __shared__ uint64_t bar;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_flag;
+  const int tid = threadIdx.x;
+  // operands: B at 0 (N rows x 128 B), A at 32 KB (128 rows x 128 B)
+  for (int i = tid; i < 48 * 1024 / 16; i += 128)
+    reinterpret_cast<uint4*>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (tid == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    tc::mbar_fence_init();
+  }
+  if (tid < 32) {
+    tc::tmem_alloc(&tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::fence_async_smem();
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = tmem_base;
+  if (tid == 0) {
+    const uint32_t sb = tc::smem_u32(smem);
+    const uint64_t b_desc = tc::smem_desc(sb, 1024, 2);
+    const uint64_t a_desc = tc::smem_desc(sb + 32768, 1024, 2);
+    constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, N);
+    const unsigned long long t0 = clock64();
+    for (uint32_t i = 0; i < iters; ++i) {
+      const uint32_t kk = i & 3u;   // the four K = 16 steps of a 128-byte row
+      if constexpr (kTs)
+        tc::mma_ts(tmem, tmem + 256 + kk * 8, b_desc + (uint64_t)(kk * 2), kIdesc, i > 0 ? 1u : 0u);
+      else
+        tc::mma_ss(tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), kIdesc,
+                   i > 0 ? 1u : 0u);
+    }
+    tc::mma_commit(&bar);
+    const bool ok = tc::mbar_wait(&bar, 0, &abort_flag, 1000000000ull);
+    cycles[blockIdx.x] = ok ? clock64() - t0 : 0ull;
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  if (tid < 32) tc::tmem_dealloc(tmem, 512);
+}
+
+template <int N, bool kTs>
+cudaError_t launch_probe_mma(uint32_t iters, uint32_t blocks, unsigned long long* cycles,
+                             cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(k_probe_mma<N, kTs>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+  if (e != cudaSuccess) return e;
+  k_probe_mma<N, kTs><<<blocks, 128, kMmaSmem, s>>>(iters, cycles);
+  return cudaGetLastError();
+}
+
+template <bool kTs>
+cudaError_t launch_probe_mma_n(int n, uint32_t iters, uint32_t blocks, unsigned long long* cycles,
+                               cudaStream_t s) {
+  switch (n) {
+    case 16: return launch_probe_mma<16, kTs>(iters, blocks, cycles, s);
+    case 32: return launch_probe_mma<32, kTs>(iters, blocks, cycles, s);
+    case 64: return launch_probe_mma<64, kTs>(iters, blocks, cycles, s);
+    case 128: return launch_probe_mma<128, kTs>(iters, blocks, cycles, s);
+    default: return launch_probe_mma<256, kTs>(iters, blocks, cycles, s);
+  }
+}
+
 int probe_grid(uint32_t blocks, uint32_t threads, uint32_t iters, const float* sink) {
   if (blocks < 1 || blocks > 65535 || threads < 32 || threads > 1024 || threads % 32 || iters < 1 ||
       !sink)
@@ -77,6 +183,25 @@ int auv_probe_tanh(uint32_t blocks, uint32_t threads, uint32_t iters, float* sin
   if (rc) return rc;
   k_probe_tanh<<<blocks, threads, 0, static_cast<cudaStream_t>(stream)>>>(iters, sink);
   return cudaGetLastError() == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
+}
+
+int auv_probe_ex2(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream) {
+  int rc = probe_grid(blocks, threads, iters, sink);
+  if (rc) return rc;
+  k_probe_ex2<<<blocks, threads, 0, static_cast<cudaStream_t>(stream)>>>(iters, sink);
+  return cudaGetLastError() == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
+}
+
+int auv_probe_mma(int n, int a_tmem, uint32_t iters, uint32_t blocks, uint64_t* cycles,
+                  void* stream) {
+  if ((n != 16 && n != 32 && n != 64 && n != 128 && n != 256) || iters < 1 || iters > (1u << 20) ||
+      blocks < 1 || blocks > 65535 || !cycles)
+    return AUV_ERR_INVALID;
+  unsigned long long* c = reinterpret_cast<unsigned long long*>(cycles);
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const cudaError_t e = a_tmem ? launch_probe_mma_n<true>(n, iters, blocks, c, s)
+                               : launch_probe_mma_n<false>(n, iters, blocks, c, s);
+  return e == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
 }
 
 int auv_probe_gemm(uint32_t precision, int n, const void* a, const void* b, void* c, void* stream) {

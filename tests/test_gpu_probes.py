@@ -61,3 +61,36 @@ def test_probes_reject_bad_arguments():
     a = torch.zeros(24, 24, device="cuda")
     with pytest.raises(auvenv.AuvError):
         auvenv.probe_gemm("tf32", a, a, a)           # n not a multiple of 16
+
+
+def test_mma_probe_costs_grow_with_n():
+    """The tcgen05 probe completes (no bounded wait gives up) and a wider
+    MMA never costs fewer cycles than a narrower one."""
+    torch = need_gpu()
+    from paper_2512_13359_gb300 import auvenv
+    cyc = torch.zeros(4, dtype=torch.int64, device="cuda")
+    per = {}
+    for n in (16, 64, 256):
+        for a_tmem in (False, True):
+            auvenv.probe_mma(n, a_tmem, 256, cyc)
+            torch.cuda.synchronize()
+            c = cyc.cpu()
+            assert int((c == 0).sum()) == 0
+            per[(n, a_tmem)] = float(c.double().median()) / 256
+    print("[probe] cycles per MMA", per)
+    for a_tmem in (False, True):
+        assert per[(16, a_tmem)] <= per[(64, a_tmem)] * 1.05 <= per[(256, a_tmem)] * 1.05
+    with pytest.raises(auvenv.AuvError):
+        auvenv.probe_mma(48, False, 16, cyc)            # not a supported N
+    with pytest.raises(auvenv.AuvError):
+        auvenv.probe_mma(64, False, 0, cyc)             # no MMA
+
+
+def test_ex2_probe_runs():
+    torch = need_gpu()
+    from paper_2512_13359_gb300 import auvenv
+    sink = torch.zeros(4 * 256, device="cuda")
+    assert auvenv.probe_ex2(4, 256, 10, sink) == 8 * 4 * 256 * 10
+    torch.cuda.synchronize()
+    with pytest.raises(auvenv.AuvError):
+        auvenv.probe_ex2(4, 100, 10, sink)
