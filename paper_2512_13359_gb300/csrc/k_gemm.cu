@@ -25,7 +25,8 @@
 // kernel with the same operand layouts and the same split-K.
 //
 // Split-K: partial tiles go to ws[z][M_pad][N_pad] (fp32); k_reduce adds
-// them in the order z = 0, 1, ... and applies beta and the output type.
+// them in a fixed order (eight interleaved partial sums over z, then those
+// eight in order) and applies beta and the output type.
 #include <cuda.h>
 
 #include <algorithm>
@@ -450,35 +451,79 @@ k_gemm_fp32(int M, int N, int K, const float* __restrict__ A, int lda, const flo
   }
 }
 
-// C = beta C + sum_z ws[z] (z in order), fp32 or bf16 output; one element
-// per thread.  A weight gradient has a few tens of thousands of elements and
-// tens of splits, so the kernel is bound by load latency: each thread issues
-// the loads of 16 partials before it adds them (in z order), so that a split
-// count below 80 costs at most five round trips to memory.
-__global__ void k_reduce(int M, int N, int splits, const float* __restrict__ ws, int m_pad,
-                         int n_pad, void* C, int ldc, int c_bf16, float beta) {
-  constexpr int kU = 16;
-  const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (size_t)M * N) return;
-  const int m = (int)(idx / N), n = (int)(idx % N);
+// C = beta C + sum_z ws[z], fp32 or bf16 output.  A weight gradient has a
+// few tens of thousands of elements and tens of splits, so one thread per
+// element summing every split in turn left the kernel bound by load latency
+// at under two blocks per SM.  Here a block of 256 threads covers 128
+// consecutive elements (32 groups of four, 16-byte loads) for 8 groups of
+// splits: thread (g, l) adds the partials z = g, g + 8, g + 16, ... of its
+// four elements in increasing z, and the eight group sums are then added in
+// the order g = 0..7: a fixed order, the same on every run.
+constexpr int kRedGroups = 8;
+constexpr int kRedQuads = 32;
+__global__ void __launch_bounds__(kRedGroups * kRedQuads)
+k_reduce(int M, int N, int splits, const float* __restrict__ ws, int m_pad, int n_pad, void* C,
+         int ldc, int c_bf16, float beta) {
+  __shared__ float4 part[kRedGroups][kRedQuads];
+  const int lane = threadIdx.x % kRedQuads, grp = threadIdx.x / kRedQuads;
+  const int qpr = (N + 3) / 4;   // groups of four per row (n_pad is a multiple of 128)
+  const long quad = (long)blockIdx.x * kRedQuads + lane;
+  const bool live = quad < (long)M * qpr;
+  const int m = live ? (int)(quad / qpr) : 0, n = live ? (int)(quad % qpr) * 4 : 0;
   const size_t zs = (size_t)m_pad * n_pad;
   const float* src = ws + (size_t)m * n_pad + n;
-  float v = 0.0f;
-  for (int z = 0; z < splits; z += kU) {
-    float p[kU];
+  // 16-byte loads when the workspace is 16-byte aligned (every offset here
+  // is a multiple of four floats), four scalar loads otherwise
+  const bool vec = (reinterpret_cast<uintptr_t>(ws) & 15u) == 0;
+  auto load4 = [&](const float* a) {
+    return vec ? __ldcs(reinterpret_cast<const float4*>(a))
+               : make_float4(__ldcs(a), __ldcs(a + 1), __ldcs(a + 2), __ldcs(a + 3));
+  };
+  float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  if (live) {
+    constexpr int kU = 4;   // loads in flight per thread
+    for (int z0 = grp; z0 < splits; z0 += kRedGroups * kU) {
+      float4 p[kU];
 #pragma unroll
-    for (int q = 0; q < kU; ++q) p[q] = z + q < splits ? __ldcs(src + (size_t)(z + q) * zs) : 0.0f;
+      for (int q = 0; q < kU; ++q) {
+        const int z = z0 + q * kRedGroups;
+        p[q] = z < splits ? load4(src + (size_t)z * zs) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      }
 #pragma unroll
-    for (int q = 0; q < kU; ++q)
-      if (z + q < splits) v += p[q];
+      for (int q = 0; q < kU; ++q)
+        if (z0 + q * kRedGroups < splits) {
+          v.x += p[q].x;
+          v.y += p[q].y;
+          v.z += p[q].z;
+          v.w += p[q].w;
+        }
+    }
   }
-  if (c_bf16) {
-    uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n;
-    if (beta != 0.0f) v = fmaf(beta, __uint_as_float((uint32_t)*c << 16), v);
-    *c = (uint16_t)(tc::pack_bf16x2(v, 0.0f) & 0xFFFFu);
-  } else {
-    float* c = static_cast<float*>(C) + (size_t)m * ldc + n;
-    *c = beta != 0.0f ? fmaf(beta, *c, v) : v;
+  part[grp][lane] = v;
+  __syncthreads();
+  if (grp != 0 || !live) return;
+  float4 s = part[0][lane];
+#pragma unroll
+  for (int g = 1; g < kRedGroups; ++g) {
+    const float4 u = part[g][lane];
+    s.x += u.x;
+    s.y += u.y;
+    s.z += u.z;
+    s.w += u.w;
+  }
+  const float r[4] = {s.x, s.y, s.z, s.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (n + j >= N) break;
+    float x = r[j];
+    if (c_bf16) {
+      uint16_t* c = static_cast<uint16_t*>(C) + (size_t)m * ldc + n + j;
+      if (beta != 0.0f) x = fmaf(beta, __uint_as_float((uint32_t)*c << 16), x);
+      *c = (uint16_t)(tc::pack_bf16x2(x, 0.0f) & 0xFFFFu);
+    } else {
+      float* c = static_cast<float*>(C) + (size_t)m * ldc + n + j;
+      *c = beta != 0.0f ? fmaf(beta, *c, x) : x;
+    }
   }
 }
 
@@ -718,9 +763,9 @@ cudaError_t launch(Prec prec, int M, int N, int K, const Operand& A_in, const Op
                         : dispatch_major<false, 128>(A.mn_major, B.mn_major, P, ma, mb, a, s);
   }
   if (e != cudaSuccess || !part) return e;
-  const size_t n = (size_t)M * N;
-  k_reduce<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(M, N, P.splits, part, P.m_pad, P.n_pad, C,
-                                                       ldc, c_bf16 ? 1 : 0, beta);
+  const size_t quads = (size_t)M * ((N + 3) / 4);
+  k_reduce<<<(unsigned)((quads + kRedQuads - 1) / kRedQuads), kRedGroups * kRedQuads, 0, s>>>(
+      M, N, P.splits, part, P.m_pad, P.n_pad, C, ldc, c_bf16 ? 1 : 0, beta);
   return cudaGetLastError();
 }
 
