@@ -573,7 +573,7 @@ def run_gae(args):
 # profiles/k_engine_ppo_65536_T128_dram.md), valid while the engine's sources
 # hash to ENGINE_SRC_HASH.
 ROLLOUT_TRAFFIC_65536x128 = 10_622_976 + 900_608_256
-ENGINE_SRC_HASH = "ce6892845323d80d"
+ENGINE_SRC_HASH = "6e8400dd6451a3f1"
 ENGINE_SRCS = ("k_bf16.cu", "auv_device.cuh", "tc_ptx.cuh", "auv_bf16.h")
 
 

@@ -40,6 +40,12 @@ cudaError_t launch_learn_forward_bf16(bool policy, const void* packed, int in_di
 size_t bf16_back_image_bytes();
 cudaError_t launch_pack_back_bf16(int in_dim, int out_dim, const float* w_f32, void* packed,
                                   cudaStream_t s);
+// The learner's forward and backward images of both networks in one launch
+// (launch_pack_bf16_dims and launch_pack_back_bf16 of each; a NULL weight
+// pointer skips that network's two images).
+cudaError_t launch_pack_learner_bf16(int in_dim, int policy_out, const float* wp_f32,
+                                     const float* wv_f32, void* wp_packed, void* wv_packed,
+                                     void* bp_packed, void* bv_packed, cudaStream_t s);
 cudaError_t launch_learn_backward_bf16(const void* packed, int out_dim, const uint16_t* gy, int ldy,
                                        size_t rows, const uint16_t* h2, const uint16_t* h1, int ldh,
                                        uint16_t* gz2, int ldz2, uint16_t* gz1, int ldz1, Status* st,

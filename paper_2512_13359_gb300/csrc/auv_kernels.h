@@ -205,6 +205,10 @@ cudaError_t launch_finish(const float* acc, float* out, cudaStream_t s);
 // flat [W1|b1|W2|b2|W3|b3] <-> augmented [W1a|W2a|W3a] of one network
 cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int Hp, int out,
                            bool to_aug, cudaStream_t s);
+// the same for the policy and the value network in one launch
+cudaError_t launch_convert_pair(float* flat_pol, float* aug_pol, int out_pol, float* flat_val,
+                                float* aug_val, int out_val, int in, int in_p, int H, int Hp,
+                                bool to_aug, cudaStream_t s);
 cudaError_t launch_fill_ones(bool bf16, void* buf, int ld, int col, int rows, cudaStream_t s);
 
 }  // namespace ppo

@@ -114,8 +114,8 @@ constexpr int kBiasCol = 30;
 // One thread per 16-byte piece of the W1/W2/W3 regions, then the vectors.
 // in_dim: network input width (18 or 12, <= 32); out_dim: 1 (value) or the
 // policy head width (<= 16; head rows out_dim..15 are packed as zeros).
-__global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
-                       uint8_t* __restrict__ img) {
+__device__ void pack_piece(const float* __restrict__ w, int in_dim, int out_dim,
+                           uint8_t* __restrict__ img, int piece) {
   const float* W1 = w;
   const float* b1 = W1 + kH * in_dim;
   const float* W2 = b1 + kH;
@@ -124,7 +124,6 @@ __global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
   const float* b3 = W3 + out_dim * kH;
   const bool policy = out_dim > 1;
   const int n_w1 = kH * 4, n_w2 = 4 * kH * 8, n_w3 = policy ? 4 * kHeadOut * 8 : 0;
-  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
   uint16_t v[8];
   uint32_t off;
   if (piece < n_w1) {
@@ -176,12 +175,11 @@ __global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
 // Backward image of one network from its flat fp32 weights (the layout of
 // k_pack): one thread per 16-byte piece of the W1 slot (W3^T, K = 32 with the
 // columns from out_dim up zero) and of the W2 slot (W2^T).
-__global__ void k_pack_back(const float* __restrict__ w, int in_dim, int out_dim,
-                            uint8_t* __restrict__ img) {
+__device__ void pack_back_piece(const float* __restrict__ w, int in_dim, int out_dim,
+                                uint8_t* __restrict__ img, int piece) {
   const float* W2 = w + kH * in_dim + kH;
   const float* W3 = W2 + kH * kH + kH;
   const int n_w1 = kH * 4, n_w2 = 4 * kH * 8;
-  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
   uint16_t v[8];
   uint32_t off;
   if (piece < n_w1) {
@@ -205,6 +203,44 @@ __global__ void k_pack_back(const float* __restrict__ w, int in_dim, int out_dim
   pk.z = v[4] | ((uint32_t)v[5] << 16);
   pk.w = v[6] | ((uint32_t)v[7] << 16);
   *reinterpret_cast<uint4*>(img + off) = pk;
+}
+
+// Pieces per image (pack_piece: W1, W2, W3 slots, then the vector entries;
+// pack_back_piece: W1 and W2 slots).
+constexpr int kPolPieces = kH * 4 + 4 * kH * 8 + 4 * kHeadOut * 8 + 2 * kH + kHeadOut;
+constexpr int kValPieces = kH * 4 + 4 * kH * 8 + 3 * kH + 1;
+constexpr int kBackPieces = kH * 4 + 4 * kH * 8;
+
+__global__ void k_pack(const float* __restrict__ w, int in_dim, int out_dim,
+                       uint8_t* __restrict__ img) {
+  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
+  if (piece < (out_dim > 1 ? kPolPieces : kValPieces)) pack_piece(w, in_dim, out_dim, img, piece);
+}
+
+__global__ void k_pack_back(const float* __restrict__ w, int in_dim, int out_dim,
+                            uint8_t* __restrict__ img) {
+  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
+  if (piece < kBackPieces) pack_back_piece(w, in_dim, out_dim, img, piece);
+}
+
+// The learner's four images in one launch: blockIdx.y = 0 policy forward,
+// 1 value forward, 2 policy backward, 3 value backward (a NULL weight
+// pointer skips its images).
+struct LearnerImages {
+  const float* w[2];   // flat fp32 weights, policy and value
+  int in_dim, out_dim[2];
+  uint8_t* fwd[2];
+  uint8_t* back[2];
+};
+__global__ void k_pack_learner(const LearnerImages L) {
+  const int job = blockIdx.y, net = job & 1;
+  const int piece = blockIdx.x * blockDim.x + threadIdx.x;
+  if (!L.w[net]) return;
+  if (job < 2) {
+    if (piece < (net ? kValPieces : kPolPieces)) pack_piece(L.w[net], L.in_dim, L.out_dim[net], L.fwd[net], piece);
+  } else if (piece < kBackPieces) {
+    pack_back_piece(L.w[net], L.in_dim, L.out_dim[net], L.back[net], piece);
+  }
 }
 
 // -------------------------------------------------------------------------
@@ -1259,9 +1295,21 @@ size_t bf16_back_image_bytes() { return kBackImage; }
 
 cudaError_t launch_pack_back_bf16(int in_dim, int out_dim, const float* w_f32, void* packed,
                                   cudaStream_t s) {
-  const int pieces = kH * 4 + 4 * kH * 8;
-  k_pack_back<<<(pieces + 255) / 256, 256, 0, s>>>(w_f32, in_dim, out_dim,
-                                                   static_cast<uint8_t*>(packed));
+  k_pack_back<<<(kBackPieces + 255) / 256, 256, 0, s>>>(w_f32, in_dim, out_dim,
+                                                        static_cast<uint8_t*>(packed));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack_learner_bf16(int in_dim, int policy_out, const float* wp_f32,
+                                     const float* wv_f32, void* wp_packed, void* wv_packed,
+                                     void* bp_packed, void* bv_packed, cudaStream_t s) {
+  const LearnerImages L = {{wp_f32, wv_f32},
+                           in_dim,
+                           {policy_out, 1},
+                           {static_cast<uint8_t*>(wp_packed), static_cast<uint8_t*>(wv_packed)},
+                           {static_cast<uint8_t*>(bp_packed), static_cast<uint8_t*>(bv_packed)}};
+  constexpr int kMax = kPolPieces > kBackPieces ? kPolPieces : kBackPieces;
+  k_pack_learner<<<dim3((kMax + 255) / 256, 4), 256, 0, s>>>(L);
   return cudaGetLastError();
 }
 
@@ -1274,16 +1322,14 @@ cudaError_t launch_pack_bf16(const Model& M, const float* wp_f32, const float* w
 cudaError_t launch_pack_bf16_dims(int in_dim, int policy_out, const float* wp_f32,
                                   const float* wv_f32, void* wp_packed, void* wv_packed,
                                   cudaStream_t s) {
-  const int pol_pieces = kH * 4 + 4 * kH * 8 + 4 * kHeadOut * 8 + 2 * kH + kHeadOut;
   cudaError_t e = cudaSuccess;
   if (wp_f32) {
-    k_pack<<<(pol_pieces + 255) / 256, 256, 0, s>>>(wp_f32, in_dim, policy_out,
+    k_pack<<<(kPolPieces + 255) / 256, 256, 0, s>>>(wp_f32, in_dim, policy_out,
                                                     static_cast<uint8_t*>(wp_packed));
     e = cudaGetLastError();
   }
   if (e != cudaSuccess || !wv_f32) return e;
-  const int val_pieces = kH * 4 + 4 * kH * 8 + 3 * kH + 1;
-  k_pack<<<(val_pieces + 255) / 256, 256, 0, s>>>(wv_f32, in_dim, 1,
+  k_pack<<<(kValPieces + 255) / 256, 256, 0, s>>>(wv_f32, in_dim, 1,
                                                   static_cast<uint8_t*>(wv_packed));
   return cudaGetLastError();
 }

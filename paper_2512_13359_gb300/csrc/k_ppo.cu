@@ -742,8 +742,8 @@ __device__ __forceinline__ long long flat_index(size_t e, int in, int in_p, int 
   return col < H ? w3 + (long long)row * H + col : col == H ? b3 + row : -1;
 }
 
-__global__ void __launch_bounds__(kT) k_convert(float* flat, float* aug, size_t n_aug, int in,
-                                                int in_p, int H, int Hp, int out, int to_aug) {
+__device__ void convert_range(float* flat, float* aug, size_t n_aug, int in, int in_p, int H, int Hp,
+                              int out, int to_aug) {
   for (size_t e = blockIdx.x * (size_t)kT + threadIdx.x; e < n_aug; e += (size_t)gridDim.x * kT) {
     const long long f = flat_index(e, in, in_p, H, Hp, out);
     if (to_aug)
@@ -751,6 +751,24 @@ __global__ void __launch_bounds__(kT) k_convert(float* flat, float* aug, size_t 
     else if (f >= 0)
       flat[f] = aug[e];
   }
+}
+
+__global__ void __launch_bounds__(kT) k_convert(float* flat, float* aug, size_t n_aug, int in,
+                                                int in_p, int H, int Hp, int out, int to_aug) {
+  convert_range(flat, aug, n_aug, in, in_p, H, Hp, out, to_aug);
+}
+
+// Both networks in one launch: blockIdx.y = 0 policy, 1 value.
+struct ConvertPair {
+  float* flat[2];
+  float* aug[2];
+  int out[2];
+  size_t n_aug[2];
+};
+__global__ void __launch_bounds__(kT) k_convert_pair(const ConvertPair c, int in, int in_p, int H,
+                                                     int Hp, int to_aug) {
+  const int net = blockIdx.y;
+  convert_range(c.flat[net], c.aug[net], c.n_aug[net], in, in_p, H, Hp, c.out[net], to_aug);
 }
 
 template <typename TX>
@@ -886,6 +904,18 @@ cudaError_t launch_convert(float* flat, float* aug, int in, int in_p, int H, int
                            bool to_aug, cudaStream_t s) {
   const size_t n = aug_count(in, in_p, H, Hp, out);
   k_convert<<<grid_for(n), kT, 0, s>>>(flat, aug, n, in, in_p, H, Hp, out, to_aug ? 1 : 0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_convert_pair(float* flat_pol, float* aug_pol, int out_pol, float* flat_val,
+                                float* aug_val, int out_val, int in, int in_p, int H, int Hp,
+                                bool to_aug, cudaStream_t s) {
+  const ConvertPair c = {{flat_pol, flat_val},
+                         {aug_pol, aug_val},
+                         {out_pol, out_val},
+                         {aug_count(in, in_p, H, Hp, out_pol), aug_count(in, in_p, H, Hp, out_val)}};
+  const size_t n = c.n_aug[0] > c.n_aug[1] ? c.n_aug[0] : c.n_aug[1];
+  k_convert_pair<<<dim3(grid_for(n), 2), kT, 0, s>>>(c, in, in_p, H, Hp, to_aug ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -328,13 +328,10 @@ int grads_impl(auv_ppo* p, const auv_ppo_batch* b, float* acc, cudaStream_t s) {
     // Both networks on the tensor-core engine: flat fp32 weights, packed bf16
     // images, then one launch per network writing H1, H2 and the head.
     if ((rc = convert(p, p->flat_eng, p->flat_eng + p->n_flat[0], p->w, false, s))) return rc;
-    if ((e = auv::launch_pack_bf16_dims(d.D, p->out[0], d.value_only ? nullptr : p->flat_eng,
-                                        p->flat_eng + p->n_flat[0], p->img_p, p->img_v, s)))
+    if ((e = auv::launch_pack_learner_bf16(d.D, p->out[0], d.value_only ? nullptr : p->flat_eng,
+                                           p->flat_eng + p->n_flat[0], p->img_p, p->img_v,
+                                           p->img_bp, p->img_bv, s)))
       return cuda_fail(p, e, "pack engine weights");
-    for (int net = d.value_only ? 1 : 0; net < 2; ++net)
-      if ((e = auv::launch_pack_back_bf16(d.D, p->out[net], p->flat_eng + (net ? p->n_flat[0] : 0),
-                                          net ? p->img_bv : p->img_bp, s)))
-        return cuda_fail(p, e, "pack engine backward weights");
     for (int net = d.value_only ? 1 : 0; net < 2; ++net) {
       if ((e = auv::launch_learn_forward_bf16(net == 0, net ? p->img_v : p->img_p, d.D, p->out[net],
                                          static_cast<const uint16_t*>(p->X), d.Dp, (size_t)d.B,
@@ -414,9 +411,8 @@ bool capture_step(auv_ppo* p, const auv_ppo_batch* b) {
 int convert(auv_ppo* p, float* flat_pol, float* flat_val, float* aug, bool to_aug,
             cudaStream_t s) {
   const ppo::Dims& d = p->d;
-  cudaError_t e = ppo::launch_convert(flat_pol, aug, d.D, d.Dp, d.H, d.Hp, p->out[0], to_aug, s);
-  if (e == cudaSuccess)
-    e = ppo::launch_convert(flat_val, aug + p->n_aug[0], d.D, d.Dp, d.H, d.Hp, p->out[1], to_aug, s);
+  const cudaError_t e = ppo::launch_convert_pair(flat_pol, aug, p->out[0], flat_val, aug + p->n_aug[0],
+                                                 p->out[1], d.D, d.Dp, d.H, d.Hp, to_aug, s);
   return e == cudaSuccess ? AUV_OK : cuda_fail(p, e, "weight layout conversion");
 }
 
