@@ -460,20 +460,21 @@ def run_probes(args):
     ffma = timed(lambda: auvenv.probe_ffma(blocks, threads, 20000, sink), max(args.steps, 5))
     tanh = timed(lambda: auvenv.probe_tanh(blocks, threads, 4000, sink), max(args.steps, 5))
     ex2 = timed(lambda: auvenv.probe_ex2(blocks, threads, 4000, sink), max(args.steps, 5))
-    mma = {}
+    mma, mma_tf32 = {}, {}
     mma_iters = 1024
     cyc = torch.zeros(sms, dtype=torch.int64, device="cuda")
-    for nn in (16, 32, 64, 128, 256):
-        for a_tmem in (False, True):
-            for _ in range(2):
-                auvenv.probe_mma(nn, a_tmem, mma_iters, cyc)
-            torch.cuda.synchronize()
-            c = cyc.cpu()
-            if int((c == 0).sum()):
-                raise RuntimeError("mma probe: a bounded wait gave up")
-            per = float(c.double().median()) / mma_iters
-            mma[f"n{nn}_{'ts' if a_tmem else 'ss'}"] = {
-                "cycles_per_mma": per, "mac_per_clk_per_sm": 128 * nn * 16 / per}
+    for tf32, out, k in ((False, mma, 16), (True, mma_tf32, 8)):
+        for nn in (16, 32, 64, 128, 256):
+            for a_tmem in (False, True):
+                for _ in range(2):
+                    auvenv.probe_mma(nn, a_tmem, mma_iters, cyc, tf32=tf32)
+                torch.cuda.synchronize()
+                c = cyc.cpu()
+                if int((c == 0).sum()):
+                    raise RuntimeError("mma probe: a bounded wait gave up")
+                per = float(c.double().median()) / mma_iters
+                out[f"n{nn}_{'ts' if a_tmem else 'ss'}"] = {
+                    "cycles_per_mma": per, "mac_per_clk_per_sm": 128 * nn * k / per}
     n = 8192
     g = torch.Generator(device="cuda").manual_seed(0)
     a32 = torch.randn(n, n, device="cuda", generator=g)
@@ -497,6 +498,7 @@ def run_probes(args):
             "mufu_ex2_gops": ex2 / 1e9,
             "mufu_ex2_per_clk_per_sm": ex2 / (sms * mhz * 1e6),
             "tcgen05_mma_m128_k16_bf16": mma,
+            "tcgen05_mma_m128_k8_tf32": mma_tf32,
             "tf32_gemm_tflops": tf32 / 1e12, "bf16_gemm_tflops": bf16 / 1e12,
             "bf16_peak_measured_tflops": peaks.get("bf16_tflops"),
             "tf32_over_bf16": tf32 / bf16, "nominal_tf32_over_bf16": 1.1 / 2.25,

@@ -751,10 +751,10 @@ int auv_gemm(uint32_t precision, int M, int N, int K, const void* A, int lda, in
  *   with A, B fp32 and tf32 tensor-core math (AUV_PPO_TF32) or bf16 operands
  *   (AUV_PPO_BF16): 2 n^3 flop.  n a multiple of 16.
  * auv_probe_mma: `blocks` CTAs (one per SM), each issuing `iters` tcgen05
- *   MMAs of shape M = 128, N = n, K = 16 (kind::f16, bf16 operands,
- *   fp32 accumulator; A in shared memory, or in tensor memory when a_tmem is
- *   nonzero) back to back from one thread, then one commit and one bounded
- *   wait.  cycles: device memory of `blocks` uint64 values, each the SM
+ *   MMAs of shape M = 128, N = n and K = 16 bf16 (kind::f16), or K = 8 tf32
+ *   (kind::tf32) when tf32 is nonzero, fp32 accumulator; A in shared memory,
+ *   or in tensor memory when a_tmem is nonzero; back to back from one
+ *   thread, then one commit and one bounded wait.  cycles: device memory of `blocks` uint64 values, each the SM
  *   cycles from the first issue to the completion (0 if the wait gave up).
  *   n in {16, 32, 64, 128, 256}, iters in [1, 2^20], blocks in [1, 65535].
  * Return AUV_OK, AUV_ERR_INVALID on bad arguments or AUV_ERR_CUDA.
@@ -762,7 +762,7 @@ int auv_gemm(uint32_t precision, int M, int N, int K, const void* A, int lda, in
 int auv_probe_ffma(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream);
 int auv_probe_tanh(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream);
 int auv_probe_ex2(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink, void* stream);
-int auv_probe_mma(int n, int a_tmem, uint32_t iters, uint32_t blocks, uint64_t* cycles,
+int auv_probe_mma(int n, int a_tmem, int tf32, uint32_t iters, uint32_t blocks, uint64_t* cycles,
                   void* stream);
 int auv_probe_gemm(uint32_t precision, int n, const void* a, const void* b, void* c, void* stream);
 

@@ -198,7 +198,7 @@ def lib(path: str | None = None):
     L.auv_probe_ffma.argtypes = [U32, U32, U32, P, P]
     L.auv_probe_tanh.argtypes = [U32, U32, U32, P, P]
     L.auv_probe_ex2.argtypes = [U32, U32, U32, P, P]
-    L.auv_probe_mma.argtypes = [I, I, U32, U32, P, P]
+    L.auv_probe_mma.argtypes = [I, I, I, U32, U32, P, P]
     L.auv_probe_gemm.argtypes = [U32, I, P, P, P, P]
     L.auv_gemm_workspace_bytes.argtypes = [I, I, I]
     L.auv_gemm_workspace_bytes.restype = C.c_size_t
@@ -605,11 +605,13 @@ def probe_ex2(blocks: int, threads: int, iters: int, sink, stream=None) -> int:
     return 8 * blocks * threads * iters
 
 
-def probe_mma(n: int, a_tmem: bool, iters: int, cycles, stream=None) -> None:
-    """Enqueue the tcgen05 MMA probe on cycles.numel() CTAs (cycles: uint64
-    device tensor, one SM-cycle span per CTA, 0 where the wait gave up)."""
-    _probe_check(lib().auv_probe_mma(n, 1 if a_tmem else 0, iters, int(cycles.numel()), _ptr(cycles),
-                                     _stream(stream)), "mma probe")
+def probe_mma(n: int, a_tmem: bool, iters: int, cycles, stream=None, tf32: bool = False) -> None:
+    """Enqueue the tcgen05 MMA probe (bf16, or tf32 with tf32=True) on
+    cycles.numel() CTAs (cycles: 64-bit device tensor, one SM-cycle span per
+    CTA, 0 where the wait gave up)."""
+    _probe_check(lib().auv_probe_mma(n, 1 if a_tmem else 0, 1 if tf32 else 0, iters,
+                                     int(cycles.numel()), _ptr(cycles), _stream(stream)),
+                 "mma probe")
 
 
 def probe_gemm(precision: str, a, b, c, stream=None) -> int:

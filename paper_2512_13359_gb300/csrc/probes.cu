@@ -76,16 +76,40 @@ __global__ void k_probe_ex2(uint32_t iters, float* sink) {
   if (s == 12345.678f) sink[blockIdx.x * blockDim.x + threadIdx.x] = s;
 }
 
+// kind::tf32 MMAs (D fp32, A and B tf32, K-major; K = 8 per instruction):
+// instruction descriptor and the two operand forms.
+__host__ __device__ constexpr uint32_t idesc_tf32_f32(int M, int N) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_tf32_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t id,
+                                            uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(id), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void mma_tf32_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t id,
+                                            uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(id), "r"(acc)
+      : "memory");
+}
+
 // One elected thread per CTA issues `iters` tcgen05 MMAs of shape M = 128,
-// N, K = 16 (bf16 operands, zero-filled; fp32 accumulator in tensor memory
-// columns 0..N-1) back to back into one accumulator, with B from shared
-// memory (128-byte swizzled K-major rows) and A from shared memory or from
-// tensor memory (columns 256..287), commits once and waits (bounded) for
-// the completion.  cycles[block] = clock64 span from the first issue to the
-// completion, or 0 if the wait gave up.  120 KB of shared memory keep one
-// CTA per SM.
+// N, K = 16 bf16 (kind::f16) or K = 8 tf32 (kind::tf32) operands,
+// zero-filled, fp32 accumulator in tensor memory columns 0..N-1, back to back
+// into one accumulator, with B from shared memory (128-byte swizzled K-major
+// rows: one K-step is 32 bytes for either type) and A from shared memory or
+// from tensor memory (columns 256..287), commits once and waits (bounded)
+// for the completion.  cycles[block] = clock64 span from the first issue to
+// the completion, or 0 if the wait gave up.  120 KB of shared memory keep
+// one CTA per SM.
 constexpr uint32_t kMmaSmem = 120u * 1024u;
-template <int N, bool kTs>
+template <int N, bool kTs, bool kTf32>
 __global__ void __launch_bounds__(128) k_probe_mma(uint32_t iters, unsigned long long* cycles) {
   extern __shared__ uint8_t mma_smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -115,15 +139,19 @@ __global__ void __launch_bounds__(128) k_probe_mma(uint32_t iters, unsigned long
     const uint32_t sb = tc::smem_u32(smem);
     const uint64_t b_desc = tc::smem_desc(sb, 1024, 2);
     const uint64_t a_desc = tc::smem_desc(sb + 32768, 1024, 2);
-    constexpr uint32_t kIdesc = tc::idesc_bf16_f32(128, N);
+    constexpr uint32_t kIdesc = kTf32 ? idesc_tf32_f32(128, N) : tc::idesc_bf16_f32(128, N);
     const unsigned long long t0 = clock64();
     for (uint32_t i = 0; i < iters; ++i) {
-      const uint32_t kk = i & 3u;   // the four K = 16 steps of a 128-byte row
-      if constexpr (kTs)
-        tc::mma_ts(tmem, tmem + 256 + kk * 8, b_desc + (uint64_t)(kk * 2), kIdesc, i > 0 ? 1u : 0u);
+      const uint32_t kk = i & 3u;   // the four 32-byte K-steps of a 128-byte row
+      const uint32_t acc = i > 0 ? 1u : 0u;
+      if constexpr (kTs && kTf32)
+        mma_tf32_ts(tmem, tmem + 256 + kk * 8, b_desc + (uint64_t)(kk * 2), kIdesc, acc);
+      else if constexpr (kTf32)
+        mma_tf32_ss(tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), kIdesc, acc);
+      else if constexpr (kTs)
+        tc::mma_ts(tmem, tmem + 256 + kk * 8, b_desc + (uint64_t)(kk * 2), kIdesc, acc);
       else
-        tc::mma_ss(tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), kIdesc,
-                   i > 0 ? 1u : 0u);
+        tc::mma_ss(tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), kIdesc, acc);
     }
     tc::mma_commit(&bar);
     const bool ok = tc::mbar_wait(&bar, 0, &abort_flag, 1000000000ull);
@@ -135,25 +163,25 @@ __global__ void __launch_bounds__(128) k_probe_mma(uint32_t iters, unsigned long
   if (tid < 32) tc::tmem_dealloc(tmem, 512);
 }
 
-template <int N, bool kTs>
+template <int N, bool kTs, bool kTf32>
 cudaError_t launch_probe_mma(uint32_t iters, uint32_t blocks, unsigned long long* cycles,
                              cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(k_probe_mma<N, kTs>,
+  cudaError_t e = cudaFuncSetAttribute(k_probe_mma<N, kTs, kTf32>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
   if (e != cudaSuccess) return e;
-  k_probe_mma<N, kTs><<<blocks, 128, kMmaSmem, s>>>(iters, cycles);
+  k_probe_mma<N, kTs, kTf32><<<blocks, 128, kMmaSmem, s>>>(iters, cycles);
   return cudaGetLastError();
 }
 
-template <bool kTs>
+template <bool kTs, bool kTf32>
 cudaError_t launch_probe_mma_n(int n, uint32_t iters, uint32_t blocks, unsigned long long* cycles,
                                cudaStream_t s) {
   switch (n) {
-    case 16: return launch_probe_mma<16, kTs>(iters, blocks, cycles, s);
-    case 32: return launch_probe_mma<32, kTs>(iters, blocks, cycles, s);
-    case 64: return launch_probe_mma<64, kTs>(iters, blocks, cycles, s);
-    case 128: return launch_probe_mma<128, kTs>(iters, blocks, cycles, s);
-    default: return launch_probe_mma<256, kTs>(iters, blocks, cycles, s);
+    case 16: return launch_probe_mma<16, kTs, kTf32>(iters, blocks, cycles, s);
+    case 32: return launch_probe_mma<32, kTs, kTf32>(iters, blocks, cycles, s);
+    case 64: return launch_probe_mma<64, kTs, kTf32>(iters, blocks, cycles, s);
+    case 128: return launch_probe_mma<128, kTs, kTf32>(iters, blocks, cycles, s);
+    default: return launch_probe_mma<256, kTs, kTf32>(iters, blocks, cycles, s);
   }
 }
 
@@ -192,15 +220,18 @@ int auv_probe_ex2(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink
   return cudaGetLastError() == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
 }
 
-int auv_probe_mma(int n, int a_tmem, uint32_t iters, uint32_t blocks, uint64_t* cycles,
+int auv_probe_mma(int n, int a_tmem, int tf32, uint32_t iters, uint32_t blocks, uint64_t* cycles,
                   void* stream) {
   if ((n != 16 && n != 32 && n != 64 && n != 128 && n != 256) || iters < 1 || iters > (1u << 20) ||
       blocks < 1 || blocks > 65535 || !cycles)
     return AUV_ERR_INVALID;
   unsigned long long* c = reinterpret_cast<unsigned long long*>(cycles);
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const cudaError_t e = a_tmem ? launch_probe_mma_n<true>(n, iters, blocks, c, s)
-                               : launch_probe_mma_n<false>(n, iters, blocks, c, s);
+  const cudaError_t e =
+      tf32 ? (a_tmem ? launch_probe_mma_n<true, true>(n, iters, blocks, c, s)
+                     : launch_probe_mma_n<false, true>(n, iters, blocks, c, s))
+           : (a_tmem ? launch_probe_mma_n<true, false>(n, iters, blocks, c, s)
+                     : launch_probe_mma_n<false, false>(n, iters, blocks, c, s));
   return e == cudaSuccess ? AUV_OK : AUV_ERR_CUDA;
 }
 

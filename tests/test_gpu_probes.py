@@ -69,17 +69,18 @@ def test_mma_probe_costs_grow_with_n():
     torch = need_gpu()
     from paper_2512_13359_gb300 import auvenv
     cyc = torch.zeros(4, dtype=torch.int64, device="cuda")
-    per = {}
-    for n in (16, 64, 256):
+    for tf32 in (False, True):
+        per = {}
+        for n in (16, 64, 256):
+            for a_tmem in (False, True):
+                auvenv.probe_mma(n, a_tmem, 256, cyc, tf32=tf32)
+                torch.cuda.synchronize()
+                c = cyc.cpu()
+                assert int((c == 0).sum()) == 0
+                per[(n, a_tmem)] = float(c.double().median()) / 256
+        print("[probe] cycles per MMA", "tf32" if tf32 else "bf16", per)
         for a_tmem in (False, True):
-            auvenv.probe_mma(n, a_tmem, 256, cyc)
-            torch.cuda.synchronize()
-            c = cyc.cpu()
-            assert int((c == 0).sum()) == 0
-            per[(n, a_tmem)] = float(c.double().median()) / 256
-    print("[probe] cycles per MMA", per)
-    for a_tmem in (False, True):
-        assert per[(16, a_tmem)] <= per[(64, a_tmem)] * 1.05 <= per[(256, a_tmem)] * 1.05
+            assert per[(16, a_tmem)] <= per[(64, a_tmem)] * 1.05 <= per[(256, a_tmem)] * 1.05
     with pytest.raises(auvenv.AuvError):
         auvenv.probe_mma(48, False, 16, cyc)            # not a supported N
     with pytest.raises(auvenv.AuvError):
