@@ -745,8 +745,9 @@ int auv_gemm(uint32_t precision, int M, int N, int K, const void* A, int lda, in
  * auv_probe_ex2: the same shape with ex2.approx.ftz.f32: 8 * iters operations
  *   per thread.
  *   blocks in [1, 65535], threads a multiple of 32 in [32, 1024], iters >= 1;
- *   sink: device memory of blocks * threads floats (written only to keep the
- *   work from being removed).
+ *   sink: device memory (of the current device) of blocks * threads floats
+ *   (written only to keep the work from being removed); a host pointer is
+ *   AUV_ERR_INVALID.
  * auv_probe_gemm: one n x n x n cuBLAS GEMM, C = A B (column-major, fp32 C),
  *   with A, B fp32 and tf32 tensor-core math (AUV_PPO_TF32) or bf16 operands
  *   (AUV_PPO_BF16): 2 n^3 flop.  n a multiple of 16.
@@ -754,8 +755,10 @@ int auv_gemm(uint32_t precision, int M, int N, int K, const void* A, int lda, in
  *   MMAs of shape M = 128, N = n and K = 16 bf16 (kind::f16), or K = 8 tf32
  *   (kind::tf32) when tf32 is nonzero, fp32 accumulator; A in shared memory,
  *   or in tensor memory when a_tmem is nonzero; back to back from one
- *   thread, then one commit and one bounded wait.  cycles: device memory of `blocks` uint64 values, each the SM
- *   cycles from the first issue to the completion (0 if the wait gave up).
+ *   thread, then one commit and one bounded wait.  cycles: device memory
+ *   (of the current device) of `blocks` uint64 values, each the SM cycles
+ *   from the first issue to the completion (0 if the wait gave up); a host
+ *   pointer is AUV_ERR_INVALID.
  *   n in {16, 32, 64, 128, 256}, iters in [1, 2^20], blocks in [1, 65535].
  * Return AUV_OK, AUV_ERR_INVALID on bad arguments or AUV_ERR_CUDA.
  * --------------------------------------------------------------------------- */

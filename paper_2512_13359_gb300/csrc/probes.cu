@@ -185,9 +185,21 @@ cudaError_t launch_probe_mma_n(int n, uint32_t iters, uint32_t blocks, unsigned 
   }
 }
 
+// Device (or managed) memory on the current device: the probes write there
+// from the GPU, so a host pointer is rejected before any launch.
+bool device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  int dev = -1;
+  if (!p || cudaPointerGetAttributes(&a, p) != cudaSuccess || cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeManaged || (a.type == cudaMemoryTypeDevice && a.device == dev);
+}
+
 int probe_grid(uint32_t blocks, uint32_t threads, uint32_t iters, const float* sink) {
   if (blocks < 1 || blocks > 65535 || threads < 32 || threads > 1024 || threads % 32 || iters < 1 ||
-      !sink)
+      !device_ptr(sink))
     return AUV_ERR_INVALID;
   return AUV_OK;
 }
@@ -223,7 +235,7 @@ int auv_probe_ex2(uint32_t blocks, uint32_t threads, uint32_t iters, float* sink
 int auv_probe_mma(int n, int a_tmem, int tf32, uint32_t iters, uint32_t blocks, uint64_t* cycles,
                   void* stream) {
   if ((n != 16 && n != 32 && n != 64 && n != 128 && n != 256) || iters < 1 || iters > (1u << 20) ||
-      blocks < 1 || blocks > 65535 || !cycles)
+      blocks < 1 || blocks > 65535 || !device_ptr(cycles))
     return AUV_ERR_INVALID;
   unsigned long long* c = reinterpret_cast<unsigned long long*>(cycles);
   const cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -85,6 +85,8 @@ def test_mma_probe_costs_grow_with_n():
         auvenv.probe_mma(48, False, 16, cyc)            # not a supported N
     with pytest.raises(auvenv.AuvError):
         auvenv.probe_mma(64, False, 0, cyc)             # no MMA
+    with pytest.raises(auvenv.AuvError):
+        auvenv.probe_mma(64, False, 16, torch.zeros(4, dtype=torch.int64))   # host memory
 
 
 def test_ex2_probe_runs():
@@ -95,3 +97,5 @@ def test_ex2_probe_runs():
     torch.cuda.synchronize()
     with pytest.raises(auvenv.AuvError):
         auvenv.probe_ex2(4, 100, 10, sink)
+    with pytest.raises(auvenv.AuvError):
+        auvenv.probe_ex2(4, 256, 10, torch.zeros(4 * 256))               # host memory
