@@ -331,7 +331,7 @@ def measure_replay(w, steps, warmup, clocks_on=True, device=0):
     return step_ms, n * T, achieved, fp32_peak, src, clock_info
 
 
-# The fp32 workloads (BASELINE's first three): 64 envs x 200 steps with the
+# The three fp32 workloads: 64 envs x 200 steps with the
 # 18-64-64-8 network on CUDA cores (hidden 64 is far below a tensor-core
 # tile), and 4,096 / 16,384 envs x 1,000 steps with the 18-256-256-8 network
 # on the tensor cores in tf32 (kind::tf32); trajectories of rewards and dones.

@@ -134,9 +134,8 @@ def _windows(w, T, win=16):
                                         ("dr_16384", 300, 20, 6)])
 def test_tf32_engine_rollout_every_step(oracle, name, n, T, L):
     """The fp32 workloads' tensor-core rollout (k_rollout_tf32): 4,096 envs x
-    1,000 steps (the paper's env count, BASELINE's second workload) and
-    16,384 envs x 1,000 steps with domain randomisation and current (the
-    third), both with auto-resets at step 500, plus ragged sizes that reset
+    1,000 steps (the paper's env count) and 16,384 envs x 1,000 steps with
+    domain randomisation and current, both with auto-resets at step 500, plus ragged sizes that reset
     inside short launches; every step of 40 sampled envs against the oracle."""
     need_gpu()
     w = W.workload(name, n_envs=n, episode_len=L, mlp="tf32")
