@@ -379,7 +379,10 @@ def measure_config(name, mlp, reps, device=0):
     pol = mlp_flops(W.obs_dim(w), w["hidden"], w["policy_out"])
     if mlp == "tf32":
         peak = peaks["bf16_tflops"] * 1.1 / 2.25
-        roof = {"bound": "tensor", "kernel": "k_rollout_tf32", "achieved": rate * pol / 1e12,
+        # a CTA pair per 128-env tile while the tiles fill at most half the SMs
+        n_sm = torch.cuda.get_device_properties(device).multi_processor_count
+        kern = "k_rollout_tf32_pair" if 2 * ((n + 127) // 128) <= n_sm else "k_rollout_tf32"
+        roof = {"bound": "tensor", "kernel": kern, "achieved": rate * pol / 1e12,
                 "peak": peak, "unit": "TFLOP/s", "frac": rate * pol / 1e12 / peak,
                 "peak_source": f"bf16 burst, {src}, x tf32/bf16 nominal 1.1/2.25"}
     else:
